@@ -1,0 +1,379 @@
+"""Float64 oracle of one ProxyFormer layer (Alg. 1), forward and backward.
+
+TEST INFRASTRUCTURE ONLY (see the package docstring): a plain restatement of
+the paper's equations, one step per function, no blocking, fusion or
+reordering.  Library matmuls serve as steps.
+
+Readings of the paper taken here (each is a descriptor flag of the library):
+  * Causal 1D routing: the tokens of block i receive the decompression of the
+    interacted proxy i-1; block 0 receives zero.  (Proxy i summarises tokens
+    that come after the early tokens of block i, so this shift is the reading
+    under which a token never sees a later token; it also matches the decode
+    rule that only completed blocks are cached, Sec. 3.8.)
+  * F is standard multi-head attention with an output projection and no
+    biases; no norm inside F for 1D; the 2D layer applies adaptive LayerNorm
+    (timestep-conditioned scale/shift) to the proxies before attention, the
+    only place conditions touch the proxies (Sec. 3.9).
+  * Gate g(X, D) = w_x*X + w_dlt*D + b_g per channel (Eq. inj-gate).
+  * H carried to the next layer is the pre-interaction H (Alg. 1 returns H).
+  * Two-level cascade: no nonlinearity between levels, biases at each level.
+  * Affine injection (Eq. inj-affine): s and t are the two halves of a
+    2*P*d-wide decompression (token p takes [s | t] from columns
+    [2pd, 2pd+d) and [2pd+d, 2(p+1)d)); Norm is LayerNorm without affine,
+    biased variance, eps 1e-6.
+  * L % P != 0: the last block is zero-padded for compression (m = ceil(L/P)).
+"""
+from __future__ import annotations
+
+import math
+from typing import Dict, Optional
+
+import numpy as np
+
+CAUSAL_1D, BIDIR_1D, BIDIR_2D = 0, 1, 2
+INJ_ADD, INJ_GATED, INJ_AFFINE = 0, 1, 2
+LN_EPS = 1e-6
+TEMB_DIM = 256
+
+
+def _f64(a):
+    return None if a is None else np.asarray(a, dtype=np.float64)
+
+
+def sigmoid(x):
+    return 1.0 / (1.0 + np.exp(-x))
+
+
+# ---------------------------------------------------------------- partition
+def partition(X, spec):
+    """Eq. partition (Sec. 3.2 "Partitioning"): split one sequence X [L, d]
+    into m = ceil(L/P) blocks X_i [P, d].  1D: contiguous non-overlapping
+    blocks, the last zero-padded.  2D: p x p spatial patches of the
+    grid_h x grid_w raster, patches in raster order, tokens inside a patch in
+    raster order (py, px)."""
+    L, d = X.shape
+    P = spec.P
+    if spec.mode == BIDIR_2D:
+        p, gh, gw = spec.patch, spec.grid_h, spec.grid_w
+        g = X.reshape(gh // p, p, gw // p, p, d)          # (by, py, bx, px, ch)
+        return g.transpose(0, 2, 1, 3, 4).reshape(-1, P, d)  # (by*bx, py*px, ch)
+    m = -(-L // P)
+    Xp = np.zeros((m * P, d))
+    Xp[:L] = X
+    return Xp.reshape(m, P, d)
+
+
+def unpartition(blocks, spec, L):
+    """Inverse of ``partition``: per-token array [L, w] from [m, P, w]."""
+    m, P, w = blocks.shape
+    if spec.mode == BIDIR_2D:
+        p, gh, gw = spec.patch, spec.grid_h, spec.grid_w
+        g = blocks.reshape(gh // p, gw // p, p, p, w).transpose(0, 2, 1, 3, 4)
+        return g.reshape(gh * gw, w)
+    return blocks.reshape(m * P, w)[:L]
+
+
+# -------------------------------------------------------------- compression
+def compress(Xb, prm, spec):
+    """Eq. compress-linear and Eq. factor-cascade: c_i = Proj(Flatten(X_i)).
+
+    Flatten is token-major (index p*d + ch).  Two levels: level 1 groups the P
+    tokens into k2 consecutive groups of k1 and projects each group's k1*d
+    vector to d (y_{i,a}); level 2 concatenates the k2 rows and projects the
+    k2*d vector to d.  Returns C [m, d] and the level-1 rows Y [m, k2, d]."""
+    m, P, d = Xb.shape
+    k1, k2 = spec.k1, spec.k2
+    groups = Xb.reshape(m, k2, k1 * d)                     # vec of each group
+    Y = groups @ _f64(prm["W_c1"]).T + _f64(prm["b_c1"])   # [m, k2, d]
+    if spec.levels == 1:
+        return Y.reshape(m, d), None
+    C = Y.reshape(m, k2 * d) @ _f64(prm["W_c2"]).T + _f64(prm["b_c2"])
+    return C, Y
+
+
+def decompress(Hbar, prm, spec):
+    """Eq. decompress-linear and Eq. factor-dec: D_i = Unflatten(Proj_up(Hbar_i)).
+
+    Two levels run in the opposite order: level 2 maps the proxy to k2 rows of
+    width d, level 1 maps each row to k1 tokens.  Output [m, P, w] with w = d,
+    or w = 2d for affine injection ([s | t] per token)."""
+    m, d = Hbar.shape
+    k1, k2 = spec.k1, spec.k2
+    if spec.levels == 2:
+        Z = Hbar @ _f64(prm["W_d2"]).T + _f64(prm["b_d2"])  # [m, k2*d]
+        rows = Z.reshape(m, k2, d)
+    else:
+        Z = None
+        rows = Hbar.reshape(m, 1, d)
+    out = rows @ _f64(prm["W_d1"]).T + _f64(prm["b_d1"])  # [m, k2, k1*w]
+    w = out.shape[-1] // k1
+    return out.reshape(m, k1 * k2, w), Z
+
+
+# ---------------------------------------------------------------- attention
+def _row_probs(q, Kh, n_vis, scale):
+    """Softmax of one query row over its visible keys 0..n_vis-1 (the mask M
+    of Eq. proxy-attn removes the rest), with the row maximum subtracted."""
+    s = (Kh[:n_vis] @ q) * scale
+    e = np.exp(s - s.max())
+    return e / e.sum()
+
+
+def attention(Hq, prm, spec):
+    """Eq. proxy-attn: Hbar = softmax(Q K^T / sqrt(dh) + M) V per head, then
+    the output projection.  M is the causal mask (proxy i sees j <= i) for the
+    autoregressive 1D mode and zero otherwise.  Evaluated one query row at a
+    time over the visible keys only."""
+    m, d = Hq.shape
+    nh, dh = spec.n_heads, d // spec.n_heads
+    W = _f64(prm["W_qkv"])
+    Q, K, V = Hq @ W[:d].T, Hq @ W[d:2 * d].T, Hq @ W[2 * d:].T
+    A = np.zeros((m, d))
+    scale = 1.0 / math.sqrt(dh)
+    causal = spec.mode == CAUSAL_1D
+    for h in range(nh):
+        cs = slice(h * dh, (h + 1) * dh)
+        Qh, Kh, Vh = Q[:, cs], K[:, cs], V[:, cs]
+        for i in range(m):
+            n_vis = i + 1 if causal else m
+            A[i, cs] = _row_probs(Qh[i], Kh, n_vis, scale) @ Vh[:n_vis]
+    Hbar = A @ _f64(prm["W_o"]).T
+    return Hbar, dict(Q=Q, K=K, V=V, A=A)
+
+
+def attention_bwd(dA, c, spec):
+    """Backward of the attention core, row by row: with p the probabilities of
+    row i, dV += p^T dO_i, dp = V dO_i, dS = p * (dp - <p, dp>),
+    dQ_i = scale dS K, dK += scale dS^T Q_i."""
+    Q, K, V = c["Q"], c["K"], c["V"]
+    m, d = Q.shape
+    nh, dh = spec.n_heads, d // spec.n_heads
+    scale = 1.0 / math.sqrt(dh)
+    causal = spec.mode == CAUSAL_1D
+    dQ, dK, dV = np.zeros_like(Q), np.zeros_like(K), np.zeros_like(V)
+    for h in range(nh):
+        cs = slice(h * dh, (h + 1) * dh)
+        Qh, Kh, Vh = Q[:, cs], K[:, cs], V[:, cs]
+        dQh, dKh, dVh = dQ[:, cs], dK[:, cs], dV[:, cs]
+        for i in range(m):
+            n_vis = i + 1 if causal else m
+            p = _row_probs(Qh[i], Kh, n_vis, scale)
+            dO = dA[i, cs]
+            dVh[:n_vis] += np.outer(p, dO)
+            dp = Vh[:n_vis] @ dO
+            dS = p * (dp - p @ dp)
+            dQh[i] = scale * (dS @ Kh[:n_vis])
+            dKh[:n_vis] += scale * np.outer(dS, Qh[i])
+    return dQ, dK, dV
+
+
+# ----------------------------------------------------------- 2D conditioning
+def timestep_embedding(t):
+    """Sinusoidal embedding of the flow-matching time t (this library's own
+    definition; the paper fixes none): e_k = cos(1000 t w_k),
+    e_{128+k} = sin(1000 t w_k), w_k = 10000^(-k/128), k < 128."""
+    half = TEMB_DIM // 2
+    w = 10000.0 ** (-np.arange(half) / half)
+    a = 1000.0 * float(t) * w
+    return np.concatenate([np.cos(a), np.sin(a)])
+
+
+def layernorm(x):
+    """LayerNorm over the last axis, no affine, biased variance, eps 1e-6."""
+    mu = x.mean(-1, keepdims=True)
+    var = ((x - mu) ** 2).mean(-1, keepdims=True)
+    return (x - mu) / np.sqrt(var + LN_EPS), mu, np.sqrt(var + LN_EPS)
+
+
+def silu(x):
+    return x * sigmoid(x)
+
+
+def adaln_params(t, prm):
+    """Timestep conditioning of the proxy stream (Sec. 3.9: conditions touch
+    only the proxies): u = SiLU(W_t1 e(t) + b_t1), [gamma | beta] = W_t2 u + b_t2."""
+    e = timestep_embedding(t)
+    a1 = _f64(prm["W_t1"]) @ e + _f64(prm["b_t1"])
+    u = silu(a1)
+    gb = _f64(prm["W_t2"]) @ u + _f64(prm["b_t2"])
+    d = gb.shape[0] // 2
+    return gb[:d], gb[d:], dict(e=e, a1=a1, u=u)
+
+
+# ------------------------------------------------------------------ forward
+def _fwd_one(spec, prm, X, H_in, t):
+    L, d = X.shape
+    Xb = partition(X, spec)                                   # Eq. partition
+    C, Y = compress(Xb, prm, spec)                            # Eq. compress-linear
+    H = C if H_in is None else H_in + C                       # Eq. proxy-res
+    cache = dict(Xb=Xb, Y=Y, H=H)
+    Hq = H
+    if spec.mode == BIDIR_2D:                                 # Sec. 3.9
+        gamma, beta, tc = adaln_params(t, prm)
+        nH, muH, sdH = layernorm(H)
+        Hq = (1.0 + gamma) * nH + beta
+        cache.update(gamma=gamma, beta=beta, tc=tc, nH=nH, sdH=sdH)
+    Hbar, ac = attention(Hq, prm, spec)                       # Eq. proxy-attn
+    D, Z = decompress(Hbar, prm, spec)                        # Eq. decompress-linear
+    cache.update(Hq=Hq, Hbar=Hbar, Z=Z, D=D, **ac)
+    m = Xb.shape[0]
+    if spec.mode == CAUSAL_1D:                                # routing shift
+        Dr = np.zeros_like(D)
+        Dr[1:] = D[:-1]
+    else:
+        Dr = D
+    Dt = unpartition(Dr, spec, L)                             # per-token update
+    cache["Dt"] = Dt
+    if spec.inject == INJ_ADD:                                # Eq. inj-add
+        Xo = X + Dt
+    elif spec.inject == INJ_GATED:                            # Eq. inj-gate
+        g = _f64(prm["w_x"]) * X + _f64(prm["w_dlt"]) * Dt + _f64(prm["b_g"])
+        sg = sigmoid(g)
+        Xo = X + sg * Dt
+        cache["sg"] = sg
+    else:                                                     # Eq. inj-affine
+        s, tau = Dt[:, :d], Dt[:, d:]
+        nX, muX, sdX = layernorm(X)
+        Xo = (1.0 + s) * nX + tau
+        cache.update(nX=nX, sdX=sdX)
+    return Xo, H, cache
+
+
+def layer_fwd(spec, prm: Dict[str, np.ndarray], X, H_in=None, t=None,
+              return_cache: bool = False):
+    """Alg. 1 over a batch: X [B, L, d] -> (X_out [B, L, d], H_out [B, m, d])."""
+    X = _f64(X)
+    outs, hs, caches = [], [], []
+    for b in range(X.shape[0]):
+        hin = None if H_in is None else _f64(H_in[b])
+        tb = None if t is None else float(t[b])
+        Xo, H, c = _fwd_one(spec, prm, X[b], hin, tb)
+        outs.append(Xo)
+        hs.append(H)
+        caches.append(c)
+    res = (np.stack(outs), np.stack(hs))
+    return res + (caches,) if return_cache else res
+
+
+# ----------------------------------------------------------------- backward
+def _layernorm_bwd(dn, n, sd):
+    """Gradient through n = (x - mean)/sd with sd = sqrt(var + eps)."""
+    return (dn - dn.mean(-1, keepdims=True)
+            - n * (dn * n).mean(-1, keepdims=True)) / sd
+
+
+def _bwd_one(spec, prm, X, c, G, dH_out, grads):
+    L, d = X.shape
+    m = c["Xb"].shape[0]
+    P, k1, k2 = spec.P, spec.k1, spec.k2
+    nh, dh = spec.n_heads, d // spec.n_heads
+    Dt = c["Dt"]
+    # injection (Eq. inj-*)
+    if spec.inject == INJ_ADD:
+        dX = G.copy()
+        dDt = G.copy()
+    elif spec.inject == INJ_GATED:
+        sg = c["sg"]
+        ds = G * Dt * sg * (1.0 - sg)                          # dL/dg
+        dX = G + ds * _f64(prm["w_x"])
+        dDt = G * sg + ds * _f64(prm["w_dlt"])
+        grads["w_x"] += (ds * X).sum(0)
+        grads["w_dlt"] += (ds * Dt).sum(0)
+        grads["b_g"] += ds.sum(0)
+    else:
+        nX, sdX = c["nX"], c["sdX"]
+        s = Dt[:, :d]
+        dDt = np.concatenate([G * nX, G], axis=1)
+        dX = _layernorm_bwd(G * (1.0 + s), nX, sdX)
+    # routing
+    w = dDt.shape[1]
+    if spec.mode == BIDIR_2D:
+        dDr = partition_w(dDt, spec)
+    else:
+        pad = np.zeros((m * P, w))
+        pad[:L] = dDt
+        dDr = pad.reshape(m, P, w)
+    if spec.mode == CAUSAL_1D:
+        dD = np.zeros_like(dDr)
+        dD[:-1] = dDr[1:]
+    else:
+        dD = dDr
+    # decompression
+    dout = dD.reshape(m, k2, k1 * w)
+    grads["b_d1"] += dout.sum((0, 1))
+    rows = c["Z"].reshape(m, k2, d) if spec.levels == 2 else c["Hbar"].reshape(m, 1, d)
+    grads["W_d1"] += np.einsum("rao,rai->oi", dout, rows)
+    drows = dout @ _f64(prm["W_d1"])                           # [m, k2, d]
+    if spec.levels == 2:
+        dZ = drows.reshape(m, k2 * d)
+        grads["b_d2"] += dZ.sum(0)
+        grads["W_d2"] += dZ.T @ c["Hbar"]
+        dHbar = dZ @ _f64(prm["W_d2"])
+    else:
+        dHbar = drows.reshape(m, d)
+    # attention
+    grads["W_o"] += dHbar.T @ c["A"]
+    dA = dHbar @ _f64(prm["W_o"])
+    dQ, dK, dV = attention_bwd(dA, c, spec)
+    dQKV = np.concatenate([dQ, dK, dV], axis=1)
+    grads["W_qkv"] += dQKV.T @ c["Hq"]
+    dHq = dQKV @ _f64(prm["W_qkv"])
+    if spec.mode == BIDIR_2D:
+        gamma = c["gamma"]
+        nH, sdH = c["nH"], c["sdH"]
+        dgamma = (dHq * nH).sum(0)
+        dbeta = dHq.sum(0)
+        dH = _layernorm_bwd(dHq * (1.0 + gamma), nH, sdH)
+        tc = c["tc"]
+        dgb = np.concatenate([dgamma, dbeta])
+        grads["b_t2"] += dgb
+        grads["W_t2"] += np.outer(dgb, tc["u"])
+        du = _f64(prm["W_t2"]).T @ dgb
+        sa = sigmoid(tc["a1"])
+        da1 = du * (sa * (1.0 + tc["a1"] * (1.0 - sa)))
+        grads["b_t1"] += da1
+        grads["W_t1"] += np.outer(da1, tc["e"])
+    else:
+        dH = dHq
+    if dH_out is not None:
+        dH = dH + dH_out
+    dH_in = dH.copy()
+    # compression
+    dC = dH
+    if spec.levels == 2:
+        grads["b_c2"] += dC.sum(0)
+        grads["W_c2"] += dC.T @ c["Y"].reshape(m, k2 * d)
+        dY = (dC @ _f64(prm["W_c2"])).reshape(m, k2, d)
+    else:
+        dY = dC.reshape(m, 1, d)
+    grads["b_c1"] += dY.sum((0, 1))
+    groups = c["Xb"].reshape(m, k2, k1 * d)
+    grads["W_c1"] += np.einsum("rao,rai->oi", dY, groups)
+    dgroups = dY @ _f64(prm["W_c1"])                          # [m, k2, k1*d]
+    dXc = unpartition(dgroups.reshape(m, P, d), spec, L)
+    return dX + dXc, dH_in
+
+
+def partition_w(A, spec):
+    """``partition`` for a per-token array of any width (2D patches)."""
+    p, gh, gw = spec.patch, spec.grid_h, spec.grid_w
+    w = A.shape[1]
+    g = A.reshape(gh // p, p, gw // p, p, w)
+    return g.transpose(0, 2, 1, 3, 4).reshape(-1, p * p, w)
+
+
+def layer_bwd(spec, prm, X, G, H_in=None, t=None, dH_out=None):
+    """Backward of ``layer_fwd`` (chain rule through Eqs. partition ...
+    inj-*).  Returns (dX [B, L, d], dH_in [B, m, d], grads{name: array})."""
+    X = _f64(X)
+    G = _f64(G)
+    _, _, caches = layer_fwd(spec, prm, X, H_in, t, return_cache=True)
+    grads = {k: np.zeros(np.shape(v)) for k, v in prm.items()
+             if k.startswith(("W_", "b_", "w_"))}
+    dXs, dHs = [], []
+    for b in range(X.shape[0]):
+        dho = None if dH_out is None else _f64(dH_out[b])
+        dX, dH_in = _bwd_one(spec, prm, X[b], caches[b], G[b], dho, grads)
+        dXs.append(dX)
+        dHs.append(dH_in)
+    return np.stack(dXs), np.stack(dHs), grads

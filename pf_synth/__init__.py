@@ -1,0 +1,259 @@
+"""Seeded synthetic inputs for the ProxyFormer layer, append and decode paths.
+
+This module is the only code shared by the CUDA path's tests/bench and the CPU
+oracle.  It draws random numbers and lays them out in the shapes of the layer's
+tensors; it holds none of the method's arithmetic (no compression, attention,
+decompression or injection).
+
+Conventions fixed here (the layer's parameter shapes, ProxyFormer Sec. 3):
+  * every weight matrix is stored [out, in] (row-major): y = W @ x + b;
+  * flattening a block of tokens is token-major: vec index p*d + ch;
+  * level 1 of a two-level cascade is the token side (k1 tokens -> 1 row),
+    level 2 the proxy side (k2 rows -> 1 proxy), P = k1*k2 (Eq. factor);
+  * decompression mirrors it: level 2 maps a proxy to k2 rows, level 1 maps
+    each row to k1 tokens (Eq. factor-dec).
+
+Random draws use numpy's PCG64 (``numpy.random.default_rng(seed)``) in the fill
+order given by ``layer_param_shapes`` followed by the activations.  Matrices are
+Xavier-uniform U(+-sqrt(6/(fan_in+fan_out))); bias and gate vectors U(+-0.1);
+norm weights 1 + U(+-0.1).  For bf16 workloads every value is rounded once to
+the nearest bf16 (ties to even) so both sides of a comparison start from the
+same representable numbers.
+"""
+from __future__ import annotations
+
+import dataclasses
+import math
+from typing import Dict, Optional
+
+import numpy as np
+
+# mode / inject / dtype codes; they mirror the C header's enums.
+CAUSAL_1D, BIDIR_1D, BIDIR_2D = 0, 1, 2
+INJ_ADD, INJ_GATED, INJ_AFFINE = 0, 1, 2
+F32, BF16 = 0, 1
+
+TEMB_DIM = 256  # width of the sinusoidal timestep embedding (2D layer)
+
+
+@dataclasses.dataclass(frozen=True)
+class LayerSpec:
+    """Shape of one ProxyFormer layer (Alg. 1) plus its variant flags."""
+
+    batch: int
+    L: int
+    d: int
+    n_heads: int
+    P: int
+    levels: int = 1
+    k1: int = 0
+    k2: int = 0
+    mode: int = CAUSAL_1D
+    inject: int = INJ_GATED
+    dtype: int = BF16
+    grid_h: int = 0
+    grid_w: int = 0
+    patch: int = 0
+
+    def __post_init__(self):
+        if self.levels == 1:
+            object.__setattr__(self, "k1", self.P)
+            object.__setattr__(self, "k2", 1)
+
+    @property
+    def m(self) -> int:
+        """Number of blocks (proxies) per sequence, m = ceil(L/P)."""
+        return -(-self.L // self.P)
+
+    @property
+    def dh(self) -> int:
+        return self.d // self.n_heads
+
+
+@dataclasses.dataclass(frozen=True)
+class DecodeSpec:
+    """Shape of the proxy KV-cache decode state (Sec. 3.7/3.8)."""
+
+    batch: int
+    d: int
+    n_heads: int
+    P: int
+    levels: int = 1
+    k1: int = 0
+    k2: int = 0
+    capacity: int = 0
+
+    def __post_init__(self):
+        if self.levels == 1:
+            object.__setattr__(self, "k1", self.P)
+            object.__setattr__(self, "k2", 1)
+
+    @property
+    def dh(self) -> int:
+        return self.d // self.n_heads
+
+
+def default_factors(P: int):
+    """k1 = 2**ceil(log2(P)/2), k2 = P/k1 (16->4x4, 64->8x8, 128->16x8)."""
+    k1 = 1 << math.ceil(math.log2(P) / 2)
+    return k1, P // k1
+
+
+def round_bf16(a: np.ndarray) -> np.ndarray:
+    """Round float32 values to the nearest bfloat16, ties to even (no NaN input)."""
+    a = np.ascontiguousarray(a, dtype=np.float32)
+    u = a.view(np.uint32).astype(np.uint64)
+    u = (u + 0x7FFF + ((u >> 16) & 1)) & 0xFFFF0000
+    return u.astype(np.uint32).view(np.float32)
+
+
+def _finish(a: np.ndarray, dtype: int) -> np.ndarray:
+    a = a.astype(np.float32)
+    return round_bf16(a) if dtype == BF16 else a
+
+
+def layer_param_shapes(spec: LayerSpec) -> Dict[str, tuple]:
+    """Parameter names and shapes, in generator fill order."""
+    d, P, k1, k2 = spec.d, spec.P, spec.k1, spec.k2
+    s = {}
+    s["W_c1"] = (d, k1 * d)
+    s["b_c1"] = (d,)
+    if spec.levels == 2:
+        s["W_c2"] = (d, k2 * d)
+        s["b_c2"] = (d,)
+    s["W_qkv"] = (3 * d, d)
+    s["W_o"] = (d, d)
+    out_tok = 2 * d if spec.inject == INJ_AFFINE else d
+    if spec.levels == 2:
+        s["W_d2"] = (k2 * d, d)
+        s["b_d2"] = (k2 * d,)
+    s["W_d1"] = (k1 * out_tok, d)
+    s["b_d1"] = (k1 * out_tok,)
+    if spec.inject == INJ_GATED:
+        s["w_x"] = (d,)
+        s["w_dlt"] = (d,)
+        s["b_g"] = (d,)
+    if spec.mode == BIDIR_2D:
+        s["W_t1"] = (d, TEMB_DIM)
+        s["b_t1"] = (d,)
+        s["W_t2"] = (2 * d, d)
+        s["b_t2"] = (2 * d,)
+    return s
+
+
+def _xavier(rng, shape):
+    fan_out, fan_in = shape
+    bound = math.sqrt(6.0 / (fan_in + fan_out))
+    return rng.uniform(-bound, bound, size=shape)
+
+
+def make_layer_params(spec: LayerSpec, seed: int) -> Dict[str, np.ndarray]:
+    rng = np.random.default_rng(seed)
+    out = {}
+    for name, shape in layer_param_shapes(spec).items():
+        if name == "W_qkv":  # three d x d matrices drawn one after another
+            d = spec.d
+            a = np.concatenate([_xavier(rng, (d, d)) for _ in range(3)], axis=0)
+        elif len(shape) == 2:
+            a = _xavier(rng, shape)
+        else:
+            a = rng.uniform(-0.1, 0.1, size=shape)
+        out[name] = _finish(a, spec.dtype)
+    return out
+
+
+def make_layer_inputs(spec: LayerSpec, seed: int, with_h_in: bool = False,
+                      with_grads: bool = True) -> Dict[str, np.ndarray]:
+    """Params + activations.  X ~ N(0,1) [B, L, d]; G (upstream grad of X_out)
+    ~ N(0,1); dH_out ~ N(0,1); H_in ~ N(0,1) if requested; t ~ U(0,1) [B]."""
+    p = make_layer_params(spec, seed)
+    rng = np.random.default_rng(seed + 0x5EED)
+    B, L, d, m = spec.batch, spec.L, spec.d, spec.m
+    p["X"] = _finish(rng.standard_normal((B, L, d), dtype=np.float32), spec.dtype)
+    if with_h_in:
+        p["H_in"] = rng.standard_normal((B, m, d), dtype=np.float32)
+    if spec.mode == BIDIR_2D:
+        p["t"] = rng.uniform(0.0, 1.0, size=(B,)).astype(np.float32)
+    if with_grads:
+        p["G"] = _finish(rng.standard_normal((B, L, d), dtype=np.float32), spec.dtype)
+        p["dH_out"] = rng.standard_normal((B, m, d), dtype=np.float32)
+    return p
+
+
+def decode_param_shapes(spec: DecodeSpec) -> Dict[str, tuple]:
+    d, k1, k2, nh = spec.d, spec.k1, spec.k2, spec.n_heads
+    s = {"W_qkv": (3 * d, d), "W_o": (d, d), "rms_w": (d,),
+         "W_a1": (d // 8, d), "b_a1": (d // 8,), "W_a2": (nh, d // 8), "b_a2": (nh,),
+         "W_c1": (d, k1 * d), "b_c1": (d,)}
+    if spec.levels == 2:
+        s["W_c2"] = (d, k2 * d)
+        s["b_c2"] = (d,)
+    s["W_kvh"] = (2 * d, d)
+    return s
+
+
+def make_decode_params(spec: DecodeSpec, seed: int) -> Dict[str, np.ndarray]:
+    rng = np.random.default_rng(seed)
+    out = {}
+    for name, shape in decode_param_shapes(spec).items():
+        if name in ("W_qkv", "W_kvh"):
+            d = spec.d
+            nmat = shape[0] // d
+            a = np.concatenate([_xavier(rng, (d, d)) for _ in range(nmat)], axis=0)
+        elif len(shape) == 2:
+            a = _xavier(rng, shape)
+        elif name == "rms_w":
+            a = 1.0 + rng.uniform(-0.1, 0.1, size=shape)
+        else:
+            a = rng.uniform(-0.1, 0.1, size=shape)
+        out[name] = round_bf16(a.astype(np.float32))
+    return out
+
+
+def make_decode_state(spec: DecodeSpec, seed: int, n_proxy, n_open):
+    """Cache contents ~ N(0,1): K/V proxy rows [B, capacity, d] (rows past
+    n_proxy[b] are filled too, and must be ignored), open-block features and
+    their K/V [B, P, d] (slots past n_open[b] likewise), new token x [B, d]."""
+    rng = np.random.default_rng(seed + 0xDEC)
+    B, d, P, cap = spec.batch, spec.d, spec.P, spec.capacity
+    st = {}
+    st["K_proxy"] = round_bf16(rng.standard_normal((B, cap, d), dtype=np.float32))
+    st["V_proxy"] = round_bf16(rng.standard_normal((B, cap, d), dtype=np.float32))
+    st["X_open"] = round_bf16(rng.standard_normal((B, P, d), dtype=np.float32))
+    st["K_open"] = round_bf16(rng.standard_normal((B, P, d), dtype=np.float32))
+    st["V_open"] = round_bf16(rng.standard_normal((B, P, d), dtype=np.float32))
+    st["x"] = round_bf16(rng.standard_normal((B, d), dtype=np.float32))
+    st["n_proxy"] = np.asarray(n_proxy, dtype=np.int32).reshape(B)
+    st["n_open"] = np.asarray(n_open, dtype=np.int32).reshape(B)
+    return st
+
+
+# Workloads used by the tests and the bench (the paper's layer shapes).
+def spec_c1():
+    """1D causal layer, fwd, fp32: L=4096, d=256, 4x64 heads, P=64 single-level."""
+    return LayerSpec(batch=1, L=4096, d=256, n_heads=4, P=64, dtype=F32)
+
+
+def spec_c2():
+    """1D causal layer, fwd+bwd, bf16: L=65536, d=1024, 16x64 heads, P=64."""
+    return LayerSpec(batch=1, L=65536, d=1024, n_heads=16, P=64)
+
+
+def spec_c3_layer(P: int = 64):
+    """One layer of the 12-layer stack: L=262144, d=1024, 16x64, factorised."""
+    k1, k2 = default_factors(P)
+    return LayerSpec(batch=1, L=262144, d=1024, n_heads=16, P=P, levels=2, k1=k1, k2=k2)
+
+
+C3_RATIOS = (16, 16, 32, 32, 64, 64, 64, 64, 128, 128, 256, 256)
+
+
+def spec_c4():
+    """Proxy-only KV decode: B=8, d=2048, 16x128 heads, P=64, 16384 cached proxies."""
+    return DecodeSpec(batch=8, d=2048, n_heads=16, P=64, capacity=16384)
+
+
+def spec_c5():
+    """2D bidirectional layer: B=4, 512x512 grid, d=512, 8x64 heads, 8x8 patches."""
+    return LayerSpec(batch=4, L=512 * 512, d=512, n_heads=8, P=64, mode=BIDIR_2D,
+                     inject=INJ_AFFINE, grid_h=512, grid_w=512, patch=8)
