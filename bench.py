@@ -1,0 +1,389 @@
+#!/usr/bin/env python
+"""ProxyFormer layer forward + backward throughput on GB300.
+
+Workload: one causal 1D layer of the 12-layer long-context stack at the P = 64
+position: L = 262144 tokens, d = 1024, 16 heads x 64, two-level 8 x 8
+compression, gated injection, bf16 with fp32 accumulation, batch 1 per GPU.
+A step is proxy_layer_fwd + proxy_layer_bwd over that sequence (inputs already
+resident in HBM); `value` is tokens per second over all ranks.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+--impl reference times the float64 CPU oracle on the host cores instead (a
+bounded slice of the same workload per step); it is a deliberately slow
+baseline, not a GPU implementation.  Prints one JSON line (rank 0).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+METRIC = "ProxyFormer layer fwd+bwd tokens/s at L=256K, P=64; % of GB300 roofline"
+UNIT = "tokens/s"
+WORKLOAD = "proxyformer_layer_causal1d_L262144_d1024_h16x64_P64_8x8_gated_bf16_fwd_bwd"
+SAMPLE_L = 2048       # tokens of one reference-arm step (32 proxies)
+BASELINE_L = 65536   # tokens of the cpu_baseline slice (1024 proxies)
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def host_cores() -> int:
+    return int(os.environ.get("OPENBLAS_NUM_THREADS") or os.cpu_count() or 1)
+
+
+def workload_spec():
+    import pf_synth as S
+    return S.spec_c3_layer(64)
+
+
+def config_dict(spec, extra=None):
+    c = {"workload": WORKLOAD, "batch_per_gpu": spec.batch, "L": spec.L, "d": spec.d,
+         "heads": spec.n_heads, "head_dim": spec.dh, "P": spec.P, "levels": spec.levels,
+         "k1": spec.k1, "k2": spec.k2, "mode": "causal_1d", "inject": "gated",
+         "l2": "inputs larger than L2 (X, dX_out, X_out, dX are 512 MiB each; L2 is 129 MB)"}
+    c.update(extra or {})
+    return c
+
+
+# ------------------------------------------------------------------ oracle leg
+def oracle_sample_seconds(L_s: int, reps: int = 1):
+    """Wall seconds of one oracle fwd+bwd over an L_s-token slice of the workload."""
+    import numpy as np
+    import pf_synth as S
+    from oracle import layer as OL
+    full = workload_spec()
+    spec = S.LayerSpec(batch=1, L=L_s, d=full.d, n_heads=full.n_heads, P=full.P,
+                       levels=full.levels, k1=full.k1, k2=full.k2)
+    inp = S.make_layer_inputs(spec, 2)
+    times = []
+    for _ in range(reps):
+        t0 = time.perf_counter()
+        OL.layer_fwd(spec, inp, inp["X"])
+        OL.layer_bwd(spec, inp, inp["X"], inp["G"], None, None, inp["dH_out"])
+        times.append(time.perf_counter() - t0)
+    return times
+
+
+def cpu_baseline_subprocess():
+    """Run the oracle slice in a fresh interpreter with an explicit BLAS thread count."""
+    cores = os.cpu_count() or 1
+    env = dict(os.environ, OPENBLAS_NUM_THREADS=str(cores), OMP_NUM_THREADS=str(cores))
+    code = ("import json, bench; t = bench.oracle_sample_seconds(%d, 1); print(json.dumps(t))"
+            % BASELINE_L)
+    r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, env=env, capture_output=True,
+                       text=True, timeout=900)
+    if r.returncode != 0:
+        return {"value": None, "unit": UNIT, "cores": cores, "kind": "oracle",
+                "sample": "failed: " + r.stderr.strip().splitlines()[-1][:200]}
+    t = json.loads(r.stdout.strip().splitlines()[-1])
+    return {"value": BASELINE_L / min(t), "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"one fwd+bwd of the float64 oracle over a {BASELINE_L}-token slice "
+                      f"({BASELINE_L // 64} proxies) of the same layer shape, {min(t):.1f} s"}
+
+
+def run_reference(args, rank: int):
+    if rank != 0:
+        return
+    cores = host_cores()
+    spec = workload_spec()
+    times = []
+    for i in range(args.warmup + args.steps):
+        t = oracle_sample_seconds(SAMPLE_L, 1)[0]
+        if i >= args.warmup:
+            times.append(t)
+    sec = statistics.mean(times)
+    value = SAMPLE_L / sec
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "impl": "reference",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": sec * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": config_dict(spec, {"oracle_slice_tokens": SAMPLE_L}),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": f"each step: float64 oracle fwd+bwd over a {SAMPLE_L}-token "
+                                       f"slice of the workload"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    """nvidia-smi samples (every 50 ms) taken while the timed region runs."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.rows = []
+        self.t0 = self.t1 = None
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", "-i", gpu_id, "--query-gpu=" + self.FIELDS,
+                                       "--format=csv,noheader,nounits", "-lms", "50"],
+                                      stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.p = None
+            return
+        self.th = threading.Thread(target=self._read, daemon=True)
+        self.th.start()
+
+    def _read(self):
+        for line in self.p.stdout:
+            self.rows.append((time.time(), [x.strip() for x in line.split(",")]))
+
+    def mark(self, start: bool):
+        if start:
+            self.t0 = time.time()
+        else:
+            self.t1 = time.time()
+
+    def stop(self):
+        if self.p is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.12)
+        self.p.terminate()
+        try:
+            self.p.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.p.kill()
+        rows = [r for t, r in self.rows if self.t0 and self.t1 and self.t0 - 0.06 <= t <= self.t1]
+        sm, mx, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for r in rows:
+            try:
+                sm.append(float(r[0]))
+                mx.append(float(r[1]))
+            except (ValueError, IndexError):
+                continue
+            for n, v in zip(names, r[4:8]):
+                if v.strip().lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def gpu_smi_id(torch, dev: int) -> str:
+    try:
+        u = str(torch.cuda.get_device_properties(dev).uuid)
+        return u if u.startswith("GPU-") else "GPU-" + u
+    except Exception:
+        vis = os.environ.get("CUDA_VISIBLE_DEVICES", "")
+        return vis.split(",")[dev] if vis else str(dev)
+
+
+# ------------------------------------------------------------------ our leg
+def source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2608_23463_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, f), "rb") as fh:
+            h.update(f.encode() + fh.read())
+    return h.hexdigest()[:16]
+
+
+def traffic_from_profile(label: str):
+    """dram bytes per launch of `label` from profiles/traffic.txt (lines:
+    label bytes_per_launch source_hash), or None when absent or stale."""
+    path = os.path.join(ROOT, "profiles", "traffic.txt")
+    if not os.path.exists(path):
+        return None
+    cur = source_hash()
+    for line in open(path):
+        parts = line.split()
+        if len(parts) >= 3 and not line.startswith("#") and parts[0] == label:
+            return float(parts[1]) if parts[2] == cur else None
+    return None
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            return json.load(f), "measured"
+    return PEAKS_FALLBACK, "fallback"
+
+
+def run_ours(args, rank: int, world: int, local_rank: int):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    import paper_2608_23463_gb300 as pf
+    import pf_synth as S
+    from paper_2608_23463_gb300.layer import ProxyLayer, to_device
+
+    torch.cuda.set_device(local_rank)
+    pf.build()
+    spec = workload_spec()
+    inp = S.make_layer_inputs(spec, 2 + 1000 * rank)
+    lay = ProxyLayer(spec, inp)
+    X = to_device(inp["X"], torch.bfloat16)
+    G = to_device(inp["G"], torch.bfloat16)
+    del inp
+    Xo, dX = lay.empty_act(), lay.empty_act()
+    stream = torch.cuda.current_stream()
+
+    def step():
+        lay.forward(X, X_out=Xo)
+        lay.backward(X, G, dX=dX)
+
+    for _ in range(max(args.warmup, 3)):
+        step()
+    pf.pf_sync_check(stream.cuda_stream)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+
+    sampler = ClockSampler(gpu_smi_id(torch, local_rank)) if rank == 0 else None
+    time.sleep(0.3)
+    pf.pf_timing_enable(True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    if sampler:
+        sampler.mark(True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if sampler:
+        sampler.mark(False)
+    if world > 1:
+        dist.barrier()
+    ms = e0.elapsed_time(e1) / args.steps
+    timing = pf.pf_timing_collect()
+    pf.pf_timing_enable(False)
+    pf.pf_sync_check(stream.cuda_stream)
+    clocks = sampler.stop() if sampler else None
+    if world > 1:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    tokens_per_step = spec.batch * spec.L * world
+    value = tokens_per_step / (ms / 1e3)
+    launches = sum(v["launches"] for v in timing.values())
+
+    # ---- end to end: pinned host inputs in, results out, every step
+    Xh = X.cpu().pin_memory()
+    Gh = G.cpu().pin_memory()
+    Xoh = torch.empty_like(Xh).pin_memory()
+    dXh = torch.empty_like(Xh).pin_memory()
+    X2, G2 = torch.empty_like(X), torch.empty_like(G)
+
+    def e2e_step():
+        X2.copy_(Xh, non_blocking=True)
+        G2.copy_(Gh, non_blocking=True)
+        lay.forward(X2, X_out=Xo)
+        lay.backward(X2, G2, dX=dX)
+        Xoh.copy_(Xo, non_blocking=True)
+        dXh.copy_(dX, non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    e0.record(stream)
+    for _ in range(args.e2e_steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms_e2e = e0.elapsed_time(e1) / args.e2e_steps
+    if world > 1:
+        t = torch.tensor([ms_e2e], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_e2e = float(t.item())
+    pf.pf_sync_check(stream.cuda_stream)
+    act_bytes = spec.batch * spec.L * spec.d * 2
+    if rank != 0:
+        return
+
+    peaks, peak_src = load_peaks()
+    # dominant kernel: largest share of the timed region
+    dom, dv = max(timing.items(), key=lambda kv: kv[1]["ms"])
+    avg_s = dv["ms"] / dv["launches"] / 1e3
+    if dv["flops"] > 0 and not dom.startswith(("inj_bwd", "colsum", "copy", "pad")):
+        achieved = dv["flops"] / avg_s / 1e12
+        peak = peaks["bf16_tflops_sustained"]
+        roof = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": achieved / peak, "traffic": traffic_from_profile(dom), "kernel": dom,
+                "launches": dv["launches"], "avg_us": avg_s * 1e6,
+                "flops_per_launch": dv["flops"],
+                "peak_source": f"{peak_src} bf16_tflops_sustained (kernel timed inside a long step)"}
+    else:
+        achieved = dv["bytes"] / avg_s / 1e9
+        peak = peaks["hbm_gbs"]
+        roof = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": achieved / peak, "traffic": traffic_from_profile(dom), "kernel": dom,
+                "launches": dv["launches"], "avg_us": avg_s * 1e6,
+                "bytes_per_launch": dv["bytes"], "peak_source": f"{peak_src} hbm_gbs"}
+    step_flops = sum(v["flops"] * v["launches"] for v in timing.values()) / args.steps
+    step_bytes = sum(v["bytes"] * v["launches"] for v in timing.values()) / args.steps
+    roof_ms = max(step_flops / (peaks["bf16_tflops_sustained"] * 1e12),
+                  step_bytes / (peaks["hbm_gbs"] * 1e9)) * 1e3
+    total_ms = sum(v["ms"] for v in timing.values())
+    breakdown = {k: {"ms_per_step": v["ms"] / args.steps, "share": v["ms"] / total_ms,
+                     "launches_per_step": v["launches"] / args.steps}
+                 for k, v in sorted(timing.items(), key=lambda kv: -kv[1]["ms"])}
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic", "config": config_dict(spec),
+            "roofline": roof,
+            "layer_roofline": {"flops_per_step": step_flops, "bytes_per_step": step_bytes,
+                               "roofline_ms": roof_ms, "frac": roof_ms / ms,
+                               "peaks": f"{peak_src}: bf16 sustained "
+                                        f"{peaks['bf16_tflops_sustained']} TFLOP/s, "
+                                        f"HBM {peaks['hbm_gbs']} GB/s"},
+            "e2e": {"value": tokens_per_step / (ms_e2e / 1e3), "unit": UNIT,
+                    "h2d_bytes_per_step": 2 * act_bytes, "d2h_bytes_per_step": 2 * act_bytes,
+                    "ms_per_step": ms_e2e},
+            "gpu_launches": launches, "clocks": clocks, "kernels": breakdown}
+    if world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline_subprocess()
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse_args()
+    rank = int(os.environ.get("RANK", 0))
+    world = int(os.environ.get("WORLD_SIZE", 1))
+    local_rank = int(os.environ.get("LOCAL_RANK", 0))
+    sys.path.insert(0, ROOT)
+    if args.impl == "reference":
+        run_reference(args, rank)
+        return
+    import torch.distributed as dist
+    if world > 1:
+        import torch
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    try:
+        run_ours(args, rank, world, local_rank)
+    finally:
+        if world > 1:
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

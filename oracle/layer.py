@@ -302,7 +302,7 @@ def _bwd_one(spec, prm, X, c, G, dH_out, grads):
     dout = dD.reshape(m, k2, k1 * w)
     grads["b_d1"] += dout.sum((0, 1))
     rows = c["Z"].reshape(m, k2, d) if spec.levels == 2 else c["Hbar"].reshape(m, 1, d)
-    grads["W_d1"] += np.einsum("rao,rai->oi", dout, rows)
+    grads["W_d1"] += dout.reshape(m * k2, k1 * w).T @ rows.reshape(m * k2, d)
     drows = dout @ _f64(prm["W_d1"])                           # [m, k2, d]
     if spec.levels == 2:
         dZ = drows.reshape(m, k2 * d)
@@ -348,7 +348,7 @@ def _bwd_one(spec, prm, X, c, G, dH_out, grads):
         dY = dC.reshape(m, 1, d)
     grads["b_c1"] += dY.sum((0, 1))
     groups = c["Xb"].reshape(m, k2, k1 * d)
-    grads["W_c1"] += np.einsum("rao,rai->oi", dY, groups)
+    grads["W_c1"] += dY.reshape(m * k2, d).T @ groups.reshape(m * k2, k1 * d)
     dgroups = dY @ _f64(prm["W_c1"])                          # [m, k2, k1*d]
     dXc = unpartition(dgroups.reshape(m, P, d), spec, L)
     return dX + dXc, dH_in

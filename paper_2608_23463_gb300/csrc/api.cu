@@ -1,0 +1,502 @@
+// C ABI of the library (include/proxyformer.h): argument validation,
+// workspace / saved-buffer planning and the launch sequence of one layer.
+#include <stdarg.h>
+#include <stdio.h>
+
+#include <algorithm>
+#include <string>
+
+#include "kernels.h"
+#include "proxyformer.h"
+
+using namespace pf;
+
+namespace {
+
+thread_local std::string g_msg;
+
+pf_status fail(pf_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_msg = buf;
+  return s;
+}
+
+#define PF_CUDA(call)                                                                 \
+  do {                                                                                \
+    cudaError_t e_ = (call);                                                          \
+    if (e_ != cudaSuccess) return fail(PF_ERR_CUDA, "%s: %s", #call, cudaGetErrorString(e_)); \
+  } while (0)
+
+// Sub-allocator over a caller buffer: 256-byte aligned slices.
+struct Carve {
+  char* base;
+  size_t off = 0;
+  explicit Carve(void* p) : base(static_cast<char*>(p)) {}
+  template <class T>
+  T* take(size_t n) {
+    off = (off + 255) & ~size_t(255);
+    T* p = base ? reinterpret_cast<T*>(base + off) : nullptr;
+    off += n * sizeof(T);
+    return p;
+  }
+};
+
+// Derived sizes of a validated 1D / 2D layer.
+struct Dims {
+  long B, L, d, nh, P, k1, k2, m, R, rows1, N1, Lp;
+  bool causal, ragged;
+};
+
+Dims dims_of(const pf_layer_desc& s) {
+  Dims g;
+  g.B = s.batch;
+  g.L = s.L;
+  g.d = s.d;
+  g.nh = s.n_heads;
+  g.P = s.P;
+  g.k1 = s.levels == 2 ? s.k1 : s.P;
+  g.k2 = s.levels == 2 ? s.k2 : 1;
+  g.m = (g.L + g.P - 1) / g.P;
+  g.R = g.B * g.m;
+  g.rows1 = g.R * g.k2;
+  g.N1 = g.k1 * g.d;
+  g.Lp = g.m * g.P;
+  g.causal = s.mode == PF_CAUSAL_1D;
+  g.ragged = g.Lp != g.L;
+  return g;
+}
+
+// Buffers the forward saves for the backward pass (order fixes the layout).
+struct Saved {
+  bf16 *Hb, *QKV, *Aatt, *Hbar, *Y, *Z, *D;
+  float* LSE;
+};
+
+Saved carve_saved(Carve& c, const pf_layer_desc& s, const Dims& g) {
+  Saved v{};
+  v.Hb = c.take<bf16>(g.R * g.d);
+  v.QKV = c.take<bf16>(g.R * 3 * g.d);
+  v.Aatt = c.take<bf16>(g.R * g.d);
+  v.Hbar = c.take<bf16>(g.R * g.d);
+  v.LSE = c.take<float>(g.B * g.nh * g.m);
+  if (s.levels == 2) {
+    v.Y = c.take<bf16>(g.rows1 * g.d);
+    v.Z = c.take<bf16>(g.R * g.k2 * g.d);
+  }
+  v.D = c.take<bf16>(g.rows1 * g.N1);
+  return v;
+}
+
+struct BwdWs {
+  bf16 *Xpad, *dD, *dZ, *dHbar, *dA, *dQKV, *dHb, *dY;
+  float *Di, *dHf, *part;
+  long part_elems;
+};
+
+BwdWs carve_bwd(Carve& c, const pf_layer_desc& s, const Dims& g) {
+  BwdWs w{};
+  w.Xpad = g.ragged ? c.take<bf16>(g.B * g.Lp * g.d) : nullptr;
+  w.dD = c.take<bf16>(g.rows1 * g.N1);
+  if (s.levels == 2) w.dZ = c.take<bf16>(g.R * g.k2 * g.d);
+  w.dHbar = c.take<bf16>(g.R * g.d);
+  w.dA = c.take<bf16>(g.R * g.d);
+  w.dQKV = c.take<bf16>(g.R * 3 * g.d);
+  w.dHb = c.take<bf16>(g.R * g.d);
+  if (s.levels == 2) w.dY = c.take<bf16>(g.rows1 * g.d);
+  w.Di = c.take<float>(g.B * g.nh * g.m);
+  w.dHf = c.take<float>(g.R * g.d);
+  long pe = (long)inj_bwd_chunks(g.rows1, (int)g.N1) * 4 * g.N1;
+  pe = std::max(pe, colsum_part_elems(g.R, (int)(g.k2 * g.d)));
+  pe = std::max(pe, colsum_part_elems(g.R, (int)g.d));
+  pe = std::max(pe, colsum_part_elems(g.rows1, (int)g.d));
+  w.part_elems = pe;
+  w.part = c.take<float>(pe);
+  return w;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+pf_status check_desc(const pf_layer_desc* s) {
+  if (s == nullptr) return fail(PF_ERR_INVALID_ARG, "descriptor is NULL");
+  if (s->batch < 1 || s->L < 1) return fail(PF_ERR_INVALID_ARG, "batch and L must be >= 1");
+  if (s->d < 64 || s->d % 64 != 0) return fail(PF_ERR_INVALID_ARG, "d must be a positive multiple of 64");
+  if (s->n_heads < 1 || s->d % s->n_heads != 0)
+    return fail(PF_ERR_INVALID_ARG, "n_heads must divide d");
+  if (s->d / s->n_heads != 64) return fail(PF_ERR_UNSUPPORTED, "head width d/n_heads must be 64");
+  if (s->P < 1) return fail(PF_ERR_INVALID_ARG, "P must be >= 1");
+  if (s->levels != 1 && s->levels != 2) return fail(PF_ERR_INVALID_ARG, "levels must be 1 or 2");
+  if (s->levels == 2 && (s->k1 < 1 || s->k2 < 1 || (long)s->k1 * s->k2 != s->P))
+    return fail(PF_ERR_INVALID_ARG, "levels == 2 needs k1 * k2 == P");
+  if (s->mode < PF_CAUSAL_1D || s->mode > PF_BIDIR_2D) return fail(PF_ERR_INVALID_ARG, "bad mode");
+  if (s->inject < PF_INJ_ADD || s->inject > PF_INJ_AFFINE)
+    return fail(PF_ERR_INVALID_ARG, "bad inject");
+  if (s->dtype != PF_F32 && s->dtype != PF_BF16) return fail(PF_ERR_INVALID_ARG, "bad dtype");
+  if (s->mode == PF_BIDIR_2D) {
+    if (s->patch < 1 || s->patch * s->patch != s->P || s->grid_h < 1 || s->grid_w < 1 ||
+        (long)s->grid_h * s->grid_w != s->L || s->grid_h % s->patch || s->grid_w % s->patch)
+      return fail(PF_ERR_INVALID_ARG, "2D layer needs L = grid_h*grid_w, P = patch^2, patch | grid");
+    return fail(PF_ERR_UNSUPPORTED, "the 2D layer is not built yet");
+  }
+  if (s->inject == PF_INJ_AFFINE) return fail(PF_ERR_UNSUPPORTED, "affine injection is 2D only");
+  if (s->dtype == PF_F32) return fail(PF_ERR_UNSUPPORTED, "fp32 layer is not built yet");
+  const long m = (s->L + (long)s->P - 1) / s->P;
+  const long k1 = s->levels == 2 ? s->k1 : s->P, k2 = s->levels == 2 ? s->k2 : 1;
+  if ((long)s->batch * m * k2 > (1L << 30) || k1 * s->d > (1L << 30))
+    return fail(PF_ERR_UNSUPPORTED, "problem too large for 32-bit GEMM extents");
+  return PF_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* pf_last_error(void) { return g_msg.c_str(); }
+
+pf_status proxy_layer_check(const pf_layer_desc* desc) { return check_desc(desc); }
+
+size_t proxy_layer_saved_size(const pf_layer_desc* desc) {
+  if (check_desc(desc) != PF_OK) return 0;
+  const Dims g = dims_of(*desc);
+  Carve c(nullptr);
+  carve_saved(c, *desc, g);
+  return (c.off + 255) & ~size_t(255);
+}
+
+size_t proxy_layer_workspace_size(const pf_layer_desc* desc, int for_backward) {
+  if (check_desc(desc) != PF_OK) return 0;
+  const Dims g = dims_of(*desc);
+  Carve c(nullptr);
+  if (for_backward) {
+    carve_bwd(c, *desc, g);
+  } else {
+    if (g.ragged) c.take<bf16>(g.B * g.Lp * g.d);
+    carve_saved(c, *desc, g);  // used when the forward is given saved == NULL
+  }
+  return ((c.off + 255) & ~size_t(255)) + 256;
+}
+
+pf_status proxy_layer_fwd(const pf_layer_desc* desc, const pf_layer_params* prm, const void* X,
+                          const float* H_in, const float* t, void* X_out, float* H_out, void* saved,
+                          void* ws, size_t ws_bytes, void* stream) {
+  pf_status st = check_desc(desc);
+  if (st != PF_OK) return st;
+  (void)t;
+  const pf_layer_desc& s = *desc;
+  const Dims g = dims_of(s);
+  if (prm == nullptr || X == nullptr || X_out == nullptr || X == X_out)
+    return fail(PF_ERR_INVALID_ARG, "params, X and X_out are required and must not alias");
+  if (!prm->W_c1 || !prm->b_c1 || !prm->W_qkv || !prm->W_o || !prm->W_d1 || !prm->b_d1 ||
+      (s.levels == 2 && (!prm->W_c2 || !prm->b_c2 || !prm->W_d2 || !prm->b_d2)) ||
+      (s.inject == PF_INJ_GATED && (!prm->w_x || !prm->w_dlt || !prm->b_g)))
+    return fail(PF_ERR_INVALID_ARG, "a parameter this layer uses is NULL");
+  if (!aligned16(X) || !aligned16(X_out) || !aligned16(saved) || !aligned16(ws) ||
+      !aligned16(H_in) || !aligned16(H_out))
+    return fail(PF_ERR_INVALID_ARG, "buffers must be 16-byte aligned");
+  Carve wc(ws);
+  bf16* Xpad = g.ragged ? wc.take<bf16>(g.B * g.Lp * g.d) : nullptr;
+  Carve sc(saved);
+  Saved sv = saved ? carve_saved(sc, s, g) : carve_saved(wc, s, g);
+  if (wc.off > ws_bytes)
+    return fail(PF_ERR_WORKSPACE, "workspace too small: need %zu bytes, got %zu", wc.off, ws_bytes);
+  if (ws == nullptr && wc.off > 0) return fail(PF_ERR_WORKSPACE, "workspace is NULL");
+  cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  const bf16* Xb = static_cast<const bf16*>(X);
+  bf16* Xo = static_cast<bf16*>(X_out);
+  const int d = (int)g.d;
+
+  // a1: partition (a zero-copy view; the ragged tail goes through a padded copy)
+  const bf16* Xsrc = Xb;
+  if (g.ragged) {
+    PF_CUDA(pad_rows(Xb, Xpad, (int)g.B, g.L, g.Lp, d, cs));
+    Xsrc = Xpad;
+  }
+  // a2 + a3: compression (Eq. compress-linear / factor-cascade), H = H_in + C
+  {
+    EpiLinearArgs e;
+    if (s.levels == 1) {
+      e.bias = prm->b_c1;
+      e.addend = H_in;
+      e.ld_add = d;
+      e.out_f32 = H_out;
+      e.ld_f32 = d;
+      e.out_bf16 = sv.Hb;
+      e.ld_bf16 = d;
+      set_gemm_tag("compress_c1", (double)g.R * d * 6.0);
+      PF_CUDA(gemm_linear((int)g.R, d, (int)g.N1, {Xsrc, g.N1, 0},
+                          {static_cast<const bf16*>(prm->W_c1), g.N1, 0}, e, cs));
+    } else {
+      e.bias = prm->b_c1;
+      e.out_bf16 = sv.Y;
+      e.ld_bf16 = d;
+      set_gemm_tag("compress_c1", (double)g.rows1 * d * 2.0);
+      PF_CUDA(gemm_linear((int)g.rows1, d, (int)g.N1, {Xsrc, g.N1, 0},
+                          {static_cast<const bf16*>(prm->W_c1), g.N1, 0}, e, cs));
+      EpiLinearArgs e2;
+      e2.bias = prm->b_c2;
+      e2.addend = H_in;
+      e2.ld_add = d;
+      e2.out_f32 = H_out;
+      e2.ld_f32 = d;
+      e2.out_bf16 = sv.Hb;
+      e2.ld_bf16 = d;
+      set_gemm_tag("compress_c2", (double)g.R * d * 10.0);
+      PF_CUDA(gemm_linear((int)g.R, d, (int)(g.k2 * d), {sv.Y, g.k2 * d, 0},
+                          {static_cast<const bf16*>(prm->W_c2), g.k2 * d, 0}, e2, cs));
+    }
+  }
+  // a4: proxy attention (Eq. proxy-attn)
+  {
+    EpiLinearArgs e;
+    e.out_bf16 = sv.QKV;
+    e.ld_bf16 = 3 * d;
+    set_gemm_tag("proxy_qkv", (double)g.R * 3 * d * 2.0);
+    PF_CUDA(gemm_linear((int)g.R, 3 * d, d, {sv.Hb, d, 0},
+                        {static_cast<const bf16*>(prm->W_qkv), d, 0}, e, cs));
+    PF_CUDA(attn_fwd(sv.QKV, sv.Aatt, sv.LSE, (int)g.B, (int)g.m, d, (int)g.nh, g.causal, cs));
+    EpiLinearArgs eo;
+    eo.out_bf16 = sv.Hbar;
+    eo.ld_bf16 = d;
+    set_gemm_tag("proxy_o", (double)g.R * d * 2.0);
+    PF_CUDA(gemm_linear((int)g.R, d, d, {sv.Aatt, d, 0}, {static_cast<const bf16*>(prm->W_o), d, 0},
+                        eo, cs));
+  }
+  // a5 + a6: decompression (Eq. decompress-linear / factor-dec), routing and
+  // injection (Eq. inj-gate / inj-add), fused into the last level's GEMM
+  const bf16* Zsrc = sv.Hbar;
+  if (s.levels == 2) {
+    EpiLinearArgs e;
+    e.bias = prm->b_d2;
+    e.out_bf16 = sv.Z;
+    e.ld_bf16 = g.k2 * d;
+    set_gemm_tag("decompress_d2", (double)g.R * g.k2 * d * 2.0);
+    PF_CUDA(gemm_linear((int)g.R, (int)(g.k2 * d), d, {sv.Hbar, d, 0},
+                        {static_cast<const bf16*>(prm->W_d2), d, 0}, e, cs));
+    Zsrc = sv.Z;
+  }
+  {
+    EpiInjectArgs e{prm->b_d1, sv.D, Xb, Xo,
+                    prm->w_x, prm->w_dlt, prm->b_g,
+                    d, (int)g.k1, (int)g.k2, (int)g.m, (int)g.L, g.causal ? 1 : 0,
+                    s.inject == PF_INJ_GATED ? 1 : 0};
+    set_gemm_tag("decompress_d1_inject", (double)g.rows1 * g.N1 * 8.0);
+    PF_CUDA(gemm_inject1d((int)g.rows1, (int)g.N1, d, {Zsrc, d, 0},
+                          {static_cast<const bf16*>(prm->W_d1), d, 0}, e, cs));
+  }
+  if (g.causal) PF_CUDA(copy_block0(Xb, Xo, (int)g.B, g.L, d, (int)std::min(g.P, g.L), cs));
+  return PF_OK;
+}
+
+pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm, const void* X,
+                          const float* H_in, const float* t, const void* saved, const void* dX_out,
+                          const float* dH_out, void* dX, float* dH_in, const pf_layer_grads* grads,
+                          void* ws, size_t ws_bytes, void* stream) {
+  pf_status st = check_desc(desc);
+  if (st != PF_OK) return st;
+  (void)H_in;
+  (void)t;
+  const pf_layer_desc& s = *desc;
+  const Dims g = dims_of(s);
+  if (!prm || !X || !saved || !dX_out || !dX || !grads)
+    return fail(PF_ERR_INVALID_ARG, "params, X, saved, dX_out, dX and grads are required");
+  if (!aligned16(X) || !aligned16(saved) || !aligned16(dX_out) || !aligned16(dX) ||
+      !aligned16(ws) || !aligned16(dH_out) || !aligned16(dH_in))
+    return fail(PF_ERR_INVALID_ARG, "buffers must be 16-byte aligned");
+  const bool gated = s.inject == PF_INJ_GATED;
+  if (!grads->b_d1 || (gated && (!grads->w_x || !grads->w_dlt || !grads->b_g)))
+    return fail(PF_ERR_INVALID_ARG, "grads->b_d1 (and the gate gradients) must be given");
+  Carve wc(ws);
+  BwdWs w = carve_bwd(wc, s, g);
+  if (ws == nullptr || wc.off > ws_bytes)
+    return fail(PF_ERR_WORKSPACE, "workspace too small: need %zu bytes, got %zu", wc.off, ws_bytes);
+  Carve sc(const_cast<void*>(saved));
+  const Saved sv = carve_saved(sc, s, g);
+  cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  const bf16* Xb = static_cast<const bf16*>(X);
+  const bf16* G = static_cast<const bf16*>(dX_out);
+  bf16* dXb = static_cast<bf16*>(dX);
+  const int d = (int)g.d, N1 = (int)g.N1;
+  const bf16* W_c1 = static_cast<const bf16*>(prm->W_c1);
+  const bf16* W_c2 = static_cast<const bf16*>(prm->W_c2);
+  const bf16* W_qkv = static_cast<const bf16*>(prm->W_qkv);
+  const bf16* W_o = static_cast<const bf16*>(prm->W_o);
+  const bf16* W_d2 = static_cast<const bf16*>(prm->W_d2);
+  const bf16* W_d1 = static_cast<const bf16*>(prm->W_d1);
+
+  const bf16* Xsrc = Xb;
+  if (g.ragged) {
+    PF_CUDA(pad_rows(Xb, w.Xpad, (int)g.B, g.L, g.Lp, d, cs));
+    Xsrc = w.Xpad;
+  }
+  // injection backward: dD (proxy order), direct dX, gate and b_d1 gradients
+  {
+    const int nch = inj_bwd_chunks(g.rows1, N1);
+    InjBwdArgs a{G, Xb, sv.D, w.dD, dXb, prm->w_x, prm->w_dlt, prm->b_g,
+                 d, (int)g.k1, (int)g.k2, (int)g.m, (int)g.L, (int)g.B, g.causal ? 1 : 0,
+                 gated ? 1 : 0};
+    PF_CUDA(inj_bwd_1d(a, w.part, nch, cs));
+    if (g.causal) PF_CUDA(copy_block0(G, dXb, (int)g.B, g.L, d, (int)std::min(g.P, g.L), cs));
+    PF_CUDA(inj_bwd_finalize(w.part, nch, N1, d, grads->b_d1, gated ? grads->w_x : nullptr,
+                             gated ? grads->w_dlt : nullptr, gated ? grads->b_g : nullptr, cs));
+  }
+  // decompression level 1 (or single level)
+  const bf16* Zsrc = s.levels == 2 ? sv.Z : sv.Hbar;
+  if (grads->W_d1) {
+    EpiLinearArgs e;
+    e.out_f32 = grads->W_d1;
+    e.ld_f32 = d;
+    set_gemm_tag("bwd_dW_d1", (double)N1 * d * 4.0);
+    PF_CUDA(gemm_linear(N1, d, (int)g.rows1, {w.dD, N1, 1}, {Zsrc, d, 1}, e, cs));
+  }
+  {
+    EpiLinearArgs e;
+    e.out_bf16 = s.levels == 2 ? w.dZ : w.dHbar;
+    e.ld_bf16 = d;
+    set_gemm_tag("bwd_dZ", (double)g.rows1 * d * 2.0);
+    PF_CUDA(gemm_linear((int)g.rows1, d, N1, {w.dD, N1, 0}, {W_d1, d, 1}, e, cs));
+  }
+  if (s.levels == 2) {
+    const int n2 = (int)(g.k2 * d);
+    if (grads->b_d2) PF_CUDA(colsum_bf16(w.dZ, g.R, n2, grads->b_d2, w.part, cs));
+    if (grads->W_d2) {
+      EpiLinearArgs e;
+      e.out_f32 = grads->W_d2;
+      e.ld_f32 = d;
+      set_gemm_tag("bwd_dW_d2", (double)n2 * d * 4.0);
+      PF_CUDA(gemm_linear(n2, d, (int)g.R, {w.dZ, n2, 1}, {sv.Hbar, d, 1}, e, cs));
+    }
+    EpiLinearArgs e;
+    e.out_bf16 = w.dHbar;
+    e.ld_bf16 = d;
+    set_gemm_tag("bwd_dHbar", (double)g.R * d * 2.0);
+    PF_CUDA(gemm_linear((int)g.R, d, n2, {w.dZ, n2, 0}, {W_d2, d, 1}, e, cs));
+  }
+  // attention output projection and attention
+  if (grads->W_o) {
+    EpiLinearArgs e;
+    e.out_f32 = grads->W_o;
+    e.ld_f32 = d;
+    set_gemm_tag("bwd_dW_o", (double)d * d * 4.0);
+    PF_CUDA(gemm_linear(d, d, (int)g.R, {w.dHbar, d, 1}, {sv.Aatt, d, 1}, e, cs));
+  }
+  {
+    EpiLinearArgs e;
+    e.out_bf16 = w.dA;
+    e.ld_bf16 = d;
+    set_gemm_tag("bwd_dA", (double)g.R * d * 2.0);
+    PF_CUDA(gemm_linear((int)g.R, d, d, {w.dHbar, d, 0}, {W_o, d, 1}, e, cs));
+  }
+  PF_CUDA(attn_bwd(sv.QKV, sv.Aatt, w.dA, sv.LSE, w.Di, w.dQKV, (int)g.B, (int)g.m, d, (int)g.nh,
+                   g.causal, cs));
+  if (grads->W_qkv) {
+    EpiLinearArgs e;
+    e.out_f32 = grads->W_qkv;
+    e.ld_f32 = d;
+    set_gemm_tag("bwd_dW_qkv", (double)3 * d * d * 4.0);
+    PF_CUDA(gemm_linear(3 * d, d, (int)g.R, {w.dQKV, 3 * d, 1}, {sv.Hb, d, 1}, e, cs));
+  }
+  float* dHf = dH_in ? dH_in : w.dHf;
+  {
+    EpiLinearArgs e;
+    e.addend = dH_out;
+    e.ld_add = d;
+    e.out_f32 = dHf;
+    e.ld_f32 = d;
+    e.out_bf16 = w.dHb;
+    e.ld_bf16 = d;
+    set_gemm_tag("bwd_dH", (double)g.R * d * 10.0);
+    PF_CUDA(gemm_linear((int)g.R, d, 3 * d, {w.dQKV, 3 * d, 0}, {W_qkv, d, 1}, e, cs));
+  }
+  // compression (H = H_in + C, so dC = dH)
+  const bf16* dYsrc = w.dHb;
+  if (s.levels == 2) {
+    const int n2 = (int)(g.k2 * d);
+    if (grads->b_c2) PF_CUDA(colsum_f32(dHf, g.R, d, grads->b_c2, w.part, cs));
+    if (grads->W_c2) {
+      EpiLinearArgs e;
+      e.out_f32 = grads->W_c2;
+      e.ld_f32 = n2;
+      set_gemm_tag("bwd_dW_c2", (double)d * n2 * 4.0);
+      PF_CUDA(gemm_linear(d, n2, (int)g.R, {w.dHb, d, 1}, {sv.Y, n2, 1}, e, cs));
+    }
+    EpiLinearArgs e;
+    e.out_bf16 = w.dY;
+    e.ld_bf16 = n2;
+    set_gemm_tag("bwd_dY", (double)g.R * n2 * 2.0);
+    PF_CUDA(gemm_linear((int)g.R, n2, d, {w.dHb, d, 0}, {W_c2, n2, 1}, e, cs));
+    if (grads->b_c1) PF_CUDA(colsum_bf16(w.dY, g.rows1, d, grads->b_c1, w.part, cs));
+    dYsrc = w.dY;
+  } else if (grads->b_c1) {
+    PF_CUDA(colsum_f32(dHf, g.R, d, grads->b_c1, w.part, cs));
+  }
+  if (grads->W_c1) {
+    EpiLinearArgs e;
+    e.out_f32 = grads->W_c1;
+    e.ld_f32 = N1;
+    set_gemm_tag("bwd_dW_c1", (double)d * N1 * 4.0);
+    PF_CUDA(gemm_linear(d, N1, (int)g.rows1, {dYsrc, d, 1}, {Xsrc, N1, 1}, e, cs));
+  }
+  {
+    EpiDXArgs e{dXb, d, (int)g.k1, (int)g.k2, (int)g.m, (int)g.L};
+    set_gemm_tag("bwd_dX", (double)g.rows1 * N1 * 4.0);
+    PF_CUDA(gemm_dx1d((int)g.rows1, N1, d, {dYsrc, d, 0}, {W_c1, N1, 1}, e, cs));
+  }
+  return PF_OK;
+}
+
+size_t proxy_decode_workspace_size(const pf_decode_desc* desc) {
+  (void)desc;
+  return 0;
+}
+size_t proxy_append_workspace_size(const pf_decode_desc* desc) {
+  (void)desc;
+  return 0;
+}
+
+pf_status proxy_decode_step(const pf_decode_desc* desc, const pf_decode_params* params,
+                            const void* x, pf_kv_cache* cache, void* y, void* ws, size_t ws_bytes,
+                            void* stream) {
+  (void)desc; (void)params; (void)x; (void)cache; (void)y; (void)ws; (void)ws_bytes; (void)stream;
+  return fail(PF_ERR_UNSUPPORTED, "decode step is not built yet");
+}
+
+pf_status proxy_kv_append(const pf_decode_desc* desc, const pf_append_params* params,
+                          const float* H_in, pf_kv_cache* cache, void* ws, size_t ws_bytes,
+                          void* stream) {
+  (void)desc; (void)params; (void)H_in; (void)cache; (void)ws; (void)ws_bytes; (void)stream;
+  return fail(PF_ERR_UNSUPPORTED, "KV append is not built yet");
+}
+
+pf_status pf_sync_check(void* stream) {
+  PF_CUDA(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
+  PF_CUDA(cudaGetLastError());
+  int e = 0;
+  for (int v : {take_dev_error_gemm(), take_dev_error_attention(), take_dev_error_elementwise()})
+    if (v != 0 && e == 0) e = v;
+  if (e < 0) return fail(PF_ERR_CUDA, "reading the device error flag failed");
+  if (e == DEVERR_TIMEOUT) return fail(PF_ERR_TIMEOUT, "a kernel's bounded wait ran out");
+  if (e == DEVERR_CAPACITY) return fail(PF_ERR_CAPACITY, "cache bookkeeping violated in a kernel");
+  return PF_OK;
+}
+
+pf_status pf_gemm_bf16(int M, int N, int K, const void* A, int a_mn, const void* B, int b_mn,
+                       float* D, int ldd, void* stream) {
+  if (M < 1 || N < 1 || K < 1 || N % 32 != 0 || !A || !B || !D || ldd < N || ldd % 4 != 0)
+    return fail(PF_ERR_INVALID_ARG, "pf_gemm_bf16: bad sizes or pointers (N must be a multiple of 32)");
+  const long lda = a_mn ? M : K, ldb = b_mn ? N : K;
+  if ((lda * 2) % 16 || (ldb * 2) % 16)
+    return fail(PF_ERR_INVALID_ARG, "pf_gemm_bf16: rows must be multiples of 16 bytes");
+  EpiLinearArgs e;
+  e.out_f32 = D;
+  e.ld_f32 = ldd;
+  set_gemm_tag("pf_gemm_bf16", (double)M * N * 4.0);
+  PF_CUDA(gemm_linear(M, N, K, {static_cast<const bf16*>(A), lda, a_mn ? 1 : 0},
+                      {static_cast<const bf16*>(B), ldb, b_mn ? 1 : 0}, e,
+                      static_cast<cudaStream_t>(stream)));
+  return PF_OK;
+}
+
+}  // extern "C"

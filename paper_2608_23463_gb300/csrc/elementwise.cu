@@ -1,0 +1,236 @@
+// Bandwidth-bound kernels of the layer: injection backward with its column
+// reductions, deterministic column sums (bias gradients), block-0 copies and
+// zero padding.  All accesses are 16-byte vectors over contiguous rows.
+#include "kernels.h"
+
+namespace pf {
+
+namespace {
+
+constexpr int EW_THREADS = 256;
+
+__global__ void copy_block0_kernel(const bf16* __restrict__ src, bf16* __restrict__ dst, long L,
+                                   int d, long per_seq_vec) {
+  const long i = (long)blockIdx.x * blockDim.x + threadIdx.x;
+  const int b = blockIdx.y;
+  if (i >= per_seq_vec) return;
+  const long off = (long)b * L * d + i * 8;
+  *reinterpret_cast<uint4*>(dst + off) = *reinterpret_cast<const uint4*>(src + off);
+}
+
+__global__ void pad_rows_kernel(const bf16* __restrict__ src, bf16* __restrict__ dst, long L,
+                                long Lp, int d) {
+  const long i = (long)blockIdx.x * blockDim.x + threadIdx.x;  // vector index in [Lp*d/8]
+  const int b = blockIdx.y;
+  if (i >= Lp * d / 8) return;
+  const long tok = i * 8 / d;
+  uint4 v = make_uint4(0, 0, 0, 0);
+  if (tok < L) v = *reinterpret_cast<const uint4*>(src + (long)b * L * d + i * 8);
+  *reinterpret_cast<uint4*>(dst + (long)b * Lp * d + i * 8) = v;
+}
+
+__global__ void __launch_bounds__(EW_THREADS) inj_bwd_kernel(InjBwdArgs a, float* __restrict__ part,
+                                                             long M, int N, long rows_per_chunk) {
+  const int col = (blockIdx.x * EW_THREADS + threadIdx.x) * 8;
+  if (col >= N) return;
+  const long r0 = (long)blockIdx.y * rows_per_chunk;
+  const long r1 = min(M, r0 + rows_per_chunk);
+  const int P = a.k1 * a.k2;
+  const int ch = col % a.d, tq = col / a.d;
+  float wx[8], wd[8], bg[8];
+  if (a.gated) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      wx[j] = a.w_x[ch + j];
+      wd[j] = a.w_dlt[ch + j];
+      bg[j] = a.b_g[ch + j];
+    }
+  }
+  float acc[4][8] = {};
+  for (long r = r0; r < r1; ++r) {
+    const int grp = (int)(r % a.k2);
+    const long prox = r / a.k2;
+    const int b = (int)(prox / a.m), i = (int)(prox % a.m);
+    const int it = i + a.shift;
+    const long tok = (long)it * P + (long)grp * a.k1 + tq;
+    float dd[8];
+    if (it < a.m && tok < a.L) {
+      const long off = ((long)b * a.L + tok) * a.d + ch;
+      float g[8], x[8], D[8], dx[8];
+      load8_bf16(a.G + off, g);
+      load8_bf16(a.X + off, x);
+      load8_bf16(a.D + r * N + col, D);
+      if (a.gated) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const float s = sigmoidf_(wx[j] * x[j] + wd[j] * D[j] + bg[j]);
+          const float ds = g[j] * D[j] * s * (1.f - s);
+          dx[j] = g[j] + ds * wx[j];
+          dd[j] = g[j] * s + ds * wd[j];
+          acc[1][j] += ds * x[j];
+          acc[2][j] += ds * D[j];
+          acc[3][j] += ds;
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          dx[j] = g[j];
+          dd[j] = g[j];
+        }
+      }
+      store8_bf16(a.dX + off, dx);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 8; ++j) dd[j] = 0.f;
+    }
+    // round dD once; the column sum uses the same rounded values the
+    // downstream GEMMs see.
+    store8_bf16(a.dD + r * N + col, dd);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc[0][j] += __bfloat162float(__float2bfloat16(dd[j]));
+  }
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    float* p = part + ((long)blockIdx.y * 4 + q) * N + col;
+    *reinterpret_cast<float4*>(p) = make_float4(acc[q][0], acc[q][1], acc[q][2], acc[q][3]);
+    *reinterpret_cast<float4*>(p + 4) = make_float4(acc[q][4], acc[q][5], acc[q][6], acc[q][7]);
+  }
+}
+
+__global__ void inj_bwd_finalize_kernel(const float* __restrict__ part, int n_chunks, int N, int d,
+                                        float* db_d1, float* gw_x, float* gw_dlt, float* gb_g) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < N) {
+    float s = 0.f;
+    for (int c = 0; c < n_chunks; ++c) s += part[((long)c * 4) * N + i];
+    db_d1[i] = s;
+    return;
+  }
+  const int j = i - N;
+  if (gw_x == nullptr || j >= 3 * d) return;
+  const int q = 1 + j / d, ch = j % d;
+  float s = 0.f;
+  for (int c = 0; c < n_chunks; ++c)
+    for (int t = 0; t < N / d; ++t) s += part[((long)c * 4 + q) * N + t * d + ch];
+  float* dst = q == 1 ? gw_x : (q == 2 ? gw_dlt : gb_g);
+  dst[ch] = s;
+}
+
+template <typename T>
+__device__ __forceinline__ void load8(const T* p, float* v);
+template <>
+__device__ __forceinline__ void load8<bf16>(const bf16* p, float* v) {
+  load8_bf16(p, v);
+}
+template <>
+__device__ __forceinline__ void load8<float>(const float* p, float* v) {
+  const float4 a = *reinterpret_cast<const float4*>(p), b = *reinterpret_cast<const float4*>(p + 4);
+  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+
+template <typename T>
+__global__ void __launch_bounds__(EW_THREADS) colsum_part_kernel(const T* __restrict__ X, long R,
+                                                                 int C, long rows_per_chunk,
+                                                                 float* __restrict__ part) {
+  const int col = (blockIdx.x * EW_THREADS + threadIdx.x) * 8;
+  if (col >= C) return;
+  const long r0 = (long)blockIdx.y * rows_per_chunk, r1 = min(R, r0 + rows_per_chunk);
+  float acc[8] = {};
+  for (long r = r0; r < r1; ++r) {
+    float v[8];
+    load8<T>(X + r * C + col, v);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc[j] += v[j];
+  }
+  float* p = part + (long)blockIdx.y * C + col;
+  *reinterpret_cast<float4*>(p) = make_float4(acc[0], acc[1], acc[2], acc[3]);
+  *reinterpret_cast<float4*>(p + 4) = make_float4(acc[4], acc[5], acc[6], acc[7]);
+}
+
+__global__ void colsum_final_kernel(const float* __restrict__ part, int n_chunks, int C,
+                                    float* __restrict__ out) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= C) return;
+  float s = 0.f;
+  for (int c = 0; c < n_chunks; ++c) s += part[(long)c * C + i];
+  out[i] = s;
+}
+
+// Row chunks of a column reduction: about 1024 CTAs in total, independent of
+// the device so that results (summation order) and workspace sizes are fixed.
+int chunks_for(long R, int C) {
+  const int gx = (C / 8 + EW_THREADS - 1) / EW_THREADS;
+  long want = (1024 + gx - 1) / gx;
+  if (want > R) want = R;
+  if (want < 1) want = 1;
+  return (int)want;
+}
+
+template <typename T>
+cudaError_t colsum_impl(const T* X, long R, int C, float* out, float* part, cudaStream_t st) {
+  const int nc = chunks_for(R, C);
+  const long rpc = (R + nc - 1) / nc;
+  dim3 grid((C / 8 + EW_THREADS - 1) / EW_THREADS, nc);
+  {
+    LaunchTimer lt("colsum", st, (double)R * C, (double)R * C * sizeof(T));
+    colsum_part_kernel<T><<<grid, EW_THREADS, 0, st>>>(X, R, C, rpc, part);
+  }
+  {
+    LaunchTimer lt("colsum_final", st, (double)nc * C, 4.0 * nc * C);
+    colsum_final_kernel<<<(C + 255) / 256, 256, 0, st>>>(part, nc, C, out);
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t copy_block0(const bf16* src, bf16* dst, int B, long L, int d, int rows,
+                        cudaStream_t st) {
+  const long nvec = (long)rows * d / 8;
+  dim3 grid((unsigned)((nvec + 255) / 256), B);
+  LaunchTimer lt("copy_block0", st, 0.0, 32.0 * nvec * B);
+  copy_block0_kernel<<<grid, 256, 0, st>>>(src, dst, L, d, nvec);
+  return cudaGetLastError();
+}
+
+cudaError_t pad_rows(const bf16* src, bf16* dst, int B, long L, long Lp, int d, cudaStream_t st) {
+  const long nvec = Lp * d / 8;
+  dim3 grid((unsigned)((nvec + 255) / 256), B);
+  LaunchTimer lt("pad_rows", st, 0.0, 2.0 * B * (L + Lp) * d);
+  pad_rows_kernel<<<grid, 256, 0, st>>>(src, dst, L, Lp, d);
+  return cudaGetLastError();
+}
+
+int inj_bwd_chunks(long M, int N) { return chunks_for(M, N); }
+
+int take_dev_error_elementwise() { return take_dev_error_tu(); }
+
+cudaError_t inj_bwd_1d(const InjBwdArgs& a, float* part, int n_chunks, cudaStream_t st) {
+  const long M = (long)a.B * a.m * a.k2;
+  const int N = a.k1 * a.d;
+  const long rpc = (M + n_chunks - 1) / n_chunks;
+  dim3 grid((N / 8 + EW_THREADS - 1) / EW_THREADS, n_chunks);
+  LaunchTimer lt("inj_bwd", st, 0.0, 10.0 * M * N + 16.0 * n_chunks * N);
+  inj_bwd_kernel<<<grid, EW_THREADS, 0, st>>>(a, part, M, N, rpc);
+  return cudaGetLastError();
+}
+
+cudaError_t inj_bwd_finalize(const float* part, int n_chunks, int N, int d, float* db_d1,
+                             float* gw_x, float* gw_dlt, float* gb_g, cudaStream_t st) {
+  const int total = N + 3 * d;
+  LaunchTimer lt("inj_bwd_finalize", st, 0.0, 16.0 * n_chunks * N);
+  inj_bwd_finalize_kernel<<<(total + 255) / 256, 256, 0, st>>>(part, n_chunks, N, d, db_d1, gw_x,
+                                                              gw_dlt, gb_g);
+  return cudaGetLastError();
+}
+
+long colsum_part_elems(long R, int C) { return (long)chunks_for(R, C) * C; }
+
+cudaError_t colsum_bf16(const bf16* X, long R, int C, float* out, float* part, cudaStream_t st) {
+  return colsum_impl<bf16>(X, R, C, out, part, st);
+}
+cudaError_t colsum_f32(const float* X, long R, int C, float* out, float* part, cudaStream_t st) {
+  return colsum_impl<float>(X, R, C, out, part, st);
+}
+
+}  // namespace pf

@@ -1,0 +1,124 @@
+// Host side of the tcgen05 GEMM: TMA tensor maps, tile-width choice and the
+// instantiations used by the layer (see gemm_tc.cuh for the kernel).
+#include <cudaTypedefs.h>
+
+#include "gemm_tc.cuh"
+#include "kernels.h"
+
+namespace pf {
+
+int take_dev_error_gemm() { return take_dev_error_tu(); }
+
+int num_sms() {
+  static int n = 0;
+  if (n == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    if (n <= 0) n = 148;
+  }
+  return n;
+}
+
+namespace {
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (fn == nullptr) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// 2D bf16 map over a row-major [outer, inner] matrix with `ld` elements per
+// row, 128-byte swizzle, zero fill outside the matrix.
+bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t ld,
+              uint32_t box_inner, uint32_t box_outer) {
+  auto fn = encode_fn();
+  if (fn == nullptr) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {ld * 2};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t es[2] = {1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// rows = M (for A) or N (for B).
+bool make_operand_map(CUtensorMap* m, const Operand& op, int rows, int K) {
+  if (op.mn) return make_map(m, op.ptr, (uint64_t)rows, (uint64_t)K, (uint64_t)op.ld, 64, 64);
+  return make_map(m, op.ptr, (uint64_t)K, (uint64_t)rows, (uint64_t)op.ld, 64, 128);
+}
+
+template <int BN, bool AMN, bool BMN, class Epi>
+cudaError_t launch(int M, int N, int K, const CUtensorMap& ta, const CUtensorMap& tb, const Epi& epi,
+                   cudaStream_t st) {
+  auto kern = gemm_tc_kernel<BN, AMN, BMN, Epi, BRowsLinear>;
+  constexpr int smem = GemmCfg<BN>::SMEM_BYTES;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  if (e != cudaSuccess) return e;
+  dim3 grid((N + BN - 1) / BN, (M + GEMM_BM - 1) / GEMM_BM);
+  kern<<<grid, GEMM_THREADS, smem, st>>>(ta, tb, M, N, K, epi, BRowsLinear{});
+  return cudaGetLastError();
+}
+
+template <int BN, class Epi>
+cudaError_t launch_majors(int M, int N, int K, const Operand& A, const Operand& B,
+                          const CUtensorMap& ta, const CUtensorMap& tb, const Epi& epi,
+                          cudaStream_t st) {
+  if (!A.mn && !B.mn) return launch<BN, false, false>(M, N, K, ta, tb, epi, st);
+  if (!A.mn && B.mn) return launch<BN, false, true>(M, N, K, ta, tb, epi, st);
+  if (A.mn && B.mn) return launch<BN, true, true>(M, N, K, ta, tb, epi, st);
+  return launch<BN, true, false>(M, N, K, ta, tb, epi, st);
+}
+
+bool operand_ok(const Operand& op) {
+  return op.ptr != nullptr && (reinterpret_cast<uintptr_t>(op.ptr) & 15) == 0 && op.ld > 0 &&
+         (op.ld * 2) % 16 == 0;
+}
+
+template <class Epi>
+cudaError_t gemm_dispatch(int M, int N, int K, Operand A, Operand B, const Epi& epi,
+                          cudaStream_t st) {
+  if (M <= 0 || N <= 0 || N % 32 != 0 || K < 0 || !operand_ok(A) || !operand_ok(B))
+    return cudaErrorInvalidValue;
+  CUtensorMap ta, tb;
+  if (!make_operand_map(&ta, A, M, K) || !make_operand_map(&tb, B, N, K))
+    return cudaErrorInvalidValue;
+  const long tiles256 = (long)((N + 255) / 256) * ((M + GEMM_BM - 1) / GEMM_BM);
+  LaunchTimer lt(gemm_tag_label(), st, 2.0 * M * N * (double)K,
+                 2.0 * ((double)M * K + (double)N * K) + gemm_tag_bytes());
+  if (N >= 256 && tiles256 >= num_sms()) return launch_majors<256>(M, N, K, A, B, ta, tb, epi, st);
+  return launch_majors<128>(M, N, K, A, B, ta, tb, epi, st);
+}
+
+}  // namespace
+
+cudaError_t gemm_linear(int M, int N, int K, Operand A, Operand B, const EpiLinearArgs& e,
+                        cudaStream_t st) {
+  EpiLinear epi{M, N, e.bias, e.addend, e.ld_add, e.out_f32, e.ld_f32, e.out_bf16, e.ld_bf16};
+  return gemm_dispatch(M, N, K, A, B, epi, st);
+}
+
+cudaError_t gemm_inject1d(int M, int N, int K, Operand A, Operand B, const EpiInjectArgs& e,
+                          cudaStream_t st) {
+  EpiInject1D epi{M, N, e.bias, e.D_save, e.X, e.X_out, e.w_x, e.w_dlt, e.b_g,
+                  e.d, e.k1, e.k2, e.m, e.L, e.shift, e.gated};
+  if (A.mn || B.mn) return cudaErrorInvalidValue;
+  return gemm_dispatch(M, N, K, A, B, epi, st);
+}
+
+cudaError_t gemm_dx1d(int M, int N, int K, Operand A, Operand B, const EpiDXArgs& e,
+                      cudaStream_t st) {
+  EpiDX1D epi{M, N, e.dX, e.d, e.k1, e.k2, e.m, e.L};
+  if (A.mn || !B.mn) return cudaErrorInvalidValue;
+  return gemm_dispatch(M, N, K, A, B, epi, st);
+}
+
+}  // namespace pf

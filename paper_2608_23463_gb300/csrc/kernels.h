@@ -1,0 +1,114 @@
+// Internal launch interface between the C ABI (api.cu) and the kernels.
+#pragma once
+
+#include "common.cuh"
+
+namespace pf {
+
+// ------------------------------------------------------------------ GEMM
+// Operand of D[M,N] = sum_k A[m,k] B[n,k]: `mn` = 0 for K-major storage
+// ([rows=M or N, K], leading dimension ld >= K), 1 for MN-major storage
+// ([K, M or N], ld >= M or N).  bf16, 16-byte aligned, ld*2 % 16 == 0.
+struct Operand {
+  const bf16* ptr;
+  long ld;
+  int mn;
+};
+
+struct EpiLinearArgs {
+  const float* bias = nullptr;    // [N]
+  const float* addend = nullptr;  // [M, ld_add] fp32
+  long ld_add = 0;
+  float* out_f32 = nullptr;
+  long ld_f32 = 0;
+  bf16* out_bf16 = nullptr;
+  long ld_bf16 = 0;
+};
+
+struct EpiInjectArgs {
+  const float* bias;  // b_d1 [k1*d]
+  bf16* D_save;       // [M, k1*d] or null
+  const bf16* X;
+  bf16* X_out;
+  const float *w_x, *w_dlt, *b_g;  // gate vectors (gated) or null (add)
+  int d, k1, k2, m, L, shift, gated;
+};
+
+struct EpiDXArgs {
+  bf16* dX;
+  int d, k1, k2, m, L;
+};
+
+cudaError_t gemm_linear(int M, int N, int K, Operand A, Operand B, const EpiLinearArgs& e,
+                        cudaStream_t st);
+cudaError_t gemm_inject1d(int M, int N, int K, Operand A, Operand B, const EpiInjectArgs& e,
+                          cudaStream_t st);
+cudaError_t gemm_dx1d(int M, int N, int K, Operand A, Operand B, const EpiDXArgs& e,
+                      cudaStream_t st);
+int num_sms();
+
+// Per-file device error flags (see common.cuh): value, cleared on read.
+int take_dev_error_gemm();
+int take_dev_error_attention();
+int take_dev_error_elementwise();
+
+// ------------------------------------------------------------- attention
+cudaError_t attn_fwd(const bf16* qkv, bf16* out, float* lse, int B, int m, int d, int nh,
+                     bool causal, cudaStream_t st);
+cudaError_t attn_bwd(const bf16* qkv, const bf16* O, const bf16* dO, const float* lse, float* Di,
+                     bf16* dqkv, int B, int m, int d, int nh, bool causal, cudaStream_t st);
+
+// ----------------------------------------------------------- elementwise
+// Copy `rows_per_seq` rows of width d from the start of each sequence of src
+// [B, L, d] to dst (block 0 of the causal routing: X_out = X, dX = dX_out).
+cudaError_t copy_block0(const bf16* src, bf16* dst, int B, long L, int d, int rows,
+                        cudaStream_t st);
+// dst [B, Lp, d] = src [B, L, d] padded with zero rows (Lp >= L).
+cudaError_t pad_rows(const bf16* src, bf16* dst, int B, long L, long Lp, int d, cudaStream_t st);
+
+// Backward of the 1D injection (Eq. inj-gate / inj-add) in proxy order.
+// Rows r of D / dD are [M = B*m*k2, N = k1*d]; row r's values belong to the
+// tokens of block i + shift.  Writes dD (zero where no token exists), the
+// direct gradient into dX, and fills `part` [n_chunks][4][N] partial column
+// sums (dD, ds*X, ds*D, ds with ds = G*D*s*(1-s)).  Returns n_chunks via out.
+struct InjBwdArgs {
+  const bf16* G;
+  const bf16* X;
+  const bf16* D;
+  bf16* dD;
+  bf16* dX;
+  const float *w_x, *w_dlt, *b_g;
+  int d, k1, k2, m, L, B, shift, gated;
+};
+int inj_bwd_chunks(long M, int N);
+cudaError_t inj_bwd_1d(const InjBwdArgs& a, float* part, int n_chunks, cudaStream_t st);
+// Reduce the partials: db_d1[c] = sum part[.][0][c]; gate grads (if non-null)
+// summed over chunks and the k1 token positions: g[ch] = sum part[.][j][q*d+ch].
+cudaError_t inj_bwd_finalize(const float* part, int n_chunks, int N, int d, float* db_d1,
+                             float* gw_x, float* gw_dlt, float* gb_g, cudaStream_t st);
+
+// out[c] = sum_r X[r, c] for a row-major [R, C] matrix (bf16 or fp32),
+// deterministic two-pass reduction using `part` (colsum_part_elems floats).
+long colsum_part_elems(long R, int C);
+cudaError_t colsum_bf16(const bf16* X, long R, int C, float* out, float* part, cudaStream_t st);
+cudaError_t colsum_f32(const float* X, long R, int C, float* out, float* part, cudaStream_t st);
+
+}  // namespace pf
+
+namespace pf {
+// ------------------------------------------------------------ launch timing
+// When enabled (pf_timing_enable), every kernel launch of the library is
+// bracketed by CUDA events recorded on its own stream and tagged with a label
+// and its algorithmic work; pf_timing_collect aggregates them after the caller
+// has synchronised.  Disabled, a LaunchTimer does nothing.
+struct LaunchTimer {
+  LaunchTimer(const char* label, cudaStream_t st, double flops, double bytes);
+  ~LaunchTimer();
+  int idx;
+  cudaStream_t st;
+};
+// Label (and epilogue bytes) of the next GEMM launches, set by the caller.
+void set_gemm_tag(const char* label, double epi_bytes);
+const char* gemm_tag_label();
+double gemm_tag_bytes();
+}  // namespace pf

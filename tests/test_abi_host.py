@@ -1,0 +1,88 @@
+"""Host-side checks of the C ABI (no GPU): the library builds, loads and exports
+every entry point declared in include/proxyformer.h; descriptor validation and
+workspace queries behave as documented."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import pf_synth as S
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def pf():
+    import paper_2608_23463_gb300 as pf
+    from paper_2608_23463_gb300.buildlib import build
+    build()
+    pf.load()
+    return pf
+
+
+def declared_functions():
+    txt = open(os.path.join(ROOT, "include", "proxyformer.h")).read()
+    txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:pf_status|size_t|const char\s*\*|void|int|double)\s*\**\s*(\w+)\s*\(",
+                                 txt, flags=re.M)))
+
+
+def test_every_declared_symbol_is_exported(pf):
+    names = declared_functions()
+    assert len(names) >= 12, names
+    lib = ctypes.CDLL(pf.LIB_PATH)
+    for n in names:
+        assert hasattr(lib, n), f"{n} declared in proxyformer.h but not exported"
+    assert set(names) == set(pf.EXPORTED)
+
+
+def test_descriptor_validation(pf):
+    ok = pf.layer_desc(S.spec_c3_layer(64))
+    assert pf.proxy_layer_check(ok) == pf.PF_OK
+    bad = pf.layer_desc(S.LayerSpec(batch=1, L=64, d=96, n_heads=1, P=4))
+    assert pf.proxy_layer_check(bad) == pf.PF_ERR_INVALID_ARG
+    bad = pf.layer_desc(S.LayerSpec(batch=1, L=64, d=128, n_heads=4, P=4))
+    assert pf.proxy_layer_check(bad) == pf.PF_ERR_UNSUPPORTED  # head width 32
+    bad = pf.layer_desc(S.LayerSpec(batch=1, L=64, d=128, n_heads=2, P=6, levels=2, k1=4, k2=2))
+    assert pf.proxy_layer_check(bad) == pf.PF_ERR_INVALID_ARG
+    assert "k1 * k2" in pf.pf_last_error()
+    bad = pf.layer_desc(S.LayerSpec(batch=0, L=64, d=128, n_heads=2, P=4))
+    assert pf.proxy_layer_check(bad) == pf.PF_ERR_INVALID_ARG
+
+
+def test_sizes_scale_with_shape(pf):
+    a = pf.layer_desc(S.LayerSpec(batch=1, L=4096, d=128, n_heads=2, P=16))
+    b = pf.layer_desc(S.LayerSpec(batch=2, L=4096, d=128, n_heads=2, P=16))
+    for f in (pf.proxy_layer_saved_size,
+              lambda d: pf.proxy_layer_workspace_size(d, 1)):
+        sa, sb = f(a), f(b)
+        assert 0 < sa < sb
+    # the saved buffer holds at least the decompressed update (bf16, L*d)
+    assert pf.proxy_layer_saved_size(a) >= 4096 * 128 * 2
+    # headline layer: saved ~ D (512 MiB) + Y + Z + proxy tensors
+    big = pf.layer_desc(S.spec_c3_layer(64))
+    assert 512 << 20 < pf.proxy_layer_saved_size(big) < 1 << 30
+
+
+def test_calls_reject_bad_arguments_before_any_launch(pf):
+    spec = S.LayerSpec(batch=1, L=256, d=128, n_heads=2, P=16)
+    desc = pf.layer_desc(spec)
+    prm = pf.layer_params({})
+    with pytest.raises(pf.ProxyFormerError) as e:
+        pf.proxy_layer_fwd(desc, prm, 16, None, None, 32, None, None, None, 0)
+    assert e.value.status == pf.PF_ERR_INVALID_ARG
+    full = pf.layer_params({k: 4096 for k in ("W_c1", "b_c1", "W_qkv", "W_o", "W_d1", "b_d1",
+                                              "w_x", "w_dlt", "b_g")})
+    with pytest.raises(pf.ProxyFormerError) as e:  # misaligned X
+        pf.proxy_layer_fwd(desc, full, 8, None, None, 4096, None, None, 4096, 1 << 30)
+    assert e.value.status == pf.PF_ERR_INVALID_ARG
+    with pytest.raises(pf.ProxyFormerError) as e:  # workspace too small
+        pf.proxy_layer_fwd(desc, full, 4096, None, None, 8192, None, None, 4096, 16)
+    assert e.value.status == pf.PF_ERR_WORKSPACE
+    with pytest.raises(pf.ProxyFormerError) as e:  # X_out aliases X
+        pf.proxy_layer_fwd(desc, full, 4096, None, None, 4096, None, None, 4096, 1 << 30)
+    assert e.value.status == pf.PF_ERR_INVALID_ARG
+    with pytest.raises(pf.ProxyFormerError) as e:
+        pf.pf_gemm_bf16(128, 100, 64, 4096, 0, 4096, 0, 4096, 100)
+    assert e.value.status == pf.PF_ERR_INVALID_ARG
