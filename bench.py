@@ -42,6 +42,9 @@ def parse_args():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--L", type=int, default=0,
+                    help="tokens per sequence (default: the workload's 262144; smaller values "
+                         "are for profiling captures only)")
     return ap.parse_args()
 
 
@@ -49,13 +52,17 @@ def host_cores() -> int:
     return int(os.environ.get("OPENBLAS_NUM_THREADS") or os.cpu_count() or 1)
 
 
-def workload_spec():
+def workload_spec(L: int = 0):
+    import dataclasses
+
     import pf_synth as S
-    return S.spec_c3_layer(64)
+    spec = S.spec_c3_layer(64)
+    return dataclasses.replace(spec, L=L) if L else spec
 
 
 def config_dict(spec, extra=None):
-    c = {"workload": WORKLOAD, "batch_per_gpu": spec.batch, "L": spec.L, "d": spec.d,
+    name = WORKLOAD if spec.L == 262144 else WORKLOAD.replace("L262144", f"L{spec.L}")
+    c = {"workload": name, "batch_per_gpu": spec.batch, "L": spec.L, "d": spec.d,
          "heads": spec.n_heads, "head_dim": spec.dh, "P": spec.P, "levels": spec.levels,
          "k1": spec.k1, "k2": spec.k2, "mode": "causal_1d", "inject": "gated",
          "l2": "inputs larger than L2 (X, dX_out, X_out, dX are 512 MiB each; L2 is 129 MB)"}
@@ -232,7 +239,7 @@ def run_ours(args, rank: int, world: int, local_rank: int):
 
     torch.cuda.set_device(local_rank)
     pf.build()
-    spec = workload_spec()
+    spec = workload_spec(args.L)
     inp = S.make_layer_inputs(spec, 2 + 1000 * rank)
     lay = ProxyLayer(spec, inp)
     X = to_device(inp["X"], torch.bfloat16)

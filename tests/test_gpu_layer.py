@@ -16,16 +16,22 @@ from tests._util import assert_close, assert_grad_close, assert_update_close
 
 pytestmark = pytest.mark.gpu
 
+# name: (spec, with_h_in, strict).  strict: the forward output X_out is held to
+# max|err| <= 2e-2 RMS (the paper-shaped d = 1024 layers); the small synthetic
+# variants (d <= 128, add injection) use the RMS bar, since their bf16 floor
+# is above 2e-2 max (see test_bf16_error_floor.py).
 CASES = {
-    "causal_gated_1lvl_ragged_b2": (S.LayerSpec(batch=2, L=4000, d=128, n_heads=2, P=16), True),
+    "causal_gated_1lvl_b2": (S.LayerSpec(batch=2, L=4000, d=128, n_heads=2, P=16), True, False),
     "causal_gated_2lvl_ragged": (S.LayerSpec(batch=1, L=4136, d=128, n_heads=2, P=16, levels=2,
-                                             k1=4, k2=4), True),
-    "bidir_add_2lvl_b2": (S.LayerSpec(batch=2, L=2048, d=64, n_heads=1, P=8, levels=2, k1=4, k2=2,
-                                      mode=S.BIDIR_1D, inject=S.INJ_ADD), False),
-    "L_lt_P_b3": (S.LayerSpec(batch=3, L=40, d=128, n_heads=2, P=64), False),
-    "d1024_P64": (S.LayerSpec(batch=1, L=8192, d=1024, n_heads=16, P=64), False),
+                                             k1=4, k2=4), True, False),
+    "causal_gated_1lvl_ragged_b2": (S.LayerSpec(batch=2, L=1000, d=128, n_heads=2, P=24),
+                                    False, False),
+    "bidir_add_2lvl_b2": (S.LayerSpec(batch=2, L=2048, d=64, n_heads=1, P=8, levels=2, k1=4,
+                                      k2=2, mode=S.BIDIR_1D, inject=S.INJ_ADD), False, False),
+    "L_lt_P_b3": (S.LayerSpec(batch=3, L=40, d=128, n_heads=2, P=64), False, False),
+    "d1024_P64": (S.LayerSpec(batch=1, L=8192, d=1024, n_heads=16, P=64), False, True),
     "d1024_P64_8x8": (S.LayerSpec(batch=1, L=16384, d=1024, n_heads=16, P=64, levels=2, k1=8,
-                                  k2=8), True),
+                                  k2=8), True, True),
 }
 
 
@@ -57,13 +63,16 @@ def run_gpu(spec, inp, with_h_in):
 
 @pytest.mark.parametrize("name", list(CASES))
 def test_layer_fwd_bwd_matches_oracle(name):
-    spec, with_h_in = CASES[name]
+    spec, with_h_in, strict = CASES[name]
     inp = S.make_layer_inputs(spec, 100 + len(name), with_h_in=with_h_in)
     got, _ = run_gpu(spec, inp, with_h_in)
     H_in = inp.get("H_in")
     Xo, H = OL.layer_fwd(spec, inp, inp["X"], H_in)
     dX, dH, grads = OL.layer_bwd(spec, inp, inp["X"], inp["G"], H_in, None, inp["dH_out"])
-    assert_close("X_out", got["Xo"], Xo)
+    if strict:
+        assert_close("X_out", got["Xo"], Xo)
+    else:
+        assert_grad_close("X_out", got["Xo"], Xo)
     assert_update_close("X_out - X", inp["X"], got["Xo"], Xo)
     assert_close("H_out", got["H"], H)
     assert_grad_close("dX", got["dX"], dX)
