@@ -197,26 +197,38 @@ def gpu_smi_id(torch, dev: int) -> str:
 
 
 # ------------------------------------------------------------------ our leg
-def source_hash() -> str:
+def kernel_files(label: str):
+    """Source files that define the kernel behind a timing label."""
+    if label.startswith("attn_"):
+        return ["attention.cu", "common.cuh"]
+    if label.startswith(("inj_bwd", "colsum", "copy_block0", "pad_rows")):
+        return ["elementwise.cu", "common.cuh"]
+    return ["gemm_tc.cuh", "gemm.cu", "common.cuh"]
+
+
+def source_hash(label: str) -> str:
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2608_23463_gb300", "csrc")
-    for f in sorted(os.listdir(csrc)):
+    for f in kernel_files(label):
         with open(os.path.join(csrc, f), "rb") as fh:
             h.update(f.encode() + fh.read())
     return h.hexdigest()[:16]
 
 
-def traffic_from_profile(label: str):
-    """dram bytes per launch of `label` from profiles/traffic.txt (lines:
-    label bytes_per_launch source_hash), or None when absent or stale."""
+def traffic_from_profile(label: str, units: float):
+    """DRAM bytes per launch of `label` from profiles/traffic.txt, whose lines
+    read: label dram_bytes_per_launch units_captured kernel_source_hash.  The
+    captured bytes are scaled to this launch by units (tokens); None when the
+    kernel has no capture or its source changed since."""
     path = os.path.join(ROOT, "profiles", "traffic.txt")
     if not os.path.exists(path):
         return None
-    cur = source_hash()
     for line in open(path):
         parts = line.split()
-        if len(parts) >= 3 and not line.startswith("#") and parts[0] == label:
-            return float(parts[1]) if parts[2] == cur else None
+        if len(parts) >= 4 and not line.startswith("#") and parts[0] == label:
+            if parts[3] != source_hash(label):
+                return None
+            return float(parts[1]) * units / float(parts[2])
     return None
 
 
@@ -333,16 +345,16 @@ def run_ours(args, rank: int, world: int, local_rank: int):
         achieved = dv["flops"] / avg_s / 1e12
         peak = peaks["bf16_tflops_sustained"]
         roof = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                "frac": achieved / peak, "traffic": traffic_from_profile(dom), "kernel": dom,
-                "launches": dv["launches"], "avg_us": avg_s * 1e6,
+                "frac": achieved / peak, "traffic": traffic_from_profile(dom, spec.batch * spec.L),
+                "kernel": dom, "launches": dv["launches"], "avg_us": avg_s * 1e6,
                 "flops_per_launch": dv["flops"],
                 "peak_source": f"{peak_src} bf16_tflops_sustained (kernel timed inside a long step)"}
     else:
         achieved = dv["bytes"] / avg_s / 1e9
         peak = peaks["hbm_gbs"]
         roof = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                "frac": achieved / peak, "traffic": traffic_from_profile(dom), "kernel": dom,
-                "launches": dv["launches"], "avg_us": avg_s * 1e6,
+                "frac": achieved / peak, "traffic": traffic_from_profile(dom, spec.batch * spec.L),
+                "kernel": dom, "launches": dv["launches"], "avg_us": avg_s * 1e6,
                 "bytes_per_launch": dv["bytes"], "peak_source": f"{peak_src} hbm_gbs"}
     step_flops = sum(v["flops"] * v["launches"] for v in timing.values()) / args.steps
     step_bytes = sum(v["bytes"] * v["launches"] for v in timing.values()) / args.steps

@@ -62,7 +62,7 @@ enum { PF_F32 = 0, PF_BF16 = 1 };
  *   grid_h, grid_w, patch : 2D only; P must equal patch*patch
  *   d, n_heads : d_fine = d_proxy = d (the paper's simplification, Sec. 4);
  *                head width d/n_heads must be 64
- *   P          : block size (compression ratio) of this layer (Sec. 3.7
+ *   P          : block size (compression ratio) of this layer (Sec. 3.6
  *                allows a different P per layer)
  *   levels     : 1 or 2 (Eq. factor with M = 2); levels == 2 needs k1*k2 == P,
  *                level 1 maps k1 tokens to one row, level 2 k2 rows to a proxy

@@ -14,8 +14,9 @@ Decode (Eq. llm-cross, Eq. llm-gate, Sec. 3.8), per sequence b and head h:
 Readings: RMSNorm has eps 1e-6 and a learnable weight; the alpha MLP's hidden
 width is d/8 (parity unpinned: the paper gives no width); no FFN.
 
-Append (Sec. 3.8 "when the new tokens ... reach the block size P"): the P
-open-block features are compressed exactly like a layer's block (Eq.
+Append (Sec. 3.8: once the generation region holds P new tokens, their block
+is compressed and appended to the cache): the P open-block features are
+compressed exactly like a layer's block (Eq.
 compress-linear / Eq. factor-cascade), H = H_in + c (Eq. proxy-res), and the
 proxy's key and value rows W_kh H, W_vh H are written at cache row n_p;
 n_p += 1, n_o = 0.

@@ -46,7 +46,7 @@ def sigmoid(x):
 
 # ---------------------------------------------------------------- partition
 def partition(X, spec):
-    """Eq. partition (Sec. 3.2 "Partitioning"): split one sequence X [L, d]
+    """Eq. partition (Sec. 3.2, partitioning): split one sequence X [L, d]
     into m = ceil(L/P) blocks X_i [P, d].  1D: contiguous non-overlapping
     blocks, the last zero-padded.  2D: p x p spatial patches of the
     grid_h x grid_w raster, patches in raster order, tokens inside a patch in

@@ -251,7 +251,7 @@ def test_p6_factorised_equals_single_level():
 
 # ----------------------------------------------------------------- P7
 def test_p7_2d_compression_is_conv_and_decompression_is_conv_transpose():
-    """Sec. 3.2/3.6: 2D patch compression is conv2d with kernel = stride = p,
+    """Sec. 3.2/3.5: 2D patch compression is conv2d with kernel = stride = p,
     and the affine decompression is the matching conv_transpose2d."""
     spec = S.LayerSpec(batch=1, L=36, d=4, n_heads=2, P=4, mode=S.BIDIR_2D,
                        inject=S.INJ_AFFINE, grid_h=6, grid_w=6, patch=2, dtype=S.F32)
