@@ -231,6 +231,34 @@ pf_status pf_gemm_bf16(int M, int N, int K, const void *A, int a_mn, const void 
                        int b_mn, float *D, int ldd, void *stream);
 
 /* ---------------------------------------------------------------------------
+ * Allocation-free backward.  The paper has no counterpart; this is a calling
+ * convenience of the library.  Some callers cannot provide a workspace: code
+ * running while a stream is captured in a mode that forbids cudaMalloc, host
+ * frameworks whose memory planner owns all device memory, and latency-critical
+ * loops that cannot pay cudaMalloc's implicit device synchronisation.  This
+ * entry point computes exactly what proxy_layer_bwd computes, with its scratch
+ * taken from a fixed device array of PF_NOALLOC_SCRATCH_BYTES inside the
+ * library instead of a caller buffer; it calls no allocator.  The caller still
+ * passes every input and output.
+ *   - Layers whose backward needs more scratch than PF_NOALLOC_SCRATCH_BYTES
+ *     (proxy_layer_workspace_size(desc, 1)) are rejected with
+ *     PF_ERR_WORKSPACE before anything is launched.
+ *   - The array exists once per GPU that loads the library and stays
+ *     allocated until the process exits.
+ *   - The first call on a device looks up the array's device address (with
+ *     that device current); make that first call before any stream capture.
+ *   - All calls share the one array and the backward writes every scratch
+ *     byte before reading it (nothing needs to start at zero); calls whose
+ *     execution overlaps on the GPU (other streams, concurrent graphs) race
+ *     on the array and must be serialised by the caller.                    */
+#define PF_NOALLOC_SCRATCH_BYTES (16u << 20)
+pf_status proxy_layer_bwd_noalloc(const pf_layer_desc *desc, const pf_layer_params *params,
+                                  const void *X, const float *H_in, const float *t,
+                                  const void *saved, const void *dX_out, const float *dH_out,
+                                  void *dX, float *dH_in, const pf_layer_grads *grads,
+                                  void *stream);
+
+/* ---------------------------------------------------------------------------
  * Launch timing (a measurement utility, not a paper operation).  While enabled,
  * every kernel the library launches is bracketed by two CUDA events recorded
  * on the stream it is launched on, tagged with a label naming the step of the

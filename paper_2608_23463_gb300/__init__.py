@@ -72,7 +72,7 @@ EXPORTED = ("proxy_layer_check", "proxy_layer_saved_size", "proxy_layer_workspac
             "proxy_decode_step", "proxy_append_workspace_size", "proxy_kv_append",
             "pf_last_error", "pf_sync_check", "pf_gemm_bf16", "pf_timing_enable",
             "pf_timing_collect", "pf_timing_label", "pf_timing_ms", "pf_timing_launches",
-            "pf_timing_flops", "pf_timing_bytes")
+            "pf_timing_flops", "pf_timing_bytes", "proxy_layer_bwd_noalloc")
 
 _lib: Optional[ctypes.CDLL] = None
 
@@ -125,6 +125,9 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     for n in ("pf_timing_ms", "pf_timing_flops", "pf_timing_bytes"):
         getattr(lib, n).argtypes = [ctypes.c_int]
         getattr(lib, n).restype = ctypes.c_double
+    lib.proxy_layer_bwd_noalloc.argtypes = [P(LayerDesc), P(LayerParams), _vp, _vp, _vp, _vp, _vp,
+                                            _vp, _vp, _vp, P(LayerGrads), _vp]
+    lib.proxy_layer_bwd_noalloc.restype = ctypes.c_int
     lib.pf_timing_launches.argtypes = [ctypes.c_int]
     lib.pf_timing_launches.restype = ctypes.c_int
     _lib = lib
@@ -179,6 +182,19 @@ def proxy_layer_bwd(desc, params, X, H_in, t, saved, dX_out, dH_out, dX, dH_in, 
                                   _ptr(t), _ptr(saved), _ptr(dX_out), _ptr(dH_out), _ptr(dX),
                                   _ptr(dH_in), ctypes.byref(grads), _ptr(ws), int(ws_bytes),
                                   stream))
+
+
+def proxy_layer_bwd_noalloc(desc, params, X, H_in, t, saved, dX_out, dH_out, dX, dH_in, grads,
+                            stream=None):
+    """proxy_layer_bwd for callers that cannot provide a workspace: scratch comes
+    from a fixed device array inside the library (PF_NOALLOC_SCRATCH_BYTES)."""
+    _check(load().proxy_layer_bwd_noalloc(ctypes.byref(desc), ctypes.byref(params), _ptr(X),
+                                          _ptr(H_in), _ptr(t), _ptr(saved), _ptr(dX_out),
+                                          _ptr(dH_out), _ptr(dX), _ptr(dH_in), ctypes.byref(grads),
+                                          stream))
+
+
+PF_NOALLOC_SCRATCH_BYTES = 16 << 20
 
 
 def proxy_decode_workspace_size(desc: DecodeDesc) -> int:

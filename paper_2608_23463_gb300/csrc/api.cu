@@ -152,6 +152,13 @@ pf_status check_desc(const pf_layer_desc* s) {
 
 }  // namespace
 
+// Sets the thread-local message returned by pf_last_error (for other files of
+// the library) and returns `s`.
+__attribute__((visibility("hidden"))) pf_status pf_set_error(pf_status s, const char* msg) {
+  g_msg = msg;
+  return s;
+}
+
 extern "C" {
 
 const char* pf_last_error(void) { return g_msg.c_str(); }
