@@ -92,7 +92,7 @@ Saved carve_saved(Carve& c, const pf_layer_desc& s, const Dims& g) {
 }
 
 struct BwdWs {
-  bf16 *Xpad, *dD, *dZ, *dHbar, *dA, *dQKV, *dHb, *dY;
+  bf16 *Xpad, *dXpad, *dD, *dZ, *dHbar, *dA, *dQKV, *dHb, *dY;
   float *Di, *dHf, *part;
   long part_elems;
 };
@@ -100,6 +100,7 @@ struct BwdWs {
 BwdWs carve_bwd(Carve& c, const pf_layer_desc& s, const Dims& g) {
   BwdWs w{};
   w.Xpad = g.ragged ? c.take<bf16>(g.B * g.Lp * g.d) : nullptr;
+  w.dXpad = g.ragged ? c.take<bf16>(g.B * g.Lp * g.d) : nullptr;
   w.dD = c.take<bf16>(g.rows1 * g.N1);
   if (s.levels == 2) w.dZ = c.take<bf16>(g.R * g.k2 * g.d);
   w.dHbar = c.take<bf16>(g.R * g.d);
@@ -119,6 +120,14 @@ BwdWs carve_bwd(Carve& c, const pf_layer_desc& s, const Dims& g) {
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+bool params_aligned(const pf_layer_params& p) {
+  const void* ptrs[] = {p.W_c1, p.b_c1, p.W_c2, p.b_c2, p.W_qkv, p.W_o,  p.W_d2,  p.b_d2, p.W_d1,
+                        p.b_d1, p.w_x,  p.w_dlt, p.b_g, p.W_t1,  p.b_t1, p.W_t2, p.b_t2};
+  for (const void* q : ptrs)
+    if (!aligned16(q)) return false;
+  return true;
+}
 
 pf_status check_desc(const pf_layer_desc* s) {
   if (s == nullptr) return fail(PF_ERR_INVALID_ARG, "descriptor is NULL");
@@ -201,7 +210,7 @@ pf_status proxy_layer_fwd(const pf_layer_desc* desc, const pf_layer_params* prm,
       (s.inject == PF_INJ_GATED && (!prm->w_x || !prm->w_dlt || !prm->b_g)))
     return fail(PF_ERR_INVALID_ARG, "a parameter this layer uses is NULL");
   if (!aligned16(X) || !aligned16(X_out) || !aligned16(saved) || !aligned16(ws) ||
-      !aligned16(H_in) || !aligned16(H_out))
+      !aligned16(H_in) || !aligned16(H_out) || !params_aligned(*prm))
     return fail(PF_ERR_INVALID_ARG, "buffers must be 16-byte aligned");
   Carve wc(ws);
   bf16* Xpad = g.ragged ? wc.take<bf16>(g.B * g.Lp * g.d) : nullptr;
@@ -285,7 +294,7 @@ pf_status proxy_layer_fwd(const pf_layer_desc* desc, const pf_layer_params* prm,
     Zsrc = sv.Z;
   }
   {
-    EpiInjectArgs e{prm->b_d1, sv.D, Xb, Xo,
+    EpiInjectArgs e{prm->b_d1, sv.D, Xsrc, Xo,
                     prm->w_x, prm->w_dlt, prm->b_g,
                     d, (int)g.k1, (int)g.k2, (int)g.m, (int)g.L, g.causal ? 1 : 0,
                     s.inject == PF_INJ_GATED ? 1 : 0};
@@ -293,7 +302,7 @@ pf_status proxy_layer_fwd(const pf_layer_desc* desc, const pf_layer_params* prm,
     PF_CUDA(gemm_inject1d((int)g.rows1, (int)g.N1, d, {Zsrc, d, 0},
                           {static_cast<const bf16*>(prm->W_d1), d, 0}, e, cs));
   }
-  if (g.causal) PF_CUDA(copy_block0(Xb, Xo, (int)g.B, g.L, d, (int)std::min(g.P, g.L), cs));
+  if (g.causal) PF_CUDA(copy_block0(Xb, g.L, Xo, g.L, (int)g.B, d, (int)std::min(g.P, g.L), cs));
   return PF_OK;
 }
 
@@ -310,7 +319,7 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
   if (!prm || !X || !saved || !dX_out || !dX || !grads)
     return fail(PF_ERR_INVALID_ARG, "params, X, saved, dX_out, dX and grads are required");
   if (!aligned16(X) || !aligned16(saved) || !aligned16(dX_out) || !aligned16(dX) ||
-      !aligned16(ws) || !aligned16(dH_out) || !aligned16(dH_in))
+      !aligned16(ws) || !aligned16(dH_out) || !aligned16(dH_in) || !params_aligned(*prm))
     return fail(PF_ERR_INVALID_ARG, "buffers must be 16-byte aligned");
   const bool gated = s.inject == PF_INJ_GATED;
   if (!grads->b_d1 || (gated && (!grads->w_x || !grads->w_dlt || !grads->b_g)))
@@ -338,14 +347,19 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
     PF_CUDA(pad_rows(Xb, w.Xpad, (int)g.B, g.L, g.Lp, d, cs));
     Xsrc = w.Xpad;
   }
+  // direct injection gradient: written into dX, or into a block-padded buffer
+  // when L % P != 0 so the dX GEMM epilogue can prefetch it as whole tiles
+  bf16* dXd = g.ragged ? w.dXpad : dXb;
   // injection backward: dD (proxy order), direct dX, gate and b_d1 gradients
   {
     const int nch = inj_bwd_chunks(g.rows1, N1);
-    InjBwdArgs a{G, Xb, sv.D, w.dD, dXb, prm->w_x, prm->w_dlt, prm->b_g,
+    InjBwdArgs a{G, Xb, sv.D, w.dD, dXd, g.ragged ? g.Lp : g.L, prm->w_x, prm->w_dlt, prm->b_g,
                  d, (int)g.k1, (int)g.k2, (int)g.m, (int)g.L, (int)g.B, g.causal ? 1 : 0,
                  gated ? 1 : 0};
     PF_CUDA(inj_bwd_1d(a, w.part, nch, cs));
-    if (g.causal) PF_CUDA(copy_block0(G, dXb, (int)g.B, g.L, d, (int)std::min(g.P, g.L), cs));
+    if (g.causal)
+      PF_CUDA(copy_block0(G, g.L, dXd, g.ragged ? g.Lp : g.L, (int)g.B, d,
+                          (int)std::min(g.P, g.L), cs));
     PF_CUDA(inj_bwd_finalize(w.part, nch, N1, d, grads->b_d1, gated ? grads->w_x : nullptr,
                              gated ? grads->w_dlt : nullptr, gated ? grads->b_g : nullptr, cs));
   }
@@ -447,7 +461,7 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
     PF_CUDA(gemm_linear(d, N1, (int)g.rows1, {dYsrc, d, 1}, {Xsrc, N1, 1}, e, cs));
   }
   {
-    EpiDXArgs e{dXb, d, (int)g.k1, (int)g.k2, (int)g.m, (int)g.L};
+    EpiDXArgs e{dXd, dXb, d, (int)g.k1, (int)g.k2, (int)g.m, (int)g.L};
     set_gemm_tag("bwd_dX", (double)g.rows1 * N1 * 4.0);
     PF_CUDA(gemm_dx1d((int)g.rows1, N1, d, {dYsrc, d, 0}, {W_c1, N1, 1}, e, cs));
   }

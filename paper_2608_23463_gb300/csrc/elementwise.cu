@@ -9,13 +9,13 @@ namespace {
 
 constexpr int EW_THREADS = 256;
 
-__global__ void copy_block0_kernel(const bf16* __restrict__ src, bf16* __restrict__ dst, long L,
-                                   int d, long per_seq_vec) {
+__global__ void copy_block0_kernel(const bf16* __restrict__ src, long Ls, bf16* __restrict__ dst,
+                                   long Ld, int d, long per_seq_vec) {
   const long i = (long)blockIdx.x * blockDim.x + threadIdx.x;
   const int b = blockIdx.y;
   if (i >= per_seq_vec) return;
-  const long off = (long)b * L * d + i * 8;
-  *reinterpret_cast<uint4*>(dst + off) = *reinterpret_cast<const uint4*>(src + off);
+  *reinterpret_cast<uint4*>(dst + (long)b * Ld * d + i * 8) =
+      *reinterpret_cast<const uint4*>(src + (long)b * Ls * d + i * 8);
 }
 
 __global__ void pad_rows_kernel(const bf16* __restrict__ src, bf16* __restrict__ dst, long L,
@@ -78,7 +78,7 @@ __global__ void __launch_bounds__(EW_THREADS) inj_bwd_kernel(InjBwdArgs a, float
           dd[j] = g[j];
         }
       }
-      store8_bf16(a.dX + off, dx);
+      store8_bf16(a.dX + ((long)b * a.Ldx + tok) * a.d + ch, dx);
     } else {
 #pragma unroll
       for (int j = 0; j < 8; ++j) dd[j] = 0.f;
@@ -184,12 +184,12 @@ cudaError_t colsum_impl(const T* X, long R, int C, float* out, float* part, cuda
 
 }  // namespace
 
-cudaError_t copy_block0(const bf16* src, bf16* dst, int B, long L, int d, int rows,
+cudaError_t copy_block0(const bf16* src, long Ls, bf16* dst, long Ld, int B, int d, int rows,
                         cudaStream_t st) {
   const long nvec = (long)rows * d / 8;
   dim3 grid((unsigned)((nvec + 255) / 256), B);
   LaunchTimer lt("copy_block0", st, 0.0, 32.0 * nvec * B);
-  copy_block0_kernel<<<grid, 256, 0, st>>>(src, dst, L, d, nvec);
+  copy_block0_kernel<<<grid, 256, 0, st>>>(src, Ls, dst, Ld, d, nvec);
   return cudaGetLastError();
 }
 

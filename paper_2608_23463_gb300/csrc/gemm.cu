@@ -2,6 +2,8 @@
 // instantiations used by the layer (see gemm_tc.cuh for the kernel).
 #include <cudaTypedefs.h>
 
+#include <algorithm>
+
 #include "gemm_tc.cuh"
 #include "kernels.h"
 
@@ -57,25 +59,26 @@ bool make_operand_map(CUtensorMap* m, const Operand& op, int rows, int K) {
 }
 
 template <int BN, bool AMN, bool BMN, class Epi>
-cudaError_t launch(int M, int N, int K, const CUtensorMap& ta, const CUtensorMap& tb, const Epi& epi,
-                   cudaStream_t st) {
-  auto kern = gemm_tc_kernel<BN, AMN, BMN, Epi, BRowsLinear>;
-  constexpr int smem = GemmCfg<BN>::SMEM_BYTES;
+cudaError_t launch(int M, int N, int K, const CUtensorMap& ta, const CUtensorMap& tb,
+                   const CUtensorMap& tx, const Epi& epi, cudaStream_t st) {
+  auto kern = gemm_tc_kernel<BN, AMN, BMN, Epi>;
+  constexpr int smem = GemmCfg<BN, Epi::kXTile>::SMEM_BYTES;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  dim3 grid((N + BN - 1) / BN, (M + GEMM_BM - 1) / GEMM_BM);
-  kern<<<grid, GEMM_THREADS, smem, st>>>(ta, tb, M, N, K, epi, BRowsLinear{});
+  const long tiles = (long)((N + BN - 1) / BN) * ((M + GEMM_BM - 1) / GEMM_BM);
+  const int grid = (int)std::min<long>(tiles, num_sms());
+  kern<<<grid, GEMM_THREADS, smem, st>>>(ta, tb, tx, M, N, K, epi);
   return cudaGetLastError();
 }
 
 template <int BN, class Epi>
 cudaError_t launch_majors(int M, int N, int K, const Operand& A, const Operand& B,
-                          const CUtensorMap& ta, const CUtensorMap& tb, const Epi& epi,
-                          cudaStream_t st) {
-  if (!A.mn && !B.mn) return launch<BN, false, false>(M, N, K, ta, tb, epi, st);
-  if (!A.mn && B.mn) return launch<BN, false, true>(M, N, K, ta, tb, epi, st);
-  if (A.mn && B.mn) return launch<BN, true, true>(M, N, K, ta, tb, epi, st);
-  return launch<BN, true, false>(M, N, K, ta, tb, epi, st);
+                          const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tx,
+                          const Epi& epi, cudaStream_t st) {
+  if (!A.mn && !B.mn) return launch<BN, false, false>(M, N, K, ta, tb, tx, epi, st);
+  if (!A.mn && B.mn) return launch<BN, false, true>(M, N, K, ta, tb, tx, epi, st);
+  if (A.mn && B.mn) return launch<BN, true, true>(M, N, K, ta, tb, tx, epi, st);
+  return launch<BN, true, false>(M, N, K, ta, tb, tx, epi, st);
 }
 
 bool operand_ok(const Operand& op) {
@@ -83,19 +86,29 @@ bool operand_ok(const Operand& op) {
          (op.ld * 2) % 16 == 0;
 }
 
+// X tile source (kXTile epilogues): the [rows, N] bf16 view the epilogue
+// prefetches by TMA; for other epilogues `xsrc` is ignored.
 template <class Epi>
 cudaError_t gemm_dispatch(int M, int N, int K, Operand A, Operand B, const Epi& epi,
-                          cudaStream_t st) {
+                          const bf16* xsrc, long x_rows, cudaStream_t st) {
   if (M <= 0 || N <= 0 || N % 32 != 0 || K < 0 || !operand_ok(A) || !operand_ok(B))
     return cudaErrorInvalidValue;
-  CUtensorMap ta, tb;
+  CUtensorMap ta, tb, tx;
   if (!make_operand_map(&ta, A, M, K) || !make_operand_map(&tb, B, N, K))
     return cudaErrorInvalidValue;
+  if (Epi::kXTile) {
+    if (xsrc == nullptr || (reinterpret_cast<uintptr_t>(xsrc) & 15) != 0 ||
+        !make_map(&tx, xsrc, (uint64_t)N, (uint64_t)x_rows, (uint64_t)N, 64, 128))
+      return cudaErrorInvalidValue;
+  } else {
+    tx = ta;
+  }
   const long tiles256 = (long)((N + 255) / 256) * ((M + GEMM_BM - 1) / GEMM_BM);
   LaunchTimer lt(gemm_tag_label(), st, 2.0 * M * N * (double)K,
                  2.0 * ((double)M * K + (double)N * K) + gemm_tag_bytes());
-  if (N >= 256 && tiles256 >= num_sms()) return launch_majors<256>(M, N, K, A, B, ta, tb, epi, st);
-  return launch_majors<128>(M, N, K, A, B, ta, tb, epi, st);
+  if (N >= 256 && tiles256 >= num_sms())
+    return launch_majors<256>(M, N, K, A, B, ta, tb, tx, epi, st);
+  return launch_majors<128>(M, N, K, A, B, ta, tb, tx, epi, st);
 }
 
 }  // namespace
@@ -103,22 +116,22 @@ cudaError_t gemm_dispatch(int M, int N, int K, Operand A, Operand B, const Epi& 
 cudaError_t gemm_linear(int M, int N, int K, Operand A, Operand B, const EpiLinearArgs& e,
                         cudaStream_t st) {
   EpiLinear epi{M, N, e.bias, e.addend, e.ld_add, e.out_f32, e.ld_f32, e.out_bf16, e.ld_bf16};
-  return gemm_dispatch(M, N, K, A, B, epi, st);
+  return gemm_dispatch(M, N, K, A, B, epi, nullptr, 0, st);
 }
 
 cudaError_t gemm_inject1d(int M, int N, int K, Operand A, Operand B, const EpiInjectArgs& e,
                           cudaStream_t st) {
-  EpiInject1D epi{M, N, e.bias, e.D_save, e.X, e.X_out, e.w_x, e.w_dlt, e.b_g,
+  EpiInject1D epi{M, N, e.bias, e.D_save, e.X_out, e.w_x, e.w_dlt, e.b_g,
                   e.d, e.k1, e.k2, e.m, e.L, e.shift, e.gated};
   if (A.mn || B.mn) return cudaErrorInvalidValue;
-  return gemm_dispatch(M, N, K, A, B, epi, st);
+  return gemm_dispatch(M, N, K, A, B, epi, e.Xsrc, M, st);
 }
 
 cudaError_t gemm_dx1d(int M, int N, int K, Operand A, Operand B, const EpiDXArgs& e,
                       cudaStream_t st) {
   EpiDX1D epi{M, N, e.dX, e.d, e.k1, e.k2, e.m, e.L};
   if (A.mn || !B.mn) return cudaErrorInvalidValue;
-  return gemm_dispatch(M, N, K, A, B, epi, st);
+  return gemm_dispatch(M, N, K, A, B, epi, e.dXd, M, st);
 }
 
 }  // namespace pf

@@ -6,14 +6,21 @@
 // or [K, N]).  Every contraction of the layer (compression, proxy Q/K/V/O,
 // decompression, and all of their weight / input gradients) is one of these.
 //
-// One CTA computes one 128 x BN output tile:
-//   warp 0   : TMA producer (one elected thread), STAGES-deep smem ring of
-//              128B-swizzled 64-wide K slices of A and B
-//   warp 1   : TMEM allocator + MMA issuer (one thread issues tcgen05.mma
-//              M=128, N=BN, K=16; tcgen05.commit frees smem stages)
-//   warps 2-5: epilogue: tcgen05.ld 32 columns at a time from the TMEM
-//              accumulator (warp w reads TMEM lanes 32*(w%4)..), applies the
-//              fused epilogue functor and writes global memory.
+// Persistent: one CTA per SM walks the 128 x BN output tiles tile = blockIdx.x
+// + k * gridDim.x (N fastest, so co-running CTAs share A panels and all of B
+// in L2).  Roles:
+//   warp 0   : TMA producer (one thread): STAGES-deep ring of 128B-swizzled
+//              64-wide K slices of A and B, continuing across tiles
+//   warp 1   : TMEM allocator + MMA issuer (one thread): tcgen05.mma M=128,
+//              N=BN, K=16 into one of two TMEM accumulators (2*BN columns),
+//              tcgen05.commit frees smem stages and hands a finished
+//              accumulator to the epilogue
+//   warps 2-5: epilogue: tcgen05.ld 32 columns at a time (warp w reads TMEM
+//              lanes 32*(w%4)..), fused epilogue functor, global stores.
+//              While they drain accumulator i, the MMA warp fills the other.
+// Epilogues that read a bf16 tile shaped like the output (the local stream X
+// for injection, the direct gradient for dX) have it prefetched by TMA into
+// shared memory (128 x BN, 128B-swizzled) while the tile's mainloop runs.
 // Every mbarrier wait is bounded (common.cuh); on a timeout the kernel flags
 // the error, drains its own copies and MMAs (bounded), frees TMEM and returns.
 #pragma once
@@ -26,157 +33,235 @@ constexpr int GEMM_BM = 128;
 constexpr int GEMM_BK = 64;
 constexpr int GEMM_THREADS = 192;
 
-template <int BN>
+template <int BN, bool XTILE>
 struct GemmCfg {
-  static constexpr int STAGES = (BN == 256) ? 4 : 6;
+  static constexpr int STAGES = XTILE ? (BN == 256 ? 3 : 5) : (BN == 256 ? 4 : 6);
   static constexpr uint32_t A_BYTES = GEMM_BM * GEMM_BK * 2;  // 16 KB
   static constexpr uint32_t B_BYTES = BN * GEMM_BK * 2;       // 16/32 KB
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr uint32_t SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*bars*/;
+  static constexpr uint32_t X_BYTES = XTILE ? GEMM_BM * BN * 2 : 0;
+  static constexpr uint32_t SMEM_BYTES =
+      STAGES * STAGE_BYTES + X_BYTES + 1024 /*align*/ + 256 /*barriers*/;
 };
 
-// Optional remap of the B tile's rows (K-major B only): B tile `n_tile` is
-// loaded as BN/128 boxes of 128 rows; box j starts at row brow(n_tile, j).
-struct BRowsLinear {
-  __device__ __forceinline__ int operator()(int n_tile, int j, int BN) const {
-    return n_tile * BN + j * 128;
-  }
-};
+// Barrier of the 128 epilogue threads (named barrier 1) that also ANDs a
+// predicate across them, so that every epilogue thread takes the same branch.
+__device__ __forceinline__ bool epi_bar_and(bool p) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred pi, po;\n\t"
+      "setp.ne.u32 pi, %1, 0;\n\t"
+      "bar.red.and.pred po, 1, 128, pi;\n\t"
+      "selp.u32 %0, 1, 0, po;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)p)
+      : "memory");
+  return r != 0;
+}
 
-template <int BN, bool A_MN, bool B_MN, class Epi, class BRows = BRowsLinear>
+// 8 bf16 of row r, columns [c, c+8) of a 128 x BN tile stored as BN/64 boxes
+// of 128 rows x 64 columns with 128-byte swizzle (TMA SWIZZLE_128B layout).
+__device__ __forceinline__ void xtile_load8(const uint8_t* xt, int r, int c, float* v) {
+  const uint8_t* p = xt + (c >> 6) * 16384 + r * 128 + ((((c & 63) >> 3) ^ (r & 7)) << 4);
+  uint4 u = *reinterpret_cast<const uint4*>(p);
+  float2 a = unpack_bf16(u.x), b = unpack_bf16(u.y), e = unpack_bf16(u.z), f = unpack_bf16(u.w);
+  v[0] = a.x; v[1] = a.y; v[2] = b.x; v[3] = b.y; v[4] = e.x; v[5] = e.y; v[6] = f.x; v[7] = f.y;
+}
+
+template <int BN, bool A_MN, bool B_MN, class Epi>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   int M, int N, int K, Epi epi, BRows brows) {
-  using Cfg = GemmCfg<BN>;
+                   const __grid_constant__ CUtensorMap tmX, int M, int N, int K, Epi epi) {
+  using Cfg = GemmCfg<BN, Epi::kXTile>;
   constexpr int STAGES = Cfg::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * Cfg::STAGE_BYTES);
-  // bars[0..S): full, bars[S..2S): empty, bars[2S]: done
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 1);
-  __shared__ int s_consumed;
+  uint8_t* xtile = smem + STAGES * Cfg::STAGE_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(xtile + Cfg::X_BYTES);
+  // bars: full[S], empty[S], tfull[2], tempty[2], xfull, done
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 6);
+  __shared__ uint32_t s_consumed;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n_tile = blockIdx.x, m_tile = blockIdx.y;
-  const int m0 = m_tile * GEMM_BM, n0 = n_tile * BN;
+  const int num_n = (N + BN - 1) / BN;
+  const int tiles = ((M + GEMM_BM - 1) / GEMM_BM) * num_n;
   const int num_k = (K + GEMM_BK - 1) / GEMM_BK;
-  const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + STAGES),
-                 done = smem_u32(bars + 2 * STAGES);
+  const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + STAGES);
+  const uint32_t tfull0 = smem_u32(bars + 2 * STAGES), tempty0 = tfull0 + 16;
+  const uint32_t xfull = tfull0 + 32, done = tfull0 + 40;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(full0 + 8 * s, 1);
       mbar_init(empty0 + 8 * s, 1);
     }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(tfull0 + 8 * b, 1);
+      mbar_init(tempty0 + 8 * b, 4);  // one arrival per epilogue warp
+    }
+    mbar_init(xfull, 1);
     mbar_init(done, 1);
     fence_barrier_init();
     s_consumed = 0;
   }
   if (warp == 1) {
-    tmem_alloc(smem_u32(tmem_slot), BN);
+    tmem_alloc(smem_u32(tmem_slot), 2 * BN);
     tmem_relinquish();
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  int issued = 0;
+  uint32_t issued = 0;
+  bool x_pending = false;
+  uint32_t x_parity = 0;
 
   if (warp == 0 && lane == 0) {
     // ---------------------------------------------------------- producer
     prefetch_tmap(&tmA);
     prefetch_tmap(&tmB);
-    for (int kt = 0; kt < num_k; ++kt) {
-      const int s = kt % STAGES;
-      const uint32_t ph = (kt / STAGES) & 1;
-      if (!mbar_wait(empty0 + 8 * s, ph ^ 1)) break;
-      const uint32_t fb = full0 + 8 * s;
-      mbar_arrive_expect_tx(fb, Cfg::STAGE_BYTES);
-      const uint32_t a_dst = smem_u32(smem + s * Cfg::STAGE_BYTES);
-      const uint32_t b_dst = a_dst + Cfg::A_BYTES;
-      const int k0 = kt * GEMM_BK;
-      if (!A_MN) {
-        tma_load_2d(a_dst, &tmA, fb, k0, m0);
-      } else {
-        tma_load_2d(a_dst, &tmA, fb, m0, k0);
-        tma_load_2d(a_dst + 8192, &tmA, fb, m0 + 64, k0);
-      }
-      if (!B_MN) {
+    uint32_t it = 0;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
+      const int m0 = (tile / num_n) * GEMM_BM, n0 = (tile % num_n) * BN;
+      for (int kt = 0; kt < num_k; ++kt, ++it) {
+        const int s = it % STAGES;
+        const uint32_t ph = (it / STAGES) & 1;
+        if (!mbar_wait(empty0 + 8 * s, ph ^ 1)) {
+          ok = false;
+          break;
+        }
+        const uint32_t fb = full0 + 8 * s;
+        mbar_arrive_expect_tx(fb, Cfg::STAGE_BYTES);
+        const uint32_t a_dst = smem_u32(smem + s * Cfg::STAGE_BYTES);
+        const uint32_t b_dst = a_dst + Cfg::A_BYTES;
+        const int k0 = kt * GEMM_BK;
+        if (!A_MN) {
+          tma_load_2d(a_dst, &tmA, fb, k0, m0);
+        } else {
+          tma_load_2d(a_dst, &tmA, fb, m0, k0);
+          tma_load_2d(a_dst + 8192, &tmA, fb, m0 + 64, k0);
+        }
+        if (!B_MN) {
 #pragma unroll
-        for (int j = 0; j < BN / 128; ++j) tma_load_2d(b_dst + j * 16384, &tmB, fb, k0, brows(n_tile, j, BN));
-      } else {
+          for (int j = 0; j < BN / 128; ++j) tma_load_2d(b_dst + j * 16384, &tmB, fb, k0, n0 + 128 * j);
+        } else {
 #pragma unroll
-        for (int j = 0; j < BN / 64; ++j) tma_load_2d(b_dst + j * 8192, &tmB, fb, n0 + 64 * j, k0);
+          for (int j = 0; j < BN / 64; ++j) tma_load_2d(b_dst + j * 8192, &tmB, fb, n0 + 64 * j, k0);
+        }
+        issued = it + 1;
       }
-      issued = kt + 1;
     }
   } else if (warp == 1 && lane == 0) {
     // ---------------------------------------------------------- MMA issuer
     constexpr uint32_t idesc = idesc_bf16_f32(GEMM_BM, BN, A_MN ? 1 : 0, B_MN ? 1 : 0);
-    int kt = 0;
-    for (; kt < num_k; ++kt) {
-      const int s = kt % STAGES;
-      const uint32_t ph = (kt / STAGES) & 1;
-      if (!mbar_wait(full0 + 8 * s, ph)) break;
+    uint32_t it = 0, lt = 0;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x, ++lt) {
+      const uint32_t buf = lt & 1, use = lt >> 1;
+      if (!mbar_wait(tempty0 + 8 * buf, (use & 1) ^ 1)) break;
       tc_fence_after();
-      const uint32_t a_base = smem_u32(smem + s * Cfg::STAGE_BYTES);
-      const uint32_t b_base = a_base + Cfg::A_BYTES;
+      const uint32_t d_tmem = tmem + buf * BN;
+      for (int kt = 0; kt < num_k; ++kt, ++it) {
+        const int s = it % STAGES;
+        const uint32_t ph = (it / STAGES) & 1;
+        if (!mbar_wait(full0 + 8 * s, ph)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t a_base = smem_u32(smem + s * Cfg::STAGE_BYTES);
+        const uint32_t b_base = a_base + Cfg::A_BYTES;
 #pragma unroll
-      for (int kk = 0; kk < GEMM_BK / 16; ++kk) {
-        // K-major: 16 K-elements = 32 bytes along the swizzled 128-byte row,
-        //          8-row groups 1024 bytes apart (SBO).
-        // MN-major: 16 K-rows = 2048 bytes; 64-wide MN slabs 8192 bytes apart
-        //          (LBO), 8-row K groups 1024 bytes apart (SBO).
-        const uint64_t ad = A_MN ? smem_desc_sw128(a_base + kk * 2048, 8192, 1024)
-                                 : smem_desc_sw128(a_base + kk * 32, 16, 1024);
-        const uint64_t bd = B_MN ? smem_desc_sw128(b_base + kk * 2048, 8192, 1024)
-                                 : smem_desc_sw128(b_base + kk * 32, 16, 1024);
-        tc_mma_f16(tmem, ad, bd, idesc, (kt | kk) != 0 ? 1u : 0u);
+        for (int kk = 0; kk < GEMM_BK / 16; ++kk) {
+          // K-major: 16 K-elements = 32 bytes along the swizzled 128-byte row,
+          //          8-row groups 1024 bytes apart (SBO).
+          // MN-major: 16 K-rows = 2048 bytes; 64-wide MN slabs 8192 bytes apart
+          //          (LBO), 8-row K groups 1024 bytes apart (SBO).
+          const uint64_t ad = A_MN ? smem_desc_sw128(a_base + kk * 2048, 8192, 1024)
+                                   : smem_desc_sw128(a_base + kk * 32, 16, 1024);
+          const uint64_t bd = B_MN ? smem_desc_sw128(b_base + kk * 2048, 8192, 1024)
+                                   : smem_desc_sw128(b_base + kk * 32, 16, 1024);
+          tc_mma_f16(d_tmem, ad, bd, idesc, (kt | kk) != 0 ? 1u : 0u);
+        }
+        tc_commit(empty0 + 8 * s);
       }
-      tc_commit(empty0 + 8 * s);
+      tc_commit(tfull0 + 8 * buf);
     }
-    s_consumed = kt;
+    s_consumed = it;
     tc_commit(done);
   } else if (warp >= 2) {
     // ---------------------------------------------------------- epilogue
-    mbar_wait(done, 0);
-    tc_fence_after();
+    const int et = threadIdx.x - 64;
     const int q = warp & 3;
-    const int row = m0 + q * 32 + lane;
-#pragma unroll 1
-    for (int c = 0; c < BN; c += 32) {
-      float v[32];
-      tmem_ld32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)c, v);
-      if (num_k == 0) {
+    uint32_t lt = 0;
+    for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++lt) {
+      const int m0 = (tile / num_n) * GEMM_BM, n0 = (tile % num_n) * BN;
+      const uint32_t buf = lt & 1, use = lt >> 1;
+      if (Epi::kXTile && et == 0) {
+        mbar_arrive_expect_tx(xfull, Cfg::X_BYTES);
+        const int xr = epi.x_row(m0);
 #pragma unroll
-        for (int i = 0; i < 32; ++i) v[i] = 0.f;
+        for (int j = 0; j < BN / 64; ++j)
+          tma_load_2d(smem_u32(xtile) + j * 16384, &tmX, xfull, n0 + 64 * j, xr);
+        x_pending = true;
+        x_parity = lt & 1;
       }
-      epi.apply(row, n0 + c, v);
+      const bool ok = mbar_wait(tfull0 + 8 * buf, use & 1);
+      tc_fence_after();
+      if (Epi::kXTile) {
+        mbar_wait(xfull, lt & 1);
+        x_pending = false;
+      }
+      const int rl = q * 32 + lane;
+#pragma unroll 1
+      for (int c = 0; c < BN; c += 32) {
+        float v[32];
+        tmem_ld32(tmem + buf * BN + ((uint32_t)(q * 32) << 16) + (uint32_t)c, v);
+        if (num_k == 0) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = 0.f;
+        }
+        epi.apply(m0 + rl, n0 + c, v, xtile, rl, c);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(tempty0 + 8 * buf);
+      // all epilogue threads are done with the X tile (free for the next
+      // prefetch); leave together if any of them saw a wait run out
+      if (!epi_bar_and(ok)) break;
     }
   }
   tc_fence_before();
   if (__syncthreads_or(*(volatile int*)&g_dev_error != 0)) {
     // error path: let in-flight TMA copies and MMAs land before TMEM/smem go.
     if (warp == 0 && lane == 0) {
-      for (int kt = s_consumed; kt < issued; ++kt)
-        mbar_wait(full0 + 8 * (kt % STAGES), (kt / STAGES) & 1);
+      for (uint32_t it = s_consumed; it < issued; ++it)
+        mbar_wait(full0 + 8 * (it % STAGES), (it / STAGES) & 1);
     }
+    if (warp == 2 && lane == 0 && x_pending) mbar_wait(xfull, x_parity);
     if (warp == 1 && lane == 0) mbar_wait(done, 0);
     __syncthreads();
+  } else if (warp == 1 && lane == 0) {
+    mbar_wait(done, 0);
   }
+  __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, BN);
+    tmem_dealloc(tmem, 2 * BN);
   }
 }
 
 // ------------------------------------------------------------------ epilogues
-// Each epilogue's apply(row, col, v) receives 32 consecutive accumulator
-// columns [col, col+32) of output row `row` (N is a multiple of 32).
+// apply(row, col, v, xt, rl, cl) receives 32 consecutive accumulator columns
+// [col, col+32) of output row `row`; rl / cl are the row and column inside the
+// tile, xt the prefetched bf16 tile (kXTile epilogues; x_row(m0) gives the row
+// of the tile's first line in the X tensor map).  N is a multiple of 32.
 
 // v = acc (+ bias[col]) (+ addend[row, col]); stored as fp32 and/or bf16.
 struct EpiLinear {
+  static constexpr bool kXTile = false;
   int M, N;
   const float* bias;
   const float* addend;
@@ -185,7 +270,8 @@ struct EpiLinear {
   long ld_f32;
   bf16* out_bf16;
   long ld_bf16;
-  __device__ __forceinline__ void apply(int row, int col, float* v) const {
+  __device__ __forceinline__ int x_row(int m0) const { return m0; }
+  __device__ __forceinline__ void apply(int row, int col, float* v, const uint8_t*, int, int) const {
     if (row >= M || col >= N) return;
     if (bias) {
 #pragma unroll
@@ -224,15 +310,19 @@ struct EpiLinear {
 // (i+shift)*P + a*k1 + c/d:
 //   gated: X_out = X + sigmoid(w_x X + w_dlt D + b_g) D    (Eq. inj-gate)
 //   add:   X_out = X + D                                    (Eq. inj-add)
+// X is read from the prefetched tile: rows r + shift*k2 of the view
+// [B*m*k2, k1*d] of X (zero-padded to whole blocks when L % P != 0).
 struct EpiInject1D {
+  static constexpr bool kXTile = true;
   int M, N;
   const float* bias;
   bf16* D_save;
-  const bf16* X;
   bf16* X_out;
   const float *w_x, *w_dlt, *b_g;
   int d, k1, k2, m, L, shift, gated;
-  __device__ __forceinline__ void apply(int row, int col, float* v) const {
+  __device__ __forceinline__ int x_row(int m0) const { return m0 + shift * k2; }
+  __device__ __forceinline__ void apply(int row, int col, float* v, const uint8_t* xt, int rl,
+                                        int cl) const {
     if (row >= M || col >= N) return;
 #pragma unroll
     for (int i = 0; i < 32; i += 4) {
@@ -255,12 +345,20 @@ struct EpiInject1D {
 #pragma unroll
     for (int i8 = 0; i8 < 32; i8 += 8) {
       float x[8], o[8];
-      load8_bf16(X + off + i8, x);
+      xtile_load8(xt, rl, cl + i8, x);
       if (gated) {
+        float4 wx0 = *reinterpret_cast<const float4*>(w_x + ch + i8);
+        float4 wx1 = *reinterpret_cast<const float4*>(w_x + ch + i8 + 4);
+        float4 wd0 = *reinterpret_cast<const float4*>(w_dlt + ch + i8);
+        float4 wd1 = *reinterpret_cast<const float4*>(w_dlt + ch + i8 + 4);
+        float4 bg0 = *reinterpret_cast<const float4*>(b_g + ch + i8);
+        float4 bg1 = *reinterpret_cast<const float4*>(b_g + ch + i8 + 4);
+        const float wx[8] = {wx0.x, wx0.y, wx0.z, wx0.w, wx1.x, wx1.y, wx1.z, wx1.w};
+        const float wd[8] = {wd0.x, wd0.y, wd0.z, wd0.w, wd1.x, wd1.y, wd1.z, wd1.w};
+        const float bg[8] = {bg0.x, bg0.y, bg0.z, bg0.w, bg1.x, bg1.y, bg1.z, bg1.w};
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
-          const int c = ch + i8 + j;
-          const float g = w_x[c] * x[j] + w_dlt[c] * v[i8 + j] + b_g[c];
+          const float g = wx[j] * x[j] + wd[j] * v[i8 + j] + bg[j];
           o[j] = x[j] + sigmoidf_(g) * v[i8 + j];
         }
       } else {
@@ -272,14 +370,19 @@ struct EpiInject1D {
   }
 };
 
-// First compression level's input gradient, accumulated onto the direct
-// injection gradient already held in dX: rows r = (b*m + i)*k2 + a, columns
-// (token c/d of the group, channel c%d) -> token i*P + a*k1 + c/d of sequence b.
+// First compression level's input gradient added to the direct injection
+// gradient: rows r = (b*m + i)*k2 + a, columns (token c/d of the group, channel
+// c%d) -> token i*P + a*k1 + c/d of sequence b.  The direct gradient is read
+// from the prefetched tile of dXd, the view [B*m*k2, k1*d] of a buffer padded
+// to whole blocks (dX itself when L % P == 0); the sum is written to dX.
 struct EpiDX1D {
+  static constexpr bool kXTile = true;
   int M, N;
   bf16* dX;
   int d, k1, k2, m, L;
-  __device__ __forceinline__ void apply(int row, int col, float* v) const {
+  __device__ __forceinline__ int x_row(int m0) const { return m0; }
+  __device__ __forceinline__ void apply(int row, int col, float* v, const uint8_t* xt, int rl,
+                                        int cl) const {
     if (row >= M || col >= N) return;
     const int per_seq = m * k2;
     const int b = row / per_seq, rr = row % per_seq;
@@ -289,7 +392,7 @@ struct EpiDX1D {
 #pragma unroll
     for (int i8 = 0; i8 < 32; i8 += 8) {
       float x[8];
-      load8_bf16(dX + off + i8, x);
+      xtile_load8(xt, rl, cl + i8, x);
 #pragma unroll
       for (int j = 0; j < 8; ++j) x[j] += v[i8 + j];
       store8_bf16(dX + off + i8, x);

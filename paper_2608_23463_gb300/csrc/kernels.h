@@ -28,13 +28,14 @@ struct EpiLinearArgs {
 struct EpiInjectArgs {
   const float* bias;  // b_d1 [k1*d]
   bf16* D_save;       // [M, k1*d] or null
-  const bf16* X;
+  const bf16* Xsrc;   // X as [B*m*k2, k1*d] (zero-padded to whole blocks if L % P != 0)
   bf16* X_out;
   const float *w_x, *w_dlt, *b_g;  // gate vectors (gated) or null (add)
   int d, k1, k2, m, L, shift, gated;
 };
 
 struct EpiDXArgs {
+  const bf16* dXd;  // direct gradient as [B*m*k2, k1*d] (padded like Xsrc)
   bf16* dX;
   int d, k1, k2, m, L;
 };
@@ -59,9 +60,9 @@ cudaError_t attn_bwd(const bf16* qkv, const bf16* O, const bf16* dO, const float
                      bf16* dqkv, int B, int m, int d, int nh, bool causal, cudaStream_t st);
 
 // ----------------------------------------------------------- elementwise
-// Copy `rows_per_seq` rows of width d from the start of each sequence of src
-// [B, L, d] to dst (block 0 of the causal routing: X_out = X, dX = dX_out).
-cudaError_t copy_block0(const bf16* src, bf16* dst, int B, long L, int d, int rows,
+// Copy the first `rows` rows (width d) of each sequence of src [B, Ls, d] to
+// dst [B, Ld, d] (block 0 of the causal routing: X_out = X, dX = dX_out).
+cudaError_t copy_block0(const bf16* src, long Ls, bf16* dst, long Ld, int B, int d, int rows,
                         cudaStream_t st);
 // dst [B, Lp, d] = src [B, L, d] padded with zero rows (Lp >= L).
 cudaError_t pad_rows(const bf16* src, bf16* dst, int B, long L, long Lp, int d, cudaStream_t st);
@@ -76,7 +77,8 @@ struct InjBwdArgs {
   const bf16* X;
   const bf16* D;
   bf16* dD;
-  bf16* dX;
+  bf16* dX;     // direct gradient, [B, Ldx, d]
+  long Ldx;     // rows per sequence of dX (L, or m*P when padded)
   const float *w_x, *w_dlt, *b_g;
   int d, k1, k2, m, L, B, shift, gated;
 };
