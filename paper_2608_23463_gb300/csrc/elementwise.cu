@@ -29,91 +29,139 @@ __global__ void pad_rows_kernel(const bf16* __restrict__ src, bf16* __restrict__
   *reinterpret_cast<uint4*>(dst + (long)b * Lp * d + i * 8) = v;
 }
 
-__global__ void __launch_bounds__(EW_THREADS) inj_bwd_kernel(InjBwdArgs a, float* __restrict__ part,
-                                                             long M, int N, long rows_per_chunk) {
-  const int col = (blockIdx.x * EW_THREADS + threadIdx.x) * 8;
+__device__ __forceinline__ void load4_bf16(const bf16* p, float* v) {
+  const uint2 u = *reinterpret_cast<const uint2*>(p);
+  const float2 a = unpack_bf16(u.x), b = unpack_bf16(u.y);
+  v[0] = a.x; v[1] = a.y; v[2] = b.x; v[3] = b.y;
+}
+__device__ __forceinline__ void store4_bf16(bf16* p, const float* v) {
+  *reinterpret_cast<uint2*>(p) = make_uint2(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]));
+}
+
+// Each thread owns 4 consecutive columns and walks a chunk of rows, INJ_U
+// rows at a time with their loads issued together.
+constexpr int INJ_COLS = 4;
+constexpr int INJ_U = 2;
+
+__global__ void __launch_bounds__(EW_THREADS, 3) inj_bwd_kernel(InjBwdArgs a, float* __restrict__ part,
+                                                                long M, int N, long rows_per_chunk) {
+  const int col = (blockIdx.x * EW_THREADS + threadIdx.x) * INJ_COLS;
   if (col >= N) return;
+  const bf16* __restrict__ G = a.G;
+  const bf16* __restrict__ X = a.X;
+  const bf16* __restrict__ D = a.D;
+  bf16* __restrict__ dD = a.dD;
+  bf16* __restrict__ dX = a.dX;
   const long r0 = (long)blockIdx.y * rows_per_chunk;
   const long r1 = min(M, r0 + rows_per_chunk);
   const int P = a.k1 * a.k2;
   const int ch = col % a.d, tq = col / a.d;
-  float wx[8], wd[8], bg[8];
-  if (a.gated) {
+  float wx[INJ_COLS], wd[INJ_COLS], bg[INJ_COLS];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      wx[j] = a.w_x[ch + j];
-      wd[j] = a.w_dlt[ch + j];
-      bg[j] = a.b_g[ch + j];
-    }
+  for (int j = 0; j < INJ_COLS; ++j) {
+    wx[j] = a.gated ? a.w_x[ch + j] : 0.f;
+    wd[j] = a.gated ? a.w_dlt[ch + j] : 0.f;
+    bg[j] = a.gated ? a.b_g[ch + j] : 0.f;
   }
-  float acc[4][8] = {};
-  for (long r = r0; r < r1; ++r) {
-    const int grp = (int)(r % a.k2);
-    const long prox = r / a.k2;
-    const int b = (int)(prox / a.m), i = (int)(prox % a.m);
-    const int it = i + a.shift;
-    const long tok = (long)it * P + (long)grp * a.k1 + tq;
-    float dd[8];
-    if (it < a.m && tok < a.L) {
-      const long off = ((long)b * a.L + tok) * a.d + ch;
-      float g[8], x[8], D[8], dx[8];
-      load8_bf16(a.G + off, g);
-      load8_bf16(a.X + off, x);
-      load8_bf16(a.D + r * N + col, D);
-      if (a.gated) {
+  float acc[4][INJ_COLS] = {};
+  for (long rb = r0; rb < r1; rb += INJ_U) {
+    long offx[INJ_U];
+    bool valid[INJ_U];
+    float g[INJ_U][INJ_COLS], x[INJ_U][INJ_COLS], Dv[INJ_U][INJ_COLS];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const float s = sigmoidf_(wx[j] * x[j] + wd[j] * D[j] + bg[j]);
-          const float ds = g[j] * D[j] * s * (1.f - s);
-          dx[j] = g[j] + ds * wx[j];
-          dd[j] = g[j] * s + ds * wd[j];
-          acc[1][j] += ds * x[j];
-          acc[2][j] += ds * D[j];
-          acc[3][j] += ds;
-        }
-      } else {
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          dx[j] = g[j];
-          dd[j] = g[j];
+    for (int u = 0; u < INJ_U; ++u) {
+      const long r = rb + u;
+      valid[u] = false;
+      offx[u] = 0;
+      if (r < r1) {
+        const int grp = (int)(r % a.k2);
+        const long prox = r / a.k2;
+        const int b = (int)(prox / a.m), i = (int)(prox % a.m);
+        const int it = i + a.shift;
+        const long tok = (long)it * P + (long)grp * a.k1 + tq;
+        if (it < a.m && tok < a.L) {
+          valid[u] = true;
+          const long off = ((long)b * a.L + tok) * a.d + ch;
+          offx[u] = ((long)b * a.Ldx + tok) * a.d + ch;
+          load4_bf16(G + off, g[u]);
+          load4_bf16(X + off, x[u]);
+          load4_bf16(D + r * N + col, Dv[u]);
         }
       }
-      store8_bf16(a.dX + ((long)b * a.Ldx + tok) * a.d + ch, dx);
-    } else {
-#pragma unroll
-      for (int j = 0; j < 8; ++j) dd[j] = 0.f;
     }
-    // round dD once; the column sum uses the same rounded values the
-    // downstream GEMMs see.
-    store8_bf16(a.dD + r * N + col, dd);
 #pragma unroll
-    for (int j = 0; j < 8; ++j) acc[0][j] += __bfloat162float(__float2bfloat16(dd[j]));
+    for (int u = 0; u < INJ_U; ++u) {
+      const long r = rb + u;
+      if (r >= r1) break;
+      float dd[INJ_COLS];
+      if (valid[u]) {
+        float dx[INJ_COLS];
+#pragma unroll
+        for (int j = 0; j < INJ_COLS; ++j) {
+          if (a.gated) {
+            const float sg = sigmoidf_(fmaf(wx[j], x[u][j], fmaf(wd[j], Dv[u][j], bg[j])));
+            const float ds = g[u][j] * Dv[u][j] * sg * (1.f - sg);
+            dx[j] = fmaf(ds, wx[j], g[u][j]);
+            dd[j] = fmaf(g[u][j], sg, ds * wd[j]);
+            acc[1][j] += ds * x[u][j];
+            acc[2][j] += ds * Dv[u][j];
+            acc[3][j] += ds;
+          } else {
+            dx[j] = g[u][j];
+            dd[j] = g[u][j];
+          }
+        }
+        store4_bf16(dX + offx[u], dx);
+      } else {
+#pragma unroll
+        for (int j = 0; j < INJ_COLS; ++j) dd[j] = 0.f;
+      }
+      // round dD once; the column sum uses the same rounded values the
+      // downstream GEMMs see.
+      store4_bf16(dD + r * N + col, dd);
+#pragma unroll
+      for (int j = 0; j < INJ_COLS; ++j) acc[0][j] += __bfloat162float(__float2bfloat16(dd[j]));
+    }
   }
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     float* p = part + ((long)blockIdx.y * 4 + q) * N + col;
     *reinterpret_cast<float4*>(p) = make_float4(acc[q][0], acc[q][1], acc[q][2], acc[q][3]);
-    *reinterpret_cast<float4*>(p + 4) = make_float4(acc[q][4], acc[q][5], acc[q][6], acc[q][7]);
   }
 }
 
+// Deterministic warp sum: lane j adds summands j, j+32, ... in order, then a
+// fixed xor-shuffle tree.
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int s = 16; s > 0; s >>= 1) v += __shfl_xor_sync(0xffffffffu, v, s);
+  return v;
+}
+
+// One warp per output: db_d1[c] = sum over chunks of part[.][0][c]; gate
+// gradients g_q[ch] = sum over chunks and the k1 token positions t of
+// part[.][q][t*d + ch] (q = 1: w_x, 2: w_dlt, 3: b_g).
 __global__ void inj_bwd_finalize_kernel(const float* __restrict__ part, int n_chunks, int N, int d,
                                         float* db_d1, float* gw_x, float* gw_dlt, float* gb_g) {
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i < N) {
+  const int o = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (o < N) {
     float s = 0.f;
-    for (int c = 0; c < n_chunks; ++c) s += part[((long)c * 4) * N + i];
-    db_d1[i] = s;
+    for (int c = lane; c < n_chunks; c += 32) s += part[((long)c * 4) * N + o];
+    s = warp_sum(s);
+    if (lane == 0) db_d1[o] = s;
     return;
   }
-  const int j = i - N;
+  const int j = o - N;
   if (gw_x == nullptr || j >= 3 * d) return;
-  const int q = 1 + j / d, ch = j % d;
+  const int q = 1 + j / d, ch = j % d, T = N / d;
   float s = 0.f;
-  for (int c = 0; c < n_chunks; ++c)
-    for (int t = 0; t < N / d; ++t) s += part[((long)c * 4 + q) * N + t * d + ch];
-  float* dst = q == 1 ? gw_x : (q == 2 ? gw_dlt : gb_g);
-  dst[ch] = s;
+  for (int e = lane; e < n_chunks * T; e += 32) {
+    const int c = e / T, t = e % T;
+    s += part[((long)c * 4 + q) * N + (long)t * d + ch];
+  }
+  s = warp_sum(s);
+  if (lane == 0) (q == 1 ? gw_x : (q == 2 ? gw_dlt : gb_g))[ch] = s;
 }
 
 template <typename T>
@@ -147,13 +195,16 @@ __global__ void __launch_bounds__(EW_THREADS) colsum_part_kernel(const T* __rest
   *reinterpret_cast<float4*>(p + 4) = make_float4(acc[4], acc[5], acc[6], acc[7]);
 }
 
+// One warp per column (deterministic order, see warp_sum).
 __global__ void colsum_final_kernel(const float* __restrict__ part, int n_chunks, int C,
                                     float* __restrict__ out) {
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  const int i = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
   if (i >= C) return;
   float s = 0.f;
-  for (int c = 0; c < n_chunks; ++c) s += part[(long)c * C + i];
-  out[i] = s;
+  for (int c = lane; c < n_chunks; c += 32) s += part[(long)c * C + i];
+  s = warp_sum(s);
+  if (lane == 0) out[i] = s;
 }
 
 // Row chunks of a column reduction: about 1024 CTAs in total, independent of
@@ -177,7 +228,7 @@ cudaError_t colsum_impl(const T* X, long R, int C, float* out, float* part, cuda
   }
   {
     LaunchTimer lt("colsum_final", st, (double)nc * C, 4.0 * nc * C);
-    colsum_final_kernel<<<(C + 255) / 256, 256, 0, st>>>(part, nc, C, out);
+    colsum_final_kernel<<<(C + 7) / 8, 256, 0, st>>>(part, nc, C, out);
   }
   return cudaGetLastError();
 }
@@ -201,7 +252,7 @@ cudaError_t pad_rows(const bf16* src, bf16* dst, int B, long L, long Lp, int d, 
   return cudaGetLastError();
 }
 
-int inj_bwd_chunks(long M, int N) { return chunks_for(M, N); }
+int inj_bwd_chunks(long M, int N) { return chunks_for(M, 2 * N); }
 
 int take_dev_error_elementwise() { return take_dev_error_tu(); }
 
@@ -209,7 +260,7 @@ cudaError_t inj_bwd_1d(const InjBwdArgs& a, float* part, int n_chunks, cudaStrea
   const long M = (long)a.B * a.m * a.k2;
   const int N = a.k1 * a.d;
   const long rpc = (M + n_chunks - 1) / n_chunks;
-  dim3 grid((N / 8 + EW_THREADS - 1) / EW_THREADS, n_chunks);
+  dim3 grid((N / INJ_COLS + EW_THREADS - 1) / EW_THREADS, n_chunks);
   LaunchTimer lt("inj_bwd", st, 0.0, 10.0 * M * N + 16.0 * n_chunks * N);
   inj_bwd_kernel<<<grid, EW_THREADS, 0, st>>>(a, part, M, N, rpc);
   return cudaGetLastError();
@@ -219,8 +270,8 @@ cudaError_t inj_bwd_finalize(const float* part, int n_chunks, int N, int d, floa
                              float* gw_x, float* gw_dlt, float* gb_g, cudaStream_t st) {
   const int total = N + 3 * d;
   LaunchTimer lt("inj_bwd_finalize", st, 0.0, 16.0 * n_chunks * N);
-  inj_bwd_finalize_kernel<<<(total + 255) / 256, 256, 0, st>>>(part, n_chunks, N, d, db_d1, gw_x,
-                                                              gw_dlt, gb_g);
+  inj_bwd_finalize_kernel<<<(total + 7) / 8, 256, 0, st>>>(part, n_chunks, N, d, db_d1, gw_x,
+                                                          gw_dlt, gb_g);
   return cudaGetLastError();
 }
 

@@ -15,9 +15,10 @@
 //              N=BN, K=16 into one of two TMEM accumulators (2*BN columns),
 //              tcgen05.commit frees smem stages and hands a finished
 //              accumulator to the epilogue
-//   warps 2-5: epilogue: tcgen05.ld 32 columns at a time (warp w reads TMEM
-//              lanes 32*(w%4)..), fused epilogue functor, global stores.
-//              While they drain accumulator i, the MMA warp fills the other.
+//   warps 2-9: epilogue: tcgen05.ld 32 columns at a time (warp w reads TMEM
+//              lanes 32*(w%4).. and half of the tile's columns), fused
+//              epilogue functor, global stores.  While they drain
+//              accumulator i, the MMA warp fills the other.
 // Epilogues that read a bf16 tile shaped like the output (the local stream X
 // for injection, the direct gradient for dX) have it prefetched by TMA into
 // shared memory (128 x BN, 128B-swizzled) while the tile's mainloop runs.
@@ -31,7 +32,8 @@ namespace pf {
 
 constexpr int GEMM_BM = 128;
 constexpr int GEMM_BK = 64;
-constexpr int GEMM_THREADS = 192;
+constexpr int GEMM_EPI_WARPS = 8;  // two per TMEM lane quarter, each owning half the columns
+constexpr int GEMM_THREADS = 64 + 32 * GEMM_EPI_WARPS;
 
 template <int BN, bool XTILE>
 struct GemmCfg {
@@ -44,17 +46,17 @@ struct GemmCfg {
       STAGES * STAGE_BYTES + X_BYTES + 1024 /*align*/ + 256 /*barriers*/;
 };
 
-// Barrier of the 128 epilogue threads (named barrier 1) that also ANDs a
-// predicate across them, so that every epilogue thread takes the same branch.
+// Barrier of the epilogue threads (named barrier 1) that also ANDs a predicate
+// across them, so that every epilogue thread takes the same branch.
 __device__ __forceinline__ bool epi_bar_and(bool p) {
   uint32_t r;
   asm volatile(
       "{\n\t.reg .pred pi, po;\n\t"
       "setp.ne.u32 pi, %1, 0;\n\t"
-      "bar.red.and.pred po, 1, 128, pi;\n\t"
+      "bar.red.and.pred po, 1, %2, pi;\n\t"
       "selp.u32 %0, 1, 0, po;\n\t}"
       : "=r"(r)
-      : "r"((uint32_t)p)
+      : "r"((uint32_t)p), "n"(32 * GEMM_EPI_WARPS)
       : "memory");
   return r != 0;
 }
@@ -98,7 +100,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(tfull0 + 8 * b, 1);
-      mbar_init(tempty0 + 8 * b, 4);  // one arrival per epilogue warp
+      mbar_init(tempty0 + 8 * b, GEMM_EPI_WARPS);  // one arrival per epilogue warp
     }
     mbar_init(xfull, 1);
     mbar_init(done, 1);
@@ -194,7 +196,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   } else if (warp >= 2) {
     // ---------------------------------------------------------- epilogue
     const int et = threadIdx.x - 64;
-    const int q = warp & 3;
+    const int q = warp & 3;                               // TMEM lane quarter
+    const int c_begin = ((warp - 2) >> 2) * (BN / 2);     // this warp's column half
     uint32_t lt = 0;
     for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++lt) {
       const int m0 = (tile / num_n) * GEMM_BM, n0 = (tile % num_n) * BN;
@@ -215,15 +218,16 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         x_pending = false;
       }
       const int rl = q * 32 + lane;
+      const typename Epi::Row ri = epi.row_info(m0 + rl);
 #pragma unroll 1
-      for (int c = 0; c < BN; c += 32) {
+      for (int c = c_begin; c < c_begin + BN / 2; c += 32) {
         float v[32];
         tmem_ld32(tmem + buf * BN + ((uint32_t)(q * 32) << 16) + (uint32_t)c, v);
         if (num_k == 0) {
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] = 0.f;
         }
-        epi.apply(m0 + rl, n0 + c, v, xtile, rl, c);
+        epi.apply(ri, m0 + rl, n0 + c, v, xtile, rl, c);
       }
       tc_fence_before();
       __syncwarp();
@@ -254,14 +258,18 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
 }
 
 // ------------------------------------------------------------------ epilogues
-// apply(row, col, v, xt, rl, cl) receives 32 consecutive accumulator columns
-// [col, col+32) of output row `row`; rl / cl are the row and column inside the
-// tile, xt the prefetched bf16 tile (kXTile epilogues; x_row(m0) gives the row
-// of the tile's first line in the X tensor map).  N is a multiple of 32.
+// row_info(row) is evaluated once per tile and output row; apply(ri, row, col,
+// v, xt, rl, cl) then receives 32 consecutive accumulator columns [col,
+// col+32) of that row, with rl / cl the row and column inside the tile and xt
+// the prefetched bf16 tile (kXTile epilogues; x_row(m0) gives the row of the
+// tile's first line in the X tensor map).  N is a multiple of 32.
 
 // v = acc (+ bias[col]) (+ addend[row, col]); stored as fp32 and/or bf16.
 struct EpiLinear {
   static constexpr bool kXTile = false;
+  struct Row {
+    bool ok;
+  };
   int M, N;
   const float* bias;
   const float* addend;
@@ -271,8 +279,10 @@ struct EpiLinear {
   bf16* out_bf16;
   long ld_bf16;
   __device__ __forceinline__ int x_row(int m0) const { return m0; }
-  __device__ __forceinline__ void apply(int row, int col, float* v, const uint8_t*, int, int) const {
-    if (row >= M || col >= N) return;
+  __device__ __forceinline__ Row row_info(int row) const { return Row{row < M}; }
+  __device__ __forceinline__ void apply(const Row& ri, int row, int col, float* v, const uint8_t*,
+                                        int, int) const {
+    if (!ri.ok || col >= N) return;
     if (bias) {
 #pragma unroll
       for (int i = 0; i < 32; i += 4) {
@@ -314,6 +324,11 @@ struct EpiLinear {
 // [B*m*k2, k1*d] of X (zero-padded to whole blocks when L % P != 0).
 struct EpiInject1D {
   static constexpr bool kXTile = true;
+  struct Row {
+    bool ok;    // row < M
+    long off0;  // element offset of the group's first token in X_out
+    int lim;    // columns < lim belong to tokens < L of a target block
+  };
   int M, N;
   const float* bias;
   bf16* D_save;
@@ -321,9 +336,22 @@ struct EpiInject1D {
   const float *w_x, *w_dlt, *b_g;
   int d, k1, k2, m, L, shift, gated;
   __device__ __forceinline__ int x_row(int m0) const { return m0 + shift * k2; }
-  __device__ __forceinline__ void apply(int row, int col, float* v, const uint8_t* xt, int rl,
-                                        int cl) const {
-    if (row >= M || col >= N) return;
+  __device__ __forceinline__ Row row_info(int row) const {
+    Row r{row < M, 0, 0};
+    const int a = row % k2, prox = row / k2;
+    const int b = prox / m, i = prox % m;
+    const int it = i + shift;
+    const long tok0 = (long)it * (k1 * k2) + (long)a * k1;
+    if (r.ok && it < m && tok0 < L) {
+      r.off0 = ((long)b * L + tok0) * d;
+      const long lim = (L - tok0) * d;
+      r.lim = lim < N ? (int)lim : N;
+    }
+    return r;
+  }
+  __device__ __forceinline__ void apply(const Row& ri, int row, int col, float* v,
+                                        const uint8_t* xt, int rl, int cl) const {
+    if (!ri.ok || col >= N) return;
 #pragma unroll
     for (int i = 0; i < 32; i += 4) {
       float4 b = *reinterpret_cast<const float4*>(bias + col + i);
@@ -334,14 +362,9 @@ struct EpiInject1D {
 #pragma unroll
       for (int i = 0; i < 32; i += 8) store8_bf16(o + i, v + i);
     }
-    const int a = row % k2, prox = row / k2;
-    const int b = prox / m, i = prox % m;
-    const int it = i + shift;
-    if (it >= m) return;
-    const long tok = (long)it * (k1 * k2) + (long)a * k1 + col / d;
-    if (tok >= L) return;
+    if (col >= ri.lim) return;
     const int ch = col % d;
-    const long off = ((long)b * L + tok) * d + ch;
+    bf16* xo = X_out + ri.off0 + col;
 #pragma unroll
     for (int i8 = 0; i8 < 32; i8 += 8) {
       float x[8], o[8];
@@ -358,14 +381,14 @@ struct EpiInject1D {
         const float bg[8] = {bg0.x, bg0.y, bg0.z, bg0.w, bg1.x, bg1.y, bg1.z, bg1.w};
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
-          const float g = wx[j] * x[j] + wd[j] * v[i8 + j] + bg[j];
-          o[j] = x[j] + sigmoidf_(g) * v[i8 + j];
+          const float g = fmaf(wx[j], x[j], fmaf(wd[j], v[i8 + j], bg[j]));
+          o[j] = fmaf(sigmoidf_(g), v[i8 + j], x[j]);
         }
       } else {
 #pragma unroll
         for (int j = 0; j < 8; ++j) o[j] = x[j] + v[i8 + j];
       }
-      store8_bf16(X_out + off + i8, o);
+      store8_bf16(xo + i8, o);
     }
   }
 };
@@ -377,25 +400,38 @@ struct EpiInject1D {
 // to whole blocks (dX itself when L % P == 0); the sum is written to dX.
 struct EpiDX1D {
   static constexpr bool kXTile = true;
+  struct Row {
+    bool ok;
+    long off0;
+    int lim;
+  };
   int M, N;
   bf16* dX;
   int d, k1, k2, m, L;
   __device__ __forceinline__ int x_row(int m0) const { return m0; }
-  __device__ __forceinline__ void apply(int row, int col, float* v, const uint8_t* xt, int rl,
-                                        int cl) const {
-    if (row >= M || col >= N) return;
+  __device__ __forceinline__ Row row_info(int row) const {
+    Row r{row < M, 0, 0};
     const int per_seq = m * k2;
     const int b = row / per_seq, rr = row % per_seq;
-    const long tok = (long)rr * k1 + col / d;
-    if (tok >= L) return;
-    const long off = ((long)b * L + tok) * d + (col % d);
+    const long tok0 = (long)rr * k1;
+    if (r.ok && tok0 < L) {
+      r.off0 = ((long)b * L + tok0) * d;
+      const long lim = (L - tok0) * d;
+      r.lim = lim < N ? (int)lim : N;
+    }
+    return r;
+  }
+  __device__ __forceinline__ void apply(const Row& ri, int, int col, float* v, const uint8_t* xt,
+                                        int rl, int cl) const {
+    if (!ri.ok || col >= ri.lim) return;
+    bf16* o = dX + ri.off0 + col;
 #pragma unroll
     for (int i8 = 0; i8 < 32; i8 += 8) {
       float x[8];
       xtile_load8(xt, rl, cl + i8, x);
 #pragma unroll
       for (int j = 0; j < 8; ++j) x[j] += v[i8 + j];
-      store8_bf16(dX + off + i8, x);
+      store8_bf16(o + i8, x);
     }
   }
 };
