@@ -42,6 +42,8 @@ def parse_args():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--decode-steps", type=int, default=128)
     ap.add_argument("--L", type=int, default=0,
                     help="tokens per sequence (default: the workload's 262144; smaller values "
                          "are for profiling captures only)")
@@ -232,6 +234,62 @@ def traffic_from_profile(label: str, units: float):
     return None
 
 
+def measure_decode(torch, pf, S, steps: int):
+    """Proxy-KV decode step at the paper's decode shape: B = 8, d = 2048, 16 x 128
+    heads, 16384 cached proxies per sequence, open block cycling through 0..63
+    tokens.  Each step is timed with CUDA events on its stream; the open block
+    is reset between passes outside the timed spans."""
+    import numpy as np
+
+    from paper_2608_23463_gb300.decode import ProxyKVCache
+    spec = S.spec_c4()
+    prm = S.make_decode_params(spec, 3)
+    st = S.make_decode_state(spec, 3, [spec.capacity] * spec.batch, [0] * spec.batch)
+    cache = ProxyKVCache(spec, prm, st)
+    del st
+    x = torch.from_numpy(S.round_bf16(np.random.default_rng(4).standard_normal(
+        (spec.batch, spec.d)).astype(np.float32))).cuda().to(torch.bfloat16)
+    y = torch.empty_like(x)
+    stream = torch.cuda.current_stream()
+    for _ in range(3):
+        cache.step(x, y)
+    cache.s["n_open"].zero_()
+    torch.cuda.synchronize()
+    pairs = []
+    pf.pf_timing_enable(True)
+    for i in range(steps):
+        if i and i % spec.P == 0:
+            cache.s["n_open"].zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        cache.step(x, y)
+        e1.record(stream)
+        pairs.append((e0, e1))
+    torch.cuda.synchronize()
+    pf.pf_sync_check(stream.cuda_stream)
+    ms = sum(a.elapsed_time(b) for a, b in pairs) / steps
+    kern = {k: v["ms"] / steps for k, v in pf.pf_timing_collect().items()}
+    pf.pf_timing_enable(False)
+    # one block-triggered append (full open blocks, one free cache row each)
+    cache.s["n_open"].fill_(spec.P)
+    cache.s["n_proxy"].fill_(spec.capacity - 1)
+    cache.append()
+    cache.s["n_open"].fill_(spec.P)
+    cache.s["n_proxy"].fill_(spec.capacity - 1)
+    torch.cuda.synchronize()
+    a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a0.record(stream)
+    cache.append()
+    a1.record(stream)
+    torch.cuda.synchronize()
+    pf.pf_sync_check(stream.cuda_stream)
+    B, d, cap = spec.batch, spec.d, spec.capacity
+    mean_open = (min(steps, spec.P) + 1) / 2.0
+    step_bytes = (2 * B * cap * d * 2 + (3 * d * d + d * d + d * d // 8) * 2
+                  + B * mean_open * 2 * d * 2 + 2 * B * d * 2)
+    return spec, ms, a0.elapsed_time(a1), step_bytes, kern
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -334,6 +392,12 @@ def run_ours(args, rank: int, world: int, local_rank: int):
         ms_e2e = float(t.item())
     pf.pf_sync_check(stream.cuda_stream)
     act_bytes = spec.batch * spec.L * spec.d * 2
+    del Xh, Gh, Xoh, dXh, X2, G2
+    decode_result = None
+    if not args.no_decode:
+        del lay, X, G, Xo, dX
+        torch.cuda.empty_cache()
+        decode_result = measure_decode(torch, pf, S, args.decode_steps)
     if rank != 0:
         return
 
@@ -378,6 +442,18 @@ def run_ours(args, rank: int, world: int, local_rank: int):
                     "h2d_bytes_per_step": 2 * act_bytes, "d2h_bytes_per_step": 2 * act_bytes,
                     "ms_per_step": ms_e2e},
             "gpu_launches": launches, "clocks": clocks, "kernels": breakdown}
+    if not args.no_decode:
+        dspec, dms, app_ms, dbytes, dkern = decode_result
+        line["decode"] = {
+            "metric": "proxy-KV decode new tokens/s per layer (B=8, 16384 cached proxies, "
+                      "d=2048, 16x128 heads, open block 0..63)",
+            "value": dspec.batch / (dms / 1e3), "unit": "tokens/s", "ms_per_step": dms,
+            "steps": args.decode_steps,
+            "roofline": {"bound": "hbm", "achieved": dbytes / (dms / 1e3) / 1e9,
+                         "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                         "frac": dbytes / (dms / 1e3) / 1e9 / peaks["hbm_gbs"],
+                         "bytes_per_step": dbytes},
+            "append_ms": app_ms, "kernels_ms_per_step": dkern}
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline_subprocess()
     print(json.dumps(line), flush=True)

@@ -468,34 +468,185 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
   return PF_OK;
 }
 
-size_t proxy_decode_workspace_size(const pf_decode_desc* desc) {
-  (void)desc;
-  return 0;
-}
-size_t proxy_append_workspace_size(const pf_decode_desc* desc) {
-  (void)desc;
-  return 0;
+}  // extern "C"
+
+namespace {
+
+pf_status check_decode_desc(const pf_decode_desc* s) {
+  if (s == nullptr) return fail(PF_ERR_INVALID_ARG, "decode descriptor is NULL");
+  if (s->batch < 1) return fail(PF_ERR_INVALID_ARG, "batch must be >= 1");
+  if (s->d < 64 || s->d % 64 != 0 || s->d > 4096)
+    return fail(PF_ERR_INVALID_ARG, "d must be a multiple of 64 in [64, 4096]");
+  if (s->n_heads < 1 || s->d % s->n_heads != 0)
+    return fail(PF_ERR_INVALID_ARG, "n_heads must divide d");
+  const int dh = s->d / s->n_heads;
+  if (dh != 64 && dh != 128) return fail(PF_ERR_UNSUPPORTED, "head width must be 64 or 128");
+  if (s->P < 1 || s->P > PF_DECODE_MAX_P)
+    return fail(PF_ERR_UNSUPPORTED, "P must be in [1, %d]", PF_DECODE_MAX_P);
+  if (s->levels != 1 && s->levels != 2) return fail(PF_ERR_INVALID_ARG, "levels must be 1 or 2");
+  if (s->levels == 2 && (s->k1 < 1 || s->k2 < 1 || (long)s->k1 * s->k2 != s->P))
+    return fail(PF_ERR_INVALID_ARG, "levels == 2 needs k1 * k2 == P");
+  if (s->capacity < 1) return fail(PF_ERR_INVALID_ARG, "capacity must be >= 1");
+  return PF_OK;
 }
 
-pf_status proxy_decode_step(const pf_decode_desc* desc, const pf_decode_params* params,
+bool cache_ok(const pf_kv_cache* c) {
+  return c && c->K_proxy && c->V_proxy && c->X_open && c->K_open && c->V_open && c->n_proxy &&
+         c->n_open && aligned16(c->K_proxy) && aligned16(c->V_proxy) && aligned16(c->X_open) &&
+         aligned16(c->K_open) && aligned16(c->V_open) && aligned16(c->n_proxy) &&
+         aligned16(c->n_open);
+}
+
+struct AppendWs {
+  bf16* Y;
+  float* Hf;
+  bf16* Hb;
+};
+
+AppendWs carve_append(Carve& c, const pf_decode_desc& s) {
+  AppendWs w{};
+  const long k2 = s.levels == 2 ? s.k2 : 1;
+  if (s.levels == 2) w.Y = c.take<bf16>((size_t)s.batch * k2 * s.d);
+  w.Hf = c.take<float>((size_t)s.batch * s.d);
+  w.Hb = c.take<bf16>((size_t)s.batch * s.d);
+  return w;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t proxy_decode_workspace_size(const pf_decode_desc* desc) {
+  if (check_decode_desc(desc) != PF_OK) return 0;
+  const int splits = decode_splits(desc->batch, desc->n_heads, desc->capacity);
+  return decode_workspace_bytes(desc->batch, desc->d, desc->n_heads, splits);
+}
+
+size_t proxy_append_workspace_size(const pf_decode_desc* desc) {
+  if (check_decode_desc(desc) != PF_OK) return 0;
+  Carve c(nullptr);
+  carve_append(c, *desc);
+  return ((c.off + 255) & ~size_t(255)) + 256;
+}
+
+pf_status proxy_decode_step(const pf_decode_desc* desc, const pf_decode_params* prm,
                             const void* x, pf_kv_cache* cache, void* y, void* ws, size_t ws_bytes,
                             void* stream) {
-  (void)desc; (void)params; (void)x; (void)cache; (void)y; (void)ws; (void)ws_bytes; (void)stream;
-  return fail(PF_ERR_UNSUPPORTED, "decode step is not built yet");
+  pf_status st = check_decode_desc(desc);
+  if (st != PF_OK) return st;
+  if (!prm || !prm->W_qkv || !prm->W_o || !prm->rms_w || !prm->W_a1 || !prm->b_a1 || !prm->W_a2 ||
+      !prm->b_a2)
+    return fail(PF_ERR_INVALID_ARG, "a decode parameter is NULL");
+  if (!x || !y || !cache_ok(cache) || !aligned16(x) || !aligned16(y) || !aligned16(ws) ||
+      !aligned16(prm->W_qkv) || !aligned16(prm->W_o) || !aligned16(prm->rms_w) ||
+      !aligned16(prm->W_a1) || !aligned16(prm->b_a1) || !aligned16(prm->W_a2) ||
+      !aligned16(prm->b_a2))
+    return fail(PF_ERR_INVALID_ARG, "x, y and every cache buffer are required, 16-byte aligned");
+  const size_t need = proxy_decode_workspace_size(desc);
+  if (ws == nullptr || ws_bytes < need)
+    return fail(PF_ERR_WORKSPACE, "workspace too small: need %zu bytes, got %zu", need, ws_bytes);
+  cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  DecodeLaunch L{};
+  L.B = desc->batch;
+  L.d = desc->d;
+  L.nh = desc->n_heads;
+  L.P = desc->P;
+  L.cap = desc->capacity;
+  L.splits = decode_splits(desc->batch, desc->n_heads, desc->capacity);
+  L.x = static_cast<const bf16*>(x);
+  L.y = static_cast<bf16*>(y);
+  L.W_qkv = static_cast<const bf16*>(prm->W_qkv);
+  L.W_o = static_cast<const bf16*>(prm->W_o);
+  L.W_a1 = static_cast<const bf16*>(prm->W_a1);
+  L.W_a2 = static_cast<const bf16*>(prm->W_a2);
+  L.rms_w = prm->rms_w;
+  L.b_a1 = prm->b_a1;
+  L.b_a2 = prm->b_a2;
+  L.K_proxy = static_cast<const bf16*>(cache->K_proxy);
+  L.V_proxy = static_cast<const bf16*>(cache->V_proxy);
+  L.X_open = static_cast<bf16*>(cache->X_open);
+  L.K_open = static_cast<bf16*>(cache->K_open);
+  L.V_open = static_cast<bf16*>(cache->V_open);
+  L.n_proxy = cache->n_proxy;
+  L.n_open = cache->n_open;
+  L.ws = static_cast<float*>(ws);
+  PF_CUDA(decode_step_launch(L, cs));
+  return PF_OK;
 }
 
-pf_status proxy_kv_append(const pf_decode_desc* desc, const pf_append_params* params,
+pf_status proxy_kv_append(const pf_decode_desc* desc, const pf_append_params* prm,
                           const float* H_in, pf_kv_cache* cache, void* ws, size_t ws_bytes,
                           void* stream) {
-  (void)desc; (void)params; (void)H_in; (void)cache; (void)ws; (void)ws_bytes; (void)stream;
-  return fail(PF_ERR_UNSUPPORTED, "KV append is not built yet");
+  pf_status st = check_decode_desc(desc);
+  if (st != PF_OK) return st;
+  const pf_decode_desc& s = *desc;
+  if (!prm || !prm->W_c1 || !prm->b_c1 || !prm->W_kvh ||
+      (s.levels == 2 && (!prm->W_c2 || !prm->b_c2)))
+    return fail(PF_ERR_INVALID_ARG, "an append parameter is NULL");
+  if (!cache_ok(cache) || !aligned16(H_in) || !aligned16(ws) || !aligned16(prm->W_c1) ||
+      !aligned16(prm->b_c1) || !aligned16(prm->W_c2) || !aligned16(prm->b_c2) ||
+      !aligned16(prm->W_kvh))
+    return fail(PF_ERR_INVALID_ARG, "every cache buffer is required; buffers 16-byte aligned");
+  Carve wc(ws);
+  const AppendWs w = carve_append(wc, s);
+  if (ws == nullptr || wc.off > ws_bytes)
+    return fail(PF_ERR_WORKSPACE, "workspace too small: need %zu bytes, got %zu", wc.off, ws_bytes);
+  cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  const int B = s.batch, d = s.d, P = s.P;
+  const long k1 = s.levels == 2 ? s.k1 : s.P, k2 = s.levels == 2 ? s.k2 : 1;
+  const bf16* Xo = static_cast<const bf16*>(cache->X_open);
+  // compression of the open block (Eq. compress-linear / factor-cascade),
+  // H = H_in + C (Eq. proxy-res)
+  if (s.levels == 1) {
+    EpiLinearArgs e;
+    e.bias = prm->b_c1;
+    e.addend = H_in;
+    e.ld_add = d;
+    e.out_f32 = w.Hf;
+    e.ld_f32 = d;
+    e.out_bf16 = w.Hb;
+    e.ld_bf16 = d;
+    set_gemm_tag("append_compress_c1", (double)B * d * 10.0);
+    PF_CUDA(gemm_linear(B, d, (int)(k1 * d), {Xo, k1 * d, 0},
+                        {static_cast<const bf16*>(prm->W_c1), k1 * d, 0}, e, cs));
+  } else {
+    EpiLinearArgs e;
+    e.bias = prm->b_c1;
+    e.out_bf16 = w.Y;
+    e.ld_bf16 = d;
+    set_gemm_tag("append_compress_c1", (double)B * k2 * d * 2.0);
+    PF_CUDA(gemm_linear((int)(B * k2), d, (int)(k1 * d), {Xo, k1 * d, 0},
+                        {static_cast<const bf16*>(prm->W_c1), k1 * d, 0}, e, cs));
+    EpiLinearArgs e2;
+    e2.bias = prm->b_c2;
+    e2.addend = H_in;
+    e2.ld_add = d;
+    e2.out_f32 = w.Hf;
+    e2.ld_f32 = d;
+    e2.out_bf16 = w.Hb;
+    e2.ld_bf16 = d;
+    set_gemm_tag("append_compress_c2", (double)B * d * 10.0);
+    PF_CUDA(gemm_linear(B, d, (int)(k2 * d), {w.Y, k2 * d, 0},
+                        {static_cast<const bf16*>(prm->W_c2), k2 * d, 0}, e2, cs));
+  }
+  // the proxy's key and value rows into cache row n_proxy[b]
+  {
+    EpiAppendArgs e{static_cast<bf16*>(cache->K_proxy), static_cast<bf16*>(cache->V_proxy),
+                    cache->n_open, cache->n_proxy, d, P, s.capacity};
+    set_gemm_tag("append_kv", (double)B * 2 * d * 2.0);
+    PF_CUDA(gemm_append_kv(B, 2 * d, d, {w.Hb, d, 0}, {static_cast<const bf16*>(prm->W_kvh), d, 0},
+                           e, cs));
+  }
+  PF_CUDA(append_finish(cache->n_open, cache->n_proxy, B, P, s.capacity, cs));
+  return PF_OK;
 }
 
 pf_status pf_sync_check(void* stream) {
   PF_CUDA(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
   PF_CUDA(cudaGetLastError());
   int e = 0;
-  for (int v : {take_dev_error_gemm(), take_dev_error_attention(), take_dev_error_elementwise()})
+  for (int v : {take_dev_error_gemm(), take_dev_error_attention(), take_dev_error_elementwise(),
+                take_dev_error_decode()})
     if (v != 0 && e == 0) e = v;
   if (e < 0) return fail(PF_ERR_CUDA, "reading the device error flag failed");
   if (e == DEVERR_TIMEOUT) return fail(PF_ERR_TIMEOUT, "a kernel's bounded wait ran out");

@@ -134,4 +134,11 @@ cudaError_t gemm_dx1d(int M, int N, int K, Operand A, Operand B, const EpiDXArgs
   return gemm_dispatch(M, N, K, A, B, epi, e.dXd, M, st);
 }
 
+cudaError_t gemm_append_kv(int M, int N, int K, Operand A, Operand B, const EpiAppendArgs& e,
+                           cudaStream_t st) {
+  EpiAppendKV epi{M, N, e.K, e.V, e.n_open, e.n_proxy, e.d, e.P, e.cap};
+  if (A.mn || B.mn) return cudaErrorInvalidValue;
+  return gemm_dispatch(M, N, K, A, B, epi, nullptr, 0, st);
+}
+
 }  // namespace pf

@@ -436,4 +436,36 @@ struct EpiDX1D {
   }
 };
 
+// KV append (Sec. 3.8): rows are sequences b, columns [0, 2d) the proxy's key
+// and value rows W_kh H and W_vh H, written as bf16 at cache row n_proxy[b] of
+// the sequences whose open block is full and whose cache has room.
+struct EpiAppendKV {
+  static constexpr bool kXTile = false;
+  struct Row {
+    bool ok;
+    long off;
+  };
+  int M, N;
+  bf16 *K, *V;
+  const int *n_open, *n_proxy;
+  int d, P, cap;
+  __device__ __forceinline__ int x_row(int m0) const { return m0; }
+  __device__ __forceinline__ Row row_info(int row) const {
+    Row r{false, 0};
+    if (row < M) {
+      const int np = n_proxy[row];
+      r.ok = n_open[row] == P && np >= 0 && np < cap;
+      r.off = ((long)row * cap + (r.ok ? np : 0)) * d;
+    }
+    return r;
+  }
+  __device__ __forceinline__ void apply(const Row& ri, int, int col, float* v, const uint8_t*, int,
+                                        int) const {
+    if (!ri.ok || col >= N) return;
+    bf16* o = col < d ? K + ri.off + col : V + ri.off + (col - d);
+#pragma unroll
+    for (int i = 0; i < 32; i += 8) store8_bf16(o + i, v + i);
+  }
+};
+
 }  // namespace pf

@@ -46,12 +46,42 @@ cudaError_t gemm_inject1d(int M, int N, int K, Operand A, Operand B, const EpiIn
                           cudaStream_t st);
 cudaError_t gemm_dx1d(int M, int N, int K, Operand A, Operand B, const EpiDXArgs& e,
                       cudaStream_t st);
+
+// KV append: rows b = sequences, columns [0, d) -> K_proxy[b, n_proxy[b]],
+// [d, 2d) -> V_proxy[b, n_proxy[b]] (bf16), only for sequences whose open
+// block is full (n_open[b] == P) and whose cache has room.
+struct EpiAppendArgs {
+  bf16 *K, *V;
+  const int *n_open, *n_proxy;
+  int d, P, cap;
+};
+cudaError_t gemm_append_kv(int M, int N, int K, Operand A, Operand B, const EpiAppendArgs& e,
+                           cudaStream_t st);
 int num_sms();
 
 // Per-file device error flags (see common.cuh): value, cleared on read.
 int take_dev_error_gemm();
+int take_dev_error_decode();
 int take_dev_error_attention();
 int take_dev_error_elementwise();
+
+// ---------------------------------------------------------------- decode
+#define PF_DECODE_MAX_P 256
+struct DecodeLaunch {
+  int B, d, nh, P, cap, splits;
+  const bf16* x;
+  bf16* y;
+  const bf16 *W_qkv, *W_o, *W_a1, *W_a2;
+  const float *rms_w, *b_a1, *b_a2;
+  const bf16 *K_proxy, *V_proxy;
+  bf16 *X_open, *K_open, *V_open;
+  int *n_proxy, *n_open;
+  float* ws;
+};
+size_t decode_workspace_bytes(int B, int d, int nh, int splits);
+int decode_splits(int B, int nh, int cap);
+cudaError_t decode_step_launch(const DecodeLaunch& L, cudaStream_t st);
+cudaError_t append_finish(int* n_open, int* n_proxy, int B, int P, int cap, cudaStream_t st);
 
 // ------------------------------------------------------------- attention
 cudaError_t attn_fwd(const bf16* qkv, bf16* out, float* lse, int B, int m, int d, int nh,

@@ -101,10 +101,11 @@ def default_factors(P: int):
 
 def round_bf16(a: np.ndarray) -> np.ndarray:
     """Round float32 values to the nearest bfloat16, ties to even (no NaN input)."""
-    a = np.ascontiguousarray(a, dtype=np.float32)
-    u = a.view(np.uint32).astype(np.uint64)
-    u = (u + 0x7FFF + ((u >> 16) & 1)) & 0xFFFF0000
-    return u.astype(np.uint32).view(np.float32)
+    a = np.array(a, dtype=np.float32, copy=True)
+    u = a.view(np.uint32)  # finite inputs: the sum below cannot wrap
+    u += np.uint32(0x7FFF) + ((u >> np.uint32(16)) & np.uint32(1))
+    u &= np.uint32(0xFFFF0000)
+    return a
 
 
 def _finish(a: np.ndarray, dtype: int) -> np.ndarray:
