@@ -119,6 +119,24 @@ BwdWs carve_bwd(Carve& c, const pf_layer_desc& s, const Dims& g) {
   return w;
 }
 
+// Workspace of the fp32 forward (all fp32).
+struct F32Ws {
+  float *Xpad, *Y, *H, *QKV, *A, *Hbar, *Z, *D;
+};
+
+F32Ws carve_f32(Carve& c, const pf_layer_desc& s, const Dims& g) {
+  F32Ws w{};
+  w.Xpad = g.ragged ? c.take<float>(g.B * g.Lp * g.d) : nullptr;
+  if (s.levels == 2) w.Y = c.take<float>(g.rows1 * g.d);
+  w.H = c.take<float>(g.R * g.d);
+  w.QKV = c.take<float>(g.R * 3 * g.d);
+  w.A = c.take<float>(g.R * g.d);
+  w.Hbar = c.take<float>(g.R * g.d);
+  if (s.levels == 2) w.Z = c.take<float>(g.R * g.k2 * g.d);
+  w.D = c.take<float>(g.rows1 * g.N1);
+  return w;
+}
+
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
 bool params_aligned(const pf_layer_params& p) {
@@ -151,11 +169,57 @@ pf_status check_desc(const pf_layer_desc* s) {
     return fail(PF_ERR_UNSUPPORTED, "the 2D layer is not built yet");
   }
   if (s->inject == PF_INJ_AFFINE) return fail(PF_ERR_UNSUPPORTED, "affine injection is 2D only");
-  if (s->dtype == PF_F32) return fail(PF_ERR_UNSUPPORTED, "fp32 layer is not built yet");
+
   const long m = (s->L + (long)s->P - 1) / s->P;
   const long k1 = s->levels == 2 ? s->k1 : s->P, k2 = s->levels == 2 ? s->k2 : 1;
   if ((long)s->batch * m * k2 > (1L << 30) || k1 * s->d > (1L << 30))
     return fail(PF_ERR_UNSUPPORTED, "problem too large for 32-bit GEMM extents");
+  return PF_OK;
+}
+
+// fp32 forward (Alg. 1) on CUDA cores; same steps as the bf16 path.
+pf_status layer_fwd_f32(const pf_layer_desc& s, const Dims& g, const pf_layer_params& p,
+                        const void* Xv, const float* H_in, void* X_out, float* H_out, void* ws,
+                        size_t ws_bytes, cudaStream_t cs) {
+  Carve wc(ws);
+  const F32Ws w = carve_f32(wc, s, g);
+  if (ws == nullptr || wc.off > ws_bytes)
+    return fail(PF_ERR_WORKSPACE, "workspace too small: need %zu bytes, got %zu", wc.off, ws_bytes);
+  const float* X = static_cast<const float*>(Xv);
+  const int d = (int)g.d, N1 = (int)g.N1;
+  const float* Xsrc = X;
+  if (g.ragged) {
+    PF_CUDA(pad_f32(X, w.Xpad, (int)g.B, g.L, g.Lp, d, cs));
+    Xsrc = w.Xpad;
+  }
+  const float* W_c1 = static_cast<const float*>(p.W_c1);
+  float* H = H_out ? H_out : w.H;
+  if (s.levels == 1) {
+    PF_CUDA(gemm_f32((int)g.R, d, N1, Xsrc, N1, W_c1, N1, H, d, p.b_c1, H_in, d, "compress_c1", cs));
+  } else {
+    PF_CUDA(gemm_f32((int)g.rows1, d, N1, Xsrc, N1, W_c1, N1, w.Y, d, p.b_c1, nullptr, 0,
+                     "compress_c1", cs));
+    const int n2 = (int)(g.k2 * d);
+    PF_CUDA(gemm_f32((int)g.R, d, n2, w.Y, n2, static_cast<const float*>(p.W_c2), n2, H, d, p.b_c2,
+                     H_in, d, "compress_c2", cs));
+  }
+  PF_CUDA(gemm_f32((int)g.R, 3 * d, d, H, d, static_cast<const float*>(p.W_qkv), d, w.QKV, 3 * d,
+                   nullptr, nullptr, 0, "proxy_qkv", cs));
+  PF_CUDA(attn_f32(w.QKV, w.A, (int)g.B, (int)g.m, d, (int)g.nh, g.causal, cs));
+  PF_CUDA(gemm_f32((int)g.R, d, d, w.A, d, static_cast<const float*>(p.W_o), d, w.Hbar, d, nullptr,
+                   nullptr, 0, "proxy_o", cs));
+  const float* Zsrc = w.Hbar;
+  if (s.levels == 2) {
+    const int n2 = (int)(g.k2 * d);
+    PF_CUDA(gemm_f32((int)g.R, n2, d, w.Hbar, d, static_cast<const float*>(p.W_d2), d, w.Z, n2,
+                     p.b_d2, nullptr, 0, "decompress_d2", cs));
+    Zsrc = w.Z;
+  }
+  PF_CUDA(gemm_f32((int)g.rows1, N1, d, Zsrc, d, static_cast<const float*>(p.W_d1), d, w.D, N1,
+                   p.b_d1, nullptr, 0, "decompress_d1", cs));
+  PF_CUDA(inject_f32(X, w.D, static_cast<float*>(X_out), p.w_x, p.w_dlt, p.b_g, (int)g.B, g.L, d,
+                     (int)g.P, (int)g.k1, (int)g.k2, (int)g.m, g.causal ? 1 : 0,
+                     s.inject == PF_INJ_GATED ? 1 : 0, cs));
   return PF_OK;
 }
 
@@ -176,6 +240,7 @@ pf_status proxy_layer_check(const pf_layer_desc* desc) { return check_desc(desc)
 
 size_t proxy_layer_saved_size(const pf_layer_desc* desc) {
   if (check_desc(desc) != PF_OK) return 0;
+  if (desc->dtype == PF_F32) return 0;  // the fp32 layer is forward-only
   const Dims g = dims_of(*desc);
   Carve c(nullptr);
   carve_saved(c, *desc, g);
@@ -186,7 +251,10 @@ size_t proxy_layer_workspace_size(const pf_layer_desc* desc, int for_backward) {
   if (check_desc(desc) != PF_OK) return 0;
   const Dims g = dims_of(*desc);
   Carve c(nullptr);
-  if (for_backward) {
+  if (desc->dtype == PF_F32) {
+    if (for_backward) return 0;
+    carve_f32(c, *desc, g);
+  } else if (for_backward) {
     carve_bwd(c, *desc, g);
   } else {
     if (g.ragged) c.take<bf16>(g.B * g.Lp * g.d);
@@ -212,6 +280,8 @@ pf_status proxy_layer_fwd(const pf_layer_desc* desc, const pf_layer_params* prm,
   if (!aligned16(X) || !aligned16(X_out) || !aligned16(saved) || !aligned16(ws) ||
       !aligned16(H_in) || !aligned16(H_out) || !params_aligned(*prm))
     return fail(PF_ERR_INVALID_ARG, "buffers must be 16-byte aligned");
+  if (s.dtype == PF_F32) return layer_fwd_f32(s, g, *prm, X, H_in, X_out, H_out, ws, ws_bytes,
+                                             static_cast<cudaStream_t>(stream));
   Carve wc(ws);
   bf16* Xpad = g.ragged ? wc.take<bf16>(g.B * g.Lp * g.d) : nullptr;
   Carve sc(saved);
@@ -321,6 +391,7 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
   if (!aligned16(X) || !aligned16(saved) || !aligned16(dX_out) || !aligned16(dX) ||
       !aligned16(ws) || !aligned16(dH_out) || !aligned16(dH_in) || !params_aligned(*prm))
     return fail(PF_ERR_INVALID_ARG, "buffers must be 16-byte aligned");
+  if (s.dtype == PF_F32) return fail(PF_ERR_UNSUPPORTED, "the fp32 layer is forward-only");
   const bool gated = s.inject == PF_INJ_GATED;
   if (!grads->b_d1 || (gated && (!grads->w_x || !grads->w_dlt || !grads->b_g)))
     return fail(PF_ERR_INVALID_ARG, "grads->b_d1 (and the gate gradients) must be given");
@@ -646,7 +717,7 @@ pf_status pf_sync_check(void* stream) {
   PF_CUDA(cudaGetLastError());
   int e = 0;
   for (int v : {take_dev_error_gemm(), take_dev_error_attention(), take_dev_error_elementwise(),
-                take_dev_error_decode()})
+                take_dev_error_decode(), take_dev_error_fp32()})
     if (v != 0 && e == 0) e = v;
   if (e < 0) return fail(PF_ERR_CUDA, "reading the device error flag failed");
   if (e == DEVERR_TIMEOUT) return fail(PF_ERR_TIMEOUT, "a kernel's bounded wait ran out");

@@ -65,6 +65,18 @@ int take_dev_error_decode();
 int take_dev_error_attention();
 int take_dev_error_elementwise();
 
+// ---------------------------------------------------------- fp32 forward
+int take_dev_error_fp32();
+cudaError_t gemm_f32(int M, int N, int K, const float* A, long lda, const float* B, long ldb,
+                     float* C, long ldc, const float* bias, const float* addend, long ld_add,
+                     const char* label, cudaStream_t st);
+cudaError_t attn_f32(const float* qkv, float* out, int B, int m, int d, int nh, bool causal,
+                     cudaStream_t st);
+cudaError_t inject_f32(const float* X, const float* D, float* Xo, const float* w_x,
+                       const float* w_dlt, const float* b_g, int B, long L, int d, int P, int k1,
+                       int k2, int m, int shift, int gated, cudaStream_t st);
+cudaError_t pad_f32(const float* src, float* dst, int B, long L, long Lp, int d, cudaStream_t st);
+
 // ---------------------------------------------------------------- decode
 #define PF_DECODE_MAX_P 256
 struct DecodeLaunch {
