@@ -119,6 +119,57 @@ BwdWs carve_bwd(Carve& c, const pf_layer_desc& s, const Dims& g) {
   return w;
 }
 
+// Saved buffer of the 2D layer (order fixes the layout).
+struct Saved2D {
+  bf16 *Xp, *S, *Hb, *QKV, *Aatt, *Hbar;
+  float *stats, *nH, *rstdH, *LSE, *e, *a1, *u, *gb;
+};
+
+Saved2D carve_saved_2d(Carve& c, const Dims& g) {
+  Saved2D v{};
+  const long T = g.B * g.L;
+  v.Xp = c.take<bf16>(g.R * g.N1);
+  v.stats = c.take<float>(2 * T);
+  v.S = c.take<bf16>(g.R * g.N1);
+  v.nH = c.take<float>(g.R * g.d);
+  v.rstdH = c.take<float>(g.R);
+  v.Hb = c.take<bf16>(g.R * g.d);
+  v.QKV = c.take<bf16>(g.R * 3 * g.d);
+  v.Aatt = c.take<bf16>(g.R * g.d);
+  v.Hbar = c.take<bf16>(g.R * g.d);
+  v.LSE = c.take<float>(g.B * g.nh * g.m);
+  v.e = c.take<float>(g.B * 256);
+  v.a1 = c.take<float>(g.B * g.d);
+  v.u = c.take<float>(g.B * g.d);
+  v.gb = c.take<float>(g.B * 2 * g.d);
+  return v;
+}
+
+struct Bwd2DWs {
+  bf16 *dD, *dXd, *dHbar, *dA, *dQKV, *dHb;
+  float *Di, *dHq, *dHf, *part, *dgb, *da1;
+};
+
+Bwd2DWs carve_bwd_2d(Carve& c, const Dims& g) {
+  Bwd2DWs w{};
+  w.dD = c.take<bf16>(g.R * 2 * g.N1);
+  w.dXd = c.take<bf16>(g.R * g.N1);
+  w.dHbar = c.take<bf16>(g.R * g.d);
+  w.dA = c.take<bf16>(g.R * g.d);
+  w.dQKV = c.take<bf16>(g.R * 3 * g.d);
+  w.dHb = c.take<bf16>(g.R * g.d);
+  w.Di = c.take<float>(g.B * g.nh * g.m);
+  w.dHq = c.take<float>(g.R * g.d);
+  w.dHf = c.take<float>(g.R * g.d);
+  long pe = colsum_part_elems(g.R, (int)(2 * g.N1));
+  pe = std::max(pe, colsum_part_elems(g.R, (int)g.d));
+  pe = std::max(pe, (long)g.B * adaln_param_chunks((int)g.m) * 2 * g.d);
+  w.part = c.take<float>(pe);
+  w.dgb = c.take<float>(g.B * 2 * g.d);
+  w.da1 = c.take<float>(g.B * g.d);
+  return w;
+}
+
 // Workspace of the fp32 forward (all fp32).
 struct F32Ws {
   float *Xpad, *Y, *H, *QKV, *A, *Hbar, *Z, *D;
@@ -166,7 +217,10 @@ pf_status check_desc(const pf_layer_desc* s) {
     if (s->patch < 1 || s->patch * s->patch != s->P || s->grid_h < 1 || s->grid_w < 1 ||
         (long)s->grid_h * s->grid_w != s->L || s->grid_h % s->patch || s->grid_w % s->patch)
       return fail(PF_ERR_INVALID_ARG, "2D layer needs L = grid_h*grid_w, P = patch^2, patch | grid");
-    return fail(PF_ERR_UNSUPPORTED, "the 2D layer is not built yet");
+    if (s->inject != PF_INJ_AFFINE || s->levels != 1 || s->dtype != PF_BF16 || s->d % 128 != 0)
+      return fail(PF_ERR_UNSUPPORTED,
+                  "the 2D layer is built for affine injection, one level, bf16, d % 128 == 0");
+    return PF_OK;
   }
   if (s->inject == PF_INJ_AFFINE) return fail(PF_ERR_UNSUPPORTED, "affine injection is 2D only");
 
@@ -223,6 +277,156 @@ pf_status layer_fwd_f32(const pf_layer_desc& s, const Dims& g, const pf_layer_pa
   return PF_OK;
 }
 
+// 2D bidirectional layer (Sec. 3.9): patch compression, timestep adaLN on
+// the proxies, bidirectional proxy attention, decompression with affine
+// injection (Eq. inj-affine).
+pf_status layer_fwd_2d(const pf_layer_desc& s, const Dims& g, const pf_layer_params& p,
+                       const void* Xv, const float* H_in, const float* t, void* X_out,
+                       float* H_out, void* saved, void* ws, size_t ws_bytes, cudaStream_t cs) {
+  if (!t) return fail(PF_ERR_INVALID_ARG, "the 2D layer needs t");
+  if (!p.W_c1 || !p.b_c1 || !p.W_qkv || !p.W_o || !p.W_d1 || !p.b_d1 || !p.W_t1 || !p.b_t1 ||
+      !p.W_t2 || !p.b_t2)
+    return fail(PF_ERR_INVALID_ARG, "a parameter of the 2D layer is NULL");
+  Carve wc(ws);
+  float* Hws = wc.take<float>(g.R * g.d);
+  Carve sc(saved);
+  const Saved2D sv = saved ? carve_saved_2d(sc, g) : carve_saved_2d(wc, g);
+  if (ws == nullptr || wc.off > ws_bytes)
+    return fail(PF_ERR_WORKSPACE, "workspace too small: need %zu bytes, got %zu", wc.off, ws_bytes);
+  const bf16* X = static_cast<const bf16*>(Xv);
+  const int d = (int)g.d, N1 = (int)g.N1;
+  const int patch = s.patch, gh = s.grid_h, gw = s.grid_w;
+  float* Hf = H_out ? H_out : Hws;
+  PF_CUDA(patch_gather(X, sv.Xp, (int)g.B, d, patch, gh, gw, cs));
+  PF_CUDA(ln_stats(X, sv.stats, g.B * g.L, d, cs));
+  {
+    EpiLinearArgs e;
+    e.bias = p.b_c1;
+    e.addend = H_in;
+    e.ld_add = d;
+    e.out_f32 = Hf;
+    e.ld_f32 = d;
+    set_gemm_tag("compress_c1", (double)g.R * d * 8.0);
+    PF_CUDA(gemm_linear((int)g.R, d, N1, {sv.Xp, N1, 0}, {static_cast<const bf16*>(p.W_c1), N1, 0},
+                        e, cs));
+  }
+  PF_CUDA(temb_fwd(t, (int)g.B, d, static_cast<const bf16*>(p.W_t1), p.b_t1,
+                   static_cast<const bf16*>(p.W_t2), p.b_t2, sv.e, sv.a1, sv.u, sv.gb, cs));
+  PF_CUDA(adaln_fwd(Hf, sv.gb, sv.nH, sv.rstdH, sv.Hb, g.R, d, (int)g.m, cs));
+  {
+    EpiLinearArgs e;
+    e.out_bf16 = sv.QKV;
+    e.ld_bf16 = 3 * d;
+    set_gemm_tag("proxy_qkv", (double)g.R * 3 * d * 2.0);
+    PF_CUDA(gemm_linear((int)g.R, 3 * d, d, {sv.Hb, d, 0},
+                        {static_cast<const bf16*>(p.W_qkv), d, 0}, e, cs));
+    PF_CUDA(attn_fwd(sv.QKV, sv.Aatt, sv.LSE, (int)g.B, (int)g.m, d, (int)g.nh, false, cs));
+    EpiLinearArgs eo;
+    eo.out_bf16 = sv.Hbar;
+    eo.ld_bf16 = d;
+    set_gemm_tag("proxy_o", (double)g.R * d * 2.0);
+    PF_CUDA(gemm_linear((int)g.R, d, d, {sv.Aatt, d, 0}, {static_cast<const bf16*>(p.W_o), d, 0},
+                        eo, cs));
+  }
+  {
+    EpiAffine2DArgs e{p.b_d1, sv.S, static_cast<bf16*>(X_out), sv.stats, sv.Xp, d, patch, gh, gw,
+                      (int)g.m};
+    set_gemm_tag("decompress_affine", (double)g.R * N1 * 8.0);
+    PF_CUDA(gemm_affine2d((int)g.R, 2 * N1, d, {sv.Hbar, d, 0},
+                          {static_cast<const bf16*>(p.W_d1), d, 0}, e, cs));
+  }
+  return PF_OK;
+}
+
+pf_status layer_bwd_2d(const pf_layer_desc& s, const Dims& g, const pf_layer_params& p,
+                       const void* Xv, const void* saved, const void* dX_out, const float* dH_out,
+                       void* dXv, float* dH_in, const pf_layer_grads& gr, void* ws,
+                       size_t ws_bytes, cudaStream_t cs) {
+  Carve wc(ws);
+  const Bwd2DWs w = carve_bwd_2d(wc, g);
+  if (ws == nullptr || wc.off > ws_bytes)
+    return fail(PF_ERR_WORKSPACE, "workspace too small: need %zu bytes, got %zu", wc.off, ws_bytes);
+  Carve sc(const_cast<void*>(saved));
+  const Saved2D sv = carve_saved_2d(sc, g);
+  const bf16* X = static_cast<const bf16*>(Xv);
+  const bf16* G = static_cast<const bf16*>(dX_out);
+  bf16* dX = static_cast<bf16*>(dXv);
+  const int d = (int)g.d, N1 = (int)g.N1, N2 = 2 * N1;
+  const int patch = s.patch, gh = s.grid_h, gw = s.grid_w;
+  const bf16* W_qkv = static_cast<const bf16*>(p.W_qkv);
+  const bf16* W_o = static_cast<const bf16*>(p.W_o);
+  const bf16* W_d1 = static_cast<const bf16*>(p.W_d1);
+  const bf16* W_c1 = static_cast<const bf16*>(p.W_c1);
+  // affine injection backward (Eq. inj-affine)
+  PF_CUDA(inj_bwd_2d(G, X, sv.stats, sv.S, w.dD, w.dXd, g.B * g.L, d, patch, gh, gw, cs));
+  if (gr.b_d1) PF_CUDA(colsum_bf16(w.dD, g.R, N2, gr.b_d1, w.part, cs));
+  if (gr.W_d1) {
+    EpiLinearArgs e;
+    e.out_f32 = gr.W_d1;
+    e.ld_f32 = d;
+    set_gemm_tag("bwd_dW_d1", (double)N2 * d * 4.0);
+    PF_CUDA(gemm_linear(N2, d, (int)g.R, {w.dD, N2, 1}, {sv.Hbar, d, 1}, e, cs));
+  }
+  {
+    EpiLinearArgs e;
+    e.out_bf16 = w.dHbar;
+    e.ld_bf16 = d;
+    set_gemm_tag("bwd_dHbar", (double)g.R * d * 2.0);
+    PF_CUDA(gemm_linear((int)g.R, d, N2, {w.dD, N2, 0}, {W_d1, d, 1}, e, cs));
+  }
+  if (gr.W_o) {
+    EpiLinearArgs e;
+    e.out_f32 = gr.W_o;
+    e.ld_f32 = d;
+    set_gemm_tag("bwd_dW_o", (double)d * d * 4.0);
+    PF_CUDA(gemm_linear(d, d, (int)g.R, {w.dHbar, d, 1}, {sv.Aatt, d, 1}, e, cs));
+  }
+  {
+    EpiLinearArgs e;
+    e.out_bf16 = w.dA;
+    e.ld_bf16 = d;
+    set_gemm_tag("bwd_dA", (double)g.R * d * 2.0);
+    PF_CUDA(gemm_linear((int)g.R, d, d, {w.dHbar, d, 0}, {W_o, d, 1}, e, cs));
+  }
+  PF_CUDA(attn_bwd(sv.QKV, sv.Aatt, w.dA, sv.LSE, w.Di, w.dQKV, (int)g.B, (int)g.m, d, (int)g.nh,
+                   false, cs));
+  if (gr.W_qkv) {
+    EpiLinearArgs e;
+    e.out_f32 = gr.W_qkv;
+    e.ld_f32 = d;
+    set_gemm_tag("bwd_dW_qkv", (double)3 * d * d * 4.0);
+    PF_CUDA(gemm_linear(3 * d, d, (int)g.R, {w.dQKV, 3 * d, 1}, {sv.Hb, d, 1}, e, cs));
+  }
+  {
+    EpiLinearArgs e;
+    e.out_f32 = w.dHq;
+    e.ld_f32 = d;
+    set_gemm_tag("bwd_dHq", (double)g.R * d * 4.0);
+    PF_CUDA(gemm_linear((int)g.R, d, 3 * d, {w.dQKV, 3 * d, 0}, {W_qkv, d, 1}, e, cs));
+  }
+  // adaLN and timestep-MLP backward
+  float* dHf = dH_in ? dH_in : w.dHf;
+  PF_CUDA(adaln_bwd(w.dHq, sv.nH, sv.rstdH, sv.gb, dH_out, dHf, w.dHb, g.R, d, (int)g.m, cs));
+  PF_CUDA(adaln_param_grads(w.dHq, sv.nH, w.part, w.dgb, (int)g.B, d, (int)g.m, cs));
+  PF_CUDA(temb_bwd(w.dgb, static_cast<const bf16*>(p.W_t2), sv.a1, sv.u, sv.e, w.da1,
+                   TembGrads{gr.W_t2, gr.b_t2, gr.W_t1, gr.b_t1}, (int)g.B, d, cs));
+  // compression backward (H = H_in + C, so dC = dH)
+  if (gr.b_c1) PF_CUDA(colsum_f32(dHf, g.R, d, gr.b_c1, w.part, cs));
+  if (gr.W_c1) {
+    EpiLinearArgs e;
+    e.out_f32 = gr.W_c1;
+    e.ld_f32 = N1;
+    set_gemm_tag("bwd_dW_c1", (double)d * N1 * 4.0);
+    PF_CUDA(gemm_linear(d, N1, (int)g.R, {w.dHb, d, 1}, {sv.Xp, N1, 1}, e, cs));
+  }
+  {
+    EpiDX2DArgs e{w.dXd, dX, d, patch, gh, gw, (int)g.m};
+    set_gemm_tag("bwd_dX", (double)g.R * N1 * 4.0);
+    PF_CUDA(gemm_dx2d((int)g.R, N1, d, {w.dHb, d, 0}, {W_c1, N1, 1}, e, cs));
+  }
+  return PF_OK;
+}
+
 }  // namespace
 
 // Sets the thread-local message returned by pf_last_error (for other files of
@@ -243,7 +447,10 @@ size_t proxy_layer_saved_size(const pf_layer_desc* desc) {
   if (desc->dtype == PF_F32) return 0;  // the fp32 layer is forward-only
   const Dims g = dims_of(*desc);
   Carve c(nullptr);
-  carve_saved(c, *desc, g);
+  if (desc->mode == PF_BIDIR_2D)
+    carve_saved_2d(c, g);
+  else
+    carve_saved(c, *desc, g);
   return (c.off + 255) & ~size_t(255);
 }
 
@@ -254,6 +461,13 @@ size_t proxy_layer_workspace_size(const pf_layer_desc* desc, int for_backward) {
   if (desc->dtype == PF_F32) {
     if (for_backward) return 0;
     carve_f32(c, *desc, g);
+  } else if (desc->mode == PF_BIDIR_2D) {
+    if (for_backward) {
+      carve_bwd_2d(c, g);
+    } else {
+      c.take<float>(g.R * g.d);  // H when H_out is NULL
+      carve_saved_2d(c, g);
+    }
   } else if (for_backward) {
     carve_bwd(c, *desc, g);
   } else {
@@ -282,6 +496,9 @@ pf_status proxy_layer_fwd(const pf_layer_desc* desc, const pf_layer_params* prm,
     return fail(PF_ERR_INVALID_ARG, "buffers must be 16-byte aligned");
   if (s.dtype == PF_F32) return layer_fwd_f32(s, g, *prm, X, H_in, X_out, H_out, ws, ws_bytes,
                                              static_cast<cudaStream_t>(stream));
+  if (s.mode == PF_BIDIR_2D)
+    return layer_fwd_2d(s, g, *prm, X, H_in, t, X_out, H_out, saved, ws, ws_bytes,
+                        static_cast<cudaStream_t>(stream));
   Carve wc(ws);
   bf16* Xpad = g.ragged ? wc.take<bf16>(g.B * g.Lp * g.d) : nullptr;
   Carve sc(saved);
@@ -392,6 +609,9 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
       !aligned16(ws) || !aligned16(dH_out) || !aligned16(dH_in) || !params_aligned(*prm))
     return fail(PF_ERR_INVALID_ARG, "buffers must be 16-byte aligned");
   if (s.dtype == PF_F32) return fail(PF_ERR_UNSUPPORTED, "the fp32 layer is forward-only");
+  if (s.mode == PF_BIDIR_2D)
+    return layer_bwd_2d(s, g, *prm, X, saved, dX_out, dH_out, dX, dH_in, *grads, ws, ws_bytes,
+                        static_cast<cudaStream_t>(stream));
   const bool gated = s.inject == PF_INJ_GATED;
   if (!grads->b_d1 || (gated && (!grads->w_x || !grads->w_dlt || !grads->b_g)))
     return fail(PF_ERR_INVALID_ARG, "grads->b_d1 (and the gate gradients) must be given");
@@ -717,7 +937,7 @@ pf_status pf_sync_check(void* stream) {
   PF_CUDA(cudaGetLastError());
   int e = 0;
   for (int v : {take_dev_error_gemm(), take_dev_error_attention(), take_dev_error_elementwise(),
-                take_dev_error_decode(), take_dev_error_fp32()})
+                take_dev_error_decode(), take_dev_error_fp32(), take_dev_error_layer2d()})
     if (v != 0 && e == 0) e = v;
   if (e < 0) return fail(PF_ERR_CUDA, "reading the device error flag failed");
   if (e == DEVERR_TIMEOUT) return fail(PF_ERR_TIMEOUT, "a kernel's bounded wait ran out");

@@ -62,7 +62,8 @@ template <int BN, bool AMN, bool BMN, class Epi>
 cudaError_t launch(int M, int N, int K, const CUtensorMap& ta, const CUtensorMap& tb,
                    const CUtensorMap& tx, const Epi& epi, cudaStream_t st) {
   auto kern = gemm_tc_kernel<BN, AMN, BMN, Epi>;
-  constexpr int smem = GemmCfg<BN, Epi::kXTile>::SMEM_BYTES;
+  constexpr int XCOLS = Epi::kXTile ? (Epi::kPaired ? BN / 2 : BN) : 0;
+  constexpr int smem = GemmCfg<BN, XCOLS>::SMEM_BYTES;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const long tiles = (long)((N + BN - 1) / BN) * ((M + GEMM_BM - 1) / GEMM_BM);
@@ -90,7 +91,8 @@ bool operand_ok(const Operand& op) {
 // prefetches by TMA; for other epilogues `xsrc` is ignored.
 template <class Epi>
 cudaError_t gemm_dispatch(int M, int N, int K, Operand A, Operand B, const Epi& epi,
-                          const bf16* xsrc, long x_rows, cudaStream_t st) {
+                          const bf16* xsrc, long x_rows, cudaStream_t st, long x_cols = -1) {
+  if (x_cols < 0) x_cols = N;
   if (M <= 0 || N <= 0 || N % 32 != 0 || K < 0 || !operand_ok(A) || !operand_ok(B))
     return cudaErrorInvalidValue;
   CUtensorMap ta, tb, tx;
@@ -98,7 +100,7 @@ cudaError_t gemm_dispatch(int M, int N, int K, Operand A, Operand B, const Epi& 
     return cudaErrorInvalidValue;
   if (Epi::kXTile) {
     if (xsrc == nullptr || (reinterpret_cast<uintptr_t>(xsrc) & 15) != 0 ||
-        !make_map(&tx, xsrc, (uint64_t)N, (uint64_t)x_rows, (uint64_t)N, 64, 128))
+        !make_map(&tx, xsrc, (uint64_t)x_cols, (uint64_t)x_rows, (uint64_t)x_cols, 64, 128))
       return cudaErrorInvalidValue;
   } else {
     tx = ta;
@@ -106,7 +108,7 @@ cudaError_t gemm_dispatch(int M, int N, int K, Operand A, Operand B, const Epi& 
   const long tiles256 = (long)((N + 255) / 256) * ((M + GEMM_BM - 1) / GEMM_BM);
   LaunchTimer lt(gemm_tag_label(), st, 2.0 * M * N * (double)K,
                  2.0 * ((double)M * K + (double)N * K) + gemm_tag_bytes());
-  if (N >= 256 && tiles256 >= num_sms())
+  if (Epi::kPaired || (N >= 256 && tiles256 >= num_sms()))
     return launch_majors<256>(M, N, K, A, B, ta, tb, tx, epi, st);
   return launch_majors<128>(M, N, K, A, B, ta, tb, tx, epi, st);
 }
@@ -115,13 +117,13 @@ cudaError_t gemm_dispatch(int M, int N, int K, Operand A, Operand B, const Epi& 
 
 cudaError_t gemm_linear(int M, int N, int K, Operand A, Operand B, const EpiLinearArgs& e,
                         cudaStream_t st) {
-  EpiLinear epi{M, N, e.bias, e.addend, e.ld_add, e.out_f32, e.ld_f32, e.out_bf16, e.ld_bf16};
+  EpiLinear epi{{}, M, N, e.bias, e.addend, e.ld_add, e.out_f32, e.ld_f32, e.out_bf16, e.ld_bf16};
   return gemm_dispatch(M, N, K, A, B, epi, nullptr, 0, st);
 }
 
 cudaError_t gemm_inject1d(int M, int N, int K, Operand A, Operand B, const EpiInjectArgs& e,
                           cudaStream_t st) {
-  EpiInject1D epi{M, N, e.bias, e.D_save, e.X_out, e.w_x, e.w_dlt, e.b_g,
+  EpiInject1D epi{{}, M, N, e.bias, e.D_save, e.X_out, e.w_x, e.w_dlt, e.b_g,
                   e.d, e.k1, e.k2, e.m, e.L, e.shift, e.gated};
   if (A.mn || B.mn) return cudaErrorInvalidValue;
   return gemm_dispatch(M, N, K, A, B, epi, e.Xsrc, M, st);
@@ -129,16 +131,30 @@ cudaError_t gemm_inject1d(int M, int N, int K, Operand A, Operand B, const EpiIn
 
 cudaError_t gemm_dx1d(int M, int N, int K, Operand A, Operand B, const EpiDXArgs& e,
                       cudaStream_t st) {
-  EpiDX1D epi{M, N, e.dX, e.d, e.k1, e.k2, e.m, e.L};
+  EpiDX1D epi{{}, M, N, e.dX, e.d, e.k1, e.k2, e.m, e.L};
   if (A.mn || !B.mn) return cudaErrorInvalidValue;
   return gemm_dispatch(M, N, K, A, B, epi, e.dXd, M, st);
 }
 
 cudaError_t gemm_append_kv(int M, int N, int K, Operand A, Operand B, const EpiAppendArgs& e,
                            cudaStream_t st) {
-  EpiAppendKV epi{M, N, e.K, e.V, e.n_open, e.n_proxy, e.d, e.P, e.cap};
+  EpiAppendKV epi{{}, M, N, e.K, e.V, e.n_open, e.n_proxy, e.d, e.P, e.cap};
   if (A.mn || B.mn) return cudaErrorInvalidValue;
   return gemm_dispatch(M, N, K, A, B, epi, nullptr, 0, st);
+}
+
+cudaError_t gemm_affine2d(int M, int N, int K, Operand A, Operand B, const EpiAffine2DArgs& e,
+                          cudaStream_t st) {
+  EpiAffine2D epi{{}, M, e.bias, e.S_save, e.X_out, e.stats, e.d, e.patch, e.gh, e.gw, e.m};
+  if (A.mn || B.mn || e.d % 128 != 0) return cudaErrorInvalidValue;
+  return gemm_dispatch(M, N, K, A, B, epi, e.Xp, M, st, (long)e.patch * e.patch * e.d);
+}
+
+cudaError_t gemm_dx2d(int M, int N, int K, Operand A, Operand B, const EpiDX2DArgs& e,
+                      cudaStream_t st) {
+  EpiDX2D epi{{}, M, N, e.dX, e.d, e.patch, e.gh, e.gw, e.m};
+  if (A.mn || !B.mn) return cudaErrorInvalidValue;
+  return gemm_dispatch(M, N, K, A, B, epi, e.dXd, M, st);
 }
 
 }  // namespace pf

@@ -35,13 +35,15 @@ constexpr int GEMM_BK = 64;
 constexpr int GEMM_EPI_WARPS = 8;  // two per TMEM lane quarter, each owning half the columns
 constexpr int GEMM_THREADS = 64 + 32 * GEMM_EPI_WARPS;
 
-template <int BN, bool XTILE>
+// XCOLS: columns of the bf16 tile an epilogue prefetches (0: none).
+template <int BN, int XCOLS>
 struct GemmCfg {
-  static constexpr int STAGES = XTILE ? (BN == 256 ? 3 : 5) : (BN == 256 ? 4 : 6);
+  static constexpr int STAGES = XCOLS ? (BN == 256 && XCOLS == 256 ? 3 : (BN == 256 ? 4 : 5))
+                                      : (BN == 256 ? 4 : 6);
   static constexpr uint32_t A_BYTES = GEMM_BM * GEMM_BK * 2;  // 16 KB
   static constexpr uint32_t B_BYTES = BN * GEMM_BK * 2;       // 16/32 KB
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr uint32_t X_BYTES = XTILE ? GEMM_BM * BN * 2 : 0;
+  static constexpr uint32_t X_BYTES = GEMM_BM * XCOLS * 2;
   static constexpr uint32_t SMEM_BYTES =
       STAGES * STAGE_BYTES + X_BYTES + 1024 /*align*/ + 256 /*barriers*/;
 };
@@ -74,7 +76,8 @@ template <int BN, bool A_MN, bool B_MN, class Epi>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmX, int M, int N, int K, Epi epi) {
-  using Cfg = GemmCfg<BN, Epi::kXTile>;
+  constexpr int XCOLS = Epi::kXTile ? (Epi::kPaired ? BN / 2 : BN) : 0;
+  using Cfg = GemmCfg<BN, XCOLS>;
   constexpr int STAGES = Cfg::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -147,7 +150,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         }
         if (!B_MN) {
 #pragma unroll
-          for (int j = 0; j < BN / 128; ++j) tma_load_2d(b_dst + j * 16384, &tmB, fb, k0, n0 + 128 * j);
+          for (int j = 0; j < BN / 128; ++j)
+            tma_load_2d(b_dst + j * 16384, &tmB, fb, k0, epi.b_row(n0, j));
         } else {
 #pragma unroll
           for (int j = 0; j < BN / 64; ++j) tma_load_2d(b_dst + j * 8192, &tmB, fb, n0 + 64 * j, k0);
@@ -206,8 +210,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         mbar_arrive_expect_tx(xfull, Cfg::X_BYTES);
         const int xr = epi.x_row(m0);
 #pragma unroll
-        for (int j = 0; j < BN / 64; ++j)
-          tma_load_2d(smem_u32(xtile) + j * 16384, &tmX, xfull, n0 + 64 * j, xr);
+        for (int j = 0; j < XCOLS / 64; ++j)
+          tma_load_2d(smem_u32(xtile) + j * 16384, &tmX, xfull, epi.x_col(n0, j), xr);
         x_pending = true;
         x_parity = lt & 1;
       }
@@ -218,16 +222,32 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         x_pending = false;
       }
       const int rl = q * 32 + lane;
-      const typename Epi::Row ri = epi.row_info(m0 + rl);
+      const typename Epi::Row ri = epi.row_info(m0 + rl, n0);
+      const uint32_t trow = tmem + buf * BN + ((uint32_t)(q * 32) << 16);
+      if constexpr (Epi::kPaired) {
+        // columns c and c + BN/2 belong together (e.g. s and t of one channel)
 #pragma unroll 1
-      for (int c = c_begin; c < c_begin + BN / 2; c += 32) {
-        float v[32];
-        tmem_ld32(tmem + buf * BN + ((uint32_t)(q * 32) << 16) + (uint32_t)c, v);
-        if (num_k == 0) {
+        for (int c = c_begin / 2; c < c_begin / 2 + BN / 4; c += 32) {
+          float v[32], w[32];
+          tmem_ld32(trow + (uint32_t)c, v);
+          tmem_ld32(trow + (uint32_t)(c + BN / 2), w);
+          if (num_k == 0) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] = 0.f;
+            for (int i = 0; i < 32; ++i) v[i] = w[i] = 0.f;
+          }
+          epi.apply_pair(ri, m0 + rl, n0, c, v, w, xtile, rl);
         }
-        epi.apply(ri, m0 + rl, n0 + c, v, xtile, rl, c);
+      } else {
+#pragma unroll 1
+        for (int c = c_begin; c < c_begin + BN / 2; c += 32) {
+          float v[32];
+          tmem_ld32(trow + (uint32_t)c, v);
+          if (num_k == 0) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = 0.f;
+          }
+          epi.apply(ri, m0 + rl, n0 + c, v, xtile, rl, c);
+        }
       }
       tc_fence_before();
       __syncwarp();
@@ -258,15 +278,28 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
 }
 
 // ------------------------------------------------------------------ epilogues
-// row_info(row) is evaluated once per tile and output row; apply(ri, row, col,
-// v, xt, rl, cl) then receives 32 consecutive accumulator columns [col,
+// row_info(row, n0) is evaluated once per tile and output row; apply(ri, row,
+// col, v, xt, rl, cl) then receives 32 consecutive accumulator columns [col,
 // col+32) of that row, with rl / cl the row and column inside the tile and xt
-// the prefetched bf16 tile (kXTile epilogues; x_row(m0) gives the row of the
-// tile's first line in the X tensor map).  N is a multiple of 32.
+// the prefetched bf16 tile (kXTile epilogues: x_row(m0) / x_col(n0, j) give the
+// coordinates of the tile's 64-column boxes in the X tensor map).  kPaired
+// epilogues receive columns c and c + BN/2 together through apply_pair, and
+// prefetch BN/2 columns.  b_row(n0, j) is the first row of B (K-major) loaded
+// for 128-row box j of the tile starting at output column n0.  N is a
+// multiple of 32.
+struct EpiBase {
+  static constexpr bool kXTile = false;
+  static constexpr bool kPaired = false;
+  __device__ __forceinline__ int x_row(int m0) const { return m0; }
+  __device__ __forceinline__ int x_col(int n0, int j) const { return n0 + 64 * j; }
+  __device__ __forceinline__ int b_row(int n0, int j) const { return n0 + 128 * j; }
+  template <class R>
+  __device__ __forceinline__ void apply_pair(const R&, int, int, int, float*, float*,
+                                             const uint8_t*, int) const {}
+};
 
 // v = acc (+ bias[col]) (+ addend[row, col]); stored as fp32 and/or bf16.
-struct EpiLinear {
-  static constexpr bool kXTile = false;
+struct EpiLinear : EpiBase {
   struct Row {
     bool ok;
   };
@@ -278,8 +311,7 @@ struct EpiLinear {
   long ld_f32;
   bf16* out_bf16;
   long ld_bf16;
-  __device__ __forceinline__ int x_row(int m0) const { return m0; }
-  __device__ __forceinline__ Row row_info(int row) const { return Row{row < M}; }
+  __device__ __forceinline__ Row row_info(int row, int) const { return Row{row < M}; }
   __device__ __forceinline__ void apply(const Row& ri, int row, int col, float* v, const uint8_t*,
                                         int, int) const {
     if (!ri.ok || col >= N) return;
@@ -322,7 +354,7 @@ struct EpiLinear {
 //   add:   X_out = X + D                                    (Eq. inj-add)
 // X is read from the prefetched tile: rows r + shift*k2 of the view
 // [B*m*k2, k1*d] of X (zero-padded to whole blocks when L % P != 0).
-struct EpiInject1D {
+struct EpiInject1D : EpiBase {
   static constexpr bool kXTile = true;
   struct Row {
     bool ok;    // row < M
@@ -336,7 +368,7 @@ struct EpiInject1D {
   const float *w_x, *w_dlt, *b_g;
   int d, k1, k2, m, L, shift, gated;
   __device__ __forceinline__ int x_row(int m0) const { return m0 + shift * k2; }
-  __device__ __forceinline__ Row row_info(int row) const {
+  __device__ __forceinline__ Row row_info(int row, int) const {
     Row r{row < M, 0, 0};
     const int a = row % k2, prox = row / k2;
     const int b = prox / m, i = prox % m;
@@ -398,7 +430,7 @@ struct EpiInject1D {
 // c%d) -> token i*P + a*k1 + c/d of sequence b.  The direct gradient is read
 // from the prefetched tile of dXd, the view [B*m*k2, k1*d] of a buffer padded
 // to whole blocks (dX itself when L % P == 0); the sum is written to dX.
-struct EpiDX1D {
+struct EpiDX1D : EpiBase {
   static constexpr bool kXTile = true;
   struct Row {
     bool ok;
@@ -408,8 +440,7 @@ struct EpiDX1D {
   int M, N;
   bf16* dX;
   int d, k1, k2, m, L;
-  __device__ __forceinline__ int x_row(int m0) const { return m0; }
-  __device__ __forceinline__ Row row_info(int row) const {
+  __device__ __forceinline__ Row row_info(int row, int) const {
     Row r{row < M, 0, 0};
     const int per_seq = m * k2;
     const int b = row / per_seq, rr = row % per_seq;
@@ -439,8 +470,7 @@ struct EpiDX1D {
 // KV append (Sec. 3.8): rows are sequences b, columns [0, 2d) the proxy's key
 // and value rows W_kh H and W_vh H, written as bf16 at cache row n_proxy[b] of
 // the sequences whose open block is full and whose cache has room.
-struct EpiAppendKV {
-  static constexpr bool kXTile = false;
+struct EpiAppendKV : EpiBase {
   struct Row {
     bool ok;
     long off;
@@ -449,8 +479,7 @@ struct EpiAppendKV {
   bf16 *K, *V;
   const int *n_open, *n_proxy;
   int d, P, cap;
-  __device__ __forceinline__ int x_row(int m0) const { return m0; }
-  __device__ __forceinline__ Row row_info(int row) const {
+  __device__ __forceinline__ Row row_info(int row, int) const {
     Row r{false, 0};
     if (row < M) {
       const int np = n_proxy[row];
@@ -465,6 +494,110 @@ struct EpiAppendKV {
     bf16* o = col < d ? K + ri.off + col : V + ri.off + (col - d);
 #pragma unroll
     for (int i = 0; i < 32; i += 8) store8_bf16(o + i, v + i);
+  }
+};
+
+// Decompression of the 2D layer fused with affine injection (Eq. inj-affine):
+// X_out = (1 + s) * LayerNorm(X) + t.  GEMM rows are patches r = (b, by, bx);
+// W_d1 [2*P*d, d] holds s for token p of a patch at rows [2pd, 2pd+d) and t at
+// [2pd+d, 2(p+1)d).  Output tile n0 = 256*nt covers token p = nt / (d/128) and
+// channels [cb, cb+128), cb = 128 * (nt % (d/128)): its B rows are loaded as
+// s (columns 0..127) then t (128..255), so each thread holds matching s and t.
+// X comes from the prefetched tile of the patch-ordered copy Xp [B*m, P*d];
+// LayerNorm statistics per token from `stats` (mean, 1/std).  s is saved in
+// patch order [B*m, P*d] for the backward.
+struct EpiAffine2D : EpiBase {
+  static constexpr bool kXTile = true;
+  static constexpr bool kPaired = true;
+  struct Row {
+    bool ok;
+    long xoff;  // element offset of (token, channel cb) in X_out
+    float mu, rs;
+  };
+  int M;
+  const float* bias;
+  bf16* S_save;
+  bf16* X_out;
+  const float* stats;
+  int d, patch, gh, gw, m;
+  __device__ __forceinline__ int ptok(int n0) const { return n0 / (2 * d); }
+  __device__ __forceinline__ int cbase(int n0) const { return ((n0 >> 8) % (d >> 7)) << 7; }
+  __device__ __forceinline__ int b_row(int n0, int j) const {
+    return ptok(n0) * 2 * d + j * d + cbase(n0);
+  }
+  __device__ __forceinline__ int x_col(int n0, int j) const {
+    return ptok(n0) * d + cbase(n0) + 64 * j;
+  }
+  __device__ __forceinline__ Row row_info(int row, int n0) const {
+    Row r{row < M, 0, 0.f, 0.f};
+    if (!r.ok) return r;
+    const int npw = gw / patch;
+    const int b = row / m, pr = row % m, by = pr / npw, bx = pr % npw;
+    const int p = ptok(n0), py = p / patch, px = p % patch;
+    const long tok = (long)b * gh * gw + (long)(by * patch + py) * gw + bx * patch + px;
+    r.xoff = tok * d + cbase(n0);
+    r.mu = stats[2 * tok];
+    r.rs = stats[2 * tok + 1];
+    return r;
+  }
+  __device__ __forceinline__ void apply_pair(const Row& ri, int row, int n0, int c, float* vs,
+                                             float* vt, const uint8_t* xt, int rl) const {
+    if (!ri.ok) return;
+    const int p = ptok(n0), ch0 = cbase(n0) + c;
+    const float* bs = bias + (long)p * 2 * d + ch0;
+    const float* bt = bs + d;
+    bf16* so = S_save + (long)row * (patch * patch * d) + (long)p * d + ch0;
+    bf16* xo = X_out + ri.xoff + c;
+#pragma unroll
+    for (int i8 = 0; i8 < 32; i8 += 8) {
+      float x[8], o[8], sv[8];
+      xtile_load8(xt, rl, c + i8, x);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        sv[j] = vs[i8 + j] + bs[i8 + j];
+        const float t = vt[i8 + j] + bt[i8 + j];
+        o[j] = fmaf(1.f + sv[j], (x[j] - ri.mu) * ri.rs, t);
+      }
+      store8_bf16(so + i8, sv);
+      store8_bf16(xo + i8, o);
+    }
+  }
+};
+
+// Compression input gradient of the 2D layer: rows are patches, columns
+// (token p = c / d of the patch, channel c % d); the direct gradient comes from
+// the prefetched tile of dXd (same patch order) and the sum is written to dX
+// at the token's raster position.
+struct EpiDX2D : EpiBase {
+  static constexpr bool kXTile = true;
+  struct Row {
+    bool ok;
+    long base;  // offset of the patch's top-left token in dX
+  };
+  int M, N;
+  bf16* dX;
+  int d, patch, gh, gw, m;
+  __device__ __forceinline__ Row row_info(int row, int) const {
+    Row r{row < M, 0};
+    if (!r.ok) return r;
+    const int npw = gw / patch;
+    const int b = row / m, pr = row % m, by = pr / npw, bx = pr % npw;
+    r.base = ((long)b * gh * gw + (long)by * patch * gw + bx * patch) * d;
+    return r;
+  }
+  __device__ __forceinline__ void apply(const Row& ri, int, int col, float* v, const uint8_t* xt,
+                                        int rl, int cl) const {
+    if (!ri.ok || col >= N) return;
+    const int p = col / d, ch = col - p * d, py = p / patch, px = p - py * patch;
+    bf16* o = dX + ri.base + ((long)py * gw + px) * d + ch;
+#pragma unroll
+    for (int i8 = 0; i8 < 32; i8 += 8) {
+      float x[8];
+      xtile_load8(xt, rl, cl + i8, x);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) x[j] += v[i8 + j];
+      store8_bf16(o + i8, x);
+    }
   }
 };
 

@@ -47,6 +47,25 @@ cudaError_t gemm_inject1d(int M, int N, int K, Operand A, Operand B, const EpiIn
 cudaError_t gemm_dx1d(int M, int N, int K, Operand A, Operand B, const EpiDXArgs& e,
                       cudaStream_t st);
 
+// 2D layer: decompression + affine injection, and the compression dX.
+struct EpiAffine2DArgs {
+  const float* bias;   // b_d1 [2*P*d]
+  bf16* S_save;        // s in patch order [B*m, P*d]
+  bf16* X_out;         // [B, gh*gw, d]
+  const float* stats;  // [B*gh*gw, 2] mean, 1/std of X per token
+  const bf16* Xp;      // X in patch order [B*m, P*d]
+  int d, patch, gh, gw, m;
+};
+cudaError_t gemm_affine2d(int M, int N, int K, Operand A, Operand B, const EpiAffine2DArgs& e,
+                          cudaStream_t st);
+struct EpiDX2DArgs {
+  const bf16* dXd;  // direct gradient in patch order [B*m, P*d]
+  bf16* dX;         // [B, gh*gw, d]
+  int d, patch, gh, gw, m;
+};
+cudaError_t gemm_dx2d(int M, int N, int K, Operand A, Operand B, const EpiDX2DArgs& e,
+                      cudaStream_t st);
+
 // KV append: rows b = sequences, columns [0, d) -> K_proxy[b, n_proxy[b]],
 // [d, 2d) -> V_proxy[b, n_proxy[b]] (bf16), only for sequences whose open
 // block is full (n_open[b] == P) and whose cache has room.
@@ -64,6 +83,31 @@ int take_dev_error_gemm();
 int take_dev_error_decode();
 int take_dev_error_attention();
 int take_dev_error_elementwise();
+
+// ------------------------------------------------------------- 2D layer
+int take_dev_error_layer2d();
+cudaError_t patch_gather(const bf16* X, bf16* Xp, int B, int d, int patch, int gh, int gw,
+                         cudaStream_t st);
+cudaError_t ln_stats(const bf16* X, float* stats, long T, int d, cudaStream_t st);
+cudaError_t temb_fwd(const float* t, int B, int d, const bf16* W_t1, const float* b_t1,
+                     const bf16* W_t2, const float* b_t2, float* e, float* a1, float* u, float* gb,
+                     cudaStream_t st);
+cudaError_t adaln_fwd(const float* H, const float* gb, float* nH, float* rstd, bf16* Hq, long R,
+                      int d, int m, cudaStream_t st);
+cudaError_t inj_bwd_2d(const bf16* G, const bf16* X, const float* stats, const bf16* S, bf16* dD,
+                       bf16* dXd, long T, int d, int patch, int gh, int gw, cudaStream_t st);
+cudaError_t adaln_bwd(const float* dHq, const float* nH, const float* rstd, const float* gb,
+                      const float* dH_out, float* dHf, bf16* dHb, long R, int d, int m,
+                      cudaStream_t st);
+int adaln_param_chunks(int m);
+cudaError_t adaln_param_grads(const float* dHq, const float* nH, float* part, float* dgb, int B,
+                              int d, int m, cudaStream_t st);
+struct TembGrads {
+  float *W_t2, *b_t2, *W_t1, *b_t1;
+};
+cudaError_t temb_bwd(const float* dgb, const bf16* W_t2, const float* a1, const float* u,
+                     const float* e, float* da1, const TembGrads& g, int B, int d,
+                     cudaStream_t st);
 
 // ---------------------------------------------------------- fp32 forward
 int take_dev_error_fp32();
