@@ -43,6 +43,8 @@ def parse_args():
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-decode", action="store_true")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the other workloads (fp32 layer, L=65536 layer, 2D layer, stack)")
     ap.add_argument("--decode-steps", type=int, default=128)
     ap.add_argument("--L", type=int, default=0,
                     help="tokens per sequence (default: the workload's 262144; smaller values "
@@ -290,6 +292,109 @@ def measure_decode(torch, pf, S, steps: int):
     return spec, ms, a0.elapsed_time(a1), step_bytes, kern
 
 
+def timed_steps(torch, pf, fn, steps: int, warmup: int):
+    """Mean ms per call of fn (CUDA events on the current stream) plus the
+    library's per-launch records: algorithmic FLOPs and bytes per call and the
+    label with the largest time."""
+    stream = torch.cuda.current_stream()
+    for _ in range(warmup):
+        fn()
+    torch.cuda.synchronize()
+    pf.pf_timing_enable(True)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        fn()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    t = pf.pf_timing_collect()
+    pf.pf_timing_enable(False)
+    pf.pf_sync_check(stream.cuda_stream)
+    flops = sum(v["flops"] * v["launches"] for v in t.values()) / steps
+    nbytes = sum(v["bytes"] * v["launches"] for v in t.values()) / steps
+    total = sum(v["ms"] for v in t.values()) or 1.0
+    dom, dv = max(t.items(), key=lambda kv: kv[1]["ms"])
+    return ms, flops, nbytes, {"kernel": dom, "share": dv["ms"] / total}
+
+
+FFMA_PEAK_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12  # SMs x fp32 lanes x 2 x max SM clock
+
+
+def config_entry(metric, tokens, ms, flops, nbytes, dom, peaks, steps, alu=False):
+    comp_peak = FFMA_PEAK_TFLOPS if alu else peaks["bf16_tflops_sustained"]
+    roof_ms = max(flops / (comp_peak * 1e12), nbytes / (peaks["hbm_gbs"] * 1e9)) * 1e3
+    return {"metric": metric, "value": tokens / (ms / 1e3), "unit": "tokens/s",
+            "ms_per_step": ms, "steps": steps,
+            "roofline": {"bound": "alu" if alu else "tensor", "flops_per_step": flops,
+                         "bytes_per_step": nbytes, "compute_peak_tflops": comp_peak,
+                         "roofline_ms": roof_ms, "frac": roof_ms / ms, **dom}}
+
+
+def measure_configs(torch, pf, S, peaks, warmup: int):
+    """The other paper workloads, each timed on its own (fresh buffers)."""
+    from paper_2608_23463_gb300.layer import ProxyLayer, to_device
+    from paper_2608_23463_gb300.stack import ProxyStack
+    out = {}
+
+    def layer_case(spec, seed, train, steps):
+        inp = S.make_layer_inputs(spec, seed, with_grads=train)
+        dt = torch.bfloat16 if spec.dtype == S.BF16 else torch.float32
+        lay = ProxyLayer(spec, inp)
+        X = to_device(inp["X"], dt)
+        G = to_device(inp["G"], dt) if train else None
+        t = to_device(inp["t"], torch.float32) if "t" in inp else None
+        del inp
+        Xo, dX = lay.empty_act(), lay.empty_act()
+
+        def step():
+            lay.forward(X, None, t, X_out=Xo, train=train)
+            if train:
+                lay.backward(X, G, None, t, dX=dX)
+        return timed_steps(torch, pf, step, steps, warmup)
+
+    s1 = S.spec_c1()
+    ms, fl, nb, dom = layer_case(s1, 0, False, 20)
+    out["c1_fp32_fwd"] = config_entry("1D causal layer fwd, fp32, L=4096 d=256 4x64 P=64",
+                                      s1.batch * s1.L, ms, fl, nb, dom, peaks, 20, alu=True)
+    torch.cuda.empty_cache()
+    s2 = S.spec_c2()
+    ms, fl, nb, dom = layer_case(s2, 1, True, 10)
+    out["c2_layer_fwd_bwd"] = config_entry(
+        "1D causal layer fwd+bwd, bf16, L=65536 d=1024 16x64 P=64", s2.batch * s2.L, ms, fl, nb,
+        dom, peaks, 10)
+    torch.cuda.empty_cache()
+    s5 = S.spec_c5()
+    ms, fl, nb, dom = layer_case(s5, 4, True, 5)
+    out["c5_2d_fwd_bwd"] = config_entry(
+        "2D bidirectional layer fwd+bwd, bf16, B=4 512x512 d=512 8x64 8x8 patches",
+        s5.batch * s5.L, ms, fl, nb, dom, peaks, 5)
+    torch.cuda.empty_cache()
+    specs, params = [], []
+    for i, P in enumerate(S.C3_RATIOS):
+        k1, k2 = S.default_factors(P)
+        sp = S.LayerSpec(batch=1, L=262144, d=1024, n_heads=16, P=P, levels=2, k1=k1, k2=k2)
+        specs.append(sp)
+        params.append(S.make_layer_params(sp, 2 + 10 * i))
+    st = ProxyStack(specs, params)
+    del params
+    inp = S.make_layer_inputs(specs[0], 2, with_grads=True)
+    X = to_device(inp["X"], torch.bfloat16)
+    G = to_device(inp["G"], torch.bfloat16)
+    del inp
+
+    def stack_step():
+        st.forward(X)
+        st.backward(G)
+    ms, fl, nb, dom = timed_steps(torch, pf, stack_step, 3, warmup)
+    out["c3_stack_fwd_bwd"] = config_entry(
+        "12-layer causal stack fwd+bwd, bf16, L=262144 d=1024 16x64, P=16..256 two-level",
+        specs[0].L, ms, fl, nb, dom, peaks, 3)
+    del st, X, G
+    torch.cuda.empty_cache()
+    return out
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -398,6 +503,14 @@ def run_ours(args, rank: int, world: int, local_rank: int):
         del lay, X, G, Xo, dX
         torch.cuda.empty_cache()
         decode_result = measure_decode(torch, pf, S, args.decode_steps)
+    configs_result = None
+    if not args.no_configs:
+        if not args.no_decode:
+            torch.cuda.empty_cache()
+        else:
+            del lay, X, G, Xo, dX
+            torch.cuda.empty_cache()
+        configs_result = measure_configs(torch, pf, S, load_peaks()[0], max(args.warmup, 3))
     if rank != 0:
         return
 
@@ -454,6 +567,8 @@ def run_ours(args, rank: int, world: int, local_rank: int):
                          "frac": dbytes / (dms / 1e3) / 1e9 / peaks["hbm_gbs"],
                          "bytes_per_step": dbytes},
             "append_ms": app_ms, "kernels_ms_per_step": dkern}
+    if configs_result is not None:
+        line["configs"] = configs_result
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline_subprocess()
     print(json.dumps(line), flush=True)

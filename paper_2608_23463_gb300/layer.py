@@ -27,7 +27,8 @@ def to_device(a: np.ndarray, dtype: torch.dtype, device="cuda") -> torch.Tensor:
 class ProxyLayer:
     """One layer (Alg. 1) with device buffers sized from the descriptor."""
 
-    def __init__(self, spec, params: Dict[str, np.ndarray], device="cuda"):
+    def __init__(self, spec, params: Dict[str, np.ndarray], device="cuda",
+                 ws: Optional[torch.Tensor] = None):
         self.spec = spec
         self.desc = layer_desc(spec)
         self.act_dtype = torch.bfloat16 if spec.dtype == PF_BF16 else torch.float32
@@ -46,8 +47,11 @@ class ProxyLayer:
                                  device=device)
         self.ws_fwd_bytes = proxy_layer_workspace_size(self.desc, 0)
         self.ws_bwd_bytes = proxy_layer_workspace_size(self.desc, 1)
-        self.ws = torch.empty(max(self.ws_fwd_bytes, self.ws_bwd_bytes, 16), dtype=torch.uint8,
-                              device=device)
+        need = max(self.ws_fwd_bytes, self.ws_bwd_bytes, 16)
+        if ws is not None and ws.numel() >= need:
+            self.ws = ws  # shared with other layers that run on the same stream
+        else:
+            self.ws = torch.empty(need, dtype=torch.uint8, device=device)
 
     def empty_act(self) -> torch.Tensor:
         s = self.spec

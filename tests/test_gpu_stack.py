@@ -1,0 +1,58 @@
+"""A stack of causal 1D layers with layer-wise ratios (Sec. 3.6) against the
+float64 oracle composed layer by layer: H is carried between layers with the
+same P and re-extracted when P changes; the backward follows the same rule."""
+import numpy as np
+import pytest
+import torch
+
+import paper_2608_23463_gb300 as pf
+import pf_synth as S
+from oracle import layer as OL
+from paper_2608_23463_gb300.stack import ProxyStack
+from tests._util import assert_grad_close
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    pf.build()
+    pf.load()
+
+
+def test_stack_matches_composed_oracle():
+    ratios = (4, 4, 8, 16, 16)
+    L, d, nh = 1024, 128, 2
+    specs = []
+    for P in ratios:
+        k1, k2 = S.default_factors(P)
+        specs.append(S.LayerSpec(batch=1, L=L, d=d, n_heads=nh, P=P, levels=2, k1=k1, k2=k2))
+    params = [S.make_layer_params(s, 70 + i) for i, s in enumerate(specs)]
+    inp = S.make_layer_inputs(specs[0], 80)
+    st = ProxyStack(specs, params)
+    X = torch.from_numpy(inp["X"]).cuda().to(torch.bfloat16)
+    G = torch.from_numpy(inp["G"]).cuda().to(torch.bfloat16)
+    Xo = st.forward(X).float().cpu().numpy()
+    dX = st.backward(G).float().cpu().numpy()
+    pf.pf_sync_check(torch.cuda.current_stream().cuda_stream)
+    # oracle: forward layer by layer, keeping each layer's input and H
+    xs, hs = [inp["X"].astype(np.float64)], []
+    for l, (s, p) in enumerate(zip(specs, params)):
+        carry = l > 0 and specs[l].P == specs[l - 1].P
+        xo, h = OL.layer_fwd(s, p, xs[-1], hs[-1] if carry else None)
+        xs.append(xo)
+        hs.append(h)
+    assert_grad_close("stack X_out", Xo, xs[-1])
+    g, dh_next, grads = inp["G"].astype(np.float64), None, []
+    for l in reversed(range(len(specs))):
+        carry = l > 0 and specs[l].P == specs[l - 1].P
+        nxt = l + 1 < len(specs) and specs[l + 1].P == specs[l].P
+        g, dh_in, gr = OL.layer_bwd(specs[l], params[l], xs[l], g, hs[l - 1] if carry else None,
+                                    None, dh_next if nxt else None)
+        dh_next = dh_in
+        grads.append((l, gr))
+    assert_grad_close("stack dX", dX, g)
+    for l, gr in grads:
+        for k in ("W_c1", "W_d1", "W_qkv", "b_g"):
+            assert_grad_close(f"layer {l} grad {k}", st.layers[l].grads[k].cpu().numpy(), gr[k])
