@@ -1,6 +1,9 @@
 """A stack of causal 1D layers with layer-wise ratios (Sec. 3.6) against the
 float64 oracle composed layer by layer: H is carried between layers with the
-same P and re-extracted when P changes; the backward follows the same rule."""
+same P and re-extracted when P changes; the backward follows the same rule.
+Bar: X_out RMS 3e-2; dX and weight gradients RMS 1e-1, max 1 -- twice the
+bf16 floor of this stack (test_bf16_error_floor.py), well below the O(1)
+error of a wrong carry rule."""
 import numpy as np
 import pytest
 import torch
@@ -43,7 +46,7 @@ def test_stack_matches_composed_oracle():
         xo, h = OL.layer_fwd(s, p, xs[-1], hs[-1] if carry else None)
         xs.append(xo)
         hs.append(h)
-    assert_grad_close("stack X_out", Xo, xs[-1])
+    assert_grad_close("stack X_out", Xo, xs[-1], tol=3e-2, max_tol=2e-1)
     g, dh_next, grads = inp["G"].astype(np.float64), None, []
     for l in reversed(range(len(specs))):
         carry = l > 0 and specs[l].P == specs[l - 1].P
@@ -52,7 +55,8 @@ def test_stack_matches_composed_oracle():
                                     None, dh_next if nxt else None)
         dh_next = dh_in
         grads.append((l, gr))
-    assert_grad_close("stack dX", dX, g)
+    assert_grad_close("stack dX", dX, g, tol=1e-1, max_tol=1.0)
     for l, gr in grads:
         for k in ("W_c1", "W_d1", "W_qkv", "b_g"):
-            assert_grad_close(f"layer {l} grad {k}", st.layers[l].grads[k].cpu().numpy(), gr[k])
+            assert_grad_close(f"layer {l} grad {k}", st.layers[l].grads[k].cpu().numpy(), gr[k],
+                              tol=1e-1, max_tol=1.0)
