@@ -5,6 +5,7 @@
 
 #include <algorithm>
 #include <string>
+#include <vector>
 
 #include "kernels.h"
 #include "proxyformer.h"
@@ -70,6 +71,37 @@ Dims dims_of(const pf_layer_desc& s) {
   return g;
 }
 
+// Largest split-K scratch needed by the layer's linear GEMMs (forward or
+// backward); the GEMM shapes below mirror the launch sequence.
+size_t splitk_need(const pf_layer_desc& s, const Dims& g, bool bwd) {
+  const int d = (int)g.d, R = (int)g.R, r1 = (int)g.rows1, N1 = (int)g.N1, n2 = (int)(g.k2 * d);
+  struct S3 {
+    int M, N, K;
+  };
+  std::vector<S3> v;
+  if (s.mode == PF_BIDIR_2D) {
+    if (!bwd) v = {{R, d, N1}, {R, 3 * d, d}, {R, d, d}};
+    else v = {{2 * N1, d, R}, {R, d, 2 * N1}, {d, d, R}, {R, d, d}, {3 * d, d, R}, {R, d, 3 * d},
+              {d, N1, R}};
+  } else if (!bwd) {
+    v = {{R, 3 * d, d}, {R, d, d}};
+    if (s.levels == 1) v.push_back({R, d, N1});
+    else v.insert(v.end(), {{r1, d, N1}, {R, d, n2}, {R, n2, d}});
+  } else {
+    v = {{N1, d, r1}, {r1, d, N1}, {d, d, R}, {R, d, d}, {3 * d, d, R}, {R, d, 3 * d}, {d, N1, r1}};
+    if (s.levels == 2) v.insert(v.end(), {{n2, d, R}, {R, d, n2}, {d, n2, R}, {R, n2, d}});
+  }
+  size_t m = 0;
+  for (const S3& x : v) m = std::max(m, splitk_scratch_bytes(x.M, x.N, x.K));
+  return m;
+}
+
+EpiLinearArgs with_sk(EpiLinearArgs e, float* sk, size_t skb) {
+  e.splitk_scratch = sk;
+  e.splitk_bytes = skb;
+  return e;
+}
+
 // Buffers the forward saves for the backward pass (order fixes the layout).
 struct Saved {
   bf16 *Hb, *QKV, *Aatt, *Hbar, *Y, *Z, *D;
@@ -93,8 +125,9 @@ Saved carve_saved(Carve& c, const pf_layer_desc& s, const Dims& g) {
 
 struct BwdWs {
   bf16 *Xpad, *dXpad, *dD, *dZ, *dHbar, *dA, *dQKV, *dHb, *dY;
-  float *Di, *dHf, *part;
+  float *Di, *dHf, *part, *sk;
   long part_elems;
+  size_t skb;
 };
 
 BwdWs carve_bwd(Carve& c, const pf_layer_desc& s, const Dims& g) {
@@ -116,6 +149,8 @@ BwdWs carve_bwd(Carve& c, const pf_layer_desc& s, const Dims& g) {
   pe = std::max(pe, colsum_part_elems(g.rows1, (int)g.d));
   w.part_elems = pe;
   w.part = c.take<float>(pe);
+  w.skb = splitk_need(s, g, true);
+  w.sk = c.take<float>(w.skb / sizeof(float));
   return w;
 }
 
@@ -147,10 +182,11 @@ Saved2D carve_saved_2d(Carve& c, const Dims& g) {
 
 struct Bwd2DWs {
   bf16 *dD, *dXd, *dHbar, *dA, *dQKV, *dHb;
-  float *Di, *dHq, *dHf, *part, *dgb, *da1;
+  float *Di, *dHq, *dHf, *part, *dgb, *da1, *sk;
+  size_t skb;
 };
 
-Bwd2DWs carve_bwd_2d(Carve& c, const Dims& g) {
+Bwd2DWs carve_bwd_2d(Carve& c, const pf_layer_desc& s, const Dims& g) {
   Bwd2DWs w{};
   w.dD = c.take<bf16>(g.R * 2 * g.N1);
   w.dXd = c.take<bf16>(g.R * g.N1);
@@ -167,6 +203,8 @@ Bwd2DWs carve_bwd_2d(Carve& c, const Dims& g) {
   w.part = c.take<float>(pe);
   w.dgb = c.take<float>(g.B * 2 * g.d);
   w.da1 = c.take<float>(g.B * g.d);
+  w.skb = splitk_need(s, g, true);
+  w.sk = c.take<float>(w.skb / sizeof(float));
   return w;
 }
 
@@ -289,6 +327,8 @@ pf_status layer_fwd_2d(const pf_layer_desc& s, const Dims& g, const pf_layer_par
     return fail(PF_ERR_INVALID_ARG, "a parameter of the 2D layer is NULL");
   Carve wc(ws);
   float* Hws = wc.take<float>(g.R * g.d);
+  const size_t skb = splitk_need(s, g, false);
+  float* sk = wc.take<float>(skb / sizeof(float));
   Carve sc(saved);
   const Saved2D sv = saved ? carve_saved_2d(sc, g) : carve_saved_2d(wc, g);
   if (ws == nullptr || wc.off > ws_bytes)
@@ -307,8 +347,7 @@ pf_status layer_fwd_2d(const pf_layer_desc& s, const Dims& g, const pf_layer_par
     e.out_f32 = Hf;
     e.ld_f32 = d;
     set_gemm_tag("compress_c1", (double)g.R * d * 8.0);
-    PF_CUDA(gemm_linear((int)g.R, d, N1, {sv.Xp, N1, 0}, {static_cast<const bf16*>(p.W_c1), N1, 0},
-                        e, cs));
+    PF_CUDA(gemm_linear((int)g.R, d, N1, {sv.Xp, N1, 0}, {static_cast<const bf16*>(p.W_c1), N1, 0}, with_sk(e, sk, skb), cs));
   }
   PF_CUDA(temb_fwd(t, (int)g.B, d, static_cast<const bf16*>(p.W_t1), p.b_t1,
                    static_cast<const bf16*>(p.W_t2), p.b_t2, sv.e, sv.a1, sv.u, sv.gb, cs));
@@ -319,14 +358,13 @@ pf_status layer_fwd_2d(const pf_layer_desc& s, const Dims& g, const pf_layer_par
     e.ld_bf16 = 3 * d;
     set_gemm_tag("proxy_qkv", (double)g.R * 3 * d * 2.0);
     PF_CUDA(gemm_linear((int)g.R, 3 * d, d, {sv.Hb, d, 0},
-                        {static_cast<const bf16*>(p.W_qkv), d, 0}, e, cs));
+                        {static_cast<const bf16*>(p.W_qkv), d, 0}, with_sk(e, sk, skb), cs));
     PF_CUDA(attn_fwd(sv.QKV, sv.Aatt, sv.LSE, (int)g.B, (int)g.m, d, (int)g.nh, false, cs));
     EpiLinearArgs eo;
     eo.out_bf16 = sv.Hbar;
     eo.ld_bf16 = d;
     set_gemm_tag("proxy_o", (double)g.R * d * 2.0);
-    PF_CUDA(gemm_linear((int)g.R, d, d, {sv.Aatt, d, 0}, {static_cast<const bf16*>(p.W_o), d, 0},
-                        eo, cs));
+    PF_CUDA(gemm_linear((int)g.R, d, d, {sv.Aatt, d, 0}, {static_cast<const bf16*>(p.W_o), d, 0}, with_sk(eo, sk, skb), cs));
   }
   {
     EpiAffine2DArgs e{p.b_d1, sv.S, static_cast<bf16*>(X_out), sv.stats, sv.Xp, d, patch, gh, gw,
@@ -343,7 +381,7 @@ pf_status layer_bwd_2d(const pf_layer_desc& s, const Dims& g, const pf_layer_par
                        void* dXv, float* dH_in, const pf_layer_grads& gr, void* ws,
                        size_t ws_bytes, cudaStream_t cs) {
   Carve wc(ws);
-  const Bwd2DWs w = carve_bwd_2d(wc, g);
+  const Bwd2DWs w = carve_bwd_2d(wc, s, g);
   if (ws == nullptr || wc.off > ws_bytes)
     return fail(PF_ERR_WORKSPACE, "workspace too small: need %zu bytes, got %zu", wc.off, ws_bytes);
   Carve sc(const_cast<void*>(saved));
@@ -365,28 +403,28 @@ pf_status layer_bwd_2d(const pf_layer_desc& s, const Dims& g, const pf_layer_par
     e.out_f32 = gr.W_d1;
     e.ld_f32 = d;
     set_gemm_tag("bwd_dW_d1", (double)N2 * d * 4.0);
-    PF_CUDA(gemm_linear(N2, d, (int)g.R, {w.dD, N2, 1}, {sv.Hbar, d, 1}, e, cs));
+    PF_CUDA(gemm_linear(N2, d, (int)g.R, {w.dD, N2, 1}, {sv.Hbar, d, 1}, with_sk(e, w.sk, w.skb), cs));
   }
   {
     EpiLinearArgs e;
     e.out_bf16 = w.dHbar;
     e.ld_bf16 = d;
     set_gemm_tag("bwd_dHbar", (double)g.R * d * 2.0);
-    PF_CUDA(gemm_linear((int)g.R, d, N2, {w.dD, N2, 0}, {W_d1, d, 1}, e, cs));
+    PF_CUDA(gemm_linear((int)g.R, d, N2, {w.dD, N2, 0}, {W_d1, d, 1}, with_sk(e, w.sk, w.skb), cs));
   }
   if (gr.W_o) {
     EpiLinearArgs e;
     e.out_f32 = gr.W_o;
     e.ld_f32 = d;
     set_gemm_tag("bwd_dW_o", (double)d * d * 4.0);
-    PF_CUDA(gemm_linear(d, d, (int)g.R, {w.dHbar, d, 1}, {sv.Aatt, d, 1}, e, cs));
+    PF_CUDA(gemm_linear(d, d, (int)g.R, {w.dHbar, d, 1}, {sv.Aatt, d, 1}, with_sk(e, w.sk, w.skb), cs));
   }
   {
     EpiLinearArgs e;
     e.out_bf16 = w.dA;
     e.ld_bf16 = d;
     set_gemm_tag("bwd_dA", (double)g.R * d * 2.0);
-    PF_CUDA(gemm_linear((int)g.R, d, d, {w.dHbar, d, 0}, {W_o, d, 1}, e, cs));
+    PF_CUDA(gemm_linear((int)g.R, d, d, {w.dHbar, d, 0}, {W_o, d, 1}, with_sk(e, w.sk, w.skb), cs));
   }
   PF_CUDA(attn_bwd(sv.QKV, sv.Aatt, w.dA, sv.LSE, w.Di, w.dQKV, (int)g.B, (int)g.m, d, (int)g.nh,
                    false, cs));
@@ -395,14 +433,14 @@ pf_status layer_bwd_2d(const pf_layer_desc& s, const Dims& g, const pf_layer_par
     e.out_f32 = gr.W_qkv;
     e.ld_f32 = d;
     set_gemm_tag("bwd_dW_qkv", (double)3 * d * d * 4.0);
-    PF_CUDA(gemm_linear(3 * d, d, (int)g.R, {w.dQKV, 3 * d, 1}, {sv.Hb, d, 1}, e, cs));
+    PF_CUDA(gemm_linear(3 * d, d, (int)g.R, {w.dQKV, 3 * d, 1}, {sv.Hb, d, 1}, with_sk(e, w.sk, w.skb), cs));
   }
   {
     EpiLinearArgs e;
     e.out_f32 = w.dHq;
     e.ld_f32 = d;
     set_gemm_tag("bwd_dHq", (double)g.R * d * 4.0);
-    PF_CUDA(gemm_linear((int)g.R, d, 3 * d, {w.dQKV, 3 * d, 0}, {W_qkv, d, 1}, e, cs));
+    PF_CUDA(gemm_linear((int)g.R, d, 3 * d, {w.dQKV, 3 * d, 0}, {W_qkv, d, 1}, with_sk(e, w.sk, w.skb), cs));
   }
   // adaLN and timestep-MLP backward
   float* dHf = dH_in ? dH_in : w.dHf;
@@ -417,7 +455,7 @@ pf_status layer_bwd_2d(const pf_layer_desc& s, const Dims& g, const pf_layer_par
     e.out_f32 = gr.W_c1;
     e.ld_f32 = N1;
     set_gemm_tag("bwd_dW_c1", (double)d * N1 * 4.0);
-    PF_CUDA(gemm_linear(d, N1, (int)g.R, {w.dHb, d, 1}, {sv.Xp, N1, 1}, e, cs));
+    PF_CUDA(gemm_linear(d, N1, (int)g.R, {w.dHb, d, 1}, {sv.Xp, N1, 1}, with_sk(e, w.sk, w.skb), cs));
   }
   {
     EpiDX2DArgs e{w.dXd, dX, d, patch, gh, gw, (int)g.m};
@@ -463,15 +501,17 @@ size_t proxy_layer_workspace_size(const pf_layer_desc* desc, int for_backward) {
     carve_f32(c, *desc, g);
   } else if (desc->mode == PF_BIDIR_2D) {
     if (for_backward) {
-      carve_bwd_2d(c, g);
+      carve_bwd_2d(c, *desc, g);
     } else {
       c.take<float>(g.R * g.d);  // H when H_out is NULL
+      c.take<float>(splitk_need(*desc, g, false) / sizeof(float));
       carve_saved_2d(c, g);
     }
   } else if (for_backward) {
     carve_bwd(c, *desc, g);
   } else {
     if (g.ragged) c.take<bf16>(g.B * g.Lp * g.d);
+    c.take<float>(splitk_need(*desc, g, false) / sizeof(float));
     carve_saved(c, *desc, g);  // used when the forward is given saved == NULL
   }
   return ((c.off + 255) & ~size_t(255)) + 256;
@@ -501,6 +541,8 @@ pf_status proxy_layer_fwd(const pf_layer_desc* desc, const pf_layer_params* prm,
                         static_cast<cudaStream_t>(stream));
   Carve wc(ws);
   bf16* Xpad = g.ragged ? wc.take<bf16>(g.B * g.Lp * g.d) : nullptr;
+  const size_t skb = splitk_need(s, g, false);
+  float* sk = wc.take<float>(skb / sizeof(float));
   Carve sc(saved);
   Saved sv = saved ? carve_saved(sc, s, g) : carve_saved(wc, s, g);
   if (wc.off > ws_bytes)
@@ -530,14 +572,14 @@ pf_status proxy_layer_fwd(const pf_layer_desc* desc, const pf_layer_params* prm,
       e.ld_bf16 = d;
       set_gemm_tag("compress_c1", (double)g.R * d * 6.0);
       PF_CUDA(gemm_linear((int)g.R, d, (int)g.N1, {Xsrc, g.N1, 0},
-                          {static_cast<const bf16*>(prm->W_c1), g.N1, 0}, e, cs));
+                          {static_cast<const bf16*>(prm->W_c1), g.N1, 0}, with_sk(e, sk, skb), cs));
     } else {
       e.bias = prm->b_c1;
       e.out_bf16 = sv.Y;
       e.ld_bf16 = d;
       set_gemm_tag("compress_c1", (double)g.rows1 * d * 2.0);
       PF_CUDA(gemm_linear((int)g.rows1, d, (int)g.N1, {Xsrc, g.N1, 0},
-                          {static_cast<const bf16*>(prm->W_c1), g.N1, 0}, e, cs));
+                          {static_cast<const bf16*>(prm->W_c1), g.N1, 0}, with_sk(e, sk, skb), cs));
       EpiLinearArgs e2;
       e2.bias = prm->b_c2;
       e2.addend = H_in;
@@ -548,7 +590,7 @@ pf_status proxy_layer_fwd(const pf_layer_desc* desc, const pf_layer_params* prm,
       e2.ld_bf16 = d;
       set_gemm_tag("compress_c2", (double)g.R * d * 10.0);
       PF_CUDA(gemm_linear((int)g.R, d, (int)(g.k2 * d), {sv.Y, g.k2 * d, 0},
-                          {static_cast<const bf16*>(prm->W_c2), g.k2 * d, 0}, e2, cs));
+                          {static_cast<const bf16*>(prm->W_c2), g.k2 * d, 0}, with_sk(e2, sk, skb), cs));
     }
   }
   // a4: proxy attention (Eq. proxy-attn)
@@ -558,14 +600,13 @@ pf_status proxy_layer_fwd(const pf_layer_desc* desc, const pf_layer_params* prm,
     e.ld_bf16 = 3 * d;
     set_gemm_tag("proxy_qkv", (double)g.R * 3 * d * 2.0);
     PF_CUDA(gemm_linear((int)g.R, 3 * d, d, {sv.Hb, d, 0},
-                        {static_cast<const bf16*>(prm->W_qkv), d, 0}, e, cs));
+                        {static_cast<const bf16*>(prm->W_qkv), d, 0}, with_sk(e, sk, skb), cs));
     PF_CUDA(attn_fwd(sv.QKV, sv.Aatt, sv.LSE, (int)g.B, (int)g.m, d, (int)g.nh, g.causal, cs));
     EpiLinearArgs eo;
     eo.out_bf16 = sv.Hbar;
     eo.ld_bf16 = d;
     set_gemm_tag("proxy_o", (double)g.R * d * 2.0);
-    PF_CUDA(gemm_linear((int)g.R, d, d, {sv.Aatt, d, 0}, {static_cast<const bf16*>(prm->W_o), d, 0},
-                        eo, cs));
+    PF_CUDA(gemm_linear((int)g.R, d, d, {sv.Aatt, d, 0}, {static_cast<const bf16*>(prm->W_o), d, 0}, with_sk(eo, sk, skb), cs));
   }
   // a5 + a6: decompression (Eq. decompress-linear / factor-dec), routing and
   // injection (Eq. inj-gate / inj-add), fused into the last level's GEMM
@@ -577,7 +618,7 @@ pf_status proxy_layer_fwd(const pf_layer_desc* desc, const pf_layer_params* prm,
     e.ld_bf16 = g.k2 * d;
     set_gemm_tag("decompress_d2", (double)g.R * g.k2 * d * 2.0);
     PF_CUDA(gemm_linear((int)g.R, (int)(g.k2 * d), d, {sv.Hbar, d, 0},
-                        {static_cast<const bf16*>(prm->W_d2), d, 0}, e, cs));
+                        {static_cast<const bf16*>(prm->W_d2), d, 0}, with_sk(e, sk, skb), cs));
     Zsrc = sv.Z;
   }
   {
@@ -661,14 +702,14 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
     e.out_f32 = grads->W_d1;
     e.ld_f32 = d;
     set_gemm_tag("bwd_dW_d1", (double)N1 * d * 4.0);
-    PF_CUDA(gemm_linear(N1, d, (int)g.rows1, {w.dD, N1, 1}, {Zsrc, d, 1}, e, cs));
+    PF_CUDA(gemm_linear(N1, d, (int)g.rows1, {w.dD, N1, 1}, {Zsrc, d, 1}, with_sk(e, w.sk, w.skb), cs));
   }
   {
     EpiLinearArgs e;
     e.out_bf16 = s.levels == 2 ? w.dZ : w.dHbar;
     e.ld_bf16 = d;
     set_gemm_tag("bwd_dZ", (double)g.rows1 * d * 2.0);
-    PF_CUDA(gemm_linear((int)g.rows1, d, N1, {w.dD, N1, 0}, {W_d1, d, 1}, e, cs));
+    PF_CUDA(gemm_linear((int)g.rows1, d, N1, {w.dD, N1, 0}, {W_d1, d, 1}, with_sk(e, w.sk, w.skb), cs));
   }
   if (s.levels == 2) {
     const int n2 = (int)(g.k2 * d);
@@ -678,13 +719,13 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
       e.out_f32 = grads->W_d2;
       e.ld_f32 = d;
       set_gemm_tag("bwd_dW_d2", (double)n2 * d * 4.0);
-      PF_CUDA(gemm_linear(n2, d, (int)g.R, {w.dZ, n2, 1}, {sv.Hbar, d, 1}, e, cs));
+      PF_CUDA(gemm_linear(n2, d, (int)g.R, {w.dZ, n2, 1}, {sv.Hbar, d, 1}, with_sk(e, w.sk, w.skb), cs));
     }
     EpiLinearArgs e;
     e.out_bf16 = w.dHbar;
     e.ld_bf16 = d;
     set_gemm_tag("bwd_dHbar", (double)g.R * d * 2.0);
-    PF_CUDA(gemm_linear((int)g.R, d, n2, {w.dZ, n2, 0}, {W_d2, d, 1}, e, cs));
+    PF_CUDA(gemm_linear((int)g.R, d, n2, {w.dZ, n2, 0}, {W_d2, d, 1}, with_sk(e, w.sk, w.skb), cs));
   }
   // attention output projection and attention
   if (grads->W_o) {
@@ -692,14 +733,14 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
     e.out_f32 = grads->W_o;
     e.ld_f32 = d;
     set_gemm_tag("bwd_dW_o", (double)d * d * 4.0);
-    PF_CUDA(gemm_linear(d, d, (int)g.R, {w.dHbar, d, 1}, {sv.Aatt, d, 1}, e, cs));
+    PF_CUDA(gemm_linear(d, d, (int)g.R, {w.dHbar, d, 1}, {sv.Aatt, d, 1}, with_sk(e, w.sk, w.skb), cs));
   }
   {
     EpiLinearArgs e;
     e.out_bf16 = w.dA;
     e.ld_bf16 = d;
     set_gemm_tag("bwd_dA", (double)g.R * d * 2.0);
-    PF_CUDA(gemm_linear((int)g.R, d, d, {w.dHbar, d, 0}, {W_o, d, 1}, e, cs));
+    PF_CUDA(gemm_linear((int)g.R, d, d, {w.dHbar, d, 0}, {W_o, d, 1}, with_sk(e, w.sk, w.skb), cs));
   }
   PF_CUDA(attn_bwd(sv.QKV, sv.Aatt, w.dA, sv.LSE, w.Di, w.dQKV, (int)g.B, (int)g.m, d, (int)g.nh,
                    g.causal, cs));
@@ -708,7 +749,7 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
     e.out_f32 = grads->W_qkv;
     e.ld_f32 = d;
     set_gemm_tag("bwd_dW_qkv", (double)3 * d * d * 4.0);
-    PF_CUDA(gemm_linear(3 * d, d, (int)g.R, {w.dQKV, 3 * d, 1}, {sv.Hb, d, 1}, e, cs));
+    PF_CUDA(gemm_linear(3 * d, d, (int)g.R, {w.dQKV, 3 * d, 1}, {sv.Hb, d, 1}, with_sk(e, w.sk, w.skb), cs));
   }
   float* dHf = dH_in ? dH_in : w.dHf;
   {
@@ -720,7 +761,7 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
     e.out_bf16 = w.dHb;
     e.ld_bf16 = d;
     set_gemm_tag("bwd_dH", (double)g.R * d * 10.0);
-    PF_CUDA(gemm_linear((int)g.R, d, 3 * d, {w.dQKV, 3 * d, 0}, {W_qkv, d, 1}, e, cs));
+    PF_CUDA(gemm_linear((int)g.R, d, 3 * d, {w.dQKV, 3 * d, 0}, {W_qkv, d, 1}, with_sk(e, w.sk, w.skb), cs));
   }
   // compression (H = H_in + C, so dC = dH)
   const bf16* dYsrc = w.dHb;
@@ -732,13 +773,13 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
       e.out_f32 = grads->W_c2;
       e.ld_f32 = n2;
       set_gemm_tag("bwd_dW_c2", (double)d * n2 * 4.0);
-      PF_CUDA(gemm_linear(d, n2, (int)g.R, {w.dHb, d, 1}, {sv.Y, n2, 1}, e, cs));
+      PF_CUDA(gemm_linear(d, n2, (int)g.R, {w.dHb, d, 1}, {sv.Y, n2, 1}, with_sk(e, w.sk, w.skb), cs));
     }
     EpiLinearArgs e;
     e.out_bf16 = w.dY;
     e.ld_bf16 = n2;
     set_gemm_tag("bwd_dY", (double)g.R * n2 * 2.0);
-    PF_CUDA(gemm_linear((int)g.R, n2, d, {w.dHb, d, 0}, {W_c2, n2, 1}, e, cs));
+    PF_CUDA(gemm_linear((int)g.R, n2, d, {w.dHb, d, 0}, {W_c2, n2, 1}, with_sk(e, w.sk, w.skb), cs));
     if (grads->b_c1) PF_CUDA(colsum_bf16(w.dY, g.rows1, d, grads->b_c1, w.part, cs));
     dYsrc = w.dY;
   } else if (grads->b_c1) {
@@ -749,7 +790,7 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
     e.out_f32 = grads->W_c1;
     e.ld_f32 = N1;
     set_gemm_tag("bwd_dW_c1", (double)d * N1 * 4.0);
-    PF_CUDA(gemm_linear(d, N1, (int)g.rows1, {dYsrc, d, 1}, {Xsrc, N1, 1}, e, cs));
+    PF_CUDA(gemm_linear(d, N1, (int)g.rows1, {dYsrc, d, 1}, {Xsrc, N1, 1}, with_sk(e, w.sk, w.skb), cs));
   }
   {
     EpiDXArgs e{dXd, dXb, d, (int)g.k1, (int)g.k2, (int)g.m, (int)g.L};

@@ -38,12 +38,27 @@ __device__ __forceinline__ void store4_bf16(bf16* p, const float* v) {
   *reinterpret_cast<uint2*>(p) = make_uint2(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]));
 }
 
-// Each thread owns 4 consecutive columns and walks a chunk of rows, INJ_U
-// rows at a time with their loads issued together.
-constexpr int INJ_COLS = 4;
+// Each thread owns 8 consecutive columns (16-byte vectors) and walks a
+// contiguous chunk of rows, INJ_U rows at a time with their loads issued
+// together (kept packed until used); the row -> (sequence, proxy, group)
+// indices advance incrementally, without divisions.
+constexpr int INJ_COLS = 8;
 constexpr int INJ_U = 2;
 
-__global__ void __launch_bounds__(EW_THREADS, 3) inj_bwd_kernel(InjBwdArgs a, float* __restrict__ part,
+struct RowIdx {  // row r = (b*m + i)*k2 + grp
+  int b, i, grp;
+  __device__ __forceinline__ void next(int k2, int m) {
+    if (++grp == k2) {
+      grp = 0;
+      if (++i == m) {
+        i = 0;
+        ++b;
+      }
+    }
+  }
+};
+
+__global__ void __launch_bounds__(EW_THREADS, 2) inj_bwd_kernel(InjBwdArgs a, float* __restrict__ part,
                                                                 long M, int N, long rows_per_chunk) {
   const int col = (blockIdx.x * EW_THREADS + threadIdx.x) * INJ_COLS;
   if (col >= N) return;
@@ -56,77 +71,99 @@ __global__ void __launch_bounds__(EW_THREADS, 3) inj_bwd_kernel(InjBwdArgs a, fl
   const long r1 = min(M, r0 + rows_per_chunk);
   const int P = a.k1 * a.k2;
   const int ch = col % a.d, tq = col / a.d;
-  float wx[INJ_COLS], wd[INJ_COLS], bg[INJ_COLS];
+  float wx[8], wd[8], bg[8];
 #pragma unroll
-  for (int j = 0; j < INJ_COLS; ++j) {
+  for (int j = 0; j < 8; ++j) {
     wx[j] = a.gated ? a.w_x[ch + j] : 0.f;
     wd[j] = a.gated ? a.w_dlt[ch + j] : 0.f;
     bg[j] = a.gated ? a.b_g[ch + j] : 0.f;
   }
-  float acc[4][INJ_COLS] = {};
+  RowIdx ix;
+  {
+    const long prox = r0 / a.k2;
+    ix.grp = (int)(r0 % a.k2);
+    ix.b = (int)(prox / a.m);
+    ix.i = (int)(prox % a.m);
+  }
+  float acc[4][8] = {};
   for (long rb = r0; rb < r1; rb += INJ_U) {
+    uint4 gv[INJ_U], xv[INJ_U], dv[INJ_U];
     long offx[INJ_U];
     bool valid[INJ_U];
-    float g[INJ_U][INJ_COLS], x[INJ_U][INJ_COLS], Dv[INJ_U][INJ_COLS];
 #pragma unroll
     for (int u = 0; u < INJ_U; ++u) {
       const long r = rb + u;
-      valid[u] = false;
-      offx[u] = 0;
-      if (r < r1) {
-        const int grp = (int)(r % a.k2);
-        const long prox = r / a.k2;
-        const int b = (int)(prox / a.m), i = (int)(prox % a.m);
-        const int it = i + a.shift;
-        const long tok = (long)it * P + (long)grp * a.k1 + tq;
-        if (it < a.m && tok < a.L) {
-          valid[u] = true;
-          const long off = ((long)b * a.L + tok) * a.d + ch;
-          offx[u] = ((long)b * a.Ldx + tok) * a.d + ch;
-          load4_bf16(G + off, g[u]);
-          load4_bf16(X + off, x[u]);
-          load4_bf16(D + r * N + col, Dv[u]);
-        }
+      const int it = ix.i + a.shift;
+      const long tok = (long)it * P + (long)ix.grp * a.k1 + tq;
+      valid[u] = r < r1 && it < a.m && tok < a.L;
+      offx[u] = ((long)ix.b * a.Ldx + tok) * a.d + ch;
+      if (valid[u]) {
+        const long off = ((long)ix.b * a.L + tok) * a.d + ch;
+        gv[u] = *reinterpret_cast<const uint4*>(G + off);
+        xv[u] = *reinterpret_cast<const uint4*>(X + off);
+        dv[u] = *reinterpret_cast<const uint4*>(D + r * N + col);
       }
+      ix.next(a.k2, a.m);
     }
 #pragma unroll
     for (int u = 0; u < INJ_U; ++u) {
       const long r = rb + u;
       if (r >= r1) break;
-      float dd[INJ_COLS];
+      float dd[8];
       if (valid[u]) {
-        float dx[INJ_COLS];
+        float g[8], x[8], Dv[8], dx[8];
+        const uint32_t* pg = &gv[u].x;
+        const uint32_t* px = &xv[u].x;
+        const uint32_t* pd = &dv[u].x;
 #pragma unroll
-        for (int j = 0; j < INJ_COLS; ++j) {
+        for (int q = 0; q < 4; ++q) {
+          const float2 a2 = unpack_bf16(pg[q]), b2 = unpack_bf16(px[q]), c2 = unpack_bf16(pd[q]);
+          g[2 * q] = a2.x; g[2 * q + 1] = a2.y;
+          x[2 * q] = b2.x; x[2 * q + 1] = b2.y;
+          Dv[2 * q] = c2.x; Dv[2 * q + 1] = c2.y;
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
           if (a.gated) {
-            const float sg = sigmoidf_(fmaf(wx[j], x[u][j], fmaf(wd[j], Dv[u][j], bg[j])));
-            const float ds = g[u][j] * Dv[u][j] * sg * (1.f - sg);
-            dx[j] = fmaf(ds, wx[j], g[u][j]);
-            dd[j] = fmaf(g[u][j], sg, ds * wd[j]);
-            acc[1][j] += ds * x[u][j];
-            acc[2][j] += ds * Dv[u][j];
+            const float sg = sigmoidf_(fmaf(wx[j], x[j], fmaf(wd[j], Dv[j], bg[j])));
+            const float ds = g[j] * Dv[j] * sg * (1.f - sg);
+            dx[j] = fmaf(ds, wx[j], g[j]);
+            dd[j] = fmaf(g[j], sg, ds * wd[j]);
+            acc[1][j] = fmaf(ds, x[j], acc[1][j]);
+            acc[2][j] = fmaf(ds, Dv[j], acc[2][j]);
             acc[3][j] += ds;
           } else {
-            dx[j] = g[u][j];
-            dd[j] = g[u][j];
+            dx[j] = g[j];
+            dd[j] = g[j];
           }
         }
-        store4_bf16(dX + offx[u], dx);
+        store8_bf16(dX + offx[u], dx);
       } else {
 #pragma unroll
-        for (int j = 0; j < INJ_COLS; ++j) dd[j] = 0.f;
+        for (int j = 0; j < 8; ++j) dd[j] = 0.f;
       }
       // round dD once; the column sum uses the same rounded values the
       // downstream GEMMs see.
-      store4_bf16(dD + r * N + col, dd);
+      uint4 o;
+      o.x = pack_bf16(dd[0], dd[1]);
+      o.y = pack_bf16(dd[2], dd[3]);
+      o.z = pack_bf16(dd[4], dd[5]);
+      o.w = pack_bf16(dd[6], dd[7]);
+      *reinterpret_cast<uint4*>(dD + r * N + col) = o;
+      const uint32_t* po = &o.x;
 #pragma unroll
-      for (int j = 0; j < INJ_COLS; ++j) acc[0][j] += __bfloat162float(__float2bfloat16(dd[j]));
+      for (int q = 0; q < 4; ++q) {
+        const float2 f = unpack_bf16(po[q]);
+        acc[0][2 * q] += f.x;
+        acc[0][2 * q + 1] += f.y;
+      }
     }
   }
 #pragma unroll
   for (int q = 0; q < 4; ++q) {
     float* p = part + ((long)blockIdx.y * 4 + q) * N + col;
     *reinterpret_cast<float4*>(p) = make_float4(acc[q][0], acc[q][1], acc[q][2], acc[q][3]);
+    *reinterpret_cast<float4*>(p + 4) = make_float4(acc[q][4], acc[q][5], acc[q][6], acc[q][7]);
   }
 }
 
@@ -252,7 +289,7 @@ cudaError_t pad_rows(const bf16* src, bf16* dst, int B, long L, long Lp, int d, 
   return cudaGetLastError();
 }
 
-int inj_bwd_chunks(long M, int N) { return chunks_for(M, 2 * N); }
+int inj_bwd_chunks(long M, int N) { return chunks_for(M, N); }
 
 int take_dev_error_elementwise() { return take_dev_error_tu(); }
 

@@ -60,26 +60,26 @@ bool make_operand_map(CUtensorMap* m, const Operand& op, int rows, int K) {
 
 template <int BN, bool AMN, bool BMN, class Epi>
 cudaError_t launch(int M, int N, int K, const CUtensorMap& ta, const CUtensorMap& tb,
-                   const CUtensorMap& tx, const Epi& epi, cudaStream_t st) {
+                   const CUtensorMap& tx, const Epi& epi, cudaStream_t st, int splits) {
   auto kern = gemm_tc_kernel<BN, AMN, BMN, Epi>;
   constexpr int XCOLS = Epi::kXTile ? (Epi::kPaired ? BN / 2 : BN) : 0;
   constexpr int smem = GemmCfg<BN, XCOLS>::SMEM_BYTES;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
-  const long tiles = (long)((N + BN - 1) / BN) * ((M + GEMM_BM - 1) / GEMM_BM);
+  const long tiles = (long)((N + BN - 1) / BN) * ((M + GEMM_BM - 1) / GEMM_BM) * splits;
   const int grid = (int)std::min<long>(tiles, num_sms());
-  kern<<<grid, GEMM_THREADS, smem, st>>>(ta, tb, tx, M, N, K, epi);
+  kern<<<grid, GEMM_THREADS, smem, st>>>(ta, tb, tx, M, N, K, splits, epi);
   return cudaGetLastError();
 }
 
 template <int BN, class Epi>
 cudaError_t launch_majors(int M, int N, int K, const Operand& A, const Operand& B,
                           const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tx,
-                          const Epi& epi, cudaStream_t st) {
-  if (!A.mn && !B.mn) return launch<BN, false, false>(M, N, K, ta, tb, tx, epi, st);
-  if (!A.mn && B.mn) return launch<BN, false, true>(M, N, K, ta, tb, tx, epi, st);
-  if (A.mn && B.mn) return launch<BN, true, true>(M, N, K, ta, tb, tx, epi, st);
-  return launch<BN, true, false>(M, N, K, ta, tb, tx, epi, st);
+                          const Epi& epi, cudaStream_t st, int splits = 1) {
+  if (!A.mn && !B.mn) return launch<BN, false, false>(M, N, K, ta, tb, tx, epi, st, splits);
+  if (!A.mn && B.mn) return launch<BN, false, true>(M, N, K, ta, tb, tx, epi, st, splits);
+  if (A.mn && B.mn) return launch<BN, true, true>(M, N, K, ta, tb, tx, epi, st, splits);
+  return launch<BN, true, false>(M, N, K, ta, tb, tx, epi, st, splits);
 }
 
 bool operand_ok(const Operand& op) {
@@ -113,10 +113,80 @@ cudaError_t gemm_dispatch(int M, int N, int K, Operand A, Operand B, const Epi& 
   return launch_majors<128>(M, N, K, A, B, ta, tb, tx, epi, st);
 }
 
+// out = sum_s part[s] (+ bias) (+ addend) -> fp32 and/or bf16, 4 columns per thread.
+__global__ void splitk_reduce_kernel(const float* __restrict__ part, int S, int M, int N,
+                                     EpiLinearArgs e) {
+  const long i = ((long)blockIdx.x * blockDim.x + threadIdx.x) * 4;
+  if (i >= (long)M * N) return;
+  const long row = i / N;
+  const int col = (int)(i % N);
+  float4 v = *reinterpret_cast<const float4*>(part + i);
+  for (int s = 1; s < S; ++s) {
+    const float4 w = *reinterpret_cast<const float4*>(part + (long)s * M * N + i);
+    v.x += w.x; v.y += w.y; v.z += w.z; v.w += w.w;
+  }
+  if (e.bias) {
+    const float4 b = *reinterpret_cast<const float4*>(e.bias + col);
+    v.x += b.x; v.y += b.y; v.z += b.z; v.w += b.w;
+  }
+  if (e.addend) {
+    const float4 a = *reinterpret_cast<const float4*>(e.addend + row * e.ld_add + col);
+    v.x += a.x; v.y += a.y; v.z += a.z; v.w += a.w;
+  }
+  if (e.out_f32) *reinterpret_cast<float4*>(e.out_f32 + row * e.ld_f32 + col) = v;
+  if (e.out_bf16)
+    *reinterpret_cast<uint2*>(e.out_bf16 + row * e.ld_bf16 + col) =
+        make_uint2(pack_bf16(v.x, v.y), pack_bf16(v.z, v.w));
+}
+
 }  // namespace
+
+int splitk_factor(int M, int N, int K) {
+  constexpr int kSms = 152;  // planning target (GB300); fixed so sizes are device-independent
+  const long tiles = (long)((N + 127) / 128) * ((M + GEMM_BM - 1) / GEMM_BM);
+  const int num_k = (K + GEMM_BK - 1) / GEMM_BK;
+  if (tiles >= kSms || num_k < 32) return 1;
+  int best = 1;
+  double best_eff = (double)tiles / kSms;
+  for (int S = 2; S <= 8 && num_k / S >= 16; ++S) {
+    const long t = tiles * S;
+    const double eff = (double)t / (((t + kSms - 1) / kSms) * kSms);
+    if (eff > best_eff + 1e-9) {
+      best = S;
+      best_eff = eff;
+    }
+  }
+  return best;
+}
+
+size_t splitk_scratch_bytes(int M, int N, int K) {
+  const int S = splitk_factor(M, N, K);
+  return S > 1 ? (size_t)S * M * N * sizeof(float) : 0;
+}
 
 cudaError_t gemm_linear(int M, int N, int K, Operand A, Operand B, const EpiLinearArgs& e,
                         cudaStream_t st) {
+  const int S = splitk_factor(M, N, K);
+  if (S > 1 && e.splitk_scratch && (size_t)S * M * N * sizeof(float) <= e.splitk_bytes &&
+      N % 4 == 0) {
+    // deterministic split-K: raw partials, then one reduce applying the epilogue
+    if (M <= 0 || N % 32 != 0 || !operand_ok(A) || !operand_ok(B)) return cudaErrorInvalidValue;
+    CUtensorMap ta, tb;
+    if (!make_operand_map(&ta, A, M, K) || !make_operand_map(&tb, B, N, K))
+      return cudaErrorInvalidValue;
+    EpiPartial epi{{}, N, e.splitk_scratch};
+    {
+      LaunchTimer lt(gemm_tag_label(), st, 2.0 * M * N * (double)K,
+                     2.0 * ((double)M * K + (double)N * K) + 4.0 * S * M * N);
+      cudaError_t err = launch_majors<128>(M, N, K, A, B, ta, tb, ta, epi, st, S);
+      if (err != cudaSuccess) return err;
+    }
+    LaunchTimer lt("splitk_reduce", st, (double)S * M * N, 4.0 * (S + 1.0) * M * N);
+    const long quads = (long)M * N / 4;
+    splitk_reduce_kernel<<<(unsigned)((quads + 255) / 256), 256, 0, st>>>(e.splitk_scratch, S, M,
+                                                                          N, e);
+    return cudaGetLastError();
+  }
   EpiLinear epi{{}, M, N, e.bias, e.addend, e.ld_add, e.out_f32, e.ld_f32, e.out_bf16, e.ld_bf16};
   return gemm_dispatch(M, N, K, A, B, epi, nullptr, 0, st);
 }

@@ -75,7 +75,8 @@ __device__ __forceinline__ void xtile_load8(const uint8_t* xt, int r, int c, flo
 template <int BN, bool A_MN, bool B_MN, class Epi>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const __grid_constant__ CUtensorMap tmX, int M, int N, int K, Epi epi) {
+                   const __grid_constant__ CUtensorMap tmX, int M, int N, int K, int splits,
+                   Epi epi) {
   constexpr int XCOLS = Epi::kXTile ? (Epi::kPaired ? BN / 2 : BN) : 0;
   using Cfg = GemmCfg<BN, XCOLS>;
   constexpr int STAGES = Cfg::STAGES;
@@ -90,8 +91,15 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int num_n = (N + BN - 1) / BN;
-  const int tiles = ((M + GEMM_BM - 1) / GEMM_BM) * num_n;
+  const int mn_tiles = ((M + GEMM_BM - 1) / GEMM_BM) * num_n;
+  const int tiles = mn_tiles * splits;
   const int num_k = (K + GEMM_BK - 1) / GEMM_BK;
+  const int kps = (num_k + splits - 1) / splits;  // K tiles per split
+  // tile t -> split t / mn_tiles (slowest), then M, then N (fastest)
+#define PF_TILE_DECODE(t)                                   \
+  const int sp = (t) / mn_tiles, rem = (t) % mn_tiles;      \
+  const int m0 = (rem / num_n) * GEMM_BM, n0 = (rem % num_n) * BN; \
+  const int kb = sp * kps, ke = min(num_k, kb + kps);
   const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + STAGES);
   const uint32_t tfull0 = smem_u32(bars + 2 * STAGES), tempty0 = tfull0 + 16;
   const uint32_t xfull = tfull0 + 32, done = tfull0 + 40;
@@ -129,8 +137,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     uint32_t it = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
-      const int m0 = (tile / num_n) * GEMM_BM, n0 = (tile % num_n) * BN;
-      for (int kt = 0; kt < num_k; ++kt, ++it) {
+      PF_TILE_DECODE(tile)
+      (void)sp;
+      for (int kt = kb; kt < ke; ++kt, ++it) {
         const int s = it % STAGES;
         const uint32_t ph = (it / STAGES) & 1;
         if (!mbar_wait(empty0 + 8 * s, ph ^ 1)) {
@@ -169,7 +178,11 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       if (!mbar_wait(tempty0 + 8 * buf, (use & 1) ^ 1)) break;
       tc_fence_after();
       const uint32_t d_tmem = tmem + buf * BN;
-      for (int kt = 0; kt < num_k; ++kt, ++it) {
+      PF_TILE_DECODE(tile)
+      (void)sp;
+      (void)m0;
+      (void)n0;
+      for (int kt = kb; kt < ke; ++kt, ++it) {
         const int s = it % STAGES;
         const uint32_t ph = (it / STAGES) & 1;
         if (!mbar_wait(full0 + 8 * s, ph)) {
@@ -189,7 +202,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                                    : smem_desc_sw128(a_base + kk * 32, 16, 1024);
           const uint64_t bd = B_MN ? smem_desc_sw128(b_base + kk * 2048, 8192, 1024)
                                    : smem_desc_sw128(b_base + kk * 32, 16, 1024);
-          tc_mma_f16(d_tmem, ad, bd, idesc, (kt | kk) != 0 ? 1u : 0u);
+          tc_mma_f16(d_tmem, ad, bd, idesc, (kt != kb || kk != 0) ? 1u : 0u);
         }
         tc_commit(empty0 + 8 * s);
       }
@@ -204,7 +217,8 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     const int c_begin = ((warp - 2) >> 2) * (BN / 2);     // this warp's column half
     uint32_t lt = 0;
     for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++lt) {
-      const int m0 = (tile / num_n) * GEMM_BM, n0 = (tile % num_n) * BN;
+      PF_TILE_DECODE(tile)
+      const bool no_k = ke <= kb;
       const uint32_t buf = lt & 1, use = lt >> 1;
       if (Epi::kXTile && et == 0) {
         mbar_arrive_expect_tx(xfull, Cfg::X_BYTES);
@@ -222,7 +236,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         x_pending = false;
       }
       const int rl = q * 32 + lane;
-      const typename Epi::Row ri = epi.row_info(m0 + rl, n0);
+      // split-K partial epilogues address row (split * M + row); -1 = out of range
+      const int erow = Epi::kSplitRows ? (m0 + rl < M ? sp * M + m0 + rl : -1) : m0 + rl;
+      const typename Epi::Row ri = epi.row_info(erow, n0);
       const uint32_t trow = tmem + buf * BN + ((uint32_t)(q * 32) << 16);
       if constexpr (Epi::kPaired) {
         // columns c and c + BN/2 belong together (e.g. s and t of one channel)
@@ -231,22 +247,22 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           float v[32], w[32];
           tmem_ld32(trow + (uint32_t)c, v);
           tmem_ld32(trow + (uint32_t)(c + BN / 2), w);
-          if (num_k == 0) {
+          if (no_k) {
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = w[i] = 0.f;
           }
-          epi.apply_pair(ri, m0 + rl, n0, c, v, w, xtile, rl);
+          epi.apply_pair(ri, erow, n0, c, v, w, xtile, rl);
         }
       } else {
 #pragma unroll 1
         for (int c = c_begin; c < c_begin + BN / 2; c += 32) {
           float v[32];
           tmem_ld32(trow + (uint32_t)c, v);
-          if (num_k == 0) {
+          if (no_k) {
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = 0.f;
           }
-          epi.apply(ri, m0 + rl, n0 + c, v, xtile, rl, c);
+          epi.apply(ri, erow, n0 + c, v, xtile, rl, c);
         }
       }
       tc_fence_before();
@@ -290,6 +306,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
 struct EpiBase {
   static constexpr bool kXTile = false;
   static constexpr bool kPaired = false;
+  static constexpr bool kSplitRows = false;
   __device__ __forceinline__ int x_row(int m0) const { return m0; }
   __device__ __forceinline__ int x_col(int n0, int j) const { return n0 + 64 * j; }
   __device__ __forceinline__ int b_row(int n0, int j) const { return n0 + 128 * j; }
@@ -598,6 +615,28 @@ struct EpiDX2D : EpiBase {
       for (int j = 0; j < 8; ++j) x[j] += v[i8 + j];
       store8_bf16(o + i8, x);
     }
+  }
+};
+
+// Split-K partial: raw fp32 accumulator of split s written to
+// part[(s * M + row) * N + col]; a reduce kernel applies the linear epilogue.
+struct EpiPartial : EpiBase {
+  static constexpr bool kSplitRows = true;
+  struct Row {
+    long off;
+  };
+  int N;
+  float* part;
+  __device__ __forceinline__ Row row_info(int erow, int) const {
+    return Row{erow < 0 ? -1L : (long)erow * N};
+  }
+  __device__ __forceinline__ void apply(const Row& ri, int, int col, float* v, const uint8_t*, int,
+                                        int) const {
+    if (ri.off < 0 || col >= N) return;
+    float* o = part + ri.off + col;
+#pragma unroll
+    for (int i = 0; i < 32; i += 4)
+      *reinterpret_cast<float4*>(o + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
   }
 };
 

@@ -23,7 +23,15 @@ struct EpiLinearArgs {
   long ld_f32 = 0;
   bf16* out_bf16 = nullptr;
   long ld_bf16 = 0;
+  // optional scratch for deterministic split-K (used when the output tiles
+  // alone cannot fill the GPU and splitk_scratch_bytes() bytes are given)
+  float* splitk_scratch = nullptr;
+  size_t splitk_bytes = 0;
 };
+// Split-K factor chosen for an M x N x K linear GEMM (1: none) and the fp32
+// scratch it needs; independent of the device.
+int splitk_factor(int M, int N, int K);
+size_t splitk_scratch_bytes(int M, int N, int K);
 
 struct EpiInjectArgs {
   const float* bias;  // b_d1 [k1*d]
