@@ -210,8 +210,19 @@ Bwd2DWs carve_bwd_2d(Carve& c, const pf_layer_desc& s, const Dims& g) {
 
 // Workspace of the fp32 forward (all fp32).
 struct F32Ws {
-  float *Xpad, *Y, *H, *QKV, *A, *Hbar, *Z, *D;
+  float *Xpad, *Y, *H, *QKV, *A, *Hbar, *Z, *D, *sk;
+  size_t skb;
 };
+
+size_t splitk_f32_need(const pf_layer_desc& s, const Dims& g) {
+  const int d = (int)g.d, R = (int)g.R, r1 = (int)g.rows1, N1 = (int)g.N1, n2 = (int)(g.k2 * d);
+  const int shapes[][3] = {{s.levels == 1 ? R : r1, d, N1}, {R, d, n2},   {R, 3 * d, d},
+                           {R, d, d},                        {R, n2, d},   {r1, N1, d}};
+  size_t m = 0;
+  for (const auto& x : shapes)
+    m = std::max(m, (size_t)splitk_f32_factor(x[0], x[1], x[2]) * x[0] * x[1] * sizeof(float));
+  return m;
+}
 
 F32Ws carve_f32(Carve& c, const pf_layer_desc& s, const Dims& g) {
   F32Ws w{};
@@ -223,6 +234,8 @@ F32Ws carve_f32(Carve& c, const pf_layer_desc& s, const Dims& g) {
   w.Hbar = c.take<float>(g.R * g.d);
   if (s.levels == 2) w.Z = c.take<float>(g.R * g.k2 * g.d);
   w.D = c.take<float>(g.rows1 * g.N1);
+  w.skb = splitk_f32_need(s, g);
+  w.sk = c.take<float>(w.skb / sizeof(float));
   return w;
 }
 
@@ -287,28 +300,28 @@ pf_status layer_fwd_f32(const pf_layer_desc& s, const Dims& g, const pf_layer_pa
   const float* W_c1 = static_cast<const float*>(p.W_c1);
   float* H = H_out ? H_out : w.H;
   if (s.levels == 1) {
-    PF_CUDA(gemm_f32((int)g.R, d, N1, Xsrc, N1, W_c1, N1, H, d, p.b_c1, H_in, d, "compress_c1", cs));
+    PF_CUDA(gemm_f32((int)g.R, d, N1, Xsrc, N1, W_c1, N1, H, d, p.b_c1, H_in, d, "compress_c1", cs, w.sk, w.skb));
   } else {
     PF_CUDA(gemm_f32((int)g.rows1, d, N1, Xsrc, N1, W_c1, N1, w.Y, d, p.b_c1, nullptr, 0,
-                     "compress_c1", cs));
+                     "compress_c1", cs, w.sk, w.skb));
     const int n2 = (int)(g.k2 * d);
     PF_CUDA(gemm_f32((int)g.R, d, n2, w.Y, n2, static_cast<const float*>(p.W_c2), n2, H, d, p.b_c2,
-                     H_in, d, "compress_c2", cs));
+                     H_in, d, "compress_c2", cs, w.sk, w.skb));
   }
   PF_CUDA(gemm_f32((int)g.R, 3 * d, d, H, d, static_cast<const float*>(p.W_qkv), d, w.QKV, 3 * d,
-                   nullptr, nullptr, 0, "proxy_qkv", cs));
+                   nullptr, nullptr, 0, "proxy_qkv", cs, w.sk, w.skb));
   PF_CUDA(attn_f32(w.QKV, w.A, (int)g.B, (int)g.m, d, (int)g.nh, g.causal, cs));
   PF_CUDA(gemm_f32((int)g.R, d, d, w.A, d, static_cast<const float*>(p.W_o), d, w.Hbar, d, nullptr,
-                   nullptr, 0, "proxy_o", cs));
+                   nullptr, 0, "proxy_o", cs, w.sk, w.skb));
   const float* Zsrc = w.Hbar;
   if (s.levels == 2) {
     const int n2 = (int)(g.k2 * d);
     PF_CUDA(gemm_f32((int)g.R, n2, d, w.Hbar, d, static_cast<const float*>(p.W_d2), d, w.Z, n2,
-                     p.b_d2, nullptr, 0, "decompress_d2", cs));
+                     p.b_d2, nullptr, 0, "decompress_d2", cs, w.sk, w.skb));
     Zsrc = w.Z;
   }
   PF_CUDA(gemm_f32((int)g.rows1, N1, d, Zsrc, d, static_cast<const float*>(p.W_d1), d, w.D, N1,
-                   p.b_d1, nullptr, 0, "decompress_d1", cs));
+                   p.b_d1, nullptr, 0, "decompress_d1", cs, w.sk, w.skb));
   PF_CUDA(inject_f32(X, w.D, static_cast<float*>(X_out), p.w_x, p.w_dlt, p.b_g, (int)g.B, g.L, d,
                      (int)g.P, (int)g.k1, (int)g.k2, (int)g.m, g.causal ? 1 : 0,
                      s.inject == PF_INJ_GATED ? 1 : 0, cs));

@@ -100,7 +100,35 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
   }
 }
 
+// Wait used on an error path, after a wait ran out: lets copies that are still
+// in flight land before the CTA's shared memory goes away.  Bounded by its own
+// limit; it does not look at the error word.
+__device__ __forceinline__ void mbar_wait_drain(uint32_t bar, uint32_t parity) {
+  unsigned long long t0 = 0;
+  for (uint32_t it = 0;; ++it) {
+    if (mbar_try_wait(bar, parity)) return;
+    if ((it & 255u) == 255u) {
+      unsigned long long now = globaltimer();
+      if (t0 == 0)
+        t0 = now;
+      else if (now - t0 > kWaitLimitNs || it > 0x7fffffffu)
+        return;
+    }
+  }
+}
+
 // ----------------------------------------------------------------------- TMA
+// Contiguous global -> shared copy (no tensor map); dst, src and bytes must be
+// multiples of 16.  Completes `bytes` of transaction count on `bar`.
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes,
+                                          uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          dst),
+      "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(bar)
+      : "memory");
+}
+
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t bar,
                                             int c0, int c1) {
   asm volatile(
@@ -201,6 +229,19 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N, int a_mn, in
          | (1u << 10)                    // B format bf16
          | ((uint32_t)a_mn << 15) | ((uint32_t)b_mn << 16) |
          ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+// ------------------------------------------------------------ warp-level MMA
+// D += A B for one m16n8k16 tile (bf16 in, fp32 accumulate), register
+// fragments in the PTX layout: a = {(g, 2t..), (g+8, 2t..), (g, 2t+8..),
+// (g+8, 2t+8..)}, b = {(2t.., g), (2t+8.., g)}, c = {(g, 2t), (g, 2t+1),
+// (g+8, 2t), (g+8, 2t+1)} with g = lane / 4, t = lane % 4.
+__device__ __forceinline__ void mma16816(float* c, const uint32_t* a, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
 // ---------------------------------------------------------------- bf16 utils

@@ -3,6 +3,8 @@
 // online-softmax proxy attention with one warp per query, and the routing +
 // injection pass.  Used when the descriptor's dtype is PF_F32 (the tensor
 // cores have no fp32 path that meets fp32 accuracy).
+#include <algorithm>
+
 #include "kernels.h"
 
 namespace pf {
@@ -17,23 +19,28 @@ constexpr int FTHREADS = 256;
 
 // C[M, N] = A[M, K] B[N, K]^T (+ bias[n]) (+ addend[m, n]), all row-major fp32
 // with leading dimensions lda, ldb, ldc.  Each thread computes 4 x 4 outputs.
+// With gridDim.z = S > 1 each z-slice reduces K range [z*Kc, (z+1)*Kc) and
+// writes raw partials to C + z*M*ldc (bias / addend are then applied by
+// splitk_f32_reduce).
 __global__ void __launch_bounds__(FTHREADS) gemm_f32_kernel(const float* __restrict__ A, long lda,
                                                            const float* __restrict__ Bm, long ldb,
                                                            float* __restrict__ C, long ldc, int M,
-                                                           int N, int K,
+                                                           int N, int K, int Kc,
                                                            const float* __restrict__ bias,
                                                            const float* __restrict__ addend,
                                                            long ld_add) {
   __shared__ float As[FK][FT + 4], Bs[FK][FT + 4];
   const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
   const int m0 = blockIdx.y * FT, n0 = blockIdx.x * FT;
+  const int kbeg = blockIdx.z * Kc, kend = min(K, kbeg + Kc);
+  C += (long)blockIdx.z * M * ldc;
   float acc[4][4] = {};
-  for (int k0 = 0; k0 < K; k0 += FK) {
+  for (int k0 = kbeg; k0 < kend; k0 += FK) {
     for (int i = threadIdx.x; i < FT * FK; i += FTHREADS) {
       const int r = i / FK, kk = i % FK;
       const int gm = m0 + r, gn = n0 + r, gk = k0 + kk;
-      As[kk][r] = (gm < M && gk < K) ? A[(long)gm * lda + gk] : 0.f;
-      Bs[kk][r] = (gn < N && gk < K) ? Bm[(long)gn * ldb + gk] : 0.f;
+      As[kk][r] = (gm < M && gk < kend) ? A[(long)gm * lda + gk] : 0.f;
+      Bs[kk][r] = (gn < N && gk < kend) ? Bm[(long)gn * ldb + gk] : 0.f;
     }
     __syncthreads();
 #pragma unroll
@@ -135,16 +142,52 @@ __global__ void pad_f32_kernel(const float* __restrict__ src, float* __restrict_
   dst[e] = (r < L * d) ? src[b * L * d + r] : 0.f;
 }
 
+
+__global__ void splitk_f32_reduce(const float* __restrict__ part, int S, int M, int N,
+                                  float* __restrict__ C, long ldc, const float* __restrict__ bias,
+                                  const float* __restrict__ addend, long ld_add) {
+  const long i = (long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (long)M * N) return;
+  const long r = i / N;
+  const int c = (int)(i % N);
+  float v = 0.f;
+  for (int s = 0; s < S; ++s) v += part[((long)s * M + r) * N + c];
+  if (bias) v += bias[c];
+  if (addend) v += addend[r * ld_add + c];
+  C[r * ldc + c] = v;
+}
+
 }  // namespace
+
+int splitk_f32_factor(int M, int N, int K) {
+  const long tiles = (long)((M + FT - 1) / FT) * ((N + FT - 1) / FT);
+  if (tiles >= 304) return 1;
+  int S = (int)((304 + tiles - 1) / tiles);
+  S = std::min(S, std::max(1, K / 512));
+  return std::min(S, 64);
+}
 
 cudaError_t gemm_f32(int M, int N, int K, const float* A, long lda, const float* B, long ldb,
                      float* C, long ldc, const float* bias, const float* addend, long ld_add,
-                     const char* label, cudaStream_t st) {
-  dim3 grid((N + FT - 1) / FT, (M + FT - 1) / FT);
+                     const char* label, cudaStream_t st, float* scratch, size_t scratch_bytes) {
+  const int S = splitk_f32_factor(M, N, K);
   LaunchTimer lt(label, st, 2.0 * M * N * (double)K, 4.0 * ((double)M * K + (double)N * K + (double)M * N));
-  gemm_f32_kernel<<<grid, FTHREADS, 0, st>>>(A, lda, B, ldb, C, ldc, M, N, K, bias, addend, ld_add);
+  if (S > 1 && scratch && (size_t)S * M * N * sizeof(float) <= scratch_bytes) {
+    const int Kc = ((K + S - 1) / S + FK - 1) / FK * FK;
+    dim3 grid((N + FT - 1) / FT, (M + FT - 1) / FT, S);
+    gemm_f32_kernel<<<grid, FTHREADS, 0, st>>>(A, lda, B, ldb, scratch, N, M, N, K, Kc, nullptr,
+                                               nullptr, 0);
+    const long total = (long)M * N;
+    splitk_f32_reduce<<<(unsigned)((total + 255) / 256), 256, 0, st>>>(scratch, S, M, N, C, ldc, bias,
+                                                                      addend, ld_add);
+    return cudaGetLastError();
+  }
+  dim3 grid((N + FT - 1) / FT, (M + FT - 1) / FT, 1);
+  gemm_f32_kernel<<<grid, FTHREADS, 0, st>>>(A, lda, B, ldb, C, ldc, M, N, K, K, bias, addend,
+                                             ld_add);
   return cudaGetLastError();
 }
+
 
 cudaError_t attn_f32(const float* qkv, float* out, int B, int m, int d, int nh, bool causal,
                      cudaStream_t st) {

@@ -278,10 +278,10 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     // error path: let in-flight TMA copies and MMAs land before TMEM/smem go.
     if (warp == 0 && lane == 0) {
       for (uint32_t it = s_consumed; it < issued; ++it)
-        mbar_wait(full0 + 8 * (it % STAGES), (it / STAGES) & 1);
+        mbar_wait_drain(full0 + 8 * (it % STAGES), (it / STAGES) & 1);
     }
-    if (warp == 2 && lane == 0 && x_pending) mbar_wait(xfull, x_parity);
-    if (warp == 1 && lane == 0) mbar_wait(done, 0);
+    if (warp == 2 && lane == 0 && x_pending) mbar_wait_drain(xfull, x_parity);
+    if (warp == 1 && lane == 0) mbar_wait_drain(done, 0);
     __syncthreads();
   } else if (warp == 1 && lane == 0) {
     mbar_wait(done, 0);

@@ -119,9 +119,13 @@ cudaError_t temb_bwd(const float* dgb, const bf16* W_t2, const float* a1, const 
 
 // ---------------------------------------------------------- fp32 forward
 int take_dev_error_fp32();
+// fp32 GEMM C = A B^T (+ bias) (+ addend); split-K over `scratch` when the
+// output tiles cannot fill the GPU (splitk_f32_factor(M, N, K) * M * N floats).
+int splitk_f32_factor(int M, int N, int K);
 cudaError_t gemm_f32(int M, int N, int K, const float* A, long lda, const float* B, long ldb,
                      float* C, long ldc, const float* bias, const float* addend, long ld_add,
-                     const char* label, cudaStream_t st);
+                     const char* label, cudaStream_t st, float* scratch = nullptr,
+                     size_t scratch_bytes = 0);
 cudaError_t attn_f32(const float* qkv, float* out, int B, int m, int d, int nh, bool causal,
                      cudaStream_t st);
 cudaError_t inject_f32(const float* X, const float* D, float* Xo, const float* w_x,

@@ -51,9 +51,9 @@ def _check_step(spec, prm, st, cache):
     return ref_st
 
 
-@pytest.mark.parametrize("dh,batch", [(128, 3), (64, 10)])
-def test_decode_step_matches_oracle(dh, batch):
-    d = 256
+@pytest.mark.parametrize("d,dh,batch", [(256, 128, 3), (256, 64, 10), (192, 64, 2)])
+def test_decode_step_matches_oracle(d, dh, batch):
+    # d = 192: the split kernel's d/8 = 24 threads fill part of one warp
     spec = S.DecodeSpec(batch=batch, d=d, n_heads=d // dh, P=16, capacity=300)
     prm = S.make_decode_params(spec, 5)
     rng = np.random.default_rng(dh)
