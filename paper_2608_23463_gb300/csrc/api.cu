@@ -846,14 +846,20 @@ struct AppendWs {
   bf16* Y;
   float* Hf;
   bf16* Hb;
+  float* sk;  // split-K partials of the compression GEMMs (M = batch rows only)
+  size_t skb;
 };
 
 AppendWs carve_append(Carve& c, const pf_decode_desc& s) {
   AppendWs w{};
-  const long k2 = s.levels == 2 ? s.k2 : 1;
+  const long k1 = s.levels == 2 ? s.k1 : s.P, k2 = s.levels == 2 ? s.k2 : 1;
   if (s.levels == 2) w.Y = c.take<bf16>((size_t)s.batch * k2 * s.d);
   w.Hf = c.take<float>((size_t)s.batch * s.d);
   w.Hb = c.take<bf16>((size_t)s.batch * s.d);
+  w.skb = splitk_scratch_bytes((int)(s.batch * k2), s.d, (int)(k1 * s.d));
+  if (s.levels == 2)
+    w.skb = std::max(w.skb, splitk_scratch_bytes(s.batch, s.d, (int)(k2 * s.d)));
+  w.sk = c.take<float>(w.skb / sizeof(float));
   return w;
 }
 
@@ -953,7 +959,8 @@ pf_status proxy_kv_append(const pf_decode_desc* desc, const pf_append_params* pr
     e.ld_bf16 = d;
     set_gemm_tag("append_compress_c1", (double)B * d * 10.0);
     PF_CUDA(gemm_linear(B, d, (int)(k1 * d), {Xo, k1 * d, 0},
-                        {static_cast<const bf16*>(prm->W_c1), k1 * d, 0}, e, cs));
+                        {static_cast<const bf16*>(prm->W_c1), k1 * d, 0}, with_sk(e, w.sk, w.skb),
+                        cs));
   } else {
     EpiLinearArgs e;
     e.bias = prm->b_c1;
@@ -961,7 +968,8 @@ pf_status proxy_kv_append(const pf_decode_desc* desc, const pf_append_params* pr
     e.ld_bf16 = d;
     set_gemm_tag("append_compress_c1", (double)B * k2 * d * 2.0);
     PF_CUDA(gemm_linear((int)(B * k2), d, (int)(k1 * d), {Xo, k1 * d, 0},
-                        {static_cast<const bf16*>(prm->W_c1), k1 * d, 0}, e, cs));
+                        {static_cast<const bf16*>(prm->W_c1), k1 * d, 0}, with_sk(e, w.sk, w.skb),
+                        cs));
     EpiLinearArgs e2;
     e2.bias = prm->b_c2;
     e2.addend = H_in;
@@ -972,7 +980,8 @@ pf_status proxy_kv_append(const pf_decode_desc* desc, const pf_append_params* pr
     e2.ld_bf16 = d;
     set_gemm_tag("append_compress_c2", (double)B * d * 10.0);
     PF_CUDA(gemm_linear(B, d, (int)(k2 * d), {w.Y, k2 * d, 0},
-                        {static_cast<const bf16*>(prm->W_c2), k2 * d, 0}, e2, cs));
+                        {static_cast<const bf16*>(prm->W_c2), k2 * d, 0}, with_sk(e2, w.sk, w.skb),
+                        cs));
   }
   // the proxy's key and value rows into cache row n_proxy[b]
   {

@@ -63,7 +63,7 @@ cudaError_t launch(int M, int N, int K, const CUtensorMap& ta, const CUtensorMap
                    const CUtensorMap& tx, const Epi& epi, cudaStream_t st, int splits) {
   auto kern = gemm_tc_kernel<BN, AMN, BMN, Epi>;
   constexpr int XCOLS = Epi::kXTile ? (Epi::kPaired ? BN / 2 : BN) : 0;
-  constexpr int smem = GemmCfg<BN, XCOLS>::SMEM_BYTES;
+  constexpr int smem = GemmCfg<BN, XCOLS, Epi::kColPar>::SMEM_BYTES;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const long tiles = (long)((N + BN - 1) / BN) * ((M + GEMM_BM - 1) / GEMM_BM) * splits;
@@ -148,7 +148,7 @@ int splitk_factor(int M, int N, int K) {
   if (tiles >= kSms || num_k < 32) return 1;
   int best = 1;
   double best_eff = (double)tiles / kSms;
-  for (int S = 2; S <= 8 && num_k / S >= 16; ++S) {
+  for (int S = 2; S <= 16 && num_k / S >= 16; ++S) {
     const long t = tiles * S;
     const double eff = (double)t / (((t + kSms - 1) / kSms) * kSms);
     if (eff > best_eff + 1e-9) {

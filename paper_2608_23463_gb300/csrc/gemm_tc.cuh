@@ -36,7 +36,9 @@ constexpr int GEMM_EPI_WARPS = 8;  // two per TMEM lane quarter, each owning hal
 constexpr int GEMM_THREADS = 64 + 32 * GEMM_EPI_WARPS;
 
 // XCOLS: columns of the bf16 tile an epilogue prefetches (0: none).
-template <int BN, int XCOLS>
+// PAR: the epilogue stages one float4 of per-column parameters per output
+// column in shared memory (two tiles' worth, filled one tile ahead).
+template <int BN, int XCOLS, bool PAR = false>
 struct GemmCfg {
   static constexpr int STAGES = XCOLS ? (BN == 256 && XCOLS == 256 ? 3 : (BN == 256 ? 4 : 5))
                                       : (BN == 256 ? 4 : 6);
@@ -44,8 +46,9 @@ struct GemmCfg {
   static constexpr uint32_t B_BYTES = BN * GEMM_BK * 2;       // 16/32 KB
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr uint32_t X_BYTES = GEMM_BM * XCOLS * 2;
+  static constexpr uint32_t PAR_BYTES = PAR ? 2 * BN * 16 : 0;
   static constexpr uint32_t SMEM_BYTES =
-      STAGES * STAGE_BYTES + X_BYTES + 1024 /*align*/ + 256 /*barriers*/;
+      STAGES * STAGE_BYTES + X_BYTES + 1024 /*align*/ + 256 /*barriers*/ + PAR_BYTES;
 };
 
 // Barrier of the epilogue threads (named barrier 1) that also ANDs a predicate
@@ -78,8 +81,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                    const __grid_constant__ CUtensorMap tmX, int M, int N, int K, int splits,
                    Epi epi) {
   constexpr int XCOLS = Epi::kXTile ? (Epi::kPaired ? BN / 2 : BN) : 0;
-  using Cfg = GemmCfg<BN, XCOLS>;
+  using Cfg = GemmCfg<BN, XCOLS, Epi::kColPar>;
   constexpr int STAGES = Cfg::STAGES;
+  static_assert(!Epi::kColPar || !Epi::kPaired, "column parameters: unpaired epilogues only");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -87,6 +91,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   uint64_t* bars = reinterpret_cast<uint64_t*>(xtile + Cfg::X_BYTES);
   // bars: full[S], empty[S], tfull[2], tempty[2], xfull, done
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 6);
+  float4* cpar = reinterpret_cast<float4*>(xtile + Cfg::X_BYTES + 256);  // [2][BN] if kColPar
   __shared__ uint32_t s_consumed;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -215,6 +220,11 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     const int et = threadIdx.x - 64;
     const int q = warp & 3;                               // TMEM lane quarter
     const int c_begin = ((warp - 2) >> 2) * (BN / 2);     // this warp's column half
+    auto tile_n0 = [&](int t) { return ((t % mn_tiles) % num_n) * BN; };
+    if constexpr (Epi::kColPar) {  // parameters of the first tile
+      if ((int)blockIdx.x < tiles && et < BN) cpar[et] = epi.col_param(tile_n0(blockIdx.x), et);
+      epi_bar_and(true);
+    }
     uint32_t lt = 0;
     for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++lt) {
       PF_TILE_DECODE(tile)
@@ -229,6 +239,12 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         x_pending = true;
         x_parity = lt & 1;
       }
+      // next tile's column parameters: loaded now, stored after this tile
+      const int ntile = tile + (int)gridDim.x;
+      float4 npar = make_float4(0.f, 0.f, 0.f, 0.f);
+      if constexpr (Epi::kColPar)
+        if (ntile < tiles && et < BN) npar = epi.col_param(tile_n0(ntile), et);
+      const float4* cp = cpar + (lt & 1) * BN;
       const bool ok = mbar_wait(tfull0 + 8 * buf, use & 1);
       tc_fence_after();
       if (Epi::kXTile) {
@@ -254,17 +270,31 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
           epi.apply_pair(ri, erow, n0, c, v, w, xtile, rl);
         }
       } else {
-#pragma unroll 1
-        for (int c = c_begin; c < c_begin + BN / 2; c += 32) {
+        // 32-column chunks, the TMEM load of chunk i+1 in flight while chunk i
+        // is processed
+        constexpr int NCH = BN / 64;
+        auto run = [&](const uint32_t* r, int c) {
           float v[32];
-          tmem_ld32(trow + (uint32_t)c, v);
-          if (no_k) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = 0.f;
-          }
-          epi.apply(ri, erow, n0 + c, v, xtile, rl, c);
+          for (int i = 0; i < 32; ++i) v[i] = no_k ? 0.f : __uint_as_float(r[i]);
+          epi.apply(ri, erow, n0 + c, v, xtile, rl, c, cp);
+        };
+        uint32_t ra[32], rb[32];
+        tmem_ld32_async(trow + (uint32_t)c_begin, ra);
+        tmem_wait_ld(ra);
+#pragma unroll 1
+        for (int ci = 0; ci < NCH; ci += 2) {
+          const int c = c_begin + ci * 32;
+          tmem_ld32_async(trow + (uint32_t)(c + 32), rb);
+          run(ra, c);
+          tmem_wait_ld(rb);
+          if (ci + 2 < NCH) tmem_ld32_async(trow + (uint32_t)(c + 64), ra);
+          run(rb, c + 32);
+          if (ci + 2 < NCH) tmem_wait_ld(ra);
         }
       }
+      if constexpr (Epi::kColPar)
+        if (ntile < tiles && et < BN) cpar[((lt + 1) & 1) * BN + et] = npar;
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(tempty0 + 8 * buf);
@@ -307,6 +337,8 @@ struct EpiBase {
   static constexpr bool kXTile = false;
   static constexpr bool kPaired = false;
   static constexpr bool kSplitRows = false;
+  static constexpr bool kColPar = false;
+  __device__ __forceinline__ float4 col_param(int, int) const { return make_float4(0, 0, 0, 0); }
   __device__ __forceinline__ int x_row(int m0) const { return m0; }
   __device__ __forceinline__ int x_col(int n0, int j) const { return n0 + 64 * j; }
   __device__ __forceinline__ int b_row(int n0, int j) const { return n0 + 128 * j; }
@@ -330,7 +362,7 @@ struct EpiLinear : EpiBase {
   long ld_bf16;
   __device__ __forceinline__ Row row_info(int row, int) const { return Row{row < M}; }
   __device__ __forceinline__ void apply(const Row& ri, int row, int col, float* v, const uint8_t*,
-                                        int, int) const {
+                                        int, int, const float4*) const {
     if (!ri.ok || col >= N) return;
     if (bias) {
 #pragma unroll
@@ -398,39 +430,38 @@ struct EpiInject1D : EpiBase {
     }
     return r;
   }
+  // staged per column: (bias, w_x, w_dlt, b_g)
+  static constexpr bool kColPar = true;
+  __device__ __forceinline__ float4 col_param(int n0, int cl) const {
+    const int col = n0 + cl;
+    if (col >= N) return make_float4(0.f, 0.f, 0.f, 0.f);
+    const float b = bias[col];
+    if (!gated) return make_float4(b, 0.f, 0.f, 0.f);
+    const int ch = col % d;
+    return make_float4(b, w_x[ch], w_dlt[ch], b_g[ch]);
+  }
   __device__ __forceinline__ void apply(const Row& ri, int row, int col, float* v,
-                                        const uint8_t* xt, int rl, int cl) const {
+                                        const uint8_t* xt, int rl, int cl,
+                                        const float4* cp) const {
     if (!ri.ok || col >= N) return;
 #pragma unroll
-    for (int i = 0; i < 32; i += 4) {
-      float4 b = *reinterpret_cast<const float4*>(bias + col + i);
-      v[i] += b.x; v[i + 1] += b.y; v[i + 2] += b.z; v[i + 3] += b.w;
-    }
+    for (int i = 0; i < 32; ++i) v[i] += cp[cl + i].x;  // D = acc + bias
     if (D_save) {
       bf16* o = D_save + (long)row * N + col;
 #pragma unroll
       for (int i = 0; i < 32; i += 8) store8_bf16(o + i, v + i);
     }
     if (col >= ri.lim) return;
-    const int ch = col % d;
     bf16* xo = X_out + ri.off0 + col;
 #pragma unroll
     for (int i8 = 0; i8 < 32; i8 += 8) {
       float x[8], o[8];
       xtile_load8(xt, rl, cl + i8, x);
       if (gated) {
-        float4 wx0 = *reinterpret_cast<const float4*>(w_x + ch + i8);
-        float4 wx1 = *reinterpret_cast<const float4*>(w_x + ch + i8 + 4);
-        float4 wd0 = *reinterpret_cast<const float4*>(w_dlt + ch + i8);
-        float4 wd1 = *reinterpret_cast<const float4*>(w_dlt + ch + i8 + 4);
-        float4 bg0 = *reinterpret_cast<const float4*>(b_g + ch + i8);
-        float4 bg1 = *reinterpret_cast<const float4*>(b_g + ch + i8 + 4);
-        const float wx[8] = {wx0.x, wx0.y, wx0.z, wx0.w, wx1.x, wx1.y, wx1.z, wx1.w};
-        const float wd[8] = {wd0.x, wd0.y, wd0.z, wd0.w, wd1.x, wd1.y, wd1.z, wd1.w};
-        const float bg[8] = {bg0.x, bg0.y, bg0.z, bg0.w, bg1.x, bg1.y, bg1.z, bg1.w};
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
-          const float g = fmaf(wx[j], x[j], fmaf(wd[j], v[i8 + j], bg[j]));
+          const float4 p = cp[cl + i8 + j];
+          const float g = fmaf(p.y, x[j], fmaf(p.z, v[i8 + j], p.w));
           o[j] = fmaf(sigmoidf_(g), v[i8 + j], x[j]);
         }
       } else {
@@ -470,7 +501,7 @@ struct EpiDX1D : EpiBase {
     return r;
   }
   __device__ __forceinline__ void apply(const Row& ri, int, int col, float* v, const uint8_t* xt,
-                                        int rl, int cl) const {
+                                        int rl, int cl, const float4*) const {
     if (!ri.ok || col >= ri.lim) return;
     bf16* o = dX + ri.off0 + col;
 #pragma unroll
@@ -506,7 +537,7 @@ struct EpiAppendKV : EpiBase {
     return r;
   }
   __device__ __forceinline__ void apply(const Row& ri, int, int col, float* v, const uint8_t*, int,
-                                        int) const {
+                                        int, const float4*) const {
     if (!ri.ok || col >= N) return;
     bf16* o = col < d ? K + ri.off + col : V + ri.off + (col - d);
 #pragma unroll
@@ -603,7 +634,7 @@ struct EpiDX2D : EpiBase {
     return r;
   }
   __device__ __forceinline__ void apply(const Row& ri, int, int col, float* v, const uint8_t* xt,
-                                        int rl, int cl) const {
+                                        int rl, int cl, const float4*) const {
     if (!ri.ok || col >= N) return;
     const int p = col / d, ch = col - p * d, py = p / patch, px = p - py * patch;
     bf16* o = dX + ri.base + ((long)py * gw + px) * d + ch;
@@ -631,7 +662,7 @@ struct EpiPartial : EpiBase {
     return Row{erow < 0 ? -1L : (long)erow * N};
   }
   __device__ __forceinline__ void apply(const Row& ri, int, int col, float* v, const uint8_t*, int,
-                                        int) const {
+                                        int, const float4*) const {
     if (ri.off < 0 || col >= N) return;
     float* o = part + ri.off + col;
 #pragma unroll

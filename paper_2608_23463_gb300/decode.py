@@ -51,6 +51,17 @@ class ProxyKVCache:
                           torch.cuda.current_stream().cuda_stream)
         return y
 
+    def capture_step(self, x: torch.Tensor, y: torch.Tensor) -> "torch.cuda.CUDAGraph":
+        """Record one decode step on fixed x / y buffers as a CUDA graph.
+
+        Capturing only records the launches; each ``replay()`` then runs one step
+        (the open-block counters live on the device, so consecutive replays fill
+        consecutive slots).  Per-launch timing must be off while capturing."""
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, capture_error_mode="thread_local"):
+            self.step(x, y)
+        return g
+
     def append(self, H_in: torch.Tensor = None) -> None:
         proxy_kv_append(self.desc, self.ap, H_in, self.cache, self.ws, self.ws.numel(),
                         torch.cuda.current_stream().cuda_stream)

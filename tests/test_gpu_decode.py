@@ -131,3 +131,24 @@ def test_capacity_errors_leave_sequences_untouched():
     assert e.value.status == pf.PF_ERR_CAPACITY
     assert cache2.s["n_proxy"].cpu().numpy().tolist() == [1, 2, 4]
     assert cache2.s["n_open"].cpu().numpy().tolist() == [0, 0, P]
+
+
+def test_graph_replay_equals_direct_steps():
+    """A captured step replays exactly like direct calls (the open-block
+    counters advance on the device, so each replay fills the next slot)."""
+    P, d = 16, 256
+    spec = S.DecodeSpec(batch=3, d=d, n_heads=2, P=P, capacity=40)
+    prm = S.make_decode_params(spec, 21)
+    st = S.make_decode_state(spec, 22, [5, 0, 40], [0, 7, 14])
+    direct, graphed = ProxyKVCache(spec, prm, st), ProxyKVCache(spec, prm, st)
+    x = torch.from_numpy(st["x"]).to("cuda", torch.bfloat16)
+    y1, y2 = torch.empty_like(x), torch.empty_like(x)
+    g = graphed.capture_step(x, y2)
+    for _ in range(2):
+        direct.step(x, y1)
+        g.replay()
+        _sync()
+        assert torch.equal(y1, y2)
+    for k in direct.s:
+        assert torch.equal(direct.s[k], graphed.s[k]), k
+    assert graphed.s["n_open"].cpu().numpy().tolist() == [2, 9, 16]
