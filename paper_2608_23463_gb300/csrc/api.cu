@@ -999,8 +999,9 @@ pf_status pf_sync_check(void* stream) {
   PF_CUDA(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
   PF_CUDA(cudaGetLastError());
   int e = 0;
-  for (int v : {take_dev_error_gemm(), take_dev_error_attention(), take_dev_error_elementwise(),
-                take_dev_error_decode(), take_dev_error_fp32(), take_dev_error_layer2d()})
+  for (int v : {take_dev_error_gemm(), take_dev_error_attention(), take_dev_error_attention_tc(),
+                take_dev_error_elementwise(), take_dev_error_decode(), take_dev_error_fp32(),
+                take_dev_error_layer2d()})
     if (v != 0 && e == 0) e = v;
   if (e < 0) return fail(PF_ERR_CUDA, "reading the device error flag failed");
   if (e == DEVERR_TIMEOUT) return fail(PF_ERR_TIMEOUT, "a kernel's bounded wait ran out");

@@ -3,11 +3,10 @@
 //
 // Q, K, V live in one [B*m, 3d] bf16 matrix (columns [Q | K | V], head h at
 // h*64 inside each third); the attention output A is [B*m, d].  The forward
-// is an online-softmax (flash) loop over 64-key tiles per 64-query tile and
-// saves LSE (log2 units) per (b, h, query).  The backward recomputes the
-// probabilities from LSE: one kernel accumulates dK, dV per key tile over the
-// query tiles, a second accumulates dQ per query tile over the key tiles, so
-// no atomics are needed and results are deterministic.
+// (attention_tc.cu) saves LSE (log2 units) per (b, h, query).  The backward
+// here recomputes the probabilities from LSE: one kernel accumulates dK, dV
+// per key tile over the query tiles, a second accumulates dQ per query tile
+// over the key tiles, so no atomics are needed and results are deterministic.
 #include "kernels.h"
 
 namespace pf {
@@ -100,112 +99,6 @@ __device__ __forceinline__ void mma_pt(float (*acc)[4], const float (*p)[4], uin
       ldsm4t(b, s + tile_off(kc * 16 + (mi & 1) * 8 + (lane & 7), dp * 2 + (mi >> 1)));
       mma16816(acc[2 * dp], a, b[0], b[1]);
       mma16816(acc[2 * dp + 1], a, b[2], b[3]);
-    }
-  }
-}
-
-__device__ __forceinline__ float quad_max(float v) {
-  v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 1));
-  return fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 2));
-}
-__device__ __forceinline__ float quad_sum(float v) {
-  v += __shfl_xor_sync(0xffffffffu, v, 1);
-  return v + __shfl_xor_sync(0xffffffffu, v, 2);
-}
-
-template <bool CAUSAL>
-__global__ void __launch_bounds__(128) attn_fwd_kernel(const bf16* __restrict__ qkv,
-                                                       bf16* __restrict__ out,
-                                                       float* __restrict__ lse, int m, int d,
-                                                       int nh, float sl2) {
-  __shared__ __align__(128) uint8_t sm[5 * AT * AT * 2];
-  const uint32_t sQ = smem_u32(sm), sK0 = sQ + 8192, sV0 = sQ + 3 * 8192;
-  const int b = blockIdx.z, h = blockIdx.y, q0 = blockIdx.x * AT;
-  const int w = threadIdx.x >> 5, lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
-  const long ld = 3L * d, rb = (long)b * m;
-  const int qc = h * AT, kc_ = d + h * AT, vc = 2 * d + h * AT;
-  const int n_kt = CAUSAL ? (min(q0 + AT, m) + AT - 1) / AT : (m + AT - 1) / AT;
-
-  load_tile(sQ, qkv, rb, q0, m, ld, qc);
-  cp_commit();
-  load_tile(sK0, qkv, rb, 0, m, ld, kc_);
-  load_tile(sV0, qkv, rb, 0, m, ld, vc);
-  cp_commit();
-
-  uint32_t qf[4][4];
-  float o[8][4] = {};
-  float rmax[2] = {-INFINITY, -INFINITY}, rsum[2] = {0.f, 0.f};
-  const int qrow0 = q0 + w * 16 + g;
-
-  for (int kt = 0; kt < n_kt; ++kt) {
-    const int buf = kt & 1;
-    if (kt + 1 < n_kt) {
-      load_tile(sK0 + (buf ^ 1) * 8192, qkv, rb, (kt + 1) * AT, m, ld, kc_);
-      load_tile(sV0 + (buf ^ 1) * 8192, qkv, rb, (kt + 1) * AT, m, ld, vc);
-      cp_commit();
-      cp_wait<1>();
-    } else {
-      cp_wait<0>();
-    }
-    __syncthreads();
-    if (kt == 0) load_afrag(qf, sQ, w);
-    float s[8][4] = {};
-    mma_abt(s, qf, sK0 + buf * 8192);
-    float tmax[2] = {-INFINITY, -INFINITY};
-#pragma unroll
-    for (int nt = 0; nt < 8; ++nt)
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int key = kt * AT + nt * 8 + 2 * t + (e & 1);
-        const int qr = qrow0 + (e >> 1) * 8;
-        float v = s[nt][e] * sl2;
-        if (key >= m || (CAUSAL && key > qr)) v = -INFINITY;
-        s[nt][e] = v;
-        tmax[e >> 1] = fmaxf(tmax[e >> 1], v);
-      }
-    float corr[2];
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      const float mx = quad_max(tmax[r]);
-      const float mnew = fmaxf(rmax[r], mx);
-      const float mref = (mnew == -INFINITY) ? 0.f : mnew;
-      corr[r] = exp2f(rmax[r] - mref);
-      rmax[r] = mnew;
-      tmax[r] = mref;
-    }
-    float psum[2] = {0.f, 0.f};
-#pragma unroll
-    for (int nt = 0; nt < 8; ++nt)
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float p = exp2f(s[nt][e] - tmax[e >> 1]);
-        s[nt][e] = p;
-        psum[e >> 1] += p;
-      }
-#pragma unroll
-    for (int r = 0; r < 2; ++r) rsum[r] = rsum[r] * corr[r] + psum[r];
-#pragma unroll
-    for (int nt = 0; nt < 8; ++nt) {
-      o[nt][0] *= corr[0];
-      o[nt][1] *= corr[0];
-      o[nt][2] *= corr[1];
-      o[nt][3] *= corr[1];
-    }
-    mma_pt(o, s, sV0 + buf * 8192);
-    __syncthreads();
-  }
-#pragma unroll
-  for (int r = 0; r < 2; ++r) {
-    rsum[r] = quad_sum(rsum[r]);
-    const int qr = qrow0 + r * 8;
-    if (qr < m) {
-      const float inv = 1.f / rsum[r];
-      bf16* op = out + (rb + qr) * d + h * AT + 2 * t;
-#pragma unroll
-      for (int nt = 0; nt < 8; ++nt)
-        *reinterpret_cast<uint32_t*>(op + nt * 8) =
-            pack_bf16(o[nt][2 * r] * inv, o[nt][2 * r + 1] * inv);
-      if (t == 0) lse[((long)b * nh + h) * m + qr] = rmax[r] + log2f(rsum[r]);
     }
   }
 }
@@ -405,20 +298,6 @@ __global__ void __launch_bounds__(128) attn_bwd_dq_kernel(
 }  // namespace
 
 int take_dev_error_attention() { return take_dev_error_tu(); }
-
-cudaError_t attn_fwd(const bf16* qkv, bf16* out, float* lse, int B, int m, int d, int nh,
-                     bool causal, cudaStream_t st) {
-  const float scale = 1.0f / sqrtf((float)AT);
-  const float sl2 = scale * 1.4426950408889634f;
-  dim3 grid((m + AT - 1) / AT, nh, B);
-  const double pairs = (double)B * nh * (causal ? 0.5 * m * (m + 1.0) : (double)m * m);
-  LaunchTimer lt("attn_fwd", st, 4.0 * AT * pairs, 2.0 * B * m * (4.0 * d) + 4.0 * B * nh * m);
-  if (causal)
-    attn_fwd_kernel<true><<<grid, 128, 0, st>>>(qkv, out, lse, m, d, nh, sl2);
-  else
-    attn_fwd_kernel<false><<<grid, 128, 0, st>>>(qkv, out, lse, m, d, nh, sl2);
-  return cudaGetLastError();
-}
 
 cudaError_t attn_bwd(const bf16* qkv, const bf16* O, const bf16* dO, const float* lse, float* Di,
                      bf16* dqkv, int B, int m, int d, int nh, bool causal, cudaStream_t st) {

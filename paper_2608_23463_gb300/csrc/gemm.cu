@@ -141,6 +141,11 @@ __global__ void splitk_reduce_kernel(const float* __restrict__ part, int S, int 
 
 }  // namespace
 
+bool tmap_bf16_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t ld,
+                  uint32_t box_inner, uint32_t box_outer) {
+  return make_map(m, base, inner, outer, ld, box_inner, box_outer);
+}
+
 int splitk_factor(int M, int N, int K) {
   constexpr int kSms = 152;  // planning target (GB300); fixed so sizes are device-independent
   const long tiles = (long)((N + 127) / 128) * ((M + GEMM_BM - 1) / GEMM_BM);

@@ -90,6 +90,7 @@ int num_sms();
 int take_dev_error_gemm();
 int take_dev_error_decode();
 int take_dev_error_attention();
+int take_dev_error_attention_tc();
 int take_dev_error_elementwise();
 
 // ------------------------------------------------------------- 2D layer
@@ -150,6 +151,11 @@ size_t decode_workspace_bytes(int B, int d, int nh, int splits);
 int decode_splits(int B, int nh, int cap);
 cudaError_t decode_step_launch(const DecodeLaunch& L, cudaStream_t st);
 cudaError_t append_finish(int* n_open, int* n_proxy, int B, int P, int cap, cudaStream_t st);
+
+// 2D bf16 TMA map over a row-major [outer, inner] matrix (ld elements per
+// row), 128-byte swizzle, zero fill outside; box box_inner x box_outer.
+bool tmap_bf16_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t ld,
+                  uint32_t box_inner, uint32_t box_outer);
 
 // ------------------------------------------------------------- attention
 cudaError_t attn_fwd(const bf16* qkv, bf16* out, float* lse, int B, int m, int d, int nh,
