@@ -1000,6 +1000,7 @@ pf_status pf_sync_check(void* stream) {
   PF_CUDA(cudaGetLastError());
   int e = 0;
   for (int v : {take_dev_error_gemm(), take_dev_error_attention(), take_dev_error_attention_tc(),
+                take_dev_error_attention_bwd_tc(),
                 take_dev_error_elementwise(), take_dev_error_decode(), take_dev_error_fp32(),
                 take_dev_error_layer2d()})
     if (v != 0 && e == 0) e = v;

@@ -1,0 +1,511 @@
+// Backward of the proxy-space attention (Eq. proxy-attn) on the tcgen05
+// tensor cores, head width 64.  With P = softmax(Q K^T / 8) recomputed from
+// the saved LSE and Di = rowsum(dO * O):
+//   dP = dO V^T,   dS = P * (dP - Di),   dV = P^T dO,   dK = dS^T Q / 8,
+//   dQ = dS K / 8.
+// Two kernels share one skeleton (no atomics, deterministic):
+//   DKDV: item = (128-key tile, head, sequence); stationary X1 = K, X2 = V;
+//         streamed 64-query tiles Y1 = Q_j, Y2 = dO_j.
+//           T1 = X1 Y1^T = S^T,  T2 = X2 Y2^T = dP^T     (TMEM, M=128 N=64)
+//           E1 = P^T, E2 = dS^T  (bf16, shared memory, by the row warps)
+//           dV += E1 Y2,  dK += E2 Y1                    (TMEM accumulators)
+//   DQ:   item = (128-query tile, head, sequence); stationary X1 = Q, X2 = dO;
+//         streamed 64-key tiles Y1 = K_j, Y2 = V_j.
+//           T1 = S,  T2 = dP,  E2 = dS,  dQ += E2 Y1
+// Roles: warp 0 TMA producer, warp 1 MMA issuer, warps 2-5 the row warps (one
+// row of T per thread = TMEM lane).  T1/T2 and E are double-buffered so the
+// MMAs of step j+1 overlap the row work of step j.  Every wait is bounded.
+#include <algorithm>
+
+#include "kernels.h"
+
+namespace pf {
+
+namespace {
+
+constexpr int BW_M = 128;  // stationary rows (TMEM lanes)
+constexpr int BW_N = 64;   // streamed rows per step
+constexpr int BW_D = 64;   // head width
+constexpr int BW_STAGES = 4;
+constexpr int BW_THREADS = 192;
+constexpr uint32_t BW_X_BYTES = BW_M * BW_D * 2;  // 16 KB per stationary tile
+constexpr uint32_t BW_Y_BYTES = BW_N * BW_D * 2;  // 8 KB per streamed tile
+constexpr uint32_t BW_E_BYTES = BW_M * BW_N * 2;  // 16 KB per E tile
+constexpr uint32_t BW_OFF_Y = 2 * 2 * BW_X_BYTES;                      // X: [2 bufs][X1, X2]
+constexpr uint32_t BW_OFF_E = BW_OFF_Y + BW_STAGES * 2 * BW_Y_BYTES;  // Y: [stage][Y1, Y2]
+constexpr uint32_t BW_OFF_LD = BW_OFF_E + 2 * 2 * BW_E_BYTES;         // E: [2 bufs][E1, E2]
+constexpr uint32_t BW_OFF_BAR = BW_OFF_LD + 2 * BW_N * 8;             // (lse, Di) [2][64]
+constexpr uint32_t BW_SMEM = BW_OFF_BAR + 256 + 1024;
+// TMEM: T1 at 0 / 64, T2 at 128 / 192, accumulators at 256 (dV or dQ), 320 (dK)
+constexpr uint32_t BW_TMEM_COLS = 512;
+
+struct BwArgs {
+  bf16* dqkv;         // [B*m, 3d]
+  const float* lse;   // [B, nh, m], log2 units
+  const float* Di;    // [B, nh, m]
+  int B, m, d, nh, causal, n_tiles, n_steps_total, n_items;
+  float sl2, scale;
+};
+
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Barrier of the 128 row threads (named barrier 1) that ANDs a predicate
+// across them, so that they leave their loops together.
+__device__ __forceinline__ bool bar_rows_and(bool p) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred pi, po;\n\t"
+      "setp.ne.u32 pi, %1, 0;\n\t"
+      "bar.red.and.pred po, 1, 128, pi;\n\t"
+      "selp.u32 %0, 1, 0, po;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)p)
+      : "memory");
+  return r != 0;
+}
+
+// Snake order over the CTAs of items ranked heaviest first.
+__device__ __forceinline__ int bw_rank(int c, int round) {
+  return round * (int)gridDim.x + ((round & 1) ? (int)gridDim.x - 1 - c : c);
+}
+
+// Item k -> stationary tile t (128 rows), head, sequence, first streamed tile
+// j0 and step count n.  DKDV: keys of tile t see queries >= key (causal), so
+// the heaviest items have the smallest t; DQ: the largest t.
+template <bool DKDV>
+__device__ __forceinline__ void bw_item(const BwArgs& a, int k, int& t, int& h, int& b, int& j0,
+                                        int& n) {
+  const int per = a.nh * a.B;
+  const int rnk = k / per, r = k % per;
+  h = r % a.nh;
+  b = r / a.nh;
+  if (DKDV) {
+    t = rnk;
+    j0 = a.causal ? 2 * t : 0;
+    n = a.n_steps_total - j0;
+  } else {
+    t = a.n_tiles - 1 - rnk;
+    j0 = 0;
+    n = a.causal ? min(2 * t + 2, a.n_steps_total) : a.n_steps_total;
+  }
+}
+
+template <bool DKDV>
+__global__ void __launch_bounds__(BW_THREADS, 1)
+    attn_bwd_tc_kernel(const __grid_constant__ CUtensorMap tmX1, const __grid_constant__ CUtensorMap tmX2,
+                       const __grid_constant__ CUtensorMap tmY1, const __grid_constant__ CUtensorMap tmY2,
+                       int x1c, int x2c, int y1c, int y2c, BwArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  const uint32_t b0 = smem_u32(smem + BW_OFF_BAR);
+  // x_full[2] x_empty[2] y_full[S] y_empty[S] t_full[2] t_free[2] e_full[2] e_free[2]
+  // acc_full acc_free done
+  const uint32_t x_full = b0, x_empty = b0 + 16, y_full = b0 + 32,
+                 y_empty = y_full + 8 * BW_STAGES, t_full = y_empty + 8 * BW_STAGES,
+                 t_free = t_full + 16, e_full = t_free + 16, e_free = e_full + 16,
+                 acc_full = e_free + 16, acc_free = acc_full + 8, done = acc_free + 8;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + BW_OFF_BAR + 240);
+  const uint32_t sbase = smem_u32(smem);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(x_full + 8 * i, 1);
+      mbar_init(x_empty + 8 * i, 1);
+      mbar_init(t_full + 8 * i, 1);
+      mbar_init(t_free + 8 * i, 128);
+      mbar_init(e_full + 8 * i, 128);
+      mbar_init(e_free + 8 * i, 1);
+    }
+    for (int i = 0; i < BW_STAGES; ++i) {
+      mbar_init(y_full + 8 * i, 1);
+      mbar_init(y_empty + 8 * i, 1);
+    }
+    mbar_init(acc_full, 1);
+    mbar_init(acc_free, 128);
+    mbar_init(done, 1);
+    fence_barrier_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), BW_TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  uint32_t y_issued = 0, x_issued = 0;
+
+  if (warp == 0 && lane == 0) {
+    // ------------------------------------------------------------ producer
+    prefetch_tmap(&tmX1);
+    prefetch_tmap(&tmX2);
+    prefetch_tmap(&tmY1);
+    prefetch_tmap(&tmY2);
+    bool ok = true;
+    uint32_t it = 0;
+    for (int rd = 0, k = bw_rank(blockIdx.x, 0); k < a.n_items && ok;
+         k = bw_rank(blockIdx.x, ++rd), ++it) {
+      int t, h, b, j0, n;
+      bw_item<DKDV>(a, k, t, h, b, j0, n);
+      const int row0 = b * a.m;
+      const uint32_t xb = it & 1;
+      if (!mbar_wait(x_empty + 8 * xb, ((it >> 1) & 1) ^ 1)) break;
+      const uint32_t xdst = sbase + xb * 2 * BW_X_BYTES;
+      mbar_arrive_expect_tx(x_full + 8 * xb, 2 * BW_X_BYTES);
+      tma_load_2d(xdst, &tmX1, x_full + 8 * xb, x1c + h * BW_D, row0 + t * BW_M);
+      tma_load_2d(xdst + BW_X_BYTES, &tmX2, x_full + 8 * xb, x2c + h * BW_D, row0 + t * BW_M);
+      x_issued = it + 1;
+      for (int j = 0; j < n; ++j) {
+        const uint32_t G = y_issued, st = G % BW_STAGES;
+        if (!mbar_wait(y_empty + 8 * st, ((G / BW_STAGES) & 1) ^ 1)) {
+          ok = false;
+          break;
+        }
+        const uint32_t ydst = sbase + BW_OFF_Y + st * 2 * BW_Y_BYTES;
+        const int yrow = row0 + (j0 + j) * BW_N;
+        mbar_arrive_expect_tx(y_full + 8 * st, 2 * BW_Y_BYTES);
+        tma_load_2d(ydst, &tmY1, y_full + 8 * st, y1c + h * BW_D, yrow);
+        tma_load_2d(ydst + BW_Y_BYTES, &tmY2, y_full + 8 * st, y2c + h * BW_D, yrow);
+        y_issued = G + 1;
+      }
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ------------------------------------------------------------ MMA issuer
+    constexpr uint32_t idesc_t = idesc_bf16_f32(BW_M, BW_N, 0, 0);
+    constexpr uint32_t idesc_a = idesc_bf16_f32(BW_M, BW_D, 0, 1);
+    bool ok = true;
+    uint32_t it = 0, G = 0;
+    // accumulate step G (local step j of its item): E_G times the step's Y tiles
+    auto acc_step = [&](uint32_t G_, int j, uint32_t it_) -> bool {
+      const uint32_t eb = G_ & 1, st = G_ % BW_STAGES;
+      if (!mbar_wait(e_full + 8 * eb, (G_ >> 1) & 1)) return false;
+      if (j == 0 && !mbar_wait(acc_free, (it_ & 1) ^ 1)) return false;
+      tc_fence_after();
+      const uint32_t e1 = sbase + BW_OFF_E + eb * 2 * BW_E_BYTES, e2 = e1 + BW_E_BYTES;
+      const uint32_t y1 = sbase + BW_OFF_Y + st * 2 * BW_Y_BYTES, y2 = y1 + BW_Y_BYTES;
+#pragma unroll
+      for (int kk = 0; kk < BW_N / 16; ++kk) {
+        const uint32_t acc = (j > 0 || kk > 0) ? 1u : 0u;
+        const uint64_t bd1 = smem_desc_sw128(y1 + kk * 2048, 8192, 1024);
+        const uint64_t ad2 = smem_desc_sw128(e2 + kk * 32, 16, 1024);
+        if (DKDV) {
+          const uint64_t ad1 = smem_desc_sw128(e1 + kk * 32, 16, 1024);
+          const uint64_t bd2 = smem_desc_sw128(y2 + kk * 2048, 8192, 1024);
+          tc_mma_f16(tmem + 256, ad1, bd2, idesc_a, acc);  // dV += P^T dO
+          tc_mma_f16(tmem + 320, ad2, bd1, idesc_a, acc);  // dK += dS^T Q
+        } else {
+          tc_mma_f16(tmem + 256, ad2, bd1, idesc_a, acc);  // dQ += dS K
+        }
+      }
+      tc_commit(e_free + 8 * eb);
+      tc_commit(y_empty + 8 * st);
+      return true;
+    };
+    for (int rd = 0, k = bw_rank(blockIdx.x, 0); k < a.n_items && ok;
+         k = bw_rank(blockIdx.x, ++rd), ++it) {
+      int t, h, b, j0, n;
+      bw_item<DKDV>(a, k, t, h, b, j0, n);
+      const uint32_t xb = it & 1;
+      if (!mbar_wait(x_full + 8 * xb, (it >> 1) & 1)) break;
+      tc_fence_after();
+      const uint32_t x1 = sbase + xb * 2 * BW_X_BYTES, x2 = x1 + BW_X_BYTES;
+      for (int j = 0; j < n; ++j) {
+        const uint32_t Gj = G + j, st = Gj % BW_STAGES, tb = Gj & 1;
+        if (!mbar_wait(y_full + 8 * st, (Gj / BW_STAGES) & 1) ||
+            !mbar_wait(t_free + 8 * tb, ((Gj >> 1) & 1) ^ 1)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t y1 = sbase + BW_OFF_Y + st * 2 * BW_Y_BYTES, y2 = y1 + BW_Y_BYTES;
+#pragma unroll
+        for (int kk = 0; kk < BW_D / 16; ++kk) {
+          tc_mma_f16(tmem + tb * BW_N, smem_desc_sw128(x1 + kk * 32, 16, 1024),
+                     smem_desc_sw128(y1 + kk * 32, 16, 1024), idesc_t, kk ? 1u : 0u);
+          tc_mma_f16(tmem + 128 + tb * BW_N, smem_desc_sw128(x2 + kk * 32, 16, 1024),
+                     smem_desc_sw128(y2 + kk * 32, 16, 1024), idesc_t, kk ? 1u : 0u);
+        }
+        tc_commit(t_full + 8 * tb);
+        if (j == n - 1) tc_commit(x_empty + 8 * xb);
+        if (j > 0 && !acc_step(Gj - 1, j - 1, it)) {
+          ok = false;
+          break;
+        }
+      }
+      if (!ok || !acc_step(G + n - 1, n - 1, it)) break;
+      tc_commit(acc_full);
+      G += n;
+    }
+    tc_commit(done);
+  } else if (warp >= 2) {
+    // ------------------------------------------------------------ row warps
+    const int q4 = warp & 3;
+    const int r = q4 * 32 + lane;  // stationary row in the tile = TMEM lane
+    const int tr = threadIdx.x - 64;  // 0..127
+    const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
+    float2* ld_s = reinterpret_cast<float2*>(smem + BW_OFF_LD);  // [2][64] (lse, Di)
+    bool ok = true;
+    uint32_t G = 0, it = 0;
+    // DKDV: (lse, Di) of the streamed queries, one step ahead: thread tr < 64
+    // fetches column tr of the next step
+    auto fetch_ld = [&](int b, int h, int q0, int c) -> float2 {
+      const int qq = q0 + c;
+      if (c >= BW_N || qq >= a.m) return make_float2(0.f, 0.f);
+      const long o = ((long)b * a.nh + h) * a.m + qq;
+      return make_float2(a.lse[o], a.Di[o]);
+    };
+    int rd = 0;
+    int k = bw_rank(blockIdx.x, 0);
+    float2 ld_next = make_float2(0.f, 0.f);
+    if (DKDV && k < a.n_items) {
+      int t, h, b, j0, n;
+      bw_item<DKDV>(a, k, t, h, b, j0, n);
+      ld_next = fetch_ld(b, h, j0 * BW_N, tr);
+    }
+    for (; k < a.n_items && ok; k = bw_rank(blockIdx.x, ++rd), ++it) {
+      int t, h, b, j0, n;
+      bw_item<DKDV>(a, k, t, h, b, j0, n);
+      const int row = t * BW_M + r;  // key (DKDV) or query (DQ) index in the sequence
+      float lse_r = 0.f, di_r = 0.f;
+      if (!DKDV && row < a.m) {
+        const long o = ((long)b * a.nh + h) * a.m + row;
+        lse_r = a.lse[o];
+        di_r = a.Di[o];
+      }
+      for (int j = 0; j < n; ++j) {
+        const uint32_t Gj = G + j, tb = Gj & 1;
+        const int c0 = (j0 + j) * BW_N;  // first streamed index of this step
+        if (DKDV) {
+          // publish this step's (lse, Di); fetch the next step's.  A thread
+          // whose wait ran out reaches this barrier too, and all leave.
+          if (tr < BW_N) ld_s[tb * BW_N + tr] = ld_next;
+          if (!bar_rows_and(ok)) {
+            ok = false;
+            break;
+          }
+          if (j + 1 < n) {
+            ld_next = fetch_ld(b, h, c0 + BW_N, tr);
+          } else {
+            const int k2 = bw_rank(blockIdx.x, rd + 1);
+            if (k2 < a.n_items) {
+              int t2, h2, b2, j02, n2;
+              bw_item<DKDV>(a, k2, t2, h2, b2, j02, n2);
+              ld_next = fetch_ld(b2, h2, j02 * BW_N, tr);
+            }
+          }
+        }
+        if (!ok) break;
+        if (!mbar_wait(t_full + 8 * tb, (Gj >> 1) & 1)) {
+          ok = false;
+          if (DKDV) continue;  // to the next barrier
+          break;
+        }
+        tc_fence_after();
+        uint32_t s1[32], s2[32], p1[32], p2[32];
+        tmem_ld32_async(tl + tb * BW_N, s1);
+        tmem_ld32_async(tl + tb * BW_N + 32, s2);
+        tmem_ld32_async(tl + 128 + tb * BW_N, p1);
+        tmem_ld32_async(tl + 128 + tb * BW_N + 32, p2);
+        tmem_wait_ld(s1);
+        tmem_wait_ld(s2);
+        tmem_wait_ld(p1);
+        tmem_wait_ld(p2);
+        tc_fence_before();
+        mbar_arrive(t_free + 8 * tb);
+        // valid streamed columns: [lo, hi)
+        int lo = 0, hi = min(BW_N, a.m - c0);
+        if (a.causal) {
+          if (DKDV)
+            lo = max(0, row - c0);  // queries >= key
+          else
+            hi = min(hi, row - c0 + 1);  // keys <= query
+        }
+        if (!mbar_wait(e_free + 8 * tb, ((Gj >> 1) & 1) ^ 1)) {
+          ok = false;
+          if (DKDV) continue;
+          break;
+        }
+        uint8_t* e1row = smem + BW_OFF_E + tb * 2 * BW_E_BYTES + r * 128;
+        uint8_t* e2row = e1row + BW_E_BYTES;
+        const float2* lds = ld_s + tb * BW_N;
+#pragma unroll
+        for (int kg = 0; kg < 8; ++kg) {
+          const uint32_t* sv = kg < 4 ? s1 + kg * 8 : s2 + (kg - 4) * 8;
+          const uint32_t* dv = kg < 4 ? p1 + kg * 8 : p2 + (kg - 4) * 8;
+          float pe[8], de[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const int c = kg * 8 + e;
+            float l2, dd;
+            if (DKDV) {
+              const float2 v = lds[c];
+              l2 = v.x;
+              dd = v.y;
+            } else {
+              l2 = lse_r;
+              dd = di_r;
+            }
+            float p = ex2_approx(fmaf(__uint_as_float(sv[e]), a.sl2, -l2));
+            if (c < lo || c >= hi) p = 0.f;
+            pe[e] = p;
+            de[e] = p * (__uint_as_float(dv[e]) - dd);
+          }
+          const int slot = (kg ^ (r & 7)) << 4;
+          if (DKDV)
+            *reinterpret_cast<uint4*>(e1row + slot) =
+                make_uint4(pack_bf16(pe[0], pe[1]), pack_bf16(pe[2], pe[3]),
+                           pack_bf16(pe[4], pe[5]), pack_bf16(pe[6], pe[7]));
+          *reinterpret_cast<uint4*>(e2row + slot) =
+              make_uint4(pack_bf16(de[0], de[1]), pack_bf16(de[2], de[3]),
+                         pack_bf16(de[4], de[5]), pack_bf16(de[6], de[7]));
+        }
+        fence_proxy_async_smem();
+        mbar_arrive(e_full + 8 * tb);
+      }
+      if (DKDV) ok = bar_rows_and(ok);
+      if (!ok) break;
+      G += n;
+      // accumulators -> dK, dV (DKDV) or dQ (DQ) rows
+      bool acc_ok = mbar_wait(acc_full, it & 1);
+      if (DKDV) acc_ok = bar_rows_and(acc_ok);
+      if (!acc_ok) break;
+      tc_fence_after();
+      uint32_t u0[32], u1[32], w0[32], w1[32];
+      tmem_ld32_async(tl + 256, u0);
+      tmem_ld32_async(tl + 256 + 32, u1);
+      if (DKDV) {
+        tmem_ld32_async(tl + 320, w0);
+        tmem_ld32_async(tl + 320 + 32, w1);
+      }
+      tmem_wait_ld(u0);
+      tmem_wait_ld(u1);
+      if (DKDV) {
+        tmem_wait_ld(w0);
+        tmem_wait_ld(w1);
+      }
+      tc_fence_before();
+      mbar_arrive(acc_free);
+      if (row < a.m) {
+        bf16* base = a.dqkv + ((long)b * a.m + row) * 3 * a.d + h * BW_D;
+        // DKDV: u = dV (column block 2d), w = dK (column block d); DQ: u = dQ
+        bf16* pu = base + (DKDV ? 2 * a.d : 0);
+        const float su = DKDV ? 1.f : a.scale;
+#pragma unroll
+        for (int i = 0; i < 32; i += 8) {
+          *reinterpret_cast<uint4*>(pu + i) = make_uint4(
+              pack_bf16(__uint_as_float(u0[i]) * su, __uint_as_float(u0[i + 1]) * su),
+              pack_bf16(__uint_as_float(u0[i + 2]) * su, __uint_as_float(u0[i + 3]) * su),
+              pack_bf16(__uint_as_float(u0[i + 4]) * su, __uint_as_float(u0[i + 5]) * su),
+              pack_bf16(__uint_as_float(u0[i + 6]) * su, __uint_as_float(u0[i + 7]) * su));
+          *reinterpret_cast<uint4*>(pu + 32 + i) = make_uint4(
+              pack_bf16(__uint_as_float(u1[i]) * su, __uint_as_float(u1[i + 1]) * su),
+              pack_bf16(__uint_as_float(u1[i + 2]) * su, __uint_as_float(u1[i + 3]) * su),
+              pack_bf16(__uint_as_float(u1[i + 4]) * su, __uint_as_float(u1[i + 5]) * su),
+              pack_bf16(__uint_as_float(u1[i + 6]) * su, __uint_as_float(u1[i + 7]) * su));
+        }
+        if (DKDV) {
+          bf16* pw = base + a.d;
+          const float sw = a.scale;
+#pragma unroll
+          for (int i = 0; i < 32; i += 8) {
+            *reinterpret_cast<uint4*>(pw + i) = make_uint4(
+                pack_bf16(__uint_as_float(w0[i]) * sw, __uint_as_float(w0[i + 1]) * sw),
+                pack_bf16(__uint_as_float(w0[i + 2]) * sw, __uint_as_float(w0[i + 3]) * sw),
+                pack_bf16(__uint_as_float(w0[i + 4]) * sw, __uint_as_float(w0[i + 5]) * sw),
+                pack_bf16(__uint_as_float(w0[i + 6]) * sw, __uint_as_float(w0[i + 7]) * sw));
+            *reinterpret_cast<uint4*>(pw + 32 + i) = make_uint4(
+                pack_bf16(__uint_as_float(w1[i]) * sw, __uint_as_float(w1[i + 1]) * sw),
+                pack_bf16(__uint_as_float(w1[i + 2]) * sw, __uint_as_float(w1[i + 3]) * sw),
+                pack_bf16(__uint_as_float(w1[i + 4]) * sw, __uint_as_float(w1[i + 5]) * sw),
+                pack_bf16(__uint_as_float(w1[i + 6]) * sw, __uint_as_float(w1[i + 7]) * sw));
+          }
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  if (__syncthreads_or(*(volatile int*)&g_dev_error != 0)) {
+    // error path: let this CTA's copies and MMAs land before smem / TMEM go
+    if (warp == 0 && lane == 0) {
+      for (uint32_t Gd = y_issued > BW_STAGES ? y_issued - BW_STAGES : 0; Gd < y_issued; ++Gd)
+        mbar_wait_drain(y_full + 8 * (Gd % BW_STAGES), (Gd / BW_STAGES) & 1);
+      for (uint32_t t = x_issued > 2 ? x_issued - 2 : 0; t < x_issued; ++t)
+        mbar_wait_drain(x_full + 8 * (t & 1), (t >> 1) & 1);
+    }
+    if (warp == 1 && lane == 0) mbar_wait_drain(done, 0);
+  } else if (warp == 1 && lane == 0) {
+    mbar_wait(done, 0);
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, BW_TMEM_COLS);
+  }
+}
+
+}  // namespace
+
+int take_dev_error_attention_bwd_tc() { return take_dev_error_tu(); }
+
+cudaError_t attn_bwd_tc(const bf16* qkv, const bf16* dO, const float* lse, const float* Di,
+                        bf16* dqkv, int B, int m, int d, int nh, bool causal, cudaStream_t st) {
+  if (d != nh * BW_D || ((uintptr_t)qkv & 15) || ((uintptr_t)dO & 15) || ((uintptr_t)dqkv & 15))
+    return cudaErrorInvalidValue;
+  const uint64_t rows = (uint64_t)B * m;
+  CUtensorMap qkv128, qkv64, do128, do64;
+  if (!tmap_bf16_2d(&qkv128, qkv, 3ull * d, rows, 3ull * d, 64, BW_M) ||
+      !tmap_bf16_2d(&qkv64, qkv, 3ull * d, rows, 3ull * d, 64, BW_N) ||
+      !tmap_bf16_2d(&do128, dO, (uint64_t)d, rows, (uint64_t)d, 64, BW_M) ||
+      !tmap_bf16_2d(&do64, dO, (uint64_t)d, rows, (uint64_t)d, 64, BW_N))
+    return cudaErrorInvalidValue;
+  BwArgs a{};
+  a.dqkv = dqkv;
+  a.lse = lse;
+  a.Di = Di;
+  a.B = B;
+  a.m = m;
+  a.d = d;
+  a.nh = nh;
+  a.causal = causal ? 1 : 0;
+  a.n_tiles = (m + BW_M - 1) / BW_M;
+  a.n_steps_total = (m + BW_N - 1) / BW_N;
+  a.n_items = a.n_tiles * nh * B;
+  a.scale = 1.0f / sqrtf((float)BW_D);
+  a.sl2 = a.scale * 1.4426950408889634f;
+  const int grid = std::min(a.n_items, num_sms());
+  const double pairs = (double)B * nh * (causal ? 0.5 * m * (m + 1.0) : (double)m * m);
+  cudaError_t e;
+  {
+    auto kern = attn_bwd_tc_kernel<true>;
+    if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, BW_SMEM)) !=
+        cudaSuccess)
+      return e;
+    LaunchTimer lt("attn_bwd_dkdv", st, 8.0 * BW_D * pairs, 2.0 * B * m * (5.0 * d));
+    // X1 = K, X2 = V (128 rows); Y1 = Q, Y2 = dO (64 rows)
+    kern<<<grid, BW_THREADS, BW_SMEM, st>>>(qkv128, qkv128, qkv64, do64, d, 2 * d, 0, 0, a);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
+  {
+    auto kern = attn_bwd_tc_kernel<false>;
+    if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, BW_SMEM)) !=
+        cudaSuccess)
+      return e;
+    LaunchTimer lt("attn_bwd_dq", st, 6.0 * BW_D * pairs, 2.0 * B * m * (4.0 * d));
+    // X1 = Q, X2 = dO (128 rows); Y1 = K, Y2 = V (64 rows)
+    kern<<<grid, BW_THREADS, BW_SMEM, st>>>(qkv128, do128, qkv64, qkv64, 0, 0, d, 2 * d, a);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+}  // namespace pf

@@ -91,6 +91,7 @@ int take_dev_error_gemm();
 int take_dev_error_decode();
 int take_dev_error_attention();
 int take_dev_error_attention_tc();
+int take_dev_error_attention_bwd_tc();
 int take_dev_error_elementwise();
 
 // ------------------------------------------------------------- 2D layer
@@ -160,6 +161,8 @@ bool tmap_bf16_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t out
 // ------------------------------------------------------------- attention
 cudaError_t attn_fwd(const bf16* qkv, bf16* out, float* lse, int B, int m, int d, int nh,
                      bool causal, cudaStream_t st);
+cudaError_t attn_bwd_tc(const bf16* qkv, const bf16* dO, const float* lse, const float* Di,
+                        bf16* dqkv, int B, int m, int d, int nh, bool causal, cudaStream_t st);
 cudaError_t attn_bwd(const bf16* qkv, const bf16* O, const bf16* dO, const float* lse, float* Di,
                      bf16* dqkv, int B, int m, int d, int nh, bool causal, cudaStream_t st);
 
