@@ -203,8 +203,12 @@ def gpu_smi_id(torch, dev: int) -> str:
 # ------------------------------------------------------------------ our leg
 def kernel_files(label: str):
     """Source files that define the kernel behind a timing label."""
+    if label == "attn_fwd":
+        return ["attention_tc.cu", "common.cuh"]
     if label.startswith("attn_"):
-        return ["attention.cu", "common.cuh"]
+        return ["attention_bwd_tc.cu", "attention.cu", "common.cuh"]
+    if label.startswith("decode_"):
+        return ["decode.cu", "common.cuh"]
     if label.startswith(("inj_bwd", "colsum", "copy_block0", "pad_rows")):
         return ["elementwise.cu", "common.cuh"]
     return ["gemm_tc.cuh", "gemm.cu", "common.cuh"]

@@ -75,6 +75,34 @@ __device__ __forceinline__ void xtile_load8(const uint8_t* xt, int r, int c, flo
   v[0] = a.x; v[1] = a.y; v[2] = b.x; v[3] = b.y; v[4] = e.x; v[5] = e.y; v[6] = f.x; v[7] = f.y;
 }
 
+// Address of 8 bf16 at row r, columns [c, c+8) of the swizzled tile above.
+__device__ __forceinline__ uint8_t* xtile_ptr(uint8_t* xt, int r, int c) {
+  return xt + (c >> 6) * 16384 + r * 128 + ((((c & 63) >> 3) ^ (r & 7)) << 4);
+}
+
+// Coalesced store of a warp's 32 rows x 32 columns (tile rows 32q.., tile
+// columns cl..) that its threads have staged, one row each, in the swizzled
+// tile: every store instruction writes 8 rows x 64 contiguous bytes.  dst(rr,
+// p) returns the global address of row rr's 16-byte piece p (or null to skip);
+// it is called by all lanes in step (it may shuffle).
+template <class F>
+__device__ __forceinline__ void warp_store_rows(uint8_t* xt, int q, int cl, F dst) {
+  const int lane = threadIdx.x & 31, p = lane & 3;
+#pragma unroll
+  for (int it = 0; it < 4; ++it) {
+    const int rr = it * 8 + (lane >> 2);
+    bf16* g = dst(rr, p);
+    const uint4 val = *reinterpret_cast<const uint4*>(xtile_ptr(xt, q * 32 + rr, cl + p * 8));
+    if (g) *reinterpret_cast<uint4*>(g) = val;
+  }
+}
+
+__device__ __forceinline__ void xtile_put8(uint8_t* xt, int r, int c, const float* v) {
+  *reinterpret_cast<uint4*>(xtile_ptr(xt, r, c)) =
+      make_uint4(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]), pack_bf16(v[4], v[5]),
+                 pack_bf16(v[6], v[7]));
+}
+
 template <int BN, bool A_MN, bool B_MN, class Epi>
 __global__ void __launch_bounds__(GEMM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
@@ -440,19 +468,14 @@ struct EpiInject1D : EpiBase {
     const int ch = col % d;
     return make_float4(b, w_x[ch], w_dlt[ch], b_g[ch]);
   }
-  __device__ __forceinline__ void apply(const Row& ri, int row, int col, float* v,
-                                        const uint8_t* xt, int rl, int cl,
-                                        const float4* cp) const {
-    if (!ri.ok || col >= N) return;
+  // The warp's 32 x 32 chunk of X_out and then of D is staged in the X tile
+  // cells it has just read and stored with whole-row segments.
+  __device__ __forceinline__ void apply(const Row& ri, int row, int col, float* v, uint8_t* xt,
+                                        int rl, int cl, const float4* cp) const {
+    if (col >= N) return;  // uniform across the warp
+    const int q = rl >> 5;
 #pragma unroll
     for (int i = 0; i < 32; ++i) v[i] += cp[cl + i].x;  // D = acc + bias
-    if (D_save) {
-      bf16* o = D_save + (long)row * N + col;
-#pragma unroll
-      for (int i = 0; i < 32; i += 8) store8_bf16(o + i, v + i);
-    }
-    if (col >= ri.lim) return;
-    bf16* xo = X_out + ri.off0 + col;
 #pragma unroll
     for (int i8 = 0; i8 < 32; i8 += 8) {
       float x[8], o[8];
@@ -468,7 +491,27 @@ struct EpiInject1D : EpiBase {
 #pragma unroll
         for (int j = 0; j < 8; ++j) o[j] = x[j] + v[i8 + j];
       }
-      store8_bf16(xo + i8, o);
+      xtile_put8(xt, rl, cl + i8, o);
+    }
+    __syncwarp();
+    const long long off = ri.off0;
+    const int lim = ri.ok ? ri.lim : 0;
+    warp_store_rows(xt, q, cl, [&](int rr, int p) -> bf16* {
+      const long long o2 = __shfl_sync(0xffffffffu, off, rr);
+      const int l2 = __shfl_sync(0xffffffffu, lim, rr);
+      return col + p * 8 < l2 ? X_out + o2 + col + p * 8 : nullptr;
+    });
+    __syncwarp();
+    if (D_save) {
+#pragma unroll
+      for (int i8 = 0; i8 < 32; i8 += 8) xtile_put8(xt, rl, cl + i8, v + i8);
+      __syncwarp();
+      const int rfirst = row - (rl & 31);
+      warp_store_rows(xt, q, cl, [&](int rr, int p) -> bf16* {
+        const int r2 = rfirst + rr;
+        return r2 < M ? D_save + (long)r2 * N + col + p * 8 : nullptr;
+      });
+      __syncwarp();
     }
   }
 };
@@ -500,18 +543,27 @@ struct EpiDX1D : EpiBase {
     }
     return r;
   }
-  __device__ __forceinline__ void apply(const Row& ri, int, int col, float* v, const uint8_t* xt,
+  // staged in the tile cells just read, stored with whole-row segments
+  __device__ __forceinline__ void apply(const Row& ri, int, int col, float* v, uint8_t* xt,
                                         int rl, int cl, const float4*) const {
-    if (!ri.ok || col >= ri.lim) return;
-    bf16* o = dX + ri.off0 + col;
+    if (col >= N) return;  // uniform across the warp
 #pragma unroll
     for (int i8 = 0; i8 < 32; i8 += 8) {
       float x[8];
       xtile_load8(xt, rl, cl + i8, x);
 #pragma unroll
       for (int j = 0; j < 8; ++j) x[j] += v[i8 + j];
-      store8_bf16(o + i8, x);
+      xtile_put8(xt, rl, cl + i8, x);
     }
+    __syncwarp();
+    const long long off = ri.off0;
+    const int lim = ri.ok ? ri.lim : 0;
+    warp_store_rows(xt, rl >> 5, cl, [&](int rr, int p) -> bf16* {
+      const long long o2 = __shfl_sync(0xffffffffu, off, rr);
+      const int l2 = __shfl_sync(0xffffffffu, lim, rr);
+      return col + p * 8 < l2 ? dX + o2 + col + p * 8 : nullptr;
+    });
+    __syncwarp();
   }
 };
 
