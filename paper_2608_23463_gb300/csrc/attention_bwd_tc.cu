@@ -53,10 +53,6 @@ __device__ __forceinline__ float ex2_approx(float x) {
   return y;
 }
 
-__device__ __forceinline__ void fence_proxy_async_smem() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-
 // Barrier of the 128 row threads (named barrier 1) that ANDs a predicate
 // across them, so that they leave their loops together.
 __device__ __forceinline__ bool bar_rows_and(bool p) {

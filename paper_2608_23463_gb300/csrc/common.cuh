@@ -117,6 +117,12 @@ __device__ __forceinline__ void mbar_wait_drain(uint32_t bar, uint32_t parity) {
   }
 }
 
+// Orders this thread's generic-proxy shared-memory accesses before later
+// async-proxy (TMA, tcgen05) accesses of the same memory.
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 // ----------------------------------------------------------------------- TMA
 // Contiguous global -> shared copy (no tensor map); dst, src and bytes must be
 // multiples of 16.  Completes `bytes` of transaction count on `bar`.

@@ -119,7 +119,16 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   uint64_t* bars = reinterpret_cast<uint64_t*>(xtile + Cfg::X_BYTES);
   // bars: full[S], empty[S], tfull[2], tempty[2], xfull, done
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 6);
-  float4* cpar = reinterpret_cast<float4*>(xtile + Cfg::X_BYTES + 256);  // [2][BN] if kColPar
+  // column parameters (kColPar), [2 tiles][BN/4 groups][4 params] float4: the
+  // float4 at (c / 4) * 4 + k holds parameter k of columns c & ~3 .. (c & ~3) + 3
+  float4* cpar = reinterpret_cast<float4*>(xtile + Cfg::X_BYTES + 256);
+  auto cpar_put = [&](int b, int col, float4 p) {
+    float* f = reinterpret_cast<float*>(cpar + b * BN) + (col >> 2) * 16 + (col & 3);
+    f[0] = p.x;
+    f[4] = p.y;
+    f[8] = p.z;
+    f[12] = p.w;
+  };
   __shared__ uint32_t s_consumed;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -250,7 +259,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     const int c_begin = ((warp - 2) >> 2) * (BN / 2);     // this warp's column half
     auto tile_n0 = [&](int t) { return ((t % mn_tiles) % num_n) * BN; };
     if constexpr (Epi::kColPar) {  // parameters of the first tile
-      if ((int)blockIdx.x < tiles && et < BN) cpar[et] = epi.col_param(tile_n0(blockIdx.x), et);
+      if ((int)blockIdx.x < tiles && et < BN) cpar_put(0, et, epi.col_param(tile_n0(blockIdx.x), et));
       epi_bar_and(true);
     }
     uint32_t lt = 0;
@@ -322,7 +331,10 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         }
       }
       if constexpr (Epi::kColPar)
-        if (ntile < tiles && et < BN) cpar[((lt + 1) & 1) * BN + et] = npar;
+        if (ntile < tiles && et < BN) cpar_put((lt + 1) & 1, et, npar);
+      // staging writes into the X tile are ordered before the next tile's
+      // TMA load of it
+      if (Epi::kXTile) fence_proxy_async_smem();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(tempty0 + 8 * buf);
@@ -469,23 +481,38 @@ struct EpiInject1D : EpiBase {
     return make_float4(b, w_x[ch], w_dlt[ch], b_g[ch]);
   }
   // The warp's 32 x 32 chunk of X_out and then of D is staged in the X tile
-  // cells it has just read and stored with whole-row segments.
+  // cells it has just read and stored with whole-row segments.  cp: the
+  // staged parameters, one float4 per (4-column group, parameter).
   __device__ __forceinline__ void apply(const Row& ri, int row, int col, float* v, uint8_t* xt,
                                         int rl, int cl, const float4* cp) const {
     if (col >= N) return;  // uniform across the warp
     const int q = rl >> 5;
+    const float4* cg = cp + (cl >> 2) * 4;
 #pragma unroll
-    for (int i = 0; i < 32; ++i) v[i] += cp[cl + i].x;  // D = acc + bias
+    for (int i4 = 0; i4 < 8; ++i4) {  // D = acc + bias
+      const float4 b = cg[i4 * 4];
+      v[4 * i4] += b.x;
+      v[4 * i4 + 1] += b.y;
+      v[4 * i4 + 2] += b.z;
+      v[4 * i4 + 3] += b.w;
+    }
 #pragma unroll
     for (int i8 = 0; i8 < 32; i8 += 8) {
       float x[8], o[8];
       xtile_load8(xt, rl, cl + i8, x);
       if (gated) {
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const float4 p = cp[cl + i8 + j];
-          const float g = fmaf(p.y, x[j], fmaf(p.z, v[i8 + j], p.w));
-          o[j] = fmaf(sigmoidf_(g), v[i8 + j], x[j]);
+        for (int h = 0; h < 2; ++h) {
+          const int g4 = (i8 >> 2) + h;
+          const float4 wx = cg[g4 * 4 + 1], wd = cg[g4 * 4 + 2], bg = cg[g4 * 4 + 3];
+          const float wxa[4] = {wx.x, wx.y, wx.z, wx.w}, wda[4] = {wd.x, wd.y, wd.z, wd.w},
+                      bga[4] = {bg.x, bg.y, bg.z, bg.w};
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const int e = h * 4 + j;
+            const float g = fmaf(wxa[j], x[e], fmaf(wda[j], v[i8 + e], bga[j]));
+            o[e] = fmaf(sigmoidf_(g), v[i8 + e], x[e]);
+          }
         }
       } else {
 #pragma unroll
