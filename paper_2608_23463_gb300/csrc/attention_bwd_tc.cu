@@ -12,10 +12,12 @@
 //   DQ:   item = (128-query tile, head, sequence); stationary X1 = Q, X2 = dO;
 //         streamed 64-key tiles Y1 = K_j, Y2 = V_j.
 //           T1 = S,  T2 = dP,  E2 = dS,  dQ += E2 Y1
-// Roles: warp 0 TMA producer, warp 1 MMA issuer, warps 2-5 the row warps (one
-// row of T per thread = TMEM lane).  T1/T2 and E are double-buffered so the
-// MMAs of step j+1 overlap the row work of step j.  Every wait is bounded.
+// Roles: warp 0 TMA producer, warp 1 MMA issuer, warps 2-9 the row warps: two
+// per TMEM lane quarter, each thread one row (TMEM lane) and one half of the
+// 64 streamed columns.  T1/T2 and E are double-buffered so the MMAs of step
+// j+1 overlap the row work of step j.  Every wait is bounded.
 #include <algorithm>
+#include <type_traits>
 
 #include "kernels.h"
 
@@ -27,7 +29,8 @@ constexpr int BW_M = 128;  // stationary rows (TMEM lanes)
 constexpr int BW_N = 64;   // streamed rows per step
 constexpr int BW_D = 64;   // head width
 constexpr int BW_STAGES = 4;
-constexpr int BW_THREADS = 192;
+constexpr int BW_ROW_THREADS = 256;  // warps 2-9
+constexpr int BW_THREADS = 64 + BW_ROW_THREADS;
 constexpr uint32_t BW_X_BYTES = BW_M * BW_D * 2;  // 16 KB per stationary tile
 constexpr uint32_t BW_Y_BYTES = BW_N * BW_D * 2;  // 8 KB per streamed tile
 constexpr uint32_t BW_E_BYTES = BW_M * BW_N * 2;  // 16 KB per E tile
@@ -53,14 +56,14 @@ __device__ __forceinline__ float ex2_approx(float x) {
   return y;
 }
 
-// Barrier of the 128 row threads (named barrier 1) that ANDs a predicate
-// across them, so that they leave their loops together.
+// Barrier of the row threads (named barrier 1) that ANDs a predicate across
+// them, so that they leave their loops together.
 __device__ __forceinline__ bool bar_rows_and(bool p) {
   uint32_t r;
   asm volatile(
       "{\n\t.reg .pred pi, po;\n\t"
       "setp.ne.u32 pi, %1, 0;\n\t"
-      "bar.red.and.pred po, 1, 128, pi;\n\t"
+      "bar.red.and.pred po, 1, 256, pi;\n\t"
       "selp.u32 %0, 1, 0, po;\n\t}"
       : "=r"(r)
       : "r"((uint32_t)p)
@@ -118,8 +121,8 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
       mbar_init(x_full + 8 * i, 1);
       mbar_init(x_empty + 8 * i, 1);
       mbar_init(t_full + 8 * i, 1);
-      mbar_init(t_free + 8 * i, 128);
-      mbar_init(e_full + 8 * i, 128);
+      mbar_init(t_free + 8 * i, BW_ROW_THREADS);
+      mbar_init(e_full + 8 * i, BW_ROW_THREADS);
       mbar_init(e_free + 8 * i, 1);
     }
     for (int i = 0; i < BW_STAGES; ++i) {
@@ -127,7 +130,7 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
       mbar_init(y_empty + 8 * i, 1);
     }
     mbar_init(acc_full, 1);
-    mbar_init(acc_free, 128);
+    mbar_init(acc_free, BW_ROW_THREADS);
     mbar_init(done, 1);
     fence_barrier_init();
   }
@@ -247,7 +250,8 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
     // ------------------------------------------------------------ row warps
     const int q4 = warp & 3;
     const int r = q4 * 32 + lane;  // stationary row in the tile = TMEM lane
-    const int tr = threadIdx.x - 64;  // 0..127
+    const int tr = threadIdx.x - 64;  // 0..255
+    const int ch = (warp - 2) >> 2;   // half of the streamed columns: [32 ch, 32 ch + 32)
     const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
     float2* ld_s = reinterpret_cast<float2*>(smem + BW_OFF_LD);  // [2][64] (lse, Di)
     bool ok = true;
@@ -307,15 +311,11 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
           break;
         }
         tc_fence_after();
-        uint32_t s1[32], s2[32], p1[32], p2[32];
-        tmem_ld32_async(tl + tb * BW_N, s1);
-        tmem_ld32_async(tl + tb * BW_N + 32, s2);
-        tmem_ld32_async(tl + 128 + tb * BW_N, p1);
-        tmem_ld32_async(tl + 128 + tb * BW_N + 32, p2);
+        uint32_t s1[32], p1[32];
+        tmem_ld32_async(tl + tb * BW_N + 32 * ch, s1);
+        tmem_ld32_async(tl + 128 + tb * BW_N + 32 * ch, p1);
         tmem_wait_ld(s1);
-        tmem_wait_ld(s2);
         tmem_wait_ld(p1);
-        tmem_wait_ld(p2);
         tc_fence_before();
         mbar_arrive(t_free + 8 * tb);
         // valid streamed columns: [lo, hi)
@@ -334,37 +334,46 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
         uint8_t* e1row = smem + BW_OFF_E + tb * 2 * BW_E_BYTES + r * 128;
         uint8_t* e2row = e1row + BW_E_BYTES;
         const float2* lds = ld_s + tb * BW_N;
+        // P and dS of this thread's 32 columns; columns outside [lo, hi) are
+        // masked (only the diagonal and tail steps have any)
+        auto emit = [&](auto masked) {
 #pragma unroll
-        for (int kg = 0; kg < 8; ++kg) {
-          const uint32_t* sv = kg < 4 ? s1 + kg * 8 : s2 + (kg - 4) * 8;
-          const uint32_t* dv = kg < 4 ? p1 + kg * 8 : p2 + (kg - 4) * 8;
-          float pe[8], de[8];
+          for (int g = 0; g < 4; ++g) {
+            const int kg = 4 * ch + g;  // 8-column group in the 64-wide row
+            const uint32_t* sv = s1 + g * 8;
+            const uint32_t* dv = p1 + g * 8;
+            float pe[8], de[8];
 #pragma unroll
-          for (int e = 0; e < 8; ++e) {
-            const int c = kg * 8 + e;
-            float l2, dd;
-            if (DKDV) {
-              const float2 v = lds[c];
-              l2 = v.x;
-              dd = v.y;
-            } else {
-              l2 = lse_r;
-              dd = di_r;
+            for (int e = 0; e < 8; ++e) {
+              const int c = kg * 8 + e;
+              float l2, dd;
+              if (DKDV) {
+                const float2 v = lds[c];
+                l2 = v.x;
+                dd = v.y;
+              } else {
+                l2 = lse_r;
+                dd = di_r;
+              }
+              float p = ex2_approx(fmaf(__uint_as_float(sv[e]), a.sl2, -l2));
+              if (decltype(masked)::value && (c < lo || c >= hi)) p = 0.f;
+              pe[e] = p;
+              de[e] = p * (__uint_as_float(dv[e]) - dd);
             }
-            float p = ex2_approx(fmaf(__uint_as_float(sv[e]), a.sl2, -l2));
-            if (c < lo || c >= hi) p = 0.f;
-            pe[e] = p;
-            de[e] = p * (__uint_as_float(dv[e]) - dd);
+            const int slot = (kg ^ (r & 7)) << 4;
+            if (DKDV)
+              *reinterpret_cast<uint4*>(e1row + slot) =
+                  make_uint4(pack_bf16(pe[0], pe[1]), pack_bf16(pe[2], pe[3]),
+                             pack_bf16(pe[4], pe[5]), pack_bf16(pe[6], pe[7]));
+            *reinterpret_cast<uint4*>(e2row + slot) =
+                make_uint4(pack_bf16(de[0], de[1]), pack_bf16(de[2], de[3]),
+                           pack_bf16(de[4], de[5]), pack_bf16(de[6], de[7]));
           }
-          const int slot = (kg ^ (r & 7)) << 4;
-          if (DKDV)
-            *reinterpret_cast<uint4*>(e1row + slot) =
-                make_uint4(pack_bf16(pe[0], pe[1]), pack_bf16(pe[2], pe[3]),
-                           pack_bf16(pe[4], pe[5]), pack_bf16(pe[6], pe[7]));
-          *reinterpret_cast<uint4*>(e2row + slot) =
-              make_uint4(pack_bf16(de[0], de[1]), pack_bf16(de[2], de[3]),
-                         pack_bf16(de[4], de[5]), pack_bf16(de[6], de[7]));
-        }
+        };
+        if (lo <= 32 * ch && hi >= 32 * ch + 32)
+          emit(std::false_type{});
+        else
+          emit(std::true_type{});
         fence_proxy_async_smem();
         mbar_arrive(e_full + 8 * tb);
       }
@@ -376,55 +385,34 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
       if (DKDV) acc_ok = bar_rows_and(acc_ok);
       if (!acc_ok) break;
       tc_fence_after();
-      uint32_t u0[32], u1[32], w0[32], w1[32];
-      tmem_ld32_async(tl + 256, u0);
-      tmem_ld32_async(tl + 256 + 32, u1);
-      if (DKDV) {
-        tmem_ld32_async(tl + 320, w0);
-        tmem_ld32_async(tl + 320 + 32, w1);
-      }
+      uint32_t u0[32], w0[32];  // this thread's 32 columns of dV / dQ and of dK
+      tmem_ld32_async(tl + 256 + 32 * ch, u0);
+      if (DKDV) tmem_ld32_async(tl + 320 + 32 * ch, w0);
       tmem_wait_ld(u0);
-      tmem_wait_ld(u1);
-      if (DKDV) {
-        tmem_wait_ld(w0);
-        tmem_wait_ld(w1);
-      }
+      if (DKDV) tmem_wait_ld(w0);
       tc_fence_before();
       mbar_arrive(acc_free);
       if (row < a.m) {
-        bf16* base = a.dqkv + ((long)b * a.m + row) * 3 * a.d + h * BW_D;
+        bf16* base = a.dqkv + ((long)b * a.m + row) * 3 * a.d + h * BW_D + 32 * ch;
         // DKDV: u = dV (column block 2d), w = dK (column block d); DQ: u = dQ
         bf16* pu = base + (DKDV ? 2 * a.d : 0);
         const float su = DKDV ? 1.f : a.scale;
 #pragma unroll
-        for (int i = 0; i < 32; i += 8) {
+        for (int i = 0; i < 32; i += 8)
           *reinterpret_cast<uint4*>(pu + i) = make_uint4(
               pack_bf16(__uint_as_float(u0[i]) * su, __uint_as_float(u0[i + 1]) * su),
               pack_bf16(__uint_as_float(u0[i + 2]) * su, __uint_as_float(u0[i + 3]) * su),
               pack_bf16(__uint_as_float(u0[i + 4]) * su, __uint_as_float(u0[i + 5]) * su),
               pack_bf16(__uint_as_float(u0[i + 6]) * su, __uint_as_float(u0[i + 7]) * su));
-          *reinterpret_cast<uint4*>(pu + 32 + i) = make_uint4(
-              pack_bf16(__uint_as_float(u1[i]) * su, __uint_as_float(u1[i + 1]) * su),
-              pack_bf16(__uint_as_float(u1[i + 2]) * su, __uint_as_float(u1[i + 3]) * su),
-              pack_bf16(__uint_as_float(u1[i + 4]) * su, __uint_as_float(u1[i + 5]) * su),
-              pack_bf16(__uint_as_float(u1[i + 6]) * su, __uint_as_float(u1[i + 7]) * su));
-        }
         if (DKDV) {
           bf16* pw = base + a.d;
-          const float sw = a.scale;
 #pragma unroll
-          for (int i = 0; i < 32; i += 8) {
+          for (int i = 0; i < 32; i += 8)
             *reinterpret_cast<uint4*>(pw + i) = make_uint4(
-                pack_bf16(__uint_as_float(w0[i]) * sw, __uint_as_float(w0[i + 1]) * sw),
-                pack_bf16(__uint_as_float(w0[i + 2]) * sw, __uint_as_float(w0[i + 3]) * sw),
-                pack_bf16(__uint_as_float(w0[i + 4]) * sw, __uint_as_float(w0[i + 5]) * sw),
-                pack_bf16(__uint_as_float(w0[i + 6]) * sw, __uint_as_float(w0[i + 7]) * sw));
-            *reinterpret_cast<uint4*>(pw + 32 + i) = make_uint4(
-                pack_bf16(__uint_as_float(w1[i]) * sw, __uint_as_float(w1[i + 1]) * sw),
-                pack_bf16(__uint_as_float(w1[i + 2]) * sw, __uint_as_float(w1[i + 3]) * sw),
-                pack_bf16(__uint_as_float(w1[i + 4]) * sw, __uint_as_float(w1[i + 5]) * sw),
-                pack_bf16(__uint_as_float(w1[i + 6]) * sw, __uint_as_float(w1[i + 7]) * sw));
-          }
+                pack_bf16(__uint_as_float(w0[i]) * a.scale, __uint_as_float(w0[i + 1]) * a.scale),
+                pack_bf16(__uint_as_float(w0[i + 2]) * a.scale, __uint_as_float(w0[i + 3]) * a.scale),
+                pack_bf16(__uint_as_float(w0[i + 4]) * a.scale, __uint_as_float(w0[i + 5]) * a.scale),
+                pack_bf16(__uint_as_float(w0[i + 6]) * a.scale, __uint_as_float(w0[i + 7]) * a.scale));
         }
       }
     }
