@@ -345,7 +345,10 @@ def timed_steps(torch, pf, fn, steps: int, warmup: int):
     nbytes = sum(v["bytes"] * v["launches"] for v in t.values()) / steps
     total = sum(v["ms"] for v in t.values()) or 1.0
     dom, dv = max(t.items(), key=lambda kv: kv[1]["ms"])
-    return ms, flops, nbytes, {"kernel": dom, "share": dv["ms"] / total}
+    top = sorted(t.items(), key=lambda kv: -kv[1]["ms"])[:8]
+    return ms, flops, nbytes, {"kernel": dom, "share": dv["ms"] / total,
+                               "kernels_ms_per_step": {k: v["ms"] / steps for k, v in top},
+                               "launches_per_step": sum(v["launches"] for v in t.values()) / steps}
 
 
 FFMA_PEAK_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12  # SMs x fp32 lanes x 2 x max SM clock

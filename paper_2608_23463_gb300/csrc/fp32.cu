@@ -14,14 +14,15 @@ int take_dev_error_fp32() { return take_dev_error_tu(); }
 namespace {
 
 constexpr int FT = 64;   // output tile (FT x FT)
-constexpr int FK = 16;   // K slab
+constexpr int FK = 32;   // K slab
 constexpr int FTHREADS = 256;
 
 // C[M, N] = A[M, K] B[N, K]^T (+ bias[n]) (+ addend[m, n]), all row-major fp32
 // with leading dimensions lda, ldb, ldc.  Each thread computes 4 x 4 outputs.
-// With gridDim.z = S > 1 each z-slice reduces K range [z*Kc, (z+1)*Kc) and
-// writes raw partials to C + z*M*ldc (bias / addend are then applied by
-// splitk_f32_reduce).
+// The next K slab is fetched into registers while the current one is used
+// (two shared-memory buffers, one barrier per slab).  With gridDim.z = S > 1
+// each z-slice reduces K range [z*Kc, (z+1)*Kc) and writes raw partials to
+// C + z*M*ldc (bias / addend are then applied by splitk_f32_reduce).
 __global__ void __launch_bounds__(FTHREADS) gemm_f32_kernel(const float* __restrict__ A, long lda,
                                                            const float* __restrict__ Bm, long ldb,
                                                            float* __restrict__ C, long ldc, int M,
@@ -29,34 +30,58 @@ __global__ void __launch_bounds__(FTHREADS) gemm_f32_kernel(const float* __restr
                                                            const float* __restrict__ bias,
                                                            const float* __restrict__ addend,
                                                            long ld_add) {
-  __shared__ float As[FK][FT + 4], Bs[FK][FT + 4];
+  __shared__ __align__(16) float As[2][FK][FT + 4], Bs[2][FK][FT + 4];
   const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
   const int m0 = blockIdx.y * FT, n0 = blockIdx.x * FT;
   const int kbeg = blockIdx.z * Kc, kend = min(K, kbeg + Kc);
   C += (long)blockIdx.z * M * ldc;
-  float acc[4][4] = {};
-  for (int k0 = kbeg; k0 < kend; k0 += FK) {
-    for (int i = threadIdx.x; i < FT * FK; i += FTHREADS) {
-      const int r = i / FK, kk = i % FK;
-      const int gm = m0 + r, gn = n0 + r, gk = k0 + kk;
-      As[kk][r] = (gm < M && gk < kend) ? A[(long)gm * lda + gk] : 0.f;
-      Bs[kk][r] = (gn < N && gk < kend) ? Bm[(long)gn * ldb + gk] : 0.f;
+  // thread t loads rows r = t / 8 + 32 i (i = 0, 1) and k = (t % 8) * 4 .. + 4
+  const int lr = threadIdx.x >> 3, lk = (threadIdx.x & 7) * 4;
+  float ra[2][4], rb[2][4];
+  auto fetch = [&](int k0) {
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const int gm = m0 + lr + 32 * i, gn = n0 + lr + 32 * i;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int gk = k0 + lk + e;
+        ra[i][e] = (gm < M && gk < kend) ? A[(long)gm * lda + gk] : 0.f;
+        rb[i][e] = (gn < N && gk < kend) ? Bm[(long)gn * ldb + gk] : 0.f;
+      }
     }
-    __syncthreads();
+  };
+  auto stash = [&](int buf) {
+#pragma unroll
+    for (int i = 0; i < 2; ++i)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        As[buf][lk + e][lr + 32 * i] = ra[i][e];
+        Bs[buf][lk + e][lr + 32 * i] = rb[i][e];
+      }
+  };
+  float acc[4][4] = {};
+  int buf = 0;
+  if (kbeg < kend) {
+    fetch(kbeg);
+    stash(0);
+  }
+  __syncthreads();
+  for (int k0 = kbeg; k0 < kend; k0 += FK) {
+    const bool more = k0 + FK < kend;
+    if (more) fetch(k0 + FK);  // in flight during the FMAs below
 #pragma unroll
     for (int kk = 0; kk < FK; ++kk) {
-      float a[4], b[4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        a[i] = As[kk][ty * 4 + i];
-        b[i] = Bs[kk][tx * 4 + i];
-      }
+      const float4 a4 = *reinterpret_cast<const float4*>(&As[buf][kk][ty * 4]);
+      const float4 b4 = *reinterpret_cast<const float4*>(&Bs[buf][kk][tx * 4]);
+      const float a[4] = {a4.x, a4.y, a4.z, a4.w}, b[4] = {b4.x, b4.y, b4.z, b4.w};
 #pragma unroll
       for (int i = 0; i < 4; ++i)
 #pragma unroll
         for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
     }
+    if (more) stash(buf ^ 1);
     __syncthreads();
+    buf ^= 1;
   }
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
@@ -74,64 +99,142 @@ __global__ void __launch_bounds__(FTHREADS) gemm_f32_kernel(const float* __restr
   }
 }
 
-// Eq. proxy-attn in fp32: one warp per (query, head, sequence), online
-// softmax over the visible keys (j <= i when causal).  Head width 64: two
-// dimensions per lane.
-__global__ void attn_f32_kernel(const float* __restrict__ qkv, float* __restrict__ out, int B,
-                                int m, int d, int nh, int causal, float scale) {
-  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
-  if (warp >= B * nh * m) return;  // whole warps only
-  const int i = warp % m, h = (warp / m) % nh, b = warp / (m * nh);
+// Eq. proxy-attn in fp32, head width 64.  CTA = (sequence, head, block of
+// ATT_Q queries), 8 warps of ATT_Q / 8 queries each.  Keys and values are
+// staged in shared memory 64 at a time (K transposed, so lane j reads key j's
+// dimensions without bank conflicts); each warp keeps an online softmax per
+// query: lane j scores keys j and j + 32 of the chunk and accumulates output
+// dimensions j and j + 32.
+constexpr int ATT_Q = 32;
+__global__ void __launch_bounds__(256) attn_f32_kernel(const float* __restrict__ qkv,
+                                                       float* __restrict__ out, int m, int d,
+                                                       int causal, float scale) {
+  __shared__ float Kt[64][65];                  // [dim][key]
+  __shared__ __align__(16) float Vs[64][64];    // [key][dim]
+  __shared__ __align__(16) float Qs[ATT_Q][64];
+  __shared__ float Ps[8][64];    // per warp: the chunk's probabilities
+  const int b = blockIdx.z, h = blockIdx.y, q0 = blockIdx.x * ATT_Q;
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
   const long ld = 3L * d, rb = (long)b * m;
-  const float* qrow = qkv + (rb + i) * ld + h * 64;
-  const float q0 = qrow[lane] * scale, q1 = qrow[lane + 32] * scale;
-  float mx = -INFINITY, l = 0.f, a0 = 0.f, a1 = 0.f;
-  const int nk = causal ? i + 1 : m;
-  for (int j = 0; j < nk; ++j) {
-    const float* krow = qkv + (rb + j) * ld + d + h * 64;
-    float s = q0 * krow[lane] + q1 * krow[lane + 32];
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
-    const float mn = fmaxf(mx, s);
-    const float c = expf(mx - mn), p = expf(s - mn);
-    const float* vrow = qkv + (rb + j) * ld + 2 * d + h * 64;
-    l = l * c + p;
-    a0 = a0 * c + p * vrow[lane];
-    a1 = a1 * c + p * vrow[lane + 32];
-    mx = mn;
+  for (int i = tid; i < ATT_Q * 16; i += 256) {
+    const int r = i >> 4, c = (i & 15) * 4;
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (q0 + r < m) v = *reinterpret_cast<const float4*>(qkv + (rb + q0 + r) * ld + h * 64 + c);
+    *reinterpret_cast<float4*>(&Qs[r][c]) = make_float4(v.x * scale, v.y * scale, v.z * scale,
+                                                        v.w * scale);
   }
-  float* o = out + (rb + i) * d + h * 64;
-  o[lane] = a0 / l;
-  o[lane + 32] = a1 / l;
+  constexpr int QW = ATT_Q / 8;
+  float mx[QW], l[QW], o0[QW], o1[QW];
+#pragma unroll
+  for (int t = 0; t < QW; ++t) {
+    mx[t] = -INFINITY;
+    l[t] = 0.f;
+    o0[t] = o1[t] = 0.f;
+  }
+  const int kend = causal ? min(m, q0 + ATT_Q) : m;
+  for (int k0 = 0; k0 < kend; k0 += 64) {
+    __syncthreads();  // previous chunk fully used (and Qs written)
+    for (int i = tid; i < 64 * 16; i += 256) {
+      const int r = i >> 4, c = (i & 15) * 4;
+      float4 kv = make_float4(0.f, 0.f, 0.f, 0.f), vv = kv;
+      if (k0 + r < m) {
+        const float* row = qkv + (rb + k0 + r) * ld + h * 64 + c;
+        kv = *reinterpret_cast<const float4*>(row + d);
+        vv = *reinterpret_cast<const float4*>(row + 2 * d);
+      }
+      Kt[c][r] = kv.x;
+      Kt[c + 1][r] = kv.y;
+      Kt[c + 2][r] = kv.z;
+      Kt[c + 3][r] = kv.w;
+      *reinterpret_cast<float4*>(&Vs[r][c]) = vv;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int t = 0; t < QW; ++t) {
+      const int ql = w * QW + t, q = q0 + ql;
+      float s0 = 0.f, s1 = 0.f;
+#pragma unroll 16
+      for (int e = 0; e < 64; ++e) {
+        const float qe = Qs[ql][e];
+        s0 = fmaf(qe, Kt[e][lane], s0);
+        s1 = fmaf(qe, Kt[e][lane + 32], s1);
+      }
+      const int j0 = k0 + lane, j1 = k0 + lane + 32;
+      if (j0 >= m || (causal && j0 > q)) s0 = -INFINITY;
+      if (j1 >= m || (causal && j1 > q)) s1 = -INFINITY;
+      float cm = fmaxf(s0, s1);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) cm = fmaxf(cm, __shfl_xor_sync(0xffffffffu, cm, o));
+      const float mn = fmaxf(mx[t], cm);
+      const float mref = (mn == -INFINITY) ? 0.f : mn;
+      const float corr = expf(mx[t] - mref);
+      const float p0 = expf(s0 - mref), p1 = expf(s1 - mref);
+      float ps = p0 + p1;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) ps += __shfl_xor_sync(0xffffffffu, ps, o);
+      l[t] = l[t] * corr + ps;
+      mx[t] = mn;
+      Ps[w][lane] = p0;
+      Ps[w][lane + 32] = p1;
+      __syncwarp();
+      float a0 = o0[t] * corr, a1 = o1[t] * corr;
+#pragma unroll 16
+      for (int j = 0; j < 64; ++j) {
+        const float pj = Ps[w][j];
+        a0 = fmaf(pj, Vs[j][lane], a0);
+        a1 = fmaf(pj, Vs[j][lane + 32], a1);
+      }
+      o0[t] = a0;
+      o1[t] = a1;
+      __syncwarp();
+    }
+  }
+#pragma unroll
+  for (int t = 0; t < QW; ++t) {
+    const int q = q0 + w * QW + t;
+    if (q >= m) continue;
+    float* op = out + (rb + q) * d + h * 64;
+    op[lane] = o0[t] / l[t];
+    op[lane + 32] = o1[t] / l[t];
+  }
 }
 
-// Routing + injection (Eq. inj-gate / inj-add) in fp32, one thread per output
-// element of X_out.  D is [B*m*k2, k1*d] in proxy order; token t of block i
-// reads the row of proxy i - shift.
+// Routing + injection (Eq. inj-gate / inj-add) in fp32, four channels per
+// thread.  D is [B*m*k2, k1*d] in proxy order; token t of block i reads the
+// row of proxy i - shift.
 __global__ void inject_f32_kernel(const float* __restrict__ X, const float* __restrict__ D,
                                   float* __restrict__ Xo, const float* __restrict__ w_x,
                                   const float* __restrict__ w_dlt, const float* __restrict__ b_g,
                                   long L, int d, int P, int k1, int k2, int m, int shift, int gated,
-                                  long total) {
-  const long e = (long)blockIdx.x * blockDim.x + threadIdx.x;
-  if (e >= total) return;
-  const long t = (e / d) % L, b = e / ((long)L * d);
-  const int ch = (int)(e % d);
-  const long i = t / P, p = t % P;
-  const float x = X[e];
+                                  long total4) {
+  const long e4 = (long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (e4 >= total4) return;
+  const int d4 = d >> 2;
+  const long tokg = e4 / d4;  // global token (b * L + t)
+  const int ch = (int)(e4 - tokg * d4) * 4;
+  const long b = tokg / L, t = tokg - b * L;
+  const long i = t / P, p = t - i * P;
+  const float4 x = *reinterpret_cast<const float4*>(X + e4 * 4);
   if (i < shift) {
-    Xo[e] = x;
+    *reinterpret_cast<float4*>(Xo + e4 * 4) = x;
     return;
   }
   const long prox = b * m + (i - shift);
   const long row = prox * k2 + p / k1;
-  const float dv = D[row * ((long)k1 * d) + (p % k1) * d + ch];
+  const float4 dv = *reinterpret_cast<const float4*>(D + row * ((long)k1 * d) + (p % k1) * d + ch);
+  float4 o;
   if (gated) {
-    const float g = w_x[ch] * x + w_dlt[ch] * dv + b_g[ch];
-    Xo[e] = x + dv / (1.f + expf(-g));
+    const float4 wx = *reinterpret_cast<const float4*>(w_x + ch);
+    const float4 wd = *reinterpret_cast<const float4*>(w_dlt + ch);
+    const float4 bg = *reinterpret_cast<const float4*>(b_g + ch);
+    o.x = x.x + dv.x / (1.f + expf(-(wx.x * x.x + wd.x * dv.x + bg.x)));
+    o.y = x.y + dv.y / (1.f + expf(-(wx.y * x.y + wd.y * dv.y + bg.y)));
+    o.z = x.z + dv.z / (1.f + expf(-(wx.z * x.z + wd.z * dv.z + bg.z)));
+    o.w = x.w + dv.w / (1.f + expf(-(wx.w * x.w + wd.w * dv.w + bg.w)));
   } else {
-    Xo[e] = x + dv;
+    o = make_float4(x.x + dv.x, x.y + dv.y, x.z + dv.z, x.w + dv.w);
   }
+  *reinterpret_cast<float4*>(Xo + e4 * 4) = o;
 }
 
 __global__ void pad_f32_kernel(const float* __restrict__ src, float* __restrict__ dst, long L,
@@ -162,8 +265,8 @@ __global__ void splitk_f32_reduce(const float* __restrict__ part, int S, int M, 
 int splitk_f32_factor(int M, int N, int K) {
   const long tiles = (long)((M + FT - 1) / FT) * ((N + FT - 1) / FT);
   if (tiles >= 304) return 1;
-  int S = (int)((304 + tiles - 1) / tiles);
-  S = std::min(S, std::max(1, K / 512));
+  int S = (int)((304 + tiles - 1) / tiles);  // about two CTAs per SM of a 152-SM part
+  S = std::min(S, std::max(1, K / 64));       // at least two 32-wide K slabs per slice
   return std::min(S, 64);
 }
 
@@ -191,21 +294,20 @@ cudaError_t gemm_f32(int M, int N, int K, const float* A, long lda, const float*
 
 cudaError_t attn_f32(const float* qkv, float* out, int B, int m, int d, int nh, bool causal,
                      cudaStream_t st) {
-  const long warps = (long)B * nh * m;
   const double pairs = (double)B * nh * (causal ? 0.5 * m * (m + 1.0) : (double)m * m);
   LaunchTimer lt("attn_f32", st, 4.0 * 64 * pairs, 4.0 * B * m * 4.0 * d);
-  attn_f32_kernel<<<(unsigned)((warps * 32 + 255) / 256), 256, 0, st>>>(
-      qkv, out, B, m, d, nh, causal ? 1 : 0, 1.0f / sqrtf(64.0f));
+  dim3 grid((m + ATT_Q - 1) / ATT_Q, nh, B);
+  attn_f32_kernel<<<grid, 256, 0, st>>>(qkv, out, m, d, causal ? 1 : 0, 1.0f / sqrtf(64.0f));
   return cudaGetLastError();
 }
 
 cudaError_t inject_f32(const float* X, const float* D, float* Xo, const float* w_x,
                        const float* w_dlt, const float* b_g, int B, long L, int d, int P, int k1,
                        int k2, int m, int shift, int gated, cudaStream_t st) {
-  const long total = (long)B * L * d;
-  LaunchTimer lt("inject_f32", st, 0.0, 12.0 * total);
-  inject_f32_kernel<<<(unsigned)((total + 255) / 256), 256, 0, st>>>(
-      X, D, Xo, w_x, w_dlt, b_g, L, d, P, k1, k2, m, shift, gated, total);
+  const long total4 = (long)B * L * d / 4;
+  LaunchTimer lt("inject_f32", st, 0.0, 48.0 * total4);
+  inject_f32_kernel<<<(unsigned)((total4 + 255) / 256), 256, 0, st>>>(
+      X, D, Xo, w_x, w_dlt, b_g, L, d, P, k1, k2, m, shift, gated, total4);
   return cudaGetLastError();
 }
 
