@@ -40,8 +40,8 @@ constexpr int GEMM_THREADS = 64 + 32 * GEMM_EPI_WARPS;
 // column in shared memory (two tiles' worth, filled one tile ahead).
 template <int BN, int XCOLS, bool PAR = false>
 struct GemmCfg {
-  static constexpr int STAGES = XCOLS ? (BN == 256 && XCOLS == 256 ? 3 : (BN == 256 ? 4 : 5))
-                                      : (BN == 256 ? 4 : 6);
+  static constexpr int STAGES =
+      XCOLS ? (BN == 256 && (XCOLS == 256 || PAR) ? 3 : (BN == 256 ? 4 : 5)) : (BN == 256 ? 4 : 6);
   static constexpr uint32_t A_BYTES = GEMM_BM * GEMM_BK * 2;  // 16 KB
   static constexpr uint32_t B_BYTES = BN * GEMM_BK * 2;       // 16/32 KB
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
@@ -111,7 +111,6 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   constexpr int XCOLS = Epi::kXTile ? (Epi::kPaired ? BN / 2 : BN) : 0;
   using Cfg = GemmCfg<BN, XCOLS, Epi::kColPar>;
   constexpr int STAGES = Cfg::STAGES;
-  static_assert(!Epi::kColPar || !Epi::kPaired, "column parameters: unpaired epilogues only");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -304,7 +303,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
 #pragma unroll
             for (int i = 0; i < 32; ++i) v[i] = w[i] = 0.f;
           }
-          epi.apply_pair(ri, erow, n0, c, v, w, xtile, rl);
+          epi.apply_pair(ri, erow, n0, c, v, w, xtile, rl, cp);
         }
       } else {
         // 32-column chunks, the TMEM load of chunk i+1 in flight while chunk i
@@ -383,8 +382,8 @@ struct EpiBase {
   __device__ __forceinline__ int x_col(int n0, int j) const { return n0 + 64 * j; }
   __device__ __forceinline__ int b_row(int n0, int j) const { return n0 + 128 * j; }
   template <class R>
-  __device__ __forceinline__ void apply_pair(const R&, int, int, int, float*, float*,
-                                             const uint8_t*, int) const {}
+  __device__ __forceinline__ void apply_pair(const R&, int, int, int, float*, float*, uint8_t*,
+                                             int, const float4*) const {}
 };
 
 // v = acc (+ bias[col]) (+ addend[row, col]); stored as fp32 and/or bf16.
@@ -667,27 +666,58 @@ struct EpiAffine2D : EpiBase {
     r.rs = stats[2 * tok + 1];
     return r;
   }
+  // staged per column c of the s half: (bias of s, bias of t)
+  static constexpr bool kColPar = true;
+  __device__ __forceinline__ float4 col_param(int n0, int cl) const {
+    if (cl >= 128) return make_float4(0.f, 0.f, 0.f, 0.f);
+    const float* bs = bias + (long)ptok(n0) * 2 * d + cbase(n0) + cl;
+    return make_float4(bs[0], bs[d], 0.f, 0.f);
+  }
+  // The warp's 32 x 32 chunk of X_out and then of S is staged in the X tile
+  // cells it has just read and stored with whole-row segments.
   __device__ __forceinline__ void apply_pair(const Row& ri, int row, int n0, int c, float* vs,
-                                             float* vt, const uint8_t* xt, int rl) const {
-    if (!ri.ok) return;
-    const int p = ptok(n0), ch0 = cbase(n0) + c;
-    const float* bs = bias + (long)p * 2 * d + ch0;
-    const float* bt = bs + d;
-    bf16* so = S_save + (long)row * (patch * patch * d) + (long)p * d + ch0;
-    bf16* xo = X_out + ri.xoff + c;
+                                             float* vt, uint8_t* xt, int rl,
+                                             const float4* cp) const {
+    const int q = rl >> 5, p = ptok(n0), ch0 = cbase(n0) + c;
+    const float4* cg = cp + (c >> 2) * 4;
 #pragma unroll
     for (int i8 = 0; i8 < 32; i8 += 8) {
-      float x[8], o[8], sv[8];
+      float x[8], o[8];
       xtile_load8(xt, rl, c + i8, x);
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        sv[j] = vs[i8 + j] + bs[i8 + j];
-        const float t = vt[i8 + j] + bt[i8 + j];
-        o[j] = fmaf(1.f + sv[j], (x[j] - ri.mu) * ri.rs, t);
+      for (int h = 0; h < 2; ++h) {
+        const int g4 = (i8 >> 2) + h;
+        const float4 bs = cg[g4 * 4], bt = cg[g4 * 4 + 1];
+        const float bsa[4] = {bs.x, bs.y, bs.z, bs.w}, bta[4] = {bt.x, bt.y, bt.z, bt.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int e = h * 4 + j;
+          const float sv = vs[i8 + e] + bsa[j];
+          vs[i8 + e] = sv;
+          o[e] = fmaf(1.f + sv, (x[e] - ri.mu) * ri.rs, vt[i8 + e] + bta[j]);
+        }
       }
-      store8_bf16(so + i8, sv);
-      store8_bf16(xo + i8, o);
+      xtile_put8(xt, rl, c + i8, o);
     }
+    __syncwarp();
+    const long long off = ri.xoff;
+    const int okr = ri.ok ? 1 : 0;
+    warp_store_rows(xt, q, c, [&](int rr, int pc) -> bf16* {
+      const long long o2 = __shfl_sync(0xffffffffu, off, rr);
+      const int k2 = __shfl_sync(0xffffffffu, okr, rr);
+      return k2 ? X_out + o2 + c + pc * 8 : nullptr;
+    });
+    __syncwarp();
+#pragma unroll
+    for (int i8 = 0; i8 < 32; i8 += 8) xtile_put8(xt, rl, c + i8, vs + i8);
+    __syncwarp();
+    const int rfirst = row - (rl & 31);
+    const long pd = (long)patch * patch * d;
+    warp_store_rows(xt, q, c, [&](int rr, int pc) -> bf16* {
+      const int r2 = rfirst + rr;
+      return r2 < M ? S_save + (long)r2 * pd + (long)p * d + ch0 + pc * 8 : nullptr;
+    });
+    __syncwarp();
   }
 };
 
