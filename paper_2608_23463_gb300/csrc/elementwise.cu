@@ -1,6 +1,8 @@
 // Bandwidth-bound kernels of the layer: injection backward with its column
 // reductions, deterministic column sums (bias gradients), block-0 copies and
 // zero padding.  All accesses are 16-byte vectors over contiguous rows.
+#include <algorithm>
+
 #include "kernels.h"
 
 namespace pf {
@@ -27,15 +29,6 @@ __global__ void pad_rows_kernel(const bf16* __restrict__ src, bf16* __restrict__
   uint4 v = make_uint4(0, 0, 0, 0);
   if (tok < L) v = *reinterpret_cast<const uint4*>(src + (long)b * L * d + i * 8);
   *reinterpret_cast<uint4*>(dst + (long)b * Lp * d + i * 8) = v;
-}
-
-__device__ __forceinline__ void load4_bf16(const bf16* p, float* v) {
-  const uint2 u = *reinterpret_cast<const uint2*>(p);
-  const float2 a = unpack_bf16(u.x), b = unpack_bf16(u.y);
-  v[0] = a.x; v[1] = a.y; v[2] = b.x; v[3] = b.y;
-}
-__device__ __forceinline__ void store4_bf16(bf16* p, const float* v) {
-  *reinterpret_cast<uint2*>(p) = make_uint2(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]));
 }
 
 // Each thread owns 8 consecutive columns (16-byte vectors) and walks a
@@ -167,6 +160,198 @@ __global__ void __launch_bounds__(EW_THREADS, 2) inj_bwd_kernel(InjBwdArgs a, fl
   }
 }
 
+// Streaming form for slices of IB_W columns (N a multiple of IB_W): two
+// 256-thread CTAs per SM, each owning one column slice and a contiguous range
+// of rows;
+// thread 0 pulls each row's slices of D, G and X (contiguous, 4 KB each) with
+// cp.async.bulk into an IB_STAGES-deep ring of IB_R-row stages, so the bytes
+// in flight per SM do not depend on registers.  Thread t handles columns
+// [8t, 8t+8) of the slice; the arithmetic and the partial sums are those of
+// inj_bwd_kernel.
+constexpr int IB_W = 2048;
+constexpr int IB_R = 2;
+constexpr int IB_STAGES = 4;
+constexpr uint32_t IB_ROW_BYTES = IB_W * 2;
+constexpr uint32_t IB_STAGE_BYTES = 3 * IB_R * IB_ROW_BYTES;  // [D | G | X] x IB_R rows
+constexpr uint32_t IB_SMEM = IB_STAGES * IB_STAGE_BYTES + 128;
+
+struct IbRow {
+  bool valid;   // the row has target tokens
+  int lim;      // valid columns of the row (tokens < L), 0 if none
+  long gx_off;  // element offset of the row's tokens in G / X
+  long dx_off;  // element offset in dX
+};
+
+__device__ __forceinline__ IbRow ib_row(const InjBwdArgs& a, const RowIdx& ix, int N) {
+  IbRow r{false, 0, 0, 0};
+  const int it = ix.i + a.shift;
+  const long tok0 = (long)it * (a.k1 * a.k2) + (long)ix.grp * a.k1;
+  if (it < a.m && tok0 < a.L) {
+    r.valid = true;
+    const long lim = (a.L - tok0) * a.d;
+    r.lim = lim < N ? (int)lim : N;
+    r.gx_off = ((long)ix.b * a.L + tok0) * a.d;
+    r.dx_off = ((long)ix.b * a.Ldx + tok0) * a.d;
+  }
+  return r;
+}
+
+__global__ void __launch_bounds__(256, 2) inj_bwd_stream_kernel(InjBwdArgs a,
+                                                               float* __restrict__ part, long M,
+                                                               int N, long rows_per_chunk) {
+  extern __shared__ __align__(128) uint8_t ib_smem[];
+  __shared__ __align__(8) uint64_t full[IB_STAGES];
+  const int tid = threadIdx.x;
+  const int col0 = blockIdx.x * IB_W, col = col0 + tid * 8;
+  const long r0 = (long)blockIdx.y * rows_per_chunk;
+  const long r1 = min(M, r0 + rows_per_chunk);
+  const int nst = (int)((max(r1 - r0, 0L) + IB_R - 1) / IB_R);
+  const uint32_t sm0 = smem_u32(ib_smem), bar0 = smem_u32(full);
+  RowIdx ix0;
+  {
+    const long prox = r0 / a.k2;
+    ix0.grp = (int)(r0 % a.k2);
+    ix0.b = (int)(prox / a.m);
+    ix0.i = (int)(prox % a.m);
+  }
+  if (tid == 0) {
+    for (int i = 0; i < IB_STAGES; ++i) mbar_init(bar0 + 8 * i, 1);
+    fence_barrier_init();
+  }
+  __syncthreads();
+  // producer state (thread 0): next stage to issue and the row index there
+  int issued = 0;
+  RowIdx pix = ix0;
+  auto issue = [&]() {
+    const int st = issued % IB_STAGES;
+    const uint32_t base = sm0 + st * IB_STAGE_BYTES, bar = bar0 + 8 * st;
+    const long rs = r0 + (long)issued * IB_R;
+    uint32_t bytes = 0;
+    uint32_t dbytes[IB_R], gbytes[IB_R];
+    long goff[IB_R];
+    for (int u = 0; u < IB_R; ++u) {
+      dbytes[u] = gbytes[u] = 0;
+      goff[u] = 0;
+      if (rs + u < r1) {
+        dbytes[u] = IB_ROW_BYTES;
+        const IbRow rr = ib_row(a, pix, N);
+        if (rr.valid && rr.lim > col0) {
+          gbytes[u] = (uint32_t)(min(rr.lim - col0, IB_W)) * 2u;
+          goff[u] = rr.gx_off + col0;
+        }
+        pix.next(a.k2, a.m);
+      }
+      bytes += dbytes[u] + 2 * gbytes[u];
+    }
+    mbar_arrive_expect_tx(bar, bytes);
+    for (int u = 0; u < IB_R; ++u) {
+      if (dbytes[u])
+        bulk_load(base + u * IB_ROW_BYTES, a.D + (rs + u) * N + col0, dbytes[u], bar);
+      if (gbytes[u]) {
+        bulk_load(base + (IB_R + u) * IB_ROW_BYTES, a.G + goff[u], gbytes[u], bar);
+        bulk_load(base + (2 * IB_R + u) * IB_ROW_BYTES, a.X + goff[u], gbytes[u], bar);
+      }
+    }
+    ++issued;
+  };
+  if (tid == 0)
+    while (issued < min(IB_STAGES, nst)) issue();
+
+  const int ch = col % a.d;
+  float wx[8], wd[8], bg[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    wx[j] = a.gated ? a.w_x[ch + j] : 0.f;
+    wd[j] = a.gated ? a.w_dlt[ch + j] : 0.f;
+    bg[j] = a.gated ? a.b_g[ch + j] : 0.f;
+  }
+  float acc[4][8] = {};
+  RowIdx ix = ix0;
+  bool failed = false;
+  int s = 0;
+  for (; s < nst; ++s) {
+    const int st = s % IB_STAGES;
+    const bool ok = mbar_wait(bar0 + 8 * st, (s / IB_STAGES) & 1);
+    const uint8_t* base = ib_smem + st * IB_STAGE_BYTES + tid * 16;
+    const long rs = r0 + (long)s * IB_R;
+#pragma unroll
+    for (int u = 0; u < IB_R; ++u) {
+      const long r = rs + u;
+      if (r >= r1) break;
+      const IbRow rr = ib_row(a, ix, N);
+      ix.next(a.k2, a.m);
+      if (!ok) continue;
+      const bool v = rr.valid && col < rr.lim;
+      float dd[8];
+      if (v) {
+        const uint4 gv = *reinterpret_cast<const uint4*>(base + (IB_R + u) * IB_ROW_BYTES);
+        const uint4 xv = *reinterpret_cast<const uint4*>(base + (2 * IB_R + u) * IB_ROW_BYTES);
+        const uint4 dv = *reinterpret_cast<const uint4*>(base + u * IB_ROW_BYTES);
+        float g[8], x[8], Dv[8], dx[8];
+        const uint32_t *pg = &gv.x, *px = &xv.x, *pd = &dv.x;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float2 a2 = unpack_bf16(pg[q]), b2 = unpack_bf16(px[q]), c2 = unpack_bf16(pd[q]);
+          g[2 * q] = a2.x; g[2 * q + 1] = a2.y;
+          x[2 * q] = b2.x; x[2 * q + 1] = b2.y;
+          Dv[2 * q] = c2.x; Dv[2 * q + 1] = c2.y;
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          if (a.gated) {
+            const float sg = sigmoidf_(fmaf(wx[j], x[j], fmaf(wd[j], Dv[j], bg[j])));
+            const float ds = g[j] * Dv[j] * sg * (1.f - sg);
+            dx[j] = fmaf(ds, wx[j], g[j]);
+            dd[j] = fmaf(g[j], sg, ds * wd[j]);
+            acc[1][j] = fmaf(ds, x[j], acc[1][j]);
+            acc[2][j] = fmaf(ds, Dv[j], acc[2][j]);
+            acc[3][j] += ds;
+          } else {
+            dx[j] = g[j];
+            dd[j] = g[j];
+          }
+        }
+        store8_bf16(a.dX + rr.dx_off + col, dx);
+      } else {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) dd[j] = 0.f;
+      }
+      uint4 o;
+      o.x = pack_bf16(dd[0], dd[1]);
+      o.y = pack_bf16(dd[2], dd[3]);
+      o.z = pack_bf16(dd[4], dd[5]);
+      o.w = pack_bf16(dd[6], dd[7]);
+      *reinterpret_cast<uint4*>(a.dD + r * N + col) = o;
+      const uint32_t* po = &o.x;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float2 f = unpack_bf16(po[q]);
+        acc[0][2 * q] += f.x;
+        acc[0][2 * q + 1] += f.y;
+      }
+    }
+    // every thread is done with stage st: refill it (or leave together)
+    if (__syncthreads_or(!ok)) {
+      failed = true;
+      break;
+    }
+    if (tid == 0 && issued < nst) issue();
+  }
+  if (failed) {  // a wait ran out: let this CTA's own copies land, then leave
+    if (tid == 0)
+      for (int it = s; it < issued; ++it)
+        mbar_wait_drain(bar0 + 8 * (it % IB_STAGES), (it / IB_STAGES) & 1);
+    __syncthreads();
+    return;
+  }
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    float* p = part + ((long)blockIdx.y * 4 + q) * N + col;
+    *reinterpret_cast<float4*>(p) = make_float4(acc[q][0], acc[q][1], acc[q][2], acc[q][3]);
+    *reinterpret_cast<float4*>(p + 4) = make_float4(acc[q][4], acc[q][5], acc[q][6], acc[q][7]);
+  }
+}
+
 // Deterministic warp sum: lane j adds summands j, j+32, ... in order, then a
 // fixed xor-shuffle tree.
 __device__ __forceinline__ float warp_sum(float v) {
@@ -289,7 +474,13 @@ cudaError_t pad_rows(const bf16* src, bf16* dst, int B, long L, long Lp, int d, 
   return cudaGetLastError();
 }
 
-int inj_bwd_chunks(long M, int N) { return chunks_for(M, N); }
+int inj_bwd_chunks(long M, int N) {
+  if (N % IB_W == 0) {  // streaming form: about two CTAs per SM of a 152-SM part
+    long c = (304 + N / IB_W - 1) / (N / IB_W);  // two CTAs per SM
+    return (int)std::max(1L, std::min(c, M));
+  }
+  return chunks_for(M, N);
+}
 
 int take_dev_error_elementwise() { return take_dev_error_tu(); }
 
@@ -297,8 +488,16 @@ cudaError_t inj_bwd_1d(const InjBwdArgs& a, float* part, int n_chunks, cudaStrea
   const long M = (long)a.B * a.m * a.k2;
   const int N = a.k1 * a.d;
   const long rpc = (M + n_chunks - 1) / n_chunks;
-  dim3 grid((N / INJ_COLS + EW_THREADS - 1) / EW_THREADS, n_chunks);
   LaunchTimer lt("inj_bwd", st, 0.0, 10.0 * M * N + 16.0 * n_chunks * N);
+  if (N % IB_W == 0) {
+    cudaError_t e = cudaFuncSetAttribute(inj_bwd_stream_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, IB_SMEM);
+    if (e != cudaSuccess) return e;
+    dim3 grid(N / IB_W, n_chunks);
+    inj_bwd_stream_kernel<<<grid, 256, IB_SMEM, st>>>(a, part, M, N, rpc);
+    return cudaGetLastError();
+  }
+  dim3 grid((N / INJ_COLS + EW_THREADS - 1) / EW_THREADS, n_chunks);
   inj_bwd_kernel<<<grid, EW_THREADS, 0, st>>>(a, part, M, N, rpc);
   return cudaGetLastError();
 }

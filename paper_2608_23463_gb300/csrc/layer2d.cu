@@ -19,18 +19,20 @@ __device__ __forceinline__ float warp_sum_f(float v) {
 
 // Xp[r, (py*p + px)*d + ch] = X[b, (by*p + py)*gw + bx*p + px, ch] for patch
 // r = (b, by, bx); 16-byte copies.
-__global__ void patch_gather_kernel(const bf16* __restrict__ X, bf16* __restrict__ Xp, int d,
-                                    int patch, int gh, int gw, long total_vec) {
-  const long e = (long)blockIdx.x * blockDim.x + threadIdx.x;
-  if (e >= total_vec) return;
-  const int dv = d / 8, P = patch * patch;
-  const long row = e / ((long)P * dv);
-  const int rem = (int)(e % ((long)P * dv)), p = rem / dv, c8 = rem % dv;
+__global__ void __launch_bounds__(256) patch_gather_kernel(const bf16* __restrict__ X,
+                                                           bf16* __restrict__ Xp, int d, int patch,
+                                                           int gh, int gw, int per_row) {
+  // grid (x: patch row, y: vectors of one patch row); 16 bytes per thread
+  const int i = blockIdx.y * blockDim.x + threadIdx.x;  // vector within the patch row
+  if (i >= per_row) return;
+  const int row = blockIdx.x;
+  const int dv = d >> 3, p = i / dv, c8 = i - p * dv;
   const int npw = gw / patch, m = (gh / patch) * npw;
-  const int b = (int)(row / m), pr = (int)(row % m), by = pr / npw, bx = pr % npw;
-  const int py = p / patch, px = p % patch;
+  const int b = row / m, pr = row - b * m, by = pr / npw, bx = pr - by * npw;
+  const int py = p / patch, px = p - py * patch;
   const long src = ((long)b * gh * gw + (long)(by * patch + py) * gw + bx * patch + px) * d + c8 * 8;
-  *reinterpret_cast<uint4*>(Xp + e * 8) = *reinterpret_cast<const uint4*>(X + src);
+  *reinterpret_cast<uint4*>(Xp + (long)row * per_row * 8 + (long)i * 8) =
+      __ldcs(reinterpret_cast<const uint4*>(X + src));
 }
 
 // stats[t] = (mean, 1/sqrt(var + 1e-6)) over the d channels of token t; one
@@ -289,10 +291,11 @@ __global__ void temb_wgrad_kernel(const float* __restrict__ dgb, const float* __
 
 cudaError_t patch_gather(const bf16* X, bf16* Xp, int B, int d, int patch, int gh, int gw,
                          cudaStream_t st) {
-  const long total_vec = (long)B * gh * gw * d / 8;
+  const int per_row = patch * patch * d / 8;  // 16-byte vectors per patch
+  const int rows = B * (gh / patch) * (gw / patch);
   LaunchTimer lt("patch_gather", st, 0.0, 4.0 * B * gh * gw * (double)d);
-  patch_gather_kernel<<<(unsigned)((total_vec + 255) / 256), 256, 0, st>>>(X, Xp, d, patch, gh, gw,
-                                                                          total_vec);
+  dim3 grid(rows, (per_row + 255) / 256);
+  patch_gather_kernel<<<grid, 256, 0, st>>>(X, Xp, d, patch, gh, gw, per_row);
   return cudaGetLastError();
 }
 
