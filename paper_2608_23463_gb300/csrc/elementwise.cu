@@ -474,12 +474,17 @@ cudaError_t pad_rows(const bf16* src, bf16* dst, int B, long L, long Lp, int d, 
   return cudaGetLastError();
 }
 
+// The streaming form needs whole IB_W slices and enough rows per CTA to fill
+// its ring (about two CTAs per SM of a 152-SM part, at least 128 rows each).
+long ib_stream_chunks(long M, int N) {
+  if (N % IB_W != 0) return 0;
+  const long c = (304 + N / IB_W - 1) / (N / IB_W);
+  return M / c >= 128 ? c : 0;
+}
+
 int inj_bwd_chunks(long M, int N) {
-  if (N % IB_W == 0) {  // streaming form: about two CTAs per SM of a 152-SM part
-    long c = (304 + N / IB_W - 1) / (N / IB_W);  // two CTAs per SM
-    return (int)std::max(1L, std::min(c, M));
-  }
-  return chunks_for(M, N);
+  const long c = ib_stream_chunks(M, N);
+  return c ? (int)c : chunks_for(M, N);
 }
 
 int take_dev_error_elementwise() { return take_dev_error_tu(); }
@@ -489,7 +494,7 @@ cudaError_t inj_bwd_1d(const InjBwdArgs& a, float* part, int n_chunks, cudaStrea
   const int N = a.k1 * a.d;
   const long rpc = (M + n_chunks - 1) / n_chunks;
   LaunchTimer lt("inj_bwd", st, 0.0, 10.0 * M * N + 16.0 * n_chunks * N);
-  if (N % IB_W == 0) {
+  if (ib_stream_chunks(M, N) == n_chunks) {
     cudaError_t e = cudaFuncSetAttribute(inj_bwd_stream_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, IB_SMEM);
     if (e != cudaSuccess) return e;

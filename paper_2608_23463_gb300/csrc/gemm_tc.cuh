@@ -8,7 +8,8 @@
 //
 // Persistent: one CTA per SM walks the 128 x BN output tiles tile = blockIdx.x
 // + k * gridDim.x (N fastest, so co-running CTAs share A panels and all of B
-// in L2).  Roles:
+// in L2; M fastest when A has at most 16 row tiles and B is wider than the
+// grid, so co-running CTAs share B tiles).  Roles:
 //   warp 0   : TMA producer (one thread): STAGES-deep ring of 128B-swizzled
 //              64-wide K slices of A and B, continuing across tiles
 //   warp 1   : TMEM allocator + MMA issuer (one thread): tcgen05.mma M=128,
@@ -131,15 +132,20 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   __shared__ uint32_t s_consumed;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int num_n = (N + BN - 1) / BN;
-  const int mn_tiles = ((M + GEMM_BM - 1) / GEMM_BM) * num_n;
+  const int num_n = (N + BN - 1) / BN, num_m = (M + GEMM_BM - 1) / GEMM_BM;
+  const int mn_tiles = num_m * num_n;
+  // N fastest keeps the co-running CTAs on one A panel with all of B in L2;
+  // when A is a few row tiles and B is wider than the grid, M fastest instead
+  // lets the co-running CTAs share each B tile (B is then read once)
+  const bool m_fast = num_m <= 16 && num_n > (int)gridDim.x;
   const int tiles = mn_tiles * splits;
   const int num_k = (K + GEMM_BK - 1) / GEMM_BK;
   const int kps = (num_k + splits - 1) / splits;  // K tiles per split
   // tile t -> split t / mn_tiles (slowest), then M, then N (fastest)
 #define PF_TILE_DECODE(t)                                   \
   const int sp = (t) / mn_tiles, rem = (t) % mn_tiles;      \
-  const int m0 = (rem / num_n) * GEMM_BM, n0 = (rem % num_n) * BN; \
+  const int m0 = (m_fast ? rem % num_m : rem / num_n) * GEMM_BM;  \
+  const int n0 = (m_fast ? rem / num_m : rem % num_n) * BN;        \
   const int kb = sp * kps, ke = min(num_k, kb + kps);
   const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + STAGES);
   const uint32_t tfull0 = smem_u32(bars + 2 * STAGES), tempty0 = tfull0 + 16;
@@ -256,7 +262,10 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     const int et = threadIdx.x - 64;
     const int q = warp & 3;                               // TMEM lane quarter
     const int c_begin = ((warp - 2) >> 2) * (BN / 2);     // this warp's column half
-    auto tile_n0 = [&](int t) { return ((t % mn_tiles) % num_n) * BN; };
+    auto tile_n0 = [&](int t) {
+      const int r = t % mn_tiles;
+      return (m_fast ? r / num_m : r % num_n) * BN;
+    };
     if constexpr (Epi::kColPar) {  // parameters of the first tile
       if ((int)blockIdx.x < tiles && et < BN) cpar_put(0, et, epi.col_param(tile_n0(blockIdx.x), et));
       epi_bar_and(true);

@@ -32,6 +32,9 @@ CASES = {
     "d1024_P64": (S.LayerSpec(batch=1, L=8192, d=1024, n_heads=16, P=64), False, True),
     "d1024_P64_8x8": (S.LayerSpec(batch=1, L=16384, d=1024, n_heads=16, P=64, levels=2, k1=8,
                                   k2=8), True, True),
+    # 9728 rows of 8192: enough rows per CTA for the streaming injection backward
+    "d1024_P64_8x8_L77824": (S.LayerSpec(batch=1, L=77824, d=1024, n_heads=16, P=64, levels=2,
+                                         k1=8, k2=8), False, True),
 }
 
 
