@@ -360,30 +360,34 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
-// One warp per output: db_d1[c] = sum over chunks of part[.][0][c]; gate
-// gradients g_q[ch] = sum over chunks and the k1 token positions t of
-// part[.][q][t*d + ch] (q = 1: w_x, 2: w_dlt, 3: b_g).
-__global__ void inj_bwd_finalize_kernel(const float* __restrict__ part, int n_chunks, int N, int d,
-                                        float* db_d1, float* gw_x, float* gw_dlt, float* gb_g) {
-  const int o = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  if (o < N) {
-    float s = 0.f;
-    for (int c = lane; c < n_chunks; c += 32) s += part[((long)c * 4) * N + o];
-    s = warp_sum(s);
-    if (lane == 0) db_d1[o] = s;
-    return;
-  }
-  const int j = o - N;
-  if (gw_x == nullptr || j >= 3 * d) return;
-  const int q = 1 + j / d, ch = j % d, T = N / d;
+// Column totals of the partials, one thread per (quantity q, column), chunks
+// added in order (coalesced across threads): q = 0 gives db_d1; the totals of
+// q = 1..3 are left in chunk 0's slots of part for the gate reduction below.
+__global__ void inj_bwd_colsum_kernel(float* __restrict__ part, int n_chunks, int N,
+                                      float* __restrict__ db_d1, int gates) {
+  const long i = (long)blockIdx.x * blockDim.x + threadIdx.x;
+  const int nq = gates ? 4 : 1;
+  if (i >= (long)nq * N) return;
+  const int q = (int)(i / N), col = (int)(i % N);
   float s = 0.f;
-  for (int e = lane; e < n_chunks * T; e += 32) {
-    const int c = e / T, t = e % T;
-    s += part[((long)c * 4 + q) * N + (long)t * d + ch];
-  }
-  s = warp_sum(s);
-  if (lane == 0) (q == 1 ? gw_x : (q == 2 ? gw_dlt : gb_g))[ch] = s;
+#pragma unroll 8
+  for (int c = 0; c < n_chunks; ++c) s += part[((long)c * 4 + q) * N + col];
+  if (q == 0)
+    db_d1[col] = s;
+  else
+    part[(long)q * N + col] = s;
+}
+
+// Gate gradients: g_q[ch] = sum over the k1 token positions t of the column
+// totals of quantity q (q = 1: w_x, 2: w_dlt, 3: b_g).
+__global__ void inj_bwd_gates_kernel(const float* __restrict__ part, int N, int d, float* gw_x,
+                                     float* gw_dlt, float* gb_g) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= 3 * d) return;
+  const int q = 1 + i / d, ch = i % d, T = N / d;
+  float s = 0.f;
+  for (int t = 0; t < T; ++t) s += part[(long)q * N + (long)t * d + ch];
+  (q == 1 ? gw_x : (q == 2 ? gw_dlt : gb_g))[ch] = s;
 }
 
 template <typename T>
@@ -509,10 +513,13 @@ cudaError_t inj_bwd_1d(const InjBwdArgs& a, float* part, int n_chunks, cudaStrea
 
 cudaError_t inj_bwd_finalize(const float* part, int n_chunks, int N, int d, float* db_d1,
                              float* gw_x, float* gw_dlt, float* gb_g, cudaStream_t st) {
-  const int total = N + 3 * d;
   LaunchTimer lt("inj_bwd_finalize", st, 0.0, 16.0 * n_chunks * N);
-  inj_bwd_finalize_kernel<<<(total + 7) / 8, 256, 0, st>>>(part, n_chunks, N, d, db_d1, gw_x,
-                                                          gw_dlt, gb_g);
+  const int gates = gw_x != nullptr ? 1 : 0;
+  const long n = (long)(gates ? 4 : 1) * N;
+  float* pw = const_cast<float*>(part);  // the column totals reuse chunk 0's slots
+  inj_bwd_colsum_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(pw, n_chunks, N, db_d1, gates);
+  if (gates)
+    inj_bwd_gates_kernel<<<(3 * d + 255) / 256, 256, 0, st>>>(part, N, d, gw_x, gw_dlt, gb_g);
   return cudaGetLastError();
 }
 

@@ -108,7 +108,12 @@ cudaError_t gemm_dispatch(int M, int N, int K, Operand A, Operand B, const Epi& 
   const long tiles256 = (long)((N + 255) / 256) * ((M + GEMM_BM - 1) / GEMM_BM);
   LaunchTimer lt(gemm_tag_label(), st, 2.0 * M * N * (double)K,
                  2.0 * ((double)M * K + (double)N * K) + gemm_tag_bytes());
-  if (Epi::kPaired || (N >= 256 && tiles256 >= num_sms()))
+  // 128 x 256 tiles move about 2/3 of the shared-memory bytes per FLOP of
+  // 128 x 128 tiles (the mainloop's bound); take them unless they need more
+  // than 1.5x the waves
+  const long tiles128 = (long)((N + 127) / 128) * ((M + GEMM_BM - 1) / GEMM_BM);
+  const long sms = num_sms(), w256 = (tiles256 + sms - 1) / sms, w128 = (tiles128 + sms - 1) / sms;
+  if (Epi::kPaired || (N >= 256 && 3 * w256 <= 2 * w128))
     return launch_majors<256>(M, N, K, A, B, ta, tb, tx, epi, st);
   return launch_majors<128>(M, N, K, A, B, ta, tb, tx, epi, st);
 }

@@ -193,6 +193,7 @@ int inj_bwd_chunks(long M, int N);
 cudaError_t inj_bwd_1d(const InjBwdArgs& a, float* part, int n_chunks, cudaStream_t st);
 // Reduce the partials: db_d1[c] = sum part[.][0][c]; gate grads (if non-null)
 // summed over chunks and the k1 token positions: g[ch] = sum part[.][j][q*d+ch].
+// part is scratch: its chunk-0 slots hold the column totals afterwards.
 cudaError_t inj_bwd_finalize(const float* part, int n_chunks, int N, int d, float* db_d1,
                              float* gw_x, float* gw_dlt, float* gb_g, cudaStream_t st);
 
