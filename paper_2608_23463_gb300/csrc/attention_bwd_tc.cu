@@ -7,15 +7,18 @@
 //   DKDV: item = (128-key tile, head, sequence); stationary X1 = K, X2 = V;
 //         streamed 64-query tiles Y1 = Q_j, Y2 = dO_j.
 //           T1 = X1 Y1^T = S^T,  T2 = X2 Y2^T = dP^T     (TMEM, M=128 N=64)
-//           E1 = P^T, E2 = dS^T  (bf16, shared memory, by the row warps)
-//           dV += E1 Y2,  dK += E2 Y1                    (TMEM accumulators)
+//           E1 = P^T, E2 = dS^T  (bf16, written to TMEM by the row warps)
+//           dV += E1 Y2,  dK += E2 Y1    (A from TMEM; TMEM accumulators)
 //   DQ:   item = (128-query tile, head, sequence); stationary X1 = Q, X2 = dO;
 //         streamed 64-key tiles Y1 = K_j, Y2 = V_j.
 //           T1 = S,  T2 = dP,  E2 = dS,  dQ += E2 Y1
 // Roles: warp 0 TMA producer, warp 1 MMA issuer, warps 2-9 the row warps: two
 // per TMEM lane quarter, each thread one row (TMEM lane) and one half of the
 // 64 streamed columns.  T1/T2 and E are double-buffered so the MMAs of step
-// j+1 overlap the row work of step j.  Every wait is bounded.
+// j+1 overlap the row work of step j.  E stays in TMEM as the A operand of the
+// accumulating MMAs, so those read only their B tile from shared memory
+// (shared-memory bandwidth, not the tensor pipe, bounds M=128 N=64 MMAs whose
+// operands both come from shared memory).  Every wait is bounded.
 #include <algorithm>
 #include <type_traits>
 
@@ -33,14 +36,15 @@ constexpr int BW_ROW_THREADS = 256;  // warps 2-9
 constexpr int BW_THREADS = 64 + BW_ROW_THREADS;
 constexpr uint32_t BW_X_BYTES = BW_M * BW_D * 2;  // 16 KB per stationary tile
 constexpr uint32_t BW_Y_BYTES = BW_N * BW_D * 2;  // 8 KB per streamed tile
-constexpr uint32_t BW_E_BYTES = BW_M * BW_N * 2;  // 16 KB per E tile
-constexpr uint32_t BW_OFF_Y = 2 * 2 * BW_X_BYTES;                      // X: [2 bufs][X1, X2]
-constexpr uint32_t BW_OFF_E = BW_OFF_Y + BW_STAGES * 2 * BW_Y_BYTES;  // Y: [stage][Y1, Y2]
-constexpr uint32_t BW_OFF_LD = BW_OFF_E + 2 * 2 * BW_E_BYTES;         // E: [2 bufs][E1, E2]
-constexpr uint32_t BW_OFF_BAR = BW_OFF_LD + 2 * BW_N * 8;             // (lse, Di) [2][64]
+constexpr uint32_t BW_OFF_Y = 2 * 2 * BW_X_BYTES;                       // X: [2 bufs][X1, X2]
+constexpr uint32_t BW_OFF_LD = BW_OFF_Y + BW_STAGES * 2 * BW_Y_BYTES;  // Y: [stage][Y1, Y2]
+constexpr uint32_t BW_OFF_BAR = BW_OFF_LD + 2 * BW_N * 8;              // (lse, Di) [2][64]
 constexpr uint32_t BW_SMEM = BW_OFF_BAR + 256 + 1024;
-// TMEM: T1 at 0 / 64, T2 at 128 / 192, accumulators at 256 (dV or dQ), 320 (dK)
+// TMEM columns: T1 at 0 / 64, T2 at 128 / 192 (fp32, per buffer), accumulators
+// at 256 (dV or dQ) and 320 (dK), E at 384 / 448 (per buffer: E1 at +0, E2 at
+// +32, bf16 pairs: streamed column c in 32-bit column c / 2)
 constexpr uint32_t BW_TMEM_COLS = 512;
+constexpr uint32_t BW_TM_E = 384;
 
 struct BwArgs {
   bf16* dqkv;         // [B*m, 3d]
@@ -178,8 +182,9 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
         y_issued = G + 1;
       }
     }
-  } else if (warp == 1 && lane == 0) {
+  } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
+    // The whole warp runs the loop; one elected lane issues and commits.
     constexpr uint32_t idesc_t = idesc_bf16_f32(BW_M, BW_N, 0, 0);
     constexpr uint32_t idesc_a = idesc_bf16_f32(BW_M, BW_D, 0, 1);
     bool ok = true;
@@ -187,27 +192,28 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
     // accumulate step G (local step j of its item): E_G times the step's Y tiles
     auto acc_step = [&](uint32_t G_, int j, uint32_t it_) -> bool {
       const uint32_t eb = G_ & 1, st = G_ % BW_STAGES;
-      if (!mbar_wait(e_full + 8 * eb, (G_ >> 1) & 1)) return false;
-      if (j == 0 && !mbar_wait(acc_free, (it_ & 1) ^ 1)) return false;
+      if (!mbar_wait_warp(e_full + 8 * eb, (G_ >> 1) & 1)) return false;
+      if (j == 0 && !mbar_wait_warp(acc_free, (it_ & 1) ^ 1)) return false;
       tc_fence_after();
-      const uint32_t e1 = sbase + BW_OFF_E + eb * 2 * BW_E_BYTES, e2 = e1 + BW_E_BYTES;
+      const uint32_t e1 = tmem + BW_TM_E + eb * 64, e2 = e1 + 32;
       const uint32_t y1 = sbase + BW_OFF_Y + st * 2 * BW_Y_BYTES, y2 = y1 + BW_Y_BYTES;
+      if (elect_one()) {
 #pragma unroll
-      for (int kk = 0; kk < BW_N / 16; ++kk) {
-        const uint32_t acc = (j > 0 || kk > 0) ? 1u : 0u;
-        const uint64_t bd1 = smem_desc_sw128(y1 + kk * 2048, 8192, 1024);
-        const uint64_t ad2 = smem_desc_sw128(e2 + kk * 32, 16, 1024);
-        if (DKDV) {
-          const uint64_t ad1 = smem_desc_sw128(e1 + kk * 32, 16, 1024);
-          const uint64_t bd2 = smem_desc_sw128(y2 + kk * 2048, 8192, 1024);
-          tc_mma_f16(tmem + 256, ad1, bd2, idesc_a, acc);  // dV += P^T dO
-          tc_mma_f16(tmem + 320, ad2, bd1, idesc_a, acc);  // dK += dS^T Q
-        } else {
-          tc_mma_f16(tmem + 256, ad2, bd1, idesc_a, acc);  // dQ += dS K
+        for (int kk = 0; kk < BW_N / 16; ++kk) {
+          const uint32_t acc = (j > 0 || kk > 0) ? 1u : 0u;
+          const uint64_t bd1 = smem_desc_sw128(y1 + kk * 2048, 8192, 1024);
+          if (DKDV) {
+            const uint64_t bd2 = smem_desc_sw128(y2 + kk * 2048, 8192, 1024);
+            tc_mma_f16_ts(tmem + 256, e1 + kk * 8, bd2, idesc_a, acc);  // dV += P^T dO
+            tc_mma_f16_ts(tmem + 320, e2 + kk * 8, bd1, idesc_a, acc);  // dK += dS^T Q
+          } else {
+            tc_mma_f16_ts(tmem + 256, e2 + kk * 8, bd1, idesc_a, acc);  // dQ += dS K
+          }
         }
+        tc_commit(e_free + 8 * eb);
+        tc_commit(y_empty + 8 * st);
       }
-      tc_commit(e_free + 8 * eb);
-      tc_commit(y_empty + 8 * st);
+      __syncwarp();
       return true;
     };
     for (int rd = 0, k = bw_rank(blockIdx.x, 0); k < a.n_items && ok;
@@ -215,37 +221,42 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
       int t, h, b, j0, n;
       bw_item<DKDV>(a, k, t, h, b, j0, n);
       const uint32_t xb = it & 1;
-      if (!mbar_wait(x_full + 8 * xb, (it >> 1) & 1)) break;
+      if (!mbar_wait_warp(x_full + 8 * xb, (it >> 1) & 1)) break;
       tc_fence_after();
       const uint32_t x1 = sbase + xb * 2 * BW_X_BYTES, x2 = x1 + BW_X_BYTES;
       for (int j = 0; j < n; ++j) {
         const uint32_t Gj = G + j, st = Gj % BW_STAGES, tb = Gj & 1;
-        if (!mbar_wait(y_full + 8 * st, (Gj / BW_STAGES) & 1) ||
-            !mbar_wait(t_free + 8 * tb, ((Gj >> 1) & 1) ^ 1)) {
+        if (!mbar_wait_warp(y_full + 8 * st, (Gj / BW_STAGES) & 1) ||
+            !mbar_wait_warp(t_free + 8 * tb, ((Gj >> 1) & 1) ^ 1)) {
           ok = false;
           break;
         }
         tc_fence_after();
         const uint32_t y1 = sbase + BW_OFF_Y + st * 2 * BW_Y_BYTES, y2 = y1 + BW_Y_BYTES;
+        if (elect_one()) {
 #pragma unroll
-        for (int kk = 0; kk < BW_D / 16; ++kk) {
-          tc_mma_f16(tmem + tb * BW_N, smem_desc_sw128(x1 + kk * 32, 16, 1024),
-                     smem_desc_sw128(y1 + kk * 32, 16, 1024), idesc_t, kk ? 1u : 0u);
-          tc_mma_f16(tmem + 128 + tb * BW_N, smem_desc_sw128(x2 + kk * 32, 16, 1024),
-                     smem_desc_sw128(y2 + kk * 32, 16, 1024), idesc_t, kk ? 1u : 0u);
+          for (int kk = 0; kk < BW_D / 16; ++kk) {
+            tc_mma_f16(tmem + tb * BW_N, smem_desc_sw128(x1 + kk * 32, 16, 1024),
+                       smem_desc_sw128(y1 + kk * 32, 16, 1024), idesc_t, kk ? 1u : 0u);
+            tc_mma_f16(tmem + 128 + tb * BW_N, smem_desc_sw128(x2 + kk * 32, 16, 1024),
+                       smem_desc_sw128(y2 + kk * 32, 16, 1024), idesc_t, kk ? 1u : 0u);
+          }
+          tc_commit(t_full + 8 * tb);
+          if (j == n - 1) tc_commit(x_empty + 8 * xb);
         }
-        tc_commit(t_full + 8 * tb);
-        if (j == n - 1) tc_commit(x_empty + 8 * xb);
+        __syncwarp();
         if (j > 0 && !acc_step(Gj - 1, j - 1, it)) {
           ok = false;
           break;
         }
       }
       if (!ok || !acc_step(G + n - 1, n - 1, it)) break;
-      tc_commit(acc_full);
+      if (elect_one()) tc_commit(acc_full);
+      __syncwarp();
       G += n;
     }
-    tc_commit(done);
+    if (elect_one()) tc_commit(done);
+    __syncwarp();
   } else if (warp >= 2) {
     // ------------------------------------------------------------ row warps
     const int q4 = warp & 3;
@@ -331,9 +342,8 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
           if (DKDV) continue;
           break;
         }
-        uint8_t* e1row = smem + BW_OFF_E + tb * 2 * BW_E_BYTES + r * 128;
-        uint8_t* e2row = e1row + BW_E_BYTES;
         const float2* lds = ld_s + tb * BW_N;
+        uint32_t pk[16], dk[16];  // this thread's 32 columns of E1 and E2, bf16 pairs
         // P and dS of this thread's 32 columns; columns outside [lo, hi) are
         // masked (only the diagonal and tail steps have any)
         auto emit = [&](auto masked) {
@@ -360,21 +370,22 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
               pe[e] = p;
               de[e] = p * (__uint_as_float(dv[e]) - dd);
             }
-            const int slot = (kg ^ (r & 7)) << 4;
-            if (DKDV)
-              *reinterpret_cast<uint4*>(e1row + slot) =
-                  make_uint4(pack_bf16(pe[0], pe[1]), pack_bf16(pe[2], pe[3]),
-                             pack_bf16(pe[4], pe[5]), pack_bf16(pe[6], pe[7]));
-            *reinterpret_cast<uint4*>(e2row + slot) =
-                make_uint4(pack_bf16(de[0], de[1]), pack_bf16(de[2], de[3]),
-                           pack_bf16(de[4], de[5]), pack_bf16(de[6], de[7]));
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              pk[4 * g + e] = pack_bf16(pe[2 * e], pe[2 * e + 1]);
+              dk[4 * g + e] = pack_bf16(de[2 * e], de[2 * e + 1]);
+            }
           }
         };
         if (lo <= 32 * ch && hi >= 32 * ch + 32)
           emit(std::false_type{});
         else
           emit(std::true_type{});
-        fence_proxy_async_smem();
+        const uint32_t te = tl + BW_TM_E + tb * 64 + 16 * ch;
+        if (DKDV) tmem_st16(te, pk);
+        tmem_st16(te + 32, dk);
+        tmem_wait_st();
+        tc_fence_before();
         mbar_arrive(e_full + 8 * tb);
       }
       if (DKDV) ok = bar_rows_and(ok);

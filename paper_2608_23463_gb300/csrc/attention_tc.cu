@@ -141,26 +141,31 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
         kv_issued = g + 1;
       }
     }
-  } else if (warp == 1 && lane == 0) {
+  } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
+    // The whole warp runs the loop; one elected lane issues and commits.
     constexpr uint32_t idesc_s = idesc_bf16_f32(FA_M, FA_N, 0, 0);
     constexpr uint32_t idesc_o = idesc_bf16_f32(FA_M, FA_D, 0, 1);
     bool ok = true;
     auto issue_o = [&](uint32_t G) -> bool {
       const uint32_t ob = G & 1, st = G % FA_STAGES;
-      if (!mbar_wait(p_full + 8 * ob, (G >> 1) & 1)) return false;
-      if (!mbar_wait(o_free + 8 * ob, ((G >> 1) & 1) ^ 1)) return false;
+      if (!mbar_wait_warp(p_full + 8 * ob, (G >> 1) & 1)) return false;
+      if (!mbar_wait_warp(o_free + 8 * ob, ((G >> 1) & 1) ^ 1)) return false;
       tc_fence_after();
       const uint32_t pb = sbase + FA_OFF_P + ob * FA_P_BYTES;
       const uint32_t vb = sbase + FA_OFF_KV + st * 2 * FA_KV_BYTES + FA_KV_BYTES;
+      if (elect_one()) {
 #pragma unroll
-      for (int kk = 0; kk < FA_N / 16; ++kk) {
-        const uint64_t ad = smem_desc_sw128(pb + (kk >> 2) * (FA_M * 128) + (kk & 3) * 32, 16, 1024);
-        const uint64_t bd = smem_desc_sw128(vb + kk * 2048, 8192, 1024);
-        tc_mma_f16(tmem + 256 + ob * FA_D, ad, bd, idesc_o, kk ? 1u : 0u);
+        for (int kk = 0; kk < FA_N / 16; ++kk) {
+          const uint64_t ad =
+              smem_desc_sw128(pb + (kk >> 2) * (FA_M * 128) + (kk & 3) * 32, 16, 1024);
+          const uint64_t bd = smem_desc_sw128(vb + kk * 2048, 8192, 1024);
+          tc_mma_f16(tmem + 256 + ob * FA_D, ad, bd, idesc_o, kk ? 1u : 0u);
+        }
+        tc_commit(o_full + 8 * ob);
+        tc_commit(kv_empty + 8 * st);
       }
-      tc_commit(o_full + 8 * ob);
-      tc_commit(kv_empty + 8 * st);
+      __syncwarp();
       return true;
     };
     uint32_t g = 0, it = 0;
@@ -169,23 +174,26 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       int qt, h, b, n;
       fa_item(a, k, qt, h, b, n);
       const uint32_t qb = it & 1;
-      if (!mbar_wait(q_full + 8 * qb, (it >> 1) & 1)) break;
+      if (!mbar_wait_warp(q_full + 8 * qb, (it >> 1) & 1)) break;
       tc_fence_after();
       const uint32_t qs = sbase + qb * FA_Q_BYTES;
       for (int j = 0; j < n; ++j) {
         const uint32_t G = g + j, st = G % FA_STAGES, sb = G & 1;
-        if (!mbar_wait(kv_full + 8 * st, (G / FA_STAGES) & 1)) {
+        if (!mbar_wait_warp(kv_full + 8 * st, (G / FA_STAGES) & 1)) {
           ok = false;
           break;
         }
         tc_fence_after();
         const uint32_t ks = sbase + FA_OFF_KV + st * 2 * FA_KV_BYTES;
+        if (elect_one()) {
 #pragma unroll
-        for (int kk = 0; kk < FA_D / 16; ++kk)
-          tc_mma_f16(tmem + sb * FA_N, smem_desc_sw128(qs + kk * 32, 16, 1024),
-                     smem_desc_sw128(ks + kk * 32, 16, 1024), idesc_s, kk ? 1u : 0u);
-        tc_commit(s_full + 8 * sb);
-        if (j == n - 1) tc_commit(q_empty + 8 * qb);
+          for (int kk = 0; kk < FA_D / 16; ++kk)
+            tc_mma_f16(tmem + sb * FA_N, smem_desc_sw128(qs + kk * 32, 16, 1024),
+                       smem_desc_sw128(ks + kk * 32, 16, 1024), idesc_s, kk ? 1u : 0u);
+          tc_commit(s_full + 8 * sb);
+          if (j == n - 1) tc_commit(q_empty + 8 * qb);
+        }
+        __syncwarp();
         if (j > 0 && !issue_o(G - 1)) {
           ok = false;
           break;
@@ -194,7 +202,8 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       if (!ok || !issue_o(g + n - 1)) break;
       g += n;
     }
-    tc_commit(done);
+    if (elect_one()) tc_commit(done);
+    __syncwarp();
   } else if (warp >= 2) {
     // ------------------------------------------------------------ softmax
     const int q4 = warp & 3;
