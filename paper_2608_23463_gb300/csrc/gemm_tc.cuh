@@ -215,14 +215,15 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         issued = it + 1;
       }
     }
-  } else if (warp == 1 && lane == 0) {
+  } else if (warp == 1) {
     // ---------------------------------------------------------- MMA issuer
+    // The whole warp runs the loop; one elected lane issues and commits.
     constexpr uint32_t idesc = idesc_bf16_f32(GEMM_BM, BN, A_MN ? 1 : 0, B_MN ? 1 : 0);
     uint32_t it = 0, lt = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x, ++lt) {
       const uint32_t buf = lt & 1, use = lt >> 1;
-      if (!mbar_wait(tempty0 + 8 * buf, (use & 1) ^ 1)) break;
+      if (!mbar_wait_warp(tempty0 + 8 * buf, (use & 1) ^ 1)) break;
       tc_fence_after();
       const uint32_t d_tmem = tmem + buf * BN;
       PF_TILE_DECODE(tile)
@@ -232,31 +233,36 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       for (int kt = kb; kt < ke; ++kt, ++it) {
         const int s = it % STAGES;
         const uint32_t ph = (it / STAGES) & 1;
-        if (!mbar_wait(full0 + 8 * s, ph)) {
+        if (!mbar_wait_warp(full0 + 8 * s, ph)) {
           ok = false;
           break;
         }
         tc_fence_after();
         const uint32_t a_base = smem_u32(smem + s * Cfg::STAGE_BYTES);
         const uint32_t b_base = a_base + Cfg::A_BYTES;
+        if (elect_one()) {
 #pragma unroll
-        for (int kk = 0; kk < GEMM_BK / 16; ++kk) {
-          // K-major: 16 K-elements = 32 bytes along the swizzled 128-byte row,
-          //          8-row groups 1024 bytes apart (SBO).
-          // MN-major: 16 K-rows = 2048 bytes; 64-wide MN slabs 8192 bytes apart
-          //          (LBO), 8-row K groups 1024 bytes apart (SBO).
-          const uint64_t ad = A_MN ? smem_desc_sw128(a_base + kk * 2048, 8192, 1024)
-                                   : smem_desc_sw128(a_base + kk * 32, 16, 1024);
-          const uint64_t bd = B_MN ? smem_desc_sw128(b_base + kk * 2048, 8192, 1024)
-                                   : smem_desc_sw128(b_base + kk * 32, 16, 1024);
-          tc_mma_f16(d_tmem, ad, bd, idesc, (kt != kb || kk != 0) ? 1u : 0u);
+          for (int kk = 0; kk < GEMM_BK / 16; ++kk) {
+            // K-major: 16 K-elements = 32 bytes along the swizzled 128-byte row,
+            //          8-row groups 1024 bytes apart (SBO).
+            // MN-major: 16 K-rows = 2048 bytes; 64-wide MN slabs 8192 bytes apart
+            //          (LBO), 8-row K groups 1024 bytes apart (SBO).
+            const uint64_t ad = A_MN ? smem_desc_sw128(a_base + kk * 2048, 8192, 1024)
+                                     : smem_desc_sw128(a_base + kk * 32, 16, 1024);
+            const uint64_t bd = B_MN ? smem_desc_sw128(b_base + kk * 2048, 8192, 1024)
+                                     : smem_desc_sw128(b_base + kk * 32, 16, 1024);
+            tc_mma_f16(d_tmem, ad, bd, idesc, (kt != kb || kk != 0) ? 1u : 0u);
+          }
+          tc_commit(empty0 + 8 * s);
         }
-        tc_commit(empty0 + 8 * s);
+        __syncwarp();
       }
-      tc_commit(tfull0 + 8 * buf);
+      if (elect_one()) tc_commit(tfull0 + 8 * buf);
+      __syncwarp();
     }
-    s_consumed = it;
-    tc_commit(done);
+    if (lane == 0) s_consumed = it;
+    if (elect_one()) tc_commit(done);
+    __syncwarp();
   } else if (warp >= 2) {
     // ---------------------------------------------------------- epilogue
     const int et = threadIdx.x - 64;
