@@ -68,7 +68,7 @@ cudaError_t launch(int M, int N, int K, const CUtensorMap& ta, const CUtensorMap
   if (e != cudaSuccess) return e;
   const long tiles = (long)((N + BN - 1) / BN) * ((M + GEMM_BM - 1) / GEMM_BM) * splits;
   const int grid = (int)std::min<long>(tiles, num_sms());
-  kern<<<grid, GEMM_THREADS, smem, st>>>(ta, tb, tx, M, N, K, splits, epi);
+  kern<<<grid, GemmRoles<Epi>::kThreads, smem, st>>>(ta, tb, tx, M, N, K, splits, epi);
   return cudaGetLastError();
 }
 

@@ -22,7 +22,13 @@
 //              accumulator i, the MMA warp fills the other.
 // Epilogues that read a bf16 tile shaped like the output (the local stream X
 // for injection, the direct gradient for dX) have it prefetched by TMA into
-// shared memory (128 x BN, 128B-swizzled) while the tile's mainloop runs.
+// shared memory (128 x BN, 128B-swizzled, 64-column boxes).  Unpaired ones get
+//   warp 10  : X loader: refills each box for the next tile as soon as the
+//              four epilogue warps of its column half are done with it, so
+//              the load overlaps the rest of the tile instead of waiting for
+//              the whole tile to drain (the single buffer has no room for a
+//              second one next to the operand stages);
+// paired ones (2D affine) load the whole tile at the start of its epilogue.
 // Every mbarrier wait is bounded (common.cuh); on a timeout the kernel flags
 // the error, drains its own copies and MMAs (bounded), frees TMEM and returns.
 #pragma once
@@ -35,6 +41,13 @@ constexpr int GEMM_BM = 128;
 constexpr int GEMM_BK = 64;
 constexpr int GEMM_EPI_WARPS = 8;  // two per TMEM lane quarter, each owning half the columns
 constexpr int GEMM_THREADS = 64 + 32 * GEMM_EPI_WARPS;
+
+// Unpaired X-tile epilogues run an X-loader warp after the epilogue warps.
+template <class Epi>
+struct GemmRoles {
+  static constexpr bool kXLoader = Epi::kXTile && !Epi::kPaired;
+  static constexpr int kThreads = GEMM_THREADS + (kXLoader ? 32 : 0);
+};
 
 // XCOLS: columns of the bf16 tile an epilogue prefetches (0: none).
 // PAR: the epilogue stages one float4 of per-column parameters per output
@@ -98,6 +111,23 @@ __device__ __forceinline__ void warp_store_rows(uint8_t* xt, int q, int cl, F ds
   }
 }
 
+// Destinations of warp_store_rows' four store instructions for whole-row
+// segments: this lane stores (in instruction it) for row 8 it + lane / 4 of
+// the warp's 32 rows, whose element offset and valid column count are
+// gathered here once per tile (not shuffled again for every chunk).
+struct SegRows {
+  long long off[4];
+  int lim[4];
+  __device__ __forceinline__ void gather(long long my_off, int my_lim) {
+    const int src = (threadIdx.x & 31) >> 2;
+#pragma unroll
+    for (int it = 0; it < 4; ++it) {
+      off[it] = __shfl_sync(0xffffffffu, my_off, it * 8 + src);
+      lim[it] = __shfl_sync(0xffffffffu, my_lim, it * 8 + src);
+    }
+  }
+};
+
 __device__ __forceinline__ void xtile_put8(uint8_t* xt, int r, int c, const float* v) {
   *reinterpret_cast<uint4*>(xtile_ptr(xt, r, c)) =
       make_uint4(pack_bf16(v[0], v[1]), pack_bf16(v[2], v[3]), pack_bf16(v[4], v[5]),
@@ -105,7 +135,7 @@ __device__ __forceinline__ void xtile_put8(uint8_t* xt, int r, int c, const floa
 }
 
 template <int BN, bool A_MN, bool B_MN, class Epi>
-__global__ void __launch_bounds__(GEMM_THREADS, 1)
+__global__ void __launch_bounds__(GemmRoles<Epi>::kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmX, int M, int N, int K, int splits,
                    Epi epi) {
@@ -117,8 +147,12 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
                                              ~uintptr_t(1023));
   uint8_t* xtile = smem + STAGES * Cfg::STAGE_BYTES;
   uint64_t* bars = reinterpret_cast<uint64_t*>(xtile + Cfg::X_BYTES);
-  // bars: full[S], empty[S], tfull[2], tempty[2], xfull, done
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 6);
+  // bars: full[S], empty[S], tfull[2], tempty[2], xfull, done, xbox_full[4],
+  // xbox_empty[4]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 14);
+  constexpr bool XL = GemmRoles<Epi>::kXLoader;
+  constexpr int XBOXES = XCOLS / 64;       // 64-column boxes of the X tile
+  constexpr int XB_HALF = XBOXES / 2;      // boxes per epilogue column half (XL)
   // column parameters (kColPar), [2 tiles][BN/4 groups][4 params] float4: the
   // float4 at (c / 4) * 4 + k holds parameter k of columns c & ~3 .. (c & ~3) + 3
   float4* cpar = reinterpret_cast<float4*>(xtile + Cfg::X_BYTES + 256);
@@ -150,6 +184,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + STAGES);
   const uint32_t tfull0 = smem_u32(bars + 2 * STAGES), tempty0 = tfull0 + 16;
   const uint32_t xfull = tfull0 + 32, done = tfull0 + 40;
+  const uint32_t xbf0 = tfull0 + 48, xbe0 = xbf0 + 32;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -162,6 +197,10 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     }
     mbar_init(xfull, 1);
     mbar_init(done, 1);
+    for (int j = 0; j < 4; ++j) {
+      mbar_init(xbf0 + 8 * j, 1);
+      mbar_init(xbe0 + 8 * j, 4);  // the four epilogue warps of the box's column half
+    }
     fence_barrier_init();
     s_consumed = 0;
   }
@@ -176,6 +215,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
   uint32_t issued = 0;
   bool x_pending = false;
   uint32_t x_parity = 0;
+  uint32_t xb_issued[4] = {0, 0, 0, 0};  // X loader: loads issued per box
 
   if (warp == 0 && lane == 0) {
     // ---------------------------------------------------------- producer
@@ -263,6 +303,34 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
     if (lane == 0) s_consumed = it;
     if (elect_one()) tc_commit(done);
     __syncwarp();
+  } else if (XL && warp == 2 + GEMM_EPI_WARPS) {
+    // ---------------------------------------------------------- X loader
+    if (lane == 0) {
+      prefetch_tmap(&tmX);
+      uint32_t lt = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x, ++lt) {
+        PF_TILE_DECODE(tile)
+        (void)sp;
+        (void)kb;
+        (void)ke;
+        const int xr = epi.x_row(m0);
+        // in the order the halves free them: box i of each half, then box i+1
+        for (int i = 0; i < XB_HALF && ok; ++i) {
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const int j = h * XB_HALF + i;
+            if (!mbar_wait(xbe0 + 8 * j, (lt & 1) ^ 1)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(xbf0 + 8 * j, 16384);
+            tma_load_2d(smem_u32(xtile) + j * 16384, &tmX, xbf0 + 8 * j, epi.x_col(n0, j), xr);
+            xb_issued[j] = lt + 1;
+          }
+        }
+      }
+    }
   } else if (warp >= 2) {
     // ---------------------------------------------------------- epilogue
     const int et = threadIdx.x - 64;
@@ -281,7 +349,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       PF_TILE_DECODE(tile)
       const bool no_k = ke <= kb;
       const uint32_t buf = lt & 1, use = lt >> 1;
-      if (Epi::kXTile && et == 0) {
+      if (Epi::kXTile && !XL && et == 0) {
         mbar_arrive_expect_tx(xfull, Cfg::X_BYTES);
         const int xr = epi.x_row(m0);
 #pragma unroll
@@ -296,9 +364,9 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
       if constexpr (Epi::kColPar)
         if (ntile < tiles && et < BN) npar = epi.col_param(tile_n0(ntile), et);
       const float4* cp = cpar + (lt & 1) * BN;
-      const bool ok = mbar_wait(tfull0 + 8 * buf, use & 1);
+      bool ok = mbar_wait(tfull0 + 8 * buf, use & 1);
       tc_fence_after();
-      if (Epi::kXTile) {
+      if (Epi::kXTile && !XL) {
         mbar_wait(xfull, lt & 1);
         x_pending = false;
       }
@@ -336,11 +404,18 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
 #pragma unroll 1
         for (int ci = 0; ci < NCH; ci += 2) {
           const int c = c_begin + ci * 32;
+          const int xb = c >> 6;  // the X box of this chunk pair (XL)
+          if (XL) ok = mbar_wait(xbf0 + 8 * xb, lt & 1) && ok;
           tmem_ld32_async(trow + (uint32_t)(c + 32), rb);
           run(ra, c);
           tmem_wait_ld(rb);
           if (ci + 2 < NCH) tmem_ld32_async(trow + (uint32_t)(c + 64), ra);
           run(rb, c + 32);
+          if (XL) {  // this warp is done with the box: staging writes before the refill
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(xbe0 + 8 * xb);
+          }
           if (ci + 2 < NCH) tmem_wait_ld(ra);
         }
       }
@@ -348,7 +423,7 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         if (ntile < tiles && et < BN) cpar_put((lt + 1) & 1, et, npar);
       // staging writes into the X tile are ordered before the next tile's
       // TMA load of it
-      if (Epi::kXTile) fence_proxy_async_smem();
+      if (Epi::kXTile && !XL) fence_proxy_async_smem();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(tempty0 + 8 * buf);
@@ -365,6 +440,10 @@ __global__ void __launch_bounds__(GEMM_THREADS, 1)
         mbar_wait_drain(full0 + 8 * (it % STAGES), (it / STAGES) & 1);
     }
     if (warp == 2 && lane == 0 && x_pending) mbar_wait_drain(xfull, x_parity);
+    if (XL && warp == 2 + GEMM_EPI_WARPS && lane == 0) {
+      for (int j = 0; j < XBOXES; ++j)
+        if (xb_issued[j]) mbar_wait_drain(xbf0 + 8 * j, (xb_issued[j] - 1) & 1);
+    }
     if (warp == 1 && lane == 0) mbar_wait_drain(done, 0);
     __syncthreads();
   } else if (warp == 1 && lane == 0) {
@@ -463,6 +542,7 @@ struct EpiInject1D : EpiBase {
     bool ok;    // row < M
     long off0;  // element offset of the group's first token in X_out
     int lim;    // columns < lim belong to tokens < L of a target block
+    SegRows seg;
   };
   int M, N;
   const float* bias;
@@ -482,6 +562,7 @@ struct EpiInject1D : EpiBase {
       const long lim = (L - tok0) * d;
       r.lim = lim < N ? (int)lim : N;
     }
+    r.seg.gather(r.off0, r.ok ? r.lim : 0);
     return r;
   }
   // staged per column: (bias, w_x, w_dlt, b_g)
@@ -535,12 +616,9 @@ struct EpiInject1D : EpiBase {
       xtile_put8(xt, rl, cl + i8, o);
     }
     __syncwarp();
-    const long long off = ri.off0;
-    const int lim = ri.ok ? ri.lim : 0;
     warp_store_rows(xt, q, cl, [&](int rr, int p) -> bf16* {
-      const long long o2 = __shfl_sync(0xffffffffu, off, rr);
-      const int l2 = __shfl_sync(0xffffffffu, lim, rr);
-      return col + p * 8 < l2 ? X_out + o2 + col + p * 8 : nullptr;
+      const int it = rr >> 3;
+      return col + p * 8 < ri.seg.lim[it] ? X_out + ri.seg.off[it] + col + p * 8 : nullptr;
     });
     __syncwarp();
     if (D_save) {
@@ -568,6 +646,7 @@ struct EpiDX1D : EpiBase {
     bool ok;
     long off0;
     int lim;
+    SegRows seg;
   };
   int M, N;
   bf16* dX;
@@ -582,6 +661,7 @@ struct EpiDX1D : EpiBase {
       const long lim = (L - tok0) * d;
       r.lim = lim < N ? (int)lim : N;
     }
+    r.seg.gather(r.off0, r.ok ? r.lim : 0);
     return r;
   }
   // staged in the tile cells just read, stored with whole-row segments
@@ -597,12 +677,9 @@ struct EpiDX1D : EpiBase {
       xtile_put8(xt, rl, cl + i8, x);
     }
     __syncwarp();
-    const long long off = ri.off0;
-    const int lim = ri.ok ? ri.lim : 0;
     warp_store_rows(xt, rl >> 5, cl, [&](int rr, int p) -> bf16* {
-      const long long o2 = __shfl_sync(0xffffffffu, off, rr);
-      const int l2 = __shfl_sync(0xffffffffu, lim, rr);
-      return col + p * 8 < l2 ? dX + o2 + col + p * 8 : nullptr;
+      const int it = rr >> 3;
+      return col + p * 8 < ri.seg.lim[it] ? dX + ri.seg.off[it] + col + p * 8 : nullptr;
     });
     __syncwarp();
   }
