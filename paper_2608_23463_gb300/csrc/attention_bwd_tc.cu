@@ -353,18 +353,24 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
             const uint32_t* sv = s1 + g * 8;
             const uint32_t* dv = p1 + g * 8;
             float pe[8], de[8];
+            // DKDV: the group's (lse, Di) with 128-bit shared loads, two columns
+            // each (the compiler cannot prove the alignment of the float2 array)
+            float l8[8], d8[8];
+            if (DKDV) {
+              const float4* l4 = reinterpret_cast<const float4*>(lds) + kg * 4;
+#pragma unroll
+              for (int e2 = 0; e2 < 4; ++e2) {
+                const float4 v = l4[e2];
+                l8[2 * e2] = v.x;
+                d8[2 * e2] = v.y;
+                l8[2 * e2 + 1] = v.z;
+                d8[2 * e2 + 1] = v.w;
+              }
+            }
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
               const int c = kg * 8 + e;
-              float l2, dd;
-              if (DKDV) {
-                const float2 v = lds[c];
-                l2 = v.x;
-                dd = v.y;
-              } else {
-                l2 = lse_r;
-                dd = di_r;
-              }
+              const float l2 = DKDV ? l8[e] : lse_r, dd = DKDV ? d8[e] : di_r;
               float p = ex2_approx(fmaf(__uint_as_float(sv[e]), a.sl2, -l2));
               if (decltype(masked)::value && (c < lo || c >= hi)) p = 0.f;
               pe[e] = p;
