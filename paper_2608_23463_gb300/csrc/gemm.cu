@@ -58,11 +58,62 @@ bool make_operand_map(CUtensorMap* m, const Operand& op, int rows, int K) {
   return make_map(m, op.ptr, (uint64_t)K, (uint64_t)rows, (uint64_t)op.ld, 64, 128);
 }
 
+// Co-resident CTA pairs of the pair kernel (at most half the SMs).
+template <class Kern>
+int max_pairs(Kern kern, int threads, int smem) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * (num_sms() / 2));
+  cfg.blockDim = dim3(threads);
+  cfg.dynamicSmemBytes = smem;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = 2;
+  at[0].val.clusterDim.y = 1;
+  at[0].val.clusterDim.z = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess || n <= 0) {
+    cudaGetLastError();
+    return 0;
+  }
+  return std::min(n, num_sms() / 2);
+}
+
 template <int BN, bool AMN, bool BMN, class Epi>
 cudaError_t launch(int M, int N, int K, const CUtensorMap& ta, const CUtensorMap& tb,
                    const CUtensorMap& tx, const Epi& epi, cudaStream_t st, int splits) {
-  auto kern = gemm_tc_kernel<BN, AMN, BMN, Epi>;
   constexpr int XCOLS = Epi::kXTile ? (Epi::kPaired ? BN / 2 : BN) : 0;
+  if constexpr (BN == 256 && Epi::kPairs) {
+    // CTA pairs (256 x 256 tiles, half of B per CTA, a deeper stage ring)
+    // when every co-resident pair gets a tile
+    auto kern2 = gemm_tc_kernel<BN, AMN, BMN, Epi, true>;
+    constexpr int smem2 = GemmCfg<BN, XCOLS, Epi::kColPar, true>::SMEM_BYTES;
+    constexpr int threads = GemmRoles<Epi>::kThreads;
+    cudaError_t e = cudaFuncSetAttribute(kern2, cudaFuncAttributeMaxDynamicSharedMemorySize, smem2);
+    if (e != cudaSuccess) return e;
+    static const int pairs = max_pairs(kern2, threads, smem2);
+    const long pair_tiles =
+        (long)((N + BN - 1) / BN) * ((M + 2 * GEMM_BM - 1) / (2 * GEMM_BM)) * splits;
+    if (pairs > 0 && pair_tiles >= pairs) {
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3(2 * (unsigned)std::min<long>(pair_tiles, pairs));
+      cfg.blockDim = dim3(threads);
+      cfg.dynamicSmemBytes = smem2;
+      cfg.stream = st;
+      cudaLaunchAttribute at[1];
+      at[0].id = cudaLaunchAttributeClusterDimension;
+      at[0].val.clusterDim.x = 2;
+      at[0].val.clusterDim.y = 1;
+      at[0].val.clusterDim.z = 1;
+      cfg.attrs = at;
+      cfg.numAttrs = 1;
+      e = cudaLaunchKernelEx(&cfg, kern2, ta, tb, tx, M, N, K, splits, epi);
+      if (e != cudaSuccess) return e;
+      return cudaGetLastError();
+    }
+  }
+  auto kern = gemm_tc_kernel<BN, AMN, BMN, Epi>;
   constexpr int smem = GemmCfg<BN, XCOLS, Epi::kColPar>::SMEM_BYTES;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;

@@ -9,13 +9,21 @@
 // Persistent: one CTA per SM walks the 128 x BN output tiles tile = blockIdx.x
 // + k * gridDim.x (N fastest, so co-running CTAs share A panels and all of B
 // in L2; M fastest when A has at most 16 row tiles and B is wider than the
-// grid, so co-running CTAs share B tiles).  Roles:
+// grid, so co-running CTAs share B tiles).  With BN = 256 and enough tiles the
+// kernel runs on CTA pairs (clusters of two): a pair owns a 256 x 256 tile,
+// rank 0 issues tcgen05.mma.cta_group::2 (M = 256) and each CTA stages its 128
+// rows of A and half of B, so a stage is 32 KB instead of 48 and 7 (4-5 with an
+// X tile) fit where 4 (3) did: the deeper ring hides the HBM latency of the
+// streamed operand (a mainloop measured at ~680 cycles per 64-deep K block
+// with 4 stages runs at ~525 with 6, the MMAs' own time being 512).  Roles:
 //   warp 0   : TMA producer (one thread): STAGES-deep ring of 128B-swizzled
 //              64-wide K slices of A and B, continuing across tiles
-//   warp 1   : TMEM allocator + MMA issuer (one thread): tcgen05.mma M=128,
-//              N=BN, K=16 into one of two TMEM accumulators (2*BN columns),
-//              tcgen05.commit frees smem stages and hands a finished
-//              accumulator to the epilogue
+//   warp 1   : TMEM allocator + MMA issuer (one elected lane): tcgen05.mma
+//              M=128 (a pair: 256), N=BN, K=16 into one of two TMEM
+//              accumulators (2*BN columns), tcgen05.commit frees smem stages
+//              and hands a finished accumulator to the epilogue (a pair: to
+//              both CTAs; both CTAs' stage loads complete on rank 0's full
+//              barriers, and rank 1's MMA warp has nothing to issue)
 //   warps 2-9: epilogue: tcgen05.ld 32 columns at a time (warp w reads TMEM
 //              lanes 32*(w%4).. and half of the tile's columns), fused
 //              epilogue functor, global stores.  While they drain
@@ -52,17 +60,25 @@ struct GemmRoles {
 // XCOLS: columns of the bf16 tile an epilogue prefetches (0: none).
 // PAR: the epilogue stages one float4 of per-column parameters per output
 // column in shared memory (two tiles' worth, filled one tile ahead).
-template <int BN, int XCOLS, bool PAR = false>
+// PAIR: the tile is shared by a CTA pair, each CTA staging half of B.
+constexpr uint32_t GEMM_SMEM_MAX = 232448;  // dynamic shared memory per CTA (227 KB)
+template <int BN, int XCOLS, bool PAR = false, bool PAIR = false>
 struct GemmCfg {
-  static constexpr int STAGES =
-      XCOLS ? (BN == 256 && (XCOLS == 256 || PAR) ? 3 : (BN == 256 ? 4 : 5)) : (BN == 256 ? 4 : 6);
+  static constexpr int B_ROWS = PAIR ? BN / 2 : BN;            // B rows staged by one CTA
   static constexpr uint32_t A_BYTES = GEMM_BM * GEMM_BK * 2;  // 16 KB
-  static constexpr uint32_t B_BYTES = BN * GEMM_BK * 2;       // 16/32 KB
+  static constexpr uint32_t B_BYTES = B_ROWS * GEMM_BK * 2;   // 16/32 KB
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr uint32_t X_BYTES = GEMM_BM * XCOLS * 2;
   static constexpr uint32_t PAR_BYTES = PAR ? 2 * BN * 16 : 0;
-  static constexpr uint32_t SMEM_BYTES =
-      STAGES * STAGE_BYTES + X_BYTES + 1024 /*align*/ + 256 /*barriers*/ + PAR_BYTES;
+  static constexpr uint32_t FIXED_BYTES = X_BYTES + 1024 /*align*/ + 256 /*barriers*/ + PAR_BYTES;
+  static constexpr int PAIR_STAGES = (int)((GEMM_SMEM_MAX - FIXED_BYTES) / STAGE_BYTES);
+  static constexpr int STAGES =
+      PAIR ? (PAIR_STAGES < 7 ? PAIR_STAGES : 7)
+           : (XCOLS ? (BN == 256 && (XCOLS == 256 || PAR) ? 3 : (BN == 256 ? 4 : 5))
+                    : (BN == 256 ? 4 : 6));
+  static constexpr uint32_t SMEM_BYTES = STAGES * STAGE_BYTES + FIXED_BYTES;
+  static_assert(SMEM_BYTES <= GEMM_SMEM_MAX, "shared memory");
+  static_assert(2 * STAGES + 14 <= 31, "barrier region");
 };
 
 // Barrier of the epilogue threads (named barrier 1) that also ANDs a predicate
@@ -134,13 +150,14 @@ __device__ __forceinline__ void xtile_put8(uint8_t* xt, int r, int c, const floa
                  pack_bf16(v[6], v[7]));
 }
 
-template <int BN, bool A_MN, bool B_MN, class Epi>
+template <int BN, bool A_MN, bool B_MN, class Epi, bool PAIR = false>
 __global__ void __launch_bounds__(GemmRoles<Epi>::kThreads, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmX, int M, int N, int K, int splits,
                    Epi epi) {
+  static_assert(!PAIR || BN == 256, "CTA pairs use 256-wide tiles");
   constexpr int XCOLS = Epi::kXTile ? (Epi::kPaired ? BN / 2 : BN) : 0;
-  using Cfg = GemmCfg<BN, XCOLS, Epi::kColPar>;
+  using Cfg = GemmCfg<BN, XCOLS, Epi::kColPar, PAIR>;
   constexpr int STAGES = Cfg::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -166,20 +183,27 @@ __global__ void __launch_bounds__(GemmRoles<Epi>::kThreads, 1)
   __shared__ uint32_t s_consumed;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int num_n = (N + BN - 1) / BN, num_m = (M + GEMM_BM - 1) / GEMM_BM;
+  // a pair (cluster of two CTAs) works on one tile of 2 x 128 rows: `unit` is
+  // the pair (or the lone CTA), `rank` this CTA's half of the rows
+  const uint32_t rank = PAIR ? cluster_ctarank() : 0u;
+  const int unit = PAIR ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+  const int n_units = PAIR ? (int)(gridDim.x >> 1) : (int)gridDim.x;
+  constexpr int TILE_M = PAIR ? 2 * GEMM_BM : GEMM_BM;
+  const int num_n = (N + BN - 1) / BN, num_m = (M + TILE_M - 1) / TILE_M;
   const int mn_tiles = num_m * num_n;
   // N fastest keeps the co-running CTAs on one A panel with all of B in L2;
   // when A is a few row tiles and B is wider than the grid, M fastest instead
   // lets the co-running CTAs share each B tile (B is then read once)
-  const bool m_fast = num_m <= 16 && num_n > (int)gridDim.x;
+  const bool m_fast = num_m <= 16 && num_n > n_units;
   const int tiles = mn_tiles * splits;
   const int num_k = (K + GEMM_BK - 1) / GEMM_BK;
   const int kps = (num_k + splits - 1) / splits;  // K tiles per split
-  // tile t -> split t / mn_tiles (slowest), then M, then N (fastest)
-#define PF_TILE_DECODE(t)                                   \
-  const int sp = (t) / mn_tiles, rem = (t) % mn_tiles;      \
-  const int m0 = (m_fast ? rem % num_m : rem / num_n) * GEMM_BM;  \
-  const int n0 = (m_fast ? rem / num_m : rem % num_n) * BN;        \
+  // tile t -> split t / mn_tiles (slowest), then M, then N (fastest); m0 is
+  // this CTA's first row
+#define PF_TILE_DECODE(t)                                                        \
+  const int sp = (t) / mn_tiles, rem = (t) % mn_tiles;                           \
+  const int m0 = (m_fast ? rem % num_m : rem / num_n) * TILE_M + (int)rank * GEMM_BM; \
+  const int n0 = (m_fast ? rem / num_m : rem % num_n) * BN;                      \
   const int kb = sp * kps, ke = min(num_k, kb + kps);
   const uint32_t full0 = smem_u32(bars), empty0 = smem_u32(bars + STAGES);
   const uint32_t tfull0 = smem_u32(bars + 2 * STAGES), tempty0 = tfull0 + 16;
@@ -193,7 +217,8 @@ __global__ void __launch_bounds__(GemmRoles<Epi>::kThreads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(tfull0 + 8 * b, 1);
-      mbar_init(tempty0 + 8 * b, GEMM_EPI_WARPS);  // one arrival per epilogue warp
+      // one arrival per epilogue warp (of both CTAs of a pair, on rank 0)
+      mbar_init(tempty0 + 8 * b, PAIR ? 2 * GEMM_EPI_WARPS : GEMM_EPI_WARPS);
     }
     mbar_init(xfull, 1);
     mbar_init(done, 1);
@@ -205,11 +230,17 @@ __global__ void __launch_bounds__(GemmRoles<Epi>::kThreads, 1)
     s_consumed = 0;
   }
   if (warp == 1) {
-    tmem_alloc(smem_u32(tmem_slot), 2 * BN);
-    tmem_relinquish();
+    if (PAIR) {
+      tmem_alloc_pair(smem_u32(tmem_slot), 2 * BN);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(smem_u32(tmem_slot), 2 * BN);
+      tmem_relinquish();
+    }
   }
   tc_fence_before();
   __syncthreads();
+  if (PAIR) cluster_sync_all();  // both CTAs' barriers exist before any remote arrival
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   uint32_t issued = 0;
@@ -223,7 +254,7 @@ __global__ void __launch_bounds__(GemmRoles<Epi>::kThreads, 1)
     prefetch_tmap(&tmB);
     uint32_t it = 0;
     bool ok = true;
-    for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x) {
+    for (int tile = unit; tile < tiles && ok; tile += n_units) {
       PF_TILE_DECODE(tile)
       (void)sp;
       for (int kt = kb; kt < ke; ++kt, ++it) {
@@ -233,35 +264,50 @@ __global__ void __launch_bounds__(GemmRoles<Epi>::kThreads, 1)
           ok = false;
           break;
         }
-        const uint32_t fb = full0 + 8 * s;
-        mbar_arrive_expect_tx(fb, Cfg::STAGE_BYTES);
+        // a pair: both CTAs' loads complete on rank 0's full barrier, which
+        // rank 0 arms for the two CTAs' bytes
+        const uint32_t fb = PAIR ? smem_map_rank(full0 + 8 * s, 0) : full0 + 8 * s;
+        if (!PAIR || rank == 0)
+          mbar_arrive_expect_tx(full0 + 8 * s, (PAIR ? 2u : 1u) * Cfg::STAGE_BYTES);
+        auto ld = [&](uint32_t dst, const CUtensorMap* map, int c0, int c1) {
+          if (PAIR)
+            tma_load_2d_pair(dst, map, fb, c0, c1);
+          else
+            tma_load_2d(dst, map, fb, c0, c1);
+        };
         const uint32_t a_dst = smem_u32(smem + s * Cfg::STAGE_BYTES);
         const uint32_t b_dst = a_dst + Cfg::A_BYTES;
         const int k0 = kt * GEMM_BK;
         if (!A_MN) {
-          tma_load_2d(a_dst, &tmA, fb, k0, m0);
+          ld(a_dst, &tmA, k0, m0);
         } else {
-          tma_load_2d(a_dst, &tmA, fb, m0, k0);
-          tma_load_2d(a_dst + 8192, &tmA, fb, m0 + 64, k0);
+          ld(a_dst, &tmA, m0, k0);
+          ld(a_dst + 8192, &tmA, m0 + 64, k0);
         }
+        // this CTA's B rows: all of them, or (a pair) its half of the columns
         if (!B_MN) {
+          constexpr int JB = Cfg::B_ROWS / 128;
 #pragma unroll
-          for (int j = 0; j < BN / 128; ++j)
-            tma_load_2d(b_dst + j * 16384, &tmB, fb, k0, epi.b_row(n0, j));
+          for (int j = 0; j < JB; ++j)
+            ld(b_dst + j * 16384, &tmB, k0, epi.b_row(n0, j + (int)rank * JB));
         } else {
+          constexpr int JB = Cfg::B_ROWS / 64;
 #pragma unroll
-          for (int j = 0; j < BN / 64; ++j) tma_load_2d(b_dst + j * 8192, &tmB, fb, n0 + 64 * j, k0);
+          for (int j = 0; j < JB; ++j)
+            ld(b_dst + j * 8192, &tmB, n0 + 64 * (j + (int)rank * JB), k0);
         }
         issued = it + 1;
       }
     }
+  } else if (warp == 1 && PAIR && rank == 1) {
+    // rank 1 of a pair: rank 0 issues the MMAs for both CTAs
   } else if (warp == 1) {
     // ---------------------------------------------------------- MMA issuer
     // The whole warp runs the loop; one elected lane issues and commits.
-    constexpr uint32_t idesc = idesc_bf16_f32(GEMM_BM, BN, A_MN ? 1 : 0, B_MN ? 1 : 0);
+    constexpr uint32_t idesc = idesc_bf16_f32(TILE_M, BN, A_MN ? 1 : 0, B_MN ? 1 : 0);
     uint32_t it = 0, lt = 0;
     bool ok = true;
-    for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x, ++lt) {
+    for (int tile = unit; tile < tiles && ok; tile += n_units, ++lt) {
       const uint32_t buf = lt & 1, use = lt >> 1;
       if (!mbar_wait_warp(tempty0 + 8 * buf, (use & 1) ^ 1)) break;
       tc_fence_after();
@@ -291,17 +337,33 @@ __global__ void __launch_bounds__(GemmRoles<Epi>::kThreads, 1)
                                      : smem_desc_sw128(a_base + kk * 32, 16, 1024);
             const uint64_t bd = B_MN ? smem_desc_sw128(b_base + kk * 2048, 8192, 1024)
                                      : smem_desc_sw128(b_base + kk * 32, 16, 1024);
-            tc_mma_f16(d_tmem, ad, bd, idesc, (kt != kb || kk != 0) ? 1u : 0u);
+            if (PAIR)
+              tc_mma_f16_pair(d_tmem, ad, bd, idesc, (kt != kb || kk != 0) ? 1u : 0u);
+            else
+              tc_mma_f16(d_tmem, ad, bd, idesc, (kt != kb || kk != 0) ? 1u : 0u);
           }
-          tc_commit(empty0 + 8 * s);
+          if (PAIR)
+            tc_commit_pair(empty0 + 8 * s);
+          else
+            tc_commit(empty0 + 8 * s);
         }
         __syncwarp();
       }
-      if (elect_one()) tc_commit(tfull0 + 8 * buf);
+      if (elect_one()) {
+        if (PAIR)
+          tc_commit_pair(tfull0 + 8 * buf);
+        else
+          tc_commit(tfull0 + 8 * buf);
+      }
       __syncwarp();
     }
     if (lane == 0) s_consumed = it;
-    if (elect_one()) tc_commit(done);
+    if (elect_one()) {
+      if (PAIR)
+        tc_commit_pair(done);
+      else
+        tc_commit(done);
+    }
     __syncwarp();
   } else if (XL && warp == 2 + GEMM_EPI_WARPS) {
     // ---------------------------------------------------------- X loader
@@ -309,7 +371,7 @@ __global__ void __launch_bounds__(GemmRoles<Epi>::kThreads, 1)
       prefetch_tmap(&tmX);
       uint32_t lt = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < tiles && ok; tile += gridDim.x, ++lt) {
+      for (int tile = unit; tile < tiles && ok; tile += n_units, ++lt) {
         PF_TILE_DECODE(tile)
         (void)sp;
         (void)kb;
@@ -341,11 +403,11 @@ __global__ void __launch_bounds__(GemmRoles<Epi>::kThreads, 1)
       return (m_fast ? r / num_m : r % num_n) * BN;
     };
     if constexpr (Epi::kColPar) {  // parameters of the first tile
-      if ((int)blockIdx.x < tiles && et < BN) cpar_put(0, et, epi.col_param(tile_n0(blockIdx.x), et));
+      if (unit < tiles && et < BN) cpar_put(0, et, epi.col_param(tile_n0(unit), et));
       epi_bar_and(true);
     }
     uint32_t lt = 0;
-    for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, ++lt) {
+    for (int tile = unit; tile < tiles; tile += n_units, ++lt) {
       PF_TILE_DECODE(tile)
       const bool no_k = ke <= kb;
       const uint32_t buf = lt & 1, use = lt >> 1;
@@ -359,7 +421,7 @@ __global__ void __launch_bounds__(GemmRoles<Epi>::kThreads, 1)
         x_parity = lt & 1;
       }
       // next tile's column parameters: loaded now, stored after this tile
-      const int ntile = tile + (int)gridDim.x;
+      const int ntile = tile + n_units;
       float4 npar = make_float4(0.f, 0.f, 0.f, 0.f);
       if constexpr (Epi::kColPar)
         if (ntile < tiles && et < BN) npar = epi.col_param(tile_n0(ntile), et);
@@ -426,7 +488,12 @@ __global__ void __launch_bounds__(GemmRoles<Epi>::kThreads, 1)
       if (Epi::kXTile && !XL) fence_proxy_async_smem();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(tempty0 + 8 * buf);
+      if (lane == 0) {
+        if (PAIR && rank == 1)
+          mbar_arrive_remote(smem_map_rank(tempty0 + 8 * buf, 0));
+        else
+          mbar_arrive(tempty0 + 8 * buf);
+      }
       // all epilogue threads are done with the X tile (free for the next
       // prefetch); leave together if any of them saw a wait run out
       if (!epi_bar_and(ok)) break;
@@ -436,8 +503,16 @@ __global__ void __launch_bounds__(GemmRoles<Epi>::kThreads, 1)
   if (__syncthreads_or(*(volatile int*)&g_dev_error != 0)) {
     // error path: let in-flight TMA copies and MMAs land before TMEM/smem go.
     if (warp == 0 && lane == 0) {
-      for (uint32_t it = s_consumed; it < issued; ++it)
-        mbar_wait_drain(full0 + 8 * (it % STAGES), (it / STAGES) & 1);
+      if (PAIR && rank == 1) {
+        // its loads complete on rank 0's barriers: give them a bounded time
+        // (far above a load's latency) to land before the CTA goes
+        const unsigned long long t0 = globaltimer();
+        while (globaltimer() - t0 < 50000ull) {
+        }
+      } else {
+        for (uint32_t it = s_consumed; it < issued; ++it)
+          mbar_wait_drain(full0 + 8 * (it % STAGES), (it / STAGES) & 1);
+      }
     }
     if (warp == 2 && lane == 0 && x_pending) mbar_wait_drain(xfull, x_parity);
     if (XL && warp == 2 + GEMM_EPI_WARPS && lane == 0) {
@@ -450,9 +525,15 @@ __global__ void __launch_bounds__(GemmRoles<Epi>::kThreads, 1)
     mbar_wait(done, 0);
   }
   __syncthreads();
+  // a pair: neither CTA leaves (or frees TMEM) while the other may still use
+  // its shared memory or TMEM
+  if (PAIR) cluster_sync_all();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, 2 * BN);
+    if (PAIR)
+      tmem_dealloc_pair(tmem, 2 * BN);
+    else
+      tmem_dealloc(tmem, 2 * BN);
   }
 }
 
@@ -471,6 +552,10 @@ struct EpiBase {
   static constexpr bool kPaired = false;
   static constexpr bool kSplitRows = false;
   static constexpr bool kColPar = false;
+  // may run on CTA pairs (256-wide tiles with enough of them); an epilogue
+  // slower than its mainloop does better on single CTAs, whose tiles do not
+  // wait for the other CTA's epilogue
+  static constexpr bool kPairs = true;
   __device__ __forceinline__ float4 col_param(int, int) const { return make_float4(0, 0, 0, 0); }
   __device__ __forceinline__ int x_row(int m0) const { return m0; }
   __device__ __forceinline__ int x_col(int n0, int j) const { return n0 + 64 * j; }
@@ -538,6 +623,7 @@ struct EpiLinear : EpiBase {
 // [B*m*k2, k1*d] of X (zero-padded to whole blocks when L % P != 0).
 struct EpiInject1D : EpiBase {
   static constexpr bool kXTile = true;
+  static constexpr bool kPairs = false;  // epilogue-bound (measured slower on pairs)
   struct Row {
     bool ok;    // row < M
     long off0;  // element offset of the group's first token in X_out

@@ -1,6 +1,8 @@
 """The tcgen05 GEMM on its own, through the C ABI (pf_gemm_bf16), against a
 float32 product of the same bf16 operands, for every operand layout and for
-shapes with ragged M, N and K tails."""
+shapes with ragged M, N and K tails.  Shapes with enough 256 x 256 tiles run
+on CTA pairs (M=256 tiles split by rows between the two CTAs); 5000 and 4904
+rows leave the second CTA of the last pair with 8 rows and with none."""
 import pytest
 import torch
 
@@ -17,7 +19,8 @@ def _lib():
 
 
 @pytest.mark.parametrize("M,N,K", [(296, 320, 200), (128, 64, 64), (1024, 2048, 4096),
-                                   (4096, 1024, 1024), (2048, 8192, 1024)])
+                                   (4096, 1024, 1024), (2048, 8192, 1024), (5000, 4096, 520),
+                                   (4904, 2560, 1000)])
 @pytest.mark.parametrize("a_mn,b_mn", [(0, 0), (0, 1), (1, 1), (1, 0)])
 def test_gemm_layouts(M, N, K, a_mn, b_mn):
     g = torch.Generator(device="cuda").manual_seed(M * 7 + N * 3 + K + a_mn * 2 + b_mn)
