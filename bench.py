@@ -410,7 +410,6 @@ def measure_configs(torch, pf, S, peaks, warmup: int):
         specs.append(sp)
         params.append(S.make_layer_params(sp, 2 + 10 * i))
     st = ProxyStack(specs, params)
-    del params
     inp = S.make_layer_inputs(specs[0], 2, with_grads=True)
     X = to_device(inp["X"], torch.bfloat16)
     G = to_device(inp["G"], torch.bfloat16)
@@ -423,9 +422,74 @@ def measure_configs(torch, pf, S, peaks, warmup: int):
     out["c3_stack_fwd_bwd"] = config_entry(
         "12-layer causal stack fwd+bwd, bf16, L=262144 d=1024 16x64, P=16..256 two-level",
         specs[0].L, ms, fl, nb, dom, peaks, 3)
-    del st, X, G
+    del G
+    out["prefill"] = measure_prefill(torch, pf, S, peaks, warmup, specs, params, st, X)
+    del st, X, params
     torch.cuda.empty_cache()
     return out
+
+
+def measure_prefill(torch, pf, S, peaks, warmup, specs, params, st, X):
+    """Prefill of the 12-layer causal stack over a 262144-token history
+    (Sec. 3.8): the inference forward plus every layer's bulk proxy-cache
+    fill, against a standard softmax-attention prefill of the same depth,
+    width and history (per layer: the QKV projection, causal attention over
+    all L tokens, the output projection).  The standard arm runs PyTorch's
+    fused attention and cuBLAS, one layer timed and scaled by the depth; its
+    FLOP floor at the measured bf16 peak is reported beside it."""
+    from paper_2608_23463_gb300.decode import ProxyKVCache
+    caches = []
+    for i, s in enumerate(specs):
+        ds = S.decode_spec_for_layer(s, s.L // s.P)
+        dp = S.decode_params_for_layer(s, params[i], 200 + i)
+        caches.append(ProxyKVCache(ds, dp, S.make_decode_state(ds, 0, [0], [0])))
+    ms, fl, nb, dom = timed_steps(torch, pf, lambda: st.prefill(X, caches), 3, warmup)
+    L, d, n = specs[0].L, specs[0].d, len(specs)
+    res = config_entry("causal stack prefill latency, 12 layers, L=262144 d=1024 16x64, "
+                       "P=16..256 two-level, proxy caches filled", L, ms, fl, nb, dom, peaks, 3)
+    res["latency_ms"] = ms
+    del caches
+    torch.cuda.empty_cache()
+    # standard prefill, one layer
+    std_flops = n * (2 * L * d * 4 * d + 2 * L * L * d)  # projections + causal QK^T and PV
+    floor_ms = std_flops / (peaks["bf16_tflops_sustained"] * 1e12) * 1e3
+    std = {"flops": std_flops, "floor_ms_at_measured_peak": floor_ms,
+           "impl": "torch scaled_dot_product_attention (fused kernels only) + cuBLAS"}
+    try:
+        from torch.nn.attention import SDPBackend, sdpa_kernel
+        g = torch.Generator(device="cuda").manual_seed(7)
+        Xs = X.reshape(L, d)
+        Wqkv = (torch.randn(3 * d, d, device="cuda", generator=g) / d ** 0.5).to(torch.bfloat16)
+        Wo = (torch.randn(d, d, device="cuda", generator=g) / d ** 0.5).to(torch.bfloat16)
+        nh = specs[0].n_heads
+
+        def layer():
+            qkv = Xs @ Wqkv.T
+            q, k, v = (qkv[:, i * d:(i + 1) * d].reshape(1, L, nh, d // nh).transpose(1, 2)
+                       for i in range(3))
+            o = torch.nn.functional.scaled_dot_product_attention(q, k, v, is_causal=True)
+            return o.transpose(1, 2).reshape(L, d) @ Wo.T
+
+        backends = [SDPBackend.CUDNN_ATTENTION, SDPBackend.FLASH_ATTENTION,
+                    SDPBackend.EFFICIENT_ATTENTION]
+        with sdpa_kernel(backends):
+            stream = torch.cuda.current_stream()
+            layer()
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for _ in range(2):
+                layer()
+            e1.record(stream)
+            torch.cuda.synchronize()
+        std["measured_ms"] = e0.elapsed_time(e1) / 2 * n
+        res["speedup_vs_standard_measured"] = std["measured_ms"] / ms
+    except Exception as e:  # the fused attention may be missing for this GPU
+        std["measured_ms"] = None
+        std["unavailable"] = str(e).splitlines()[0][:200]
+    res["standard_attention_prefill"] = std
+    res["speedup_vs_standard_floor"] = floor_ms / ms
+    return res
 
 
 def load_peaks():

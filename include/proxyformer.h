@@ -214,6 +214,31 @@ pf_status proxy_kv_append(const pf_decode_desc *desc, const pf_append_params *pa
                           const float *H_in, pf_kv_cache *cache,
                           void *ws, size_t ws_bytes, void *stream);
 
+size_t proxy_prefill_workspace_size(const pf_decode_desc *desc, int32_t L_hist);
+
+/* Bulk prefill of the proxy cache from a history (Sec. 3.8: the prefill stage
+ * compresses the historical blocks and caches only their proxies' keys and
+ * values).  For every sequence b the history X_hist[b] ([L_hist, d] bf16,
+ * sequences contiguous) is split into m = floor(L_hist / P) complete blocks
+ * and r = L_hist - m P remaining tokens:
+ *   H_i = H_in[b, i] + C(block i)               (Eq. proxy-res, Eq. compress-
+ *                                                 linear / factor-cascade)
+ *   K_proxy[b, i] = W_kh H_i, V_proxy[b, i] = W_vh H_i       (i < m)
+ *   X_open[b, j] = x, K_open[b, j] = W_k x, V_open[b, j] = W_v x   (j < r, x the
+ *                                                 history's token m P + j)
+ *   n_proxy[b] = m, n_open[b] = r.
+ * This equals m block appends (proxy_kv_append) followed by the open-slot
+ * writes of r decode steps, and replaces the cache's previous contents.
+ * H_in fp32 or NULL, laid out as a layer's proxy stream over the history:
+ * [batch, ceil(L_hist / P), d], the row of a partial last block (r > 0)
+ * unused.  W_k, W_v are rows [d, 3d) of the decode parameters' W_qkv
+ * (dparams is only read when r > 0).  Requires
+ * m <= capacity (else PF_ERR_CAPACITY, nothing launched).                    */
+pf_status proxy_kv_prefill(const pf_decode_desc *desc, const pf_append_params *aparams,
+                           const pf_decode_params *dparams, const void *X_hist, int32_t L_hist,
+                           const float *H_in, pf_kv_cache *cache, void *ws, size_t ws_bytes,
+                           void *stream);
+
 /* Thread-local message describing the last non-OK status of this thread. */
 const char *pf_last_error(void);
 

@@ -20,6 +20,12 @@ compressed exactly like a layer's block (Eq.
 compress-linear / Eq. factor-cascade), H = H_in + c (Eq. proxy-res), and the
 proxy's key and value rows W_kh H, W_vh H are written at cache row n_p;
 n_p += 1, n_o = 0.
+
+Prefill (Sec. 3.8: the prefill stage compresses the historical blocks and
+caches only their proxies): a history of L tokens gives m = floor(L / P)
+complete blocks, each compressed and projected as an append does, and the
+r = L - m P remaining tokens fill the open block with their features and the
+decode step's keys W_k x and values W_v x; n_p = m, n_o = r.
 """
 from __future__ import annotations
 
@@ -125,3 +131,35 @@ def kv_append(spec, prm, state, H_in=None):
         new["n_proxy"][b] = npx + 1
         new["n_open"][b] = 0
     return new
+
+
+def kv_prefill(spec, prm, X_hist, H_in=None):
+    """Cache state after prefilling from a history X_hist [B, L, d]: all
+    complete blocks compressed at once (the blocks' rows of k1 tokens through
+    W_c1, their k2 rows through W_c2 with two levels), H = H_in + C, proxy
+    rows W_kh H / W_vh H; the remaining tokens' features, W_k x and W_v x in
+    the open block.  H_in [B, ceil(L / P), d] (a layer's proxy stream; the
+    partial block's row unused) or None.  Rows past n_proxy / n_open are
+    zero."""
+    X = _f64(X_hist)
+    B, L, d = X.shape
+    P, k1, k2 = spec.P, spec.k1, spec.k2
+    m, r = L // P, L % P
+    Y = X[:, :m * P].reshape(B * m * k2, k1 * d) @ _f64(prm["W_c1"]).T + _f64(prm["b_c1"])
+    if spec.levels == 1:
+        C = Y.reshape(B, m, d)
+    else:
+        C = (Y.reshape(B * m, k2 * d) @ _f64(prm["W_c2"]).T + _f64(prm["b_c2"])).reshape(B, m, d)
+    H = C if H_in is None else C + _f64(H_in)[:, :m]
+    Wkv, Wqkv = _f64(prm["W_kvh"]), _f64(prm["W_qkv"])
+    st = {k: np.zeros((B, spec.capacity, d)) for k in ("K_proxy", "V_proxy")}
+    st.update({k: np.zeros((B, P, d)) for k in ("X_open", "K_open", "V_open")})
+    st["K_proxy"][:, :m] = H @ Wkv[:d].T
+    st["V_proxy"][:, :m] = H @ Wkv[d:].T
+    Xr = X[:, m * P:]
+    st["X_open"][:, :r] = Xr
+    st["K_open"][:, :r] = Xr @ Wqkv[d:2 * d].T
+    st["V_open"][:, :r] = Xr @ Wqkv[2 * d:].T
+    st["n_proxy"] = np.full(B, m, dtype=np.int32)
+    st["n_open"] = np.full(B, r, dtype=np.int32)
+    return st

@@ -70,6 +70,7 @@ class AppendParams(ctypes.Structure):
 EXPORTED = ("proxy_layer_check", "proxy_layer_saved_size", "proxy_layer_workspace_size",
             "proxy_layer_fwd", "proxy_layer_bwd", "proxy_decode_workspace_size",
             "proxy_decode_step", "proxy_append_workspace_size", "proxy_kv_append",
+            "proxy_prefill_workspace_size", "proxy_kv_prefill",
             "pf_last_error", "pf_sync_check", "pf_gemm_bf16", "pf_timing_enable",
             "pf_timing_collect", "pf_timing_label", "pf_timing_ms", "pf_timing_launches",
             "pf_timing_flops", "pf_timing_bytes", "proxy_layer_bwd_noalloc")
@@ -109,6 +110,11 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.proxy_append_workspace_size.restype = sz
     lib.proxy_kv_append.argtypes = [P(DecodeDesc), P(AppendParams), _vp, P(KVCache), _vp, sz, _vp]
     lib.proxy_kv_append.restype = ctypes.c_int
+    lib.proxy_prefill_workspace_size.argtypes = [P(DecodeDesc), ctypes.c_int32]
+    lib.proxy_prefill_workspace_size.restype = sz
+    lib.proxy_kv_prefill.argtypes = [P(DecodeDesc), P(AppendParams), P(DecodeParams), _vp,
+                                     ctypes.c_int32, _vp, P(KVCache), _vp, sz, _vp]
+    lib.proxy_kv_prefill.restype = ctypes.c_int
     lib.pf_last_error.argtypes = []
     lib.pf_last_error.restype = ctypes.c_char_p
     lib.pf_sync_check.argtypes = [_vp]
@@ -213,6 +219,17 @@ def proxy_append_workspace_size(desc: DecodeDesc) -> int:
 def proxy_kv_append(desc, params, H_in, cache, ws, ws_bytes, stream=None):
     _check(load().proxy_kv_append(ctypes.byref(desc), ctypes.byref(params), _ptr(H_in),
                                   ctypes.byref(cache), _ptr(ws), int(ws_bytes), stream))
+
+
+def proxy_prefill_workspace_size(desc: DecodeDesc, L_hist: int) -> int:
+    return load().proxy_prefill_workspace_size(ctypes.byref(desc), int(L_hist))
+
+
+def proxy_kv_prefill(desc, aparams, dparams, X_hist, L_hist, H_in, cache, ws, ws_bytes,
+                     stream=None):
+    _check(load().proxy_kv_prefill(ctypes.byref(desc), ctypes.byref(aparams),
+                                   ctypes.byref(dparams), _ptr(X_hist), int(L_hist), _ptr(H_in),
+                                   ctypes.byref(cache), _ptr(ws), int(ws_bytes), stream))
 
 
 def pf_sync_check(stream=None) -> None:

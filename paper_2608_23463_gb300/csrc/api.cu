@@ -995,6 +995,142 @@ pf_status proxy_kv_append(const pf_decode_desc* desc, const pf_append_params* pr
   return PF_OK;
 }
 
+// ---------------------------------------------------------------- prefill
+namespace {
+
+struct PrefillWs {
+  bf16 *Xc, *Y, *Hb;  // gathered blocks [B m P, d] (remainder and B > 1), level-1 rows
+                      // [B m k2, d] (two levels), proxies [B m, d]
+};
+
+PrefillWs carve_prefill(Carve& c, const pf_decode_desc& s, long L_hist) {
+  PrefillWs w{};
+  const long m = L_hist / s.P, r = L_hist - m * s.P, B = s.batch;
+  const long k2 = s.levels == 2 ? s.k2 : 1;
+  if (r > 0 && B > 1) w.Xc = c.take<bf16>((size_t)B * m * s.P * s.d);
+  if (s.levels == 2) w.Y = c.take<bf16>((size_t)B * m * k2 * s.d);
+  w.Hb = c.take<bf16>((size_t)B * m * s.d);
+  return w;
+}
+
+}  // namespace
+
+size_t proxy_prefill_workspace_size(const pf_decode_desc* desc, int32_t L_hist) {
+  if (check_decode_desc(desc) != PF_OK || L_hist < 0) return 0;
+  Carve c(nullptr);
+  carve_prefill(c, *desc, L_hist);
+  return ((c.off + 255) & ~size_t(255)) + 256;
+}
+
+pf_status proxy_kv_prefill(const pf_decode_desc* desc, const pf_append_params* ap,
+                           const pf_decode_params* dp, const void* X_hist, int32_t L_hist,
+                           const float* H_in, pf_kv_cache* cache, void* ws, size_t ws_bytes,
+                           void* stream) {
+  pf_status st = check_decode_desc(desc);
+  if (st != PF_OK) return st;
+  const pf_decode_desc& s = *desc;
+  if (L_hist < 0) return fail(PF_ERR_INVALID_ARG, "L_hist must be >= 0");
+  const long P = s.P, d = s.d, B = s.batch;
+  const long m = L_hist / P, r = L_hist - m * P;
+  if (m > s.capacity)
+    return fail(PF_ERR_CAPACITY, "history of %d tokens needs %ld proxies; capacity %d", L_hist, m,
+                s.capacity);
+  if (!ap || !ap->W_c1 || !ap->b_c1 || !ap->W_kvh || (s.levels == 2 && (!ap->W_c2 || !ap->b_c2)))
+    return fail(PF_ERR_INVALID_ARG, "an append parameter is NULL");
+  if (r > 0 && (!dp || !dp->W_qkv))
+    return fail(PF_ERR_INVALID_ARG, "the decode W_qkv is required for an open remainder");
+  if ((L_hist > 0 && X_hist == nullptr) || !cache_ok(cache) || !aligned16(X_hist) ||
+      !aligned16(H_in) || !aligned16(ws) || !aligned16(ap->W_c1) || !aligned16(ap->b_c1) ||
+      !aligned16(ap->W_c2) || !aligned16(ap->b_c2) || !aligned16(ap->W_kvh) ||
+      (dp && !aligned16(dp->W_qkv)))
+    return fail(PF_ERR_INVALID_ARG, "every cache buffer is required; buffers 16-byte aligned");
+  Carve wc(ws);
+  const PrefillWs w = carve_prefill(wc, s, L_hist);
+  if ((m > 0 && ws == nullptr) || wc.off > ws_bytes)
+    return fail(PF_ERR_WORKSPACE, "workspace too small: need %zu bytes, got %zu", wc.off, ws_bytes);
+  cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  const long k1 = s.levels == 2 ? s.k1 : P, k2 = s.levels == 2 ? s.k2 : 1;
+  const bf16* X = static_cast<const bf16*>(X_hist);
+  const bf16* Wkv = static_cast<const bf16*>(ap->W_kvh);
+  if (m > 0) {
+    // all sequences' complete blocks as one matrix of rows of k1 tokens:
+    // in place when they are contiguous, else gathered
+    const bf16* Xb = X;
+    if (r > 0 && B > 1) {
+      PF_CUDA(cudaMemcpy2DAsync(w.Xc, (size_t)m * P * d * sizeof(bf16), X,
+                                (size_t)L_hist * d * sizeof(bf16), (size_t)m * P * d * sizeof(bf16),
+                                (size_t)B, cudaMemcpyDeviceToDevice, cs));
+      Xb = w.Xc;
+    }
+    // the proxies H = H_in + C(block) (Eq. proxy-res, Eq. compress-linear /
+    // factor-cascade), rows (b, i) in sequence order.  H_in has ceil(L_hist/P)
+    // rows per sequence: with a partial block and several sequences its rows
+    // are not those of the output, and the last GEMM runs per sequence.
+    const long mh = m + (r > 0 ? 1 : 0);
+    const bool per_seq = H_in != nullptr && mh != m && B > 1;
+    const bf16* Wc1 = static_cast<const bf16*>(ap->W_c1);
+    if (s.levels == 2) {
+      EpiLinearArgs e;
+      e.bias = ap->b_c1;
+      e.out_bf16 = w.Y;
+      e.ld_bf16 = d;
+      set_gemm_tag("prefill_compress_c1", (double)B * m * k2 * d * 2.0);
+      PF_CUDA(gemm_linear((int)(B * m * k2), (int)d, (int)(k1 * d), {Xb, k1 * d, 0},
+                          {Wc1, k1 * d, 0}, e, cs));
+    }
+    // the last level: W_c1 over the blocks (one level) or W_c2 over the
+    // level-1 rows (two levels), plus b and H_in
+    const bf16* A = s.levels == 2 ? w.Y : Xb;
+    const long lda = s.levels == 2 ? k2 * d : k1 * d;
+    const bf16* Wl = s.levels == 2 ? static_cast<const bf16*>(ap->W_c2) : Wc1;
+    const float* bl = s.levels == 2 ? ap->b_c2 : ap->b_c1;
+    for (long b = 0; b < (per_seq ? B : 1); ++b) {
+      EpiLinearArgs e;
+      e.bias = bl;
+      e.addend = H_in ? H_in + b * mh * d : nullptr;
+      e.ld_add = d;
+      e.out_bf16 = w.Hb + b * m * d;
+      e.ld_bf16 = d;
+      const long rows = per_seq ? m : B * m;
+      set_gemm_tag(s.levels == 2 ? "prefill_compress_c2" : "prefill_compress_c1",
+                   (double)rows * d * 2.0);
+      PF_CUDA(gemm_linear((int)rows, (int)d, (int)lda, {A + b * m * lda, lda, 0}, {Wl, lda, 0},
+                          e, cs));
+    }
+    // their key and value rows into cache rows 0..m-1 of each sequence (one
+    // GEMM over all sequences when the cache rows are contiguous, m = capacity)
+    const bool whole = m == s.capacity;
+    for (long b = 0; b < (whole ? 1 : B); ++b)
+      for (int kv = 0; kv < 2; ++kv) {
+        EpiLinearArgs e;
+        e.out_bf16 =
+            static_cast<bf16*>(kv ? cache->V_proxy : cache->K_proxy) + b * (long)s.capacity * d;
+        e.ld_bf16 = d;
+        const long rows = whole ? B * m : m;
+        set_gemm_tag("prefill_kv", (double)rows * d * 2.0);
+        PF_CUDA(gemm_linear((int)rows, (int)d, (int)d, {w.Hb + b * m * d, d, 0},
+                            {Wkv + kv * d * d, d, 0}, e, cs));
+      }
+  }
+  // the remaining tokens: the open block's features, keys and values
+  for (long b = 0; b < B && r > 0; ++b) {
+    const bf16* Xr = X + (b * (long)L_hist + m * P) * d;
+    bf16* Xo = static_cast<bf16*>(cache->X_open) + b * P * d;
+    PF_CUDA(cudaMemcpyAsync(Xo, Xr, (size_t)r * d * sizeof(bf16), cudaMemcpyDeviceToDevice, cs));
+    const bf16* Wqkv = static_cast<const bf16*>(dp->W_qkv);
+    for (int kv = 0; kv < 2; ++kv) {
+      EpiLinearArgs e;
+      e.out_bf16 = static_cast<bf16*>(kv ? cache->V_open : cache->K_open) + b * P * d;
+      e.ld_bf16 = d;
+      set_gemm_tag("prefill_open_kv", (double)r * d * 2.0);
+      PF_CUDA(gemm_linear((int)r, (int)d, (int)d, {Xr, d, 0}, {Wqkv + (1 + kv) * d * d, d, 0}, e,
+                          cs));
+    }
+  }
+  PF_CUDA(prefill_counts(cache->n_open, cache->n_proxy, (int)B, (int)m, (int)r, cs));
+  return PF_OK;
+}
+
 pf_status pf_sync_check(void* stream) {
   PF_CUDA(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
   PF_CUDA(cudaGetLastError());

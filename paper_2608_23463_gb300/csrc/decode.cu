@@ -517,6 +517,21 @@ cudaError_t decode_step_launch(const DecodeLaunch& L, cudaStream_t st) {
   return cudaSuccess;
 }
 
+// Prefill: every sequence's cache holds m proxies and r open tokens.
+__global__ void prefill_counts_kernel(int* n_open, int* n_proxy, int B, int m, int r) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b < B) {
+    n_proxy[b] = m;
+    n_open[b] = r;
+  }
+}
+
+cudaError_t prefill_counts(int* n_open, int* n_proxy, int B, int m, int r, cudaStream_t st) {
+  LaunchTimer lt("prefill_counts", st, 0.0, 8.0 * B);
+  prefill_counts_kernel<<<(B + 127) / 128, 128, 0, st>>>(n_open, n_proxy, B, m, r);
+  return cudaGetLastError();
+}
+
 cudaError_t append_finish(int* n_open, int* n_proxy, int B, int P, int cap, cudaStream_t st) {
   LaunchTimer lt("append_finish", st, 0.0, 16.0 * B);
   append_finish_kernel<<<1, 32 * ((B + 31) / 32), 0, st>>>(n_open, n_proxy, B, P, cap);

@@ -152,6 +152,8 @@ size_t decode_workspace_bytes(int B, int d, int nh, int splits);
 int decode_splits(int B, int nh, int cap);
 cudaError_t decode_step_launch(const DecodeLaunch& L, cudaStream_t st);
 cudaError_t append_finish(int* n_open, int* n_proxy, int B, int P, int cap, cudaStream_t st);
+// n_proxy[b] = m, n_open[b] = r for every sequence (bulk prefill)
+cudaError_t prefill_counts(int* n_open, int* n_proxy, int B, int m, int r, cudaStream_t st);
 
 // 2D bf16 TMA map over a row-major [outer, inner] matrix (ld elements per
 // row), 128-byte swizzle, zero fill outside; box box_inner x box_outer.

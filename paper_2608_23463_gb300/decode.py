@@ -2,7 +2,8 @@
 
 ``ProxyKVCache`` keeps the decode-side parameters, the cache state and the
 workspaces on the device and calls ``proxy_decode_step`` / ``proxy_kv_append``
-on the current CUDA stream.  It does no arithmetic of its own.
+/ ``proxy_kv_prefill`` on the current CUDA stream.  It does no arithmetic of
+its own.
 """
 from __future__ import annotations
 
@@ -12,7 +13,8 @@ import numpy as np
 import torch
 
 from . import (AppendParams, DecodeDesc, DecodeParams, KVCache, _ptr, proxy_append_workspace_size,
-               proxy_decode_step, proxy_decode_workspace_size, proxy_kv_append)
+               proxy_decode_step, proxy_decode_workspace_size, proxy_kv_append, proxy_kv_prefill,
+               proxy_prefill_workspace_size)
 
 
 def _dev(a, dtype, device):
@@ -65,3 +67,16 @@ class ProxyKVCache:
     def append(self, H_in: torch.Tensor = None) -> None:
         proxy_kv_append(self.desc, self.ap, H_in, self.cache, self.ws, self.ws.numel(),
                         torch.cuda.current_stream().cuda_stream)
+
+    def prefill(self, X_hist: torch.Tensor, H_in: torch.Tensor = None,
+                ws: torch.Tensor = None) -> None:
+        """Fill the cache from a history X_hist [batch, L_hist, d] (bf16): its
+        complete blocks' proxies and the remaining tokens' open block.  ``ws``
+        may hold a workspace of proxy_prefill_workspace_size bytes (allocated
+        here if None)."""
+        L_hist = int(X_hist.shape[1])
+        need = proxy_prefill_workspace_size(self.desc, L_hist)
+        if ws is None or ws.numel() < need:
+            ws = torch.empty(max(need, 16), dtype=torch.uint8, device=X_hist.device)
+        proxy_kv_prefill(self.desc, self.ap, self.dp, X_hist, L_hist, H_in, self.cache, ws,
+                         ws.numel(), torch.cuda.current_stream().cuda_stream)

@@ -34,12 +34,23 @@ class ProxyStack:
         """True if layer l receives H from layer l-1 (same block size)."""
         return l > 0 and self.specs[l].P == self.specs[l - 1].P
 
-    def forward(self, X0: torch.Tensor) -> torch.Tensor:
+    def forward(self, X0: torch.Tensor, train: bool = True) -> torch.Tensor:
         self.X[0].copy_(X0)
         for l, lay in enumerate(self.layers):
             H_in = self.H[l - 1] if self.carries(l) else None
-            lay.forward(self.X[l], H_in, X_out=self.X[l + 1], H_out=self.H[l])
+            lay.forward(self.X[l], H_in, X_out=self.X[l + 1], H_out=self.H[l], train=train)
         return self.X[-1]
+
+    def prefill(self, X_hist: torch.Tensor, caches: List) -> torch.Tensor:
+        """Prefill stage (Sec. 3.8): the stack's inference forward over the
+        history, then each layer's proxy KV cache (a ProxyKVCache holding that
+        layer's compression weights) filled from the layer's input X[l] and
+        the proxy stream it received.  Returns the last layer's output."""
+        assert len(caches) == len(self.layers)
+        out = self.forward(X_hist, train=False)
+        for l, cache in enumerate(caches):
+            cache.prefill(self.X[l], self.H[l - 1] if self.carries(l) else None, ws=self.ws)
+        return out
 
     def backward(self, G: torch.Tensor) -> torch.Tensor:
         n = len(self.layers)

@@ -211,6 +211,28 @@ def make_decode_params(spec: DecodeSpec, seed: int) -> Dict[str, np.ndarray]:
     return out
 
 
+def decode_spec_for_layer(spec: "LayerSpec", capacity: int) -> DecodeSpec:
+    """The proxy KV cache of one causal layer: its width, heads and block
+    factors, room for `capacity` proxies per sequence."""
+    return DecodeSpec(batch=spec.batch, d=spec.d, n_heads=spec.n_heads, P=spec.P,
+                      levels=spec.levels, k1=spec.k1 if spec.levels == 2 else 0,
+                      k2=spec.k2 if spec.levels == 2 else 0, capacity=capacity)
+
+
+def decode_params_for_layer(spec: "LayerSpec", layer_params: Dict[str, np.ndarray],
+                            seed: int) -> Dict[str, np.ndarray]:
+    """Decode-side parameters of a layer: the layer's own compression weights
+    (W_c1, b_c1, W_c2, b_c2) and, as the proxy key/value projection W_kvh, the
+    key and value rows of the layer's W_qkv; the decode-only weights (token
+    W_qkv, W_o, RMSNorm, gate MLP) drawn from `seed`."""
+    out = make_decode_params(decode_spec_for_layer(spec, 1), seed)
+    for k in ("W_c1", "b_c1", "W_c2", "b_c2"):
+        if k in layer_params:
+            out[k] = layer_params[k]
+    out["W_kvh"] = np.ascontiguousarray(layer_params["W_qkv"][spec.d:])
+    return out
+
+
 def make_decode_state(spec: DecodeSpec, seed: int, n_proxy, n_open):
     """Cache contents ~ N(0,1): K/V proxy rows [B, capacity, d] (rows past
     n_proxy[b] are filled too, and must be ignored), open-block features and

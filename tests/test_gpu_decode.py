@@ -5,7 +5,8 @@ open blocks from empty to the last slot, batches beyond one 8-sequence GEMV
 launch, single- and two-level append compression, the streaming rule (P
 decode steps then an append), the paper-size decode (B = 8, d = 2048, 16 x 128
 heads, 16384 cached proxies, 63 open tokens), and capacity errors that must
-leave the offending sequence untouched.
+leave the offending sequence untouched, and the bulk prefill from a history
+(gathered and in-place blocks, empty and sub-block histories, paper width).
 """
 import numpy as np
 import pytest
@@ -152,3 +153,67 @@ def test_graph_replay_equals_direct_steps():
     for k in direct.s:
         assert torch.equal(direct.s[k], graphed.s[k]), k
     assert graphed.s["n_open"].cpu().numpy().tolist() == [2, 9, 16]
+
+
+_PREFILL_CASES = [
+    # levels, batch, P blocks m, remainder r, capacity, with H_in
+    (1, 3, 4, 5, 6, True),     # remainder with B > 1: blocks gathered first
+    (2, 3, 4, 0, 4, False),    # m == capacity: one K/V GEMM over all sequences
+    (2, 1, 3, 15, 10, True),   # one sequence: blocks read in place
+    (1, 2, 0, 9, 3, False),    # shorter than a block: open block only
+    (2, 2, 0, 0, 3, False),    # empty history
+]
+
+
+@pytest.mark.parametrize("levels,batch,m,r,cap,with_h", _PREFILL_CASES)
+def test_prefill_matches_oracle(levels, batch, m, r, cap, with_h):
+    """Bulk prefill (Sec. 3.8) against the oracle's: proxy K/V rows below m,
+    open-block rows below r, counters m and r.  The cache starts full of
+    unrelated rows, which prefill must overwrite from row 0."""
+    P, d = 16, 256
+    spec = S.DecodeSpec(batch=batch, d=d, n_heads=2, P=P, levels=levels,
+                        k1=4 if levels == 2 else 0, k2=4 if levels == 2 else 0, capacity=cap)
+    prm = S.make_decode_params(spec, 30 + levels)
+    st0 = S.make_decode_state(spec, 31, [cap] * batch, [P - 1] * batch)
+    cache = ProxyKVCache(spec, prm, st0)
+    rng = np.random.default_rng(32)
+    X = S.round_bf16(rng.standard_normal((batch, m * P + r, d)).astype(np.float32))
+    H = rng.standard_normal((batch, m + (r > 0), d)).astype(np.float32) if with_h else None
+    cache.prefill(torch.from_numpy(X).to("cuda", torch.bfloat16),
+                  None if H is None else torch.from_numpy(H).cuda())
+    _sync()
+    ref = OD.kv_prefill(spec, prm, X, H)
+    assert cache.s["n_proxy"].cpu().numpy().tolist() == [m] * batch
+    assert cache.s["n_open"].cpu().numpy().tolist() == [r] * batch
+    if m:
+        for k in ("K_proxy", "V_proxy"):
+            assert_close(k, _np(cache.s[k][:, :m]), ref[k][:, :m])
+    if r:
+        assert np.array_equal(_np(cache.s["X_open"][:, :r]), ref["X_open"][:, :r])
+        for k in ("K_open", "V_open"):
+            assert_close(k, _np(cache.s[k][:, :r]), ref[k][:, :r])
+    # the next decode step reads the prefilled cache
+    st = {k: (_np(v) if v.dtype == torch.bfloat16 else v.cpu().numpy()) for k, v in cache.s.items()}
+    st["x"] = S.round_bf16(rng.standard_normal((batch, d)).astype(np.float32))
+    _check_step(spec, prm, st, cache)
+
+
+def test_prefill_paper_width():
+    """d = 2048, 16 x 128 heads, P = 64 as 8 x 8 factors, eight sequences of
+    3 blocks and 17 open tokens (a short history keeps the float64 oracle fast)."""
+    spec = S.DecodeSpec(batch=8, d=2048, n_heads=16, P=64, levels=2, k1=8, k2=8, capacity=5)
+    prm = S.make_decode_params(spec, 40)
+    cache = ProxyKVCache(spec, prm, S.make_decode_state(spec, 41, [5] * 8, [0] * 8))
+    rng = np.random.default_rng(42)
+    X = S.round_bf16(rng.standard_normal((8, 3 * 64 + 17, 2048)).astype(np.float32))
+    H = rng.standard_normal((8, 4, 2048)).astype(np.float32)  # 3 blocks + the partial one
+    cache.prefill(torch.from_numpy(X).to("cuda", torch.bfloat16), torch.from_numpy(H).cuda())
+    _sync()
+    ref = OD.kv_prefill(spec, prm, X, H)
+    for k in ("K_proxy", "V_proxy"):
+        assert_close(k, _np(cache.s[k][:, :3]), ref[k][:, :3])
+    assert np.array_equal(_np(cache.s["X_open"][:, :17]), ref["X_open"][:, :17])
+    for k in ("K_open", "V_open"):
+        assert_close(k, _np(cache.s[k][:, :17]), ref[k][:, :17])
+    assert cache.s["n_proxy"].cpu().numpy().tolist() == [3] * 8
+    assert cache.s["n_open"].cpu().numpy().tolist() == [17] * 8

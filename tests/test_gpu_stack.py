@@ -3,7 +3,8 @@ float64 oracle composed layer by layer: H is carried between layers with the
 same P and re-extracted when P changes; the backward follows the same rule.
 Bar: X_out RMS 3e-2; dX and weight gradients RMS 1e-1, max 1 -- twice the
 bf16 floor of this stack (test_bf16_error_floor.py), well below the O(1)
-error of a wrong carry rule."""
+error of a wrong carry rule.  The stack prefill must fill every layer's proxy
+KV cache from that layer's own input and proxy stream."""
 import numpy as np
 import pytest
 import torch
@@ -60,3 +61,42 @@ def test_stack_matches_composed_oracle():
         for k in ("W_c1", "W_d1", "W_qkv", "b_g"):
             assert_grad_close(f"layer {l} grad {k}", st.layers[l].grads[k].cpu().numpy(), gr[k],
                               tol=1e-1, max_tol=1.0)
+
+
+def test_stack_prefill_fills_every_layer_cache():
+    """Prefill (Sec. 3.8) through a stack: each layer's cache must equal the
+    oracle's bulk prefill of that layer's own input X[l] and incoming proxy
+    stream.  Ragged history (partial last block) with two sequences, so the
+    carried stream's extra row per sequence is skipped; P changes once."""
+    from oracle import decode as OD
+    from paper_2608_23463_gb300.decode import ProxyKVCache
+    ratios = (16, 16, 32)
+    B, L, d, nh = 2, 1000, 128, 2
+    specs = []
+    for P in ratios:
+        k1, k2 = S.default_factors(P)
+        specs.append(S.LayerSpec(batch=B, L=L, d=d, n_heads=nh, P=P, levels=2, k1=k1, k2=k2))
+    specs[2] = S.LayerSpec(batch=B, L=L, d=d, n_heads=nh, P=32)  # one level
+    params = [S.make_layer_params(s, 90 + i) for i, s in enumerate(specs)]
+    st = ProxyStack(specs, params)
+    dspecs = [S.decode_spec_for_layer(s, L // s.P + 2) for s in specs]
+    dprms = [S.decode_params_for_layer(s, p, 95 + i) for i, (s, p) in enumerate(zip(specs, params))]
+    caches = [ProxyKVCache(ds, dp, S.make_decode_state(ds, 96, [ds.capacity] * B, [5] * B))
+              for ds, dp in zip(dspecs, dprms)]
+    X = torch.from_numpy(S.make_layer_inputs(specs[0], 97, with_grads=False)["X"])
+    st.prefill(X.cuda().to(torch.bfloat16), caches)
+    pf.pf_sync_check(torch.cuda.current_stream().cuda_stream)
+    for l, (ds, dp, c) in enumerate(zip(dspecs, dprms, caches)):
+        m, r = L // ds.P, L % ds.P
+        Xl = st.X[l].float().cpu().numpy()
+        H = st.H[l - 1].cpu().numpy() if st.carries(l) else None
+        ref = OD.kv_prefill(ds, dp, Xl, H)
+        assert c.s["n_proxy"].cpu().numpy().tolist() == [m] * B
+        assert c.s["n_open"].cpu().numpy().tolist() == [r] * B
+        for k in ("K_proxy", "V_proxy"):
+            assert_grad_close(f"layer {l} {k}", c.s[k][:, :m].float().cpu().numpy(), ref[k][:, :m],
+                              tol=2e-2, max_tol=1e-1)
+        assert np.array_equal(c.s["X_open"][:, :r].float().cpu().numpy(), Xl[:, m * ds.P:])
+        for k in ("K_open", "V_open"):
+            assert_grad_close(f"layer {l} {k}", c.s[k][:, :r].float().cpu().numpy(), ref[k][:, :r],
+                              tol=2e-2, max_tol=1e-1)

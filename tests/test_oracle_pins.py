@@ -375,6 +375,35 @@ def test_p8_alpha_limits():
 
 
 @pytest.mark.parametrize("levels", [1, 2])
+@pytest.mark.parametrize("with_h", [False, True])
+def test_prefill_equals_appends_and_decode_writes(levels, with_h):
+    """Bulk prefill of a history of m P + r tokens equals the streaming path
+    it replaces (Sec. 3.8): m times (P decode steps filling the open block,
+    then an append), then r decode steps -- compared on every cached proxy
+    row, the open block's features, keys and values, and the counters."""
+    spec, prm, st = _dec_setup([0, 0, 0], [0, 0, 0], levels)
+    rng = np.random.default_rng(11)
+    m, r = 2, 3  # r < P
+    X = rng.standard_normal((3, m * spec.P + r, spec.d))
+    # H_in is a layer's proxy stream: one row per block, the partial one included
+    H_in = rng.standard_normal((3, m + 1, spec.d)) if with_h else None
+    for i in range(m):
+        for j in range(spec.P):
+            st = dict(st, x=X[:, i * spec.P + j])
+            _, st = OD.decode_step(spec, prm, st)
+        st = OD.kv_append(spec, prm, st, None if H_in is None else H_in[:, i])
+    for j in range(r):
+        st = dict(st, x=X[:, m * spec.P + j])
+        _, st = OD.decode_step(spec, prm, st)
+    pre = OD.kv_prefill(spec, prm, X, H_in)
+    assert (pre["n_proxy"] == st["n_proxy"]).all() and (pre["n_open"] == st["n_open"]).all()
+    for k in ("K_proxy", "V_proxy"):
+        np.testing.assert_allclose(pre[k][:, :m], st[k][:, :m], rtol=1e-12, atol=1e-12)
+    for k in ("X_open", "K_open", "V_open"):
+        np.testing.assert_allclose(pre[k][:, :r], st[k][:, :r], rtol=1e-12, atol=1e-12)
+
+
+@pytest.mark.parametrize("levels", [1, 2])
 def test_p8_streaming_append_equals_layer_compression(levels):
     """P decode steps fill the open block; the append then caches the same
     proxy the layer's compression (Eq. compress-linear, Eq. proxy-res) makes
