@@ -239,6 +239,26 @@ pf_status proxy_kv_prefill(const pf_decode_desc *desc, const pf_append_params *a
                            const float *H_in, pf_kv_cache *cache, void *ws, size_t ws_bytes,
                            void *stream);
 
+/* Prefill of one causal layer (Sec. 3.8: the prefill stage runs compression
+ * and proxy interaction over the history, then keeps only the proxies' keys
+ * and values).  Runs the layer's inference forward over the history X
+ * ([batch, L, d] bf16, exactly proxy_layer_fwd with saved = NULL, writing
+ * X_out and H_out) and fills `cache` from it:
+ *   K_proxy[b, i], V_proxy[b, i] = the keys and values the forward's proxy
+ *     attention projected for proxy i < m = floor(L / P) (Eq. proxy-attn), so
+ *     the cache's W_kh, W_vh are this layer's W_k, W_v (rows [d, 3d) of its
+ *     W_qkv) and later appends must use those same rows as W_kvh;
+ *   the open block from the last r = L mod P tokens as in proxy_kv_prefill
+ *     (dparams->W_qkv, read only when r > 0); n_proxy[b] = m, n_open[b] = r.
+ * cdesc must match the layer (batch, d, n_heads, P, levels, k1, k2); the
+ * layer must be PF_CAUSAL_1D in PF_BF16 (else PF_ERR_UNSUPPORTED).  ws needs
+ * proxy_layer_workspace_size(desc, 0) bytes.  m > capacity gives
+ * PF_ERR_CAPACITY with nothing launched.                                      */
+pf_status proxy_layer_prefill(const pf_layer_desc *desc, const pf_layer_params *params,
+                              const pf_decode_desc *cdesc, const pf_decode_params *dparams,
+                              const void *X, const float *H_in, void *X_out, float *H_out,
+                              pf_kv_cache *cache, void *ws, size_t ws_bytes, void *stream);
+
 /* Thread-local message describing the last non-OK status of this thread. */
 const char *pf_last_error(void);
 

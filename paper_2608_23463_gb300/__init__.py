@@ -70,7 +70,7 @@ class AppendParams(ctypes.Structure):
 EXPORTED = ("proxy_layer_check", "proxy_layer_saved_size", "proxy_layer_workspace_size",
             "proxy_layer_fwd", "proxy_layer_bwd", "proxy_decode_workspace_size",
             "proxy_decode_step", "proxy_append_workspace_size", "proxy_kv_append",
-            "proxy_prefill_workspace_size", "proxy_kv_prefill",
+            "proxy_prefill_workspace_size", "proxy_kv_prefill", "proxy_layer_prefill",
             "pf_last_error", "pf_sync_check", "pf_gemm_bf16", "pf_timing_enable",
             "pf_timing_collect", "pf_timing_label", "pf_timing_ms", "pf_timing_launches",
             "pf_timing_flops", "pf_timing_bytes", "proxy_layer_bwd_noalloc")
@@ -115,6 +115,10 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.proxy_kv_prefill.argtypes = [P(DecodeDesc), P(AppendParams), P(DecodeParams), _vp,
                                      ctypes.c_int32, _vp, P(KVCache), _vp, sz, _vp]
     lib.proxy_kv_prefill.restype = ctypes.c_int
+    lib.proxy_layer_prefill.argtypes = [P(LayerDesc), P(LayerParams), P(DecodeDesc),
+                                        P(DecodeParams), _vp, _vp, _vp, _vp, P(KVCache), _vp, sz,
+                                        _vp]
+    lib.proxy_layer_prefill.restype = ctypes.c_int
     lib.pf_last_error.argtypes = []
     lib.pf_last_error.restype = ctypes.c_char_p
     lib.pf_sync_check.argtypes = [_vp]
@@ -230,6 +234,14 @@ def proxy_kv_prefill(desc, aparams, dparams, X_hist, L_hist, H_in, cache, ws, ws
     _check(load().proxy_kv_prefill(ctypes.byref(desc), ctypes.byref(aparams),
                                    ctypes.byref(dparams), _ptr(X_hist), int(L_hist), _ptr(H_in),
                                    ctypes.byref(cache), _ptr(ws), int(ws_bytes), stream))
+
+
+def proxy_layer_prefill(desc, params, cdesc, dparams, X, H_in, X_out, H_out, cache, ws,
+                        ws_bytes, stream=None):
+    _check(load().proxy_layer_prefill(ctypes.byref(desc), ctypes.byref(params),
+                                      ctypes.byref(cdesc), ctypes.byref(dparams), _ptr(X),
+                                      _ptr(H_in), _ptr(X_out), _ptr(H_out), ctypes.byref(cache),
+                                      _ptr(ws), int(ws_bytes), stream))
 
 
 def pf_sync_check(stream=None) -> None:

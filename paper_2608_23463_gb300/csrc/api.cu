@@ -123,6 +123,25 @@ Saved carve_saved(Carve& c, const pf_layer_desc& s, const Dims& g) {
   return v;
 }
 
+// The bf16 forward's workspace: padded copy of a ragged X, split-K partials,
+// and the saved activations (in `saved` when given, else here).
+struct FwdWs {
+  bf16* Xpad;
+  float* sk;
+  size_t skb;
+  Saved sv;
+};
+
+FwdWs carve_fwd(Carve& wc, const pf_layer_desc& s, const Dims& g, void* saved) {
+  FwdWs f{};
+  f.Xpad = g.ragged ? wc.take<bf16>(g.B * g.Lp * g.d) : nullptr;
+  f.skb = splitk_need(s, g, false);
+  f.sk = wc.take<float>(f.skb / sizeof(float));
+  Carve sc(saved);
+  f.sv = saved ? carve_saved(sc, s, g) : carve_saved(wc, s, g);
+  return f;
+}
+
 struct BwdWs {
   bf16 *Xpad, *dXpad, *dD, *dZ, *dHbar, *dA, *dQKV, *dHb, *dY;
   float *Di, *dHf, *part, *sk;
@@ -523,9 +542,7 @@ size_t proxy_layer_workspace_size(const pf_layer_desc* desc, int for_backward) {
   } else if (for_backward) {
     carve_bwd(c, *desc, g);
   } else {
-    if (g.ragged) c.take<bf16>(g.B * g.Lp * g.d);
-    c.take<float>(splitk_need(*desc, g, false) / sizeof(float));
-    carve_saved(c, *desc, g);  // used when the forward is given saved == NULL
+    carve_fwd(c, *desc, g, nullptr);  // saved activations here when saved == NULL
   }
   return ((c.off + 255) & ~size_t(255)) + 256;
 }
@@ -553,11 +570,11 @@ pf_status proxy_layer_fwd(const pf_layer_desc* desc, const pf_layer_params* prm,
     return layer_fwd_2d(s, g, *prm, X, H_in, t, X_out, H_out, saved, ws, ws_bytes,
                         static_cast<cudaStream_t>(stream));
   Carve wc(ws);
-  bf16* Xpad = g.ragged ? wc.take<bf16>(g.B * g.Lp * g.d) : nullptr;
-  const size_t skb = splitk_need(s, g, false);
-  float* sk = wc.take<float>(skb / sizeof(float));
-  Carve sc(saved);
-  Saved sv = saved ? carve_saved(sc, s, g) : carve_saved(wc, s, g);
+  const FwdWs fw = carve_fwd(wc, s, g, saved);
+  bf16* Xpad = fw.Xpad;
+  const size_t skb = fw.skb;
+  float* sk = fw.sk;
+  const Saved sv = fw.sv;
   if (wc.off > ws_bytes)
     return fail(PF_ERR_WORKSPACE, "workspace too small: need %zu bytes, got %zu", wc.off, ws_bytes);
   if (ws == nullptr && wc.off > 0) return fail(PF_ERR_WORKSPACE, "workspace is NULL");
@@ -1013,6 +1030,31 @@ PrefillWs carve_prefill(Carve& c, const pf_decode_desc& s, long L_hist) {
   return w;
 }
 
+// The tail of a prefill: each sequence's last r = L_hist mod P tokens become
+// its open block (features, W_k x, W_v x with the decode W_qkv), and the
+// counters are set to m = floor(L_hist / P) proxies and r open tokens.
+pf_status prefill_open(const pf_decode_desc& s, const pf_decode_params* dp, const bf16* X,
+                       long L_hist, pf_kv_cache* cache, cudaStream_t cs) {
+  const long P = s.P, d = s.d, B = s.batch;
+  const long m = L_hist / P, r = L_hist - m * P;
+  for (long b = 0; b < B && r > 0; ++b) {
+    const bf16* Xr = X + (b * L_hist + m * P) * d;
+    bf16* Xo = static_cast<bf16*>(cache->X_open) + b * P * d;
+    PF_CUDA(cudaMemcpyAsync(Xo, Xr, (size_t)r * d * sizeof(bf16), cudaMemcpyDeviceToDevice, cs));
+    const bf16* Wqkv = static_cast<const bf16*>(dp->W_qkv);
+    for (int kv = 0; kv < 2; ++kv) {
+      EpiLinearArgs e;
+      e.out_bf16 = static_cast<bf16*>(kv ? cache->V_open : cache->K_open) + b * P * d;
+      e.ld_bf16 = d;
+      set_gemm_tag("prefill_open_kv", (double)r * d * 2.0);
+      PF_CUDA(gemm_linear((int)r, (int)d, (int)d, {Xr, d, 0}, {Wqkv + (1 + kv) * d * d, d, 0}, e,
+                          cs));
+    }
+  }
+  PF_CUDA(prefill_counts(cache->n_open, cache->n_proxy, (int)B, (int)m, (int)r, cs));
+  return PF_OK;
+}
+
 }  // namespace
 
 size_t proxy_prefill_workspace_size(const pf_decode_desc* desc, int32_t L_hist) {
@@ -1112,23 +1154,49 @@ pf_status proxy_kv_prefill(const pf_decode_desc* desc, const pf_append_params* a
                             {Wkv + kv * d * d, d, 0}, e, cs));
       }
   }
-  // the remaining tokens: the open block's features, keys and values
-  for (long b = 0; b < B && r > 0; ++b) {
-    const bf16* Xr = X + (b * (long)L_hist + m * P) * d;
-    bf16* Xo = static_cast<bf16*>(cache->X_open) + b * P * d;
-    PF_CUDA(cudaMemcpyAsync(Xo, Xr, (size_t)r * d * sizeof(bf16), cudaMemcpyDeviceToDevice, cs));
-    const bf16* Wqkv = static_cast<const bf16*>(dp->W_qkv);
+  return prefill_open(s, dp, X, L_hist, cache, cs);
+}
+
+pf_status proxy_layer_prefill(const pf_layer_desc* desc, const pf_layer_params* prm,
+                              const pf_decode_desc* cdesc, const pf_decode_params* dp,
+                              const void* X, const float* H_in, void* X_out, float* H_out,
+                              pf_kv_cache* cache, void* ws, size_t ws_bytes, void* stream) {
+  pf_status st = check_desc(desc);
+  if (st != PF_OK) return st;
+  st = check_decode_desc(cdesc);
+  if (st != PF_OK) return st;
+  const pf_layer_desc& s = *desc;
+  const pf_decode_desc& c = *cdesc;
+  if (s.mode != PF_CAUSAL_1D || s.dtype != PF_BF16)
+    return fail(PF_ERR_UNSUPPORTED, "prefill needs a causal 1D bf16 layer");
+  if (c.batch != s.batch || c.d != s.d || c.n_heads != s.n_heads || c.P != s.P ||
+      c.levels != s.levels || (s.levels == 2 && (c.k1 != s.k1 || c.k2 != s.k2)))
+    return fail(PF_ERR_INVALID_ARG, "the cache descriptor does not match the layer");
+  const Dims g = dims_of(s);
+  const long m = s.L / s.P, r = s.L - m * s.P, d = s.d, B = s.batch;
+  if (m > c.capacity)
+    return fail(PF_ERR_CAPACITY, "history of %ld tokens needs %ld proxies; capacity %d", (long)s.L,
+                m, c.capacity);
+  if (r > 0 && (!dp || !dp->W_qkv || !aligned16(dp->W_qkv)))
+    return fail(PF_ERR_INVALID_ARG, "the decode W_qkv is required for an open remainder");
+  if (!cache_ok(cache)) return fail(PF_ERR_INVALID_ARG, "every cache buffer is required, 16-byte aligned");
+  // the layer's inference forward; its proxy attention projects K and V of
+  // the proxies H = H_in + C(block) into the saved-activation area of ws
+  st = proxy_layer_fwd(desc, prm, X, H_in, nullptr, X_out, H_out, nullptr, ws, ws_bytes, stream);
+  if (st != PF_OK) return st;
+  cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  Carve wc(ws);
+  const bf16* QKV = carve_fwd(wc, s, g, nullptr).sv.QKV;  // [B, ceil(L/P), 3d]
+  // complete blocks' key and value columns into cache rows 0..m-1
+  const bool whole = m == g.m && m == c.capacity;  // source and cache rows both contiguous
+  for (long b = 0; b < (whole ? 1 : B) && m > 0; ++b)
     for (int kv = 0; kv < 2; ++kv) {
-      EpiLinearArgs e;
-      e.out_bf16 = static_cast<bf16*>(kv ? cache->V_open : cache->K_open) + b * P * d;
-      e.ld_bf16 = d;
-      set_gemm_tag("prefill_open_kv", (double)r * d * 2.0);
-      PF_CUDA(gemm_linear((int)r, (int)d, (int)d, {Xr, d, 0}, {Wqkv + (1 + kv) * d * d, d, 0}, e,
-                          cs));
+      bf16* dst = static_cast<bf16*>(kv ? cache->V_proxy : cache->K_proxy) + b * c.capacity * d;
+      const bf16* src = QKV + b * g.m * 3 * d + (1 + kv) * d;
+      PF_CUDA(cudaMemcpy2DAsync(dst, d * sizeof(bf16), src, 3 * d * sizeof(bf16),
+                                d * sizeof(bf16), whole ? B * m : m, cudaMemcpyDeviceToDevice, cs));
     }
-  }
-  PF_CUDA(prefill_counts(cache->n_open, cache->n_proxy, (int)B, (int)m, (int)r, cs));
-  return PF_OK;
+  return prefill_open(c, dp, static_cast<const bf16*>(X), s.L, cache, cs);
 }
 
 pf_status pf_sync_check(void* stream) {

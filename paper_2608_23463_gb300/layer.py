@@ -12,7 +12,7 @@ import numpy as np
 import torch
 
 from . import (PF_BF16, layer_desc, layer_params, proxy_layer_bwd, proxy_layer_fwd,
-               proxy_layer_saved_size, proxy_layer_workspace_size)
+               proxy_layer_prefill, proxy_layer_saved_size, proxy_layer_workspace_size)
 
 
 def _stream() -> int:
@@ -65,6 +65,15 @@ class ProxyLayer:
         X_out = self.empty_act() if X_out is None else X_out
         proxy_layer_fwd(self.desc, self.p_struct, X, H_in, t, X_out, H_out,
                         self.saved if train else None, self.ws, self.ws.numel(), _stream())
+        return X_out
+
+    def prefill(self, X, cache, H_in=None, X_out=None, H_out=None):
+        """Inference forward over a history plus the fill of `cache` (a
+        ProxyKVCache of this layer) from the forward's own proxy keys and
+        values (Sec. 3.8); see proxy_layer_prefill."""
+        X_out = self.empty_act() if X_out is None else X_out
+        proxy_layer_prefill(self.desc, self.p_struct, cache.desc, cache.dp, X, H_in, X_out, H_out,
+                            cache.cache, self.ws, self.ws.numel(), _stream())
         return X_out
 
     def backward(self, X, dX_out, H_in=None, t=None, dH_out=None, dX=None, dH_in=None):

@@ -42,15 +42,17 @@ class ProxyStack:
         return self.X[-1]
 
     def prefill(self, X_hist: torch.Tensor, caches: List) -> torch.Tensor:
-        """Prefill stage (Sec. 3.8): the stack's inference forward over the
-        history, then each layer's proxy KV cache (a ProxyKVCache holding that
-        layer's compression weights) filled from the layer's input X[l] and
-        the proxy stream it received.  Returns the last layer's output."""
+        """Prefill stage (Sec. 3.8): each layer's inference forward over the
+        history, which also fills that layer's proxy KV cache (a ProxyKVCache
+        whose proxy key/value projection is the layer's own W_k, W_v) with the
+        keys and values its proxy attention computed.  Returns the last
+        layer's output."""
         assert len(caches) == len(self.layers)
-        out = self.forward(X_hist, train=False)
-        for l, cache in enumerate(caches):
-            cache.prefill(self.X[l], self.H[l - 1] if self.carries(l) else None, ws=self.ws)
-        return out
+        self.X[0].copy_(X_hist)
+        for l, (lay, cache) in enumerate(zip(self.layers, caches)):
+            H_in = self.H[l - 1] if self.carries(l) else None
+            lay.prefill(self.X[l], cache, H_in, X_out=self.X[l + 1], H_out=self.H[l])
+        return self.X[-1]
 
     def backward(self, G: torch.Tensor) -> torch.Tensor:
         n = len(self.layers)

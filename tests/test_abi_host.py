@@ -86,3 +86,39 @@ def test_calls_reject_bad_arguments_before_any_launch(pf):
     with pytest.raises(pf.ProxyFormerError) as e:
         pf.pf_gemm_bf16(128, 100, 64, 4096, 0, 4096, 0, 4096, 100)
     assert e.value.status == pf.PF_ERR_INVALID_ARG
+
+
+def test_prefill_rejects_bad_arguments_before_any_launch(pf):
+    """proxy_layer_prefill / proxy_kv_prefill validate the cache descriptor
+    against the layer, the capacity and the cache buffers on the host."""
+    spec = S.LayerSpec(batch=2, L=100, d=128, n_heads=2, P=16)  # m = 6, r = 4
+    desc = pf.layer_desc(spec)
+    prm = pf.layer_params({})
+    cache = pf.KVCache(*([4096] * 7))
+    dp = pf.DecodeParams(*([4096] * 7))
+
+    def call(cdesc, c=cache, d=dp, ldesc=desc):
+        with pytest.raises(pf.ProxyFormerError) as e:
+            pf.proxy_layer_prefill(ldesc, prm, cdesc, d, 4096, None, 8192, None, c, 4096, 1 << 30)
+        return e.value.status
+
+    ok = S.decode_spec_for_layer(spec, 6)
+    mk = lambda ds: pf.DecodeDesc(ds.batch, ds.d, ds.n_heads, ds.P, ds.levels, ds.k1, ds.k2,
+                                  ds.capacity)
+    assert call(mk(S.decode_spec_for_layer(S.LayerSpec(batch=2, L=100, d=128, n_heads=2, P=8),
+                                           6))) == pf.PF_ERR_INVALID_ARG  # other P
+    assert call(mk(S.decode_spec_for_layer(spec, 5))) == pf.PF_ERR_CAPACITY
+    assert call(mk(ok), c=pf.KVCache(*([4096] * 6 + [None]))) == pf.PF_ERR_INVALID_ARG
+    assert call(mk(ok), d=pf.DecodeParams()) == pf.PF_ERR_INVALID_ARG  # r > 0 needs W_qkv
+    s2d = S.spec_c5()
+    assert call(mk(ok), ldesc=pf.layer_desc(s2d)) == pf.PF_ERR_UNSUPPORTED
+    # the standalone prefill from a history
+    ap = pf.AppendParams(*([4096] * 5))
+    with pytest.raises(pf.ProxyFormerError) as e:
+        pf.proxy_kv_prefill(mk(S.decode_spec_for_layer(spec, 5)), ap, dp, 4096, 100, None, cache,
+                            4096, 1 << 30)
+    assert e.value.status == pf.PF_ERR_CAPACITY
+    with pytest.raises(pf.ProxyFormerError) as e:
+        pf.proxy_kv_prefill(mk(ok), ap, dp, 4096, -1, None, cache, 4096, 1 << 30)
+    assert e.value.status == pf.PF_ERR_INVALID_ARG
+    assert pf.proxy_prefill_workspace_size(mk(ok), 100) > pf.proxy_prefill_workspace_size(mk(ok), 0)

@@ -84,8 +84,11 @@ def test_stack_prefill_fills_every_layer_cache():
     caches = [ProxyKVCache(ds, dp, S.make_decode_state(ds, 96, [ds.capacity] * B, [5] * B))
               for ds, dp in zip(dspecs, dprms)]
     X = torch.from_numpy(S.make_layer_inputs(specs[0], 97, with_grads=False)["X"])
-    st.prefill(X.cuda().to(torch.bfloat16), caches)
+    X = X.cuda().to(torch.bfloat16)
+    out = st.prefill(X, caches).clone()
     pf.pf_sync_check(torch.cuda.current_stream().cuda_stream)
+    # the prefill's forward is the plain inference forward (no atomics: bitwise)
+    assert torch.equal(out, st.forward(X, train=False))
     for l, (ds, dp, c) in enumerate(zip(dspecs, dprms, caches)):
         m, r = L // ds.P, L % ds.P
         Xl = st.X[l].float().cpu().numpy()
