@@ -22,6 +22,14 @@ Readings of the paper taken here (each is a descriptor flag of the library):
     [2pd, 2pd+d) and [2pd+d, 2(p+1)d)); Norm is LayerNorm without affine,
     biased variance, eps 1e-6.
   * L % P != 0: the last block is zero-padded for compression (m = ceil(L/P)).
+  * Cross-attention injection (Eq. inj-cross) in its gated form, the way the
+    language model uses it (Eq. llm-cross / llm-gate): every token queries,
+    per head, the interacted proxies it may see (causal: proxies of earlier
+    blocks only, the same one-block shift as above; bidirectional: all of
+    them); a per-head linear gate alpha = sigmoid(W_a x + b_a) scales each
+    head's result; X_out = X + W_ox (alpha * A).  W_qa stacks the token-query
+    projection [d, d] over the gate's rows [heads, d]; W_kvx maps proxies to
+    the injection's keys and values.  No decompression is used.
 """
 from __future__ import annotations
 
@@ -31,7 +39,7 @@ from typing import Dict, Optional
 import numpy as np
 
 CAUSAL_1D, BIDIR_1D, BIDIR_2D = 0, 1, 2
-INJ_ADD, INJ_GATED, INJ_AFFINE = 0, 1, 2
+INJ_ADD, INJ_GATED, INJ_AFFINE, INJ_CROSS = 0, 1, 2, 3
 LN_EPS = 1e-6
 TEMB_DIM = 256
 
@@ -167,6 +175,73 @@ def attention_bwd(dA, c, spec):
     return dQ, dK, dV
 
 
+# ------------------------------------------------- cross-attention injection
+def _cross_visible(t, spec, m):
+    """Proxies token t may read: those of earlier blocks (causal), else all."""
+    return t // spec.P if spec.mode == CAUSAL_1D else m
+
+
+def cross_inject(X, Hbar, prm, spec):
+    """Gated Eq. inj-cross over one sequence: Q = X W_q^T, alpha = sigmoid(
+    X W_a^T + b_a) per head, K, V = Hbar W_k^T, Hbar W_v^T; row t of head h
+    is the softmax over its visible proxies (a token that sees none gets 0);
+    X_out = X + (alpha * A) W_ox^T."""
+    L, d = X.shape
+    m = Hbar.shape[0]
+    nh, dh = spec.n_heads, d // spec.n_heads
+    Wqa, Wkv = _f64(prm["W_qa"]), _f64(prm["W_kvx"])
+    Q = X @ Wqa[:d].T
+    alpha = sigmoid(X @ Wqa[d:].T + _f64(prm["b_a"]))           # [L, heads]
+    K, V = Hbar @ Wkv[:d].T, Hbar @ Wkv[d:].T
+    A = np.zeros((L, d))
+    scale = 1.0 / math.sqrt(dh)
+    for h in range(nh):
+        cs = slice(h * dh, (h + 1) * dh)
+        for t in range(L):
+            n_vis = _cross_visible(t, spec, m)
+            if n_vis:
+                A[t, cs] = _row_probs(Q[t, cs], K[:, cs], n_vis, scale) @ V[:n_vis, cs]
+    Ag = A * np.repeat(alpha, dh, axis=1)
+    Xo = X + Ag @ _f64(prm["W_ox"]).T
+    return Xo, dict(Qx=Q, Kx=K, Vx=V, Ax=A, alpha=alpha, Ag=Ag)
+
+
+def cross_inject_bwd(G, X, Hbar, c, prm, spec, grads):
+    """Chain rule through ``cross_inject``: returns (dX, dHbar) and adds the
+    gradients of W_ox, W_qa, b_a and W_kvx to ``grads``."""
+    L, d = X.shape
+    m = Hbar.shape[0]
+    nh, dh = spec.n_heads, d // spec.n_heads
+    scale = 1.0 / math.sqrt(dh)
+    Q, K, V, A, alpha = c["Qx"], c["Kx"], c["Vx"], c["Ax"], c["alpha"]
+    grads["W_ox"] += G.T @ c["Ag"]
+    dAg = G @ _f64(prm["W_ox"])
+    s = (dAg * A).reshape(L, nh, dh).sum(-1)                     # dL/dalpha
+    da = s * alpha * (1.0 - alpha)                                # through the sigmoid
+    dA = dAg * np.repeat(alpha, dh, axis=1)
+    dQ, dK, dV = np.zeros_like(Q), np.zeros_like(K), np.zeros_like(V)
+    for h in range(nh):
+        cs = slice(h * dh, (h + 1) * dh)
+        for t in range(L):
+            n_vis = _cross_visible(t, spec, m)
+            if not n_vis:
+                continue
+            p = _row_probs(Q[t, cs], K[:, cs], n_vis, scale)
+            dO = dA[t, cs]
+            dV[:n_vis, cs] += np.outer(p, dO)
+            dp = V[:n_vis, cs] @ dO
+            dS = p * (dp - p @ dp)
+            dQ[t, cs] = scale * (dS @ K[:n_vis, cs])
+            dK[:n_vis, cs] += scale * np.outer(dS, Q[t, cs])
+    dQA = np.concatenate([dQ, da], axis=1)
+    Wqa, Wkv = _f64(prm["W_qa"]), _f64(prm["W_kvx"])
+    grads["W_qa"] += dQA.T @ X
+    grads["b_a"] += da.sum(0)
+    dKV = np.concatenate([dK, dV], axis=1)
+    grads["W_kvx"] += dKV.T @ Hbar
+    return G + dQA @ Wqa, dKV @ Wkv
+
+
 # ----------------------------------------------------------- 2D conditioning
 def timestep_embedding(t):
     """Sinusoidal embedding of the flow-matching time t (this library's own
@@ -214,8 +289,13 @@ def _fwd_one(spec, prm, X, H_in, t):
         Hq = (1.0 + gamma) * nH + beta
         cache.update(gamma=gamma, beta=beta, tc=tc, nH=nH, sdH=sdH)
     Hbar, ac = attention(Hq, prm, spec)                       # Eq. proxy-attn
+    cache.update(Hq=Hq, Hbar=Hbar, **ac)
+    if spec.inject == INJ_CROSS:                              # Eq. inj-cross (gated)
+        Xo, cc = cross_inject(X, Hbar, prm, spec)
+        cache.update(cc)
+        return Xo, H, cache
     D, Z = decompress(Hbar, prm, spec)                        # Eq. decompress-linear
-    cache.update(Hq=Hq, Hbar=Hbar, Z=Z, D=D, **ac)
+    cache.update(Z=Z, D=D)
     m = Xb.shape[0]
     if spec.mode == CAUSAL_1D:                                # routing shift
         Dr = np.zeros_like(D)
@@ -262,13 +342,13 @@ def _layernorm_bwd(dn, n, sd):
             - n * (dn * n).mean(-1, keepdims=True)) / sd
 
 
-def _bwd_one(spec, prm, X, c, G, dH_out, grads):
+def _inject_decompress_bwd(spec, prm, X, c, G, grads):
+    """Backward of the decompression, routing and Eq. inj-add / inj-gate /
+    inj-affine: returns (dX direct, dHbar)."""
     L, d = X.shape
     m = c["Xb"].shape[0]
     P, k1, k2 = spec.P, spec.k1, spec.k2
-    nh, dh = spec.n_heads, d // spec.n_heads
     Dt = c["Dt"]
-    # injection (Eq. inj-*)
     if spec.inject == INJ_ADD:
         dX = G.copy()
         dDt = G.copy()
@@ -311,6 +391,18 @@ def _bwd_one(spec, prm, X, c, G, dH_out, grads):
         dHbar = dZ @ _f64(prm["W_d2"])
     else:
         dHbar = drows.reshape(m, d)
+    return dX, dHbar
+
+
+def _bwd_one(spec, prm, X, c, G, dH_out, grads):
+    L, d = X.shape
+    m = c["Xb"].shape[0]
+    P, k1, k2 = spec.P, spec.k1, spec.k2
+    nh, dh = spec.n_heads, d // spec.n_heads
+    if spec.inject == INJ_CROSS:
+        dX, dHbar = cross_inject_bwd(G, X, c["Hbar"], c, prm, spec, grads)
+    else:
+        dX, dHbar = _inject_decompress_bwd(spec, prm, X, c, G, grads)
     # attention
     grads["W_o"] += dHbar.T @ c["A"]
     dA = dHbar @ _f64(prm["W_o"])

@@ -30,7 +30,7 @@ import numpy as np
 
 # mode / inject / dtype codes; they mirror the C header's enums.
 CAUSAL_1D, BIDIR_1D, BIDIR_2D = 0, 1, 2
-INJ_ADD, INJ_GATED, INJ_AFFINE = 0, 1, 2
+INJ_ADD, INJ_GATED, INJ_AFFINE, INJ_CROSS = 0, 1, 2, 3
 F32, BF16 = 0, 1
 
 TEMB_DIM = 256  # width of the sinusoidal timestep embedding (2D layer)
@@ -124,6 +124,14 @@ def layer_param_shapes(spec: LayerSpec) -> Dict[str, tuple]:
         s["b_c2"] = (d,)
     s["W_qkv"] = (3 * d, d)
     s["W_o"] = (d, d)
+    if spec.inject == INJ_CROSS:
+        # token queries stacked over the per-head gate rows; proxy keys and
+        # values of the injection; its output projection
+        s["W_qa"] = (d + spec.n_heads, d)
+        s["b_a"] = (spec.n_heads,)
+        s["W_kvx"] = (2 * d, d)
+        s["W_ox"] = (d, d)
+        return s
     out_tok = 2 * d if spec.inject == INJ_AFFINE else d
     if spec.levels == 2:
         s["W_d2"] = (k2 * d, d)
@@ -152,9 +160,9 @@ def make_layer_params(spec: LayerSpec, seed: int) -> Dict[str, np.ndarray]:
     rng = np.random.default_rng(seed)
     out = {}
     for name, shape in layer_param_shapes(spec).items():
-        if name == "W_qkv":  # three d x d matrices drawn one after another
+        if name in ("W_qkv", "W_kvx"):  # d x d matrices drawn one after another
             d = spec.d
-            a = np.concatenate([_xavier(rng, (d, d)) for _ in range(3)], axis=0)
+            a = np.concatenate([_xavier(rng, (d, d)) for _ in range(shape[0] // d)], axis=0)
         elif len(shape) == 2:
             a = _xavier(rng, shape)
         else:

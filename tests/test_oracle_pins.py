@@ -191,6 +191,10 @@ FD_SPECS = {
                                   mode=S.BIDIR_1D, inject=S.INJ_ADD, dtype=S.F32),
     "2d_affine": S.LayerSpec(batch=2, L=64, d=8, n_heads=2, P=4, mode=S.BIDIR_2D,
                              inject=S.INJ_AFFINE, grid_h=8, grid_w=8, patch=2, dtype=S.F32),
+    "causal_cross_1lvl": S.LayerSpec(batch=2, L=22, d=8, n_heads=2, P=4, inject=S.INJ_CROSS,
+                                     dtype=S.F32),
+    "bidir_cross_2lvl": S.LayerSpec(batch=1, L=24, d=8, n_heads=2, P=4, levels=2, k1=2, k2=2,
+                                    mode=S.BIDIR_1D, inject=S.INJ_CROSS, dtype=S.F32),
 }
 
 
@@ -221,6 +225,89 @@ def test_p5_finite_differences(name):
             fd = (lp - lm) / (2 * eps)
             a = an.reshape(-1)[j]
             assert abs(fd - a) <= 1e-6 * max(1.0, abs(a)), (key, j, fd, a)
+
+
+# --------------------------------------------------- cross-attention injection
+@pytest.mark.parametrize("causal", [True, False])
+def test_cross_injection_equals_masked_sdpa(causal):
+    """Gated Eq. inj-cross against torch SDPA with an explicit boolean mask
+    (token t of block i sees proxies j < i when causal, all otherwise),
+    projections and gate recomputed here with torch: X_out - X must equal
+    (sigmoid(X W_a^T + b_a) * A) W_ox^T, and a token that sees no proxy gets
+    exactly nothing."""
+    P, L, d, nh = 4, 23, 8, 2
+    spec = S.LayerSpec(batch=1, L=L, d=d, n_heads=nh, P=P, inject=S.INJ_CROSS, dtype=S.F32,
+                       mode=S.CAUSAL_1D if causal else S.BIDIR_1D)
+    prm = {k: v.astype(np.float64) for k, v in S.make_layer_params(spec, 41).items()}
+    rng = np.random.default_rng(42)
+    X = rng.standard_normal((L, d))
+    Hbar = rng.standard_normal((spec.m, d))
+    Xo, _ = OL.cross_inject(X, Hbar, prm, spec)
+    T = lambda a: torch.from_numpy(np.asarray(a, np.float64))
+    Xt, Ht = T(X), T(Hbar)
+    Wqa, Wkv = T(prm["W_qa"]), T(prm["W_kvx"])
+    q, k, v = Xt @ Wqa[:d].T, Ht @ Wkv[:d].T, Ht @ Wkv[d:].T
+    alpha = torch.sigmoid(Xt @ Wqa[d:].T + T(prm["b_a"]))
+    vis = torch.ones(L, spec.m, dtype=torch.bool)
+    if causal:
+        vis = torch.arange(spec.m)[None, :] < (torch.arange(L) // P)[:, None]
+    sh = lambda a: a.reshape(a.shape[0], nh, d // nh).transpose(0, 1)
+    rows = vis.any(1)
+    o = F.scaled_dot_product_attention(sh(q[rows]), sh(k), sh(v), attn_mask=vis[rows])
+    A = torch.zeros(L, d, dtype=torch.float64)
+    A[rows] = o.transpose(0, 1).reshape(-1, d)
+    ref = X + ((A.reshape(L, nh, -1) * alpha[:, :, None]).reshape(L, d) @ T(prm["W_ox"]).T).numpy()
+    np.testing.assert_allclose(Xo, ref, rtol=1e-12, atol=1e-12)
+    if causal:
+        assert (Xo[:P] == X[:P]).all()
+
+
+def test_cross_injection_routing_probe():
+    """Uniform attention (W_q = 0) over proxies Hbar_j = 2^j e_0 with identity
+    W_v and W_ox and a zero gate map (alpha = 1/2): token t must receive
+    mean_{j < t//P} 2^j / 2 (to rounding) in every channel, which decodes the
+    set of proxies it read."""
+    P, m, d = 4, 6, 4
+    spec = S.LayerSpec(batch=1, L=P * m - 1, d=d, n_heads=1, P=P, inject=S.INJ_CROSS,
+                       dtype=S.F32)
+    prm = {"W_qa": np.zeros((d + 1, d)), "b_a": np.zeros(1),
+           "W_kvx": np.concatenate([np.eye(d), np.eye(d)]), "W_ox": np.zeros((d, d))}
+    prm["W_ox"][:, 0] = 1.0
+    Hbar = np.zeros((m, d))
+    Hbar[:, 0] = 2.0 ** np.arange(m)
+    X = np.zeros((spec.L, d))
+    Xo, _ = OL.cross_inject(X, Hbar, prm, spec)
+    cand = np.array([0.0] + [np.mean(2.0 ** np.arange(i)) / 2 for i in range(1, m)])
+    for t in range(spec.L):
+        assert np.ptp(Xo[t]) == 0.0
+        i = int(np.argmin(np.abs(cand - Xo[t, 0])))
+        assert i == t // P and abs(Xo[t, 0] - cand[i]) < 1e-12, (t, Xo[t], i)
+
+
+@pytest.mark.parametrize("mode", [S.CAUSAL_1D, S.BIDIR_1D])
+def test_cross_injection_causality(mode):
+    """Causal: perturbing X[t0] leaves X_out bit-identical before the end of
+    t0's block except at t0 (its own query), and changes later blocks.
+    Bidirectional: later blocks' proxies reach earlier tokens."""
+    P = 4
+    spec = S.LayerSpec(batch=1, L=22, d=8, n_heads=2, P=P, mode=mode, inject=S.INJ_CROSS,
+                       dtype=S.F32)
+    inp = S.make_layer_inputs(spec, 43, with_grads=False)
+    X = inp["X"].astype(np.float64)
+    Xo, _ = OL.layer_fwd(spec, inp, X)
+    for t0 in (1, 9, 21):
+        X2 = X.copy()
+        X2[0, t0] += 0.75
+        Xo2, _ = OL.layer_fwd(spec, inp, X2)
+        lim = (t0 // P + 1) * P
+        same = np.ones(spec.L, bool)
+        same[t0] = False
+        if mode == S.CAUSAL_1D:
+            assert (Xo2[0, :lim][same[:lim]] == Xo[0, :lim][same[:lim]]).all()
+            if lim < spec.L:
+                assert np.abs(Xo2[0, lim:] - Xo[0, lim:]).max() > 1e-6
+        else:
+            assert np.abs(Xo2[0, :t0 // P * P] - Xo[0, :t0 // P * P]).max(initial=1.0) > 1e-6
 
 
 # ----------------------------------------------------------------- P6
