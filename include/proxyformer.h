@@ -53,7 +53,7 @@ typedef enum {
 } pf_status;
 
 enum { PF_CAUSAL_1D = 0, PF_BIDIR_1D = 1, PF_BIDIR_2D = 2 };
-enum { PF_INJ_ADD = 0, PF_INJ_GATED = 1, PF_INJ_AFFINE = 2 };
+enum { PF_INJ_ADD = 0, PF_INJ_GATED = 1, PF_INJ_AFFINE = 2, PF_INJ_CROSS = 3 };
 enum { PF_F32 = 0, PF_BF16 = 1 };
 
 /* One ProxyFormer layer (Alg. 1; m = ceil(L/P), Sec. 3.1).
@@ -67,7 +67,14 @@ enum { PF_F32 = 0, PF_BF16 = 1 };
  *   levels     : 1 or 2 (Eq. factor with M = 2); levels == 2 needs k1*k2 == P,
  *                level 1 maps k1 tokens to one row, level 2 k2 rows to a proxy
  *   mode       : PF_CAUSAL_1D | PF_BIDIR_1D | PF_BIDIR_2D (Eq. proxy-attn mask)
- *   inject     : PF_INJ_ADD | PF_INJ_GATED (1D) | PF_INJ_AFFINE (2D)
+ *   inject     : PF_INJ_ADD | PF_INJ_GATED (1D) | PF_INJ_AFFINE (2D) |
+ *                PF_INJ_CROSS (1D, bf16): gated cross-attention (Eq. inj-cross
+ *                in the gated form of Eq. llm-cross / llm-gate): token t of
+ *                block i queries, per head, the interacted proxies j < i
+ *                (causal) or all proxies (bidirectional); a per-head gate
+ *                alpha = sigmoid(W_a x + b_a) scales each head; X_out = X +
+ *                W_ox (alpha * A).  No decompression; a token that sees no
+ *                proxy is left unchanged
  *   dtype      : PF_BF16 (fp32 accumulation) or PF_F32                         */
 typedef struct {
   int32_t batch, L;
@@ -92,6 +99,11 @@ typedef struct {
  *   W_t1 [d, 256] mat, b_t1 [d] vec,       timestep conditioning of the 2D
  *   W_t2 [2d, d] mat, b_t2 [2d] vec        proxies: u = SiLU(W_t1 e(t) + b_t1),
  *                                          [gamma|beta] = W_t2 u + b_t2
+ *   W_qa [d + n_heads, d] mat              PF_INJ_CROSS: token queries (rows
+ *                                          [0, d)) over the gate rows W_a
+ *   b_a [n_heads] vec                      PF_INJ_CROSS: gate bias
+ *   W_kvx [2d, d] mat                      PF_INJ_CROSS: proxy keys, values
+ *   W_ox [d, d] mat                        PF_INJ_CROSS: output projection
  * Unused pointers may be NULL.                                                  */
 typedef struct {
   const void *W_c1;  const float *b_c1;
@@ -102,6 +114,8 @@ typedef struct {
   const float *w_x, *w_dlt, *b_g;
   const void *W_t1;  const float *b_t1;
   const void *W_t2;  const float *b_t2;
+  const void *W_qa;  const float *b_a;
+  const void *W_kvx; const void *W_ox;
 } pf_layer_params;
 
 /* Parameter gradients, fp32 device buffers shaped like pf_layer_params.
@@ -109,6 +123,7 @@ typedef struct {
 typedef struct {
   float *W_c1, *b_c1, *W_c2, *b_c2, *W_qkv, *W_o, *W_d2, *b_d2, *W_d1, *b_d1;
   float *w_x, *w_dlt, *b_g, *W_t1, *b_t1, *W_t2, *b_t2;
+  float *W_qa, *b_a, *W_kvx, *W_ox;
 } pf_layer_grads;
 
 /* Validates a descriptor; PF_OK or the reason it is rejected. */

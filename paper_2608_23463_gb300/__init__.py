@@ -19,7 +19,7 @@ LIB_PATH = os.path.join(_HERE, "libproxyformer.so")
 PF_OK, PF_ERR_INVALID_ARG, PF_ERR_UNSUPPORTED, PF_ERR_WORKSPACE = 0, 1, 2, 3
 PF_ERR_CAPACITY, PF_ERR_CUDA, PF_ERR_TIMEOUT = 4, 5, 6
 PF_CAUSAL_1D, PF_BIDIR_1D, PF_BIDIR_2D = 0, 1, 2
-PF_INJ_ADD, PF_INJ_GATED, PF_INJ_AFFINE = 0, 1, 2
+PF_INJ_ADD, PF_INJ_GATED, PF_INJ_AFFINE, PF_INJ_CROSS = 0, 1, 2, 3
 PF_F32, PF_BF16 = 0, 1
 
 _c_i32 = ctypes.c_int32
@@ -38,7 +38,8 @@ class LayerDesc(ctypes.Structure):
 
 
 _PARAM_NAMES = ("W_c1", "b_c1", "W_c2", "b_c2", "W_qkv", "W_o", "W_d2", "b_d2", "W_d1", "b_d1",
-                "w_x", "w_dlt", "b_g", "W_t1", "b_t1", "W_t2", "b_t2")
+                "w_x", "w_dlt", "b_g", "W_t1", "b_t1", "W_t2", "b_t2", "W_qa", "b_a", "W_kvx",
+                "W_ox")
 
 
 class LayerParams(ctypes.Structure):

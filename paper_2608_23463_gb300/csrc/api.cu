@@ -49,7 +49,8 @@ struct Carve {
 // Derived sizes of a validated 1D / 2D layer.
 struct Dims {
   long B, L, d, nh, P, k1, k2, m, R, rows1, N1, Lp;
-  bool causal, ragged;
+  long T, ldq;  // tokens B*L; width of the token-query matrix [Q | gate | 0] (cross)
+  bool causal, ragged, cross;
 };
 
 Dims dims_of(const pf_layer_desc& s) {
@@ -68,6 +69,9 @@ Dims dims_of(const pf_layer_desc& s) {
   g.Lp = g.m * g.P;
   g.causal = s.mode == PF_CAUSAL_1D;
   g.ragged = g.Lp != g.L;
+  g.cross = s.inject == PF_INJ_CROSS;
+  g.T = g.B * g.L;
+  g.ldq = g.d + 64;  // the gate's n_heads <= 64 rows, zero-padded to 64
   return g;
 }
 
@@ -91,6 +95,12 @@ size_t splitk_need(const pf_layer_desc& s, const Dims& g, bool bwd) {
     v = {{N1, d, r1}, {r1, d, N1}, {d, d, R}, {R, d, d}, {3 * d, d, R}, {R, d, 3 * d}, {d, N1, r1}};
     if (s.levels == 2) v.insert(v.end(), {{n2, d, R}, {R, d, n2}, {d, n2, R}, {R, n2, d}});
   }
+  if (g.cross) {  // token queries + gate, proxy keys / values, output projection
+    const int T = (int)g.T, q = (int)g.ldq, nh = (int)g.nh;
+    if (!bwd) v.insert(v.end(), {{T, q, d}, {R, 2 * d, d}, {T, d, d}});
+    else v.insert(v.end(), {{d, d, T}, {T, d, d}, {d + nh, d, T}, {2 * d, d, R}, {R, d, 2 * d},
+                            {T, d, q}});
+  }
   size_t m = 0;
   for (const S3& x : v) m = std::max(m, splitk_scratch_bytes(x.M, x.N, x.K));
   return m;
@@ -102,10 +112,24 @@ EpiLinearArgs with_sk(EpiLinearArgs e, float* sk, size_t skb) {
   return e;
 }
 
+// W_qa [d + nh, d] copied into a [ldq, d] buffer whose extra rows are zero,
+// so the token-query GEMM writes whole 64-column groups and its transpose
+// reads only zeros past the gate rows.
+cudaError_t pad_qa(const void* W_qa, bf16* dst, const Dims& g, cudaStream_t cs) {
+  const size_t live = (size_t)(g.d + g.nh) * g.d;
+  cudaError_t e = cudaMemcpyAsync(dst, W_qa, live * sizeof(bf16), cudaMemcpyDeviceToDevice, cs);
+  if (e != cudaSuccess) return e;
+  return cudaMemsetAsync(dst + live, 0, ((size_t)g.ldq * g.d - live) * sizeof(bf16), cs);
+}
+
 // Buffers the forward saves for the backward pass (order fixes the layout).
 struct Saved {
   bf16 *Hb, *QKV, *Aatt, *Hbar, *Y, *Z, *D;
   float* LSE;
+  // cross injection: [Q | gate] of the tokens, proxy K | V, attention output
+  // ungated and gated, its LSE
+  bf16 *QA, *KVx, *Ax, *Ag;
+  float* LSEx;
 };
 
 Saved carve_saved(Carve& c, const pf_layer_desc& s, const Dims& g) {
@@ -115,10 +139,16 @@ Saved carve_saved(Carve& c, const pf_layer_desc& s, const Dims& g) {
   v.Aatt = c.take<bf16>(g.R * g.d);
   v.Hbar = c.take<bf16>(g.R * g.d);
   v.LSE = c.take<float>(g.B * g.nh * g.m);
-  if (s.levels == 2) {
-    v.Y = c.take<bf16>(g.rows1 * g.d);
-    v.Z = c.take<bf16>(g.R * g.k2 * g.d);
+  if (s.levels == 2) v.Y = c.take<bf16>(g.rows1 * g.d);
+  if (g.cross) {
+    v.QA = c.take<bf16>(g.T * g.ldq);
+    v.KVx = c.take<bf16>(g.R * 2 * g.d);
+    v.Ax = c.take<bf16>(g.T * g.d);
+    v.Ag = c.take<bf16>(g.T * g.d);
+    v.LSEx = c.take<float>(g.B * g.nh * g.L);
+    return v;
   }
+  if (s.levels == 2) v.Z = c.take<bf16>(g.R * g.k2 * g.d);
   v.D = c.take<bf16>(g.rows1 * g.N1);
   return v;
 }
@@ -129,6 +159,7 @@ struct FwdWs {
   bf16* Xpad;
   float* sk;
   size_t skb;
+  bf16* Wqa;  // cross: W_qa zero-padded to [d + 64, d]
   Saved sv;
 };
 
@@ -137,6 +168,7 @@ FwdWs carve_fwd(Carve& wc, const pf_layer_desc& s, const Dims& g, void* saved) {
   f.Xpad = g.ragged ? wc.take<bf16>(g.B * g.Lp * g.d) : nullptr;
   f.skb = splitk_need(s, g, false);
   f.sk = wc.take<float>(f.skb / sizeof(float));
+  if (g.cross) f.Wqa = wc.take<bf16>(g.ldq * g.d);
   Carve sc(saved);
   f.sv = saved ? carve_saved(sc, s, g) : carve_saved(wc, s, g);
   return f;
@@ -147,14 +179,31 @@ struct BwdWs {
   float *Di, *dHf, *part, *sk;
   long part_elems;
   size_t skb;
+  // cross injection: padded W_qa, dL/d(alpha A), dL/dA, [dQ | d gate | 0],
+  // proxy dK | dV, gate pre-activation gradient (fp32), Di of the tokens
+  bf16 *Wqa, *dAg, *dOx, *dQA, *dKVx;
+  float *ga, *gsum, *Dix;  // ga: [T, ldga], columns past n_heads zero
+  int ldga;
 };
 
 BwdWs carve_bwd(Carve& c, const pf_layer_desc& s, const Dims& g) {
   BwdWs w{};
   w.Xpad = g.ragged ? c.take<bf16>(g.B * g.Lp * g.d) : nullptr;
   w.dXpad = g.ragged ? c.take<bf16>(g.B * g.Lp * g.d) : nullptr;
-  w.dD = c.take<bf16>(g.rows1 * g.N1);
-  if (s.levels == 2) w.dZ = c.take<bf16>(g.R * g.k2 * g.d);
+  if (g.cross) {
+    w.Wqa = c.take<bf16>(g.ldq * g.d);
+    w.dAg = c.take<bf16>(g.T * g.d);
+    w.dOx = c.take<bf16>(g.T * g.d);
+    w.dQA = c.take<bf16>(g.T * g.ldq);
+    w.dKVx = c.take<bf16>(g.R * 2 * g.d);
+    w.ldga = (int)((g.nh + 7) & ~7L);  // whole 8-column groups for the column sum
+    w.ga = c.take<float>(g.T * w.ldga);
+    w.gsum = c.take<float>(w.ldga);
+    w.Dix = c.take<float>(g.B * g.nh * g.L);
+  } else {
+    w.dD = c.take<bf16>(g.rows1 * g.N1);
+    if (s.levels == 2) w.dZ = c.take<bf16>(g.R * g.k2 * g.d);
+  }
   w.dHbar = c.take<bf16>(g.R * g.d);
   w.dA = c.take<bf16>(g.R * g.d);
   w.dQKV = c.take<bf16>(g.R * 3 * g.d);
@@ -166,6 +215,7 @@ BwdWs carve_bwd(Carve& c, const pf_layer_desc& s, const Dims& g) {
   pe = std::max(pe, colsum_part_elems(g.R, (int)(g.k2 * g.d)));
   pe = std::max(pe, colsum_part_elems(g.R, (int)g.d));
   pe = std::max(pe, colsum_part_elems(g.rows1, (int)g.d));
+  if (g.cross) pe = std::max(pe, colsum_part_elems(g.T, (int)((g.nh + 7) & ~7L)));
   w.part_elems = pe;
   w.part = c.take<float>(pe);
   w.skb = splitk_need(s, g, true);
@@ -261,8 +311,9 @@ F32Ws carve_f32(Carve& c, const pf_layer_desc& s, const Dims& g) {
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
 bool params_aligned(const pf_layer_params& p) {
-  const void* ptrs[] = {p.W_c1, p.b_c1, p.W_c2, p.b_c2, p.W_qkv, p.W_o,  p.W_d2,  p.b_d2, p.W_d1,
-                        p.b_d1, p.w_x,  p.w_dlt, p.b_g, p.W_t1,  p.b_t1, p.W_t2, p.b_t2};
+  const void* ptrs[] = {p.W_c1, p.b_c1, p.W_c2,  p.b_c2, p.W_qkv, p.W_o,  p.W_d2,  p.b_d2,
+                        p.W_d1, p.b_d1, p.w_x,   p.w_dlt, p.b_g,  p.W_t1, p.b_t1, p.W_t2,
+                        p.b_t2, p.W_qa, p.b_a,   p.W_kvx, p.W_ox};
   for (const void* q : ptrs)
     if (!aligned16(q)) return false;
   return true;
@@ -280,7 +331,7 @@ pf_status check_desc(const pf_layer_desc* s) {
   if (s->levels == 2 && (s->k1 < 1 || s->k2 < 1 || (long)s->k1 * s->k2 != s->P))
     return fail(PF_ERR_INVALID_ARG, "levels == 2 needs k1 * k2 == P");
   if (s->mode < PF_CAUSAL_1D || s->mode > PF_BIDIR_2D) return fail(PF_ERR_INVALID_ARG, "bad mode");
-  if (s->inject < PF_INJ_ADD || s->inject > PF_INJ_AFFINE)
+  if (s->inject < PF_INJ_ADD || s->inject > PF_INJ_CROSS)
     return fail(PF_ERR_INVALID_ARG, "bad inject");
   if (s->dtype != PF_F32 && s->dtype != PF_BF16) return fail(PF_ERR_INVALID_ARG, "bad dtype");
   if (s->mode == PF_BIDIR_2D) {
@@ -293,6 +344,10 @@ pf_status check_desc(const pf_layer_desc* s) {
     return PF_OK;
   }
   if (s->inject == PF_INJ_AFFINE) return fail(PF_ERR_UNSUPPORTED, "affine injection is 2D only");
+  if (s->inject == PF_INJ_CROSS && (s->dtype != PF_BF16 || s->n_heads > 64))
+    return fail(PF_ERR_UNSUPPORTED, "cross-attention injection is built for bf16, <= 64 heads");
+  if (s->inject == PF_INJ_CROSS && (long)s->batch * s->L > (1L << 30))
+    return fail(PF_ERR_UNSUPPORTED, "problem too large for 32-bit GEMM extents");
 
   const long m = (s->L + (long)s->P - 1) / s->P;
   const long k1 = s->levels == 2 ? s->k1 : s->P, k2 = s->levels == 2 ? s->k2 : 1;
@@ -557,9 +612,12 @@ pf_status proxy_layer_fwd(const pf_layer_desc* desc, const pf_layer_params* prm,
   const Dims g = dims_of(s);
   if (prm == nullptr || X == nullptr || X_out == nullptr || X == X_out)
     return fail(PF_ERR_INVALID_ARG, "params, X and X_out are required and must not alias");
-  if (!prm->W_c1 || !prm->b_c1 || !prm->W_qkv || !prm->W_o || !prm->W_d1 || !prm->b_d1 ||
-      (s.levels == 2 && (!prm->W_c2 || !prm->b_c2 || !prm->W_d2 || !prm->b_d2)) ||
-      (s.inject == PF_INJ_GATED && (!prm->w_x || !prm->w_dlt || !prm->b_g)))
+  const bool cross = s.inject == PF_INJ_CROSS;
+  if (!prm->W_c1 || !prm->b_c1 || !prm->W_qkv || !prm->W_o ||
+      (!cross && (!prm->W_d1 || !prm->b_d1)) || (s.levels == 2 && (!prm->W_c2 || !prm->b_c2)) ||
+      (s.levels == 2 && !cross && (!prm->W_d2 || !prm->b_d2)) ||
+      (s.inject == PF_INJ_GATED && (!prm->w_x || !prm->w_dlt || !prm->b_g)) ||
+      (cross && (!prm->W_qa || !prm->b_a || !prm->W_kvx || !prm->W_ox)))
     return fail(PF_ERR_INVALID_ARG, "a parameter this layer uses is NULL");
   if (!aligned16(X) || !aligned16(X_out) || !aligned16(saved) || !aligned16(ws) ||
       !aligned16(H_in) || !aligned16(H_out) || !params_aligned(*prm))
@@ -638,6 +696,39 @@ pf_status proxy_layer_fwd(const pf_layer_desc* desc, const pf_layer_params* prm,
     set_gemm_tag("proxy_o", (double)g.R * d * 2.0);
     PF_CUDA(gemm_linear((int)g.R, d, d, {sv.Aatt, d, 0}, {static_cast<const bf16*>(prm->W_o), d, 0}, with_sk(eo, sk, skb), cs));
   }
+  if (g.cross) {
+    // a5 + a6 as gated cross-attention (Eq. inj-cross with the gate of Eq.
+    // llm-gate): [Q | gate] of the tokens, the proxies' keys and values, the
+    // attention with its per-head gate, and the output projection plus X
+    PF_CUDA(pad_qa(prm->W_qa, fw.Wqa, g, cs));
+    {
+      EpiLinearArgs e;
+      e.out_bf16 = sv.QA;
+      e.ld_bf16 = g.ldq;
+      set_gemm_tag("cross_qa", (double)g.T * (d + g.ldq) * 2.0);
+      PF_CUDA(gemm_linear((int)g.T, (int)g.ldq, d, {Xb, d, 0}, {fw.Wqa, d, 0}, with_sk(e, sk, skb), cs));
+    }
+    {
+      EpiLinearArgs e;
+      e.out_bf16 = sv.KVx;
+      e.ld_bf16 = 2 * d;
+      set_gemm_tag("cross_kv", (double)g.R * 3 * d * 2.0);
+      PF_CUDA(gemm_linear((int)g.R, 2 * d, d, {sv.Hbar, d, 0},
+                          {static_cast<const bf16*>(prm->W_kvx), d, 0}, with_sk(e, sk, skb), cs));
+    }
+    PF_CUDA(attn_cross_fwd(sv.QA, g.ldq, sv.KVx, prm->b_a, saved ? sv.Ax : nullptr, sv.Ag,
+                           sv.LSEx, (int)g.B, (int)g.L, (int)g.m, d, (int)g.nh, (int)g.P,
+                           g.causal, cs));
+    EpiLinearArgs e;
+    e.add_bf16 = Xb;
+    e.ld_add_bf16 = d;
+    e.out_bf16 = Xo;
+    e.ld_bf16 = d;
+    set_gemm_tag("cross_out", (double)g.T * d * 6.0);
+    PF_CUDA(gemm_linear((int)g.T, d, d, {sv.Ag, d, 0}, {static_cast<const bf16*>(prm->W_ox), d, 0},
+                        with_sk(e, sk, skb), cs));
+    return PF_OK;
+  }
   // a5 + a6: decompression (Eq. decompress-linear / factor-dec), routing and
   // injection (Eq. inj-gate / inj-add), fused into the last level's GEMM
   const bf16* Zsrc = sv.Hbar;
@@ -684,8 +775,10 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
     return layer_bwd_2d(s, g, *prm, X, saved, dX_out, dH_out, dX, dH_in, *grads, ws, ws_bytes,
                         static_cast<cudaStream_t>(stream));
   const bool gated = s.inject == PF_INJ_GATED;
-  if (!grads->b_d1 || (gated && (!grads->w_x || !grads->w_dlt || !grads->b_g)))
-    return fail(PF_ERR_INVALID_ARG, "grads->b_d1 (and the gate gradients) must be given");
+  if (g.cross ? (!prm->W_qa || !prm->b_a || !prm->W_kvx || !prm->W_ox)
+              : (!grads->b_d1 || (gated && (!grads->w_x || !grads->w_dlt || !grads->b_g))))
+    return fail(PF_ERR_INVALID_ARG, g.cross ? "a cross-injection parameter is NULL"
+                                            : "grads->b_d1 (and the gate gradients) must be given");
   Carve wc(ws);
   BwdWs w = carve_bwd(wc, s, g);
   if (ws == nullptr || wc.off > ws_bytes)
@@ -712,50 +805,121 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
   // direct injection gradient: written into dX, or into a block-padded buffer
   // when L % P != 0 so the dX GEMM epilogue can prefetch it as whole tiles
   bf16* dXd = g.ragged ? w.dXpad : dXb;
-  // injection backward: dD (proxy order), direct dX, gate and b_d1 gradients
-  {
-    const int nch = inj_bwd_chunks(g.rows1, N1);
-    InjBwdArgs a{G, Xb, sv.D, w.dD, dXd, g.ragged ? g.Lp : g.L, prm->w_x, prm->w_dlt, prm->b_g,
-                 d, (int)g.k1, (int)g.k2, (int)g.m, (int)g.L, (int)g.B, g.causal ? 1 : 0,
-                 gated ? 1 : 0};
-    PF_CUDA(inj_bwd_1d(a, w.part, nch, cs));
-    if (g.causal)
-      PF_CUDA(copy_block0(G, g.L, dXd, g.ragged ? g.Lp : g.L, (int)g.B, d,
-                          (int)std::min(g.P, g.L), cs));
-    PF_CUDA(inj_bwd_finalize(w.part, nch, N1, d, grads->b_d1, gated ? grads->w_x : nullptr,
-                             gated ? grads->w_dlt : nullptr, gated ? grads->b_g : nullptr, cs));
-  }
-  // decompression level 1 (or single level)
-  const bf16* Zsrc = s.levels == 2 ? sv.Z : sv.Hbar;
-  if (grads->W_d1) {
-    EpiLinearArgs e;
-    e.out_f32 = grads->W_d1;
-    e.ld_f32 = d;
-    set_gemm_tag("bwd_dW_d1", (double)N1 * d * 4.0);
-    PF_CUDA(gemm_linear(N1, d, (int)g.rows1, {w.dD, N1, 1}, {Zsrc, d, 1}, with_sk(e, w.sk, w.skb), cs));
-  }
-  {
-    EpiLinearArgs e;
-    e.out_bf16 = s.levels == 2 ? w.dZ : w.dHbar;
-    e.ld_bf16 = d;
-    set_gemm_tag("bwd_dZ", (double)g.rows1 * d * 2.0);
-    PF_CUDA(gemm_linear((int)g.rows1, d, N1, {w.dD, N1, 0}, {W_d1, d, 1}, with_sk(e, w.sk, w.skb), cs));
-  }
-  if (s.levels == 2) {
-    const int n2 = (int)(g.k2 * d);
-    if (grads->b_d2) PF_CUDA(colsum_bf16(w.dZ, g.R, n2, grads->b_d2, w.part, cs));
-    if (grads->W_d2) {
+  if (g.cross) {
+    // the gated cross injection backward: output projection, gate, the
+    // cross-attention (dQ of the tokens, dK / dV of the proxies), then the
+    // direct dX = dX_out + [dQ | d gate] W_qa and dHbar = [dK | dV] W_kvx
+    const bf16* W_ox = static_cast<const bf16*>(prm->W_ox);
+    const bf16* W_kvx = static_cast<const bf16*>(prm->W_kvx);
+    const int T = (int)g.T, q = (int)g.ldq;
+    PF_CUDA(pad_qa(prm->W_qa, w.Wqa, g, cs));
+    if (grads->W_ox) {
       EpiLinearArgs e;
-      e.out_f32 = grads->W_d2;
+      e.out_f32 = grads->W_ox;
       e.ld_f32 = d;
-      set_gemm_tag("bwd_dW_d2", (double)n2 * d * 4.0);
-      PF_CUDA(gemm_linear(n2, d, (int)g.R, {w.dZ, n2, 1}, {sv.Hbar, d, 1}, with_sk(e, w.sk, w.skb), cs));
+      set_gemm_tag("bwd_dW_ox", (double)d * d * 4.0);
+      PF_CUDA(gemm_linear(d, d, T, {G, d, 1}, {sv.Ag, d, 1}, with_sk(e, w.sk, w.skb), cs));
     }
-    EpiLinearArgs e;
-    e.out_bf16 = w.dHbar;
-    e.ld_bf16 = d;
-    set_gemm_tag("bwd_dHbar", (double)g.R * d * 2.0);
-    PF_CUDA(gemm_linear((int)g.R, d, n2, {w.dZ, n2, 0}, {W_d2, d, 1}, with_sk(e, w.sk, w.skb), cs));
+    {
+      EpiLinearArgs e;
+      e.out_bf16 = w.dAg;
+      e.ld_bf16 = d;
+      set_gemm_tag("bwd_dAg", (double)T * d * 4.0);
+      PF_CUDA(gemm_linear(T, d, d, {G, d, 0}, {W_ox, d, 1}, with_sk(e, w.sk, w.skb), cs));
+    }
+    PF_CUDA(cross_gate_bwd(w.dAg, sv.Ax, sv.QA, g.ldq, prm->b_a, w.dOx, w.Dix, w.dQA, w.ga,
+                           w.ldga, (int)g.B, (int)g.L, d, (int)g.nh, cs));
+    if (grads->b_a) {
+      PF_CUDA(colsum_f32(w.ga, g.T, w.ldga, w.gsum, w.part, cs));
+      PF_CUDA(cudaMemcpyAsync(grads->b_a, w.gsum, g.nh * sizeof(float), cudaMemcpyDeviceToDevice,
+                              cs));
+    }
+    PF_CUDA(attn_cross_bwd(sv.QA, g.ldq, sv.KVx, w.dOx, sv.LSEx, w.Dix, w.dQA, w.dKVx, (int)g.B,
+                           (int)g.L, (int)g.m, d, (int)g.nh, (int)g.P, g.causal, cs));
+    if (grads->W_qa) {
+      EpiLinearArgs e;
+      e.out_f32 = grads->W_qa;
+      e.ld_f32 = d;
+      set_gemm_tag("bwd_dW_qa", (double)(d + g.nh) * d * 4.0);
+      PF_CUDA(gemm_linear(d + (int)g.nh, d, T, {w.dQA, g.ldq, 1}, {Xb, d, 1},
+                          with_sk(e, w.sk, w.skb), cs));
+    }
+    if (grads->W_kvx) {
+      EpiLinearArgs e;
+      e.out_f32 = grads->W_kvx;
+      e.ld_f32 = d;
+      set_gemm_tag("bwd_dW_kvx", (double)2 * d * d * 4.0);
+      PF_CUDA(gemm_linear(2 * d, d, (int)g.R, {w.dKVx, 2 * d, 1}, {sv.Hbar, d, 1},
+                          with_sk(e, w.sk, w.skb), cs));
+    }
+    {
+      EpiLinearArgs e;
+      e.out_bf16 = w.dHbar;
+      e.ld_bf16 = d;
+      set_gemm_tag("bwd_dHbar", (double)g.R * 3 * d * 2.0);
+      PF_CUDA(gemm_linear((int)g.R, d, 2 * d, {w.dKVx, 2 * d, 0}, {W_kvx, d, 1},
+                          with_sk(e, w.sk, w.skb), cs));
+    }
+    // direct dX, in the block-padded layout when L % P != 0 (per sequence
+    // then, as the rows of different sequences are spaced differently)
+    const bool per_seq = g.ragged && g.B > 1;
+    for (long b = 0; b < (per_seq ? g.B : 1); ++b) {
+      EpiLinearArgs e;
+      e.add_bf16 = G + b * g.L * d;
+      e.ld_add_bf16 = d;
+      e.out_bf16 = dXd + b * (g.ragged ? g.Lp : g.L) * d;
+      e.ld_bf16 = d;
+      const int rows = per_seq ? (int)g.L : T;
+      set_gemm_tag("bwd_dX_direct", (double)rows * (q + 2 * d) * 2.0);
+      PF_CUDA(gemm_linear(rows, d, q, {w.dQA + b * g.L * q, q, 0}, {w.Wqa, d, 1},
+                          with_sk(e, w.sk, w.skb), cs));
+    }
+  } else {
+    // injection backward: dD (proxy order), direct dX, gate and b_d1 gradients
+    {
+      const int nch = inj_bwd_chunks(g.rows1, N1);
+      InjBwdArgs a{G, Xb, sv.D, w.dD, dXd, g.ragged ? g.Lp : g.L, prm->w_x, prm->w_dlt, prm->b_g,
+                   d, (int)g.k1, (int)g.k2, (int)g.m, (int)g.L, (int)g.B, g.causal ? 1 : 0,
+                   gated ? 1 : 0};
+      PF_CUDA(inj_bwd_1d(a, w.part, nch, cs));
+      if (g.causal)
+        PF_CUDA(copy_block0(G, g.L, dXd, g.ragged ? g.Lp : g.L, (int)g.B, d,
+                            (int)std::min(g.P, g.L), cs));
+      PF_CUDA(inj_bwd_finalize(w.part, nch, N1, d, grads->b_d1, gated ? grads->w_x : nullptr,
+                               gated ? grads->w_dlt : nullptr, gated ? grads->b_g : nullptr, cs));
+    }
+    // decompression level 1 (or single level)
+    const bf16* Zsrc = s.levels == 2 ? sv.Z : sv.Hbar;
+    if (grads->W_d1) {
+      EpiLinearArgs e;
+      e.out_f32 = grads->W_d1;
+      e.ld_f32 = d;
+      set_gemm_tag("bwd_dW_d1", (double)N1 * d * 4.0);
+      PF_CUDA(gemm_linear(N1, d, (int)g.rows1, {w.dD, N1, 1}, {Zsrc, d, 1}, with_sk(e, w.sk, w.skb), cs));
+    }
+    {
+      EpiLinearArgs e;
+      e.out_bf16 = s.levels == 2 ? w.dZ : w.dHbar;
+      e.ld_bf16 = d;
+      set_gemm_tag("bwd_dZ", (double)g.rows1 * d * 2.0);
+      PF_CUDA(gemm_linear((int)g.rows1, d, N1, {w.dD, N1, 0}, {W_d1, d, 1}, with_sk(e, w.sk, w.skb), cs));
+    }
+    if (s.levels == 2) {
+      const int n2 = (int)(g.k2 * d);
+      if (grads->b_d2) PF_CUDA(colsum_bf16(w.dZ, g.R, n2, grads->b_d2, w.part, cs));
+      if (grads->W_d2) {
+        EpiLinearArgs e;
+        e.out_f32 = grads->W_d2;
+        e.ld_f32 = d;
+        set_gemm_tag("bwd_dW_d2", (double)n2 * d * 4.0);
+        PF_CUDA(gemm_linear(n2, d, (int)g.R, {w.dZ, n2, 1}, {sv.Hbar, d, 1}, with_sk(e, w.sk, w.skb), cs));
+      }
+      EpiLinearArgs e;
+      e.out_bf16 = w.dHbar;
+      e.ld_bf16 = d;
+      set_gemm_tag("bwd_dHbar", (double)g.R * d * 2.0);
+      PF_CUDA(gemm_linear((int)g.R, d, n2, {w.dZ, n2, 0}, {W_d2, d, 1}, with_sk(e, w.sk, w.skb), cs));
+    }
   }
   // attention output projection and attention
   if (grads->W_o) {

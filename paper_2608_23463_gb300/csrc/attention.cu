@@ -34,7 +34,54 @@ __global__ void attn_bwd_dot_kernel(const bf16* __restrict__ dO, const bf16* __r
   }
 }
 
+// Gate of the cross injection, backward: one warp per (token row, head),
+// each lane two of the head's 64 columns.
+__global__ void cross_gate_bwd_kernel(const bf16* __restrict__ dAg, const bf16* __restrict__ A,
+                                      const bf16* __restrict__ qa, long ldq,
+                                      const float* __restrict__ b_a, bf16* __restrict__ dO,
+                                      float* __restrict__ Di, bf16* __restrict__ dqa,
+                                      float* __restrict__ ga, int ldga, long rows, int L, int d,
+                                      int nh) {
+  const long wid = ((long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (wid >= rows * nh) return;
+  const long row = wid / nh;
+  const int h = (int)(wid % nh);
+  const long off = row * d + h * AT + lane * 2;
+  const float2 g = unpack_bf16(*reinterpret_cast<const uint32_t*>(dAg + off));
+  const float2 a = unpack_bf16(*reinterpret_cast<const uint32_t*>(A + off));
+  float sum = g.x * a.x + g.y * a.y;
+#pragma unroll
+  for (int s = 16; s > 0; s >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, s);
+  const float x = __bfloat162float(qa[row * ldq + d + h]) + b_a[h];
+  const float al = 1.f / (1.f + __expf(-x));
+  *reinterpret_cast<uint32_t*>(dO + off) = pack_bf16(al * g.x, al * g.y);
+  if (lane == 0) {
+    const long b = row / L, t = row % L;
+    Di[(b * nh + h) * L + t] = al * sum;
+    const float gp = sum * al * (1.f - al);
+    dqa[row * ldq + d + h] = __float2bfloat16(gp);
+    ga[row * ldga + h] = gp;
+  }
+  if (h == 0) {  // the padding columns past the gate rows stay zero
+    for (long c = d + nh + lane; c < ldq; c += 32) dqa[row * ldq + c] = __float2bfloat16(0.f);
+    for (int c = nh + lane; c < ldga; c += 32) ga[row * ldga + c] = 0.f;
+  }
+}
+
 }  // namespace
+
+cudaError_t cross_gate_bwd(const bf16* dAg, const bf16* A, const bf16* qa, long ldq,
+                           const float* b_a, bf16* dO, float* Di, bf16* dqa, float* ga, int ldga,
+                           int B, int L, int d, int nh, cudaStream_t st) {
+  if (d != nh * AT || ldq < d + nh || ldga < nh) return cudaErrorInvalidValue;
+  const long rows = (long)B * L, warps = rows * nh;
+  LaunchTimer lt("cross_gate_bwd", st, 4.0 * rows * d,
+                 6.0 * rows * d + 2.0 * rows * ldq / 8.0 + 8.0 * rows * nh);
+  cross_gate_bwd_kernel<<<(unsigned)((warps * 32 + 255) / 256), 256, 0, st>>>(
+      dAg, A, qa, ldq, b_a, dO, Di, dqa, ga, ldga, rows, L, d, nh);
+  return cudaGetLastError();
+}
 
 int take_dev_error_attention() { return take_dev_error_tu(); }
 

@@ -19,6 +19,12 @@
 // accumulating MMAs, so those read only their B tile from shared memory
 // (shared-memory bandwidth, not the tensor pipe, bounds M=128 N=64 MMAs whose
 // operands both come from shared memory).  Every wait is bounded.
+//
+// The cross-attention of the injection (Eq. inj-cross) runs on the same
+// kernels: queries are tokens, keys / values proxies (separate matrices, Lq
+// and Lk rows per sequence), and token q sees proxies j < q / P (causal) or
+// all.  Stationary tiles that no pair reaches are not work items; the host
+// zero-fills their output rows.
 #include <algorithm>
 #include <type_traits>
 
@@ -47,12 +53,28 @@ constexpr uint32_t BW_TMEM_COLS = 512;
 constexpr uint32_t BW_TM_E = 384;
 
 struct BwArgs {
-  bf16* dqkv;         // [B*m, 3d]
-  const float* lse;   // [B, nh, m], log2 units
-  const float* Di;    // [B, nh, m]
-  int B, m, d, nh, causal, n_tiles, n_steps_total, n_items;
+  // outputs, head h of stationary row (b, r) at out + (b*Lx + r)*ld + col + 64h:
+  // DKDV u = dV, w = dK; DQ u = dQ
+  bf16 *out_u, *out_w;
+  long ld_u, ld_w;
+  int col_u, col_w;
+  const float* lse;   // [B, nh, Lq], log2 units
+  const float* Di;    // [B, nh, Lq]
+  int B, Lq, Lk, d, nh, causal, P;  // P > 0: cross-attention with block size P
+  int Lx, Ly;         // stationary / streamed rows per sequence
+  int n_tiles, n_steps_total, n_items;
   float sl2, scale;
 };
+
+// Keys visible to query q (all, causal prefix, or the proxies of earlier
+// blocks), and the first query that sees key k.
+__host__ __device__ __forceinline__ int bw_vis(const BwArgs& a, int q) {
+  const int v = !a.causal ? a.Lk : a.P ? q / a.P : q + 1;
+  return v < a.Lk ? v : a.Lk;
+}
+__host__ __device__ __forceinline__ int bw_first_q(const BwArgs& a, int k) {
+  return !a.causal ? 0 : a.P ? (k + 1) * a.P : k;
+}
 
 __device__ __forceinline__ float ex2_approx(float x) {
   float y;
@@ -81,8 +103,9 @@ __device__ __forceinline__ int bw_rank(int c, int round) {
 }
 
 // Item k -> stationary tile t (128 rows), head, sequence, first streamed tile
-// j0 and step count n.  DKDV: keys of tile t see queries >= key (causal), so
-// the heaviest items have the smallest t; DQ: the largest t.
+// j0 and step count n.  DKDV: the keys of tile t are seen by the queries from
+// bw_first_q on, so the heaviest items have the smallest t; DQ: the largest t.
+// The host sizes n_items so that every item has n >= 1.
 template <bool DKDV>
 __device__ __forceinline__ void bw_item(const BwArgs& a, int k, int& t, int& h, int& b, int& j0,
                                         int& n) {
@@ -92,12 +115,12 @@ __device__ __forceinline__ void bw_item(const BwArgs& a, int k, int& t, int& h, 
   b = r / a.nh;
   if (DKDV) {
     t = rnk;
-    j0 = a.causal ? 2 * t : 0;
+    j0 = bw_first_q(a, t * BW_M) / BW_N;
     n = a.n_steps_total - j0;
   } else {
     t = a.n_tiles - 1 - rnk;
     j0 = 0;
-    n = a.causal ? min(2 * t + 2, a.n_steps_total) : a.n_steps_total;
+    n = min((bw_vis(a, min(t * BW_M + BW_M - 1, a.Lq - 1)) + BW_N - 1) / BW_N, a.n_steps_total);
   }
 }
 
@@ -160,7 +183,7 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
          k = bw_rank(blockIdx.x, ++rd), ++it) {
       int t, h, b, j0, n;
       bw_item<DKDV>(a, k, t, h, b, j0, n);
-      const int row0 = b * a.m;
+      const int row0 = b * a.Lx;
       const uint32_t xb = it & 1;
       if (!mbar_wait(x_empty + 8 * xb, ((it >> 1) & 1) ^ 1)) break;
       const uint32_t xdst = sbase + xb * 2 * BW_X_BYTES;
@@ -175,7 +198,7 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
           break;
         }
         const uint32_t ydst = sbase + BW_OFF_Y + st * 2 * BW_Y_BYTES;
-        const int yrow = row0 + (j0 + j) * BW_N;
+        const int yrow = b * a.Ly + (j0 + j) * BW_N;
         mbar_arrive_expect_tx(y_full + 8 * st, 2 * BW_Y_BYTES);
         tma_load_2d(ydst, &tmY1, y_full + 8 * st, y1c + h * BW_D, yrow);
         tma_load_2d(ydst + BW_Y_BYTES, &tmY2, y_full + 8 * st, y2c + h * BW_D, yrow);
@@ -271,8 +294,8 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
     // fetches column tr of the next step
     auto fetch_ld = [&](int b, int h, int q0, int c) -> float2 {
       const int qq = q0 + c;
-      if (c >= BW_N || qq >= a.m) return make_float2(0.f, 0.f);
-      const long o = ((long)b * a.nh + h) * a.m + qq;
+      if (c >= BW_N || qq >= a.Lq) return make_float2(0.f, 0.f);
+      const long o = ((long)b * a.nh + h) * a.Lq + qq;
       return make_float2(a.lse[o], a.Di[o]);
     };
     int rd = 0;
@@ -288,8 +311,8 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
       bw_item<DKDV>(a, k, t, h, b, j0, n);
       const int row = t * BW_M + r;  // key (DKDV) or query (DQ) index in the sequence
       float lse_r = 0.f, di_r = 0.f;
-      if (!DKDV && row < a.m) {
-        const long o = ((long)b * a.nh + h) * a.m + row;
+      if (!DKDV && row < a.Lq) {
+        const long o = ((long)b * a.nh + h) * a.Lq + row;
         lse_r = a.lse[o];
         di_r = a.Di[o];
       }
@@ -330,13 +353,11 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
         tc_fence_before();
         mbar_arrive(t_free + 8 * tb);
         // valid streamed columns: [lo, hi)
-        int lo = 0, hi = min(BW_N, a.m - c0);
-        if (a.causal) {
-          if (DKDV)
-            lo = max(0, row - c0);  // queries >= key
-          else
-            hi = min(hi, row - c0 + 1);  // keys <= query
-        }
+        int lo = 0, hi = min(BW_N, a.Ly - c0);
+        if (DKDV)
+          lo = max(0, bw_first_q(a, row) - c0);  // the queries that see this key
+        else
+          hi = min(hi, bw_vis(a, row) - c0);  // the keys this query sees
         if (!mbar_wait(e_free + 8 * tb, ((Gj >> 1) & 1) ^ 1)) {
           ok = false;
           if (DKDV) continue;
@@ -409,10 +430,9 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
       if (DKDV) tmem_wait_ld(w0);
       tc_fence_before();
       mbar_arrive(acc_free);
-      if (row < a.m) {
-        bf16* base = a.dqkv + ((long)b * a.m + row) * 3 * a.d + h * BW_D + 32 * ch;
-        // DKDV: u = dV (column block 2d), w = dK (column block d); DQ: u = dQ
-        bf16* pu = base + (DKDV ? 2 * a.d : 0);
+      if (row < a.Lx) {
+        const long srow = (long)b * a.Lx + row;
+        bf16* pu = a.out_u + srow * a.ld_u + a.col_u + h * BW_D + 32 * ch;
         const float su = DKDV ? 1.f : a.scale;
 #pragma unroll
         for (int i = 0; i < 32; i += 8)
@@ -422,7 +442,7 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
               pack_bf16(__uint_as_float(u0[i + 4]) * su, __uint_as_float(u0[i + 5]) * su),
               pack_bf16(__uint_as_float(u0[i + 6]) * su, __uint_as_float(u0[i + 7]) * su));
         if (DKDV) {
-          bf16* pw = base + a.d;
+          bf16* pw = a.out_w + srow * a.ld_w + a.col_w + h * BW_D + 32 * ch;
 #pragma unroll
           for (int i = 0; i < 32; i += 8)
             *reinterpret_cast<uint4*>(pw + i) = make_uint4(
@@ -458,6 +478,53 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
 
 int take_dev_error_attention_bwd_tc() { return take_dev_error_tu(); }
 
+namespace {
+
+// zero rows [r0, r1) of every sequence in a [B*Lx, ld] matrix, columns [col, col + d)
+cudaError_t zero_rows(bf16* o, long ld, int col, int d, int B, int Lx, int r0, int r1,
+                      cudaStream_t st) {
+  if (r1 <= r0) return cudaSuccess;
+  for (int b = 0; b < B; ++b) {
+    const cudaError_t e = cudaMemset2DAsync(o + ((long)b * Lx + r0) * ld + col, ld * sizeof(bf16),
+                                            0, (size_t)d * sizeof(bf16), (size_t)(r1 - r0), st);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+template <bool DKDV>
+cudaError_t bw_launch(const CUtensorMap& x1, const CUtensorMap& x2, const CUtensorMap& y1,
+                      const CUtensorMap& y2, int x1c, int x2c, int y1c, int y2c, BwArgs a,
+                      const char* label, double flops, double bytes, cudaStream_t st) {
+  a.Lx = DKDV ? a.Lk : a.Lq;
+  a.Ly = DKDV ? a.Lq : a.Lk;
+  a.n_tiles = (a.Lx + BW_M - 1) / BW_M;
+  a.n_steps_total = (a.Ly + BW_N - 1) / BW_N;
+  a.scale = 1.0f / sqrtf((float)BW_D);
+  a.sl2 = a.scale * 1.4426950408889634f;
+  // stationary tiles with work: DKDV [0, hi), DQ [lo, n_tiles)
+  int lo = 0, hi = a.n_tiles;
+  if (DKDV)
+    while (hi > 0 && bw_first_q(a, (hi - 1) * BW_M) >= a.Lq) --hi;
+  else
+    while (lo < a.n_tiles && bw_vis(a, std::min(lo * BW_M + BW_M - 1, a.Lq - 1)) == 0) ++lo;
+  a.n_items = (hi - lo) * a.nh * a.B;
+  auto kern = attn_bwd_tc_kernel<DKDV>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, BW_SMEM);
+  if (e != cudaSuccess) return e;
+  LaunchTimer lt(label, st, flops, bytes);
+  const int r0 = DKDV ? std::min(hi * BW_M, a.Lx) : 0, r1 = DKDV ? a.Lx : std::min(lo * BW_M, a.Lx);
+  if ((e = zero_rows(a.out_u, a.ld_u, a.col_u, a.d, a.B, a.Lx, r0, r1, st)) != cudaSuccess) return e;
+  if (DKDV && (e = zero_rows(a.out_w, a.ld_w, a.col_w, a.d, a.B, a.Lx, r0, r1, st)) != cudaSuccess)
+    return e;
+  if (a.n_items == 0) return cudaSuccess;
+  const int grid = std::min(a.n_items, num_sms());
+  kern<<<grid, BW_THREADS, BW_SMEM, st>>>(x1, x2, y1, y2, x1c, x2c, y1c, y2c, a);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
 cudaError_t attn_bwd_tc(const bf16* qkv, const bf16* dO, const float* lse, const float* Di,
                         bf16* dqkv, int B, int m, int d, int nh, bool causal, cudaStream_t st) {
   if (d != nh * BW_D || ((uintptr_t)qkv & 15) || ((uintptr_t)dO & 15) || ((uintptr_t)dqkv & 15))
@@ -470,43 +537,80 @@ cudaError_t attn_bwd_tc(const bf16* qkv, const bf16* dO, const float* lse, const
       !tmap_bf16_2d(&do64, dO, (uint64_t)d, rows, (uint64_t)d, 64, BW_N))
     return cudaErrorInvalidValue;
   BwArgs a{};
-  a.dqkv = dqkv;
   a.lse = lse;
   a.Di = Di;
   a.B = B;
-  a.m = m;
+  a.Lq = a.Lk = m;
   a.d = d;
   a.nh = nh;
   a.causal = causal ? 1 : 0;
-  a.n_tiles = (m + BW_M - 1) / BW_M;
-  a.n_steps_total = (m + BW_N - 1) / BW_N;
-  a.n_items = a.n_tiles * nh * B;
-  a.scale = 1.0f / sqrtf((float)BW_D);
-  a.sl2 = a.scale * 1.4426950408889634f;
-  const int grid = std::min(a.n_items, num_sms());
+  a.P = 0;
+  a.out_u = a.out_w = dqkv;
+  a.ld_u = a.ld_w = 3L * d;
   const double pairs = (double)B * nh * (causal ? 0.5 * m * (m + 1.0) : (double)m * m);
   cudaError_t e;
-  {
-    auto kern = attn_bwd_tc_kernel<true>;
-    if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, BW_SMEM)) !=
-        cudaSuccess)
-      return e;
-    LaunchTimer lt("attn_bwd_dkdv", st, 8.0 * BW_D * pairs, 2.0 * B * m * (5.0 * d));
-    // X1 = K, X2 = V (128 rows); Y1 = Q, Y2 = dO (64 rows)
-    kern<<<grid, BW_THREADS, BW_SMEM, st>>>(qkv128, qkv128, qkv64, do64, d, 2 * d, 0, 0, a);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  // DKDV: X1 = K, X2 = V (128 rows); Y1 = Q, Y2 = dO (64 rows); u = dV, w = dK
+  a.col_u = 2 * d;
+  a.col_w = d;
+  if ((e = bw_launch<true>(qkv128, qkv128, qkv64, do64, d, 2 * d, 0, 0, a, "attn_bwd_dkdv",
+                           8.0 * BW_D * pairs, 2.0 * B * m * (5.0 * d), st)) != cudaSuccess)
+    return e;
+  // DQ: X1 = Q, X2 = dO (128 rows); Y1 = K, Y2 = V (64 rows); u = dQ
+  a.col_u = 0;
+  return bw_launch<false>(qkv128, do128, qkv64, qkv64, 0, 0, d, 2 * d, a, "attn_bwd_dq",
+                          6.0 * BW_D * pairs, 2.0 * B * m * (4.0 * d), st);
+}
+
+cudaError_t attn_cross_bwd(const bf16* qa, long ldq, const bf16* kv, const bf16* dO,
+                           const float* lse, const float* Di, bf16* dqa, bf16* dkv, int B, int Lq,
+                           int Lk, int d, int nh, int P, bool causal, cudaStream_t st) {
+  if (d != nh * BW_D || P < 1 || ldq < d || ((uintptr_t)qa & 15) || ((uintptr_t)kv & 15) ||
+      ((uintptr_t)dO & 15) || ((uintptr_t)dqa & 15) || ((uintptr_t)dkv & 15) || (ldq * 2) % 16)
+    return cudaErrorInvalidValue;
+  const uint64_t rq = (uint64_t)B * Lq, rk = (uint64_t)B * Lk;
+  CUtensorMap qa128, qa64, kv128, kv64, do128, do64;
+  if (!tmap_bf16_2d(&qa128, qa, (uint64_t)ldq, rq, (uint64_t)ldq, 64, BW_M) ||
+      !tmap_bf16_2d(&qa64, qa, (uint64_t)ldq, rq, (uint64_t)ldq, 64, BW_N) ||
+      !tmap_bf16_2d(&kv128, kv, 2ull * d, rk, 2ull * d, 64, BW_M) ||
+      !tmap_bf16_2d(&kv64, kv, 2ull * d, rk, 2ull * d, 64, BW_N) ||
+      !tmap_bf16_2d(&do128, dO, (uint64_t)d, rq, (uint64_t)d, 64, BW_M) ||
+      !tmap_bf16_2d(&do64, dO, (uint64_t)d, rq, (uint64_t)d, 64, BW_N))
+    return cudaErrorInvalidValue;
+  BwArgs a{};
+  a.lse = lse;
+  a.Di = Di;
+  a.B = B;
+  a.Lq = Lq;
+  a.Lk = Lk;
+  a.d = d;
+  a.nh = nh;
+  a.causal = causal ? 1 : 0;
+  a.P = P;
+  double pairs = 0.0;  // visible (token, proxy) pairs per head and sequence
+  if (!causal) {
+    pairs = (double)Lq * Lk;
+  } else {
+    for (int i = 0; (long)i * P < Lq; ++i) pairs += (double)std::min(P, Lq - i * P) * std::min(i, Lk);
   }
-  {
-    auto kern = attn_bwd_tc_kernel<false>;
-    if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, BW_SMEM)) !=
-        cudaSuccess)
-      return e;
-    LaunchTimer lt("attn_bwd_dq", st, 6.0 * BW_D * pairs, 2.0 * B * m * (4.0 * d));
-    // X1 = Q, X2 = dO (128 rows); Y1 = K, Y2 = V (64 rows)
-    kern<<<grid, BW_THREADS, BW_SMEM, st>>>(qkv128, do128, qkv64, qkv64, 0, 0, d, 2 * d, a);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  }
-  return cudaSuccess;
+  pairs *= (double)B * nh;
+  cudaError_t e;
+  // DKDV: X1 = K, X2 = V (proxies, 128 rows); Y1 = Q, Y2 = dO (tokens, 64 rows);
+  // u = dV (dkv columns [d, 2d)), w = dK (columns [0, d))
+  a.out_u = a.out_w = dkv;
+  a.ld_u = a.ld_w = 2L * d;
+  a.col_u = d;
+  a.col_w = 0;
+  if ((e = bw_launch<true>(kv128, kv128, qa64, do64, 0, d, 0, 0, a, "attn_cross_bwd_dkdv",
+                           8.0 * BW_D * pairs, 2.0 * B * (Lk * 4.0 * d + Lq * 2.0 * d), st)) !=
+      cudaSuccess)
+    return e;
+  // DQ: X1 = Q, X2 = dO (tokens, 128 rows); Y1 = K, Y2 = V (proxies, 64 rows);
+  // u = dQ (dqa columns [0, d))
+  a.out_u = dqa;
+  a.ld_u = ldq;
+  a.col_u = 0;
+  return bw_launch<false>(qa128, do128, kv64, kv64, 0, 0, 0, d, a, "attn_cross_bwd_dq",
+                          6.0 * BW_D * pairs, 2.0 * B * (Lq * 3.0 * d + Lk * 2.0 * d), st);
 }
 
 }  // namespace pf

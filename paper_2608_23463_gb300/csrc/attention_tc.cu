@@ -16,6 +16,14 @@
 //             running-max correction
 // Saved per (b, h, query): LSE = max + log2(sum) (log2 units), the input of
 // the backward.  Every mbarrier wait is bounded.
+//
+// The same kernel serves the cross-attention injection (Eq. inj-cross): the
+// queries are tokens and the keys / values proxies, from separate matrices,
+// and token q sees the proxies of earlier blocks, j < q / P (causal) or all
+// of them.  Query tiles that see no proxy are not work items (the host
+// zero-fills their rows); a row that sees none writes zeros and LSE 0.  An
+// optional second output applies the per-head gate sigmoid(a + b_a) (the
+// ungated output is optional too, for inference).
 #include <algorithm>
 
 #include "kernels.h"
@@ -40,11 +48,24 @@ constexpr uint32_t FA_SMEM = FA_OFF_BAR + 256 + 1024;
 constexpr uint32_t FA_TMEM_COLS = 512;
 
 struct FaArgs {
-  bf16* out;   // [B*m, d]
-  float* lse;  // [B, nh, m]
-  int B, m, d, nh, causal, n_qt, n_kt, n_items;
+  bf16* out;          // [B*Lq, ldo], head h at column h*64
+  bf16* out_g;        // gated copy sigmoid(gate + b_a[h]) * out, or null
+  const bf16* gpre;   // gate pre-activations: row b*Lq + q, column gcol + h
+  const float* b_a;   // [nh]
+  float* lse;         // [B, nh, Lq]
+  long ldo, ldg;
+  int gcol, qcol, kcol, vcol;  // column offsets of gate, Q, K, V in their matrices
+  int B, Lq, Lk, d, nh, causal, P;  // P > 0: cross-attention with block size P
+  int n_qt, qt_min, n_kt, n_items;
   float sl2;  // log2(e) / sqrt(64)
 };
+
+// Keys visible to query q: all, the causal prefix j <= q, or (cross) the
+// proxies of the blocks before q's.
+__host__ __device__ __forceinline__ int fa_vis(const FaArgs& a, int q) {
+  const int v = !a.causal ? a.Lk : a.P ? q / a.P : q + 1;
+  return v < a.Lk ? v : a.Lk;
+}
 
 // Items are ranked heaviest first (causal: the query tiles with the most key
 // tiles); CTA c takes rank c of round 0, rank G-1-c of round 1, and so on
@@ -59,7 +80,7 @@ __device__ __forceinline__ void fa_item(const FaArgs& a, int k, int& qt, int& h,
   const int r = k % per;
   h = r % a.nh;
   b = r / a.nh;
-  n = a.causal ? min(qt + 1, a.n_kt) : a.n_kt;
+  n = (fa_vis(a, min(qt * FA_M + FA_M - 1, a.Lq - 1)) + FA_N - 1) / FA_N;
 }
 
 // 2^x on the SFU (ex2.approx, flush-to-zero): relative error about 2^-22,
@@ -71,7 +92,8 @@ __device__ __forceinline__ float ex2_approx(float x) {
 }
 
 __global__ void __launch_bounds__(FA_THREADS, 1)
-    attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQKV, FaArgs a) {
+    attn_fwd_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
+                       const __grid_constant__ CUtensorMap tmKV, FaArgs a) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
@@ -114,18 +136,20 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
 
   if (warp == 0 && lane == 0) {
     // ------------------------------------------------------------ producer
-    prefetch_tmap(&tmQKV);
+    prefetch_tmap(&tmQ);
+    prefetch_tmap(&tmKV);
     bool ok = true;
     uint32_t it = 0;
     for (int rd = 0, k = fa_rank(blockIdx.x, 0); k < a.n_items && ok;
          k = fa_rank(blockIdx.x, ++rd), ++it) {
       int qt, h, b, n;
       fa_item(a, k, qt, h, b, n);
-      const int row0 = b * a.m;
+      const int krow0 = b * a.Lk;
       const uint32_t qb = it & 1;
       if (!mbar_wait(q_empty + 8 * qb, ((it >> 1) & 1) ^ 1)) break;
       mbar_arrive_expect_tx(q_full + 8 * qb, FA_Q_BYTES);
-      tma_load_2d(sbase + qb * FA_Q_BYTES, &tmQKV, q_full + 8 * qb, h * FA_D, row0 + qt * FA_M);
+      tma_load_2d(sbase + qb * FA_Q_BYTES, &tmQ, q_full + 8 * qb, a.qcol + h * FA_D,
+                  b * a.Lq + qt * FA_M);
       q_issued = it + 1;
       for (int j = 0; j < n; ++j) {
         const uint32_t g = kv_issued, st = g % FA_STAGES;
@@ -135,9 +159,9 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
         }
         const uint32_t kdst = sbase + FA_OFF_KV + st * 2 * FA_KV_BYTES;
         mbar_arrive_expect_tx(kv_full + 8 * st, 2 * FA_KV_BYTES);
-        tma_load_2d(kdst, &tmQKV, kv_full + 8 * st, a.d + h * FA_D, row0 + j * FA_N);
-        tma_load_2d(kdst + FA_KV_BYTES, &tmQKV, kv_full + 8 * st, 2 * a.d + h * FA_D,
-                    row0 + j * FA_N);
+        tma_load_2d(kdst, &tmKV, kv_full + 8 * st, a.kcol + h * FA_D, krow0 + j * FA_N);
+        tma_load_2d(kdst + FA_KV_BYTES, &tmKV, kv_full + 8 * st, a.vcol + h * FA_D,
+                    krow0 + j * FA_N);
         kv_issued = g + 1;
       }
     }
@@ -216,6 +240,7 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       int qt, h, b, n;
       fa_item(a, k, qt, h, b, n);
       const int q = qt * FA_M + r;  // query index in the sequence
+      const int vis = fa_vis(a, q);
       float mrun = -INFINITY, l = 0.f, corr_prev = 1.f;
       float o[FA_D];
 #pragma unroll
@@ -247,9 +272,10 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
         tc_fence_after();
         // two passes over the 128 scores, 64 TMEM columns at a time: the row
         // maximum, then the probabilities (keeps the live registers low).
-        // Keys c >= lim of this tile are masked (causal diagonal, sequence end).
+        // Keys c >= lim of this tile are masked (causal diagonal or block
+        // boundary, sequence end); lim <= 0 masks the whole tile.
         const int key0 = j * FA_N;
-        const int lim = min(FA_N, min(a.m - key0, a.causal ? q - key0 + 1 : FA_N));
+        const int lim = min(FA_N, min(a.Lk, vis) - key0);
         const uint32_t ts = tl + sb * FA_N;
         uint32_t ra[32], rb[32];
         float m8[8];
@@ -318,18 +344,31 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       }
       if (!ok || !consume_o(g + n - 1, corr_prev)) break;
       g += n;
-      if (q < a.m) {
-        const float inv = 1.f / l;
-        bf16* op = a.out + ((long)b * a.m + q) * a.d + h * FA_D;
+      if (q < a.Lq) {
+        const float inv = l > 0.f ? 1.f / l : 0.f;  // a row that sees no key: 0
+        const long row = (long)b * a.Lq + q;
+        if (a.out) {
+          bf16* op = a.out + row * a.ldo + h * FA_D;
 #pragma unroll
-        for (int i = 0; i < FA_D; i += 8) {
-          const uint4 v = make_uint4(pack_bf16(o[i] * inv, o[i + 1] * inv),
-                                     pack_bf16(o[i + 2] * inv, o[i + 3] * inv),
-                                     pack_bf16(o[i + 4] * inv, o[i + 5] * inv),
-                                     pack_bf16(o[i + 6] * inv, o[i + 7] * inv));
-          *reinterpret_cast<uint4*>(op + i) = v;
+          for (int i = 0; i < FA_D; i += 8) {
+            const uint4 v = make_uint4(pack_bf16(o[i] * inv, o[i + 1] * inv),
+                                       pack_bf16(o[i + 2] * inv, o[i + 3] * inv),
+                                       pack_bf16(o[i + 4] * inv, o[i + 5] * inv),
+                                       pack_bf16(o[i + 6] * inv, o[i + 7] * inv));
+            *reinterpret_cast<uint4*>(op + i) = v;
+          }
         }
-        a.lse[((long)b * a.nh + h) * a.m + q] = mrun + log2f(l);  // log2 units
+        if (a.out_g) {
+          const float x = __bfloat162float(a.gpre[row * a.ldg + a.gcol + h]) + a.b_a[h];
+          const float gi = inv / (1.f + __expf(-x));
+          bf16* gp = a.out_g + row * a.ldo + h * FA_D;
+#pragma unroll
+          for (int i = 0; i < FA_D; i += 8)
+            *reinterpret_cast<uint4*>(gp + i) =
+                make_uint4(pack_bf16(o[i] * gi, o[i + 1] * gi), pack_bf16(o[i + 2] * gi, o[i + 3] * gi),
+                           pack_bf16(o[i + 4] * gi, o[i + 5] * gi), pack_bf16(o[i + 6] * gi, o[i + 7] * gi));
+        }
+        a.lse[((long)b * a.nh + h) * a.Lq + q] = l > 0.f ? mrun + log2f(l) : 0.f;  // log2 units
       }
     }
   }
@@ -357,6 +396,50 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
 
 int take_dev_error_attention_tc() { return take_dev_error_tu(); }
 
+namespace {
+
+cudaError_t fa_launch(const CUtensorMap& tq, const CUtensorMap& tkv, FaArgs& a, const char* label,
+                      double pairs, double bytes, cudaStream_t st) {
+  a.n_qt = (a.Lq + FA_M - 1) / FA_M;
+  a.n_kt = (a.Lk + FA_N - 1) / FA_N;
+  a.qt_min = 0;
+  while (a.qt_min < a.n_qt && fa_vis(a, std::min(a.qt_min * FA_M + FA_M - 1, a.Lq - 1)) == 0)
+    ++a.qt_min;
+  a.n_items = (a.n_qt - a.qt_min) * a.nh * a.B;
+  a.sl2 = 1.4426950408889634f / sqrtf((float)FA_D);
+  auto kern = attn_fwd_tc_kernel;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, FA_SMEM);
+  if (e != cudaSuccess) return e;
+  LaunchTimer lt(label, st, 4.0 * FA_D * pairs, bytes);
+  if (a.qt_min > 0) {  // query tiles that see no key: zero rows, LSE 0
+    const size_t rows = (size_t)std::min(a.qt_min * FA_M, a.Lq);
+    for (int b = 0; b < a.B; ++b) {
+      bf16* dsts[2] = {a.out, a.out_g};
+      for (bf16* o : dsts)
+        if (o && (e = cudaMemset2DAsync(o + (long)b * a.Lq * a.ldo, a.ldo * sizeof(bf16), 0,
+                                        (size_t)a.d * sizeof(bf16), rows, st)) != cudaSuccess)
+          return e;
+    }
+    if ((e = cudaMemset2DAsync(a.lse, (size_t)a.Lq * sizeof(float), 0, rows * sizeof(float),
+                               (size_t)a.B * a.nh, st)) != cudaSuccess)
+      return e;
+  }
+  if (a.n_items == 0) return cudaSuccess;
+  const int grid = std::min(a.n_items, num_sms());
+  kern<<<grid, FA_THREADS, FA_SMEM, st>>>(tq, tkv, a);
+  return cudaGetLastError();
+}
+
+double cross_pairs(int Lq, int Lk, int P, bool causal) {
+  if (!causal) return (double)Lq * Lk;
+  double s = 0.0;
+  for (int i = 0; (long)i * P < Lq; ++i)  // block i's tokens see min(i, Lk) proxies
+    s += (double)std::min(P, Lq - i * P) * std::min(i, Lk);
+  return s;
+}
+
+}  // namespace
+
 cudaError_t attn_fwd(const bf16* qkv, bf16* out, float* lse, int B, int m, int d, int nh,
                         bool causal, cudaStream_t st) {
   if (d != nh * FA_D || ((uintptr_t)qkv & 15) || ((uintptr_t)out & 15))
@@ -367,23 +450,53 @@ cudaError_t attn_fwd(const bf16* qkv, bf16* out, float* lse, int B, int m, int d
   FaArgs a{};
   a.out = out;
   a.lse = lse;
+  a.ldo = d;
+  a.qcol = 0;
+  a.kcol = d;
+  a.vcol = 2 * d;
   a.B = B;
-  a.m = m;
+  a.Lq = a.Lk = m;
   a.d = d;
   a.nh = nh;
   a.causal = causal ? 1 : 0;
-  a.n_qt = (m + FA_M - 1) / FA_M;
-  a.n_kt = (m + FA_N - 1) / FA_N;
-  a.n_items = a.n_qt * nh * B;
-  a.sl2 = 1.4426950408889634f / sqrtf((float)FA_D);
-  auto kern = attn_fwd_tc_kernel;
-  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, FA_SMEM);
-  if (e != cudaSuccess) return e;
+  a.P = 0;
   const double pairs = (double)B * nh * (causal ? 0.5 * m * (m + 1.0) : (double)m * m);
-  LaunchTimer lt("attn_fwd", st, 4.0 * FA_D * pairs, 2.0 * B * m * (4.0 * d) + 4.0 * B * nh * m);
-  const int grid = std::min(a.n_items, num_sms());
-  kern<<<grid, FA_THREADS, FA_SMEM, st>>>(tm, a);
-  return cudaGetLastError();
+  return fa_launch(tm, tm, a, "attn_fwd", pairs, 2.0 * B * m * (4.0 * d) + 4.0 * B * nh * m, st);
+}
+
+cudaError_t attn_cross_fwd(const bf16* qa, long ldq, const bf16* kv, const float* b_a, bf16* out,
+                           bf16* out_g, float* lse, int B, int Lq, int Lk, int d, int nh, int P,
+                           bool causal, cudaStream_t st) {
+  if (d != nh * FA_D || P < 1 || ldq < d + nh || ((uintptr_t)qa & 15) || ((uintptr_t)kv & 15) ||
+      ((uintptr_t)out & 15) || ((uintptr_t)out_g & 15) || (ldq * 2) % 16 || !b_a)
+    return cudaErrorInvalidValue;
+  CUtensorMap tq, tkv;
+  if (!tmap_bf16_2d(&tq, qa, (uint64_t)ldq, (uint64_t)B * Lq, (uint64_t)ldq, 64, 128) ||
+      !tmap_bf16_2d(&tkv, kv, (uint64_t)2 * d, (uint64_t)B * Lk, (uint64_t)2 * d, 64, 128))
+    return cudaErrorInvalidValue;
+  FaArgs a{};
+  a.out = out;
+  a.out_g = out_g;
+  a.gpre = qa;
+  a.b_a = b_a;
+  a.lse = lse;
+  a.ldo = d;
+  a.ldg = ldq;
+  a.gcol = d;
+  a.qcol = 0;
+  a.kcol = 0;
+  a.vcol = d;
+  a.B = B;
+  a.Lq = Lq;
+  a.Lk = Lk;
+  a.d = d;
+  a.nh = nh;
+  a.causal = causal ? 1 : 0;
+  a.P = P;
+  const double pairs = (double)B * nh * cross_pairs(Lq, Lk, P, causal);
+  const double bytes = 2.0 * B * ((double)Lq * (d + nh) + 2.0 * Lk * d +
+                                  (out_g ? 2.0 : 1.0) * Lq * d) + 4.0 * B * nh * Lq;
+  return fa_launch(tq, tkv, a, "attn_cross_fwd", pairs, bytes, st);
 }
 
 }  // namespace pf

@@ -189,6 +189,11 @@ __global__ void splitk_reduce_kernel(const float* __restrict__ part, int S, int 
     const float4 a = *reinterpret_cast<const float4*>(e.addend + row * e.ld_add + col);
     v.x += a.x; v.y += a.y; v.z += a.z; v.w += a.w;
   }
+  if (e.add_bf16) {
+    const uint2 u = *reinterpret_cast<const uint2*>(e.add_bf16 + row * e.ld_add_bf16 + col);
+    const float2 a0 = unpack_bf16(u.x), a1 = unpack_bf16(u.y);
+    v.x += a0.x; v.y += a0.y; v.z += a1.x; v.w += a1.y;
+  }
   if (e.out_f32) *reinterpret_cast<float4*>(e.out_f32 + row * e.ld_f32 + col) = v;
   if (e.out_bf16)
     *reinterpret_cast<uint2*>(e.out_bf16 + row * e.ld_bf16 + col) =
@@ -248,7 +253,10 @@ cudaError_t gemm_linear(int M, int N, int K, Operand A, Operand B, const EpiLine
                                                                           N, e);
     return cudaGetLastError();
   }
-  EpiLinear epi{{}, M, N, e.bias, e.addend, e.ld_add, e.out_f32, e.ld_f32, e.out_bf16, e.ld_bf16};
+  if ((e.add_bf16 && ((uintptr_t)e.add_bf16 & 15)) || (e.add_bf16 && e.ld_add_bf16 % 8))
+    return cudaErrorInvalidValue;
+  EpiLinear epi{{},         M,          N,        e.bias,     e.addend,  e.ld_add,
+                e.out_f32,  e.ld_f32,   e.out_bf16, e.ld_bf16, e.add_bf16, e.ld_add_bf16};
   return gemm_dispatch(M, N, K, A, B, epi, nullptr, 0, st);
 }
 

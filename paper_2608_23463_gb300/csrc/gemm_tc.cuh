@@ -578,6 +578,8 @@ struct EpiLinear : EpiBase {
   long ld_f32;
   bf16* out_bf16;
   long ld_bf16;
+  const bf16* add_bf16;
+  long ld_add_bf16;
   __device__ __forceinline__ Row row_info(int row, int) const { return Row{row < M}; }
   __device__ __forceinline__ void apply(const Row& ri, int row, int col, float* v, const uint8_t*,
                                         int, int, const float4*) const {
@@ -595,6 +597,20 @@ struct EpiLinear : EpiBase {
       for (int i = 0; i < 32; i += 4) {
         float4 b = *reinterpret_cast<const float4*>(a + i);
         v[i] += b.x; v[i + 1] += b.y; v[i + 2] += b.z; v[i + 3] += b.w;
+      }
+    }
+    if (add_bf16) {
+      const bf16* a = add_bf16 + (long)row * ld_add_bf16 + col;
+#pragma unroll
+      for (int i = 0; i < 32; i += 8) {
+        const uint4 u = *reinterpret_cast<const uint4*>(a + i);
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const float2 f = unpack_bf16(w[j]);
+          v[i + 2 * j] += f.x;
+          v[i + 2 * j + 1] += f.y;
+        }
       }
     }
     if (out_f32) {

@@ -19,6 +19,8 @@ struct EpiLinearArgs {
   const float* bias = nullptr;    // [N]
   const float* addend = nullptr;  // [M, ld_add] fp32
   long ld_add = 0;
+  const bf16* add_bf16 = nullptr;  // [M, ld_add_bf16] bf16, added like addend
+  long ld_add_bf16 = 0;
   float* out_f32 = nullptr;
   long ld_f32 = 0;
   bf16* out_bf16 = nullptr;
@@ -163,6 +165,29 @@ bool tmap_bf16_2d(CUtensorMap* m, const void* base, uint64_t inner, uint64_t out
 // ------------------------------------------------------------- attention
 cudaError_t attn_fwd(const bf16* qkv, bf16* out, float* lse, int B, int m, int d, int nh,
                      bool causal, cudaStream_t st);
+// Cross-attention of the injection (Eq. inj-cross): queries from qa [B*Lq,
+// ldq] (columns [0, d), the gate pre-activations at [d, d + nh)), keys and
+// values from kv [B*Lk, 2d]; token q sees proxies j < q / P (causal) or all.
+// Writes out (ungated), out_g = sigmoid(gate + b_a) * out per head (if not
+// null), both [B*Lq, d], and LSE [B, nh, Lq].
+cudaError_t attn_cross_fwd(const bf16* qa, long ldq, const bf16* kv, const float* b_a, bf16* out,
+                           bf16* out_g, float* lse, int B, int Lq, int Lk, int d, int nh, int P,
+                           bool causal, cudaStream_t st);
+// Its backward, given dO (the gradient of the ungated output) and Di =
+// rowsum(dO * O): dQ into dqa columns [0, d) (row stride ldq), dK and dV into
+// dkv [B*Lk, 2d].
+cudaError_t attn_cross_bwd(const bf16* qa, long ldq, const bf16* kv, const bf16* dO,
+                           const float* lse, const float* Di, bf16* dqa, bf16* dkv, int B, int Lq,
+                           int Lk, int d, int nh, int P, bool causal, cudaStream_t st);
+// Gate of the cross injection, backward, one warp per (token row, head):
+// s = sum over the head's columns of dAg * A, alpha = sigmoid(qa[row, d + h] +
+// b_a[h]); dO = alpha * dAg, Di = alpha * s (= rowsum(dO * A)), and the gate
+// pre-activation gradient s alpha (1 - alpha) into dqa[row, d + h] (bf16;
+// columns [d + nh, ldq) zeroed) and ga[row, h] (fp32, row stride ldga,
+// columns [nh, ldga) zeroed).
+cudaError_t cross_gate_bwd(const bf16* dAg, const bf16* A, const bf16* qa, long ldq,
+                           const float* b_a, bf16* dO, float* Di, bf16* dqa, float* ga, int ldga,
+                           int B, int L, int d, int nh, cudaStream_t st);
 cudaError_t attn_bwd_tc(const bf16* qkv, const bf16* dO, const float* lse, const float* Di,
                         bf16* dqkv, int B, int m, int d, int nh, bool causal, cudaStream_t st);
 cudaError_t attn_bwd(const bf16* qkv, const bf16* O, const bf16* dO, const float* lse, float* Di,

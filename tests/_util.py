@@ -17,6 +17,10 @@ import numpy as np
 BF16_TOL = 2e-2
 BF16_MAX_TOL = 1e-1
 F32_TOL = 1e-4
+# gated cross-attention injection: its gradients' bf16 floor is RMS 1-2e-2,
+# max up to 2.3e-1 (test_bf16_error_floor.py); the bar is about twice that
+CROSS_TOL = 4e-2
+CROSS_MAX_TOL = 3e-1
 
 
 def rms(a):
