@@ -397,6 +397,12 @@ def measure_configs(torch, pf, S, peaks, warmup: int):
         "1D causal layer fwd+bwd, bf16, L=65536 d=1024 16x64 P=64", s2.batch * s2.L, ms, fl, nb,
         dom, peaks, 10)
     torch.cuda.empty_cache()
+    sx = S.spec_cross_layer()
+    ms, fl, nb, dom = layer_case(sx, 5, True, 5)
+    out["cross_layer_fwd_bwd"] = config_entry(
+        "1D causal layer fwd+bwd with gated cross-attention injection (Eq. inj-cross), bf16, "
+        "L=262144 d=1024 16x64 P=64 8x8", sx.batch * sx.L, ms, fl, nb, dom, peaks, 5)
+    torch.cuda.empty_cache()
     s5 = S.spec_c5()
     ms, fl, nb, dom = layer_case(s5, 4, True, 5)
     out["c5_2d_fwd_bwd"] = config_entry(

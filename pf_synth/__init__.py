@@ -276,6 +276,13 @@ def spec_c3_layer(P: int = 64):
     return LayerSpec(batch=1, L=262144, d=1024, n_heads=16, P=P, levels=2, k1=k1, k2=k2)
 
 
+def spec_cross_layer():
+    """The causal headline layer with gated cross-attention injection:
+    L=262144, d=1024, 16x64 heads, P=64 as 8x8."""
+    return LayerSpec(batch=1, L=262144, d=1024, n_heads=16, P=64, levels=2, k1=8, k2=8,
+                     inject=INJ_CROSS)
+
+
 C3_RATIOS = (16, 16, 32, 32, 64, 64, 64, 64, 128, 128, 256, 256)
 
 

@@ -20,7 +20,8 @@ import pf_synth as S
 from oracle import layer as OL
 from paper_2608_23463_gb300.layer import ProxyLayer, to_device
 from paper_2608_23463_gb300.stack import ProxyStack
-from tests._util import assert_close, assert_grad_close, assert_update_close
+from tests._util import (CROSS_MAX_TOL, CROSS_TOL, assert_close, assert_grad_close,
+                         assert_update_close)
 
 pytestmark = pytest.mark.gpu
 
@@ -65,17 +66,29 @@ def _layer_prefix_case(spec, seed):
     return inp, got, (ref_Xo, ref_H, ref_dX, ref_g)
 
 
-@pytest.mark.parametrize("which", ["layer_L262144_P64_8x8", "c2_L65536_P64"])
+@pytest.mark.parametrize("which", ["layer_L262144_P64_8x8", "c2_L65536_P64",
+                                   "cross_L262144_P64_8x8"])
 def test_causal_layer_full_size_prefix(which):
-    spec, seed = ((S.spec_c3_layer(64), 2) if which.startswith("layer") else (S.spec_c2(), 1))
+    """The gated cross-attention layer (Eq. inj-cross) keeps the prefix
+    property: a token reads only the proxies of earlier blocks."""
+    if which == "cross_L262144_P64_8x8":
+        spec, seed = S.spec_cross_layer(), 5
+    else:
+        spec, seed = ((S.spec_c3_layer(64), 2) if which.startswith("layer") else (S.spec_c2(), 1))
+    cross = spec.inject == S.INJ_CROSS
+    tol, max_tol = (CROSS_TOL, CROSS_MAX_TOL) if cross else (2e-2, 1e-1)
     inp, got, (Xo, H, dX, grads) = _layer_prefix_case(spec, seed)
     assert got["dX_tail_max"] == 0.0  # no gradient reaches tokens after T
-    assert_close("X_out", got["Xo"], Xo)
-    assert_update_close("X_out - X", inp["X"][:, :T], got["Xo"], Xo)
+    if cross:  # bf16 floor of this variant: X_out up to 5e-2 max (test_bf16_error_floor.py)
+        assert_grad_close("X_out", got["Xo"], Xo)
+    else:
+        assert_close("X_out", got["Xo"], Xo)
+    assert_update_close("X_out - X", inp["X"][:, :T], got["Xo"], Xo,
+                        max_tol=2e-1 if cross else 1e-1)
     assert_close("H_out", got["H"], H)
-    assert_grad_close("dX", got["dX"], dX)
+    assert_grad_close("dX", got["dX"], dX, tol, max_tol)
     for k, v in grads.items():
-        assert_grad_close("grad " + k, got["grads"][k], v)
+        assert_grad_close("grad " + k, got["grads"][k], v, tol, max_tol)
 
 
 def _rel(a, b):
