@@ -22,6 +22,9 @@ Readings of the paper taken here (each is a descriptor flag of the library):
     [2pd, 2pd+d) and [2pd+d, 2(p+1)d)); Norm is LayerNorm without affine,
     biased variance, eps 1e-6.
   * L % P != 0: the last block is zero-padded for compression (m = ceil(L/P)).
+  * Widths: tokens are d_fine wide and proxies d wide (d_fine = d unless the
+    spec says otherwise, the asymmetric history stream of the language
+    model); both compression levels output d, both decompression levels read d.
   * Cross-attention injection (Eq. inj-cross) in its gated form, the way the
     language model uses it (Eq. llm-cross / llm-gate): every token queries,
     per head, the interacted proxies it may see (causal: proxies of earlier
@@ -85,13 +88,14 @@ def unpartition(blocks, spec, L):
 def compress(Xb, prm, spec):
     """Eq. compress-linear and Eq. factor-cascade: c_i = Proj(Flatten(X_i)).
 
-    Flatten is token-major (index p*d + ch).  Two levels: level 1 groups the P
-    tokens into k2 consecutive groups of k1 and projects each group's k1*d
-    vector to d (y_{i,a}); level 2 concatenates the k2 rows and projects the
-    k2*d vector to d.  Returns C [m, d] and the level-1 rows Y [m, k2, d]."""
-    m, P, d = Xb.shape
-    k1, k2 = spec.k1, spec.k2
-    groups = Xb.reshape(m, k2, k1 * d)                     # vec of each group
+    Flatten is token-major (index p*d_fine + ch).  Two levels: level 1 groups
+    the P tokens into k2 consecutive groups of k1 and projects each group's
+    k1*d_fine vector to d (y_{i,a}); level 2 concatenates the k2 rows and
+    projects the k2*d vector to d.  Returns C [m, d] and the level-1 rows Y
+    [m, k2, d]."""
+    m, P, df = Xb.shape
+    k1, k2, d = spec.k1, spec.k2, spec.d
+    groups = Xb.reshape(m, k2, k1 * df)                    # vec of each group
     Y = groups @ _f64(prm["W_c1"]).T + _f64(prm["b_c1"])   # [m, k2, d]
     if spec.levels == 1:
         return Y.reshape(m, d), None
@@ -103,8 +107,8 @@ def decompress(Hbar, prm, spec):
     """Eq. decompress-linear and Eq. factor-dec: D_i = Unflatten(Proj_up(Hbar_i)).
 
     Two levels run in the opposite order: level 2 maps the proxy to k2 rows of
-    width d, level 1 maps each row to k1 tokens.  Output [m, P, w] with w = d,
-    or w = 2d for affine injection ([s | t] per token)."""
+    width d, level 1 maps each row to k1 tokens.  Output [m, P, w] with w =
+    d_fine, or w = 2d for affine injection ([s | t] per token)."""
     m, d = Hbar.shape
     k1, k2 = spec.k1, spec.k2
     if spec.levels == 2:
@@ -345,7 +349,8 @@ def _layernorm_bwd(dn, n, sd):
 def _inject_decompress_bwd(spec, prm, X, c, G, grads):
     """Backward of the decompression, routing and Eq. inj-add / inj-gate /
     inj-affine: returns (dX direct, dHbar)."""
-    L, d = X.shape
+    L, d = X.shape                                             # token width
+    dp = spec.d                                                # proxy width
     m = c["Xb"].shape[0]
     P, k1, k2 = spec.P, spec.k1, spec.k2
     Dt = c["Dt"]
@@ -381,24 +386,24 @@ def _inject_decompress_bwd(spec, prm, X, c, G, grads):
     # decompression
     dout = dD.reshape(m, k2, k1 * w)
     grads["b_d1"] += dout.sum((0, 1))
-    rows = c["Z"].reshape(m, k2, d) if spec.levels == 2 else c["Hbar"].reshape(m, 1, d)
-    grads["W_d1"] += dout.reshape(m * k2, k1 * w).T @ rows.reshape(m * k2, d)
-    drows = dout @ _f64(prm["W_d1"])                           # [m, k2, d]
+    rows = c["Z"].reshape(m, k2, dp) if spec.levels == 2 else c["Hbar"].reshape(m, 1, dp)
+    grads["W_d1"] += dout.reshape(m * k2, k1 * w).T @ rows.reshape(m * k2, dp)
+    drows = dout @ _f64(prm["W_d1"])                           # [m, k2, dp]
     if spec.levels == 2:
-        dZ = drows.reshape(m, k2 * d)
+        dZ = drows.reshape(m, k2 * dp)
         grads["b_d2"] += dZ.sum(0)
         grads["W_d2"] += dZ.T @ c["Hbar"]
         dHbar = dZ @ _f64(prm["W_d2"])
     else:
-        dHbar = drows.reshape(m, d)
+        dHbar = drows.reshape(m, dp)
     return dX, dHbar
 
 
 def _bwd_one(spec, prm, X, c, G, dH_out, grads):
-    L, d = X.shape
+    L, df = X.shape                                            # token width
+    d = spec.d                                                 # proxy width
     m = c["Xb"].shape[0]
     P, k1, k2 = spec.P, spec.k1, spec.k2
-    nh, dh = spec.n_heads, d // spec.n_heads
     if spec.inject == INJ_CROSS:
         dX, dHbar = cross_inject_bwd(G, X, c["Hbar"], c, prm, spec, grads)
     else:
@@ -439,10 +444,10 @@ def _bwd_one(spec, prm, X, c, G, dH_out, grads):
     else:
         dY = dC.reshape(m, 1, d)
     grads["b_c1"] += dY.sum((0, 1))
-    groups = c["Xb"].reshape(m, k2, k1 * d)
-    grads["W_c1"] += dY.reshape(m * k2, d).T @ groups.reshape(m * k2, k1 * d)
-    dgroups = dY @ _f64(prm["W_c1"])                          # [m, k2, k1*d]
-    dXc = unpartition(dgroups.reshape(m, P, d), spec, L)
+    groups = c["Xb"].reshape(m, k2, k1 * df)
+    grads["W_c1"] += dY.reshape(m * k2, d).T @ groups.reshape(m * k2, k1 * df)
+    dgroups = dY @ _f64(prm["W_c1"])                          # [m, k2, k1*df]
+    dXc = unpartition(dgroups.reshape(m, P, df), spec, L)
     return dX + dXc, dH_in
 
 

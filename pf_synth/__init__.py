@@ -54,11 +54,17 @@ class LayerSpec:
     grid_h: int = 0
     grid_w: int = 0
     patch: int = 0
+    d_fine: int = 0  # token width when it differs from the proxy width d
 
     def __post_init__(self):
         if self.levels == 1:
             object.__setattr__(self, "k1", self.P)
             object.__setattr__(self, "k2", 1)
+
+    @property
+    def df(self) -> int:
+        """Token (local stream) width: d_fine, else d."""
+        return self.d_fine or self.d
 
     @property
     def m(self) -> int:
@@ -115,9 +121,9 @@ def _finish(a: np.ndarray, dtype: int) -> np.ndarray:
 
 def layer_param_shapes(spec: LayerSpec) -> Dict[str, tuple]:
     """Parameter names and shapes, in generator fill order."""
-    d, P, k1, k2 = spec.d, spec.P, spec.k1, spec.k2
+    d, P, k1, k2, df = spec.d, spec.P, spec.k1, spec.k2, spec.df
     s = {}
-    s["W_c1"] = (d, k1 * d)
+    s["W_c1"] = (d, k1 * df)
     s["b_c1"] = (d,)
     if spec.levels == 2:
         s["W_c2"] = (d, k2 * d)
@@ -132,16 +138,16 @@ def layer_param_shapes(spec: LayerSpec) -> Dict[str, tuple]:
         s["W_kvx"] = (2 * d, d)
         s["W_ox"] = (d, d)
         return s
-    out_tok = 2 * d if spec.inject == INJ_AFFINE else d
+    out_tok = 2 * d if spec.inject == INJ_AFFINE else df
     if spec.levels == 2:
         s["W_d2"] = (k2 * d, d)
         s["b_d2"] = (k2 * d,)
     s["W_d1"] = (k1 * out_tok, d)
     s["b_d1"] = (k1 * out_tok,)
     if spec.inject == INJ_GATED:
-        s["w_x"] = (d,)
-        s["w_dlt"] = (d,)
-        s["b_g"] = (d,)
+        s["w_x"] = (df,)
+        s["w_dlt"] = (df,)
+        s["b_g"] = (df,)
     if spec.mode == BIDIR_2D:
         s["W_t1"] = (d, TEMB_DIM)
         s["b_t1"] = (d,)
@@ -177,14 +183,14 @@ def make_layer_inputs(spec: LayerSpec, seed: int, with_h_in: bool = False,
     ~ N(0,1); dH_out ~ N(0,1); H_in ~ N(0,1) if requested; t ~ U(0,1) [B]."""
     p = make_layer_params(spec, seed)
     rng = np.random.default_rng(seed + 0x5EED)
-    B, L, d, m = spec.batch, spec.L, spec.d, spec.m
-    p["X"] = _finish(rng.standard_normal((B, L, d), dtype=np.float32), spec.dtype)
+    B, L, d, m, df = spec.batch, spec.L, spec.d, spec.m, spec.df
+    p["X"] = _finish(rng.standard_normal((B, L, df), dtype=np.float32), spec.dtype)
     if with_h_in:
         p["H_in"] = rng.standard_normal((B, m, d), dtype=np.float32)
     if spec.mode == BIDIR_2D:
         p["t"] = rng.uniform(0.0, 1.0, size=(B,)).astype(np.float32)
     if with_grads:
-        p["G"] = _finish(rng.standard_normal((B, L, d), dtype=np.float32), spec.dtype)
+        p["G"] = _finish(rng.standard_normal((B, L, df), dtype=np.float32), spec.dtype)
         p["dH_out"] = rng.standard_normal((B, m, d), dtype=np.float32)
     return p
 

@@ -193,6 +193,8 @@ FD_SPECS = {
                              inject=S.INJ_AFFINE, grid_h=8, grid_w=8, patch=2, dtype=S.F32),
     "causal_cross_1lvl": S.LayerSpec(batch=2, L=22, d=8, n_heads=2, P=4, inject=S.INJ_CROSS,
                                      dtype=S.F32),
+    "causal_gated_2lvl_dfine4": S.LayerSpec(batch=2, L=22, d=8, n_heads=2, P=4, levels=2, k1=2,
+                                            k2=2, d_fine=4, dtype=S.F32),
     "bidir_cross_2lvl": S.LayerSpec(batch=1, L=24, d=8, n_heads=2, P=4, levels=2, k1=2, k2=2,
                                     mode=S.BIDIR_1D, inject=S.INJ_CROSS, dtype=S.F32),
 }
@@ -308,6 +310,44 @@ def test_cross_injection_causality(mode):
                 assert np.abs(Xo2[0, lim:] - Xo[0, lim:]).max() > 1e-6
         else:
             assert np.abs(Xo2[0, :t0 // P * P] - Xo[0, :t0 // P * P]).max(initial=1.0) > 1e-6
+
+
+# ------------------------------------------------------ asymmetric widths
+@pytest.mark.parametrize("inject,levels", [(S.INJ_GATED, 2), (S.INJ_ADD, 1)])
+def test_asymmetric_widths_embed_in_a_symmetric_layer(inject, levels):
+    """A layer with d_fine = 4-wide tokens and d = 8-wide proxies equals the
+    symmetric d = 8 layer run on the tokens zero-padded to 8 channels, when
+    that layer's compression reads the real channels with the same weights
+    (its weights on the padding channels are arbitrary: they multiply zeros)
+    and its decompression writes zero into the padding channels.  The padded
+    channels of X_out must stay exactly zero."""
+    kw = dict(batch=2, L=22, d=8, n_heads=2, P=4, levels=levels, inject=inject, dtype=S.F32,
+              k1=2 if levels == 2 else 0, k2=2 if levels == 2 else 0)
+    sa, ss = S.LayerSpec(d_fine=4, **kw), S.LayerSpec(**kw)
+    pa = {k: v.astype(np.float64) for k, v in S.make_layer_params(sa, 51).items()}
+    ps = {k: v.astype(np.float64) for k, v in S.make_layer_params(ss, 52).items()}
+    k1, df, d = sa.k1, 4, 8
+    for k in ("b_c1", "W_c2", "b_c2", "W_qkv", "W_o", "W_d2", "b_d2"):
+        if k in pa:
+            ps[k] = pa[k]
+    for t in range(k1):  # token slot t of a k1-group: channels [t*d, t*d + df)
+        ps["W_c1"][:, t * d:t * d + df] = pa["W_c1"][:, t * df:(t + 1) * df]
+        ps["W_d1"][t * d:(t + 1) * d] = 0.0
+        ps["W_d1"][t * d:t * d + df] = pa["W_d1"][t * df:(t + 1) * df]
+        ps["b_d1"][t * d:(t + 1) * d] = 0.0
+        ps["b_d1"][t * d:t * d + df] = pa["b_d1"][t * df:(t + 1) * df]
+    if inject == S.INJ_GATED:
+        for k in ("w_x", "w_dlt", "b_g"):
+            ps[k][:df] = pa[k]
+    rng = np.random.default_rng(53)
+    Xa = rng.standard_normal((2, sa.L, df))
+    Xs = np.concatenate([Xa, np.zeros((2, sa.L, d - df))], axis=2)
+    H_in = rng.standard_normal((2, sa.m, d))
+    oa, ha = OL.layer_fwd(sa, pa, Xa, H_in)
+    os_, hs = OL.layer_fwd(ss, ps, Xs, H_in)
+    np.testing.assert_allclose(oa, os_[..., :df], rtol=1e-12, atol=1e-12)
+    assert (os_[..., df:] == 0.0).all()
+    np.testing.assert_allclose(ha, hs, rtol=1e-12, atol=1e-12)
 
 
 # ----------------------------------------------------------------- P6
