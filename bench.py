@@ -397,6 +397,13 @@ def measure_configs(torch, pf, S, peaks, warmup: int):
         "1D causal layer fwd+bwd, bf16, L=65536 d=1024 16x64 P=64", s2.batch * s2.L, ms, fl, nb,
         dom, peaks, 10)
     torch.cuda.empty_cache()
+    sh = S.spec_lm_history()
+    ms, fl, nb, dom = layer_case(sh, 6, True, 10)
+    out["lm_history_fwd_bwd"] = config_entry(
+        "1D causal layer fwd+bwd with 64-wide tokens and 512-wide proxies (the language model's "
+        "history stream), bf16, L=1048576 8x64 heads P=64", sh.batch * sh.L, ms, fl, nb, dom,
+        peaks, 10)
+    torch.cuda.empty_cache()
     sx = S.spec_cross_layer()
     ms, fl, nb, dom = layer_case(sx, 5, True, 5)
     out["cross_layer_fwd_bwd"] = config_entry(

@@ -60,8 +60,14 @@ enum { PF_F32 = 0, PF_BF16 = 1 };
  *   batch, L   : sequences and tokens per sequence (2D: L = grid_h*grid_w,
  *                tokens in raster order)
  *   grid_h, grid_w, patch : 2D only; P must equal patch*patch
- *   d, n_heads : d_fine = d_proxy = d (the paper's simplification, Sec. 4);
- *                head width d/n_heads must be 64
+ *   d, n_heads : proxy width d_proxy = d; head width d/n_heads must be 64
+ *   d_fine     : token (local stream) width; 0 means d (the paper's
+ *                simplification, Sec. 4).  Another positive multiple of 64
+ *                gives the asymmetric history stream of the language model
+ *                (Sec. 3.3: d_h = 64 against d = 512): X, X_out, dX are
+ *                [batch, L, d_fine], W_c1 is [d, k1*d_fine], W_d1 [k1*d_fine,
+ *                d], the gate vectors d_fine wide; 1D bf16 layers with add or
+ *                gated injection only
  *   P          : block size (compression ratio) of this layer (Sec. 3.6
  *                allows a different P per layer)
  *   levels     : 1 or 2 (Eq. factor with M = 2); levels == 2 needs k1*k2 == P,
@@ -82,19 +88,21 @@ typedef struct {
   int32_t d, n_heads;
   int32_t P, levels, k1, k2;
   int32_t mode, inject, dtype;
+  int32_t d_fine;
 } pf_layer_desc;
 
 /* Layer parameters (device pointers).  "mat" = dtype, "vec" = fp32.
- *   W_c1 [d, k1*d] mat, b_c1 [d] vec       compression level 1 (or single)
+ *   W_c1 [d, k1*df] mat, b_c1 [d] vec      compression level 1 (or single);
+ *                                          df = d_fine (d when 0)
  *   W_c2 [d, k2*d] mat, b_c2 [d] vec       compression level 2 (levels == 2)
  *   W_qkv [3d, d] mat                      proxy Q, K, V projections, stacked
  *   W_o  [d, d] mat                        proxy attention output projection
  *   W_d2 [k2*d, d] mat, b_d2 [k2*d] vec    decompression level 2 (levels == 2)
  *   W_d1 [k1*w, d] mat, b_d1 [k1*w] vec    decompression level 1 (or single);
- *                                          w = d, or 2d for PF_INJ_AFFINE where
+ *                                          w = df, or 2d for PF_INJ_AFFINE where
  *                                          token p's rows are [s | t] at
  *                                          [2pd, 2pd+d) and [2pd+d, 2(p+1)d)
- *   w_x, w_dlt, b_g [d] vec                gate g = w_x*X + w_dlt*D + b_g
+ *   w_x, w_dlt, b_g [df] vec               gate g = w_x*X + w_dlt*D + b_g
  *                                          (PF_INJ_GATED, Eq. inj-gate)
  *   W_t1 [d, 256] mat, b_t1 [d] vec,       timestep conditioning of the 2D
  *   W_t2 [2d, d] mat, b_t2 [2d] vec        proxies: u = SiLU(W_t1 e(t) + b_t1),

@@ -34,7 +34,8 @@ class ProxyFormerError(RuntimeError):
 
 class LayerDesc(ctypes.Structure):
     _fields_ = [(n, _c_i32) for n in ("batch", "L", "grid_h", "grid_w", "patch", "d", "n_heads",
-                                      "P", "levels", "k1", "k2", "mode", "inject", "dtype")]
+                                      "P", "levels", "k1", "k2", "mode", "inject", "dtype",
+                                      "d_fine")]
 
 
 _PARAM_NAMES = ("W_c1", "b_c1", "W_c2", "b_c2", "W_qkv", "W_o", "W_d2", "b_d2", "W_d1", "b_d1",

@@ -48,7 +48,7 @@ struct Carve {
 
 // Derived sizes of a validated 1D / 2D layer.
 struct Dims {
-  long B, L, d, nh, P, k1, k2, m, R, rows1, N1, Lp;
+  long B, L, d, df, nh, P, k1, k2, m, R, rows1, N1, Lp;  // d: proxy width, df: token width
   long T, ldq;  // tokens B*L; width of the token-query matrix [Q | gate | 0] (cross)
   bool causal, ragged, cross;
 };
@@ -58,6 +58,7 @@ Dims dims_of(const pf_layer_desc& s) {
   g.B = s.batch;
   g.L = s.L;
   g.d = s.d;
+  g.df = s.d_fine > 0 ? s.d_fine : s.d;
   g.nh = s.n_heads;
   g.P = s.P;
   g.k1 = s.levels == 2 ? s.k1 : s.P;
@@ -65,7 +66,7 @@ Dims dims_of(const pf_layer_desc& s) {
   g.m = (g.L + g.P - 1) / g.P;
   g.R = g.B * g.m;
   g.rows1 = g.R * g.k2;
-  g.N1 = g.k1 * g.d;
+  g.N1 = g.k1 * g.df;
   g.Lp = g.m * g.P;
   g.causal = s.mode == PF_CAUSAL_1D;
   g.ragged = g.Lp != g.L;
@@ -165,7 +166,7 @@ struct FwdWs {
 
 FwdWs carve_fwd(Carve& wc, const pf_layer_desc& s, const Dims& g, void* saved) {
   FwdWs f{};
-  f.Xpad = g.ragged ? wc.take<bf16>(g.B * g.Lp * g.d) : nullptr;
+  f.Xpad = g.ragged ? wc.take<bf16>(g.B * g.Lp * g.df) : nullptr;
   f.skb = splitk_need(s, g, false);
   f.sk = wc.take<float>(f.skb / sizeof(float));
   if (g.cross) f.Wqa = wc.take<bf16>(g.ldq * g.d);
@@ -188,8 +189,8 @@ struct BwdWs {
 
 BwdWs carve_bwd(Carve& c, const pf_layer_desc& s, const Dims& g) {
   BwdWs w{};
-  w.Xpad = g.ragged ? c.take<bf16>(g.B * g.Lp * g.d) : nullptr;
-  w.dXpad = g.ragged ? c.take<bf16>(g.B * g.Lp * g.d) : nullptr;
+  w.Xpad = g.ragged ? c.take<bf16>(g.B * g.Lp * g.df) : nullptr;
+  w.dXpad = g.ragged ? c.take<bf16>(g.B * g.Lp * g.df) : nullptr;
   if (g.cross) {
     w.Wqa = c.take<bf16>(g.ldq * g.d);
     w.dAg = c.take<bf16>(g.T * g.d);
@@ -331,6 +332,12 @@ pf_status check_desc(const pf_layer_desc* s) {
   if (s->levels == 2 && (s->k1 < 1 || s->k2 < 1 || (long)s->k1 * s->k2 != s->P))
     return fail(PF_ERR_INVALID_ARG, "levels == 2 needs k1 * k2 == P");
   if (s->mode < PF_CAUSAL_1D || s->mode > PF_BIDIR_2D) return fail(PF_ERR_INVALID_ARG, "bad mode");
+  if (s->d_fine < 0 || s->d_fine % 64 != 0)
+    return fail(PF_ERR_INVALID_ARG, "d_fine must be 0 (= d) or a positive multiple of 64");
+  if (s->d_fine > 0 && s->d_fine != s->d &&
+      (s->mode == PF_BIDIR_2D || s->dtype != PF_BF16 || s->inject == PF_INJ_CROSS))
+    return fail(PF_ERR_UNSUPPORTED,
+                "d_fine != d is built for 1D bf16 layers with add or gated injection");
   if (s->inject < PF_INJ_ADD || s->inject > PF_INJ_CROSS)
     return fail(PF_ERR_INVALID_ARG, "bad inject");
   if (s->dtype != PF_F32 && s->dtype != PF_BF16) return fail(PF_ERR_INVALID_ARG, "bad dtype");
@@ -639,12 +646,12 @@ pf_status proxy_layer_fwd(const pf_layer_desc* desc, const pf_layer_params* prm,
   cudaStream_t cs = static_cast<cudaStream_t>(stream);
   const bf16* Xb = static_cast<const bf16*>(X);
   bf16* Xo = static_cast<bf16*>(X_out);
-  const int d = (int)g.d;
+  const int d = (int)g.d, df = (int)g.df;  // proxy and token widths
 
   // a1: partition (a zero-copy view; the ragged tail goes through a padded copy)
   const bf16* Xsrc = Xb;
   if (g.ragged) {
-    PF_CUDA(pad_rows(Xb, Xpad, (int)g.B, g.L, g.Lp, d, cs));
+    PF_CUDA(pad_rows(Xb, Xpad, (int)g.B, g.L, g.Lp, df, cs));
     Xsrc = Xpad;
   }
   // a2 + a3: compression (Eq. compress-linear / factor-cascade), H = H_in + C
@@ -745,13 +752,13 @@ pf_status proxy_layer_fwd(const pf_layer_desc* desc, const pf_layer_params* prm,
   {
     EpiInjectArgs e{prm->b_d1, sv.D, Xsrc, Xo,
                     prm->w_x, prm->w_dlt, prm->b_g,
-                    d, (int)g.k1, (int)g.k2, (int)g.m, (int)g.L, g.causal ? 1 : 0,
+                    df, (int)g.k1, (int)g.k2, (int)g.m, (int)g.L, g.causal ? 1 : 0,
                     s.inject == PF_INJ_GATED ? 1 : 0};
     set_gemm_tag("decompress_d1_inject", (double)g.rows1 * g.N1 * 8.0);
     PF_CUDA(gemm_inject1d((int)g.rows1, (int)g.N1, d, {Zsrc, d, 0},
                           {static_cast<const bf16*>(prm->W_d1), d, 0}, e, cs));
   }
-  if (g.causal) PF_CUDA(copy_block0(Xb, g.L, Xo, g.L, (int)g.B, d, (int)std::min(g.P, g.L), cs));
+  if (g.causal) PF_CUDA(copy_block0(Xb, g.L, Xo, g.L, (int)g.B, df, (int)std::min(g.P, g.L), cs));
   return PF_OK;
 }
 
@@ -789,7 +796,7 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
   const bf16* Xb = static_cast<const bf16*>(X);
   const bf16* G = static_cast<const bf16*>(dX_out);
   bf16* dXb = static_cast<bf16*>(dX);
-  const int d = (int)g.d, N1 = (int)g.N1;
+  const int d = (int)g.d, N1 = (int)g.N1, df = (int)g.df;  // proxy and token widths
   const bf16* W_c1 = static_cast<const bf16*>(prm->W_c1);
   const bf16* W_c2 = static_cast<const bf16*>(prm->W_c2);
   const bf16* W_qkv = static_cast<const bf16*>(prm->W_qkv);
@@ -799,7 +806,7 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
 
   const bf16* Xsrc = Xb;
   if (g.ragged) {
-    PF_CUDA(pad_rows(Xb, w.Xpad, (int)g.B, g.L, g.Lp, d, cs));
+    PF_CUDA(pad_rows(Xb, w.Xpad, (int)g.B, g.L, g.Lp, df, cs));
     Xsrc = w.Xpad;
   }
   // direct injection gradient: written into dX, or into a block-padded buffer
@@ -879,13 +886,13 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
     {
       const int nch = inj_bwd_chunks(g.rows1, N1);
       InjBwdArgs a{G, Xb, sv.D, w.dD, dXd, g.ragged ? g.Lp : g.L, prm->w_x, prm->w_dlt, prm->b_g,
-                   d, (int)g.k1, (int)g.k2, (int)g.m, (int)g.L, (int)g.B, g.causal ? 1 : 0,
+                   df, (int)g.k1, (int)g.k2, (int)g.m, (int)g.L, (int)g.B, g.causal ? 1 : 0,
                    gated ? 1 : 0};
       PF_CUDA(inj_bwd_1d(a, w.part, nch, cs));
       if (g.causal)
-        PF_CUDA(copy_block0(G, g.L, dXd, g.ragged ? g.Lp : g.L, (int)g.B, d,
+        PF_CUDA(copy_block0(G, g.L, dXd, g.ragged ? g.Lp : g.L, (int)g.B, df,
                             (int)std::min(g.P, g.L), cs));
-      PF_CUDA(inj_bwd_finalize(w.part, nch, N1, d, grads->b_d1, gated ? grads->w_x : nullptr,
+      PF_CUDA(inj_bwd_finalize(w.part, nch, N1, df, grads->b_d1, gated ? grads->w_x : nullptr,
                                gated ? grads->w_dlt : nullptr, gated ? grads->b_g : nullptr, cs));
     }
     // decompression level 1 (or single level)
@@ -987,7 +994,7 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
     PF_CUDA(gemm_linear(d, N1, (int)g.rows1, {dYsrc, d, 1}, {Xsrc, N1, 1}, with_sk(e, w.sk, w.skb), cs));
   }
   {
-    EpiDXArgs e{dXd, dXb, d, (int)g.k1, (int)g.k2, (int)g.m, (int)g.L};
+    EpiDXArgs e{dXd, dXb, df, (int)g.k1, (int)g.k2, (int)g.m, (int)g.L};
     set_gemm_tag("bwd_dX", (double)g.rows1 * N1 * 4.0);
     PF_CUDA(gemm_dx1d((int)g.rows1, N1, d, {dYsrc, d, 0}, {W_c1, N1, 1}, e, cs));
   }
@@ -1331,8 +1338,8 @@ pf_status proxy_layer_prefill(const pf_layer_desc* desc, const pf_layer_params* 
   if (st != PF_OK) return st;
   const pf_layer_desc& s = *desc;
   const pf_decode_desc& c = *cdesc;
-  if (s.mode != PF_CAUSAL_1D || s.dtype != PF_BF16)
-    return fail(PF_ERR_UNSUPPORTED, "prefill needs a causal 1D bf16 layer");
+  if (s.mode != PF_CAUSAL_1D || s.dtype != PF_BF16 || (s.d_fine > 0 && s.d_fine != s.d))
+    return fail(PF_ERR_UNSUPPORTED, "prefill needs a causal 1D bf16 layer with d_fine == d");
   if (c.batch != s.batch || c.d != s.d || c.n_heads != s.n_heads || c.P != s.P ||
       c.levels != s.levels || (s.levels == 2 && (c.k1 != s.k1 || c.k2 != s.k2)))
     return fail(PF_ERR_INVALID_ARG, "the cache descriptor does not match the layer");

@@ -55,7 +55,8 @@ class ProxyLayer:
 
     def empty_act(self) -> torch.Tensor:
         s = self.spec
-        return torch.empty((s.batch, s.L, s.d), dtype=self.act_dtype, device=self.device)
+        width = getattr(s, "d_fine", 0) or s.d  # token width
+        return torch.empty((s.batch, s.L, width), dtype=self.act_dtype, device=self.device)
 
     def empty_proxy(self) -> torch.Tensor:
         s = self.spec

@@ -24,7 +24,8 @@ class ProxyStack:
         self.ws = torch.empty(max(need, 16), dtype=torch.uint8, device=device)
         self.layers = [ProxyLayer(s, p, device, ws=self.ws) for s, p in zip(specs, params)]
         s0 = specs[0]
-        self.X = [torch.empty((s0.batch, s0.L, s0.d), dtype=torch.bfloat16, device=device)
+        width = getattr(s0, "d_fine", 0) or s0.d  # token width
+        self.X = [torch.empty((s0.batch, s0.L, width), dtype=torch.bfloat16, device=device)
                   for _ in range(len(specs) + 1)]
         self.H = [lay.empty_proxy() for lay in self.layers]
         self.dX = [torch.empty_like(self.X[0]) for _ in range(2)]

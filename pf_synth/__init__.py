@@ -289,6 +289,13 @@ def spec_cross_layer():
                      inject=INJ_CROSS)
 
 
+def spec_lm_history():
+    """The language model's history layer (Sec. 3.3, Sec. 5.1): 64-wide
+    tokens compressed into 512-wide proxies, 8x64 heads, P = 64, a
+    1048576-token history."""
+    return LayerSpec(batch=1, L=1048576, d=512, n_heads=8, P=64, d_fine=64)
+
+
 C3_RATIOS = (16, 16, 32, 32, 64, 64, 64, 64, 128, 128, 256, 256)
 
 

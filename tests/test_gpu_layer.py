@@ -54,6 +54,16 @@ CASES = {
                         False, False),
     "cross_d1024_P64_8x8": (S.LayerSpec(batch=1, L=4096, d=1024, n_heads=16, P=64, levels=2,
                                         k1=8, k2=8, inject=S.INJ_CROSS), True, True),
+    # asymmetric widths (the language model's history stream, d_h = 64 tokens
+    # against d = 512 proxies): ragged with two sequences, 8x8 factors,
+    # bidirectional add injection with 128-wide tokens
+    "asym_dfine64_d512_P64_ragged_b2": (S.LayerSpec(batch=2, L=2000, d=512, n_heads=8, P=64,
+                                                    d_fine=64), True, False),
+    "asym_dfine64_d512_P64_8x8": (S.LayerSpec(batch=1, L=8192, d=512, n_heads=8, P=64, levels=2,
+                                              k1=8, k2=8, d_fine=64), False, False),
+    "asym_bidir_add_dfine128": (S.LayerSpec(batch=1, L=1024, d=256, n_heads=4, P=16,
+                                            mode=S.BIDIR_1D, inject=S.INJ_ADD, d_fine=128),
+                                False, False),
 }
 
 
