@@ -22,6 +22,10 @@ Readings of the paper taken here (each is a descriptor flag of the library):
     [2pd, 2pd+d) and [2pd+d, 2(p+1)d)); Norm is LayerNorm without affine,
     biased variance, eps 1e-6.
   * L % P != 0: the last block is zero-padded for compression (m = ceil(L/P)).
+  * Proxy interaction F (Sec. 3.4): attention (Eq. proxy-attn), identity
+    (Hbar = H) or a single-proxy MLP Hbar = W_m2 SiLU(W_m1 H + b_m1) + b_m2 of
+    hidden width 4d; attention may rotate the proxies' queries and keys by
+    their index (RoPE, base 10000, pairs (2j, 2j+1) of each head).
   * Widths: tokens are d_fine wide and proxies d wide (d_fine = d unless the
     spec says otherwise, the asymmetric history stream of the language
     model); both compression levels output d, both decompression levels read d.
@@ -42,6 +46,8 @@ from typing import Dict, Optional
 import numpy as np
 
 CAUSAL_1D, BIDIR_1D, BIDIR_2D = 0, 1, 2
+F_ATTENTION, F_IDENTITY, F_MLP = 0, 1, 2
+ROPE_BASE = 10000.0
 INJ_ADD, INJ_GATED, INJ_AFFINE, INJ_CROSS = 0, 1, 2, 3
 LN_EPS = 1e-6
 TEMB_DIM = 256
@@ -131,15 +137,78 @@ def _row_probs(q, Kh, n_vis, scale):
     return e / e.sum()
 
 
+def rope(Z, nh, inverse=False):
+    """Rotary position embedding of rows Z [m, d] by their index i: within
+    each head, the pair (2j, 2j+1) turns by the angle i * ROPE_BASE^(-2j/dh)
+    (backwards when ``inverse``, the transpose of the rotation)."""
+    m, d = Z.shape
+    dh = d // nh
+    j = np.arange(dh // 2)
+    ang = np.arange(m)[:, None] * ROPE_BASE ** (-2.0 * j / dh)[None, :]  # [m, dh/2]
+    c, s = np.cos(ang), np.sin(ang)
+    if inverse:
+        s = -s
+    out = np.empty_like(Z)
+    for h in range(nh):
+        a = Z[:, h * dh:(h + 1) * dh:2]
+        b = Z[:, h * dh + 1:(h + 1) * dh:2]
+        out[:, h * dh:(h + 1) * dh:2] = a * c - b * s
+        out[:, h * dh + 1:(h + 1) * dh:2] = a * s + b * c
+    return out
+
+
+def silu_grad(u):
+    sg = sigmoid(u)
+    return sg * (1.0 + u * (1.0 - sg))
+
+
+def interact(Hq, prm, spec):
+    """The proxy interaction F (Sec. 3.4): identity, single-proxy MLP, or
+    attention (below)."""
+    f = getattr(spec, "interact", F_ATTENTION)
+    if f == F_IDENTITY:
+        return Hq.copy(), {}
+    if f == F_MLP:
+        U = Hq @ _f64(prm["W_m1"]).T + _f64(prm["b_m1"])
+        Am = silu(U)
+        return Am @ _f64(prm["W_m2"]).T + _f64(prm["b_m2"]), dict(U=U, Am=Am)
+    return attention(Hq, prm, spec)
+
+
+def interact_bwd(dHbar, c, prm, spec, grads):
+    """Backward of ``interact``: dHq, adding the interaction's weight gradients."""
+    f = getattr(spec, "interact", F_ATTENTION)
+    if f == F_IDENTITY:
+        return dHbar
+    if f == F_MLP:
+        grads["W_m2"] += dHbar.T @ c["Am"]
+        grads["b_m2"] += dHbar.sum(0)
+        dU = (dHbar @ _f64(prm["W_m2"])) * silu_grad(c["U"])
+        grads["W_m1"] += dU.T @ c["Hq"]
+        grads["b_m1"] += dU.sum(0)
+        return dU @ _f64(prm["W_m1"])
+    grads["W_o"] += dHbar.T @ c["A"]
+    dA = dHbar @ _f64(prm["W_o"])
+    dQ, dK, dV = attention_bwd(dA, c, spec)
+    if getattr(spec, "rope", 0):                          # back through the rotation
+        dQ, dK = rope(dQ, spec.n_heads, True), rope(dK, spec.n_heads, True)
+    dQKV = np.concatenate([dQ, dK, dV], axis=1)
+    grads["W_qkv"] += dQKV.T @ c["Hq"]
+    return dQKV @ _f64(prm["W_qkv"])
+
+
 def attention(Hq, prm, spec):
     """Eq. proxy-attn: Hbar = softmax(Q K^T / sqrt(dh) + M) V per head, then
     the output projection.  M is the causal mask (proxy i sees j <= i) for the
     autoregressive 1D mode and zero otherwise.  Evaluated one query row at a
-    time over the visible keys only."""
+    time over the visible keys only.  With RoPE, Q and K are rotated by the
+    proxy index first."""
     m, d = Hq.shape
     nh, dh = spec.n_heads, d // spec.n_heads
     W = _f64(prm["W_qkv"])
     Q, K, V = Hq @ W[:d].T, Hq @ W[d:2 * d].T, Hq @ W[2 * d:].T
+    if getattr(spec, "rope", 0):
+        Q, K = rope(Q, nh), rope(K, nh)
     A = np.zeros((m, d))
     scale = 1.0 / math.sqrt(dh)
     causal = spec.mode == CAUSAL_1D
@@ -292,7 +361,7 @@ def _fwd_one(spec, prm, X, H_in, t):
         nH, muH, sdH = layernorm(H)
         Hq = (1.0 + gamma) * nH + beta
         cache.update(gamma=gamma, beta=beta, tc=tc, nH=nH, sdH=sdH)
-    Hbar, ac = attention(Hq, prm, spec)                       # Eq. proxy-attn
+    Hbar, ac = interact(Hq, prm, spec)                        # F: Eq. proxy-attn, ...
     cache.update(Hq=Hq, Hbar=Hbar, **ac)
     if spec.inject == INJ_CROSS:                              # Eq. inj-cross (gated)
         Xo, cc = cross_inject(X, Hbar, prm, spec)
@@ -408,13 +477,8 @@ def _bwd_one(spec, prm, X, c, G, dH_out, grads):
         dX, dHbar = cross_inject_bwd(G, X, c["Hbar"], c, prm, spec, grads)
     else:
         dX, dHbar = _inject_decompress_bwd(spec, prm, X, c, G, grads)
-    # attention
-    grads["W_o"] += dHbar.T @ c["A"]
-    dA = dHbar @ _f64(prm["W_o"])
-    dQ, dK, dV = attention_bwd(dA, c, spec)
-    dQKV = np.concatenate([dQ, dK, dV], axis=1)
-    grads["W_qkv"] += dQKV.T @ c["Hq"]
-    dHq = dQKV @ _f64(prm["W_qkv"])
+    # proxy interaction
+    dHq = interact_bwd(dHbar, c, prm, spec, grads)
     if spec.mode == BIDIR_2D:
         gamma = c["gamma"]
         nH, sdH = c["nH"], c["sdH"]

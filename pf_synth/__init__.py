@@ -30,6 +30,7 @@ import numpy as np
 
 # mode / inject / dtype codes; they mirror the C header's enums.
 CAUSAL_1D, BIDIR_1D, BIDIR_2D = 0, 1, 2
+F_ATTENTION, F_IDENTITY, F_MLP = 0, 1, 2  # proxy interaction
 INJ_ADD, INJ_GATED, INJ_AFFINE, INJ_CROSS = 0, 1, 2, 3
 F32, BF16 = 0, 1
 
@@ -55,6 +56,8 @@ class LayerSpec:
     grid_w: int = 0
     patch: int = 0
     d_fine: int = 0  # token width when it differs from the proxy width d
+    interact: int = F_ATTENTION
+    rope: int = 0  # rotate the proxies' queries and keys (attention only)
 
     def __post_init__(self):
         if self.levels == 1:
@@ -128,8 +131,14 @@ def layer_param_shapes(spec: LayerSpec) -> Dict[str, tuple]:
     if spec.levels == 2:
         s["W_c2"] = (d, k2 * d)
         s["b_c2"] = (d,)
-    s["W_qkv"] = (3 * d, d)
-    s["W_o"] = (d, d)
+    if spec.interact == F_ATTENTION:
+        s["W_qkv"] = (3 * d, d)
+        s["W_o"] = (d, d)
+    elif spec.interact == F_MLP:
+        s["W_m1"] = (4 * d, d)
+        s["b_m1"] = (4 * d,)
+        s["W_m2"] = (d, 4 * d)
+        s["b_m2"] = (d,)
     if spec.inject == INJ_CROSS:
         # token queries stacked over the per-head gate rows; proxy keys and
         # values of the injection; its output projection

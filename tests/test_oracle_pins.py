@@ -195,6 +195,12 @@ FD_SPECS = {
                                      dtype=S.F32),
     "causal_gated_2lvl_dfine4": S.LayerSpec(batch=2, L=22, d=8, n_heads=2, P=4, levels=2, k1=2,
                                             k2=2, d_fine=4, dtype=S.F32),
+    "causal_gated_mlp": S.LayerSpec(batch=2, L=22, d=8, n_heads=2, P=4, interact=S.F_MLP,
+                                    dtype=S.F32),
+    "bidir_add_identity_2lvl": S.LayerSpec(batch=1, L=24, d=8, n_heads=2, P=4, levels=2, k1=2,
+                                           k2=2, mode=S.BIDIR_1D, inject=S.INJ_ADD,
+                                           interact=S.F_IDENTITY, dtype=S.F32),
+    "causal_gated_rope": S.LayerSpec(batch=2, L=30, d=8, n_heads=2, P=4, rope=1, dtype=S.F32),
     "bidir_cross_2lvl": S.LayerSpec(batch=1, L=24, d=8, n_heads=2, P=4, levels=2, k1=2, k2=2,
                                     mode=S.BIDIR_1D, inject=S.INJ_CROSS, dtype=S.F32),
 }
@@ -348,6 +354,59 @@ def test_asymmetric_widths_embed_in_a_symmetric_layer(inject, levels):
     np.testing.assert_allclose(oa, os_[..., :df], rtol=1e-12, atol=1e-12)
     assert (os_[..., df:] == 0.0).all()
     np.testing.assert_allclose(ha, hs, rtol=1e-12, atol=1e-12)
+
+
+# ------------------------------------------------- proxy interaction variants
+def test_identity_interaction_closed_form():
+    """F = identity (Hbar = H) with P = 1 and identity compression and
+    decompression: each token receives the previous token (causal routing),
+    the first nothing -- X_out[t] = X[t] + X[t-1] exactly."""
+    spec = _spec(inject=S.INJ_ADD, interact=S.F_IDENTITY)
+    d = spec.d
+    prm = {"W_c1": np.eye(d), "b_c1": np.zeros(d), "W_d1": np.eye(d), "b_d1": np.zeros(d)}
+    X = np.random.default_rng(61).standard_normal((1, spec.L, d))
+    Xo, H = OL.layer_fwd(spec, prm, X)
+    np.testing.assert_array_equal(Xo[0, 0], X[0, 0])
+    np.testing.assert_array_equal(Xo[0, 1:], X[0, 1:] + X[0, :-1])
+    np.testing.assert_array_equal(H[0], X[0])
+
+
+def test_mlp_interaction_equals_torch():
+    """The single-proxy MLP is torch's linear -> SiLU -> linear on every row."""
+    spec = S.LayerSpec(batch=1, L=40, d=8, n_heads=2, P=4, interact=S.F_MLP, dtype=S.F32)
+    prm = {k: v.astype(np.float64) for k, v in S.make_layer_params(spec, 62).items()}
+    H = np.random.default_rng(63).standard_normal((spec.m, spec.d))
+    got, _ = OL.interact(H, prm, spec)
+    T = lambda a: torch.from_numpy(np.asarray(a, np.float64))
+    ref = F.linear(F.silu(F.linear(T(H), T(prm["W_m1"]), T(prm["b_m1"]))), T(prm["W_m2"]),
+                   T(prm["b_m2"]))
+    np.testing.assert_allclose(got, ref.numpy(), rtol=1e-12, atol=1e-12)
+
+
+def test_rope_rotation_properties():
+    """RoPE on the proxies: position 0 is the identity; position 1 turns pair
+    j of a head by base^(-2j/dh) radians; the inverse is the transpose; and a
+    rotated query-key dot product depends only on the distance of the two
+    positions (shifting both leaves it unchanged)."""
+    nh, dh, m = 2, 8, 12
+    d = nh * dh
+    rng = np.random.default_rng(64)
+    Z = rng.standard_normal((m, d))
+    R = OL.rope(Z, nh)
+    np.testing.assert_array_equal(R[0], Z[0])
+    e = np.zeros((2, d))
+    e[1, 2] = 1.0  # head 0, pair j = 1, first element, at position 1
+    r = OL.rope(e, nh)[1]
+    a = OL.ROPE_BASE ** (-2.0 / dh)
+    np.testing.assert_allclose(r[2:4], [math.cos(a), math.sin(a)], rtol=1e-14, atol=1e-15)
+    np.testing.assert_allclose(OL.rope(R, nh, inverse=True), Z, rtol=1e-12, atol=1e-12)
+    q, k = rng.standard_normal(d), rng.standard_normal(d)
+    def dot_at(i, j):
+        Q = np.zeros((m, d)); K = np.zeros((m, d))
+        Q[i], K[j] = q, k
+        return float(OL.rope(Q, nh)[i] @ OL.rope(K, nh)[j])
+    for i, j, s in ((5, 2, 3), (7, 7, 4), (1, 9, 2)):
+        assert abs(dot_at(i, j) - dot_at(i + s, j + s)) < 1e-12
 
 
 # ----------------------------------------------------------------- P6
