@@ -404,6 +404,15 @@ def measure_configs(torch, pf, S, peaks, warmup: int):
         "history stream), bf16, L=1048576 8x64 heads P=64", sh.batch * sh.L, ms, fl, nb, dom,
         peaks, 10)
     torch.cuda.empty_cache()
+    for key, kw in (("mlp_interaction_fwd_bwd", dict(interact=S.F_MLP)),
+                    ("rope_attention_fwd_bwd", dict(rope=1))):
+        sv = S.LayerSpec(batch=1, L=262144, d=1024, n_heads=16, P=64, levels=2, k1=8, k2=8, **kw)
+        ms, fl, nb, dom = layer_case(sv, 7, True, 10)
+        what = ("single-proxy MLP interaction (hidden 4d, SiLU)" if "mlp" in key
+                else "proxy attention with RoPE on queries and keys")
+        out[key] = config_entry(f"1D causal layer fwd+bwd with {what}, bf16, L=262144 d=1024 "
+                                "16x64 P=64 8x8", sv.L, ms, fl, nb, dom, peaks, 10)
+        torch.cuda.empty_cache()
     sx = S.spec_cross_layer()
     ms, fl, nb, dom = layer_case(sx, 5, True, 5)
     out["cross_layer_fwd_bwd"] = config_entry(

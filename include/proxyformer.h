@@ -55,6 +55,7 @@ typedef enum {
 enum { PF_CAUSAL_1D = 0, PF_BIDIR_1D = 1, PF_BIDIR_2D = 2 };
 enum { PF_INJ_ADD = 0, PF_INJ_GATED = 1, PF_INJ_AFFINE = 2, PF_INJ_CROSS = 3 };
 enum { PF_F32 = 0, PF_BF16 = 1 };
+enum { PF_F_ATTENTION = 0, PF_F_IDENTITY = 1, PF_F_MLP = 2 };
 
 /* One ProxyFormer layer (Alg. 1; m = ceil(L/P), Sec. 3.1).
  *   batch, L   : sequences and tokens per sequence (2D: L = grid_h*grid_w,
@@ -68,6 +69,13 @@ enum { PF_F32 = 0, PF_BF16 = 1 };
  *                [batch, L, d_fine], W_c1 is [d, k1*d_fine], W_d1 [k1*d_fine,
  *                d], the gate vectors d_fine wide; 1D bf16 layers with add or
  *                gated injection only
+ *   interact   : proxy interaction F (Sec. 3.4): PF_F_ATTENTION (Eq.
+ *                proxy-attn), PF_F_IDENTITY (Hbar = H) or PF_F_MLP (Hbar =
+ *                W_m2 SiLU(W_m1 H + b_m1) + b_m2, hidden width 4d, one proxy
+ *                at a time); other than attention: 1D bf16 only
+ *   rope       : 1 rotates the proxies' queries and keys by proxy index before
+ *                the attention (RoPE, base 10000, pairs (2j, 2j+1) of each
+ *                head); attention, 1D bf16 only
  *   P          : block size (compression ratio) of this layer (Sec. 3.6
  *                allows a different P per layer)
  *   levels     : 1 or 2 (Eq. factor with M = 2); levels == 2 needs k1*k2 == P,
@@ -89,6 +97,7 @@ typedef struct {
   int32_t P, levels, k1, k2;
   int32_t mode, inject, dtype;
   int32_t d_fine;
+  int32_t interact, rope;
 } pf_layer_desc;
 
 /* Layer parameters (device pointers).  "mat" = dtype, "vec" = fp32.
@@ -112,6 +121,8 @@ typedef struct {
  *   b_a [n_heads] vec                      PF_INJ_CROSS: gate bias
  *   W_kvx [2d, d] mat                      PF_INJ_CROSS: proxy keys, values
  *   W_ox [d, d] mat                        PF_INJ_CROSS: output projection
+ *   W_m1 [4d, d] mat, b_m1 [4d] vec,       PF_F_MLP: the single-proxy MLP
+ *   W_m2 [d, 4d] mat, b_m2 [d] vec
  * Unused pointers may be NULL.                                                  */
 typedef struct {
   const void *W_c1;  const float *b_c1;
@@ -124,6 +135,8 @@ typedef struct {
   const void *W_t2;  const float *b_t2;
   const void *W_qa;  const float *b_a;
   const void *W_kvx; const void *W_ox;
+  const void *W_m1;  const float *b_m1;
+  const void *W_m2;  const float *b_m2;
 } pf_layer_params;
 
 /* Parameter gradients, fp32 device buffers shaped like pf_layer_params.
@@ -132,6 +145,7 @@ typedef struct {
   float *W_c1, *b_c1, *W_c2, *b_c2, *W_qkv, *W_o, *W_d2, *b_d2, *W_d1, *b_d1;
   float *w_x, *w_dlt, *b_g, *W_t1, *b_t1, *W_t2, *b_t2;
   float *W_qa, *b_a, *W_kvx, *W_ox;
+  float *W_m1, *b_m1, *W_m2, *b_m2;
 } pf_layer_grads;
 
 /* Validates a descriptor; PF_OK or the reason it is rejected. */

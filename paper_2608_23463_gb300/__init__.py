@@ -21,6 +21,7 @@ PF_ERR_CAPACITY, PF_ERR_CUDA, PF_ERR_TIMEOUT = 4, 5, 6
 PF_CAUSAL_1D, PF_BIDIR_1D, PF_BIDIR_2D = 0, 1, 2
 PF_INJ_ADD, PF_INJ_GATED, PF_INJ_AFFINE, PF_INJ_CROSS = 0, 1, 2, 3
 PF_F32, PF_BF16 = 0, 1
+PF_F_ATTENTION, PF_F_IDENTITY, PF_F_MLP = 0, 1, 2
 
 _c_i32 = ctypes.c_int32
 _vp = ctypes.c_void_p
@@ -35,12 +36,12 @@ class ProxyFormerError(RuntimeError):
 class LayerDesc(ctypes.Structure):
     _fields_ = [(n, _c_i32) for n in ("batch", "L", "grid_h", "grid_w", "patch", "d", "n_heads",
                                       "P", "levels", "k1", "k2", "mode", "inject", "dtype",
-                                      "d_fine")]
+                                      "d_fine", "interact", "rope")]
 
 
 _PARAM_NAMES = ("W_c1", "b_c1", "W_c2", "b_c2", "W_qkv", "W_o", "W_d2", "b_d2", "W_d1", "b_d1",
                 "w_x", "w_dlt", "b_g", "W_t1", "b_t1", "W_t2", "b_t2", "W_qa", "b_a", "W_kvx",
-                "W_ox")
+                "W_ox", "W_m1", "b_m1", "W_m2", "b_m2")
 
 
 class LayerParams(ctypes.Structure):

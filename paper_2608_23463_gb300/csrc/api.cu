@@ -51,6 +51,8 @@ struct Dims {
   long B, L, d, df, nh, P, k1, k2, m, R, rows1, N1, Lp;  // d: proxy width, df: token width
   long T, ldq;  // tokens B*L; width of the token-query matrix [Q | gate | 0] (cross)
   bool causal, ragged, cross;
+  int f;      // proxy interaction: PF_F_ATTENTION / PF_F_IDENTITY / PF_F_MLP
+  bool rope;  // RoPE on the proxies' queries and keys
 };
 
 Dims dims_of(const pf_layer_desc& s) {
@@ -71,6 +73,8 @@ Dims dims_of(const pf_layer_desc& s) {
   g.causal = s.mode == PF_CAUSAL_1D;
   g.ragged = g.Lp != g.L;
   g.cross = s.inject == PF_INJ_CROSS;
+  g.f = s.interact;
+  g.rope = s.rope != 0;
   g.T = g.B * g.L;
   g.ldq = g.d + 64;  // the gate's n_heads <= 64 rows, zero-padded to 64
   return g;
@@ -95,6 +99,10 @@ size_t splitk_need(const pf_layer_desc& s, const Dims& g, bool bwd) {
   } else {
     v = {{N1, d, r1}, {r1, d, N1}, {d, d, R}, {R, d, d}, {3 * d, d, R}, {R, d, 3 * d}, {d, N1, r1}};
     if (s.levels == 2) v.insert(v.end(), {{n2, d, R}, {R, d, n2}, {d, n2, R}, {R, n2, d}});
+  }
+  if (g.f == PF_F_MLP) {  // the single-proxy MLP and its backward
+    if (!bwd) v.insert(v.end(), {{R, 4 * d, d}, {R, d, 4 * d}});
+    else v.insert(v.end(), {{d, 4 * d, R}, {R, 4 * d, d}, {4 * d, d, R}, {R, d, 4 * d}});
   }
   if (g.cross) {  // token queries + gate, proxy keys / values, output projection
     const int T = (int)g.T, q = (int)g.ldq, nh = (int)g.nh;
@@ -131,15 +139,22 @@ struct Saved {
   // ungated and gated, its LSE
   bf16 *QA, *KVx, *Ax, *Ag;
   float* LSEx;
+  bf16 *U, *Am;  // single-proxy MLP: pre-activation and SiLU of its hidden layer
 };
 
 Saved carve_saved(Carve& c, const pf_layer_desc& s, const Dims& g) {
   Saved v{};
   v.Hb = c.take<bf16>(g.R * g.d);
-  v.QKV = c.take<bf16>(g.R * 3 * g.d);
-  v.Aatt = c.take<bf16>(g.R * g.d);
+  if (g.f == PF_F_ATTENTION) {
+    v.QKV = c.take<bf16>(g.R * 3 * g.d);
+    v.Aatt = c.take<bf16>(g.R * g.d);
+  }
   v.Hbar = c.take<bf16>(g.R * g.d);
-  v.LSE = c.take<float>(g.B * g.nh * g.m);
+  if (g.f == PF_F_ATTENTION) v.LSE = c.take<float>(g.B * g.nh * g.m);
+  if (g.f == PF_F_MLP) {
+    v.U = c.take<bf16>(g.R * 4 * g.d);
+    v.Am = c.take<bf16>(g.R * 4 * g.d);
+  }
   if (s.levels == 2) v.Y = c.take<bf16>(g.rows1 * g.d);
   if (g.cross) {
     v.QA = c.take<bf16>(g.T * g.ldq);
@@ -185,6 +200,7 @@ struct BwdWs {
   bf16 *Wqa, *dAg, *dOx, *dQA, *dKVx;
   float *ga, *gsum, *Dix;  // ga: [T, ldga], columns past n_heads zero
   int ldga;
+  bf16* dU;  // single-proxy MLP: gradient of the hidden pre-activation
 };
 
 BwdWs carve_bwd(Carve& c, const pf_layer_desc& s, const Dims& g) {
@@ -206,8 +222,11 @@ BwdWs carve_bwd(Carve& c, const pf_layer_desc& s, const Dims& g) {
     if (s.levels == 2) w.dZ = c.take<bf16>(g.R * g.k2 * g.d);
   }
   w.dHbar = c.take<bf16>(g.R * g.d);
-  w.dA = c.take<bf16>(g.R * g.d);
-  w.dQKV = c.take<bf16>(g.R * 3 * g.d);
+  if (g.f == PF_F_ATTENTION) {
+    w.dA = c.take<bf16>(g.R * g.d);
+    w.dQKV = c.take<bf16>(g.R * 3 * g.d);
+  }
+  if (g.f == PF_F_MLP) w.dU = c.take<bf16>(g.R * 4 * g.d);
   w.dHb = c.take<bf16>(g.R * g.d);
   if (s.levels == 2) w.dY = c.take<bf16>(g.rows1 * g.d);
   w.Di = c.take<float>(g.B * g.nh * g.m);
@@ -217,6 +236,7 @@ BwdWs carve_bwd(Carve& c, const pf_layer_desc& s, const Dims& g) {
   pe = std::max(pe, colsum_part_elems(g.R, (int)g.d));
   pe = std::max(pe, colsum_part_elems(g.rows1, (int)g.d));
   if (g.cross) pe = std::max(pe, colsum_part_elems(g.T, (int)((g.nh + 7) & ~7L)));
+  if (g.f == PF_F_MLP) pe = std::max(pe, colsum_part_elems(g.R, (int)(4 * g.d)));
   w.part_elems = pe;
   w.part = c.take<float>(pe);
   w.skb = splitk_need(s, g, true);
@@ -314,7 +334,8 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 
 bool params_aligned(const pf_layer_params& p) {
   const void* ptrs[] = {p.W_c1, p.b_c1, p.W_c2,  p.b_c2, p.W_qkv, p.W_o,  p.W_d2,  p.b_d2,
                         p.W_d1, p.b_d1, p.w_x,   p.w_dlt, p.b_g,  p.W_t1, p.b_t1, p.W_t2,
-                        p.b_t2, p.W_qa, p.b_a,   p.W_kvx, p.W_ox};
+                        p.b_t2, p.W_qa, p.b_a,   p.W_kvx, p.W_ox, p.W_m1, p.b_m1, p.W_m2,
+                        p.b_m2};
   for (const void* q : ptrs)
     if (!aligned16(q)) return false;
   return true;
@@ -332,6 +353,13 @@ pf_status check_desc(const pf_layer_desc* s) {
   if (s->levels == 2 && (s->k1 < 1 || s->k2 < 1 || (long)s->k1 * s->k2 != s->P))
     return fail(PF_ERR_INVALID_ARG, "levels == 2 needs k1 * k2 == P");
   if (s->mode < PF_CAUSAL_1D || s->mode > PF_BIDIR_2D) return fail(PF_ERR_INVALID_ARG, "bad mode");
+  if (s->interact < PF_F_ATTENTION || s->interact > PF_F_MLP || s->rope < 0 || s->rope > 1)
+    return fail(PF_ERR_INVALID_ARG, "bad interact or rope");
+  if ((s->interact != PF_F_ATTENTION || s->rope) &&
+      (s->mode == PF_BIDIR_2D || s->dtype != PF_BF16))
+    return fail(PF_ERR_UNSUPPORTED, "identity / MLP interaction and RoPE are built for 1D bf16");
+  if (s->rope && s->interact != PF_F_ATTENTION)
+    return fail(PF_ERR_INVALID_ARG, "RoPE needs the attention interaction");
   if (s->d_fine < 0 || s->d_fine % 64 != 0)
     return fail(PF_ERR_INVALID_ARG, "d_fine must be 0 (= d) or a positive multiple of 64");
   if (s->d_fine > 0 && s->d_fine != s->d &&
@@ -620,7 +648,9 @@ pf_status proxy_layer_fwd(const pf_layer_desc* desc, const pf_layer_params* prm,
   if (prm == nullptr || X == nullptr || X_out == nullptr || X == X_out)
     return fail(PF_ERR_INVALID_ARG, "params, X and X_out are required and must not alias");
   const bool cross = s.inject == PF_INJ_CROSS;
-  if (!prm->W_c1 || !prm->b_c1 || !prm->W_qkv || !prm->W_o ||
+  const bool attn = s.interact == PF_F_ATTENTION, mlp = s.interact == PF_F_MLP;
+  if (!prm->W_c1 || !prm->b_c1 || (attn && (!prm->W_qkv || !prm->W_o)) ||
+      (mlp && (!prm->W_m1 || !prm->b_m1 || !prm->W_m2 || !prm->b_m2)) ||
       (!cross && (!prm->W_d1 || !prm->b_d1)) || (s.levels == 2 && (!prm->W_c2 || !prm->b_c2)) ||
       (s.levels == 2 && !cross && (!prm->W_d2 || !prm->b_d2)) ||
       (s.inject == PF_INJ_GATED && (!prm->w_x || !prm->w_dlt || !prm->b_g)) ||
@@ -688,14 +718,35 @@ pf_status proxy_layer_fwd(const pf_layer_desc* desc, const pf_layer_params* prm,
                           {static_cast<const bf16*>(prm->W_c2), g.k2 * d, 0}, with_sk(e2, sk, skb), cs));
     }
   }
-  // a4: proxy attention (Eq. proxy-attn)
-  {
+  // a4: proxy interaction F (Sec. 3.4)
+  if (g.f == PF_F_IDENTITY) {
+    PF_CUDA(cudaMemcpyAsync(sv.Hbar, sv.Hb, g.R * d * sizeof(bf16), cudaMemcpyDeviceToDevice, cs));
+  } else if (g.f == PF_F_MLP) {  // Hbar = W_m2 SiLU(W_m1 H + b_m1) + b_m2, one proxy at a time
+    EpiLinearArgs e;
+    e.bias = prm->b_m1;
+    e.pre_bf16 = sv.U;
+    e.ld_pre = 4 * d;
+    e.act_silu = 1;
+    e.out_bf16 = sv.Am;
+    e.ld_bf16 = 4 * d;
+    set_gemm_tag("proxy_mlp1", (double)g.R * 9 * d * 2.0);
+    PF_CUDA(gemm_linear((int)g.R, 4 * d, d, {sv.Hb, d, 0},
+                        {static_cast<const bf16*>(prm->W_m1), d, 0}, e, cs));
+    EpiLinearArgs e2;
+    e2.bias = prm->b_m2;
+    e2.out_bf16 = sv.Hbar;
+    e2.ld_bf16 = d;
+    set_gemm_tag("proxy_mlp2", (double)g.R * 5 * d * 2.0);
+    PF_CUDA(gemm_linear((int)g.R, d, 4 * d, {sv.Am, 4 * d, 0},
+                        {static_cast<const bf16*>(prm->W_m2), 4 * d, 0}, with_sk(e2, sk, skb), cs));
+  } else {  // attention (Eq. proxy-attn), queries and keys rotated first with RoPE
     EpiLinearArgs e;
     e.out_bf16 = sv.QKV;
     e.ld_bf16 = 3 * d;
     set_gemm_tag("proxy_qkv", (double)g.R * 3 * d * 2.0);
     PF_CUDA(gemm_linear((int)g.R, 3 * d, d, {sv.Hb, d, 0},
                         {static_cast<const bf16*>(prm->W_qkv), d, 0}, with_sk(e, sk, skb), cs));
+    if (g.rope) PF_CUDA(rope_qk(sv.QKV, 3 * d, (int)g.B, (int)g.m, d, false, cs));
     PF_CUDA(attn_fwd(sv.QKV, sv.Aatt, sv.LSE, (int)g.B, (int)g.m, d, (int)g.nh, g.causal, cs));
     EpiLinearArgs eo;
     eo.out_bf16 = sv.Hbar;
@@ -928,32 +979,40 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
       PF_CUDA(gemm_linear((int)g.R, d, n2, {w.dZ, n2, 0}, {W_d2, d, 1}, with_sk(e, w.sk, w.skb), cs));
     }
   }
-  // attention output projection and attention
-  if (grads->W_o) {
-    EpiLinearArgs e;
-    e.out_f32 = grads->W_o;
-    e.ld_f32 = d;
-    set_gemm_tag("bwd_dW_o", (double)d * d * 4.0);
-    PF_CUDA(gemm_linear(d, d, (int)g.R, {w.dHbar, d, 1}, {sv.Aatt, d, 1}, with_sk(e, w.sk, w.skb), cs));
-  }
-  {
-    EpiLinearArgs e;
-    e.out_bf16 = w.dA;
-    e.ld_bf16 = d;
-    set_gemm_tag("bwd_dA", (double)g.R * d * 2.0);
-    PF_CUDA(gemm_linear((int)g.R, d, d, {w.dHbar, d, 0}, {W_o, d, 1}, with_sk(e, w.sk, w.skb), cs));
-  }
-  PF_CUDA(attn_bwd(sv.QKV, sv.Aatt, w.dA, sv.LSE, w.Di, w.dQKV, (int)g.B, (int)g.m, d, (int)g.nh,
-                   g.causal, cs));
-  if (grads->W_qkv) {
-    EpiLinearArgs e;
-    e.out_f32 = grads->W_qkv;
-    e.ld_f32 = d;
-    set_gemm_tag("bwd_dW_qkv", (double)3 * d * d * 4.0);
-    PF_CUDA(gemm_linear(3 * d, d, (int)g.R, {w.dQKV, 3 * d, 1}, {sv.Hb, d, 1}, with_sk(e, w.sk, w.skb), cs));
-  }
+  // proxy interaction F: identity, single-proxy MLP, or attention
   float* dHf = dH_in ? dH_in : w.dHf;
-  {
+  if (g.f == PF_F_IDENTITY) {
+    PF_CUDA(add_f32_bf16(w.dHbar, dH_out, dHf, w.dHb, g.R * d, cs));
+  } else if (g.f == PF_F_MLP) {
+    const bf16* W_m1 = static_cast<const bf16*>(prm->W_m1);
+    const bf16* W_m2 = static_cast<const bf16*>(prm->W_m2);
+    if (grads->W_m2) {
+      EpiLinearArgs e;
+      e.out_f32 = grads->W_m2;
+      e.ld_f32 = 4 * d;
+      set_gemm_tag("bwd_dW_m2", (double)4 * d * d * 4.0);
+      PF_CUDA(gemm_linear(d, 4 * d, (int)g.R, {w.dHbar, d, 1}, {sv.Am, 4 * d, 1},
+                          with_sk(e, w.sk, w.skb), cs));
+    }
+    if (grads->b_m2) PF_CUDA(colsum_bf16(w.dHbar, g.R, d, grads->b_m2, w.part, cs));
+    {
+      EpiLinearArgs e;  // dU = (dHbar W_m2) * SiLU'(U)
+      e.dsilu_of = sv.U;
+      e.ld_dsilu = 4 * d;
+      e.out_bf16 = w.dU;
+      e.ld_bf16 = 4 * d;
+      set_gemm_tag("bwd_dU", (double)g.R * 9 * d * 2.0);
+      PF_CUDA(gemm_linear((int)g.R, 4 * d, d, {w.dHbar, d, 0}, {W_m2, 4 * d, 1}, e, cs));
+    }
+    if (grads->W_m1) {
+      EpiLinearArgs e;
+      e.out_f32 = grads->W_m1;
+      e.ld_f32 = d;
+      set_gemm_tag("bwd_dW_m1", (double)4 * d * d * 4.0);
+      PF_CUDA(gemm_linear(4 * d, d, (int)g.R, {w.dU, 4 * d, 1}, {sv.Hb, d, 1},
+                          with_sk(e, w.sk, w.skb), cs));
+    }
+    if (grads->b_m1) PF_CUDA(colsum_bf16(w.dU, g.R, 4 * d, grads->b_m1, w.part, cs));
     EpiLinearArgs e;
     e.addend = dH_out;
     e.ld_add = d;
@@ -961,8 +1020,45 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
     e.ld_f32 = d;
     e.out_bf16 = w.dHb;
     e.ld_bf16 = d;
-    set_gemm_tag("bwd_dH", (double)g.R * d * 10.0);
-    PF_CUDA(gemm_linear((int)g.R, d, 3 * d, {w.dQKV, 3 * d, 0}, {W_qkv, d, 1}, with_sk(e, w.sk, w.skb), cs));
+    set_gemm_tag("bwd_dH", (double)g.R * d * 14.0);
+    PF_CUDA(gemm_linear((int)g.R, d, 4 * d, {w.dU, 4 * d, 0}, {W_m1, d, 1},
+                        with_sk(e, w.sk, w.skb), cs));
+  } else {
+    if (grads->W_o) {
+      EpiLinearArgs e;
+      e.out_f32 = grads->W_o;
+      e.ld_f32 = d;
+      set_gemm_tag("bwd_dW_o", (double)d * d * 4.0);
+      PF_CUDA(gemm_linear(d, d, (int)g.R, {w.dHbar, d, 1}, {sv.Aatt, d, 1}, with_sk(e, w.sk, w.skb), cs));
+    }
+    {
+      EpiLinearArgs e;
+      e.out_bf16 = w.dA;
+      e.ld_bf16 = d;
+      set_gemm_tag("bwd_dA", (double)g.R * d * 2.0);
+      PF_CUDA(gemm_linear((int)g.R, d, d, {w.dHbar, d, 0}, {W_o, d, 1}, with_sk(e, w.sk, w.skb), cs));
+    }
+    PF_CUDA(attn_bwd(sv.QKV, sv.Aatt, w.dA, sv.LSE, w.Di, w.dQKV, (int)g.B, (int)g.m, d, (int)g.nh,
+                     g.causal, cs));
+    if (g.rope) PF_CUDA(rope_qk(w.dQKV, 3 * d, (int)g.B, (int)g.m, d, true, cs));  // back through it
+    if (grads->W_qkv) {
+      EpiLinearArgs e;
+      e.out_f32 = grads->W_qkv;
+      e.ld_f32 = d;
+      set_gemm_tag("bwd_dW_qkv", (double)3 * d * d * 4.0);
+      PF_CUDA(gemm_linear(3 * d, d, (int)g.R, {w.dQKV, 3 * d, 1}, {sv.Hb, d, 1}, with_sk(e, w.sk, w.skb), cs));
+    }
+    {
+      EpiLinearArgs e;
+      e.addend = dH_out;
+      e.ld_add = d;
+      e.out_f32 = dHf;
+      e.ld_f32 = d;
+      e.out_bf16 = w.dHb;
+      e.ld_bf16 = d;
+      set_gemm_tag("bwd_dH", (double)g.R * d * 10.0);
+      PF_CUDA(gemm_linear((int)g.R, d, 3 * d, {w.dQKV, 3 * d, 0}, {W_qkv, d, 1}, with_sk(e, w.sk, w.skb), cs));
+    }
   }
   // compression (H = H_in + C, so dC = dH)
   const bf16* dYsrc = w.dHb;
@@ -1338,8 +1434,10 @@ pf_status proxy_layer_prefill(const pf_layer_desc* desc, const pf_layer_params* 
   if (st != PF_OK) return st;
   const pf_layer_desc& s = *desc;
   const pf_decode_desc& c = *cdesc;
-  if (s.mode != PF_CAUSAL_1D || s.dtype != PF_BF16 || (s.d_fine > 0 && s.d_fine != s.d))
-    return fail(PF_ERR_UNSUPPORTED, "prefill needs a causal 1D bf16 layer with d_fine == d");
+  if (s.mode != PF_CAUSAL_1D || s.dtype != PF_BF16 || (s.d_fine > 0 && s.d_fine != s.d) ||
+      s.interact != PF_F_ATTENTION || s.rope)
+    return fail(PF_ERR_UNSUPPORTED,
+                "prefill needs a causal 1D bf16 attention layer with d_fine == d, no RoPE");
   if (c.batch != s.batch || c.d != s.d || c.n_heads != s.n_heads || c.P != s.P ||
       c.levels != s.levels || (s.levels == 2 && (c.k1 != s.k1 || c.k2 != s.k2)))
     return fail(PF_ERR_INVALID_ARG, "the cache descriptor does not match the layer");

@@ -523,6 +523,64 @@ cudaError_t inj_bwd_finalize(const float* part, int n_chunks, int N, int d, floa
   return cudaGetLastError();
 }
 
+namespace {
+
+// RoPE on Q | K, one thread per rotated pair: the angle i * 10000^(-2j/64)
+// is formed and reduced modulo 2 pi in double precision, then sin / cos in
+// single precision.
+__global__ void rope_qk_kernel(bf16* __restrict__ qk, long ld, long rows, int m, int d,
+                               float sgn) {
+  const long t = (long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= rows * d) return;  // d pairs per row: d / 2 in Q, d / 2 in K
+  const long row = t / d;
+  const int col = 2 * (int)(t % d);
+  const int j = (col & 63) >> 1;  // pair within the 64-wide head
+  const double theta = exp2(-(double)(2 * j) / 64.0 * 13.287712379549449);  // log2(10000)
+  double a = (double)(row % m) * theta;
+  a -= 6.283185307179586 * rint(a / 6.283185307179586);
+  float sn, cs;
+  sincosf((float)a, &sn, &cs);
+  sn *= sgn;
+  uint32_t* q = reinterpret_cast<uint32_t*>(qk + row * ld + col);
+  const float2 v = unpack_bf16(*q);
+  *q = pack_bf16(v.x * cs - v.y * sn, v.x * sn + v.y * cs);
+}
+
+__global__ void add_f32_bf16_kernel(const bf16* __restrict__ a, const float* __restrict__ b,
+                                    float* __restrict__ of, bf16* __restrict__ ob, long n4) {
+  const long t = (long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= n4) return;
+  const uint2 u = reinterpret_cast<const uint2*>(a)[t];
+  const float2 x = unpack_bf16(u.x), y = unpack_bf16(u.y);
+  float4 v = make_float4(x.x, x.y, y.x, y.y);
+  if (b) {
+    const float4 c = reinterpret_cast<const float4*>(b)[t];
+    v.x += c.x; v.y += c.y; v.z += c.z; v.w += c.w;
+  }
+  reinterpret_cast<float4*>(of)[t] = v;
+  reinterpret_cast<uint2*>(ob)[t] = make_uint2(pack_bf16(v.x, v.y), pack_bf16(v.z, v.w));
+}
+
+}  // namespace
+
+cudaError_t rope_qk(bf16* qk, long ld, int B, int m, int d, bool inverse, cudaStream_t st) {
+  if (d % 64 || ld < 2 * d) return cudaErrorInvalidValue;
+  const long rows = (long)B * m, n = rows * d;
+  LaunchTimer lt("rope_qk", st, 6.0 * n, 8.0 * n);
+  rope_qk_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(qk, ld, rows, m, d,
+                                                              inverse ? -1.f : 1.f);
+  return cudaGetLastError();
+}
+
+cudaError_t add_f32_bf16(const bf16* a, const float* b, float* out_f, bf16* out_b, long n,
+                         cudaStream_t st) {
+  if (n % 4) return cudaErrorInvalidValue;
+  const long n4 = n / 4;
+  LaunchTimer lt("add_f32_bf16", st, (double)n, 2.0 * n + (b ? 4.0 : 0.0) * n + 6.0 * n);
+  add_f32_bf16_kernel<<<(unsigned)((n4 + 255) / 256), 256, 0, st>>>(a, b, out_f, out_b, n4);
+  return cudaGetLastError();
+}
+
 long colsum_part_elems(long R, int C) { return (long)chunks_for(R, C) * C; }
 
 cudaError_t colsum_bf16(const bf16* X, long R, int C, float* out, float* part, cudaStream_t st) {

@@ -234,7 +234,7 @@ cudaError_t gemm_linear(int M, int N, int K, Operand A, Operand B, const EpiLine
                         cudaStream_t st) {
   const int S = splitk_factor(M, N, K);
   if (S > 1 && e.splitk_scratch && (size_t)S * M * N * sizeof(float) <= e.splitk_bytes &&
-      N % 4 == 0) {
+      N % 4 == 0 && !e.act_silu && !e.pre_bf16 && !e.dsilu_of) {
     // deterministic split-K: raw partials, then one reduce applying the epilogue
     if (M <= 0 || N % 32 != 0 || !operand_ok(A) || !operand_ok(B)) return cudaErrorInvalidValue;
     CUtensorMap ta, tb;
@@ -255,8 +255,12 @@ cudaError_t gemm_linear(int M, int N, int K, Operand A, Operand B, const EpiLine
   }
   if ((e.add_bf16 && ((uintptr_t)e.add_bf16 & 15)) || (e.add_bf16 && e.ld_add_bf16 % 8))
     return cudaErrorInvalidValue;
-  EpiLinear epi{{},         M,          N,        e.bias,     e.addend,  e.ld_add,
-                e.out_f32,  e.ld_f32,   e.out_bf16, e.ld_bf16, e.add_bf16, e.ld_add_bf16};
+  if ((e.pre_bf16 && ((uintptr_t)e.pre_bf16 & 15 || e.ld_pre % 8)) ||
+      (e.dsilu_of && ((uintptr_t)e.dsilu_of & 15 || e.ld_dsilu % 8)))
+    return cudaErrorInvalidValue;
+  EpiLinear epi{{},         M,          N,          e.bias,      e.addend,  e.ld_add,
+                e.out_f32,  e.ld_f32,   e.out_bf16, e.ld_bf16,   e.add_bf16, e.ld_add_bf16,
+                e.act_silu, e.pre_bf16, e.ld_pre,   e.dsilu_of,  e.ld_dsilu};
   return gemm_dispatch(M, N, K, A, B, epi, nullptr, 0, st);
 }
 

@@ -580,6 +580,11 @@ struct EpiLinear : EpiBase {
   long ld_bf16;
   const bf16* add_bf16;
   long ld_add_bf16;
+  int act_silu;
+  bf16* pre_bf16;
+  long ld_pre;
+  const bf16* dsilu_of;
+  long ld_dsilu;
   __device__ __forceinline__ Row row_info(int row, int) const { return Row{row < M}; }
   __device__ __forceinline__ void apply(const Row& ri, int row, int col, float* v, const uint8_t*,
                                         int, int, const float4*) const {
@@ -610,6 +615,30 @@ struct EpiLinear : EpiBase {
           const float2 f = unpack_bf16(w[j]);
           v[i + 2 * j] += f.x;
           v[i + 2 * j + 1] += f.y;
+        }
+      }
+    }
+    if (pre_bf16) {
+      bf16* o = pre_bf16 + (long)row * ld_pre + col;
+#pragma unroll
+      for (int i = 0; i < 32; i += 8) store8_bf16(o + i, v + i);
+    }
+    if (act_silu) {
+#pragma unroll
+      for (int i = 0; i < 32; ++i) v[i] = v[i] / (1.f + __expf(-v[i]));
+    }
+    if (dsilu_of) {
+      const bf16* u = dsilu_of + (long)row * ld_dsilu + col;
+#pragma unroll
+      for (int i = 0; i < 32; i += 8) {
+        const uint4 q = *reinterpret_cast<const uint4*>(u + i);
+        const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const float2 f = unpack_bf16(w[j]);
+          const float s0 = 1.f / (1.f + __expf(-f.x)), s1 = 1.f / (1.f + __expf(-f.y));
+          v[i + 2 * j] *= s0 * (1.f + f.x * (1.f - s0));
+          v[i + 2 * j + 1] *= s1 * (1.f + f.y * (1.f - s1));
         }
       }
     }

@@ -21,6 +21,14 @@ struct EpiLinearArgs {
   long ld_add = 0;
   const bf16* add_bf16 = nullptr;  // [M, ld_add_bf16] bf16, added like addend
   long ld_add_bf16 = 0;
+  // SiLU: the value after bias / addends is stored to pre_bf16 (if given),
+  // then out = SiLU(value); dsilu_of: out = value * SiLU'(u), u read from a
+  // bf16 matrix [M, ld_dsilu].  Either one disables split-K.
+  int act_silu = 0;
+  bf16* pre_bf16 = nullptr;
+  long ld_pre = 0;
+  const bf16* dsilu_of = nullptr;
+  long ld_dsilu = 0;
   float* out_f32 = nullptr;
   long ld_f32 = 0;
   bf16* out_bf16 = nullptr;
@@ -188,6 +196,13 @@ cudaError_t attn_cross_bwd(const bf16* qa, long ldq, const bf16* kv, const bf16*
 cudaError_t cross_gate_bwd(const bf16* dAg, const bf16* A, const bf16* qa, long ldq,
                            const float* b_a, bf16* dO, float* Di, bf16* dqa, float* ga, int ldga,
                            int B, int L, int d, int nh, cudaStream_t st);
+// RoPE on the proxies' queries and keys, in place: rows (b, i) of a [B*m, ld]
+// matrix, columns [0, 2d) = Q | K, pair (2j, 2j+1) of head h turned by the
+// angle i * 10000^(-2j/64) (backwards when inverse).
+cudaError_t rope_qk(bf16* qk, long ld, int B, int m, int d, bool inverse, cudaStream_t st);
+// out_f = a + b (b may be null), out_b = bf16(out_f), n elements (n % 4 == 0)
+cudaError_t add_f32_bf16(const bf16* a, const float* b, float* out_f, bf16* out_b, long n,
+                         cudaStream_t st);
 cudaError_t attn_bwd_tc(const bf16* qkv, const bf16* dO, const float* lse, const float* Di,
                         bf16* dqkv, int B, int m, int d, int nh, bool causal, cudaStream_t st);
 cudaError_t attn_bwd(const bf16* qkv, const bf16* O, const bf16* dO, const float* lse, float* Di,

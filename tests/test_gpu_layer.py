@@ -64,6 +64,20 @@ CASES = {
     "asym_bidir_add_dfine128": (S.LayerSpec(batch=1, L=1024, d=256, n_heads=4, P=16,
                                             mode=S.BIDIR_1D, inject=S.INJ_ADD, d_fine=128),
                                 False, False),
+    # proxy interaction variants (Sec. 3.4): single-proxy MLP, identity, and
+    # attention with RoPE on the proxies' queries and keys
+    "mlp_causal_gated_2lvl_ragged_b2": (S.LayerSpec(batch=2, L=2000, d=128, n_heads=2, P=16,
+                                                    levels=2, k1=4, k2=4, interact=S.F_MLP),
+                                        True, False),
+    "mlp_d1024_P64": (S.LayerSpec(batch=1, L=8192, d=1024, n_heads=16, P=64, interact=S.F_MLP),
+                      False, False),
+    "identity_bidir_add_b2": (S.LayerSpec(batch=2, L=1000, d=128, n_heads=2, P=16,
+                                          mode=S.BIDIR_1D, inject=S.INJ_ADD,
+                                          interact=S.F_IDENTITY), True, False),
+    "rope_causal_gated_b2": (S.LayerSpec(batch=2, L=4000, d=128, n_heads=2, P=16, rope=1),
+                             True, False),
+    "rope_d1024_P64_8x8": (S.LayerSpec(batch=1, L=16384, d=1024, n_heads=16, P=64, levels=2,
+                                       k1=8, k2=8, rope=1), False, False),
 }
 
 
