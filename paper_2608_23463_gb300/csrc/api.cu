@@ -175,7 +175,8 @@ struct FwdWs {
   bf16* Xpad;
   float* sk;
   size_t skb;
-  bf16* Wqa;  // cross: W_qa zero-padded to [d + 64, d]
+  bf16* Wqa;     // cross: W_qa zero-padded to [d + 64, d]
+  float2* rtab;  // RoPE: (cos, sin) per proxy position and pair [m, 32]
   Saved sv;
 };
 
@@ -185,6 +186,7 @@ FwdWs carve_fwd(Carve& wc, const pf_layer_desc& s, const Dims& g, void* saved) {
   f.skb = splitk_need(s, g, false);
   f.sk = wc.take<float>(f.skb / sizeof(float));
   if (g.cross) f.Wqa = wc.take<bf16>(g.ldq * g.d);
+  if (g.rope) f.rtab = wc.take<float2>(g.m * 32);
   Carve sc(saved);
   f.sv = saved ? carve_saved(sc, s, g) : carve_saved(wc, s, g);
   return f;
@@ -200,7 +202,8 @@ struct BwdWs {
   bf16 *Wqa, *dAg, *dOx, *dQA, *dKVx;
   float *ga, *gsum, *Dix;  // ga: [T, ldga], columns past n_heads zero
   int ldga;
-  bf16* dU;  // single-proxy MLP: gradient of the hidden pre-activation
+  bf16* dU;      // single-proxy MLP: gradient of the hidden pre-activation
+  float2* rtab;  // RoPE angle table [m, 32]
 };
 
 BwdWs carve_bwd(Carve& c, const pf_layer_desc& s, const Dims& g) {
@@ -227,6 +230,7 @@ BwdWs carve_bwd(Carve& c, const pf_layer_desc& s, const Dims& g) {
     w.dQKV = c.take<bf16>(g.R * 3 * g.d);
   }
   if (g.f == PF_F_MLP) w.dU = c.take<bf16>(g.R * 4 * g.d);
+  if (g.rope) w.rtab = c.take<float2>(g.m * 32);
   w.dHb = c.take<bf16>(g.R * g.d);
   if (s.levels == 2) w.dY = c.take<bf16>(g.rows1 * g.d);
   w.Di = c.take<float>(g.B * g.nh * g.m);
@@ -746,7 +750,7 @@ pf_status proxy_layer_fwd(const pf_layer_desc* desc, const pf_layer_params* prm,
     set_gemm_tag("proxy_qkv", (double)g.R * 3 * d * 2.0);
     PF_CUDA(gemm_linear((int)g.R, 3 * d, d, {sv.Hb, d, 0},
                         {static_cast<const bf16*>(prm->W_qkv), d, 0}, with_sk(e, sk, skb), cs));
-    if (g.rope) PF_CUDA(rope_qk(sv.QKV, 3 * d, (int)g.B, (int)g.m, d, false, cs));
+    if (g.rope) PF_CUDA(rope_qk(sv.QKV, 3 * d, (int)g.B, (int)g.m, d, fw.rtab, false, cs));
     PF_CUDA(attn_fwd(sv.QKV, sv.Aatt, sv.LSE, (int)g.B, (int)g.m, d, (int)g.nh, g.causal, cs));
     EpiLinearArgs eo;
     eo.out_bf16 = sv.Hbar;
@@ -1040,7 +1044,7 @@ pf_status proxy_layer_bwd(const pf_layer_desc* desc, const pf_layer_params* prm,
     }
     PF_CUDA(attn_bwd(sv.QKV, sv.Aatt, w.dA, sv.LSE, w.Di, w.dQKV, (int)g.B, (int)g.m, d, (int)g.nh,
                      g.causal, cs));
-    if (g.rope) PF_CUDA(rope_qk(w.dQKV, 3 * d, (int)g.B, (int)g.m, d, true, cs));  // back through it
+    if (g.rope) PF_CUDA(rope_qk(w.dQKV, 3 * d, (int)g.B, (int)g.m, d, w.rtab, true, cs));  // back
     if (grads->W_qkv) {
       EpiLinearArgs e;
       e.out_f32 = grads->W_qkv;

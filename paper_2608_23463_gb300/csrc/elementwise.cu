@@ -525,25 +525,33 @@ cudaError_t inj_bwd_finalize(const float* part, int n_chunks, int N, int d, floa
 
 namespace {
 
-// RoPE on Q | K, one thread per rotated pair: the angle i * 10000^(-2j/64)
-// is formed and reduced modulo 2 pi in double precision, then sin / cos in
-// single precision.
+// RoPE angles, one thread per (position i < m, pair j < 32): i * 10000^(-2j/64)
+// formed and reduced modulo 2 pi in double precision, (cos, sin) stored in
+// single precision.  Shared by every sequence, head and by Q and K.
+__global__ void rope_table_kernel(float2* __restrict__ tab, int m) {
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= m * 32) return;
+  const int i = t >> 5, j = t & 31;
+  const double theta = exp2(-(double)(2 * j) / 64.0 * 13.287712379549449);  // log2(10000)
+  double a = (double)i * theta;
+  a -= 6.283185307179586 * rint(a / 6.283185307179586);
+  float sn, cs;
+  sincosf((float)a, &sn, &cs);
+  tab[t] = make_float2(cs, sn);
+}
+
+// RoPE on Q | K in place, one thread per rotated pair, angles from the table.
 __global__ void rope_qk_kernel(bf16* __restrict__ qk, long ld, long rows, int m, int d,
-                               float sgn) {
+                               const float2* __restrict__ tab, float sgn) {
   const long t = (long)blockIdx.x * blockDim.x + threadIdx.x;
   if (t >= rows * d) return;  // d pairs per row: d / 2 in Q, d / 2 in K
   const long row = t / d;
   const int col = 2 * (int)(t % d);
-  const int j = (col & 63) >> 1;  // pair within the 64-wide head
-  const double theta = exp2(-(double)(2 * j) / 64.0 * 13.287712379549449);  // log2(10000)
-  double a = (double)(row % m) * theta;
-  a -= 6.283185307179586 * rint(a / 6.283185307179586);
-  float sn, cs;
-  sincosf((float)a, &sn, &cs);
-  sn *= sgn;
+  const float2 cs = tab[(row % m) * 32 + ((col & 63) >> 1)];  // pair within the 64-wide head
+  const float sn = sgn * cs.y;
   uint32_t* q = reinterpret_cast<uint32_t*>(qk + row * ld + col);
   const float2 v = unpack_bf16(*q);
-  *q = pack_bf16(v.x * cs - v.y * sn, v.x * sn + v.y * cs);
+  *q = pack_bf16(v.x * cs.x - v.y * sn, v.x * sn + v.y * cs.x);
 }
 
 __global__ void add_f32_bf16_kernel(const bf16* __restrict__ a, const float* __restrict__ b,
@@ -563,11 +571,16 @@ __global__ void add_f32_bf16_kernel(const bf16* __restrict__ a, const float* __r
 
 }  // namespace
 
-cudaError_t rope_qk(bf16* qk, long ld, int B, int m, int d, bool inverse, cudaStream_t st) {
-  if (d % 64 || ld < 2 * d) return cudaErrorInvalidValue;
+cudaError_t rope_qk(bf16* qk, long ld, int B, int m, int d, float2* tab, bool inverse,
+                    cudaStream_t st) {
+  if (d % 64 || ld < 2 * d || !tab) return cudaErrorInvalidValue;
   const long rows = (long)B * m, n = rows * d;
+  {
+    LaunchTimer lt("rope_table", st, 0.0, 8.0 * m * 32);
+    rope_table_kernel<<<(m * 32 + 255) / 256, 256, 0, st>>>(tab, m);
+  }
   LaunchTimer lt("rope_qk", st, 6.0 * n, 8.0 * n);
-  rope_qk_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(qk, ld, rows, m, d,
+  rope_qk_kernel<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(qk, ld, rows, m, d, tab,
                                                               inverse ? -1.f : 1.f);
   return cudaGetLastError();
 }

@@ -198,8 +198,10 @@ cudaError_t cross_gate_bwd(const bf16* dAg, const bf16* A, const bf16* qa, long 
                            int B, int L, int d, int nh, cudaStream_t st);
 // RoPE on the proxies' queries and keys, in place: rows (b, i) of a [B*m, ld]
 // matrix, columns [0, 2d) = Q | K, pair (2j, 2j+1) of head h turned by the
-// angle i * 10000^(-2j/64) (backwards when inverse).
-cudaError_t rope_qk(bf16* qk, long ld, int B, int m, int d, bool inverse, cudaStream_t st);
+// angle i * 10000^(-2j/64) (backwards when inverse).  tab: scratch of m * 32
+// float2 for the (cos, sin) table.
+cudaError_t rope_qk(bf16* qk, long ld, int B, int m, int d, float2* tab, bool inverse,
+                    cudaStream_t st);
 // out_f = a + b (b may be null), out_b = bf16(out_f), n elements (n % 4 == 0)
 cudaError_t add_f32_bf16(const bf16* a, const float* b, float* out_f, bf16* out_b, long n,
                          cudaStream_t st);
