@@ -110,6 +110,28 @@ def cpu_baseline_subprocess():
                       f"({BASELINE_L // 64} proxies) of the same layer shape, {min(t):.1f} s"}
 
 
+# ------------------------------------------------------------ ranks (N > 1)
+def rank_seed(rank: int) -> int:
+    """Input seed of a rank: every replica draws its own batch (weak scaling)."""
+    return 2 + 1000 * rank
+
+
+def max_over_ranks(x: float, world: int, device: str = "cuda") -> float:
+    """The slowest rank's time: all_reduce(MAX) over the process group."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(tokens_per_rank: float, world: int, ms: float) -> float:
+    """Whole-job tokens/s: every rank's tokens over the slowest rank's step."""
+    return tokens_per_rank * world / (ms / 1e3)
+
+
 def run_reference(args, rank: int):
     if rank != 0:
         return
@@ -534,7 +556,7 @@ def run_ours(args, rank: int, world: int, local_rank: int):
     torch.cuda.set_device(local_rank)
     pf.build()
     spec = workload_spec(args.L)
-    inp = S.make_layer_inputs(spec, 2 + 1000 * rank)
+    inp = S.make_layer_inputs(spec, rank_seed(rank))
     lay = ProxyLayer(spec, inp)
     X = to_device(inp["X"], torch.bfloat16)
     G = to_device(inp["G"], torch.bfloat16)
@@ -588,12 +610,9 @@ def run_ours(args, rank: int, world: int, local_rank: int):
     for v in timing.values():
         v["ms"] *= args.steps / bsteps
         v["launches"] = v["launches"] * args.steps // bsteps
-    if world > 1:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(ms, world)
     tokens_per_step = spec.batch * spec.L * world
-    value = tokens_per_step / (ms / 1e3)
+    value = job_throughput(spec.batch * spec.L, world, ms)
     launches = sum(v["launches"] for v in timing.values())
 
     # ---- end to end: pinned host inputs in, results out, every step.  The
@@ -644,10 +663,7 @@ def run_ours(args, rank: int, world: int, local_rank: int):
     e1.record(stream)
     torch.cuda.synchronize()
     ms_e2e = e0.elapsed_time(e1) / args.e2e_steps
-    if world > 1:
-        t = torch.tensor([ms_e2e], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_e2e = float(t.item())
+    ms_e2e = max_over_ranks(ms_e2e, world)
     pf.pf_sync_check(stream.cuda_stream)
     act_bytes = spec.batch * spec.L * spec.d * 2
     del Xh, Gh, Xoh, dXh, Xd, Gd, Xod, dXd
