@@ -51,6 +51,37 @@ def test_descriptor_validation(pf):
     assert pf.proxy_layer_check(bad) == pf.PF_ERR_INVALID_ARG
 
 
+def test_variant_descriptor_validation(pf):
+    """d_fine, the interaction F, RoPE and the cross injection are accepted
+    exactly where they are built (1D bf16) and rejected elsewhere."""
+    L = dict(batch=1, L=256, n_heads=2, P=16)
+    check = lambda **kw: pf.proxy_layer_check(pf.layer_desc(S.LayerSpec(**{**L, **kw})))
+    assert check(d=128, d_fine=64) == pf.PF_OK
+    assert check(d=128, d_fine=32) == pf.PF_ERR_INVALID_ARG  # not a multiple of 64
+    assert check(d=128, d_fine=64, dtype=S.F32) == pf.PF_ERR_UNSUPPORTED
+    assert check(d=128, d_fine=64, inject=S.INJ_CROSS) == pf.PF_ERR_UNSUPPORTED
+    assert check(d=128, inject=S.INJ_CROSS) == pf.PF_OK
+    assert check(d=128, inject=S.INJ_CROSS, dtype=S.F32) == pf.PF_ERR_UNSUPPORTED
+    assert check(d=128, interact=S.F_MLP) == pf.PF_OK
+    assert check(d=128, interact=S.F_IDENTITY, mode=S.BIDIR_1D) == pf.PF_OK
+    assert check(d=128, interact=3) == pf.PF_ERR_INVALID_ARG
+    assert check(d=128, interact=S.F_MLP, dtype=S.F32) == pf.PF_ERR_UNSUPPORTED
+    assert check(d=128, rope=1) == pf.PF_OK
+    assert check(d=128, rope=1, interact=S.F_MLP) == pf.PF_ERR_INVALID_ARG
+    s2d = S.spec_c5()
+    assert pf.proxy_layer_check(pf.layer_desc(s2d)) == pf.PF_OK
+    for kw in (dict(rope=1), dict(interact=S.F_IDENTITY), dict(d_fine=256)):
+        bad = S.LayerSpec(**{**s2d.__dict__, **kw})
+        assert pf.proxy_layer_check(pf.layer_desc(bad)) == pf.PF_ERR_UNSUPPORTED, kw
+    # saved activations follow the variant: the MLP keeps its hidden layer,
+    # identity drops Q/K/V, the cross injection keeps the token queries
+    size = lambda **kw: pf.proxy_layer_saved_size(pf.layer_desc(S.LayerSpec(**{**L, **kw})))
+    base = size(d=128)
+    assert size(d=128, interact=S.F_IDENTITY) < base < size(d=128, interact=S.F_MLP)
+    assert size(d=128, inject=S.INJ_CROSS) > 0
+    assert size(d=128, d_fine=64) < base  # the decompressed update is d_fine wide
+
+
 def test_sizes_scale_with_shape(pf):
     a = pf.layer_desc(S.LayerSpec(batch=1, L=4096, d=128, n_heads=2, P=16))
     b = pf.layer_desc(S.LayerSpec(batch=2, L=4096, d=128, n_heads=2, P=16))
