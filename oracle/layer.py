@@ -26,6 +26,11 @@ Readings of the paper taken here (each is a descriptor flag of the library):
     (Hbar = H) or a single-proxy MLP Hbar = W_m2 SiLU(W_m1 H + b_m1) + b_m2 of
     hidden width 4d; attention may rotate the proxies' queries and keys by
     their index (RoPE, base 10000, pairs (2j, 2j+1) of each head).
+  * Temporal-distance ratios (Sec. 3.6): a causal sequence split into
+    segments with their own block size (coarse blocks for distant history),
+    each with its own compression / decompression weights; one causal
+    attention over all proxies in time order; a block receives the proxy
+    just before it in time, decompressed by its own segment's weights.
   * Widths: tokens are d_fine wide and proxies d wide (d_fine = d unless the
     spec says otherwise, the asymmetric history stream of the language
     model); both compression levels output d, both decompression levels read d.
@@ -513,6 +518,116 @@ def _bwd_one(spec, prm, X, c, G, dH_out, grads):
     dgroups = dY @ _f64(prm["W_c1"])                          # [m, k2, k1*df]
     dXc = unpartition(dgroups.reshape(m, P, df), spec, L)
     return dX + dXc, dH_in
+
+
+# ------------------------------------------- temporal-distance ratios (Sec. 3.6)
+def _seg_spec(spec, seg):
+    """The single-ratio view of one segment: seg = (L, P) or, with two
+    levels, (L, P, k1, k2)."""
+    import dataclasses
+    L, P = seg[0], seg[1]
+    if spec.levels == 2:
+        return dataclasses.replace(spec, L=L, P=P, k1=seg[2], k2=seg[3])
+    return dataclasses.replace(spec, L=L, P=P, k1=0, k2=0)
+
+
+def layer_fwd_segments(spec, segs, seg_prm, prm, X):
+    """A causal 1D layer whose blocks grow coarser with temporal distance
+    (Sec. 3.6): segs = [(L_s, P_s[, k1_s, k2_s]), ...] in time order (L_s a
+    multiple of P_s except the last), X [sum L_s, d] one sequence.  Segment s compresses its
+    blocks with its own weights seg_prm[s] (W_c1, b_c1[, W_c2, b_c2]); all
+    proxies, in time order, share one causal attention (prm: W_qkv, W_o); the
+    block with global proxy index g receives the interacted proxy g - 1
+    decompressed by its own segment's weights (W_d*, b_d*), block 0 nothing;
+    gated injection with the shared gate vectors in prm.  Returns X_out and
+    the cache ``layer_bwd_segments`` reads."""
+    X = _f64(X)
+    Hs, parts, off = [], [], 0
+    for seg, sp in zip(segs, seg_prm):
+        ss = _seg_spec(spec, seg)
+        Ls = ss.L
+        Xb = partition(X[off:off + Ls], ss)
+        C, Y = compress(Xb, sp, ss)
+        Hs.append(C)
+        parts.append(dict(ss=ss, Xb=Xb, Y=Y, off=off, m=Xb.shape[0]))
+        off += Ls
+    H = np.concatenate(Hs)
+    Hbar, ac = attention(H, prm, spec)                       # causal over all proxies
+    Xo = X.copy()
+    g0 = 0
+    for part, sp in zip(parts, seg_prm):
+        ss, m, o = part["ss"], part["m"], part["off"]
+        src = np.zeros((m, Hbar.shape[1]))                   # proxy g - 1 for block g
+        lo = max(g0 - 1, 0)
+        src[(1 if g0 == 0 else 0):] = Hbar[lo:g0 + m - 1]
+        D, Z = decompress(src, sp, ss)
+        if g0 == 0:
+            D[0] = 0.0                                       # block 0 receives nothing
+        Dt = unpartition(D, ss, ss.L)
+        Xs = X[o:o + ss.L]
+        sg = sigmoid(_f64(prm["w_x"]) * Xs + _f64(prm["w_dlt"]) * Dt + _f64(prm["b_g"]))
+        Xo[o:o + ss.L] = Xs + sg * Dt
+        part.update(src=src, Z=Z, Dt=Dt, sg=sg, g0=g0)
+        g0 += m
+    return Xo, dict(parts=parts, H=H, Hbar=Hbar, **ac)
+
+
+def layer_bwd_segments(spec, segs, seg_prm, prm, X, G):
+    """Backward of ``layer_fwd_segments`` for one sequence: (dX, seg_grads,
+    grads) with the per-segment and shared weight gradients."""
+    X, G = _f64(X), _f64(G)
+    _, c = layer_fwd_segments(spec, segs, seg_prm, prm, X)
+    d = spec.d
+    grads = {k: np.zeros(np.shape(v)) for k, v in prm.items()}
+    sgr = [{k: np.zeros(np.shape(v)) for k, v in sp.items()} for sp in seg_prm]
+    dX = np.zeros_like(X)
+    dHbar = np.zeros_like(c["Hbar"])
+    for part, sp, gr in zip(c["parts"], seg_prm, sgr):
+        ss, m, o, g0 = part["ss"], part["m"], part["off"], part["g0"]
+        Xs, Gs, Dt, sg = X[o:o + ss.L], G[o:o + ss.L], part["Dt"], part["sg"]
+        ds = Gs * Dt * sg * (1.0 - sg)                       # through the gate
+        dX[o:o + ss.L] += Gs + ds * _f64(prm["w_x"])
+        dDt = Gs * sg + ds * _f64(prm["w_dlt"])
+        grads["w_x"] += (ds * Xs).sum(0)
+        grads["w_dlt"] += (ds * Dt).sum(0)
+        grads["b_g"] += ds.sum(0)
+        pad = np.zeros((m * ss.P, d))
+        pad[:ss.L] = dDt
+        dout = pad.reshape(m, ss.k2, ss.k1 * d)
+        if g0 == 0:
+            dout[0] = 0.0                                    # block 0's update was zeroed
+        gr["b_d1"] += dout.sum((0, 1))
+        rows = part["Z"].reshape(m, ss.k2, d) if ss.levels == 2 else part["src"].reshape(m, 1, d)
+        gr["W_d1"] += dout.reshape(m * ss.k2, ss.k1 * d).T @ rows.reshape(m * ss.k2, d)
+        drows = dout @ _f64(sp["W_d1"])
+        if ss.levels == 2:
+            dZ = drows.reshape(m, ss.k2 * d)
+            gr["b_d2"] += dZ.sum(0)
+            gr["W_d2"] += dZ.T @ part["src"]
+            dsrc = dZ @ _f64(sp["W_d2"])
+        else:
+            dsrc = drows.reshape(m, d)
+        lo = max(g0 - 1, 0)
+        dHbar[lo:g0 + m - 1] += dsrc[(1 if g0 == 0 else 0):]
+    cc = dict(Q=c["Q"], K=c["K"], V=c["V"], A=c["A"], Hq=c["H"])
+    dH = interact_bwd(dHbar, cc, prm, spec, grads)
+    g0 = 0
+    for part, sp, gr in zip(c["parts"], seg_prm, sgr):
+        ss, m, o = part["ss"], part["m"], part["off"]
+        dC = dH[g0:g0 + m]
+        if ss.levels == 2:
+            gr["b_c2"] += dC.sum(0)
+            gr["W_c2"] += dC.T @ part["Y"].reshape(m, ss.k2 * d)
+            dY = (dC @ _f64(sp["W_c2"])).reshape(m, ss.k2, d)
+        else:
+            dY = dC.reshape(m, 1, d)
+        gr["b_c1"] += dY.sum((0, 1))
+        groups = part["Xb"].reshape(m, ss.k2, ss.k1 * d)
+        gr["W_c1"] += dY.reshape(m * ss.k2, d).T @ groups.reshape(m * ss.k2, ss.k1 * d)
+        dgroups = dY @ _f64(sp["W_c1"])
+        dX[o:o + ss.L] += unpartition(dgroups.reshape(m, ss.P, d), ss, ss.L)
+        g0 += m
+    return dX, sgr, grads
 
 
 def partition_w(A, spec):

@@ -671,3 +671,97 @@ def test_golden_complexity_ratios():
             _, st = OD.decode_step(spec, prm, st)
         st = OD.kv_append(spec, prm, st)
     assert (2 * P) // int(st["n_proxy"][0]) == g["kv_cache_compression"]
+
+
+# ------------------------------------- temporal-distance ratios (Sec. 3.6)
+_SEG_KEYS = ("W_c1", "b_c1", "W_c2", "b_c2", "W_d1", "b_d1", "W_d2", "b_d2")
+
+
+def _split(prm):
+    seg = {k: v for k, v in prm.items() if k in _SEG_KEYS}
+    shared = {k: v for k, v in prm.items() if k not in _SEG_KEYS and k.startswith(("W_", "w_", "b_"))}
+    return seg, shared
+
+
+@pytest.mark.parametrize("levels", [1, 2])
+def test_segments_one_segment_is_the_layer(levels):
+    """A single segment is the ordinary causal layer, ragged tail included."""
+    kw = dict(k1=2, k2=2) if levels == 2 else {}
+    spec = S.LayerSpec(batch=1, L=22, d=8, n_heads=2, P=4, levels=levels, dtype=S.F32, **kw)
+    inp = S.make_layer_inputs(spec, 71, with_grads=False)
+    prm = {k: v.astype(np.float64) for k, v in inp.items()}
+    seg, shared = _split(prm)
+    segs = [(22, 4, 2, 2)] if levels == 2 else [(22, 4)]
+    Xo, _ = OL.layer_fwd_segments(spec, segs, [seg], shared, prm["X"][0])
+    ref, _ = OL.layer_fwd(spec, prm, prm["X"])
+    np.testing.assert_allclose(Xo, ref[0], rtol=1e-12, atol=1e-12)
+
+
+def test_segments_equal_ratio_split_is_the_layer():
+    """Two segments with the same block size and the same weights are the
+    ordinary layer over their concatenation: the routing across the segment
+    boundary (the first block of segment 2 receives the last proxy of
+    segment 1) and the shared attention must line up exactly."""
+    spec = S.LayerSpec(batch=1, L=30, d=8, n_heads=2, P=4, dtype=S.F32)
+    inp = S.make_layer_inputs(spec, 72, with_grads=False)
+    prm = {k: v.astype(np.float64) for k, v in inp.items()}
+    seg, shared = _split(prm)
+    Xo, _ = OL.layer_fwd_segments(spec, [(12, 4), (18, 4)], [seg, seg], shared, prm["X"][0])
+    ref, _ = OL.layer_fwd(spec, prm, prm["X"])
+    np.testing.assert_allclose(Xo, ref[0], rtol=1e-12, atol=1e-12)
+
+
+def _seg_case():
+    """Coarse blocks (P = 8) for the distant 16 tokens, fine (P = 4) for the
+    recent 14."""
+    specs = [S.LayerSpec(batch=1, L=16, d=8, n_heads=2, P=8, dtype=S.F32),
+             S.LayerSpec(batch=1, L=14, d=8, n_heads=2, P=4, dtype=S.F32)]
+    seg_prm, shared = [], None
+    for i, sp in enumerate(specs):
+        p = {k: v.astype(np.float64) for k, v in S.make_layer_params(sp, 73 + i).items()}
+        sgp, sh = _split(p)
+        seg_prm.append(sgp)
+        shared = shared or sh
+    rng = np.random.default_rng(75)
+    return specs[1], [(16, 8), (14, 4)], seg_prm, shared, rng.standard_normal((30, 8)), \
+        rng.standard_normal((30, 8))
+
+
+def test_segments_causality():
+    """Coarse-then-fine blocks keep causality: perturbing X[t0] leaves every
+    output before the end of t0's block bit-identical except t0 itself."""
+    spec, segs, seg_prm, shared, X, _ = _seg_case()
+    Xo, _ = OL.layer_fwd_segments(spec, segs, seg_prm, shared, X)
+    ends = [8, 16, 20, 24, 28, 30]  # block ends: two P = 8 blocks, then P = 4 blocks
+    for t0 in (3, 12, 17, 29):
+        X2 = X.copy()
+        X2[t0] += 0.5
+        Xo2, _ = OL.layer_fwd_segments(spec, segs, seg_prm, shared, X2)
+        lim = next(e for e in ends if e > t0)
+        same = np.ones(30, bool)
+        same[t0] = False
+        assert (Xo2[:lim][same[:lim]] == Xo[:lim][same[:lim]]).all(), t0
+        if lim < 30:
+            assert np.abs(Xo2[lim:] - Xo[lim:]).max() > 1e-6
+
+
+def test_segments_finite_differences():
+    spec, segs, seg_prm, shared, X, G = _seg_case()
+    dX, sgr, gr = OL.layer_bwd_segments(spec, segs, seg_prm, shared, X, G)
+    loss = lambda: float((OL.layer_fwd_segments(spec, segs, seg_prm, shared, X)[0] * G).sum())
+    rng = np.random.default_rng(76)
+    eps = 1e-6
+    targets = [("X", X, dX)] + [(f"shared {k}", shared[k], gr[k]) for k in shared] + \
+        [(f"seg{i} {k}", seg_prm[i][k], sgr[i][k]) for i in range(2) for k in seg_prm[i]]
+    for name, base, an in targets:
+        flat = base.reshape(-1)
+        for j in rng.choice(flat.size, size=min(8, flat.size), replace=False):
+            old = flat[j]
+            flat[j] = old + eps
+            lp = loss()
+            flat[j] = old - eps
+            lm = loss()
+            flat[j] = old
+            fd = (lp - lm) / (2 * eps)
+            a = an.reshape(-1)[j]
+            assert abs(fd - a) <= 1e-6 * max(1.0, abs(a)), (name, j, fd, a)
