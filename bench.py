@@ -435,6 +435,8 @@ def measure_configs(torch, pf, S, peaks, warmup: int):
         out[key] = config_entry(f"1D causal layer fwd+bwd with {what}, bf16, L=262144 d=1024 "
                                 "16x64 P=64 8x8", sv.L, ms, fl, nb, dom, peaks, 10)
         torch.cuda.empty_cache()
+    out["segments_fwd_bwd"] = measure_segments(torch, pf, S, peaks, warmup)
+    torch.cuda.empty_cache()
     sx = S.spec_cross_layer()
     ms, fl, nb, dom = layer_case(sx, 5, True, 5)
     out["cross_layer_fwd_bwd"] = config_entry(
@@ -471,6 +473,33 @@ def measure_configs(torch, pf, S, peaks, warmup: int):
     del st, X, params
     torch.cuda.empty_cache()
     return out
+
+
+def measure_segments(torch, pf, S, peaks, warmup):
+    """Temporal-distance ratios (Sec. 3.6) on the 262144-token causal layer,
+    d = 1024, 16x64 heads, two levels: the distant 131072 tokens in P = 256
+    blocks, the next 98304 in P = 64, the recent 32768 in P = 16 (4096
+    proxies, as many as uniform P = 64)."""
+    from paper_2608_23463_gb300.segments import ProxySegmentLayer
+    segs = [(131072, 256, 16, 16), (98304, 64, 8, 8), (32768, 16, 4, 4)]
+    try:
+        spec = S.LayerSpec(batch=1, L=262144, d=1024, n_heads=16, P=256, levels=2, k1=16, k2=16)
+        shared, seg_prm = S.make_segment_params(1024, 16, 2, segs, 90)
+        lay = ProxySegmentLayer(spec, segs, shared, seg_prm)
+        g = torch.Generator(device="cuda").manual_seed(91)
+        X = torch.randn(1, spec.L, 1024, device="cuda", generator=g).to(torch.bfloat16)
+        G = torch.randn(1, spec.L, 1024, device="cuda", generator=g).to(torch.bfloat16)
+        Xo, dX = torch.empty_like(X), torch.empty_like(X)
+
+        def step():
+            lay.forward(X, Xo)
+            lay.backward(X, G, dX)
+        ms, fl, nb, dom = timed_steps(torch, pf, step, 5, warmup)
+        return config_entry("1D causal layer fwd+bwd with temporal-distance ratios (P = 256 / 64 / "
+                            "16 from distant to recent), bf16, L=262144 d=1024 16x64 two-level",
+                            spec.L, ms, fl, nb, dom, peaks, 5)
+    except Exception as e:  # reported in the JSON line rather than ending the run
+        return {"error": str(e).splitlines()[0][:200]}
 
 
 def measure_prefill(torch, pf, S, peaks, warmup, specs, params, st, X):

@@ -296,6 +296,46 @@ pf_status proxy_layer_prefill(const pf_layer_desc *desc, const pf_layer_params *
                               const void *X, const float *H_in, void *X_out, float *H_out,
                               pf_kv_cache *cache, void *ws, size_t ws_bytes, void *stream);
 
+/* ---------------------------------------------------------------------------
+ * Temporal-distance ratios (Sec. 3.6): one causal 1D sequence whose blocks
+ * grow coarser with temporal distance.  The sequence is split into n_seg
+ * segments in time order; segment s has L tokens, block size P (and, with
+ * levels == 2, factors k1 * k2 == P) and its own compression / decompression
+ * weights.  The proxies of all segments, in time order, share one causal
+ * attention (Eq. proxy-attn, W_qkv and W_o of the shared parameters); the
+ * block with global proxy index g receives the interacted proxy g - 1
+ * through its own segment's decompression, block 0 nothing; gated (or add)
+ * injection with the shared gate vectors.  One segment is the ordinary
+ * layer.
+ * desc: batch 1, PF_CAUSAL_1D, PF_BF16, PF_INJ_GATED or PF_INJ_ADD,
+ * attention interaction without RoPE, d_fine 0, L = the segments' total;
+ * its P, k1, k2 are not used (give segs[0]'s).  Every segment but the last
+ * has L a multiple of P.  The shared parameters are pf_layer_params' W_qkv,
+ * W_o, w_x, w_dlt, b_g; the gradients land in the same fields of
+ * pf_layer_grads.  Buffers: X, X_out, dX_out, dX [L, d] bf16.                */
+typedef struct { int32_t L, P, k1, k2; } pf_segment;
+typedef struct {
+  const void *W_c1; const float *b_c1; const void *W_c2; const float *b_c2;  /* [d, k1*d] ... */
+  const void *W_d1; const float *b_d1; const void *W_d2; const float *b_d2;  /* [k1*d, d] ... */
+} pf_segment_params;
+typedef struct {
+  float *W_c1, *b_c1, *W_c2, *b_c2, *W_d1, *b_d1, *W_d2, *b_d2;
+} pf_segment_grads;
+
+size_t proxy_segments_saved_size(const pf_layer_desc *desc, int32_t n_seg,
+                                 const pf_segment *segs);
+size_t proxy_segments_workspace_size(const pf_layer_desc *desc, int32_t n_seg,
+                                     const pf_segment *segs, int for_backward);
+pf_status proxy_segments_fwd(const pf_layer_desc *desc, int32_t n_seg, const pf_segment *segs,
+                             const pf_layer_params *shared, const pf_segment_params *seg_params,
+                             const void *X, void *X_out, void *saved, void *ws, size_t ws_bytes,
+                             void *stream);
+pf_status proxy_segments_bwd(const pf_layer_desc *desc, int32_t n_seg, const pf_segment *segs,
+                             const pf_layer_params *shared, const pf_segment_params *seg_params,
+                             const void *X, const void *saved, const void *dX_out, void *dX,
+                             const pf_layer_grads *grads, const pf_segment_grads *seg_grads,
+                             void *ws, size_t ws_bytes, void *stream);
+
 /* Thread-local message describing the last non-OK status of this thread. */
 const char *pf_last_error(void);
 

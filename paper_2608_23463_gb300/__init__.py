@@ -52,6 +52,17 @@ class LayerGrads(ctypes.Structure):
     _fields_ = [(n, _vp) for n in _PARAM_NAMES]
 
 
+class Segment(ctypes.Structure):
+    _fields_ = [(n, _c_i32) for n in ("L", "P", "k1", "k2")]
+
+
+_SEG_NAMES = ("W_c1", "b_c1", "W_c2", "b_c2", "W_d1", "b_d1", "W_d2", "b_d2")
+
+
+class SegmentParams(ctypes.Structure):
+    _fields_ = [(n, _vp) for n in _SEG_NAMES]
+
+
 class DecodeDesc(ctypes.Structure):
     _fields_ = [(n, _c_i32) for n in ("batch", "d", "n_heads", "P", "levels", "k1", "k2",
                                       "capacity")]
@@ -74,6 +85,8 @@ EXPORTED = ("proxy_layer_check", "proxy_layer_saved_size", "proxy_layer_workspac
             "proxy_layer_fwd", "proxy_layer_bwd", "proxy_decode_workspace_size",
             "proxy_decode_step", "proxy_append_workspace_size", "proxy_kv_append",
             "proxy_prefill_workspace_size", "proxy_kv_prefill", "proxy_layer_prefill",
+            "proxy_segments_saved_size", "proxy_segments_workspace_size", "proxy_segments_fwd",
+            "proxy_segments_bwd",
             "pf_last_error", "pf_sync_check", "pf_gemm_bf16", "pf_timing_enable",
             "pf_timing_collect", "pf_timing_label", "pf_timing_ms", "pf_timing_launches",
             "pf_timing_flops", "pf_timing_bytes", "proxy_layer_bwd_noalloc")
@@ -122,6 +135,18 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
                                         P(DecodeParams), _vp, _vp, _vp, _vp, P(KVCache), _vp, sz,
                                         _vp]
     lib.proxy_layer_prefill.restype = ctypes.c_int
+    lib.proxy_segments_saved_size.argtypes = [P(LayerDesc), ctypes.c_int32, P(Segment)]
+    lib.proxy_segments_saved_size.restype = sz
+    lib.proxy_segments_workspace_size.argtypes = [P(LayerDesc), ctypes.c_int32, P(Segment),
+                                                  ctypes.c_int]
+    lib.proxy_segments_workspace_size.restype = sz
+    lib.proxy_segments_fwd.argtypes = [P(LayerDesc), ctypes.c_int32, P(Segment), P(LayerParams),
+                                       P(SegmentParams), _vp, _vp, _vp, _vp, sz, _vp]
+    lib.proxy_segments_fwd.restype = ctypes.c_int
+    lib.proxy_segments_bwd.argtypes = [P(LayerDesc), ctypes.c_int32, P(Segment), P(LayerParams),
+                                       P(SegmentParams), _vp, _vp, _vp, _vp, P(LayerGrads),
+                                       P(SegmentParams), _vp, sz, _vp]
+    lib.proxy_segments_bwd.restype = ctypes.c_int
     lib.pf_last_error.argtypes = []
     lib.pf_last_error.restype = ctypes.c_char_p
     lib.pf_sync_check.argtypes = [_vp]
@@ -245,6 +270,48 @@ def proxy_layer_prefill(desc, params, cdesc, dparams, X, H_in, X_out, H_out, cac
                                       ctypes.byref(cdesc), ctypes.byref(dparams), _ptr(X),
                                       _ptr(H_in), _ptr(X_out), _ptr(H_out), ctypes.byref(cache),
                                       _ptr(ws), int(ws_bytes), stream))
+
+
+def segments(specs) -> "ctypes.Array":
+    """pf_segment array from (L, P[, k1, k2]) tuples."""
+    arr = (Segment * len(specs))()
+    for a, sp in zip(arr, specs):
+        a.L, a.P = int(sp[0]), int(sp[1])
+        a.k1, a.k2 = (int(sp[2]), int(sp[3])) if len(sp) > 2 else (0, 0)
+    return arr
+
+
+def segment_params(tensors_list) -> "ctypes.Array":
+    """pf_segment_params (or pf_segment_grads, same layout) array."""
+    arr = (SegmentParams * len(tensors_list))()
+    for a, t in zip(arr, tensors_list):
+        for n in _SEG_NAMES:
+            setattr(a, n, _ptr(t.get(n)))
+    return arr
+
+
+def proxy_segments_saved_size(desc, segs) -> int:
+    return load().proxy_segments_saved_size(ctypes.byref(desc), len(segs), segs)
+
+
+def proxy_segments_workspace_size(desc, segs, for_backward: int) -> int:
+    return load().proxy_segments_workspace_size(ctypes.byref(desc), len(segs), segs,
+                                                int(for_backward))
+
+
+def proxy_segments_fwd(desc, segs, shared, seg_params, X, X_out, saved, ws, ws_bytes,
+                       stream=None):
+    _check(load().proxy_segments_fwd(ctypes.byref(desc), len(segs), segs, ctypes.byref(shared),
+                                     seg_params, _ptr(X), _ptr(X_out), _ptr(saved), _ptr(ws),
+                                     int(ws_bytes), stream))
+
+
+def proxy_segments_bwd(desc, segs, shared, seg_params, X, saved, dX_out, dX, grads, seg_grads,
+                       ws, ws_bytes, stream=None):
+    _check(load().proxy_segments_bwd(ctypes.byref(desc), len(segs), segs, ctypes.byref(shared),
+                                     seg_params, _ptr(X), _ptr(saved), _ptr(dX_out), _ptr(dX),
+                                     ctypes.byref(grads), seg_grads, _ptr(ws), int(ws_bytes),
+                                     stream))
 
 
 def pf_sync_check(stream=None) -> None:

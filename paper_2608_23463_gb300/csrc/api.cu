@@ -5,6 +5,7 @@
 
 #include <algorithm>
 #include <string>
+#include <array>
 #include <vector>
 
 #include "kernels.h"
@@ -1470,6 +1471,480 @@ pf_status proxy_layer_prefill(const pf_layer_desc* desc, const pf_layer_params* 
                                 d * sizeof(bf16), whole ? B * m : m, cudaMemcpyDeviceToDevice, cs));
     }
   return prefill_open(c, dp, static_cast<const bf16*>(X), s.L, cache, cs);
+}
+
+// ------------------------------------------- temporal-distance ratios (Sec. 3.6)
+namespace {
+
+struct Seg {
+  long L, P, k1, k2, m, off, g0, rows1, N1;
+  bool ragged;
+};
+struct SegPlan {
+  long d, nh, M;
+  int levels;
+  bool gated;
+  std::vector<Seg> s;
+};
+
+pf_status seg_plan(const pf_layer_desc* desc, int32_t n, const pf_segment* segs, SegPlan& p) {
+  pf_status st = check_desc(desc);
+  if (st != PF_OK) return st;
+  const pf_layer_desc& q = *desc;
+  if (q.batch != 1 || q.mode != PF_CAUSAL_1D || q.dtype != PF_BF16 ||
+      (q.inject != PF_INJ_GATED && q.inject != PF_INJ_ADD) || q.interact != PF_F_ATTENTION ||
+      q.rope || (q.d_fine > 0 && q.d_fine != q.d))
+    return fail(PF_ERR_UNSUPPORTED,
+                "segments need batch 1, causal 1D, bf16, gated or add injection, attention");
+  if (n < 1 || segs == nullptr) return fail(PF_ERR_INVALID_ARG, "no segments");
+  p.d = q.d;
+  p.nh = q.n_heads;
+  p.levels = q.levels;
+  p.gated = q.inject == PF_INJ_GATED;
+  p.s.clear();
+  long off = 0, g0 = 0;
+  for (int i = 0; i < n; ++i) {
+    const pf_segment& a = segs[i];
+    if (a.L < 1 || a.P < 1) return fail(PF_ERR_INVALID_ARG, "segment %d: L and P must be >= 1", i);
+    if (q.levels == 2 && (a.k1 < 1 || a.k2 < 1 || (long)a.k1 * a.k2 != a.P))
+      return fail(PF_ERR_INVALID_ARG, "segment %d: levels == 2 needs k1 * k2 == P", i);
+    if (i + 1 < n && a.L % a.P != 0)
+      return fail(PF_ERR_INVALID_ARG, "segment %d: only the last segment may end mid-block", i);
+    Seg g;
+    g.L = a.L;
+    g.P = a.P;
+    g.k1 = q.levels == 2 ? a.k1 : a.P;
+    g.k2 = q.levels == 2 ? a.k2 : 1;
+    g.m = (a.L + a.P - 1) / a.P;
+    g.off = off;
+    g.g0 = g0;
+    g.rows1 = g.m * g.k2;
+    g.N1 = g.k1 * q.d;
+    g.ragged = g.m * g.P != g.L;
+    if (g.N1 > (1L << 30)) return fail(PF_ERR_UNSUPPORTED, "segment %d too large", i);
+    p.s.push_back(g);
+    off += a.L;
+    g0 += g.m;
+  }
+  if (off != q.L) return fail(PF_ERR_INVALID_ARG, "segment lengths sum to %ld, desc L is %d", off, q.L);
+  p.M = g0;
+  return PF_OK;
+}
+
+struct SegSaved {
+  bf16 *Hb, *QKV, *Aatt, *Hbar;
+  float* LSE;
+  std::vector<bf16*> Y, Z, D;
+};
+
+SegSaved carve_seg_saved(Carve& c, const SegPlan& p) {
+  SegSaved v;
+  v.Hb = c.take<bf16>(p.M * p.d);
+  v.QKV = c.take<bf16>(p.M * 3 * p.d);
+  v.Aatt = c.take<bf16>(p.M * p.d);
+  v.Hbar = c.take<bf16>(p.M * p.d);
+  v.LSE = c.take<float>(p.nh * p.M);
+  for (const Seg& g : p.s) {
+    v.Y.push_back(p.levels == 2 ? c.take<bf16>(g.rows1 * p.d) : nullptr);
+    v.Z.push_back(p.levels == 2 ? c.take<bf16>(g.m * g.k2 * p.d) : nullptr);
+    v.D.push_back(c.take<bf16>(g.rows1 * g.N1));
+  }
+  return v;
+}
+
+size_t seg_splitk(const SegPlan& p, bool bwd) {
+  const int d = (int)p.d, M = (int)p.M;
+  std::vector<std::array<int, 3>> v;
+  if (!bwd) v = {{M, 3 * d, d}, {M, d, d}};
+  else v = {{d, d, M}, {M, d, d}, {3 * d, d, M}, {M, d, 3 * d}};
+  for (const Seg& g : p.s) {
+    const int m = (int)g.m, r1 = (int)g.rows1, N1 = (int)g.N1, n2 = (int)(g.k2 * d);
+    if (!bwd) {
+      v.push_back({r1, d, N1});
+      if (p.levels == 2) v.insert(v.end(), {{m, d, n2}, {m, n2, d}});
+    } else {
+      v.insert(v.end(), {{N1, d, r1}, {r1, d, N1}, {d, N1, r1}});
+      if (p.levels == 2) v.insert(v.end(), {{n2, d, m}, {m, d, n2}, {d, n2, m}, {m, n2, d}});
+    }
+  }
+  size_t b = 0;
+  for (const auto& x : v) b = std::max(b, splitk_scratch_bytes(x[0], x[1], x[2]));
+  return b;
+}
+
+struct SegFwdWs {
+  bf16* Xpad;  // the last segment, zero-padded to whole blocks (if ragged)
+  float* sk;
+  size_t skb;
+  SegSaved sv;
+};
+
+SegFwdWs carve_seg_fwd(Carve& wc, const SegPlan& p, void* saved) {
+  SegFwdWs f;
+  const Seg& z = p.s.back();
+  f.Xpad = z.ragged ? wc.take<bf16>(z.m * z.P * p.d) : nullptr;
+  f.skb = seg_splitk(p, false);
+  f.sk = wc.take<float>(f.skb / sizeof(float));
+  Carve sc(saved);
+  f.sv = saved ? carve_seg_saved(sc, p) : carve_seg_saved(wc, p);
+  return f;
+}
+
+struct SegBwdWs {
+  bf16 *Xpad, *dXpad, *dD, *dZ, *dHbar, *dA, *dQKV, *dHb, *dY;
+  float *Di, *dHf, *part, *sk, *gtmp, *gsum;
+  size_t skb;
+};
+
+SegBwdWs carve_seg_bwd(Carve& c, const SegPlan& p) {
+  SegBwdWs w{};
+  const Seg& z = p.s.back();
+  long dD = 0, dZ = 0, dY = 0, pe = 0;
+  for (const Seg& g : p.s) {
+    dD = std::max(dD, g.rows1 * g.N1);
+    dZ = std::max(dZ, g.m * g.k2 * p.d);
+    dY = std::max(dY, g.rows1 * p.d);
+    pe = std::max(pe, (long)inj_bwd_chunks(g.rows1, (int)g.N1) * 4 * g.N1);
+    pe = std::max(pe, colsum_part_elems(g.m, (int)(g.k2 * p.d)));
+    pe = std::max(pe, colsum_part_elems(g.m, (int)p.d));
+    pe = std::max(pe, colsum_part_elems(g.rows1, (int)p.d));
+  }
+  pe = std::max(pe, colsum_part_elems((long)p.s.size(), (int)(3 * p.d)));
+  w.Xpad = z.ragged ? c.take<bf16>(z.m * z.P * p.d) : nullptr;
+  w.dXpad = z.ragged ? c.take<bf16>(z.m * z.P * p.d) : nullptr;
+  w.dD = c.take<bf16>(dD);
+  if (p.levels == 2) w.dZ = c.take<bf16>(dZ);
+  w.dHbar = c.take<bf16>(p.M * p.d);
+  w.dA = c.take<bf16>(p.M * p.d);
+  w.dQKV = c.take<bf16>(p.M * 3 * p.d);
+  w.dHb = c.take<bf16>(p.M * p.d);
+  if (p.levels == 2) w.dY = c.take<bf16>(dY);
+  w.Di = c.take<float>(p.nh * p.M);
+  w.dHf = c.take<float>(p.M * p.d);
+  w.part = c.take<float>(pe);
+  w.skb = seg_splitk(p, true);
+  w.sk = c.take<float>(w.skb / sizeof(float));
+  w.gtmp = c.take<float>((long)p.s.size() * 3 * p.d);
+  w.gsum = c.take<float>(3 * p.d);
+  return w;
+}
+
+bool seg_params_ok(const SegPlan& p, const pf_segment_params* sp) {
+  if (!sp) return false;
+  for (size_t i = 0; i < p.s.size(); ++i) {
+    const pf_segment_params& a = sp[i];
+    if (!a.W_c1 || !a.b_c1 || !a.W_d1 || !a.b_d1 ||
+        (p.levels == 2 && (!a.W_c2 || !a.b_c2 || !a.W_d2 || !a.b_d2)))
+      return false;
+    const void* ptrs[] = {a.W_c1, a.b_c1, a.W_c2, a.b_c2, a.W_d1, a.b_d1, a.W_d2, a.b_d2};
+    for (const void* q : ptrs)
+      if (!aligned16(q)) return false;
+  }
+  return true;
+}
+
+// the source rows of segment i's decompression: proxy g0 - 1 onwards, or for
+// the first segment proxy 0 onwards with the usual one-block routing shift
+const bf16* seg_src(const SegSaved& sv, const SegPlan& p, size_t i) {
+  return i == 0 ? sv.Hbar : sv.Hbar + (p.s[i].g0 - 1) * p.d;
+}
+
+}  // namespace
+
+size_t proxy_segments_saved_size(const pf_layer_desc* desc, int32_t n_seg, const pf_segment* segs) {
+  SegPlan p;
+  if (seg_plan(desc, n_seg, segs, p) != PF_OK) return 0;
+  Carve c(nullptr);
+  carve_seg_saved(c, p);
+  return (c.off + 255) & ~size_t(255);
+}
+
+size_t proxy_segments_workspace_size(const pf_layer_desc* desc, int32_t n_seg,
+                                     const pf_segment* segs, int for_backward) {
+  SegPlan p;
+  if (seg_plan(desc, n_seg, segs, p) != PF_OK) return 0;
+  Carve c(nullptr);
+  if (for_backward)
+    carve_seg_bwd(c, p);
+  else
+    carve_seg_fwd(c, p, nullptr);
+  return ((c.off + 255) & ~size_t(255)) + 256;
+}
+
+pf_status proxy_segments_fwd(const pf_layer_desc* desc, int32_t n_seg, const pf_segment* segs,
+                             const pf_layer_params* prm, const pf_segment_params* sp,
+                             const void* X, void* X_out, void* saved, void* ws, size_t ws_bytes,
+                             void* stream) {
+  SegPlan p;
+  pf_status st = seg_plan(desc, n_seg, segs, p);
+  if (st != PF_OK) return st;
+  if (!prm || !prm->W_qkv || !prm->W_o || (p.gated && (!prm->w_x || !prm->w_dlt || !prm->b_g)) ||
+      !seg_params_ok(p, sp) || !X || !X_out || X == X_out || !params_aligned(*prm) ||
+      !aligned16(X) || !aligned16(X_out) || !aligned16(saved) || !aligned16(ws))
+    return fail(PF_ERR_INVALID_ARG, "a parameter or buffer is NULL, aliased or misaligned");
+  Carve wc(ws);
+  const SegFwdWs f = carve_seg_fwd(wc, p, saved);
+  if (ws == nullptr || wc.off > ws_bytes)
+    return fail(PF_ERR_WORKSPACE, "workspace too small: need %zu bytes, got %zu", wc.off, ws_bytes);
+  cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  const SegSaved& sv = f.sv;
+  const int d = (int)p.d;
+  const bf16* Xb = static_cast<const bf16*>(X);
+  bf16* Xo = static_cast<bf16*>(X_out);
+  // compression, segment by segment, into the proxies' rows g0 .. g0 + m - 1
+  std::vector<const bf16*> xs(p.s.size());
+  for (size_t i = 0; i < p.s.size(); ++i) {
+    const Seg& g = p.s[i];
+    const bf16* Xs = Xb + g.off * d;
+    if (g.ragged) {
+      PF_CUDA(pad_rows(Xs, f.Xpad, 1, g.L, g.m * g.P, d, cs));
+      Xs = f.Xpad;
+    }
+    xs[i] = Xs;
+    const bf16* W_c1 = static_cast<const bf16*>(sp[i].W_c1);
+    EpiLinearArgs e;
+    e.bias = sp[i].b_c1;
+    e.ld_bf16 = d;
+    if (p.levels == 1) {
+      e.out_bf16 = sv.Hb + g.g0 * d;
+      set_gemm_tag("seg_compress_c1", (double)g.m * d * 2.0);
+      PF_CUDA(gemm_linear((int)g.m, d, (int)g.N1, {Xs, g.N1, 0}, {W_c1, g.N1, 0},
+                          with_sk(e, f.sk, f.skb), cs));
+    } else {
+      const int n2 = (int)(g.k2 * d);
+      e.out_bf16 = sv.Y[i];
+      set_gemm_tag("seg_compress_c1", (double)g.rows1 * d * 2.0);
+      PF_CUDA(gemm_linear((int)g.rows1, d, (int)g.N1, {Xs, g.N1, 0}, {W_c1, g.N1, 0},
+                          with_sk(e, f.sk, f.skb), cs));
+      EpiLinearArgs e2;
+      e2.bias = sp[i].b_c2;
+      e2.out_bf16 = sv.Hb + g.g0 * d;
+      e2.ld_bf16 = d;
+      set_gemm_tag("seg_compress_c2", (double)g.m * d * 2.0);
+      PF_CUDA(gemm_linear((int)g.m, d, n2, {sv.Y[i], n2, 0},
+                          {static_cast<const bf16*>(sp[i].W_c2), n2, 0}, with_sk(e2, f.sk, f.skb),
+                          cs));
+    }
+  }
+  // one causal attention over all proxies in time order (Eq. proxy-attn)
+  {
+    EpiLinearArgs e;
+    e.out_bf16 = sv.QKV;
+    e.ld_bf16 = 3 * d;
+    set_gemm_tag("proxy_qkv", (double)p.M * 3 * d * 2.0);
+    PF_CUDA(gemm_linear((int)p.M, 3 * d, d, {sv.Hb, d, 0},
+                        {static_cast<const bf16*>(prm->W_qkv), d, 0}, with_sk(e, f.sk, f.skb), cs));
+    PF_CUDA(attn_fwd(sv.QKV, sv.Aatt, sv.LSE, 1, (int)p.M, d, (int)p.nh, true, cs));
+    EpiLinearArgs eo;
+    eo.out_bf16 = sv.Hbar;
+    eo.ld_bf16 = d;
+    set_gemm_tag("proxy_o", (double)p.M * d * 2.0);
+    PF_CUDA(gemm_linear((int)p.M, d, d, {sv.Aatt, d, 0}, {static_cast<const bf16*>(prm->W_o), d, 0},
+                        with_sk(eo, f.sk, f.skb), cs));
+  }
+  // decompression and injection, each block through its own segment's weights
+  for (size_t i = 0; i < p.s.size(); ++i) {
+    const Seg& g = p.s[i];
+    const bf16* src = seg_src(sv, p, i);
+    const bf16* Zsrc = src;
+    if (p.levels == 2) {
+      const int n2 = (int)(g.k2 * d);
+      EpiLinearArgs e;
+      e.bias = sp[i].b_d2;
+      e.out_bf16 = sv.Z[i];
+      e.ld_bf16 = n2;
+      set_gemm_tag("seg_decompress_d2", (double)g.m * n2 * 2.0);
+      PF_CUDA(gemm_linear((int)g.m, n2, d, {src, d, 0}, {static_cast<const bf16*>(sp[i].W_d2), d, 0},
+                          with_sk(e, f.sk, f.skb), cs));
+      Zsrc = sv.Z[i];
+    }
+    EpiInjectArgs e{sp[i].b_d1, sv.D[i], xs[i], Xo + g.off * d, prm->w_x, prm->w_dlt, prm->b_g,
+                    d, (int)g.k1, (int)g.k2, (int)g.m, (int)g.L, i == 0 ? 1 : 0, p.gated ? 1 : 0};
+    set_gemm_tag("seg_decompress_d1_inject", (double)g.rows1 * g.N1 * 8.0);
+    PF_CUDA(gemm_inject1d((int)g.rows1, (int)g.N1, d, {Zsrc, d, 0},
+                          {static_cast<const bf16*>(sp[i].W_d1), d, 0}, e, cs));
+  }
+  const Seg& g0 = p.s.front();
+  PF_CUDA(copy_block0(Xb, g0.L, Xo, g0.L, 1, d, (int)std::min(g0.P, g0.L), cs));
+  return PF_OK;
+}
+
+pf_status proxy_segments_bwd(const pf_layer_desc* desc, int32_t n_seg, const pf_segment* segs,
+                             const pf_layer_params* prm, const pf_segment_params* sp,
+                             const void* X, const void* saved, const void* dX_out, void* dX,
+                             const pf_layer_grads* grads, const pf_segment_grads* sg, void* ws,
+                             size_t ws_bytes, void* stream) {
+  SegPlan p;
+  pf_status st = seg_plan(desc, n_seg, segs, p);
+  if (st != PF_OK) return st;
+  if (!prm || !prm->W_qkv || !prm->W_o || (p.gated && (!prm->w_x || !prm->w_dlt || !prm->b_g)) ||
+      !seg_params_ok(p, sp) || !X || !saved || !dX_out || !dX || !grads || !sg ||
+      !params_aligned(*prm) || !aligned16(X) || !aligned16(saved) || !aligned16(dX_out) ||
+      !aligned16(dX) || !aligned16(ws))
+    return fail(PF_ERR_INVALID_ARG, "a parameter or buffer is NULL or misaligned");
+  for (size_t i = 0; i < p.s.size(); ++i)
+    if (!sg[i].b_d1) return fail(PF_ERR_INVALID_ARG, "seg_grads[%zu].b_d1 must be given", i);
+  Carve wc(ws);
+  const SegBwdWs w = carve_seg_bwd(wc, p);
+  if (ws == nullptr || wc.off > ws_bytes)
+    return fail(PF_ERR_WORKSPACE, "workspace too small: need %zu bytes, got %zu", wc.off, ws_bytes);
+  Carve sc(const_cast<void*>(saved));
+  const SegSaved sv = carve_seg_saved(sc, p);
+  cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  const int d = (int)p.d;
+  const bf16* Xb = static_cast<const bf16*>(X);
+  const bf16* G = static_cast<const bf16*>(dX_out);
+  bf16* dXb = static_cast<bf16*>(dX);
+  const bf16* W_qkv = static_cast<const bf16*>(prm->W_qkv);
+  const bf16* W_o = static_cast<const bf16*>(prm->W_o);
+  // the last proxy feeds no block
+  PF_CUDA(cudaMemsetAsync(w.dHbar + (p.M - 1) * d, 0, d * sizeof(bf16), cs));
+  if (p.gated) PF_CUDA(cudaMemsetAsync(w.gtmp, 0, p.s.size() * 3 * d * sizeof(float), cs));
+  std::vector<const bf16*> xs(p.s.size());
+  std::vector<bf16*> dxd(p.s.size());
+  // injection and decompression backward, segment by segment (segment 0 first:
+  // its last proxy row, which feeds no block of its own, is overwritten by
+  // segment 1's first source row)
+  for (size_t i = 0; i < p.s.size(); ++i) {
+    const Seg& g = p.s[i];
+    const bf16* Xs = Xb + g.off * d;
+    xs[i] = Xs;
+    dxd[i] = dXb + g.off * d;
+    if (g.ragged) {
+      PF_CUDA(pad_rows(Xs, w.Xpad, 1, g.L, g.m * g.P, d, cs));
+      xs[i] = w.Xpad;
+      dxd[i] = w.dXpad;
+    }
+    const int N1 = (int)g.N1, r1 = (int)g.rows1;
+    const int nch = inj_bwd_chunks(g.rows1, N1);
+    InjBwdArgs a{G + g.off * d, Xs, sv.D[i], w.dD, dxd[i], g.ragged ? g.m * g.P : g.L, prm->w_x,
+                 prm->w_dlt, prm->b_g, d, (int)g.k1, (int)g.k2, (int)g.m, (int)g.L, 1,
+                 i == 0 ? 1 : 0, p.gated ? 1 : 0};
+    PF_CUDA(inj_bwd_1d(a, w.part, nch, cs));
+    if (i == 0)
+      PF_CUDA(copy_block0(G, g.L, dxd[0], g.ragged ? g.m * g.P : g.L, 1, d,
+                          (int)std::min(g.P, g.L), cs));
+    float* gt = w.gtmp + i * 3 * d;
+    PF_CUDA(inj_bwd_finalize(w.part, nch, N1, d, sg[i].b_d1, p.gated ? gt : nullptr,
+                             p.gated ? gt + d : nullptr, p.gated ? gt + 2 * d : nullptr, cs));
+    const bf16* src = seg_src(sv, p, i);
+    bf16* dsrc = w.dHbar + (i == 0 ? 0 : (g.g0 - 1)) * d;
+    const bf16* Zsrc = p.levels == 2 ? sv.Z[i] : src;
+    if (sg[i].W_d1) {
+      EpiLinearArgs e;
+      e.out_f32 = sg[i].W_d1;
+      e.ld_f32 = d;
+      set_gemm_tag("seg_bwd_dW_d1", (double)N1 * d * 4.0);
+      PF_CUDA(gemm_linear(N1, d, r1, {w.dD, N1, 1}, {Zsrc, d, 1}, with_sk(e, w.sk, w.skb), cs));
+    }
+    EpiLinearArgs e;
+    e.out_bf16 = p.levels == 2 ? w.dZ : dsrc;
+    e.ld_bf16 = d;
+    set_gemm_tag("seg_bwd_dZ", (double)r1 * d * 2.0);
+    PF_CUDA(gemm_linear(r1, d, N1, {w.dD, N1, 0}, {static_cast<const bf16*>(sp[i].W_d1), d, 1},
+                        with_sk(e, w.sk, w.skb), cs));
+    if (p.levels == 2) {
+      const int n2 = (int)(g.k2 * d), m = (int)g.m;
+      if (sg[i].b_d2) PF_CUDA(colsum_bf16(w.dZ, g.m, n2, sg[i].b_d2, w.part, cs));
+      if (sg[i].W_d2) {
+        EpiLinearArgs e2;
+        e2.out_f32 = sg[i].W_d2;
+        e2.ld_f32 = d;
+        set_gemm_tag("seg_bwd_dW_d2", (double)n2 * d * 4.0);
+        PF_CUDA(gemm_linear(n2, d, m, {w.dZ, n2, 1}, {src, d, 1}, with_sk(e2, w.sk, w.skb), cs));
+      }
+      EpiLinearArgs e3;
+      e3.out_bf16 = dsrc;
+      e3.ld_bf16 = d;
+      set_gemm_tag("seg_bwd_dHbar", (double)m * d * 2.0);
+      PF_CUDA(gemm_linear(m, d, n2, {w.dZ, n2, 0}, {static_cast<const bf16*>(sp[i].W_d2), d, 1},
+                          with_sk(e3, w.sk, w.skb), cs));
+    }
+  }
+  if (p.gated) {  // the gate vectors are shared: sum the segments' contributions
+    PF_CUDA(colsum_f32(w.gtmp, (long)p.s.size(), 3 * d, w.gsum, w.part, cs));
+    float* dst[3] = {grads->w_x, grads->w_dlt, grads->b_g};
+    for (int k = 0; k < 3; ++k)
+      if (dst[k])
+        PF_CUDA(cudaMemcpyAsync(dst[k], w.gsum + k * d, d * sizeof(float),
+                                cudaMemcpyDeviceToDevice, cs));
+  }
+  // the shared attention
+  if (grads->W_o) {
+    EpiLinearArgs e;
+    e.out_f32 = grads->W_o;
+    e.ld_f32 = d;
+    set_gemm_tag("bwd_dW_o", (double)d * d * 4.0);
+    PF_CUDA(gemm_linear(d, d, (int)p.M, {w.dHbar, d, 1}, {sv.Aatt, d, 1}, with_sk(e, w.sk, w.skb), cs));
+  }
+  {
+    EpiLinearArgs e;
+    e.out_bf16 = w.dA;
+    e.ld_bf16 = d;
+    set_gemm_tag("bwd_dA", (double)p.M * d * 2.0);
+    PF_CUDA(gemm_linear((int)p.M, d, d, {w.dHbar, d, 0}, {W_o, d, 1}, with_sk(e, w.sk, w.skb), cs));
+  }
+  PF_CUDA(attn_bwd(sv.QKV, sv.Aatt, w.dA, sv.LSE, w.Di, w.dQKV, 1, (int)p.M, d, (int)p.nh, true,
+                   cs));
+  if (grads->W_qkv) {
+    EpiLinearArgs e;
+    e.out_f32 = grads->W_qkv;
+    e.ld_f32 = d;
+    set_gemm_tag("bwd_dW_qkv", (double)3 * d * d * 4.0);
+    PF_CUDA(gemm_linear(3 * d, d, (int)p.M, {w.dQKV, 3 * d, 1}, {sv.Hb, d, 1},
+                        with_sk(e, w.sk, w.skb), cs));
+  }
+  {
+    EpiLinearArgs e;
+    e.out_f32 = w.dHf;
+    e.ld_f32 = d;
+    e.out_bf16 = w.dHb;
+    e.ld_bf16 = d;
+    set_gemm_tag("bwd_dH", (double)p.M * d * 10.0);
+    PF_CUDA(gemm_linear((int)p.M, d, 3 * d, {w.dQKV, 3 * d, 0}, {W_qkv, d, 1},
+                        with_sk(e, w.sk, w.skb), cs));
+  }
+  // compression backward and dX, segment by segment
+  for (size_t i = 0; i < p.s.size(); ++i) {
+    const Seg& g = p.s[i];
+    const int N1 = (int)g.N1, r1 = (int)g.rows1, m = (int)g.m;
+    const bf16* dHb = w.dHb + g.g0 * d;
+    const float* dHf = w.dHf + g.g0 * d;
+    const bf16* dYsrc = dHb;
+    if (p.levels == 2) {
+      const int n2 = (int)(g.k2 * d);
+      if (sg[i].b_c2) PF_CUDA(colsum_f32(dHf, g.m, d, sg[i].b_c2, w.part, cs));
+      if (sg[i].W_c2) {
+        EpiLinearArgs e;
+        e.out_f32 = sg[i].W_c2;
+        e.ld_f32 = n2;
+        set_gemm_tag("seg_bwd_dW_c2", (double)d * n2 * 4.0);
+        PF_CUDA(gemm_linear(d, n2, m, {dHb, d, 1}, {sv.Y[i], n2, 1}, with_sk(e, w.sk, w.skb), cs));
+      }
+      EpiLinearArgs e;
+      e.out_bf16 = w.dY;
+      e.ld_bf16 = n2;
+      set_gemm_tag("seg_bwd_dY", (double)m * n2 * 2.0);
+      PF_CUDA(gemm_linear(m, n2, d, {dHb, d, 0}, {static_cast<const bf16*>(sp[i].W_c2), n2, 1},
+                          with_sk(e, w.sk, w.skb), cs));
+      if (sg[i].b_c1) PF_CUDA(colsum_bf16(w.dY, g.rows1, d, sg[i].b_c1, w.part, cs));
+      dYsrc = w.dY;
+    } else if (sg[i].b_c1) {
+      PF_CUDA(colsum_f32(dHf, g.m, d, sg[i].b_c1, w.part, cs));
+    }
+    if (sg[i].W_c1) {
+      EpiLinearArgs e;
+      e.out_f32 = sg[i].W_c1;
+      e.ld_f32 = N1;
+      set_gemm_tag("seg_bwd_dW_c1", (double)d * N1 * 4.0);
+      PF_CUDA(gemm_linear(d, N1, r1, {dYsrc, d, 1}, {xs[i], N1, 1}, with_sk(e, w.sk, w.skb), cs));
+    }
+    EpiDXArgs e{dxd[i], dXb + g.off * d, d, (int)g.k1, (int)g.k2, (int)g.m, (int)g.L};
+    set_gemm_tag("seg_bwd_dX", (double)r1 * N1 * 4.0);
+    PF_CUDA(gemm_dx1d(r1, N1, d, {dYsrc, d, 0}, {static_cast<const bf16*>(sp[i].W_c1), N1, 1}, e,
+                      cs));
+  }
+  return PF_OK;
 }
 
 pf_status pf_sync_check(void* stream) {

@@ -305,6 +305,24 @@ def spec_lm_history():
     return LayerSpec(batch=1, L=1048576, d=512, n_heads=8, P=64, d_fine=64)
 
 
+SEGMENT_KEYS = ("W_c1", "b_c1", "W_c2", "b_c2", "W_d1", "b_d1", "W_d2", "b_d2")
+
+
+def make_segment_params(d: int, n_heads: int, levels: int, segs, seed: int):
+    """Parameters of a layer with temporal-distance ratios: the shared ones
+    (proxy attention and gate: W_qkv, W_o, w_x, w_dlt, b_g) and one set of
+    compression / decompression weights per segment (L, P[, k1, k2])."""
+    shared, per = None, []
+    for i, sg in enumerate(segs):
+        kw = dict(k1=sg[2], k2=sg[3]) if levels == 2 else {}
+        sp = LayerSpec(batch=1, L=sg[0], d=d, n_heads=n_heads, P=sg[1], levels=levels, **kw)
+        p = make_layer_params(sp, seed + i)
+        per.append({k: v for k, v in p.items() if k in SEGMENT_KEYS})
+        if shared is None:
+            shared = {k: v for k, v in p.items() if k not in SEGMENT_KEYS}
+    return shared, per
+
+
 C3_RATIOS = (16, 16, 32, 32, 64, 64, 64, 64, 128, 128, 256, 256)
 
 

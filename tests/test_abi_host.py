@@ -153,3 +153,26 @@ def test_prefill_rejects_bad_arguments_before_any_launch(pf):
         pf.proxy_kv_prefill(mk(ok), ap, dp, 4096, -1, None, cache, 4096, 1 << 30)
     assert e.value.status == pf.PF_ERR_INVALID_ARG
     assert pf.proxy_prefill_workspace_size(mk(ok), 100) > pf.proxy_prefill_workspace_size(mk(ok), 0)
+
+
+def test_segments_plan_checks(pf):
+    """Temporal-distance ratios: the segments must tile L, only the last may
+    end mid-block, two levels need k1 * k2 == P per segment, and the layer
+    must be batch 1, causal, bf16."""
+    spec = S.LayerSpec(batch=1, L=300, d=128, n_heads=2, P=32)
+    desc = pf.layer_desc(spec)
+    ok = pf.segments([(256, 32), (44, 8)])
+    assert pf.proxy_segments_saved_size(desc, ok) > 0
+    assert pf.proxy_segments_workspace_size(desc, ok, 1) > 0
+    assert pf.proxy_segments_saved_size(desc, pf.segments([(256, 32), (40, 8)])) == 0  # sum != L
+    assert pf.proxy_segments_saved_size(desc, pf.segments([(250, 32), (50, 8)])) == 0  # mid-block
+    two = pf.layer_desc(S.LayerSpec(batch=1, L=300, d=128, n_heads=2, P=32, levels=2, k1=8, k2=4))
+    assert pf.proxy_segments_saved_size(two, pf.segments([(256, 32, 8, 4), (44, 8, 4, 2)])) > 0
+    assert pf.proxy_segments_saved_size(two, pf.segments([(256, 32, 8, 8), (44, 8, 4, 2)])) == 0
+    b2 = pf.layer_desc(S.LayerSpec(batch=2, L=300, d=128, n_heads=2, P=32))
+    assert pf.proxy_segments_saved_size(b2, ok) == 0
+    shared = pf.layer_params({})
+    sp = pf.segment_params([{}, {}])
+    with pytest.raises(pf.ProxyFormerError) as e:  # parameters missing: rejected on the host
+        pf.proxy_segments_fwd(desc, ok, shared, sp, 4096, 8192, None, 4096, 1 << 30)
+    assert e.value.status == pf.PF_ERR_INVALID_ARG
