@@ -272,7 +272,7 @@ def proxy_layer_prefill(desc, params, cdesc, dparams, X, H_in, X_out, H_out, cac
                                       _ptr(ws), int(ws_bytes), stream))
 
 
-def segments(specs) -> "ctypes.Array":
+def segment_array(specs) -> "ctypes.Array":
     """pf_segment array from (L, P[, k1, k2]) tuples."""
     arr = (Segment * len(specs))()
     for a, sp in zip(arr, specs):

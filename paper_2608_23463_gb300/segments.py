@@ -13,7 +13,8 @@ import numpy as np
 import torch
 
 from . import (layer_desc, layer_params, proxy_segments_bwd, proxy_segments_fwd,
-               proxy_segments_saved_size, proxy_segments_workspace_size, segment_params, segments)
+               proxy_segments_saved_size, proxy_segments_workspace_size, segment_array,
+               segment_params)
 
 
 def _dev(a, device):
@@ -26,7 +27,7 @@ class ProxySegmentLayer:
                  seg_params: List[Dict[str, np.ndarray]], device="cuda"):
         self.spec, self.device = spec, device
         self.desc = layer_desc(spec)
-        self.segs = segments(segs)
+        self.segs = segment_array(segs)
         self.p = {k: _dev(v, device) for k, v in shared.items()}
         self.sp = [{k: _dev(v, device) for k, v in d.items()} for d in seg_params]
         self.p_struct = layer_params(self.p)

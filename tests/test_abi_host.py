@@ -161,14 +161,14 @@ def test_segments_plan_checks(pf):
     must be batch 1, causal, bf16."""
     spec = S.LayerSpec(batch=1, L=300, d=128, n_heads=2, P=32)
     desc = pf.layer_desc(spec)
-    ok = pf.segments([(256, 32), (44, 8)])
+    ok = pf.segment_array([(256, 32), (44, 8)])
     assert pf.proxy_segments_saved_size(desc, ok) > 0
     assert pf.proxy_segments_workspace_size(desc, ok, 1) > 0
-    assert pf.proxy_segments_saved_size(desc, pf.segments([(256, 32), (40, 8)])) == 0  # sum != L
-    assert pf.proxy_segments_saved_size(desc, pf.segments([(250, 32), (50, 8)])) == 0  # mid-block
+    assert pf.proxy_segments_saved_size(desc, pf.segment_array([(256, 32), (40, 8)])) == 0  # sum != L
+    assert pf.proxy_segments_saved_size(desc, pf.segment_array([(250, 32), (50, 8)])) == 0  # mid-block
     two = pf.layer_desc(S.LayerSpec(batch=1, L=300, d=128, n_heads=2, P=32, levels=2, k1=8, k2=4))
-    assert pf.proxy_segments_saved_size(two, pf.segments([(256, 32, 8, 4), (44, 8, 4, 2)])) > 0
-    assert pf.proxy_segments_saved_size(two, pf.segments([(256, 32, 8, 8), (44, 8, 4, 2)])) == 0
+    assert pf.proxy_segments_saved_size(two, pf.segment_array([(256, 32, 8, 4), (44, 8, 4, 2)])) > 0
+    assert pf.proxy_segments_saved_size(two, pf.segment_array([(256, 32, 8, 8), (44, 8, 4, 2)])) == 0
     b2 = pf.layer_desc(S.LayerSpec(batch=2, L=300, d=128, n_heads=2, P=32))
     assert pf.proxy_segments_saved_size(b2, ok) == 0
     shared = pf.layer_params({})
