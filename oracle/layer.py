@@ -254,9 +254,22 @@ def attention_bwd(dA, c, spec):
 
 
 # ------------------------------------------------- cross-attention injection
-def _cross_visible(t, spec, m):
-    """Proxies token t may read: those of earlier blocks (causal), else all."""
-    return t // spec.P if spec.mode == CAUSAL_1D else m
+def _cross_visible(L, m, spec):
+    """[L, m] mask of the proxies each token may read: those of earlier
+    blocks (causal, proxy j < t // P), else all."""
+    if spec.mode == CAUSAL_1D:
+        return np.arange(m)[None, :] < (np.arange(L) // spec.P)[:, None]
+    return np.ones((L, m), dtype=bool)
+
+
+def _cross_probs(Qh, Kh, vis, scale):
+    """Row-wise softmax of the scores Q K^T * scale over the visible
+    proxies (the row maximum subtracted); a row that sees none is zero."""
+    S = np.where(vis, (Qh @ Kh.T) * scale, -np.inf)
+    mx = np.where(vis.any(1), S.max(1, initial=-np.inf), 0.0)
+    E = np.where(vis, np.exp(S - mx[:, None]), 0.0)
+    l = E.sum(1)
+    return E / np.where(l > 0, l, 1.0)[:, None]
 
 
 def cross_inject(X, Hbar, prm, spec):
@@ -273,12 +286,10 @@ def cross_inject(X, Hbar, prm, spec):
     K, V = Hbar @ Wkv[:d].T, Hbar @ Wkv[d:].T
     A = np.zeros((L, d))
     scale = 1.0 / math.sqrt(dh)
+    vis = _cross_visible(L, m, spec)
     for h in range(nh):
         cs = slice(h * dh, (h + 1) * dh)
-        for t in range(L):
-            n_vis = _cross_visible(t, spec, m)
-            if n_vis:
-                A[t, cs] = _row_probs(Q[t, cs], K[:, cs], n_vis, scale) @ V[:n_vis, cs]
+        A[:, cs] = _cross_probs(Q[:, cs], K[:, cs], vis, scale) @ V[:, cs]
     Ag = A * np.repeat(alpha, dh, axis=1)
     Xo = X + Ag @ _f64(prm["W_ox"]).T
     return Xo, dict(Qx=Q, Kx=K, Vx=V, Ax=A, alpha=alpha, Ag=Ag)
@@ -298,19 +309,16 @@ def cross_inject_bwd(G, X, Hbar, c, prm, spec, grads):
     da = s * alpha * (1.0 - alpha)                                # through the sigmoid
     dA = dAg * np.repeat(alpha, dh, axis=1)
     dQ, dK, dV = np.zeros_like(Q), np.zeros_like(K), np.zeros_like(V)
-    for h in range(nh):
-        cs = slice(h * dh, (h + 1) * dh)
-        for t in range(L):
-            n_vis = _cross_visible(t, spec, m)
-            if not n_vis:
-                continue
-            p = _row_probs(Q[t, cs], K[:, cs], n_vis, scale)
-            dO = dA[t, cs]
-            dV[:n_vis, cs] += np.outer(p, dO)
-            dp = V[:n_vis, cs] @ dO
-            dS = p * (dp - p @ dp)
-            dQ[t, cs] = scale * (dS @ K[:n_vis, cs])
-            dK[:n_vis, cs] += scale * np.outer(dS, Q[t, cs])
+    vis = _cross_visible(L, m, spec)
+    for h in range(nh):     # with p the probabilities of each row: dV = p^T dO,
+        cs = slice(h * dh, (h + 1) * dh)        # dS = p * (dp - <p, dp>), dp = dO V^T
+        p = _cross_probs(Q[:, cs], K[:, cs], vis, scale)
+        dO = dA[:, cs]
+        dV[:, cs] = p.T @ dO
+        dp = dO @ V[:, cs].T
+        dS = p * (dp - (p * dp).sum(1, keepdims=True))
+        dQ[:, cs] = scale * (dS @ K[:, cs])
+        dK[:, cs] = scale * (dS.T @ Q[:, cs])
     dQA = np.concatenate([dQ, da], axis=1)
     Wqa, Wkv = _f64(prm["W_qa"]), _f64(prm["W_kvx"])
     grads["W_qa"] += dQA.T @ X
