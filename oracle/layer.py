@@ -134,12 +134,21 @@ def decompress(Hbar, prm, spec):
 
 
 # ---------------------------------------------------------------- attention
-def _row_probs(q, Kh, n_vis, scale):
-    """Softmax of one query row over its visible keys 0..n_vis-1 (the mask M
-    of Eq. proxy-attn removes the rest), with the row maximum subtracted."""
-    s = (Kh[:n_vis] @ q) * scale
-    e = np.exp(s - s.max())
-    return e / e.sum()
+def proxy_mask(m, spec):
+    """The mask M of Eq. proxy-attn as a boolean [m, m] matrix of visible
+    (query, key) pairs: proxy i sees j <= i in the autoregressive 1D mode and
+    every proxy otherwise."""
+    if spec.mode == CAUSAL_1D:
+        return np.tril(np.ones((m, m), dtype=bool))
+    return np.ones((m, m), dtype=bool)
+
+
+def _probs(Qh, Kh, vis, scale):
+    """softmax(Q K^T * scale + M) row by row, M = -inf where ``vis`` is
+    False, with each row's maximum subtracted (every row sees its own key)."""
+    S = np.where(vis, (Qh @ Kh.T) * scale, -np.inf)
+    E = np.exp(S - S.max(1, keepdims=True))
+    return E / E.sum(1, keepdims=True)
 
 
 def rope(Z, nh, inverse=False):
@@ -205,9 +214,9 @@ def interact_bwd(dHbar, c, prm, spec, grads):
 def attention(Hq, prm, spec):
     """Eq. proxy-attn: Hbar = softmax(Q K^T / sqrt(dh) + M) V per head, then
     the output projection.  M is the causal mask (proxy i sees j <= i) for the
-    autoregressive 1D mode and zero otherwise.  Evaluated one query row at a
-    time over the visible keys only.  With RoPE, Q and K are rotated by the
-    proxy index first."""
+    autoregressive 1D mode and zero otherwise; each head's m x m probability
+    matrix is formed whole.  With RoPE, Q and K are rotated by the proxy index
+    first."""
     m, d = Hq.shape
     nh, dh = spec.n_heads, d // spec.n_heads
     W = _f64(prm["W_qkv"])
@@ -216,40 +225,33 @@ def attention(Hq, prm, spec):
         Q, K = rope(Q, nh), rope(K, nh)
     A = np.zeros((m, d))
     scale = 1.0 / math.sqrt(dh)
-    causal = spec.mode == CAUSAL_1D
+    vis = proxy_mask(m, spec)
     for h in range(nh):
         cs = slice(h * dh, (h + 1) * dh)
-        Qh, Kh, Vh = Q[:, cs], K[:, cs], V[:, cs]
-        for i in range(m):
-            n_vis = i + 1 if causal else m
-            A[i, cs] = _row_probs(Qh[i], Kh, n_vis, scale) @ Vh[:n_vis]
+        A[:, cs] = _probs(Q[:, cs], K[:, cs], vis, scale) @ V[:, cs]
     Hbar = A @ _f64(prm["W_o"]).T
     return Hbar, dict(Q=Q, K=K, V=V, A=A)
 
 
 def attention_bwd(dA, c, spec):
-    """Backward of the attention core, row by row: with p the probabilities of
-    row i, dV += p^T dO_i, dp = V dO_i, dS = p * (dp - <p, dp>),
-    dQ_i = scale dS K, dK += scale dS^T Q_i."""
+    """Backward of the attention core per head: with P the probability
+    matrix, dV = P^T dO, dP = dO V^T, dS = P * (dP - rowsum(P * dP)),
+    dQ = scale dS K, dK = scale dS^T Q."""
     Q, K, V = c["Q"], c["K"], c["V"]
     m, d = Q.shape
     nh, dh = spec.n_heads, d // spec.n_heads
     scale = 1.0 / math.sqrt(dh)
-    causal = spec.mode == CAUSAL_1D
+    vis = proxy_mask(m, spec)
     dQ, dK, dV = np.zeros_like(Q), np.zeros_like(K), np.zeros_like(V)
     for h in range(nh):
         cs = slice(h * dh, (h + 1) * dh)
-        Qh, Kh, Vh = Q[:, cs], K[:, cs], V[:, cs]
-        dQh, dKh, dVh = dQ[:, cs], dK[:, cs], dV[:, cs]
-        for i in range(m):
-            n_vis = i + 1 if causal else m
-            p = _row_probs(Qh[i], Kh, n_vis, scale)
-            dO = dA[i, cs]
-            dVh[:n_vis] += np.outer(p, dO)
-            dp = Vh[:n_vis] @ dO
-            dS = p * (dp - p @ dp)
-            dQh[i] = scale * (dS @ Kh[:n_vis])
-            dKh[:n_vis] += scale * np.outer(dS, Qh[i])
+        Pm = _probs(Q[:, cs], K[:, cs], vis, scale)
+        dO = dA[:, cs]
+        dV[:, cs] = Pm.T @ dO
+        dP = dO @ V[:, cs].T
+        dS = Pm * (dP - (Pm * dP).sum(1, keepdims=True))
+        dQ[:, cs] = scale * (dS @ K[:, cs])
+        dK[:, cs] = scale * (dS.T @ Q[:, cs])
     return dQ, dK, dV
 
 

@@ -631,20 +631,22 @@ def test_p9_null_h_in_equals_zero_h_in():
 # ----------------------------------------------------------- golden: Sec. 4
 def test_golden_complexity_ratios():
     """Sec. 4 prints, for P=64, a 4096x cheaper proxy attention and a 64x
-    smaller history cache.  Count the oracle's score evaluations (visible keys
-    summed over queries) for bidirectional attention over L tokens vs over
-    L/P proxies, and its cache rows after streaming L_h tokens."""
+    smaller history cache.  Count the oracle's score evaluations (the visible
+    (query, key) pairs of the mask it applies) for bidirectional attention
+    over L tokens vs over L/P proxies, and its cache rows after streaming L_h
+    tokens."""
     with open(os.path.join(GOLDEN, "complexity_p64.json")) as f:
         g = json.load(f)
     P = g["P"]
     calls = []
-    orig = OL._row_probs
+    orig = OL.proxy_mask
 
-    def counting(q, Kh, n_vis, scale):
-        calls.append(n_vis)
-        return orig(q, Kh, n_vis, scale)
+    def counting(m, spec):
+        vis = orig(m, spec)
+        calls.append(int(vis.sum()))
+        return vis
 
-    OL._row_probs = counting
+    OL.proxy_mask = counting
     try:
         L, d = 2 * P, 1
         full = S.LayerSpec(batch=1, L=L, d=d, n_heads=1, P=1, mode=S.BIDIR_1D, inject=S.INJ_ADD,
@@ -660,7 +662,7 @@ def test_golden_complexity_ratios():
             else:
                 n_prox = sp_count
     finally:
-        OL._row_probs = orig
+        OL.proxy_mask = orig
     assert n_full // n_prox == g["attention_speedup"]
     spec = S.DecodeSpec(batch=1, d=4, n_heads=1, P=P, capacity=4)
     prm = S.make_decode_params(spec, 1)
