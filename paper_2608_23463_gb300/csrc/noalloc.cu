@@ -1,12 +1,13 @@
 // Allocation-free variant of proxy_layer_bwd (see proxyformer.h).
 //
-// Some callers cannot hand the library a workspace: code that runs while a
-// stream is being captured in a mode that forbids cudaMalloc, host frameworks
-// whose memory planner owns every device byte and gives plugins no scratch,
-// and latency-critical loops that cannot afford cudaMalloc's implicit device
+// Some callers cannot hand the library a workspace: host frameworks whose
+// memory planner owns every device byte and gives plugins no scratch, and
+// latency-critical loops that cannot afford cudaMalloc's implicit device
 // synchronisation.  For them the backward's scratch lives in the fixed
 // file-scope device array below instead of a caller buffer.
 #include <stdio.h>
+
+#include <atomic>
 
 #include "kernels.h"
 #include "proxyformer.h"
@@ -20,7 +21,10 @@ namespace {
 static __device__ __align__(256) unsigned char g_noalloc_scratch[PF_NOALLOC_SCRATCH_BYTES];
 
 constexpr int kMaxDevices = 64;
-void* g_scratch_addr[kMaxDevices] = {};
+// Device address of the array per device, filled on a device's first call.
+// Host threads may race on the first call: each looks the (same) address up
+// and stores it; readers see either null (and look it up too) or the address.
+std::atomic<void*> g_scratch_addr[kMaxDevices] = {};
 
 thread_local char g_noalloc_msg[256];
 
@@ -46,7 +50,8 @@ extern "C" pf_status proxy_layer_bwd_noalloc(const pf_layer_desc* desc,
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess || dev < 0 || dev >= kMaxDevices)
     return pf_set_error(PF_ERR_CUDA, "proxy_layer_bwd_noalloc: no usable current device");
-  if (g_scratch_addr[dev] == nullptr) {
+  void* scratch = g_scratch_addr[dev].load(std::memory_order_acquire);
+  if (scratch == nullptr) {
     // Host code must not use g_noalloc_scratch directly (on the host it is a
     // stand-in symbol, not a device address): look the device address up once
     // per device, with that device current.
@@ -57,8 +62,9 @@ extern "C" pf_status proxy_layer_bwd_noalloc(const pf_layer_desc* desc,
                "proxy_layer_bwd_noalloc: cudaGetSymbolAddress failed: %s", cudaGetErrorString(e));
       return pf_set_error(PF_ERR_CUDA, g_noalloc_msg);
     }
-    g_scratch_addr[dev] = p;
+    g_scratch_addr[dev].store(p, std::memory_order_release);
+    scratch = p;
   }
   return proxy_layer_bwd(desc, params, X, H_in, t, saved, dX_out, dH_out, dX, dH_in, grads,
-                         g_scratch_addr[dev], (size_t)PF_NOALLOC_SCRATCH_BYTES, stream);
+                         scratch, (size_t)PF_NOALLOC_SCRATCH_BYTES, stream);
 }
