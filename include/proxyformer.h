@@ -352,12 +352,27 @@ pf_status pf_sync_check(void *stream);
 pf_status pf_gemm_bf16(int M, int N, int K, const void *A, int a_mn, const void *B,
                        int b_mn, float *D, int ldd, void *stream);
 
+/* Test utilities for the bounded waits (not paper operations).  Every
+ * mbarrier wait of the library's kernels gives up after a time limit (4 s by
+ * default), records PF_ERR_TIMEOUT for pf_sync_check, lets its own copies and
+ * MMAs land (a separately bounded wait), frees its tensor memory and returns.
+ *   pf_debug_set_wait_limit_ns(ns): sets that limit for every kernel launched
+ *     afterwards; 0 restores the default.  Synchronous (the device is idle
+ *     when it returns).  Returns PF_ERR_CUDA if the device write fails.
+ *   pf_debug_gemm_skip_loads(on): while on, the GEMM kernel (pf_gemm_bf16 and
+ *     every contraction of the layer) issues none of its operand loads, so its
+ *     MMA warp waits for data that never comes and the wait runs out.  Nothing
+ *     is in flight when the kernel leaves; the outputs hold garbage.  For tests
+ *     of the timeout path only; off by default.                              */
+pf_status pf_debug_set_wait_limit_ns(unsigned long long ns);
+pf_status pf_debug_gemm_skip_loads(int on);
+
 /* ---------------------------------------------------------------------------
  * Allocation-free backward.  The paper has no counterpart; this is a calling
- * convenience of the library.  Some callers cannot provide a workspace: code
- * running while a stream is captured in a mode that forbids cudaMalloc, host
- * frameworks whose memory planner owns all device memory, and latency-critical
- * loops that cannot pay cudaMalloc's implicit device synchronisation.  This
+ * convenience of the library.  Some callers cannot provide a workspace: host
+ * frameworks whose memory planner owns all device memory and hands plugins no
+ * scratch, and latency-critical loops that cannot pay cudaMalloc's implicit
+ * device synchronisation.  This
  * entry point computes exactly what proxy_layer_bwd computes, with its scratch
  * taken from a fixed device array of PF_NOALLOC_SCRATCH_BYTES inside the
  * library instead of a caller buffer; it calls no allocator.  The caller still
@@ -390,6 +405,11 @@ pf_status proxy_layer_bwd_noalloc(const pf_layer_desc *desc, const pf_layer_para
  * elapsed milliseconds, launch count and per-launch algorithmic FLOPs and
  * bytes.  pf_timing_enable(0/1) discards previous records.  Not thread safe.  */
 void        pf_timing_enable(int on);
+/* FP32 FMA peak probe (measurement utility): `blocks` CTAs of 512 threads,
+ * each thread 8 independent fmaf chains of `iters` steps, i.e.
+ * blocks * 512 * 8 * iters FMAs = twice that many FLOPs; `out` (device,
+ * blocks * 512 floats) receives one value per thread.  The caller times it.  */
+pf_status   pf_probe_ffma(void *out, int blocks, int iters, void *stream);
 int         pf_timing_collect(void);
 const char *pf_timing_label(int i);
 double      pf_timing_ms(int i);

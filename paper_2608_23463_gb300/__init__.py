@@ -89,7 +89,8 @@ EXPORTED = ("proxy_layer_check", "proxy_layer_saved_size", "proxy_layer_workspac
             "proxy_segments_bwd",
             "pf_last_error", "pf_sync_check", "pf_gemm_bf16", "pf_timing_enable",
             "pf_timing_collect", "pf_timing_label", "pf_timing_ms", "pf_timing_launches",
-            "pf_timing_flops", "pf_timing_bytes", "proxy_layer_bwd_noalloc")
+            "pf_timing_flops", "pf_timing_bytes", "proxy_layer_bwd_noalloc",
+            "pf_debug_set_wait_limit_ns", "pf_debug_gemm_skip_loads", "pf_probe_ffma")
 
 _lib: Optional[ctypes.CDLL] = None
 
@@ -168,6 +169,12 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
     lib.proxy_layer_bwd_noalloc.restype = ctypes.c_int
     lib.pf_timing_launches.argtypes = [ctypes.c_int]
     lib.pf_timing_launches.restype = ctypes.c_int
+    lib.pf_debug_set_wait_limit_ns.argtypes = [ctypes.c_ulonglong]
+    lib.pf_debug_set_wait_limit_ns.restype = ctypes.c_int
+    lib.pf_debug_gemm_skip_loads.argtypes = [ctypes.c_int]
+    lib.pf_debug_gemm_skip_loads.restype = ctypes.c_int
+    lib.pf_probe_ffma.argtypes = [_vp, ctypes.c_int, ctypes.c_int, _vp]
+    lib.pf_probe_ffma.restype = ctypes.c_int
     _lib = lib
     return lib
 
@@ -326,6 +333,21 @@ def pf_last_error() -> str:
 def pf_gemm_bf16(M, N, K, A, a_mn, B, b_mn, D, ldd, stream=None):
     _check(load().pf_gemm_bf16(int(M), int(N), int(K), _ptr(A), int(a_mn), _ptr(B), int(b_mn),
                                _ptr(D), int(ldd), stream))
+
+
+def pf_debug_set_wait_limit_ns(ns: int) -> None:
+    """Time limit of every bounded wait in the library's kernels (0: default)."""
+    _check(load().pf_debug_set_wait_limit_ns(int(ns)))
+
+
+def pf_debug_gemm_skip_loads(on: bool) -> None:
+    """Test hook: the GEMM kernel issues no operand loads while on."""
+    _check(load().pf_debug_gemm_skip_loads(1 if on else 0))
+
+
+def pf_probe_ffma(out, blocks: int, iters: int, stream=None) -> None:
+    """Launch the fp32 FMA peak probe (2 * blocks * 512 * 8 * iters FLOPs)."""
+    _check(load().pf_probe_ffma(_ptr(out), int(blocks), int(iters), stream))
 
 
 def pf_timing_enable(on: bool) -> None:

@@ -1962,6 +1962,24 @@ pf_status pf_sync_check(void* stream) {
   return PF_OK;
 }
 
+pf_status pf_debug_set_wait_limit_ns(unsigned long long ns) {
+  if (ns == 0) ns = kWaitLimitNs;
+  int bad = 0;
+  for (int r : {set_wait_limit_gemm(ns), set_wait_limit_attention(ns),
+                set_wait_limit_attention_tc(ns), set_wait_limit_attention_bwd_tc(ns),
+                set_wait_limit_elementwise(ns), set_wait_limit_decode(ns), set_wait_limit_fp32(ns),
+                set_wait_limit_layer2d(ns)})
+    bad |= r;
+  if (bad) return fail(PF_ERR_CUDA, "pf_debug_set_wait_limit_ns: writing the limit failed");
+  return PF_OK;
+}
+
+pf_status pf_debug_gemm_skip_loads(int on) {
+  if (set_debug_skip_loads_gemm(on ? 1 : 0))
+    return fail(PF_ERR_CUDA, "pf_debug_gemm_skip_loads: writing the flag failed");
+  return PF_OK;
+}
+
 pf_status pf_gemm_bf16(int M, int N, int K, const void* A, int a_mn, const void* B, int b_mn,
                        float* D, int ldd, void* stream) {
   if (M < 1 || N < 1 || K < 1 || N % 32 != 0 || !A || !B || !D || ldd < N || ldd % 4 != 0)

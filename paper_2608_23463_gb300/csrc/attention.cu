@@ -84,6 +84,7 @@ cudaError_t cross_gate_bwd(const bf16* dAg, const bf16* A, const bf16* qa, long 
 }
 
 int take_dev_error_attention() { return take_dev_error_tu(); }
+int set_wait_limit_attention(unsigned long long ns) { return set_wait_limit_tu(ns); }
 
 cudaError_t attn_bwd(const bf16* qkv, const bf16* O, const bf16* dO, const float* lse, float* Di,
                      bf16* dqkv, int B, int m, int d, int nh, bool causal, cudaStream_t st) {

@@ -477,6 +477,7 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
 }  // namespace
 
 int take_dev_error_attention_bwd_tc() { return take_dev_error_tu(); }
+int set_wait_limit_attention_bwd_tc(unsigned long long ns) { return set_wait_limit_tu(ns); }
 
 namespace {
 

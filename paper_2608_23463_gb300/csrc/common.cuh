@@ -32,9 +32,18 @@ static inline int take_dev_error_tu() {
   return v;
 }
 
-// A wait gives up after this long (the longest single kernel of the library
-// runs for a few milliseconds).
+// A wait gives up after this long by default (the longest single kernel of
+// the library runs for a few milliseconds).  The limit is a per-file device
+// word so that a test can shorten it (pf_debug_set_wait_limit_ns).
 constexpr unsigned long long kWaitLimitNs = 4000000000ull;
+static __device__ unsigned long long g_wait_limit_ns = kWaitLimitNs;
+// Test hook of the GEMM producer: when nonzero it issues no operand loads, so
+// the MMA warp's first wait runs out (read only by gemm_tc_kernel).
+static __device__ int g_debug_skip_loads;
+
+static inline int set_wait_limit_tu(unsigned long long ns) {
+  return cudaMemcpyToSymbol(g_wait_limit_ns, &ns, sizeof(ns)) == cudaSuccess ? 0 : -1;
+}
 
 __device__ __forceinline__ void set_dev_error(int code) {
   atomicCAS(&g_dev_error, 0, code);
@@ -81,7 +90,7 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 }
 
 // Bounded wait for the phase with the given parity to complete.  Returns false
-// (and records DEVERR_TIMEOUT) if it does not complete within kWaitLimitNs or
+// (and records DEVERR_TIMEOUT) if it does not complete within g_wait_limit_ns or
 // if another thread already recorded an error.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
   unsigned long long t0 = 0;
@@ -91,7 +100,7 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
       unsigned long long now = globaltimer();
       if (t0 == 0) {
         t0 = now;
-      } else if (now - t0 > kWaitLimitNs || it > 0x7fffffffu) {
+      } else if (now - t0 > g_wait_limit_ns || it > 0x7fffffffu) {
         set_dev_error(DEVERR_TIMEOUT);
         return false;
       }
@@ -131,7 +140,7 @@ __device__ __forceinline__ void mbar_wait_drain(uint32_t bar, uint32_t parity) {
       unsigned long long now = globaltimer();
       if (t0 == 0)
         t0 = now;
-      else if (now - t0 > kWaitLimitNs || it > 0x7fffffffu)
+      else if (now - t0 > g_wait_limit_ns || it > 0x7fffffffu)
         return;
     }
   }

@@ -30,6 +30,7 @@
 namespace pf {
 
 int take_dev_error_decode() { return take_dev_error_tu(); }
+int set_wait_limit_decode(unsigned long long ns) { return set_wait_limit_tu(ns); }
 
 namespace {
 

@@ -492,6 +492,7 @@ int inj_bwd_chunks(long M, int N) {
 }
 
 int take_dev_error_elementwise() { return take_dev_error_tu(); }
+int set_wait_limit_elementwise(unsigned long long ns) { return set_wait_limit_tu(ns); }
 
 cudaError_t inj_bwd_1d(const InjBwdArgs& a, float* part, int n_chunks, cudaStream_t st) {
   const long M = (long)a.B * a.m * a.k2;

@@ -10,6 +10,7 @@
 namespace pf {
 
 int take_dev_error_fp32() { return take_dev_error_tu(); }
+int set_wait_limit_fp32(unsigned long long ns) { return set_wait_limit_tu(ns); }
 
 namespace {
 

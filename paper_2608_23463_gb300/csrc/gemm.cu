@@ -10,6 +10,10 @@
 namespace pf {
 
 int take_dev_error_gemm() { return take_dev_error_tu(); }
+int set_wait_limit_gemm(unsigned long long ns) { return set_wait_limit_tu(ns); }
+int set_debug_skip_loads_gemm(int on) {
+  return cudaMemcpyToSymbol(g_debug_skip_loads, &on, sizeof(on)) == cudaSuccess ? 0 : -1;
+}
 
 int num_sms() {
   static int n = 0;

@@ -252,6 +252,9 @@ __global__ void __launch_bounds__(GemmRoles<Epi>::kThreads, 1)
     // ---------------------------------------------------------- producer
     prefetch_tmap(&tmA);
     prefetch_tmap(&tmB);
+    // test hook: arm no stage and issue no load, so that nothing is ever in
+    // flight and the MMA warp's first wait runs out
+    const bool skip_loads = *(volatile int*)&g_debug_skip_loads != 0;
     uint32_t it = 0;
     bool ok = true;
     for (int tile = unit; tile < tiles && ok; tile += n_units) {
@@ -264,6 +267,7 @@ __global__ void __launch_bounds__(GemmRoles<Epi>::kThreads, 1)
           ok = false;
           break;
         }
+        if (skip_loads) continue;
         // a pair: both CTAs' loads complete on rank 0's full barrier, which
         // rank 0 arms for the two CTAs' bytes
         const uint32_t fb = PAIR ? smem_map_rank(full0 + 8 * s, 0) : full0 + 8 * s;

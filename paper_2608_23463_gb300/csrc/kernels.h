@@ -96,7 +96,18 @@ cudaError_t gemm_append_kv(int M, int N, int K, Operand A, Operand B, const EpiA
                            cudaStream_t st);
 int num_sms();
 
-// Per-file device error flags (see common.cuh): value, cleared on read.
+// Per-file device error flags (see common.cuh): value, cleared on read.  The
+// per-file wait limits (set_wait_limit_*) and the GEMM producer's load-skip
+// hook serve the timeout test (pf_debug_set_wait_limit_ns); 0 = success.
+int set_wait_limit_gemm(unsigned long long ns);
+int set_wait_limit_decode(unsigned long long ns);
+int set_wait_limit_attention(unsigned long long ns);
+int set_wait_limit_attention_tc(unsigned long long ns);
+int set_wait_limit_attention_bwd_tc(unsigned long long ns);
+int set_wait_limit_elementwise(unsigned long long ns);
+int set_wait_limit_fp32(unsigned long long ns);
+int set_wait_limit_layer2d(unsigned long long ns);
+int set_debug_skip_loads_gemm(int on);
 int take_dev_error_gemm();
 int take_dev_error_decode();
 int take_dev_error_attention();

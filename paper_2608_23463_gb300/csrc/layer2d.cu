@@ -8,6 +8,7 @@
 namespace pf {
 
 int take_dev_error_layer2d() { return take_dev_error_tu(); }
+int set_wait_limit_layer2d(unsigned long long ns) { return set_wait_limit_tu(ns); }
 
 namespace {
 

@@ -108,3 +108,34 @@ double pf_timing_bytes(int i) {
 }
 
 }  // extern "C"
+
+// ------------------------------------------------------------ FFMA probe
+// Peak of the fp32 FMA pipe, measured: every thread runs 8 independent FMA
+// chains of `iters` steps (8 chains hide the FMA latency at 16 warps per SM
+// sub-partition), then stores one value so the chains are not dead code.
+namespace pf {
+namespace {
+__global__ void __launch_bounds__(512) ffma_probe_kernel(float* out, int iters, float a0) {
+  float v[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) v[j] = a0 + 0.001f * (float)(threadIdx.x + j);
+  const float b = 0.999f, c = 0.001f;
+  for (int i = 0; i < iters; ++i) {
+#pragma unroll
+    for (int j = 0; j < 8; ++j) v[j] = fmaf(v[j], b, c);
+  }
+  float acc = 0.f;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) acc += v[j];
+  out[(long)blockIdx.x * blockDim.x + threadIdx.x] = acc;
+}
+}  // namespace
+}  // namespace pf
+
+extern "C" pf_status pf_probe_ffma(void* out, int blocks, int iters, void* stream) {
+  if (out == nullptr || blocks < 1 || iters < 1) return PF_ERR_INVALID_ARG;
+  pf::ffma_probe_kernel<<<blocks, 512, 0, static_cast<cudaStream_t>(stream)>>>(
+      static_cast<float*>(out), iters, 1.0f);
+  return cudaGetLastError() == cudaSuccess ? PF_OK : PF_ERR_CUDA;
+}
+
