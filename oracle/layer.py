@@ -648,12 +648,15 @@ def partition_w(A, spec):
     return g.transpose(0, 2, 1, 3, 4).reshape(-1, p * p, w)
 
 
-def layer_bwd(spec, prm, X, G, H_in=None, t=None, dH_out=None):
+def layer_bwd(spec, prm, X, G, H_in=None, t=None, dH_out=None, caches=None):
     """Backward of ``layer_fwd`` (chain rule through Eqs. partition ...
-    inj-*).  Returns (dX [B, L, d], dH_in [B, m, d], grads{name: array})."""
+    inj-*).  Returns (dX [B, L, d], dH_in [B, m, d], grads{name: array}).
+    ``caches`` may pass the activations a ``layer_fwd(..., return_cache=True)``
+    of the same inputs returned, instead of recomputing them."""
     X = _f64(X)
     G = _f64(G)
-    _, _, caches = layer_fwd(spec, prm, X, H_in, t, return_cache=True)
+    if caches is None:
+        _, _, caches = layer_fwd(spec, prm, X, H_in, t, return_cache=True)
     grads = {k: np.zeros(np.shape(v)) for k, v in prm.items()
              if k.startswith(("W_", "b_", "w_"))}
     dXs, dHs = [], []

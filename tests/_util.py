@@ -12,6 +12,9 @@ Floating-point bars (bf16 storage, fp32 accumulation):
     derivation is in test_bf16_error_floor.py, which rounds the float64
     oracle's intermediates at the library's bf16 storage points.
 """
+import json
+import os
+
 import numpy as np
 
 BF16_TOL = 2e-2
@@ -21,6 +24,20 @@ F32_TOL = 1e-4
 # max up to 2.3e-1 (test_bf16_error_floor.py); the bar is about twice that
 CROSS_TOL = 4e-2
 CROSS_MAX_TOL = 3e-1
+
+
+def record(name, gpu, ref, bar=""):
+    """Append the measured errors of one compared tensor (RMS and max-abs
+    error, both relative to RMS(ref)) to the JSON-lines file named by the
+    environment variable PF_PARITY_LOG, when it is set."""
+    path = os.environ.get("PF_PARITY_LOG")
+    if not path:
+        return
+    test = os.environ.get("PYTEST_CURRENT_TEST", "").split(" ")[0]
+    row = {"test": test, "tensor": name, "rms_err": rms_rel_err(gpu, ref),
+           "max_err": max_rel_err(gpu, ref), "n": int(np.asarray(ref).size), "bar": bar}
+    with open(path, "a") as f:
+        f.write(json.dumps(row) + "\n")
 
 
 def rms(a):
@@ -46,6 +63,7 @@ def rms_rel_err(gpu, ref):
 def assert_close(name, gpu, ref, tol=BF16_TOL):
     """Output bar: max-abs error relative to the reference RMS."""
     e = max_rel_err(gpu, ref)
+    record(name, gpu, ref, f"max {tol:g}")
     assert e <= tol, f"{name}: max|gpu-ref|/rms(ref) = {e:.3e} > {tol:.1e}"
     return e
 
@@ -54,6 +72,7 @@ def assert_grad_close(name, gpu, ref, tol=BF16_TOL, max_tol=BF16_MAX_TOL):
     """Gradient bar: RMS-normalised error and a bound on the worst element."""
     e = rms_rel_err(gpu, ref)
     m = max_rel_err(gpu, ref)
+    record(name, gpu, ref, f"rms {tol:g}, max {max_tol:g}")
     assert e <= tol and m <= max_tol, (f"{name}: rms err {e:.3e} (tol {tol:.0e}), "
                                        f"max err {m:.3e} (tol {max_tol:.0e})")
     return e, m
@@ -64,6 +83,7 @@ def assert_update_close(name, X, gpu_out, ref_out, tol=BF16_TOL, max_tol=BF16_MA
     X = np.asarray(X, np.float64)
     du_g = np.asarray(gpu_out, np.float64) - X
     du_r = np.asarray(ref_out, np.float64) - X
+    record(name, du_g, du_r, f"rms {tol:g} (+ X_out rounding), max {max_tol:g}")
     e = rms(du_g - du_r)
     bound = tol * rms(du_r) + 2.0 ** -9 * rms(ref_out)
     m = float(np.abs(du_g - du_r).max())
