@@ -46,6 +46,13 @@ def parse_args():
     ap.add_argument("--no-configs", action="store_true",
                     help="skip the other workloads (fp32 layer, L=65536 layer, 2D layer, stack)")
     ap.add_argument("--decode-steps", type=int, default=128)
+    ap.add_argument("--case", default="",
+                    choices=("", "layer", "c2", "c5", "cross", "lm_history", "decode"),
+                    help="profiling helper: run only this workload's step (--batch / --L shrink "
+                         "it) and print its time; not the benchmark line")
+    ap.add_argument("--batch", type=int, default=0, help="batch of --case (default: its own)")
+    ap.add_argument("--detail", default="",
+                    help="also write the per-kernel breakdowns of every workload to this JSON file")
     ap.add_argument("--L", type=int, default=0,
                     help="tokens per sequence (default: the workload's 262144; smaller values "
                          "are for profiling captures only)")
@@ -187,16 +194,12 @@ class ClockSampler:
         else:
             self.t1 = time.time()
 
-    def stop(self):
+    def window(self, t0, t1):
+        """Median SM clock, maximum clock and active throttle reasons of the
+        samples taken between wall times t0 and t1."""
         if self.p is None:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
-        time.sleep(0.12)
-        self.p.terminate()
-        try:
-            self.p.wait(timeout=5)
-        except subprocess.TimeoutExpired:
-            self.p.kill()
-        rows = [r for t, r in self.rows if self.t0 and self.t1 and self.t0 - 0.06 <= t <= self.t1]
+        rows = [r for t, r in list(self.rows) if t0 - 0.06 <= t <= t1]
         sm, mx, reasons = [], [], set()
         names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
         for r in rows:
@@ -211,6 +214,18 @@ class ClockSampler:
         return {"sm_mhz": statistics.median(sm) if sm else None,
                 "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons),
                 "samples": len(sm)}
+
+    def stop(self):
+        """Ends sampling; the statistics of the window marked by mark()."""
+        if self.p is None:
+            return self.window(0, 0)
+        time.sleep(0.12)
+        self.p.terminate()
+        try:
+            self.p.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.p.kill()
+        return self.window(self.t0 or 0, self.t1 or 0)
 
 
 def gpu_smi_id(torch, dev: int) -> str:
@@ -341,19 +356,22 @@ def measure_decode(torch, pf, S, steps: int):
 
 
 def timed_steps(torch, pf, fn, steps: int, warmup: int):
-    """Mean ms per call of fn (CUDA events on the current stream) plus the
-    library's per-launch records: algorithmic FLOPs and bytes per call and the
-    label with the largest time."""
+    """Mean ms per call of fn (CUDA events on the current stream), the wall
+    times bracketing the timed calls (for the clock samples), and the
+    library's per-launch records: FLOPs and bytes per call as the kernels
+    count them, and the label with the largest time."""
     stream = torch.cuda.current_stream()
     for _ in range(warmup):
         fn()
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    w0 = time.time()
     e0.record(stream)
     for _ in range(steps):
         fn()
     e1.record(stream)
     torch.cuda.synchronize()
+    w1 = time.time()
     ms = e0.elapsed_time(e1) / steps
     pf.pf_sync_check(stream.cuda_stream)
     pf.pf_timing_enable(True)  # breakdown pass
@@ -368,29 +386,155 @@ def timed_steps(torch, pf, fn, steps: int, warmup: int):
     total = sum(v["ms"] for v in t.values()) or 1.0
     dom, dv = max(t.items(), key=lambda kv: kv[1]["ms"])
     top = sorted(t.items(), key=lambda kv: -kv[1]["ms"])[:8]
-    return ms, flops, nbytes, {"kernel": dom, "share": dv["ms"] / total,
-                               "kernels_ms_per_step": {k: v["ms"] / steps for k, v in top},
-                               "launches_per_step": sum(v["launches"] for v in t.values()) / steps}
+    return ms, (flops, nbytes), {"kernel": dom, "share": dv["ms"] / total,
+                                 "kernels_ms_per_step": {k: v["ms"] / steps for k, v in top},
+                                 "launches_per_step": sum(v["launches"] for v in t.values())
+                                 / steps}, (w0, w1)
 
 
-FFMA_PEAK_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12  # SMs x fp32 lanes x 2 x max SM clock
+# ------------------------------------------------------- algorithmic work
+def layer_work(spec, train: bool = True):
+    """Algorithmic FLOPs and HBM bytes of one layer step (forward, plus the
+    backward when `train`), from the method's own operation counts (Eq.
+    complexity, Sec. 4), not from what the kernels happen to move.
+
+    FLOPs, per sequence (m = ceil(L/P) proxies, tokens df wide, proxies d):
+      compression 2 m P df d (level 1) + 2 m k2 d d (level 2);
+      decompression the mirror image, w = df (2 df for affine injection);
+      proxy attention 8 m d^2 (Q, K, V, O) + 4 d per visible (query, key)
+      pair (m(m+1)/2 causal, m^2 bidirectional); the MLP interaction
+      16 m d^2; the cross injection 2 L df (d + heads) + 4 m d^2 + 4 d per
+      visible (token, proxy) pair + 2 L d df instead of the decompression.
+      The backward costs twice the linear terms and 2.5 times the attention.
+    Bytes: the forward reads X twice (compression, injection) and writes
+    X_out; the backward reads dX_out and X and writes dX; every weight is
+    read once per pass and its fp32 gradient written once."""
+    B, L, d, df, P = spec.batch, spec.L, spec.d, spec.df, spec.P
+    m = -(-L // P)
+    nh = spec.n_heads
+    k2 = spec.k2 if spec.levels == 2 else 1
+    elt = 2 if spec.dtype == 1 else 4
+    affine = spec.inject == 2
+    cross = spec.inject == 3
+    w_tok = 2 * df if affine else df
+    lin = 2.0 * m * P * df * d + (2.0 * m * k2 * d * d if spec.levels == 2 else 0.0)
+    wts = P // k2 * df * d + (k2 * d * d if spec.levels == 2 else 0)
+    if cross:
+        vis_x = (P * m * (m - 1) / 2.0) if spec.mode == 0 else float(L) * m
+        lin += 2.0 * L * df * (d + nh) + 4.0 * m * d * d + 2.0 * L * d * df
+        wts += df * (d + nh) + 2 * d * d + d * df
+        att_x = 4.0 * d * vis_x
+    else:
+        lin += 2.0 * m * k2 * d * (P // k2) * w_tok + (2.0 * m * d * k2 * d if spec.levels == 2
+                                                        else 0.0)
+        wts += d * (P // k2) * w_tok + (d * k2 * d if spec.levels == 2 else 0)
+        att_x = 0.0
+    interact = getattr(spec, "interact", 0)
+    att = 0.0
+    if interact == 0:
+        lin += 8.0 * m * d * d
+        wts += 4 * d * d
+        vis = m * (m + 1) / 2.0 if spec.mode == 0 else float(m) * m
+        att = 4.0 * d * vis
+    elif interact == 2:
+        lin += 16.0 * m * d * d
+        wts += 8 * d * d
+    fwd_flops = B * (lin + att + att_x)
+    act = B * L * df * elt
+    flops = fwd_flops
+    nbytes = 3.0 * act + wts * elt
+    if train:
+        flops += B * (2.0 * lin + 2.5 * (att + att_x))
+        nbytes += 3.0 * act + wts * elt + 4.0 * wts
+    return flops, nbytes
 
 
-def config_entry(metric, tokens, ms, flops, nbytes, dom, peaks, steps, alu=False):
-    comp_peak = FFMA_PEAK_TFLOPS if alu else peaks["bf16_tflops_sustained"]
-    roof_ms = max(flops / (comp_peak * 1e12), nbytes / (peaks["hbm_gbs"] * 1e9)) * 1e3
-    return {"metric": metric, "value": tokens / (ms / 1e3), "unit": "tokens/s",
-            "ms_per_step": ms, "steps": steps,
-            "roofline": {"bound": "alu" if alu else "tensor", "flops_per_step": flops,
-                         "bytes_per_step": nbytes, "compute_peak_tflops": comp_peak,
-                         "roofline_ms": roof_ms, "frac": roof_ms / ms, **dom}}
+def segments_work(d, nh, levels, segs):
+    """``layer_work`` of a layer with temporal-distance ratios: each segment's
+    compression and decompression at its own ratio, one causal attention over
+    all the proxies, weights of every segment."""
+    import pf_synth as S
+    flops = nbytes = 0.0
+    m_tot = 0
+    for sg in segs:
+        kw = dict(k1=sg[2], k2=sg[3]) if levels == 2 else {}
+        sp = S.LayerSpec(batch=1, L=sg[0], d=d, n_heads=nh, P=sg[1], levels=levels,
+                         interact=S.F_IDENTITY, **kw)
+        f, b = layer_work(sp)
+        flops += f
+        nbytes += b
+        m_tot += -(-sg[0] // sg[1])
+    att = 4.0 * d * m_tot * (m_tot + 1) / 2.0
+    flops += 8.0 * m_tot * d * d * 3 + 3.5 * att
+    nbytes += 4 * d * d * 8
+    return flops, nbytes
 
 
-def measure_configs(torch, pf, S, peaks, warmup: int):
-    """The other paper workloads, each timed on its own (fresh buffers)."""
+def compute_peak(peaks, clocks):
+    """bf16 dense peak for a kernel timed at the sampled SM clock: the burst
+    figure (measured at the maximum clock) scaled by median / maximum clock,
+    never above the burst figure."""
+    burst = peaks["bf16_tflops"]
+    mhz, mx = (clocks or {}).get("sm_mhz"), (clocks or {}).get("sm_max_mhz")
+    if mhz and mx:
+        return burst * min(1.0, mhz / mx), f"bf16_tflops (burst) x {mhz:.0f}/{mx:.0f} MHz"
+    return burst, "bf16_tflops (burst; no clock samples)"
+
+
+def measure_ffma_peak(torch, pf):
+    """The fp32 FMA pipe's peak, measured with the library's probe kernel
+    (CUDA events, best of 5): TFLOP/s."""
+    blocks, iters = 8 * 152, 4096
+    out = torch.empty(blocks * 512, dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+    pf.pf_probe_ffma(out, blocks, iters, stream.cuda_stream)
+    torch.cuda.synchronize()
+    best = float("inf")
+    for _ in range(5):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        pf.pf_probe_ffma(out, blocks, iters, stream.cuda_stream)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        best = min(best, e0.elapsed_time(e1))
+    return 2.0 * blocks * 512 * 8 * iters / (best / 1e3) / 1e12
+
+
+def config_entry(metric, tokens, ms, work, dom, peaks, steps, clocks=None, ffma=None,
+                 rec=None):
+    """One workload's line: throughput and its roofline fraction, the bound
+    being the larger of algorithmic FLOPs at the compute peak (bf16 tensor, or
+    the measured FFMA peak for fp32) and algorithmic bytes at HBM bandwidth."""
+    flops, nbytes = work
+    if ffma:
+        comp_peak, src = ffma, "fp32 FFMA, measured by the probe kernel"
+    else:
+        comp_peak, src = compute_peak(peaks, clocks)
+    t_c = flops / (comp_peak * 1e12) * 1e3
+    t_b = nbytes / (peaks["hbm_gbs"] * 1e9) * 1e3
+    roof_ms = max(t_c, t_b)
+    bound = ("alu" if ffma else "tensor") if t_c >= t_b else "hbm"
+    e = {"metric": metric, "value": tokens / (ms / 1e3), "unit": "tokens/s",
+         "ms_per_step": ms, "steps": steps,
+         "roofline": {"bound": bound, "flops_per_step": flops, "bytes_per_step": nbytes,
+                      "compute_peak_tflops": comp_peak, "compute_peak_source": src,
+                      "roofline_ms": roof_ms, "frac": roof_ms / ms, **dom}}
+    if rec:
+        e["roofline"]["flops_per_step_kernel_records"] = rec[0]
+    if clocks:
+        e["clocks"] = clocks
+    return e
+
+
+def measure_configs(torch, pf, S, peaks, warmup: int, sampler=None, ffma=None):
+    """The other paper workloads, each timed on its own (fresh buffers); the
+    clock samples of each one's timed window set its compute peak."""
     from paper_2608_23463_gb300.layer import ProxyLayer, to_device
     from paper_2608_23463_gb300.stack import ProxyStack
     out = {}
+
+    def clk(win):
+        return sampler.window(*win) if sampler else None
 
     def layer_case(spec, seed, train, steps):
         inp = S.make_layer_inputs(spec, seed, with_grads=train)
@@ -408,47 +552,33 @@ def measure_configs(torch, pf, S, peaks, warmup: int):
                 lay.backward(X, G, None, t, dX=dX)
         return timed_steps(torch, pf, step, steps, warmup)
 
-    s1 = S.spec_c1()
-    ms, fl, nb, dom = layer_case(s1, 0, False, 20)
-    out["c1_fp32_fwd"] = config_entry("1D causal layer fwd, fp32, L=4096 d=256 4x64 P=64",
-                                      s1.batch * s1.L, ms, fl, nb, dom, peaks, 20, alu=True)
-    torch.cuda.empty_cache()
-    s2 = S.spec_c2()
-    ms, fl, nb, dom = layer_case(s2, 1, True, 10)
-    out["c2_layer_fwd_bwd"] = config_entry(
-        "1D causal layer fwd+bwd, bf16, L=65536 d=1024 16x64 P=64", s2.batch * s2.L, ms, fl, nb,
-        dom, peaks, 10)
-    torch.cuda.empty_cache()
-    sh = S.spec_lm_history()
-    ms, fl, nb, dom = layer_case(sh, 6, True, 10)
-    out["lm_history_fwd_bwd"] = config_entry(
-        "1D causal layer fwd+bwd with 64-wide tokens and 512-wide proxies (the language model's "
-        "history stream), bf16, L=1048576 8x64 heads P=64", sh.batch * sh.L, ms, fl, nb, dom,
-        peaks, 10)
-    torch.cuda.empty_cache()
+    def entry(key, metric, spec, seed, train, steps, **kw):
+        ms, rec, dom, win = layer_case(spec, seed, train, steps)
+        out[key] = config_entry(metric, spec.batch * spec.L, ms, layer_work(spec, train), dom,
+                                peaks, steps, clocks=clk(win), rec=rec, **kw)
+        torch.cuda.empty_cache()
+
+    entry("c1_fp32_fwd", "1D causal layer fwd, fp32, L=4096 d=256 4x64 P=64", S.spec_c1(), 0,
+          False, 20, ffma=ffma)
+    entry("c2_layer_fwd_bwd", "1D causal layer fwd+bwd, bf16, L=65536 d=1024 16x64 P=64",
+          S.spec_c2(), 1, True, 10)
+    entry("lm_history_fwd_bwd", "1D causal layer fwd+bwd with 64-wide tokens and 512-wide "
+          "proxies (the language model's history stream), bf16, L=1048576 8x64 heads P=64",
+          S.spec_lm_history(), 6, True, 10)
     for key, kw in (("mlp_interaction_fwd_bwd", dict(interact=S.F_MLP)),
                     ("rope_attention_fwd_bwd", dict(rope=1))):
         sv = S.LayerSpec(batch=1, L=262144, d=1024, n_heads=16, P=64, levels=2, k1=8, k2=8, **kw)
-        ms, fl, nb, dom = layer_case(sv, 7, True, 10)
         what = ("single-proxy MLP interaction (hidden 4d, SiLU)" if "mlp" in key
                 else "proxy attention with RoPE on queries and keys")
-        out[key] = config_entry(f"1D causal layer fwd+bwd with {what}, bf16, L=262144 d=1024 "
-                                "16x64 P=64 8x8", sv.L, ms, fl, nb, dom, peaks, 10)
-        torch.cuda.empty_cache()
-    out["segments_fwd_bwd"] = measure_segments(torch, pf, S, peaks, warmup)
+        entry(key, f"1D causal layer fwd+bwd with {what}, bf16, L=262144 d=1024 16x64 P=64 8x8",
+              sv, 7, True, 10)
+    out["segments_fwd_bwd"] = measure_segments(torch, pf, S, peaks, warmup, clk)
     torch.cuda.empty_cache()
-    sx = S.spec_cross_layer()
-    ms, fl, nb, dom = layer_case(sx, 5, True, 5)
-    out["cross_layer_fwd_bwd"] = config_entry(
-        "1D causal layer fwd+bwd with gated cross-attention injection (Eq. inj-cross), bf16, "
-        "L=262144 d=1024 16x64 P=64 8x8", sx.batch * sx.L, ms, fl, nb, dom, peaks, 5)
-    torch.cuda.empty_cache()
-    s5 = S.spec_c5()
-    ms, fl, nb, dom = layer_case(s5, 4, True, 5)
-    out["c5_2d_fwd_bwd"] = config_entry(
-        "2D bidirectional layer fwd+bwd, bf16, B=4 512x512 d=512 8x64 8x8 patches",
-        s5.batch * s5.L, ms, fl, nb, dom, peaks, 5)
-    torch.cuda.empty_cache()
+    entry("cross_layer_fwd_bwd", "1D causal layer fwd+bwd with gated cross-attention injection "
+          "(Eq. inj-cross), bf16, L=262144 d=1024 16x64 P=64 8x8", S.spec_cross_layer(), 5,
+          True, 5)
+    entry("c5_2d_fwd_bwd", "2D bidirectional layer fwd+bwd, bf16, B=4 512x512 d=512 8x64 8x8 "
+          "patches", S.spec_c5(), 4, True, 5)
     specs, params = [], []
     for i, P in enumerate(S.C3_RATIOS):
         k1, k2 = S.default_factors(P)
@@ -464,24 +594,28 @@ def measure_configs(torch, pf, S, peaks, warmup: int):
     def stack_step():
         st.forward(X)
         st.backward(G)
-    ms, fl, nb, dom = timed_steps(torch, pf, stack_step, 3, warmup)
+    ms, rec, dom, win = timed_steps(torch, pf, stack_step, 3, warmup)
+    work = [sum(w) for w in zip(*(layer_work(sp) for sp in specs))]
     out["c3_stack_fwd_bwd"] = config_entry(
         "12-layer causal stack fwd+bwd, bf16, L=262144 d=1024 16x64, P=16..256 two-level",
-        specs[0].L, ms, fl, nb, dom, peaks, 3)
+        specs[0].L, ms, work, dom, peaks, 3, clocks=clk(win), rec=rec)
     del G
-    out["prefill"] = measure_prefill(torch, pf, S, peaks, warmup, specs, params, st, X)
+    out["prefill"] = measure_prefill(torch, pf, S, peaks, warmup, specs, params, st, X, clk)
     del st, X, params
     torch.cuda.empty_cache()
     return out
 
 
-def measure_segments(torch, pf, S, peaks, warmup):
+SEGMENTS = [(131072, 256, 16, 16), (98304, 64, 8, 8), (32768, 16, 4, 4)]
+
+
+def measure_segments(torch, pf, S, peaks, warmup, clk):
     """Temporal-distance ratios (Sec. 3.6) on the 262144-token causal layer,
     d = 1024, 16x64 heads, two levels: the distant 131072 tokens in P = 256
     blocks, the next 98304 in P = 64, the recent 32768 in P = 16 (4096
     proxies, as many as uniform P = 64)."""
     from paper_2608_23463_gb300.segments import ProxySegmentLayer
-    segs = [(131072, 256, 16, 16), (98304, 64, 8, 8), (32768, 16, 4, 4)]
+    segs = SEGMENTS
     try:
         spec = S.LayerSpec(batch=1, L=262144, d=1024, n_heads=16, P=256, levels=2, k1=16, k2=16)
         shared, seg_prm = S.make_segment_params(1024, 16, 2, segs, 90)
@@ -494,38 +628,43 @@ def measure_segments(torch, pf, S, peaks, warmup):
         def step():
             lay.forward(X, Xo)
             lay.backward(X, G, dX)
-        ms, fl, nb, dom = timed_steps(torch, pf, step, 5, warmup)
+        ms, rec, dom, win = timed_steps(torch, pf, step, 5, warmup)
         return config_entry("1D causal layer fwd+bwd with temporal-distance ratios (P = 256 / 64 / "
                             "16 from distant to recent), bf16, L=262144 d=1024 16x64 two-level",
-                            spec.L, ms, fl, nb, dom, peaks, 5)
+                            spec.L, ms, segments_work(1024, 16, 2, segs), dom, peaks, 5,
+                            clocks=clk(win), rec=rec)
     except Exception as e:  # reported in the JSON line rather than ending the run
         return {"error": str(e).splitlines()[0][:200]}
 
 
-def measure_prefill(torch, pf, S, peaks, warmup, specs, params, st, X):
+def measure_prefill(torch, pf, S, peaks, warmup, specs, params, st, X, clk):
     """Prefill of the 12-layer causal stack over a 262144-token history
     (Sec. 3.8): the inference forward plus every layer's bulk proxy-cache
     fill, against a standard softmax-attention prefill of the same depth,
     width and history (per layer: the QKV projection, causal attention over
     all L tokens, the output projection).  The standard arm runs PyTorch's
     fused attention and cuBLAS, one layer timed and scaled by the depth; its
-    FLOP floor at the measured bf16 peak is reported beside it."""
+    FLOP floor at the measured (burst) bf16 peak is reported beside it."""
     from paper_2608_23463_gb300.decode import ProxyKVCache
     caches = []
     for i, s in enumerate(specs):
         ds = S.decode_spec_for_layer(s, s.L // s.P)
         dp = S.decode_params_for_layer(s, params[i], 200 + i)
         caches.append(ProxyKVCache(ds, dp, S.make_decode_state(ds, 0, [0], [0])))
-    ms, fl, nb, dom = timed_steps(torch, pf, lambda: st.prefill(X, caches), 3, warmup)
+    ms, rec, dom, win = timed_steps(torch, pf, lambda: st.prefill(X, caches), 3, warmup)
     L, d, n = specs[0].L, specs[0].d, len(specs)
+    # the inference forward of every layer plus its cache rows (K and V, bf16)
+    work = [sum(w) for w in zip(*(layer_work(sp, False) for sp in specs))]
+    work[1] += sum(2 * (sp.L // sp.P) * sp.d * 2 for sp in specs)
     res = config_entry("causal stack prefill latency, 12 layers, L=262144 d=1024 16x64, "
-                       "P=16..256 two-level, proxy caches filled", L, ms, fl, nb, dom, peaks, 3)
+                       "P=16..256 two-level, proxy caches filled", L, ms, work, dom, peaks, 3,
+                       clocks=clk(win), rec=rec)
     res["latency_ms"] = ms
     del caches
     torch.cuda.empty_cache()
     # standard prefill, one layer
     std_flops = n * (2 * L * d * 4 * d + 2 * L * L * d)  # projections + causal QK^T and PV
-    floor_ms = std_flops / (peaks["bf16_tflops_sustained"] * 1e12) * 1e3
+    floor_ms = std_flops / (peaks["bf16_tflops"] * 1e12) * 1e3
     std = {"flops": std_flops, "floor_ms_at_measured_peak": floor_ms,
            "impl": "torch scaled_dot_product_attention (fused kernels only) + cuBLAS"}
     try:
@@ -563,6 +702,63 @@ def measure_prefill(torch, pf, S, peaks, warmup, specs, params, st, X):
     res["standard_attention_prefill"] = std
     res["speedup_vs_standard_floor"] = floor_ms / ms
     return res
+
+
+
+
+def run_case(args):
+    """A small run of one workload's step for profiler captures: W warm-up
+    steps, then K steps; prints the mean step time."""
+    import dataclasses
+
+    import torch
+
+    import paper_2608_23463_gb300 as pf
+    import pf_synth as S
+    from paper_2608_23463_gb300.layer import ProxyLayer, to_device
+    pf.build()
+    stream = torch.cuda.current_stream()
+    if args.case == "decode":
+        spec, ms, _, _, _, _ = measure_decode(torch, pf, S, max(args.steps, 1))
+        print(json.dumps({"case": "decode", "ms_per_step": ms}), flush=True)
+        return
+    spec = {"layer": S.spec_c3_layer(64), "c2": S.spec_c2(), "c5": S.spec_c5(),
+            "cross": S.spec_cross_layer(), "lm_history": S.spec_lm_history()}[args.case]
+    if args.batch:
+        spec = dataclasses.replace(spec, batch=args.batch)
+    if args.L:
+        spec = dataclasses.replace(spec, L=args.L)
+    inp = S.make_layer_inputs(spec, 2)
+    lay = ProxyLayer(spec, inp)
+    X = to_device(inp["X"], torch.bfloat16)
+    G = to_device(inp["G"], torch.bfloat16)
+    t = to_device(inp["t"], torch.float32) if "t" in inp else None
+    del inp
+    Xo, dX = lay.empty_act(), lay.empty_act()
+
+    def step():
+        lay.forward(X, None, t, X_out=Xo)
+        lay.backward(X, G, None, t, dX=dX)
+    for _ in range(max(args.warmup, 1)):
+        step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    pf.pf_sync_check(stream.cuda_stream)
+    ms = e0.elapsed_time(e1) / max(args.steps, 1)
+    pf.pf_timing_enable(True)  # per-kernel breakdown of one more step
+    step()
+    torch.cuda.synchronize()
+    t = pf.pf_timing_collect()
+    pf.pf_timing_enable(False)
+    pf.pf_sync_check(stream.cuda_stream)
+    top = sorted(t.items(), key=lambda kv: -kv[1]["ms"])[:10]
+    print(json.dumps({"case": args.case, "batch": spec.batch, "L": spec.L, "ms_per_step": ms,
+                      "kernels_ms": {k: round(v["ms"], 4) for k, v in top}}), flush=True)
 
 
 def load_peaks():
@@ -625,7 +821,7 @@ def run_ours(args, rank: int, world: int, local_rank: int):
         dist.barrier()
     ms = e0.elapsed_time(e1) / args.steps
     pf.pf_sync_check(stream.cuda_stream)
-    clocks = sampler.stop() if sampler else None
+    clocks = sampler.window(sampler.t0, sampler.t1) if sampler else None
     # breakdown pass: the same steps with CUDA events around every launch,
     # scaled to the timed step count
     bsteps = min(args.steps, 10)
@@ -702,39 +898,44 @@ def run_ours(args, rank: int, world: int, local_rank: int):
         torch.cuda.empty_cache()
         decode_result = measure_decode(torch, pf, S, args.decode_steps)
     configs_result = None
+    ffma = measure_ffma_peak(torch, pf) if not args.no_configs else None
     if not args.no_configs:
         if not args.no_decode:
             torch.cuda.empty_cache()
         else:
             del lay, X, G, Xo, dX
             torch.cuda.empty_cache()
-        configs_result = measure_configs(torch, pf, S, load_peaks()[0], max(args.warmup, 3))
+        configs_result = measure_configs(torch, pf, S, load_peaks()[0], max(args.warmup, 3),
+                                         sampler, ffma)
+    if sampler:
+        sampler.stop()
     if rank != 0:
         return
 
     peaks, peak_src = load_peaks()
+    comp_peak, comp_src = compute_peak(peaks, clocks)
     # dominant kernel: largest share of the timed region
     dom, dv = max(timing.items(), key=lambda kv: kv[1]["ms"])
     avg_s = dv["ms"] / dv["launches"] / 1e3
+    units = spec.batch * spec.L
     if dv["flops"] > 0 and not dom.startswith(("inj_bwd", "colsum", "copy", "pad")):
         achieved = dv["flops"] / avg_s / 1e12
-        peak = peaks["bf16_tflops_sustained"]
-        roof = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                "frac": achieved / peak, "traffic": traffic_from_profile(dom, spec.batch * spec.L),
+        roof = {"bound": "tensor", "achieved": achieved, "peak": comp_peak, "unit": "TFLOP/s",
+                "frac": achieved / comp_peak, "traffic": traffic_from_profile(dom, units),
                 "kernel": dom, "launches": dv["launches"], "avg_us": avg_s * 1e6,
                 "flops_per_launch": dv["flops"],
-                "peak_source": f"{peak_src} bf16_tflops_sustained (kernel timed inside a long step)"}
+                "peak_source": f"{peak_src} {comp_src} (of measured)"}
     else:
         achieved = dv["bytes"] / avg_s / 1e9
         peak = peaks["hbm_gbs"]
         roof = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                "frac": achieved / peak, "traffic": traffic_from_profile(dom, spec.batch * spec.L),
+                "frac": achieved / peak, "traffic": traffic_from_profile(dom, units),
                 "kernel": dom, "launches": dv["launches"], "avg_us": avg_s * 1e6,
                 "bytes_per_launch": dv["bytes"], "peak_source": f"{peak_src} hbm_gbs"}
-    step_flops = sum(v["flops"] * v["launches"] for v in timing.values()) / args.steps
-    step_bytes = sum(v["bytes"] * v["launches"] for v in timing.values()) / args.steps
-    roof_ms = max(step_flops / (peaks["bf16_tflops_sustained"] * 1e12),
-                  step_bytes / (peaks["hbm_gbs"] * 1e9)) * 1e3
+    step_flops, step_bytes = layer_work(spec)
+    t_c = step_flops / (comp_peak * 1e12) * 1e3
+    t_b = step_bytes / (peaks["hbm_gbs"] * 1e9) * 1e3
+    roof_ms = max(t_c, t_b)
     total_ms = sum(v["ms"] for v in timing.values())
     breakdown = {k: {"ms_per_step": v["ms"] / args.steps, "share": v["ms"] / total_ms,
                      "launches_per_step": v["launches"] / args.steps}
@@ -745,19 +946,22 @@ def run_ours(args, rank: int, world: int, local_rank: int):
             "data": "synthetic", "config": config_dict(spec),
             "roofline": roof,
             "layer_roofline": {"flops_per_step": step_flops, "bytes_per_step": step_bytes,
+                               "bound": "tensor" if t_c >= t_b else "hbm",
                                "roofline_ms": roof_ms, "frac": roof_ms / ms,
-                               "peaks": f"{peak_src}: bf16 sustained "
-                                        f"{peaks['bf16_tflops_sustained']} TFLOP/s, "
-                                        f"HBM {peaks['hbm_gbs']} GB/s"},
+                               "peaks": f"{peak_src}: bf16 {comp_peak:.1f} TFLOP/s "
+                                        f"({comp_src}), HBM {peaks['hbm_gbs']} GB/s",
+                               "work": "algorithmic (Eq. complexity, Sec. 4)"},
             "e2e": {"value": tokens_per_step / (ms_e2e / 1e3), "unit": UNIT,
                     "h2d_bytes_per_step": 2 * act_bytes, "d2h_bytes_per_step": 2 * act_bytes,
                     "ms_per_step": ms_e2e,
                     "copies": "pinned host X, dX_out in and X_out, dX out every step, on two "
                               "copy streams overlapping the previous / next step's kernels"},
-            "gpu_launches": launches, "clocks": clocks, "kernels": breakdown}
+            "gpu_launches": launches, "clocks": clocks,
+            "kernels": {k: round(v["ms_per_step"], 4) for k, v in list(breakdown.items())[:6]}}
+    detail = {"kernels": breakdown}
     if not args.no_decode:
         dspec, dms, dms_direct, app_ms, dbytes, dkern = decode_result
-        line["decode"] = {
+        dec = {
             "metric": "proxy-KV decode new tokens/s per layer (B=8, 16384 cached proxies, "
                       "d=2048, 16x128 heads, open block 0..63)",
             "value": dspec.batch / (dms / 1e3), "unit": "tokens/s", "ms_per_step": dms,
@@ -769,10 +973,29 @@ def run_ours(args, rank: int, world: int, local_rank: int):
             "timing": "CUDA graph of one step, replayed back to back; events per 64-step span",
             "direct_call_ms_per_step": dms_direct,
             "append_ms": app_ms, "kernels_ms_per_step": dkern}
+        detail["decode"] = dec
+        line["decode"] = {"tok_s": round(dec["value"]), "ms": round(dms, 4),
+                          "frac_hbm": round(dec["roofline"]["frac"], 3),
+                          "direct_ms": round(dms_direct, 4), "append_ms": round(app_ms, 4)}
     if configs_result is not None:
-        line["configs"] = configs_result
+        detail["configs"] = configs_result
+        detail["ffma_tflops_measured"] = ffma
+        compact = {}
+        for k, v in configs_result.items():
+            if "roofline" not in v:
+                compact[k] = v
+                continue
+            r = v["roofline"]
+            compact[k] = {"tok_s": float(f"{v['value']:.4g}"), "ms": round(v["ms_per_step"], 4),
+                          "frac": round(r["frac"], 3), "bound": r["bound"],
+                          "top": r.get("kernel")}
+        compact["ffma_tflops"] = round(ffma, 1) if ffma else None
+        line["configs"] = compact
     if world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline_subprocess()
+    if args.detail:
+        with open(args.detail, "w") as f:
+            json.dump(detail, f, indent=1)
     print(json.dumps(line), flush=True)
 
 
@@ -784,6 +1007,9 @@ def main():
     sys.path.insert(0, ROOT)
     if args.impl == "reference":
         run_reference(args, rank)
+        return
+    if args.case:
+        run_case(args)
         return
     import torch.distributed as dist
     if world > 1:
