@@ -47,7 +47,7 @@ def parse_args():
                     help="skip the other workloads (fp32 layer, L=65536 layer, 2D layer, stack)")
     ap.add_argument("--decode-steps", type=int, default=128)
     ap.add_argument("--case", default="",
-                    choices=("", "layer", "c2", "c5", "cross", "lm_history", "decode"),
+                    choices=("", "layer", "c1", "c2", "c5", "cross", "lm_history", "decode"),
                     help="profiling helper: run only this workload's step (--batch / --L shrink "
                          "it) and print its time; not the benchmark line")
     ap.add_argument("--batch", type=int, default=0, help="batch of --case (default: its own)")
@@ -722,23 +722,26 @@ def run_case(args):
         spec, ms, _, _, _, _ = measure_decode(torch, pf, S, max(args.steps, 1))
         print(json.dumps({"case": "decode", "ms_per_step": ms}), flush=True)
         return
-    spec = {"layer": S.spec_c3_layer(64), "c2": S.spec_c2(), "c5": S.spec_c5(),
+    spec = {"layer": S.spec_c3_layer(64), "c1": S.spec_c1(), "c2": S.spec_c2(), "c5": S.spec_c5(),
             "cross": S.spec_cross_layer(), "lm_history": S.spec_lm_history()}[args.case]
     if args.batch:
         spec = dataclasses.replace(spec, batch=args.batch)
     if args.L:
         spec = dataclasses.replace(spec, L=args.L)
+    train = spec.dtype == S.BF16  # the fp32 layer is forward-only
+    dt = torch.bfloat16 if train else torch.float32
     inp = S.make_layer_inputs(spec, 2)
     lay = ProxyLayer(spec, inp)
-    X = to_device(inp["X"], torch.bfloat16)
-    G = to_device(inp["G"], torch.bfloat16)
+    X = to_device(inp["X"], dt)
+    G = to_device(inp["G"], dt)
     t = to_device(inp["t"], torch.float32) if "t" in inp else None
     del inp
     Xo, dX = lay.empty_act(), lay.empty_act()
 
     def step():
-        lay.forward(X, None, t, X_out=Xo)
-        lay.backward(X, G, None, t, dX=dX)
+        lay.forward(X, None, t, X_out=Xo, train=train)
+        if train:
+            lay.backward(X, G, None, t, dX=dX)
     for _ in range(max(args.warmup, 1)):
         step()
     torch.cuda.synchronize()

@@ -292,7 +292,7 @@ Bwd2DWs carve_bwd_2d(Carve& c, const pf_layer_desc& s, const Dims& g) {
   w.Di = c.take<float>(g.B * g.nh * g.m);
   w.dHq = c.take<float>(g.R * g.d);
   w.dHf = c.take<float>(g.R * g.d);
-  long pe = colsum_part_elems(g.R, (int)(2 * g.N1));
+  long pe = inj_bwd_2d_part_elems(g.R, (int)g.d, s.patch);
   pe = std::max(pe, colsum_part_elems(g.R, (int)g.d));
   pe = std::max(pe, (long)g.B * adaln_param_chunks((int)g.m) * 2 * g.d);
   w.part = c.take<float>(pe);
@@ -378,9 +378,10 @@ pf_status check_desc(const pf_layer_desc* s) {
     if (s->patch < 1 || s->patch * s->patch != s->P || s->grid_h < 1 || s->grid_w < 1 ||
         (long)s->grid_h * s->grid_w != s->L || s->grid_h % s->patch || s->grid_w % s->patch)
       return fail(PF_ERR_INVALID_ARG, "2D layer needs L = grid_h*grid_w, P = patch^2, patch | grid");
-    if (s->inject != PF_INJ_AFFINE || s->levels != 1 || s->dtype != PF_BF16 || s->d % 128 != 0)
-      return fail(PF_ERR_UNSUPPORTED,
-                  "the 2D layer is built for affine injection, one level, bf16, d % 128 == 0");
+    if (s->inject != PF_INJ_AFFINE || s->levels != 1 || s->dtype != PF_BF16 || s->d % 128 != 0 ||
+        s->d > 512)
+      return fail(PF_ERR_UNSUPPORTED, "the 2D layer is built for affine injection, one level, "
+                                      "bf16, d % 128 == 0, d <= 512");
     return PF_OK;
   }
   if (s->inject == PF_INJ_AFFINE) return fail(PF_ERR_UNSUPPORTED, "affine injection is 2D only");
@@ -434,11 +435,10 @@ pf_status layer_fwd_f32(const pf_layer_desc& s, const Dims& g, const pf_layer_pa
                      p.b_d2, nullptr, 0, "decompress_d2", cs, w.sk, w.skb));
     Zsrc = w.Z;
   }
-  PF_CUDA(gemm_f32((int)g.rows1, N1, d, Zsrc, d, static_cast<const float*>(p.W_d1), d, w.D, N1,
-                   p.b_d1, nullptr, 0, "decompress_d1", cs, w.sk, w.skb));
-  PF_CUDA(inject_f32(X, w.D, static_cast<float*>(X_out), p.w_x, p.w_dlt, p.b_g, (int)g.B, g.L, d,
-                     (int)g.P, (int)g.k1, (int)g.k2, (int)g.m, g.causal ? 1 : 0,
-                     s.inject == PF_INJ_GATED ? 1 : 0, cs));
+  PF_CUDA(gemm_f32_inject((int)g.rows1, N1, d, Zsrc, d, static_cast<const float*>(p.W_d1), d,
+                          p.b_d1, X, static_cast<float*>(X_out), p.w_x, p.w_dlt, p.b_g, (int)g.B,
+                          g.L, d, (int)g.P, (int)g.k1, (int)g.k2, (int)g.m, g.causal ? 1 : 0,
+                          s.inject == PF_INJ_GATED ? 1 : 0, cs));
   return PF_OK;
 }
 
@@ -464,8 +464,9 @@ pf_status layer_fwd_2d(const pf_layer_desc& s, const Dims& g, const pf_layer_par
   const int d = (int)g.d, N1 = (int)g.N1;
   const int patch = s.patch, gh = s.grid_h, gw = s.grid_w;
   float* Hf = H_out ? H_out : Hws;
-  PF_CUDA(patch_gather(X, sv.Xp, (int)g.B, d, patch, gh, gw, cs));
-  PF_CUDA(ln_stats(X, sv.stats, g.B * g.L, d, cs));
+  PF_CUDA(patch_gather_stats(X, sv.Xp, sv.stats, (int)g.B, d, patch, gh, gw, cs));
+  // the patch matrix (Eq. partition): X itself through the patch view, else the gathered copy
+
   {
     EpiLinearArgs e;
     e.bias = p.b_c1;
@@ -523,8 +524,8 @@ pf_status layer_bwd_2d(const pf_layer_desc& s, const Dims& g, const pf_layer_par
   const bf16* W_d1 = static_cast<const bf16*>(p.W_d1);
   const bf16* W_c1 = static_cast<const bf16*>(p.W_c1);
   // affine injection backward (Eq. inj-affine)
-  PF_CUDA(inj_bwd_2d(G, X, sv.stats, sv.S, w.dD, w.dXd, g.B * g.L, d, patch, gh, gw, cs));
-  if (gr.b_d1) PF_CUDA(colsum_bf16(w.dD, g.R, N2, gr.b_d1, w.part, cs));
+  PF_CUDA(inj_bwd_2d(G, X, sv.stats, sv.S, w.dD, w.dXd, gr.b_d1, w.part, g.R, d, patch, gh, gw,
+                     cs));
   if (gr.W_d1) {
     EpiLinearArgs e;
     e.out_f32 = gr.W_d1;

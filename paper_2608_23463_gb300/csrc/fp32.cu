@@ -18,19 +18,33 @@ constexpr int FT = 64;   // output tile (FT x FT)
 constexpr int FK = 32;   // K slab
 constexpr int FTHREADS = 256;
 
+// Routing + injection (Eq. inj-gate / inj-add) applied to the last
+// decompression's output instead of storing it: output (row r, column c) of
+// that GEMM is D for token (i + shift) * P + a * k1 + c / d, channel c % d of
+// sequence b, with r = (b * m + i) * k2 + a.
+struct InjF32 {
+  const float* X;    // [B, L, d]
+  float* Xo;         // null: a plain GEMM epilogue
+  const float *w_x, *w_dlt, *b_g;
+  long L;
+  int d, P, k1, k2, m, shift, gated;
+};
+
 // C[M, N] = A[M, K] B[N, K]^T (+ bias[n]) (+ addend[m, n]), all row-major fp32
 // with leading dimensions lda, ldb, ldc.  Each thread computes 4 x 4 outputs.
 // The next K slab is fetched into registers while the current one is used
-// (two shared-memory buffers, one barrier per slab).  With gridDim.z = S > 1
-// each z-slice reduces K range [z*Kc, (z+1)*Kc) and writes raw partials to
-// C + z*M*ldc (bias / addend are then applied by splitk_f32_reduce).
+// (two shared-memory buffers, one barrier per slab); with `vec` the fetch
+// uses 16-byte loads (lda, ldb, the K range and the pointers 4-aligned).
+// With gridDim.z = S > 1 each z-slice reduces K range [z*Kc, (z+1)*Kc) and
+// writes raw partials to C + z*M*ldc (bias / addend are then applied by
+// splitk_f32_reduce).  With inj.Xo the epilogue injects instead of storing C.
 __global__ void __launch_bounds__(FTHREADS) gemm_f32_kernel(const float* __restrict__ A, long lda,
                                                            const float* __restrict__ Bm, long ldb,
                                                            float* __restrict__ C, long ldc, int M,
                                                            int N, int K, int Kc,
                                                            const float* __restrict__ bias,
                                                            const float* __restrict__ addend,
-                                                           long ld_add) {
+                                                           long ld_add, int vec, InjF32 inj) {
   __shared__ __align__(16) float As[2][FK][FT + 4], Bs[2][FK][FT + 4];
   const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
   const int m0 = blockIdx.y * FT, n0 = blockIdx.x * FT;
@@ -43,11 +57,19 @@ __global__ void __launch_bounds__(FTHREADS) gemm_f32_kernel(const float* __restr
 #pragma unroll
     for (int i = 0; i < 2; ++i) {
       const int gm = m0 + lr + 32 * i, gn = n0 + lr + 32 * i;
+      const int gk = k0 + lk;
+      if (vec) {
+        const float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+        const float4 va = (gm < M && gk < kend) ? *reinterpret_cast<const float4*>(A + (long)gm * lda + gk) : z;
+        const float4 vb = (gn < N && gk < kend) ? *reinterpret_cast<const float4*>(Bm + (long)gn * ldb + gk) : z;
+        ra[i][0] = va.x; ra[i][1] = va.y; ra[i][2] = va.z; ra[i][3] = va.w;
+        rb[i][0] = vb.x; rb[i][1] = vb.y; rb[i][2] = vb.z; rb[i][3] = vb.w;
+      } else {
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int gk = k0 + lk + e;
-        ra[i][e] = (gm < M && gk < kend) ? A[(long)gm * lda + gk] : 0.f;
-        rb[i][e] = (gn < N && gk < kend) ? Bm[(long)gn * ldb + gk] : 0.f;
+        for (int e = 0; e < 4; ++e) {
+          ra[i][e] = (gm < M && gk + e < kend) ? A[(long)gm * lda + gk + e] : 0.f;
+          rb[i][e] = (gn < N && gk + e < kend) ? Bm[(long)gn * ldb + gk + e] : 0.f;
+        }
       }
     }
   };
@@ -88,6 +110,28 @@ __global__ void __launch_bounds__(FTHREADS) gemm_f32_kernel(const float* __restr
   for (int i = 0; i < 4; ++i) {
     const int gm = m0 + ty * 4 + i;
     if (gm >= M) continue;
+    if (inj.Xo) {
+      // row gm = (b * m + iprox) * k2 + a: the target block and first token
+      const int a = gm % inj.k2, prox = gm / inj.k2;
+      const int b = prox / inj.m, ip = prox % inj.m + inj.shift;
+      const long tok0 = (long)ip * inj.P + (long)a * inj.k1;
+      if (ip >= inj.m) continue;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int gn = n0 + tx * 4 + j;
+        if (gn >= N) continue;
+        const long t = tok0 + gn / inj.d;
+        if (t >= inj.L) continue;
+        const int ch = gn % inj.d;
+        const float v = acc[i][j] + (bias ? bias[gn] : 0.f);
+        const long o = ((long)b * inj.L + t) * inj.d + ch;
+        const float x = inj.X[o];
+        inj.Xo[o] = inj.gated
+                        ? x + v / (1.f + expf(-(inj.w_x[ch] * x + inj.w_dlt[ch] * v + inj.b_g[ch])))
+                        : x + v;
+      }
+      continue;
+    }
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
       const int gn = n0 + tx * 4 + j;
@@ -271,16 +315,24 @@ int splitk_f32_factor(int M, int N, int K) {
   return std::min(S, 64);
 }
 
+namespace {
+int vec_ok(const float* A, long lda, const float* B, long ldb, int K) {
+  return ((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(B)) & 15) == 0 &&
+         lda % 4 == 0 && ldb % 4 == 0 && K % 4 == 0;
+}
+}  // namespace
+
 cudaError_t gemm_f32(int M, int N, int K, const float* A, long lda, const float* B, long ldb,
                      float* C, long ldc, const float* bias, const float* addend, long ld_add,
                      const char* label, cudaStream_t st, float* scratch, size_t scratch_bytes) {
   const int S = splitk_f32_factor(M, N, K);
+  const int vec = vec_ok(A, lda, B, ldb, K);
   LaunchTimer lt(label, st, 2.0 * M * N * (double)K, 4.0 * ((double)M * K + (double)N * K + (double)M * N));
   if (S > 1 && scratch && (size_t)S * M * N * sizeof(float) <= scratch_bytes) {
     const int Kc = ((K + S - 1) / S + FK - 1) / FK * FK;
     dim3 grid((N + FT - 1) / FT, (M + FT - 1) / FT, S);
     gemm_f32_kernel<<<grid, FTHREADS, 0, st>>>(A, lda, B, ldb, scratch, N, M, N, K, Kc, nullptr,
-                                               nullptr, 0);
+                                               nullptr, 0, vec, InjF32{});
     const long total = (long)M * N;
     splitk_f32_reduce<<<(unsigned)((total + 255) / 256), 256, 0, st>>>(scratch, S, M, N, C, ldc, bias,
                                                                       addend, ld_add);
@@ -288,10 +340,33 @@ cudaError_t gemm_f32(int M, int N, int K, const float* A, long lda, const float*
   }
   dim3 grid((N + FT - 1) / FT, (M + FT - 1) / FT, 1);
   gemm_f32_kernel<<<grid, FTHREADS, 0, st>>>(A, lda, B, ldb, C, ldc, M, N, K, K, bias, addend,
-                                             ld_add);
+                                             ld_add, vec, InjF32{});
   return cudaGetLastError();
 }
 
+cudaError_t gemm_f32_inject(int M, int N, int K, const float* A, long lda, const float* B, long ldb,
+                            const float* bias, const float* X, float* Xo, const float* w_x,
+                            const float* w_dlt, const float* b_g, int Bsz, long L, int d, int P,
+                            int k1, int k2, int m, int shift, int gated, cudaStream_t st) {
+  const int vec = vec_ok(A, lda, B, ldb, K);
+  {
+    LaunchTimer lt("decompress_d1_inject", st, 2.0 * M * N * (double)K,
+                   4.0 * ((double)M * K + (double)N * K) + 12.0 * Bsz * L * (double)d);
+    dim3 grid((N + FT - 1) / FT, (M + FT - 1) / FT, 1);
+    gemm_f32_kernel<<<grid, FTHREADS, 0, st>>>(
+        A, lda, B, ldb, nullptr, 0, M, N, K, K, bias, nullptr, 0, vec,
+        InjF32{X, Xo, w_x, w_dlt, b_g, L, d, P, k1, k2, m, shift, gated});
+  }
+  if (shift > 0) {  // the first block of every sequence receives nothing: X_out = X
+    const long rows = std::min<long>((long)shift * P, L);
+    cudaError_t e = cudaMemcpy2DAsync(Xo, (size_t)L * d * sizeof(float), X,
+                                      (size_t)L * d * sizeof(float),
+                                      (size_t)rows * d * sizeof(float), (size_t)Bsz,
+                                      cudaMemcpyDeviceToDevice, st);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaGetLastError();
+}
 
 cudaError_t attn_f32(const float* qkv, float* out, int B, int m, int d, int nh, bool causal,
                      cudaStream_t st) {

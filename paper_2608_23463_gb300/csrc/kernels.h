@@ -117,16 +117,24 @@ int take_dev_error_elementwise();
 
 // ------------------------------------------------------------- 2D layer
 int take_dev_error_layer2d();
-cudaError_t patch_gather(const bf16* X, bf16* Xp, int B, int d, int patch, int gh, int gw,
-                         cudaStream_t st);
-cudaError_t ln_stats(const bf16* X, float* stats, long T, int d, cudaStream_t st);
+// The patch-order copy Xp [B*m, P*d] of X [B, gh*gw, d] and every token's
+// LayerNorm statistics (mean, 1/std), in one pass over X (d <= 512).
+cudaError_t patch_gather_stats(const bf16* X, bf16* Xp, float* stats, int B, int d, int patch,
+                               int gh, int gw, cudaStream_t st);
+
 cudaError_t temb_fwd(const float* t, int B, int d, const bf16* W_t1, const float* b_t1,
                      const bf16* W_t2, const float* b_t2, float* e, float* a1, float* u, float* gb,
                      cudaStream_t st);
 cudaError_t adaln_fwd(const float* H, const float* gb, float* nH, float* rstd, bf16* Hq, long R,
                       int d, int m, cudaStream_t st);
+// Backward of the affine injection over R patches (d <= 512): dD, the direct
+// dX in patch order, and (db_d1 non-null) the bias gradient of the
+// decompression from per-block partial sums in `part`
+// (inj_bwd_2d_part_elems floats).
+long inj_bwd_2d_part_elems(long R, int d, int patch);
 cudaError_t inj_bwd_2d(const bf16* G, const bf16* X, const float* stats, const bf16* S, bf16* dD,
-                       bf16* dXd, long T, int d, int patch, int gh, int gw, cudaStream_t st);
+                       bf16* dXd, float* db_d1, float* part, long R, int d, int patch, int gh,
+                       int gw, cudaStream_t st);
 cudaError_t adaln_bwd(const float* dHq, const float* nH, const float* rstd, const float* gb,
                       const float* dH_out, float* dHf, bf16* dHb, long R, int d, int m,
                       cudaStream_t st);
@@ -149,6 +157,13 @@ cudaError_t gemm_f32(int M, int N, int K, const float* A, long lda, const float*
                      float* C, long ldc, const float* bias, const float* addend, long ld_add,
                      const char* label, cudaStream_t st, float* scratch = nullptr,
                      size_t scratch_bytes = 0);
+// The last decompression level fused with routing and injection (Eq. inj-gate
+// / inj-add): X_out instead of D; block 0 of every sequence (shift = 1) is
+// copied from X.
+cudaError_t gemm_f32_inject(int M, int N, int K, const float* A, long lda, const float* B, long ldb,
+                            const float* bias, const float* X, float* Xo, const float* w_x,
+                            const float* w_dlt, const float* b_g, int Bsz, long L, int d, int P,
+                            int k1, int k2, int m, int shift, int gated, cudaStream_t st);
 cudaError_t attn_f32(const float* qkv, float* out, int B, int m, int d, int nh, bool causal,
                      cudaStream_t st);
 cudaError_t inject_f32(const float* X, const float* D, float* Xo, const float* w_x,

@@ -18,46 +18,51 @@ __device__ __forceinline__ float warp_sum_f(float v) {
   return v;
 }
 
-// Xp[r, (py*p + px)*d + ch] = X[b, (by*p + py)*gw + bx*p + px, ch] for patch
-// r = (b, by, bx); 16-byte copies.
-__global__ void __launch_bounds__(256) patch_gather_kernel(const bf16* __restrict__ X,
-                                                           bf16* __restrict__ Xp, int d, int patch,
-                                                           int gh, int gw, int per_row) {
-  // grid (x: patch row, y: vectors of one patch row); 16 bytes per thread
-  const int i = blockIdx.y * blockDim.x + threadIdx.x;  // vector within the patch row
-  if (i >= per_row) return;
-  const int row = blockIdx.x;
-  const int dv = d >> 3, p = i / dv, c8 = i - p * dv;
-  const int npw = gw / patch, m = (gh / patch) * npw;
-  const int b = row / m, pr = row - b * m, by = pr / npw, bx = pr - by * npw;
-  const int py = p / patch, px = p - py * patch;
-  const long src = ((long)b * gh * gw + (long)(by * patch + py) * gw + bx * patch + px) * d + c8 * 8;
-  *reinterpret_cast<uint4*>(Xp + (long)row * per_row * 8 + (long)i * 8) =
-      __ldcs(reinterpret_cast<const uint4*>(X + src));
-}
-
-// stats[t] = (mean, 1/sqrt(var + 1e-6)) over the d channels of token t; one
-// warp per token, two passes over the row (the second hits L1).
-__global__ void ln_stats_kernel(const bf16* __restrict__ X, float* __restrict__ stats, long T,
-                                int d) {
+// One pass over the tokens of the 2D layer, one warp per token t = (b, y, x):
+// the patch copy Xp[r, (py*p + px)*d + ch] = X[t, ch] for patch r = (b, by, bx)
+// (Eq. partition, the compression GEMM's operand) and the token's LayerNorm
+// statistics stats[t] = (mean, 1/sqrt(var + 1e-6)) (Eq. inj-affine), from
+// registers (two passes over the row held by the warp).  d <= 512.
+__global__ void __launch_bounds__(256) patch_gather_stats_kernel(
+    const bf16* __restrict__ X, bf16* __restrict__ Xp, float* __restrict__ stats, long T, int d,
+    int patch, int gh, int gw) {
   const long t = ((long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (t >= T) return;
-  const bf16* x = X + t * d;
+  const long HW = (long)gh * gw;
+  const int b = (int)(t / HW), yx = (int)(t % HW), y = yx / gw, x = yx % gw;
+  const int npw = gw / patch, m = (gh / patch) * npw;
+  const long row = (long)b * m + (y / patch) * npw + x / patch;
+  const int p = (y % patch) * patch + (x % patch);
+  const bf16* src = X + t * d;
+  bf16* dst = Xp + row * ((long)patch * patch * d) + (long)p * d;
+  uint4 u[2];
   float s = 0.f;
-  for (int c = lane * 8; c < d; c += 256) {
-    float v[8];
-    load8_bf16(x + c, v);
 #pragma unroll
-    for (int j = 0; j < 8; ++j) s += v[j];
+  for (int i = 0; i < 2; ++i) {
+    const int c = lane * 8 + 256 * i;
+    if (c >= d) break;
+    u[i] = __ldcs(reinterpret_cast<const uint4*>(src + c));
+    *reinterpret_cast<uint4*>(dst + c) = u[i];
+    const uint32_t w[4] = {u[i].x, u[i].y, u[i].z, u[i].w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float2 f = unpack_bf16(w[j]);
+      s += f.x + f.y;
+    }
   }
   const float mu = warp_sum_f(s) / d;
   float q = 0.f;
-  for (int c = lane * 8; c < d; c += 256) {
-    float v[8];
-    load8_bf16(x + c, v);
 #pragma unroll
-    for (int j = 0; j < 8; ++j) q += (v[j] - mu) * (v[j] - mu);
+  for (int i = 0; i < 2; ++i) {
+    const int c = lane * 8 + 256 * i;
+    if (c >= d) break;
+    const uint32_t w[4] = {u[i].x, u[i].y, u[i].z, u[i].w};
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float2 f = unpack_bf16(w[j]);
+      q += (f.x - mu) * (f.x - mu) + (f.y - mu) * (f.y - mu);
+    }
   }
   const float var = warp_sum_f(q) / d;
   if (lane == 0) {
@@ -140,55 +145,106 @@ __global__ void adaln_fwd_kernel(const float* __restrict__ H, const float* __res
 // Backward of X_out = (1 + s) n + t, n = LayerNorm(X), one warp per token:
 // ds = G n, dt = G, dn = G (1 + s), dX = rstd (dn - mean(dn) - n mean(dn n)).
 // dD [B*m, 2*P*d] (patch order: token p of a patch at columns [2pd, 2pd+d) for
-// ds and [2pd+d, 2(p+1)d) for dt) and dXd [B*m, P*d] (patch order).
-__global__ void inj_bwd_2d_kernel(const bf16* __restrict__ G, const bf16* __restrict__ X,
-                                  const float* __restrict__ stats, const bf16* __restrict__ S,
-                                  bf16* __restrict__ dD, bf16* __restrict__ dXd, long T, int d,
-                                  int patch, int gh, int gw) {
-  const long t = ((long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  if (t >= T) return;
-  const long HW = (long)gh * gw;
-  const int b = (int)(t / HW), yx = (int)(t % HW), y = yx / gw, x = yx % gw;
+// ds and [2pd+d, 2(p+1)d) for dt) and dXd [B*m, P*d] (patch order).  A block
+// takes the tokens at one position p of their patch for IB2_CP consecutive
+// patches and also sums its ds and dt over them: part[chunk][2pd + c], the
+// first pass of the deterministic bias gradient (no second read of dD).
+// d <= 512.
+constexpr int IB2_CP = 256;   // patches per block
+constexpr int IB2_MAXI = 2;   // channel groups of 256 per lane: d <= 512
+__global__ void __launch_bounds__(256) inj_bwd_2d_kernel(
+    const bf16* __restrict__ G, const bf16* __restrict__ X, const float* __restrict__ stats,
+    const bf16* __restrict__ S, bf16* __restrict__ dD, bf16* __restrict__ dXd,
+    float* __restrict__ part, long R, int d, int patch, int gh, int gw) {
+  __shared__ float red[8][2 * 256 * IB2_MAXI];
+  const int p = blockIdx.y, chunk = blockIdx.x;
+  const int py = p / patch, px = p % patch;
   const int npw = gw / patch, m = (gh / patch) * npw, P = patch * patch;
-  const long row = (long)b * m + (y / patch) * npw + x / patch;
-  const int p = (y % patch) * patch + (x % patch);
-  const float mu = stats[2 * t], rs = stats[2 * t + 1];
-  const bf16* g = G + t * d;
-  const bf16* xr = X + t * d;
-  const bf16* sr = S + row * ((long)P * d) + (long)p * d;
-  bf16* dds = dD + row * (2L * P * d) + (long)p * 2 * d;
-  bf16* ddt = dds + d;
-  bf16* dxo = dXd + row * ((long)P * d) + (long)p * d;
-  float s1 = 0.f, s2 = 0.f;
-  for (int c = lane * 8; c < d; c += 256) {
-    float gv[8], xv[8], sv[8], o[8];
-    load8_bf16(g + c, gv);
-    load8_bf16(xr + c, xv);
-    load8_bf16(sr + c, sv);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  float cs[IB2_MAXI][8], ct[IB2_MAXI][8];
+#pragma unroll
+  for (int i = 0; i < IB2_MAXI; ++i)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) cs[i][j] = ct[i][j] = 0.f;
+  const long r1 = min(R, (long)(chunk + 1) * IB2_CP);
+  for (long row = (long)chunk * IB2_CP + warp; row < r1; row += 8) {
+    const int b = (int)(row / m), pr = (int)(row % m), by = pr / npw, bx = pr % npw;
+    const long t = ((long)b * gh + by * patch + py) * gw + bx * patch + px;
+    const float mu = stats[2 * t], rs = stats[2 * t + 1];
+    const bf16* g = G + t * d;
+    const bf16* xr = X + t * d;
+    const bf16* sr = S + row * ((long)P * d) + (long)p * d;
+    bf16* dds = dD + row * (2L * P * d) + (long)p * 2 * d;
+    bf16* ddt = dds + d;
+    bf16* dxo = dXd + row * ((long)P * d) + (long)p * d;
+    float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+    for (int i = 0; i < IB2_MAXI; ++i) {
+      const int c = lane * 8 + 256 * i;
+      if (c >= d) break;
+      float gv[8], xv[8], sv[8], o[8];
+      load8_bf16(g + c, gv);
+      load8_bf16(xr + c, xv);
+      load8_bf16(sr + c, sv);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float n = (xv[j] - mu) * rs, dn = gv[j] * (1.f + sv[j]);
+        o[j] = gv[j] * n;
+        s1 += dn;
+        s2 += dn * n;
+        cs[i][j] += o[j];
+        ct[i][j] += gv[j];
+      }
+      store8_bf16(dds + c, o);
+      *reinterpret_cast<uint4*>(ddt + c) = *reinterpret_cast<const uint4*>(g + c);
+    }
+    const float m1 = warp_sum_f(s1) / d, m2 = warp_sum_f(s2) / d;
+#pragma unroll
+    for (int i = 0; i < IB2_MAXI; ++i) {
+      const int c = lane * 8 + 256 * i;
+      if (c >= d) break;
+      float gv[8], xv[8], sv[8], o[8];
+      load8_bf16(g + c, gv);
+      load8_bf16(xr + c, xv);
+      load8_bf16(sr + c, sv);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const float n = (xv[j] - mu) * rs, dn = gv[j] * (1.f + sv[j]);
+        o[j] = rs * (dn - m1 - n * m2);
+      }
+      store8_bf16(dxo + c, o);
+    }
+  }
+  // the block's sums over its patches, in a fixed order (deterministic)
+#pragma unroll
+  for (int i = 0; i < IB2_MAXI; ++i) {
+    const int c = lane * 8 + 256 * i;
+    if (c >= d) break;
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
-      const float n = (xv[j] - mu) * rs, dn = gv[j] * (1.f + sv[j]);
-      o[j] = gv[j] * n;
-      s1 += dn;
-      s2 += dn * n;
+      red[warp][c + j] = cs[i][j];
+      red[warp][d + c + j] = ct[i][j];
     }
-    store8_bf16(dds + c, o);
-    *reinterpret_cast<uint4*>(ddt + c) = *reinterpret_cast<const uint4*>(g + c);
   }
-  const float m1 = warp_sum_f(s1) / d, m2 = warp_sum_f(s2) / d;
-  for (int c = lane * 8; c < d; c += 256) {
-    float gv[8], xv[8], sv[8], o[8];
-    load8_bf16(g + c, gv);
-    load8_bf16(xr + c, xv);
-    load8_bf16(sr + c, sv);
+  __syncthreads();
+  float* dst = part + (long)chunk * (2L * P * d) + (long)p * 2 * d;
+  for (int c = threadIdx.x; c < 2 * d; c += 256) {
+    float v = 0.f;
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const float n = (xv[j] - mu) * rs, dn = gv[j] * (1.f + sv[j]);
-      o[j] = rs * (dn - m1 - n * m2);
-    }
-    store8_bf16(dxo + c, o);
+    for (int w = 0; w < 8; ++w) v += red[w][c];
+    dst[c] = v;
   }
+}
+
+// out[c] = sum over chunks of part[chunk][c] (the bias gradient), one thread
+// per column, chunks in order.
+__global__ void colsum_chunks_kernel(const float* __restrict__ part, int n_chunks, long C,
+                                     float* __restrict__ out) {
+  const long c = (long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (c >= C) return;
+  float v = 0.f;
+  for (int k = 0; k < n_chunks; ++k) v += part[(long)k * C + c];
+  out[c] = v;
 }
 
 // Backward of Hq = (1 + gamma) n + beta, n = LayerNorm(H), one warp per row:
@@ -290,19 +346,13 @@ __global__ void temb_wgrad_kernel(const float* __restrict__ dgb, const float* __
 
 }  // namespace
 
-cudaError_t patch_gather(const bf16* X, bf16* Xp, int B, int d, int patch, int gh, int gw,
-                         cudaStream_t st) {
-  const int per_row = patch * patch * d / 8;  // 16-byte vectors per patch
-  const int rows = B * (gh / patch) * (gw / patch);
-  LaunchTimer lt("patch_gather", st, 0.0, 4.0 * B * gh * gw * (double)d);
-  dim3 grid(rows, (per_row + 255) / 256);
-  patch_gather_kernel<<<grid, 256, 0, st>>>(X, Xp, d, patch, gh, gw, per_row);
-  return cudaGetLastError();
-}
-
-cudaError_t ln_stats(const bf16* X, float* stats, long T, int d, cudaStream_t st) {
-  LaunchTimer lt("ln_stats", st, 0.0, 2.0 * T * d + 8.0 * T);
-  ln_stats_kernel<<<(unsigned)((T * 32 + 255) / 256), 256, 0, st>>>(X, stats, T, d);
+cudaError_t patch_gather_stats(const bf16* X, bf16* Xp, float* stats, int B, int d, int patch,
+                               int gh, int gw, cudaStream_t st) {
+  if (d > 512 || d % 8 != 0) return cudaErrorInvalidValue;
+  const long T = (long)B * gh * gw;
+  LaunchTimer lt("patch_gather_stats", st, 0.0, 4.0 * T * d + 8.0 * T);
+  patch_gather_stats_kernel<<<(unsigned)((T * 32 + 255) / 256), 256, 0, st>>>(X, Xp, stats, T, d,
+                                                                             patch, gh, gw);
   return cudaGetLastError();
 }
 
@@ -322,11 +372,26 @@ cudaError_t adaln_fwd(const float* H, const float* gb, float* nH, float* rstd, b
   return cudaGetLastError();
 }
 
+long inj_bwd_2d_part_elems(long R, int d, int patch) {
+  return (R + IB2_CP - 1) / IB2_CP * 2L * patch * patch * d;
+}
+
 cudaError_t inj_bwd_2d(const bf16* G, const bf16* X, const float* stats, const bf16* S, bf16* dD,
-                       bf16* dXd, long T, int d, int patch, int gh, int gw, cudaStream_t st) {
-  LaunchTimer lt("inj_bwd_2d", st, 0.0, 18.0 * T * d);
-  inj_bwd_2d_kernel<<<(unsigned)((T * 32 + 255) / 256), 256, 0, st>>>(G, X, stats, S, dD, dXd, T, d,
-                                                                      patch, gh, gw);
+                       bf16* dXd, float* db_d1, float* part, long R, int d, int patch, int gh,
+                       int gw, cudaStream_t st) {
+  if (d > 256 * IB2_MAXI || d % 8 != 0) return cudaErrorInvalidValue;
+  const int P = patch * patch;
+  const int n_chunks = (int)((R + IB2_CP - 1) / IB2_CP);
+  {
+    LaunchTimer lt("inj_bwd_2d", st, 0.0, 12.0 * R * P * (double)d);
+    dim3 grid(n_chunks, P);
+    inj_bwd_2d_kernel<<<grid, 256, 0, st>>>(G, X, stats, S, dD, dXd, part, R, d, patch, gh, gw);
+  }
+  if (db_d1) {
+    const long C = 2L * P * d;
+    LaunchTimer lt("colsum_final", st, (double)n_chunks * C, 4.0 * n_chunks * C);
+    colsum_chunks_kernel<<<(unsigned)((C + 255) / 256), 256, 0, st>>>(part, n_chunks, C, db_d1);
+  }
   return cudaGetLastError();
 }
 
