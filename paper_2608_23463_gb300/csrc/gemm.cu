@@ -92,7 +92,7 @@ cudaError_t launch(int M, int N, int K, const CUtensorMap& ta, const CUtensorMap
     // CTA pairs (256 x 256 tiles, half of B per CTA, a deeper stage ring)
     // when every co-resident pair gets a tile
     auto kern2 = gemm_tc_kernel<BN, AMN, BMN, Epi, true>;
-    constexpr int smem2 = GemmCfg<BN, XCOLS, Epi::kColPar, true>::SMEM_BYTES;
+    constexpr int smem2 = GemmCfg<BN, XCOLS, Epi::kColPar, true, Epi::kStageBytes>::SMEM_BYTES;
     constexpr int threads = GemmRoles<Epi>::kThreads;
     cudaError_t e = cudaFuncSetAttribute(kern2, cudaFuncAttributeMaxDynamicSharedMemorySize, smem2);
     if (e != cudaSuccess) return e;
@@ -118,7 +118,7 @@ cudaError_t launch(int M, int N, int K, const CUtensorMap& ta, const CUtensorMap
     }
   }
   auto kern = gemm_tc_kernel<BN, AMN, BMN, Epi>;
-  constexpr int smem = GemmCfg<BN, XCOLS, Epi::kColPar>::SMEM_BYTES;
+  constexpr int smem = GemmCfg<BN, XCOLS, Epi::kColPar, false, Epi::kStageBytes>::SMEM_BYTES;
   cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
   if (e != cudaSuccess) return e;
   const long tiles = (long)((N + BN - 1) / BN) * ((M + GEMM_BM - 1) / GEMM_BM) * splits;
@@ -262,6 +262,13 @@ cudaError_t gemm_linear(int M, int N, int K, Operand A, Operand B, const EpiLine
   if ((e.pre_bf16 && ((uintptr_t)e.pre_bf16 & 15 || e.ld_pre % 8)) ||
       (e.dsilu_of && ((uintptr_t)e.dsilu_of & 15 || e.ld_dsilu % 8)))
     return cudaErrorInvalidValue;
+  // a short contraction with a plain (bias) epilogue stores whole rows from a
+  // shared-memory stage: its output, not its mainloop, would bound it
+  if (K <= 2048 && !e.addend && !e.add_bf16 && !e.act_silu && !e.pre_bf16 && !e.dsilu_of &&
+      (e.out_f32 == nullptr || e.ld_f32 % 4 == 0) && (e.out_bf16 == nullptr || e.ld_bf16 % 8 == 0)) {
+    EpiLinearStaged epi{{}, M, N, e.bias, e.out_f32, e.ld_f32, e.out_bf16, e.ld_bf16};
+    return gemm_dispatch(M, N, K, A, B, epi, nullptr, 0, st);
+  }
   EpiLinear epi{{},         M,          N,          e.bias,      e.addend,  e.ld_add,
                 e.out_f32,  e.ld_f32,   e.out_bf16, e.ld_bf16,   e.add_bf16, e.ld_add_bf16,
                 e.act_silu, e.pre_bf16, e.ld_pre,   e.dsilu_of,  e.ld_dsilu};

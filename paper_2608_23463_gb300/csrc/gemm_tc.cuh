@@ -62,7 +62,8 @@ struct GemmRoles {
 // column in shared memory (two tiles' worth, filled one tile ahead).
 // PAIR: the tile is shared by a CTA pair, each CTA staging half of B.
 constexpr uint32_t GEMM_SMEM_MAX = 232448;  // dynamic shared memory per CTA (227 KB)
-template <int BN, int XCOLS, bool PAR = false, bool PAIR = false>
+// SB: bytes of shared memory the epilogue stages its output in (0: none).
+template <int BN, int XCOLS, bool PAR = false, bool PAIR = false, uint32_t SB = 0>
 struct GemmCfg {
   static constexpr int B_ROWS = PAIR ? BN / 2 : BN;            // B rows staged by one CTA
   static constexpr uint32_t A_BYTES = GEMM_BM * GEMM_BK * 2;  // 16 KB
@@ -70,12 +71,14 @@ struct GemmCfg {
   static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr uint32_t X_BYTES = GEMM_BM * XCOLS * 2;
   static constexpr uint32_t PAR_BYTES = PAR ? 2 * BN * 16 : 0;
-  static constexpr uint32_t FIXED_BYTES = X_BYTES + 1024 /*align*/ + 256 /*barriers*/ + PAR_BYTES;
+  static constexpr uint32_t FIXED_BYTES =
+      X_BYTES + 1024 /*align*/ + 256 /*barriers*/ + PAR_BYTES + SB;
   static constexpr int PAIR_STAGES = (int)((GEMM_SMEM_MAX - FIXED_BYTES) / STAGE_BYTES);
-  static constexpr int STAGES =
-      PAIR ? (PAIR_STAGES < 7 ? PAIR_STAGES : 7)
+  static constexpr int TABLE_STAGES =
+      PAIR ? 7
            : (XCOLS ? (BN == 256 && (XCOLS == 256 || PAR) ? 3 : (BN == 256 ? 4 : 5))
                     : (BN == 256 ? 4 : 6));
+  static constexpr int STAGES = PAIR_STAGES < TABLE_STAGES ? PAIR_STAGES : TABLE_STAGES;
   static constexpr uint32_t SMEM_BYTES = STAGES * STAGE_BYTES + FIXED_BYTES;
   static_assert(SMEM_BYTES <= GEMM_SMEM_MAX, "shared memory");
   static_assert(2 * STAGES + 14 <= 31, "barrier region");
@@ -157,7 +160,7 @@ __global__ void __launch_bounds__(GemmRoles<Epi>::kThreads, 1)
                    Epi epi) {
   static_assert(!PAIR || BN == 256, "CTA pairs use 256-wide tiles");
   constexpr int XCOLS = Epi::kXTile ? (Epi::kPaired ? BN / 2 : BN) : 0;
-  using Cfg = GemmCfg<BN, XCOLS, Epi::kColPar, PAIR>;
+  using Cfg = GemmCfg<BN, XCOLS, Epi::kColPar, PAIR, Epi::kStageBytes>;
   constexpr int STAGES = Cfg::STAGES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -181,6 +184,10 @@ __global__ void __launch_bounds__(GemmRoles<Epi>::kThreads, 1)
     f[12] = p.w;
   };
   __shared__ uint32_t s_consumed;
+  // output staging of the epilogue warps (kStageBytes epilogues), after the
+  // column parameters; other epilogues get the X tile
+  uint8_t* const epi_smem =
+      Epi::kStageBytes ? xtile + Cfg::X_BYTES + 256 + Cfg::PAR_BYTES : xtile;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // a pair (cluster of two CTAs) works on one tile of 2 x 128 rows: `unit` is
@@ -462,7 +469,7 @@ __global__ void __launch_bounds__(GemmRoles<Epi>::kThreads, 1)
           float v[32];
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] = no_k ? 0.f : __uint_as_float(r[i]);
-          epi.apply(ri, erow, n0 + c, v, xtile, rl, c, cp);
+          epi.apply(ri, erow, n0 + c, v, epi_smem, rl, c, cp);
         };
         uint32_t ra[32], rb[32];
         tmem_ld32_async(trow + (uint32_t)c_begin, ra);
@@ -560,6 +567,8 @@ struct EpiBase {
   // slower than its mainloop does better on single CTAs, whose tiles do not
   // wait for the other CTA's epilogue
   static constexpr bool kPairs = true;
+  // shared memory for staging the output (0: the epilogue stores from registers)
+  static constexpr uint32_t kStageBytes = 0;
   __device__ __forceinline__ float4 col_param(int, int) const { return make_float4(0, 0, 0, 0); }
   __device__ __forceinline__ int x_row(int m0) const { return m0; }
   __device__ __forceinline__ int x_col(int n0, int j) const { return n0 + 64 * j; }
@@ -657,6 +666,67 @@ struct EpiLinear : EpiBase {
 #pragma unroll
       for (int i = 0; i < 32; i += 8) store8_bf16(o + i, v + i);
     }
+  }
+};
+
+// A linear epilogue (v = acc + bias, fp32 and / or bf16 out) that stores
+// whole rows: each warp stages its 32 x 32 chunk in shared memory (rows 36
+// floats apart, so neither the row-per-lane writes nor the row reads conflict)
+// and writes it back row by row, 128 contiguous bytes of fp32 per row.
+// Used where the output is large next to the contraction (short K), so that
+// the stores from one row per lane would bound the epilogue.
+struct EpiLinearStaged : EpiBase {
+  static constexpr int kRowF = 36;  // floats per staged row
+  static constexpr uint32_t kStageBytes = GEMM_EPI_WARPS * 32 * kRowF * 4;
+  struct Row {
+    bool ok;
+  };
+  int M, N;
+  const float* bias;
+  float* out_f32;
+  long ld_f32;
+  bf16* out_bf16;
+  long ld_bf16;
+  __device__ __forceinline__ Row row_info(int row, int) const { return Row{row < M}; }
+  __device__ __forceinline__ void apply(const Row&, int row, int col, float* v, uint8_t* stg,
+                                        int rl, int, const float4*) const {
+    if (col >= N) return;  // uniform across the warp
+    const int lane = threadIdx.x & 31, ew = (threadIdx.x >> 5) - 2;
+    float* s = reinterpret_cast<float*>(stg) + ew * (32 * kRowF);
+    if (bias) {
+#pragma unroll
+      for (int i = 0; i < 32; i += 4) {
+        const float4 b = *reinterpret_cast<const float4*>(bias + col + i);
+        v[i] += b.x; v[i + 1] += b.y; v[i + 2] += b.z; v[i + 3] += b.w;
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 32; i += 4)
+      *reinterpret_cast<float4*>(s + lane * kRowF + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+    __syncwarp();
+    const int rfirst = row - (rl & 31);
+    if (out_f32) {  // 8 lanes per row, 4 rows per instruction
+#pragma unroll
+      for (int it = 0; it < 8; ++it) {
+        const int rr = it * 4 + (lane >> 3), pc = (lane & 7) * 4;
+        const float4 val = *reinterpret_cast<const float4*>(s + rr * kRowF + pc);
+        if (rfirst + rr < M)
+          *reinterpret_cast<float4*>(out_f32 + (long)(rfirst + rr) * ld_f32 + col + pc) = val;
+      }
+    }
+    if (out_bf16) {  // 4 lanes per row (8 values each), 8 rows per instruction
+#pragma unroll
+      for (int it = 0; it < 4; ++it) {
+        const int rr = it * 8 + (lane >> 2), pc = (lane & 3) * 8;
+        const float4 a = *reinterpret_cast<const float4*>(s + rr * kRowF + pc);
+        const float4 b = *reinterpret_cast<const float4*>(s + rr * kRowF + pc + 4);
+        if (rfirst + rr < M)
+          *reinterpret_cast<uint4*>(out_bf16 + (long)(rfirst + rr) * ld_bf16 + col + pc) =
+              make_uint4(pack_bf16(a.x, a.y), pack_bf16(a.z, a.w), pack_bf16(b.x, b.y),
+                         pack_bf16(b.z, b.w));
+      }
+    }
+    __syncwarp();  // the staging is reused by the next chunk
   }
 };
 
