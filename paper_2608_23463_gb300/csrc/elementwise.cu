@@ -421,29 +421,16 @@ __global__ void __launch_bounds__(EW_THREADS) colsum_part_kernel(const T* __rest
   *reinterpret_cast<float4*>(p + 4) = make_float4(acc[4], acc[5], acc[6], acc[7]);
 }
 
-// out[c] = sum over chunks of part[chunk][c]: a block per 32 columns, warp w
-// sums the chunks w, w + 8, ... with one column per lane (coalesced rows of
-// the partials), then the eight warp sums are added in a fixed order
-// (deterministic).
-__global__ void __launch_bounds__(256) colsum_final_kernel(const float* __restrict__ part,
-                                                           int n_chunks, int C,
-                                                           float* __restrict__ out) {
-  __shared__ float red[8][32];
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int c = blockIdx.x * 32 + lane;
+// One warp per column (deterministic order, see warp_sum).
+__global__ void colsum_final_kernel(const float* __restrict__ part, int n_chunks, int C,
+                                    float* __restrict__ out) {
+  const int i = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (i >= C) return;
   float s = 0.f;
-  if (c < C) {
-#pragma unroll 4
-    for (int k = warp; k < n_chunks; k += 8) s += part[(long)k * C + c];
-  }
-  red[warp][lane] = s;
-  __syncthreads();
-  if (warp == 0 && c < C) {
-    float v = 0.f;
-#pragma unroll
-    for (int w = 0; w < 8; ++w) v += red[w][lane];
-    out[c] = v;
-  }
+  for (int c = lane; c < n_chunks; c += 32) s += part[(long)c * C + i];
+  s = warp_sum(s);
+  if (lane == 0) out[i] = s;
 }
 
 // Row chunks of a column reduction: about 1024 CTAs in total, independent of
@@ -467,7 +454,7 @@ cudaError_t colsum_impl(const T* X, long R, int C, float* out, float* part, cuda
   }
   {
     LaunchTimer lt("colsum_final", st, (double)nc * C, 4.0 * nc * C);
-    colsum_final_kernel<<<(C + 31) / 32, 256, 0, st>>>(part, nc, C, out);
+    colsum_final_kernel<<<(C + 7) / 8, 256, 0, st>>>(part, nc, C, out);
   }
   return cudaGetLastError();
 }
