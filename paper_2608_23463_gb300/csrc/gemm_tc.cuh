@@ -465,10 +465,14 @@ __global__ void __launch_bounds__(GemmRoles<Epi>::kThreads, 1)
         // 32-column chunks, the TMEM load of chunk i+1 in flight while chunk i
         // is processed
         constexpr int NCH = BN / 64;
-        auto run = [&](const uint32_t* r, int c) {
+        auto run = [&](uint32_t* r, int c) {
+          if (no_k) {  // uniform: a split with no K blocks
+#pragma unroll
+            for (int i = 0; i < 32; ++i) r[i] = 0u;
+          }
           float v[32];
 #pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] = no_k ? 0.f : __uint_as_float(r[i]);
+          for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
           epi.apply(ri, erow, n0 + c, v, epi_smem, rl, c, cp);
         };
         uint32_t ra[32], rb[32];
@@ -782,59 +786,86 @@ struct EpiInject1D : EpiBase {
   }
   // The warp's 32 x 32 chunk of X_out and then of D is staged in the X tile
   // cells it has just read and stored with whole-row segments.  cp: the
-  // staged parameters, one float4 per (4-column group, parameter).
+  // staged parameters, one float4 per (4-column group, parameter).  The gate
+  // arithmetic runs on column pairs with packed fp32x2 FMAs (each lane an
+  // IEEE fp32 FMA, as the scalar form), and the cell addresses are formed
+  // once per chunk.
   __device__ __forceinline__ void apply(const Row& ri, int row, int col, float* v, uint8_t* xt,
                                         int rl, int cl, const float4* cp) const {
     if (col >= N) return;  // uniform across the warp
-    const int q = rl >> 5;
+    const int lane = threadIdx.x & 31, q = rl >> 5;
     const float4* cg = cp + (cl >> 2) * 4;
+    // this row's four 16-byte cells of the chunk (128-byte swizzle)
+    const int c8 = (cl & 63) >> 3, sw = rl & 7;
+    uint8_t* const rowp = xt + (cl >> 6) * 16384 + rl * 128;
+    uint4* cell[4];
 #pragma unroll
-    for (int i4 = 0; i4 < 8; ++i4) {  // D = acc + bias
-      const float4 b = cg[i4 * 4];
-      v[4 * i4] += b.x;
-      v[4 * i4 + 1] += b.y;
-      v[4 * i4 + 2] += b.z;
-      v[4 * i4 + 3] += b.w;
-    }
+    for (int j = 0; j < 4; ++j) cell[j] = reinterpret_cast<uint4*>(rowp + (((c8 | j) ^ sw) << 4));
+    uint32_t dpk[16];  // D = acc + bias, bf16 pairs
 #pragma unroll
-    for (int i8 = 0; i8 < 32; i8 += 8) {
-      float x[8], o[8];
-      xtile_load8(xt, rl, cl + i8, x);
-      if (gated) {
+    for (int j = 0; j < 4; ++j) {
+      const uint4 xu = *cell[j];
+      const uint32_t xw[4] = {xu.x, xu.y, xu.z, xu.w};
+      uint32_t ow[4];
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int g4 = (i8 >> 2) + h;
-          const float4 wx = cg[g4 * 4 + 1], wd = cg[g4 * 4 + 2], bg = cg[g4 * 4 + 3];
-          const float wxa[4] = {wx.x, wx.y, wx.z, wx.w}, wda[4] = {wd.x, wd.y, wd.z, wd.w},
-                      bga[4] = {bg.x, bg.y, bg.z, bg.w};
-#pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            const int e = h * 4 + j;
-            const float g = fmaf(wxa[j], x[e], fmaf(wda[j], v[i8 + e], bga[j]));
-            o[e] = fmaf(sigmoidf_(g), v[i8 + e], x[e]);
-          }
+      for (int h = 0; h < 2; ++h) {
+        const int g4 = 2 * j + h;  // 4-column group of the chunk
+        const float4 b = cg[g4 * 4];
+        const float bb[4] = {b.x, b.y, b.z, b.w};
+        float wx[4], wd[4], bg[4];
+        if (gated) {
+          const float4 a = cg[g4 * 4 + 1], dd = cg[g4 * 4 + 2], e = cg[g4 * 4 + 3];
+          wx[0] = a.x; wx[1] = a.y; wx[2] = a.z; wx[3] = a.w;
+          wd[0] = dd.x; wd[1] = dd.y; wd[2] = dd.z; wd[3] = dd.w;
+          bg[0] = e.x; bg[1] = e.y; bg[2] = e.z; bg[3] = e.w;
         }
-      } else {
 #pragma unroll
-        for (int j = 0; j < 8; ++j) o[j] = x[j] + v[i8 + j];
+        for (int pr = 0; pr < 2; ++pr) {
+          const int e0 = 8 * j + 4 * h + 2 * pr, k = 2 * pr;
+          const float2 x2 = unpack_bf16(xw[2 * h + pr]);
+          const float2 d2 = __fadd2_rn(make_float2(v[e0], v[e0 + 1]), make_float2(bb[k], bb[k + 1]));
+          float2 o2;
+          if (gated) {
+            const float2 g2 = __ffma2_rn(make_float2(wx[k], wx[k + 1]), x2,
+                                         __ffma2_rn(make_float2(wd[k], wd[k + 1]), d2,
+                                                    make_float2(bg[k], bg[k + 1])));
+            const float2 hg = __fmul2_rn(g2, make_float2(0.5f, 0.5f));
+            const float2 t2 = make_float2(tanh_approx(hg.x), tanh_approx(hg.y));
+            const float2 s2 = __ffma2_rn(make_float2(0.5f, 0.5f), t2, make_float2(0.5f, 0.5f));
+            o2 = __ffma2_rn(s2, d2, x2);
+          } else {
+            o2 = __fadd2_rn(x2, d2);
+          }
+          ow[2 * h + pr] = pack_bf16(o2.x, o2.y);
+          dpk[(e0 >> 1)] = pack_bf16(d2.x, d2.y);
+        }
       }
-      xtile_put8(xt, rl, cl + i8, o);
+      *cell[j] = make_uint4(ow[0], ow[1], ow[2], ow[3]);
     }
     __syncwarp();
-    warp_store_rows(xt, q, cl, [&](int rr, int p) -> bf16* {
-      const int it = rr >> 3;
-      return col + p * 8 < ri.seg.lim[it] ? X_out + ri.seg.off[it] + col + p * 8 : nullptr;
-    });
+    // whole-row stores: instruction it writes rows 8 it + lane / 4 of the warp,
+    // 16-byte piece p = lane % 4; the swizzle phase of those rows is lane / 4
+    const int p = lane & 3, rq = lane >> 2;
+    const uint8_t* srow = xt + (cl >> 6) * 16384 + (q * 32 + rq) * 128 + (((c8 | p) ^ rq) << 4);
+#pragma unroll
+    for (int it = 0; it < 4; ++it) {
+      const uint4 val = *reinterpret_cast<const uint4*>(srow + it * 8 * 128);
+      if (col + p * 8 < ri.seg.lim[it])
+        *reinterpret_cast<uint4*>(X_out + ri.seg.off[it] + col + p * 8) = val;
+    }
     __syncwarp();
     if (D_save) {
 #pragma unroll
-      for (int i8 = 0; i8 < 32; i8 += 8) xtile_put8(xt, rl, cl + i8, v + i8);
+      for (int j = 0; j < 4; ++j)
+        *cell[j] = make_uint4(dpk[4 * j], dpk[4 * j + 1], dpk[4 * j + 2], dpk[4 * j + 3]);
       __syncwarp();
       const int rfirst = row - (rl & 31);
-      warp_store_rows(xt, q, cl, [&](int rr, int p) -> bf16* {
-        const int r2 = rfirst + rr;
-        return r2 < M ? D_save + (long)r2 * N + col + p * 8 : nullptr;
-      });
+      bf16* dbase = D_save + (long)(rfirst + rq) * N + col + p * 8;
+#pragma unroll
+      for (int it = 0; it < 4; ++it) {
+        const uint4 val = *reinterpret_cast<const uint4*>(srow + it * 8 * 128);
+        if (rfirst + rq + 8 * it < M) *reinterpret_cast<uint4*>(dbase + (long)it * 8 * N) = val;
+      }
       __syncwarp();
     }
   }
