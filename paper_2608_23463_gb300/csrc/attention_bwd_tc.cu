@@ -148,8 +148,8 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
       mbar_init(x_full + 8 * i, 1);
       mbar_init(x_empty + 8 * i, 1);
       mbar_init(t_full + 8 * i, 1);
-      mbar_init(t_free + 8 * i, BW_ROW_THREADS);
-      mbar_init(e_full + 8 * i, BW_ROW_THREADS);
+      mbar_init(t_free + 8 * i, BW_ROW_THREADS / 32);  // one arrival per row warp
+      mbar_init(e_full + 8 * i, BW_ROW_THREADS / 32);
       mbar_init(e_free + 8 * i, 1);
     }
     for (int i = 0; i < BW_STAGES; ++i) {
@@ -157,7 +157,7 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
       mbar_init(y_empty + 8 * i, 1);
     }
     mbar_init(acc_full, 1);
-    mbar_init(acc_free, BW_ROW_THREADS);
+    mbar_init(acc_free, BW_ROW_THREADS / 32);
     mbar_init(done, 1);
     fence_barrier_init();
   }
@@ -351,7 +351,7 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
         tmem_wait_ld(s1);
         tmem_wait_ld(p1);
         tc_fence_before();
-        mbar_arrive(t_free + 8 * tb);
+        mbar_arrive_warp(t_free + 8 * tb);
         // valid streamed columns: [lo, hi)
         int lo = 0, hi = min(BW_N, a.Ly - c0);
         if (DKDV)
@@ -413,7 +413,7 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
         tmem_st16(te + 32, dk);
         tmem_wait_st();
         tc_fence_before();
-        mbar_arrive(e_full + 8 * tb);
+        mbar_arrive_warp(e_full + 8 * tb);
       }
       if (DKDV) ok = bar_rows_and(ok);
       if (!ok) break;
@@ -429,7 +429,7 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
       tmem_wait_ld(u0);
       if (DKDV) tmem_wait_ld(w0);
       tc_fence_before();
-      mbar_arrive(acc_free);
+      mbar_arrive_warp(acc_free);
       if (row < a.Lx) {
         const long srow = (long)b * a.Lx + row;
         bf16* pu = a.out_u + srow * a.ld_u + a.col_u + h * BW_D + 32 * ch;

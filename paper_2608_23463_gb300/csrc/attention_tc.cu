@@ -135,11 +135,11 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       mbar_init(q_full + 8 * i, 1);
       mbar_init(q_empty + 8 * i, 1);
       mbar_init(s_full(i), 1);
-      mbar_init(s_free(i), 128);
-      mbar_init(p_full(i), 128);
+      mbar_init(s_free(i), 4);  // one arrival per softmax warp of the group
+      mbar_init(p_full(i), 4);
       mbar_init(p_free(i), 1);
       mbar_init(o_full(i), 1);
-      mbar_init(o_free(i), 128);
+      mbar_init(o_free(i), 4);
     }
     for (int i = 0; i < FA_STAGES; ++i) {
       mbar_init(kv_full + 8 * i, 1);
@@ -390,12 +390,12 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
           }
         }
         tc_fence_before();
-        mbar_arrive(s_free(w));  // this group's scores are no longer read
+        mbar_arrive_warp(s_free(w));  // this group's scores are no longer read
         l = fmaf(l, corr, psum);
         mref = mnew;
         tmem_wait_st();
         tc_fence_before();
-        mbar_arrive(p_full(w));
+        mbar_arrive_warp(p_full(w));
       }
       if (!ok) break;
       // the item's O: after its last P.V
@@ -408,7 +408,7 @@ __global__ void __launch_bounds__(FA_THREADS, 1)
       tmem_wait_ld(ov);
       tmem_wait_ld(ov + 32);
       tc_fence_before();
-      mbar_arrive(o_free(w));
+      mbar_arrive_warp(o_free(w));
       if (q < a.Lq) {
         const float inv = l > 0.f ? 1.f / l : 0.f;  // a row that sees no key: 0
         const long row = (long)b * a.Lq + q;

@@ -115,6 +115,14 @@ __device__ __forceinline__ bool mbar_wait_warp(uint32_t bar, uint32_t parity) {
   return __all_sync(0xffffffffu, mbar_wait(bar, parity));
 }
 
+// One arrival for a converged warp (barriers counted in warps): every lane's
+// earlier accesses, and after a tcgen05.fence::before_thread_sync its tensor
+// memory accesses, are ordered before lane 0's arrive by the warp barrier.
+__device__ __forceinline__ void mbar_arrive_warp(uint32_t bar) {
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) mbar_arrive(bar);
+}
+
 // True in exactly one lane of a converged warp (elect.sync's leader).  An MMA
 // issuer that runs its loop on the whole warp and issues from this lane keeps
 // its operand arithmetic warp-uniform, which issues tcgen05.mma at the tensor
