@@ -12,9 +12,10 @@
 //   DQ:   item = (128-query tile, head, sequence); stationary X1 = Q, X2 = dO;
 //         streamed 64-key tiles Y1 = K_j, Y2 = V_j.
 //           T1 = S,  T2 = dP,  E2 = dS,  dQ += E2 Y1
-// Roles: warp 0 TMA producer, warp 1 MMA issuer, warps 2-9 the row warps: two
-// per TMEM lane quarter, each thread one row (TMEM lane) and one half of the
-// 64 streamed columns.  T1/T2 and E are double-buffered so the MMAs of step
+// Roles: warp 0 TMA producer (DKDV: it also stages each step's (LSE, Di)
+// pairs of the streamed queries in shared memory), warp 1 MMA issuer, warps
+// 2-9 the row warps: two per TMEM lane quarter, each thread one row (TMEM
+// lane) and one half of the 64 streamed columns.  T1/T2 and E are double-buffered so the MMAs of step
 // j+1 overlap the row work of step j.  E stays in TMEM as the A operand of the
 // accumulating MMAs, so those read only their B tile from shared memory
 // (shared-memory bandwidth, not the tensor pipe, bounds M=128 N=64 MMAs whose
@@ -44,7 +45,7 @@ constexpr uint32_t BW_X_BYTES = BW_M * BW_D * 2;  // 16 KB per stationary tile
 constexpr uint32_t BW_Y_BYTES = BW_N * BW_D * 2;  // 8 KB per streamed tile
 constexpr uint32_t BW_OFF_Y = 2 * 2 * BW_X_BYTES;                       // X: [2 bufs][X1, X2]
 constexpr uint32_t BW_OFF_LD = BW_OFF_Y + BW_STAGES * 2 * BW_Y_BYTES;  // Y: [stage][Y1, Y2]
-constexpr uint32_t BW_OFF_BAR = BW_OFF_LD + 2 * BW_N * 8;              // (lse, Di) [2][64]
+constexpr uint32_t BW_OFF_BAR = BW_OFF_LD + BW_STAGES * BW_N * 8;      // (lse, Di) [stage][64]
 constexpr uint32_t BW_SMEM = BW_OFF_BAR + 256 + 1024;
 // TMEM columns: T1 at 0 / 64, T2 at 128 / 192 (fp32, per buffer), accumulators
 // at 256 (dV or dQ) and 320 (dK), E at 384 / 448 (per buffer: E1 at +0, E2 at
@@ -80,21 +81,6 @@ __device__ __forceinline__ float ex2_approx(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
-}
-
-// Barrier of the row threads (named barrier 1) that ANDs a predicate across
-// them, so that they leave their loops together.
-__device__ __forceinline__ bool bar_rows_and(bool p) {
-  uint32_t r;
-  asm volatile(
-      "{\n\t.reg .pred pi, po;\n\t"
-      "setp.ne.u32 pi, %1, 0;\n\t"
-      "bar.red.and.pred po, 1, 256, pi;\n\t"
-      "selp.u32 %0, 1, 0, po;\n\t}"
-      : "=r"(r)
-      : "r"((uint32_t)p)
-      : "memory");
-  return r != 0;
 }
 
 // Snake order over the CTAs of items ranked heaviest first.
@@ -171,38 +157,82 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
   const uint32_t tmem = *tmem_slot;
   uint32_t y_issued = 0, x_issued = 0;
 
-  if (warp == 0 && lane == 0) {
+  if (warp == 0) {
     // ------------------------------------------------------------ producer
-    prefetch_tmap(&tmX1);
-    prefetch_tmap(&tmX2);
-    prefetch_tmap(&tmY1);
-    prefetch_tmap(&tmY2);
+    // Lane 0 issues the copies.  DKDV: the whole warp also stages the (lse,
+    // Di) pairs of each step's 64 streamed queries in the stage's slot before
+    // lane 0 arms the stage's full barrier, so that the row warps read them
+    // after that barrier (the values for the next step are loaded one step
+    // ahead, two queries per lane).
+    if (lane == 0) {
+      prefetch_tmap(&tmX1);
+      prefetch_tmap(&tmX2);
+      prefetch_tmap(&tmY1);
+      prefetch_tmap(&tmY2);
+    }
+    float2* ld_ring = reinterpret_cast<float2*>(smem + BW_OFF_LD);
+    auto fetch_ld = [&](int b, int h, int q0, int c) -> float2 {
+      const int qq = q0 + c;
+      if (qq >= a.Lq) return make_float2(0.f, 0.f);
+      const long o = ((long)b * a.nh + h) * a.Lq + qq;
+      return make_float2(a.lse[o], a.Di[o]);
+    };
+    float2 ld0 = make_float2(0.f, 0.f), ld1 = ld0;  // next step's pairs of queries lane, lane + 32
+    int k = bw_rank(blockIdx.x, 0);
+    if (DKDV && k < a.n_items) {
+      int t, h, b, j0, n;
+      bw_item<DKDV>(a, k, t, h, b, j0, n);
+      ld0 = fetch_ld(b, h, j0 * BW_N, lane);
+      ld1 = fetch_ld(b, h, j0 * BW_N, lane + 32);
+    }
     bool ok = true;
     uint32_t it = 0;
-    for (int rd = 0, k = bw_rank(blockIdx.x, 0); k < a.n_items && ok;
-         k = bw_rank(blockIdx.x, ++rd), ++it) {
+    for (int rd = 0; k < a.n_items && ok; k = bw_rank(blockIdx.x, ++rd), ++it) {
       int t, h, b, j0, n;
       bw_item<DKDV>(a, k, t, h, b, j0, n);
       const int row0 = b * a.Lx;
       const uint32_t xb = it & 1;
-      if (!mbar_wait(x_empty + 8 * xb, ((it >> 1) & 1) ^ 1)) break;
-      const uint32_t xdst = sbase + xb * 2 * BW_X_BYTES;
-      mbar_arrive_expect_tx(x_full + 8 * xb, 2 * BW_X_BYTES);
-      tma_load_2d(xdst, &tmX1, x_full + 8 * xb, x1c + h * BW_D, row0 + t * BW_M);
-      tma_load_2d(xdst + BW_X_BYTES, &tmX2, x_full + 8 * xb, x2c + h * BW_D, row0 + t * BW_M);
+      if (!mbar_wait_warp(x_empty + 8 * xb, ((it >> 1) & 1) ^ 1)) break;
+      if (lane == 0) {
+        const uint32_t xdst = sbase + xb * 2 * BW_X_BYTES;
+        mbar_arrive_expect_tx(x_full + 8 * xb, 2 * BW_X_BYTES);
+        tma_load_2d(xdst, &tmX1, x_full + 8 * xb, x1c + h * BW_D, row0 + t * BW_M);
+        tma_load_2d(xdst + BW_X_BYTES, &tmX2, x_full + 8 * xb, x2c + h * BW_D, row0 + t * BW_M);
+      }
       x_issued = it + 1;
       for (int j = 0; j < n; ++j) {
         const uint32_t G = y_issued, st = G % BW_STAGES;
-        if (!mbar_wait(y_empty + 8 * st, ((G / BW_STAGES) & 1) ^ 1)) {
+        if (!mbar_wait_warp(y_empty + 8 * st, ((G / BW_STAGES) & 1) ^ 1)) {
           ok = false;
           break;
         }
-        const uint32_t ydst = sbase + BW_OFF_Y + st * 2 * BW_Y_BYTES;
-        const int yrow = b * a.Ly + (j0 + j) * BW_N;
-        mbar_arrive_expect_tx(y_full + 8 * st, 2 * BW_Y_BYTES);
-        tma_load_2d(ydst, &tmY1, y_full + 8 * st, y1c + h * BW_D, yrow);
-        tma_load_2d(ydst + BW_Y_BYTES, &tmY2, y_full + 8 * st, y2c + h * BW_D, yrow);
+        if (DKDV) {
+          ld_ring[st * BW_N + lane] = ld0;
+          ld_ring[st * BW_N + 32 + lane] = ld1;
+          __syncwarp();
+        }
+        if (lane == 0) {
+          const uint32_t ydst = sbase + BW_OFF_Y + st * 2 * BW_Y_BYTES;
+          const int yrow = b * a.Ly + (j0 + j) * BW_N;
+          mbar_arrive_expect_tx(y_full + 8 * st, 2 * BW_Y_BYTES);
+          tma_load_2d(ydst, &tmY1, y_full + 8 * st, y1c + h * BW_D, yrow);
+          tma_load_2d(ydst + BW_Y_BYTES, &tmY2, y_full + 8 * st, y2c + h * BW_D, yrow);
+        }
         y_issued = G + 1;
+        if (DKDV) {  // the pairs of the next step (this item's or the next item's first)
+          if (j + 1 < n) {
+            ld0 = fetch_ld(b, h, (j0 + j + 1) * BW_N, lane);
+            ld1 = fetch_ld(b, h, (j0 + j + 1) * BW_N, lane + 32);
+          } else {
+            const int k2 = bw_rank(blockIdx.x, rd + 1);
+            if (k2 < a.n_items) {
+              int t2, h2, b2, j02, n2;
+              bw_item<DKDV>(a, k2, t2, h2, b2, j02, n2);
+              ld0 = fetch_ld(b2, h2, j02 * BW_N, lane);
+              ld1 = fetch_ld(b2, h2, j02 * BW_N, lane + 32);
+            }
+          }
+        }
       }
     }
   } else if (warp == 1) {
@@ -284,29 +314,13 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
     // ------------------------------------------------------------ row warps
     const int q4 = warp & 3;
     const int r = q4 * 32 + lane;  // stationary row in the tile = TMEM lane
-    const int tr = threadIdx.x - 64;  // 0..255
     const int ch = (warp - 2) >> 2;   // half of the streamed columns: [32 ch, 32 ch + 32)
     const uint32_t tl = tmem + ((uint32_t)(q4 * 32) << 16);
-    float2* ld_s = reinterpret_cast<float2*>(smem + BW_OFF_LD);  // [2][64] (lse, Di)
+    const float2* ld_ring = reinterpret_cast<const float2*>(smem + BW_OFF_LD);  // [stage][64]
     bool ok = true;
     uint32_t G = 0, it = 0;
-    // DKDV: (lse, Di) of the streamed queries, one step ahead: thread tr < 64
-    // fetches column tr of the next step
-    auto fetch_ld = [&](int b, int h, int q0, int c) -> float2 {
-      const int qq = q0 + c;
-      if (c >= BW_N || qq >= a.Lq) return make_float2(0.f, 0.f);
-      const long o = ((long)b * a.nh + h) * a.Lq + qq;
-      return make_float2(a.lse[o], a.Di[o]);
-    };
-    int rd = 0;
-    int k = bw_rank(blockIdx.x, 0);
-    float2 ld_next = make_float2(0.f, 0.f);
-    if (DKDV && k < a.n_items) {
-      int t, h, b, j0, n;
-      bw_item<DKDV>(a, k, t, h, b, j0, n);
-      ld_next = fetch_ld(b, h, j0 * BW_N, tr);
-    }
-    for (; k < a.n_items && ok; k = bw_rank(blockIdx.x, ++rd), ++it) {
+    for (int rd = 0, k = bw_rank(blockIdx.x, 0); k < a.n_items && ok;
+         k = bw_rank(blockIdx.x, ++rd), ++it) {
       int t, h, b, j0, n;
       bw_item<DKDV>(a, k, t, h, b, j0, n);
       const int row = t * BW_M + r;  // key (DKDV) or query (DQ) index in the sequence
@@ -319,29 +333,15 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
       for (int j = 0; j < n; ++j) {
         const uint32_t Gj = G + j, tb = Gj & 1;
         const int c0 = (j0 + j) * BW_N;  // first streamed index of this step
-        if (DKDV) {
-          // publish this step's (lse, Di); fetch the next step's.  A thread
-          // whose wait ran out reaches this barrier too, and all leave.
-          if (tr < BW_N) ld_s[tb * BW_N + tr] = ld_next;
-          if (!bar_rows_and(ok)) {
-            ok = false;
-            break;
-          }
-          if (j + 1 < n) {
-            ld_next = fetch_ld(b, h, c0 + BW_N, tr);
-          } else {
-            const int k2 = bw_rank(blockIdx.x, rd + 1);
-            if (k2 < a.n_items) {
-              int t2, h2, b2, j02, n2;
-              bw_item<DKDV>(a, k2, t2, h2, b2, j02, n2);
-              ld_next = fetch_ld(b2, h2, j02 * BW_N, tr);
-            }
-          }
+        // DKDV: the step's (lse, Di) pairs, staged by the producer before the
+        // stage's full barrier (already complete: the step's scores used it;
+        // the slot is refilled only after this step's E has been consumed)
+        if (DKDV && !mbar_wait(y_full + 8 * (Gj % BW_STAGES), (Gj / BW_STAGES) & 1)) {
+          ok = false;
+          break;
         }
-        if (!ok) break;
         if (!mbar_wait(t_full + 8 * tb, (Gj >> 1) & 1)) {
           ok = false;
-          if (DKDV) continue;  // to the next barrier
           break;
         }
         tc_fence_after();
@@ -360,10 +360,9 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
           hi = min(hi, bw_vis(a, row) - c0);  // the keys this query sees
         if (!mbar_wait(e_free + 8 * tb, ((Gj >> 1) & 1) ^ 1)) {
           ok = false;
-          if (DKDV) continue;
           break;
         }
-        const float2* lds = ld_s + tb * BW_N;
+        const float2* lds = ld_ring + (Gj % BW_STAGES) * BW_N;
         uint32_t pk[16], dk[16];  // this thread's 32 columns of E1 and E2, bf16 pairs
         // P and dS of this thread's 32 columns; columns outside [lo, hi) are
         // masked (only the diagonal and tail steps have any)
@@ -415,13 +414,10 @@ __global__ void __launch_bounds__(BW_THREADS, 1)
         tc_fence_before();
         mbar_arrive_warp(e_full + 8 * tb);
       }
-      if (DKDV) ok = bar_rows_and(ok);
       if (!ok) break;
       G += n;
       // accumulators -> dK, dV (DKDV) or dQ (DQ) rows
-      bool acc_ok = mbar_wait(acc_full, it & 1);
-      if (DKDV) acc_ok = bar_rows_and(acc_ok);
-      if (!acc_ok) break;
+      if (!mbar_wait(acc_full, it & 1)) break;
       tc_fence_after();
       uint32_t u0[32], w0[32];  // this thread's 32 columns of dV / dQ and of dK
       tmem_ld32_async(tl + 256 + 32 * ch, u0);
