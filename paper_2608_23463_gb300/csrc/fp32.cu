@@ -144,13 +144,159 @@ __global__ void __launch_bounds__(FTHREADS) gemm_f32_kernel(const float* __restr
   }
 }
 
+// The same product with a CP_STAGES-deep ring of cp.async copies (16-byte,
+// zero-filled past M, N and the K range), for 16-byte aligned operands with
+// K, lda, ldb multiples of 4.  A and B tiles stay row-major in shared memory
+// (rows 36 floats apart), and each thread reads four K values of a row with
+// one 16-byte load, so a 4-deep K group costs eight shared loads for 64 FMAs.
+// A thread owns rows 4 ty .. 4 ty + 3 and columns tx + 16 j: the B rows that
+// eight consecutive lanes read are 36 floats apart, so their 16-byte loads
+// fall in distinct banks (contiguous column quartets, 144 floats apart, would
+// collide eight ways).
+constexpr int CP_STAGES = 4;
+constexpr int CP_LD = FK + 4;  // floats per row of a shared tile
+constexpr int CP_SMEM = CP_STAGES * 2 * FT * CP_LD * 4;
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src, bool valid) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
+               "r"(valid ? 16 : 0)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+__global__ void __launch_bounds__(FTHREADS, 2) gemm_f32_cp_kernel(
+    const float* __restrict__ A, long lda, const float* __restrict__ Bm, long ldb,
+    float* __restrict__ C, long ldc, int M, int N, int K, int Kc, const float* __restrict__ bias,
+    const float* __restrict__ addend, long ld_add, InjF32 inj) {
+  extern __shared__ __align__(16) float cps[];
+  float* As = cps;                              // [stage][FT][CP_LD]
+  float* Bs = cps + CP_STAGES * FT * CP_LD;     // [stage][FT][CP_LD]
+  const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
+  const int m0 = blockIdx.y * FT, n0 = blockIdx.x * FT;
+  const int kbeg = blockIdx.z * Kc, kend = min(K, kbeg + Kc);
+  const int nslab = kend > kbeg ? (kend - kbeg + FK - 1) / FK : 0;
+  C += (long)blockIdx.z * M * ldc;
+  // thread t copies rows t / 8 and t / 8 + 32, K offset (t % 8) * 4, of A and B
+  const int lr = threadIdx.x >> 3, lk = (threadIdx.x & 7) * 4;
+  const uint32_t as0 = static_cast<uint32_t>(__cvta_generic_to_shared(As));
+  const uint32_t bs0 = static_cast<uint32_t>(__cvta_generic_to_shared(Bs));
+  auto load = [&](int buf, int slab) {
+    const int gk = kbeg + slab * FK + lk;
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+      const int r = lr + 32 * i, gm = m0 + r, gn = n0 + r;
+      const bool ka = gk < kend;
+      const uint32_t off = (uint32_t)(((buf * FT + r) * CP_LD + lk) * 4);
+      cp_async16(as0 + off, A + (long)(gm < M ? gm : 0) * lda + (ka ? gk : 0), ka && gm < M);
+      cp_async16(bs0 + off, Bm + (long)(gn < N ? gn : 0) * ldb + (ka ? gk : 0), ka && gn < N);
+    }
+  };
+#pragma unroll
+  for (int st = 0; st < CP_STAGES - 1; ++st) {
+    if (st < nslab) load(st, st);
+    cp_async_commit();
+  }
+  float acc[4][4] = {};
+  for (int sl = 0; sl < nslab; ++sl) {
+    cp_async_wait<CP_STAGES - 2>();
+    __syncthreads();  // slab sl landed for all threads; buffer (sl - 1) % S is free
+    if (sl + CP_STAGES - 1 < nslab) load((sl + CP_STAGES - 1) % CP_STAGES, sl + CP_STAGES - 1);
+    cp_async_commit();
+    const float* a_t = As + (sl % CP_STAGES) * FT * CP_LD + (ty * 4) * CP_LD;
+    const float* b_t = Bs + (sl % CP_STAGES) * FT * CP_LD + tx * CP_LD;
+#pragma unroll
+    for (int kk = 0; kk < FK; kk += 4) {
+      float4 a4[4], b4[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        a4[i] = *reinterpret_cast<const float4*>(a_t + i * CP_LD + kk);
+        b4[i] = *reinterpret_cast<const float4*>(b_t + i * 16 * CP_LD + kk);
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          acc[i][j] = fmaf(a4[i].x, b4[j].x, acc[i][j]);
+          acc[i][j] = fmaf(a4[i].y, b4[j].y, acc[i][j]);
+          acc[i][j] = fmaf(a4[i].z, b4[j].z, acc[i][j]);
+          acc[i][j] = fmaf(a4[i].w, b4[j].w, acc[i][j]);
+        }
+    }
+  }
+  cp_async_wait<0>();
+  if (inj.Xo) {
+    // per-column parameters once, then all X loads before any X_out store (X
+    // and X_out are distinct tensors, but the compiler cannot know it)
+    float pb[4], pwx[4], pwd[4], pbg[4];
+    int chs[4], tko[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int gn = min(n0 + tx + 16 * j, N - 1);
+      chs[j] = gn % inj.d;
+      tko[j] = gn / inj.d;
+      pb[j] = bias ? bias[gn] : 0.f;
+      pwx[j] = inj.gated ? inj.w_x[chs[j]] : 0.f;
+      pwd[j] = inj.gated ? inj.w_dlt[chs[j]] : 0.f;
+      pbg[j] = inj.gated ? inj.b_g[chs[j]] : 0.f;
+    }
+    const float* __restrict__ Xr = inj.X;
+    float* __restrict__ Xw = inj.Xo;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {  // a row: its four X loads, then its stores
+      const int gm = m0 + ty * 4 + i;
+      if (gm >= M) continue;
+      // row gm = (b * m + iprox) * k2 + a: the target block and first token
+      const int a = gm % inj.k2, prox = gm / inj.k2;
+      const int b = prox / inj.m, ip = prox % inj.m + inj.shift;
+      if (ip >= inj.m) continue;
+      const long tok0 = (long)ip * inj.P + (long)a * inj.k1, seq0 = (long)b * inj.L;
+      float xv[4];
+      bool ok[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const long t = tok0 + tko[j];
+        ok[j] = n0 + tx + 16 * j < N && t < inj.L;
+        xv[j] = ok[j] ? Xr[(seq0 + t) * inj.d + chs[j]] : 0.f;
+      }
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        if (!ok[j]) continue;
+        const float v = acc[i][j] + pb[j], x = xv[j];
+        Xw[(seq0 + tok0 + tko[j]) * inj.d + chs[j]] =
+            inj.gated ? x + v / (1.f + expf(-(pwx[j] * x + pwd[j] * v + pbg[j]))) : x + v;
+      }
+    }
+    return;
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int gm = m0 + ty * 4 + i;
+    if (gm >= M) continue;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int gn = n0 + tx + 16 * j;
+      if (gn >= N) continue;
+      float v = acc[i][j];
+      if (bias) v += bias[gn];
+      if (addend) v += addend[(long)gm * ld_add + gn];
+      C[(long)gm * ldc + gn] = v;
+    }
+  }
+}
+
 // Eq. proxy-attn in fp32, head width 64.  CTA = (sequence, head, block of
 // ATT_Q queries), 8 warps of ATT_Q / 8 queries each.  Keys and values are
 // staged in shared memory 64 at a time (K transposed, so lane j reads key j's
 // dimensions without bank conflicts); each warp keeps an online softmax per
 // query: lane j scores keys j and j + 32 of the chunk and accumulates output
 // dimensions j and j + 32.
-constexpr int ATT_Q = 32;
+constexpr int ATT_Q = 8;  // one query per warp: 4x the CTAs of 32, a quarter of the serial chains
 __global__ void __launch_bounds__(256) attn_f32_kernel(const float* __restrict__ qkv,
                                                        float* __restrict__ out, int m, int d,
                                                        int causal, float scale) {
@@ -291,27 +437,67 @@ __global__ void pad_f32_kernel(const float* __restrict__ src, float* __restrict_
 }
 
 
-__global__ void splitk_f32_reduce(const float* __restrict__ part, int S, int M, int N,
-                                  float* __restrict__ C, long ldc, const float* __restrict__ bias,
-                                  const float* __restrict__ addend, long ld_add) {
-  const long i = (long)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= (long)M * N) return;
-  const long r = i / N;
-  const int c = (int)(i % N);
-  float v = 0.f;
-  for (int s = 0; s < S; ++s) v += part[((long)s * M + r) * N + c];
-  if (bias) v += bias[c];
-  if (addend) v += addend[r * ld_add + c];
-  C[r * ldc + c] = v;
+// Deterministic split-K reduction: C = sum_s part[s] (+ bias) (+ addend).  A
+// CTA takes 32 four-column groups of one row segment and 8 split groups; split
+// group g sums splits g, g + 8, ... in that order, and the 8 group sums are
+// added in order 0..7, so the result does not depend on scheduling.
+constexpr int RED_G = 8;
+__global__ void __launch_bounds__(256) splitk_f32_reduce(const float* __restrict__ part, int S, int M,
+                                                         int N, float* __restrict__ C, long ldc,
+                                                         const float* __restrict__ bias,
+                                                         const float* __restrict__ addend,
+                                                         long ld_add) {
+  __shared__ float4 sums[RED_G][32];
+  const int g = threadIdx.x >> 5, l = threadIdx.x & 31;
+  const long n4 = (long)(N + 3) / 4;
+  const long q = (long)blockIdx.x * 32 + l;  // four-column group over [M, N / 4]
+  const bool in = q < (long)M * n4;
+  const long r = in ? q / n4 : 0;
+  const int c = in ? (int)(q % n4) * 4 : 0;
+  const bool vec4 = (N % 4) == 0;
+  float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (in) {
+    for (int s = g; s < S; s += RED_G) {
+      const float* p = part + ((long)s * M + r) * N + c;
+      if (vec4) {
+        const float4 x = *reinterpret_cast<const float4*>(p);
+        v.x += x.x; v.y += x.y; v.z += x.z; v.w += x.w;
+      } else {
+        v.x += p[0];
+        if (c + 1 < N) v.y += p[1];
+        if (c + 2 < N) v.z += p[2];
+        if (c + 3 < N) v.w += p[3];
+      }
+    }
+  }
+  sums[g][l] = v;
+  __syncthreads();
+  if (g != 0 || !in) return;
+  float4 t = sums[0][l];
+#pragma unroll
+  for (int k = 1; k < RED_G; ++k) {
+    const float4 u = sums[k][l];
+    t.x += u.x; t.y += u.y; t.z += u.z; t.w += u.w;
+  }
+  const float tv[4] = {t.x, t.y, t.z, t.w};
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    if (c + j >= N) break;
+    float o = tv[j];
+    if (bias) o += bias[c + j];
+    if (addend) o += addend[r * ld_add + c + j];
+    C[r * ldc + c + j] = o;
+  }
 }
 
 }  // namespace
 
 int splitk_f32_factor(int M, int N, int K) {
+  // about one wave of a 152-SM part; slices of at least two 32-wide K slabs
   const long tiles = (long)((M + FT - 1) / FT) * ((N + FT - 1) / FT);
-  if (tiles >= 304) return 1;
-  int S = (int)((304 + tiles - 1) / tiles);  // about two CTAs per SM of a 152-SM part
-  S = std::min(S, std::max(1, K / 64));       // at least two 32-wide K slabs per slice
+  if (tiles >= 152) return 1;
+  int S = (int)((152 + tiles - 1) / tiles);
+  S = std::min(S, std::max(1, K / 64));
   return std::min(S, 64);
 }
 
@@ -319,6 +505,25 @@ namespace {
 int vec_ok(const float* A, long lda, const float* B, long ldb, int K) {
   return ((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(B)) & 15) == 0 &&
          lda % 4 == 0 && ldb % 4 == 0 && K % 4 == 0;
+}
+}  // namespace
+
+namespace {
+// launch the product (cp.async ring when the operands allow it)
+cudaError_t launch_f32(dim3 grid, int vec, const float* A, long lda, const float* B, long ldb,
+                       float* C, long ldc, int M, int N, int K, int Kc, const float* bias,
+                       const float* addend, long ld_add, const InjF32& inj, cudaStream_t st) {
+  if (vec) {
+    static const cudaError_t attr = cudaFuncSetAttribute(
+        gemm_f32_cp_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, CP_SMEM);
+    if (attr != cudaSuccess) return attr;
+    gemm_f32_cp_kernel<<<grid, FTHREADS, CP_SMEM, st>>>(A, lda, B, ldb, C, ldc, M, N, K, Kc, bias,
+                                                        addend, ld_add, inj);
+  } else {
+    gemm_f32_kernel<<<grid, FTHREADS, 0, st>>>(A, lda, B, ldb, C, ldc, M, N, K, Kc, bias, addend,
+                                               ld_add, 0, inj);
+  }
+  return cudaGetLastError();
 }
 }  // namespace
 
@@ -331,17 +536,17 @@ cudaError_t gemm_f32(int M, int N, int K, const float* A, long lda, const float*
   if (S > 1 && scratch && (size_t)S * M * N * sizeof(float) <= scratch_bytes) {
     const int Kc = ((K + S - 1) / S + FK - 1) / FK * FK;
     dim3 grid((N + FT - 1) / FT, (M + FT - 1) / FT, S);
-    gemm_f32_kernel<<<grid, FTHREADS, 0, st>>>(A, lda, B, ldb, scratch, N, M, N, K, Kc, nullptr,
-                                               nullptr, 0, vec, InjF32{});
-    const long total = (long)M * N;
-    splitk_f32_reduce<<<(unsigned)((total + 255) / 256), 256, 0, st>>>(scratch, S, M, N, C, ldc, bias,
-                                                                      addend, ld_add);
+    cudaError_t e = launch_f32(grid, vec, A, lda, B, ldb, scratch, N, M, N, K, Kc, nullptr, nullptr,
+                               0, InjF32{}, st);
+    if (e != cudaSuccess) return e;
+    const long groups = (long)M * ((N + 3) / 4);
+    splitk_f32_reduce<<<(unsigned)((groups + 31) / 32), 256, 0, st>>>(scratch, S, M, N, C, ldc, bias,
+                                                                     addend, ld_add);
     return cudaGetLastError();
   }
   dim3 grid((N + FT - 1) / FT, (M + FT - 1) / FT, 1);
-  gemm_f32_kernel<<<grid, FTHREADS, 0, st>>>(A, lda, B, ldb, C, ldc, M, N, K, K, bias, addend,
-                                             ld_add, vec, InjF32{});
-  return cudaGetLastError();
+  return launch_f32(grid, vec, A, lda, B, ldb, C, ldc, M, N, K, K, bias, addend, ld_add, InjF32{},
+                    st);
 }
 
 cudaError_t gemm_f32_inject(int M, int N, int K, const float* A, long lda, const float* B, long ldb,
@@ -353,9 +558,11 @@ cudaError_t gemm_f32_inject(int M, int N, int K, const float* A, long lda, const
     LaunchTimer lt("decompress_d1_inject", st, 2.0 * M * N * (double)K,
                    4.0 * ((double)M * K + (double)N * K) + 12.0 * Bsz * L * (double)d);
     dim3 grid((N + FT - 1) / FT, (M + FT - 1) / FT, 1);
-    gemm_f32_kernel<<<grid, FTHREADS, 0, st>>>(
-        A, lda, B, ldb, nullptr, 0, M, N, K, K, bias, nullptr, 0, vec,
-        InjF32{X, Xo, w_x, w_dlt, b_g, L, d, P, k1, k2, m, shift, gated});
+    const cudaError_t e = launch_f32(grid, vec, A, lda, B, ldb, nullptr, 0, M, N, K, K, bias,
+                                     nullptr, 0, InjF32{X, Xo, w_x, w_dlt, b_g, L, d, P, k1, k2, m,
+                                                        shift, gated},
+                                     st);
+    if (e != cudaSuccess) return e;
   }
   if (shift > 0) {  // the first block of every sequence receives nothing: X_out = X
     const long rows = std::min<long>((long)shift * P, L);
