@@ -307,7 +307,7 @@ cudaError_t gemm_affine2d(int M, int N, int K, Operand A, Operand B, const EpiAf
 cudaError_t gemm_dx2d(int M, int N, int K, Operand A, Operand B, const EpiDX2DArgs& e,
                       cudaStream_t st) {
   EpiDX2D epi{{}, M, N, e.dX, e.d, e.patch, e.gh, e.gw, e.m};
-  if (A.mn || !B.mn) return cudaErrorInvalidValue;
+  if (A.mn || !B.mn || e.d % 32 != 0) return cudaErrorInvalidValue;
   return gemm_dispatch(M, N, K, A, B, epi, e.dXd, M, st);
 }
 

@@ -1058,31 +1058,43 @@ struct EpiDX2D : EpiBase {
   struct Row {
     bool ok;
     long base;  // offset of the patch's top-left token in dX
+    SegRows seg;
   };
   int M, N;
   bf16* dX;
   int d, patch, gh, gw, m;
   __device__ __forceinline__ Row row_info(int row, int) const {
     Row r{row < M, 0};
-    if (!r.ok) return r;
-    const int npw = gw / patch;
-    const int b = row / m, pr = row % m, by = pr / npw, bx = pr % npw;
-    r.base = ((long)b * gh * gw + (long)by * patch * gw + bx * patch) * d;
+    if (r.ok) {
+      const int npw = gw / patch;
+      const int b = row / m, pr = row % m, by = pr / npw, bx = pr % npw;
+      r.base = ((long)b * gh * gw + (long)by * patch * gw + bx * patch) * d;
+    }
+    r.seg.gather(r.base, r.ok ? N : 0);
     return r;
   }
-  __device__ __forceinline__ void apply(const Row& ri, int, int col, float* v, const uint8_t* xt,
+  // staged in the tile cells just read, stored with whole-row segments: a
+  // 32-column chunk is 32 channels of one token of the patch (d is a multiple
+  // of 32), 64 contiguous bytes of dX per row
+  __device__ __forceinline__ void apply(const Row& ri, int, int col, float* v, uint8_t* xt,
                                         int rl, int cl, const float4*) const {
-    if (!ri.ok || col >= N) return;
-    const int p = col / d, ch = col - p * d, py = p / patch, px = p - py * patch;
-    bf16* o = dX + ri.base + ((long)py * gw + px) * d + ch;
+    if (col >= N) return;  // uniform across the warp
 #pragma unroll
     for (int i8 = 0; i8 < 32; i8 += 8) {
       float x[8];
       xtile_load8(xt, rl, cl + i8, x);
 #pragma unroll
       for (int j = 0; j < 8; ++j) x[j] += v[i8 + j];
-      store8_bf16(o + i8, x);
+      xtile_put8(xt, rl, cl + i8, x);
     }
+    __syncwarp();
+    const int p = col / d, ch = col - p * d, py = p / patch, px = p - py * patch;
+    const long colofs = ((long)py * gw + px) * d + ch;
+    warp_store_rows(xt, rl >> 5, cl, [&](int rr, int q) -> bf16* {
+      const int it = rr >> 3;
+      return col + q * 8 < ri.seg.lim[it] ? dX + ri.seg.off[it] + colofs + q * 8 : nullptr;
+    });
+    __syncwarp();
   }
 };
 
