@@ -967,6 +967,7 @@ struct EpiAffine2D : EpiBase {
     bool ok;
     long xoff;  // element offset of (token, channel cb) in X_out
     float mu, rs;
+    SegRows seg;  // X_out offsets of the rows this lane stores (lim 1: row exists)
   };
   int M;
   const float* bias;
@@ -984,14 +985,16 @@ struct EpiAffine2D : EpiBase {
   }
   __device__ __forceinline__ Row row_info(int row, int n0) const {
     Row r{row < M, 0, 0.f, 0.f};
-    if (!r.ok) return r;
-    const int npw = gw / patch;
-    const int b = row / m, pr = row % m, by = pr / npw, bx = pr % npw;
-    const int p = ptok(n0), py = p / patch, px = p % patch;
-    const long tok = (long)b * gh * gw + (long)(by * patch + py) * gw + bx * patch + px;
-    r.xoff = tok * d + cbase(n0);
-    r.mu = stats[2 * tok];
-    r.rs = stats[2 * tok + 1];
+    if (r.ok) {
+      const int npw = gw / patch;
+      const int b = row / m, pr = row % m, by = pr / npw, bx = pr % npw;
+      const int p = ptok(n0), py = p / patch, px = p % patch;
+      const long tok = (long)b * gh * gw + (long)(by * patch + py) * gw + bx * patch + px;
+      r.xoff = tok * d + cbase(n0);
+      r.mu = stats[2 * tok];
+      r.rs = stats[2 * tok + 1];
+    }
+    r.seg.gather(r.xoff, r.ok ? 1 : 0);
     return r;
   }
   // staged per column c of the s half: (bias of s, bias of t)
@@ -1028,12 +1031,9 @@ struct EpiAffine2D : EpiBase {
       xtile_put8(xt, rl, c + i8, o);
     }
     __syncwarp();
-    const long long off = ri.xoff;
-    const int okr = ri.ok ? 1 : 0;
     warp_store_rows(xt, q, c, [&](int rr, int pc) -> bf16* {
-      const long long o2 = __shfl_sync(0xffffffffu, off, rr);
-      const int k2 = __shfl_sync(0xffffffffu, okr, rr);
-      return k2 ? X_out + o2 + c + pc * 8 : nullptr;
+      const int it = rr >> 3;
+      return ri.seg.lim[it] ? X_out + ri.seg.off[it] + c + pc * 8 : nullptr;
     });
     __syncwarp();
 #pragma unroll
