@@ -34,29 +34,45 @@ __global__ void attn_bwd_dot_kernel(const bf16* __restrict__ dO, const bf16* __r
   }
 }
 
-// Gate of the cross injection, backward: one warp per (token row, head),
-// each lane two of the head's 64 columns.
+// Gate of the cross injection, backward: eight lanes per (token row, head),
+// each lane eight of the head's 64 columns with 16-byte loads and stores, so
+// a warp covers four items per instruction (one item per warp, with 4-byte
+// loads, left too few bytes in flight to stream at HBM speed).
 __global__ void cross_gate_bwd_kernel(const bf16* __restrict__ dAg, const bf16* __restrict__ A,
                                       const bf16* __restrict__ qa, long ldq,
                                       const float* __restrict__ b_a, bf16* __restrict__ dO,
                                       float* __restrict__ Di, bf16* __restrict__ dqa,
                                       float* __restrict__ ga, int ldga, long rows, int L, int d,
                                       int nh) {
-  const long wid = ((long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  if (wid >= rows * nh) return;
+  const long gid = ((long)blockIdx.x * blockDim.x + threadIdx.x) >> 3;  // item
+  const int sub = threadIdx.x & 7;                                      // lane in the item
+  const long items = rows * nh;
+  const bool live = gid < items;
+  const long wid = live ? gid : items - 1;
   const long row = wid / nh;
   const int h = (int)(wid % nh);
-  const long off = row * d + h * AT + lane * 2;
-  const float2 g = unpack_bf16(*reinterpret_cast<const uint32_t*>(dAg + off));
-  const float2 a = unpack_bf16(*reinterpret_cast<const uint32_t*>(A + off));
-  float sum = g.x * a.x + g.y * a.y;
-#pragma unroll
-  for (int s = 16; s > 0; s >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, s);
+  const long off = row * d + h * AT + sub * 8;
+  const uint4 gu = *reinterpret_cast<const uint4*>(dAg + off);
+  const uint4 au = *reinterpret_cast<const uint4*>(A + off);
   const float x = __bfloat162float(qa[row * ldq + d + h]) + b_a[h];
+  const uint32_t gw[4] = {gu.x, gu.y, gu.z, gu.w}, aw[4] = {au.x, au.y, au.z, au.w};
+  float sum = 0.f;
+  float2 g2[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    g2[k] = unpack_bf16(gw[k]);
+    const float2 a2 = unpack_bf16(aw[k]);
+    sum = fmaf(g2[k].x, a2.x, sum);
+    sum = fmaf(g2[k].y, a2.y, sum);
+  }
+#pragma unroll
+  for (int s = 4; s > 0; s >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, s);
+  if (!live) return;
   const float al = 1.f / (1.f + __expf(-x));
-  *reinterpret_cast<uint32_t*>(dO + off) = pack_bf16(al * g.x, al * g.y);
-  if (lane == 0) {
+  *reinterpret_cast<uint4*>(dO + off) =
+      make_uint4(pack_bf16(al * g2[0].x, al * g2[0].y), pack_bf16(al * g2[1].x, al * g2[1].y),
+                 pack_bf16(al * g2[2].x, al * g2[2].y), pack_bf16(al * g2[3].x, al * g2[3].y));
+  if (sub == 0) {
     const long b = row / L, t = row % L;
     Di[(b * nh + h) * L + t] = al * sum;
     const float gp = sum * al * (1.f - al);
@@ -64,8 +80,8 @@ __global__ void cross_gate_bwd_kernel(const bf16* __restrict__ dAg, const bf16* 
     ga[row * ldga + h] = gp;
   }
   if (h == 0) {  // the padding columns past the gate rows stay zero
-    for (long c = d + nh + lane; c < ldq; c += 32) dqa[row * ldq + c] = __float2bfloat16(0.f);
-    for (int c = nh + lane; c < ldga; c += 32) ga[row * ldga + c] = 0.f;
+    for (long c = d + nh + sub; c < ldq; c += 8) dqa[row * ldq + c] = __float2bfloat16(0.f);
+    for (int c = nh + sub; c < ldga; c += 8) ga[row * ldga + c] = 0.f;
   }
 }
 
@@ -78,7 +94,8 @@ cudaError_t cross_gate_bwd(const bf16* dAg, const bf16* A, const bf16* qa, long 
   const long rows = (long)B * L, warps = rows * nh;
   LaunchTimer lt("cross_gate_bwd", st, 4.0 * rows * d,
                  6.0 * rows * d + 2.0 * rows * ldq / 8.0 + 8.0 * rows * nh);
-  cross_gate_bwd_kernel<<<(unsigned)((warps * 32 + 255) / 256), 256, 0, st>>>(
+  if (((uintptr_t)dAg | (uintptr_t)A | (uintptr_t)dO) & 15) return cudaErrorInvalidValue;
+  cross_gate_bwd_kernel<<<(unsigned)((warps * 8 + 255) / 256), 256, 0, st>>>(
       dAg, A, qa, ldq, b_a, dO, Di, dqa, ga, ldga, rows, L, d, nh);
   return cudaGetLastError();
 }
