@@ -14,21 +14,31 @@ namespace {
 
 constexpr int AT = 64;  // head width
 
-// Di = rowsum(dO * O) per (b, h, query): one warp per (row, head).
+// Di = rowsum(dO * O) per (b, h, query): eight lanes per (row, head), each
+// eight of the head's 64 columns with 16-byte loads.
 __global__ void attn_bwd_dot_kernel(const bf16* __restrict__ dO, const bf16* __restrict__ O,
                                     float* __restrict__ Dout, int rows, int m, int d, int nh) {
-  const long wid = ((long)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  if (wid >= (long)rows * nh) return;
+  const long gid = ((long)blockIdx.x * blockDim.x + threadIdx.x) >> 3;
+  const int sub = threadIdx.x & 7;
+  const long items = (long)rows * nh;
+  const bool live = gid < items;
+  const long wid = live ? gid : items - 1;
   const long row = wid / nh;
   const int h = (int)(wid % nh);
-  const long off = row * d + h * AT + lane * 2;
-  const float2 a = unpack_bf16(*reinterpret_cast<const uint32_t*>(dO + off));
-  const float2 c = unpack_bf16(*reinterpret_cast<const uint32_t*>(O + off));
-  float v = a.x * c.x + a.y * c.y;
+  const long off = row * d + h * AT + sub * 8;
+  const uint4 gu = *reinterpret_cast<const uint4*>(dO + off);
+  const uint4 ou = *reinterpret_cast<const uint4*>(O + off);
+  const uint32_t gw[4] = {gu.x, gu.y, gu.z, gu.w}, ow[4] = {ou.x, ou.y, ou.z, ou.w};
+  float v = 0.f;
 #pragma unroll
-  for (int s = 16; s > 0; s >>= 1) v += __shfl_xor_sync(0xffffffffu, v, s);
-  if (lane == 0) {
+  for (int k = 0; k < 4; ++k) {
+    const float2 a = unpack_bf16(gw[k]), c = unpack_bf16(ow[k]);
+    v = fmaf(a.x, c.x, v);
+    v = fmaf(a.y, c.y, v);
+  }
+#pragma unroll
+  for (int s = 4; s > 0; s >>= 1) v += __shfl_xor_sync(0xffffffffu, v, s);
+  if (live && sub == 0) {
     const long b = row / m, i = row % m;
     Dout[(b * nh + h) * m + i] = v;
   }
@@ -108,8 +118,9 @@ cudaError_t attn_bwd(const bf16* qkv, const bf16* O, const bf16* dO, const float
   const long warps = (long)B * m * nh;
   {
     LaunchTimer lt("attn_bwd_dot", st, 2.0 * B * m * d, 4.0 * B * m * d + 4.0 * B * nh * m);
-    attn_bwd_dot_kernel<<<(unsigned)((warps * 32 + 255) / 256), 256, 0, st>>>(dO, O, Di, B * m, m,
-                                                                              d, nh);
+    if (((uintptr_t)dO | (uintptr_t)O) & 15) return cudaErrorInvalidValue;
+    attn_bwd_dot_kernel<<<(unsigned)((warps * 8 + 255) / 256), 256, 0, st>>>(dO, O, Di, B * m, m,
+                                                                             d, nh);
     const cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
