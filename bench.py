@@ -759,7 +759,7 @@ def run_case(args):
     t = pf.pf_timing_collect()
     pf.pf_timing_enable(False)
     pf.pf_sync_check(stream.cuda_stream)
-    top = sorted(t.items(), key=lambda kv: -kv[1]["ms"])[:10]
+    top = sorted(t.items(), key=lambda kv: -kv[1]["ms"])[:24]
     print(json.dumps({"case": args.case, "batch": spec.batch, "L": spec.L, "ms_per_step": ms,
                       "kernels_ms": {k: round(v["ms"], 4) for k, v in top}}), flush=True)
 
