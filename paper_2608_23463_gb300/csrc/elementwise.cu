@@ -402,35 +402,73 @@ __device__ __forceinline__ void load8<float>(const float* p, float* v) {
   v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
 }
 
+// Column sums of an [R, C] matrix (C a multiple of 8), pass 1: CTA (x, y)
+// adds rows chunk y of the CG * 8 columns from x * CG * 8 on.  Thread t reads
+// 8 columns (16 or 32 bytes) of every 256 / CG-th row from row (t / CG), so
+// a warp reads whole row segments; the 256 / CG row lanes are then added in
+// lane order through shared memory.  CG: the smallest power of two of
+// 8-column groups covering C, at most 32.
 template <typename T>
 __global__ void __launch_bounds__(EW_THREADS) colsum_part_kernel(const T* __restrict__ X, long R,
-                                                                 int C, long rows_per_chunk,
+                                                                 int C, int CG, long rows_per_chunk,
                                                                  float* __restrict__ part) {
-  const int col = (blockIdx.x * EW_THREADS + threadIdx.x) * 8;
-  if (col >= C) return;
+  __shared__ float s_acc[EW_THREADS * 8];
+  const int RL = EW_THREADS / CG, cg = threadIdx.x % CG, rl = threadIdx.x / CG;
+  const int col = (blockIdx.x * CG + cg) * 8;
   const long r0 = (long)blockIdx.y * rows_per_chunk, r1 = min(R, r0 + rows_per_chunk);
   float acc[8] = {};
-  for (long r = r0; r < r1; ++r) {
-    float v[8];
-    load8<T>(X + r * C + col, v);
+  if (col < C) {
+    long r = r0 + rl;
+#pragma unroll 1
+    for (; r + 3 * RL < r1; r += 4 * RL) {  // four rows' loads in flight
+      float v[4][8];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) acc[j] += v[j];
+      for (int u = 0; u < 4; ++u) load8<T>(X + (r + u * RL) * C + col, v[u]);
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[j] += v[u][j];
+    }
+    for (; r < r1; r += RL) {
+      float v[8];
+      load8<T>(X + r * C + col, v);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) acc[j] += v[j];
+    }
   }
-  float* p = part + (long)blockIdx.y * C + col;
-  *reinterpret_cast<float4*>(p) = make_float4(acc[0], acc[1], acc[2], acc[3]);
-  *reinterpret_cast<float4*>(p + 4) = make_float4(acc[4], acc[5], acc[6], acc[7]);
+#pragma unroll
+  for (int j = 0; j < 8; ++j) s_acc[rl * CG * 8 + cg * 8 + j] = acc[j];
+  __syncthreads();
+  const int c = threadIdx.x;  // one column of the CTA's CG * 8 per thread
+  const int gcol = blockIdx.x * CG * 8 + c;
+  if (c < CG * 8 && gcol < C) {
+    float t = 0.f;
+    for (int l = 0; l < RL; ++l) t += s_acc[l * CG * 8 + c];
+    part[(long)blockIdx.y * C + gcol] = t;
+  }
 }
 
-// One warp per column (deterministic order, see warp_sum).
-__global__ void colsum_final_kernel(const float* __restrict__ part, int n_chunks, int C,
-                                    float* __restrict__ out) {
-  const int i = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  if (i >= C) return;
-  float s = 0.f;
-  for (int c = lane; c < n_chunks; c += 32) s += part[(long)c * C + i];
-  s = warp_sum(s);
-  if (lane == 0) out[i] = s;
+// Pass 2: block = 32 consecutive columns x CS_WARPS warps; warp w adds chunks
+// w, w + CS_WARPS, ... of its lane's column (a chunk row is one 128-byte
+// segment per warp), then the warp totals are added in warp order.
+constexpr int CS_WARPS = 16;
+__global__ void __launch_bounds__(32 * CS_WARPS)
+    colsum_final_kernel(const float* __restrict__ part, int n_chunks, int C,
+                        float* __restrict__ out) {
+  __shared__ float s_w[CS_WARPS][32];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int col = blockIdx.x * 32 + lane;
+  float a = 0.f;
+  if (col < C)
+    for (int c = w; c < n_chunks; c += CS_WARPS) a += part[(long)c * C + col];
+  s_w[w][lane] = a;
+  __syncthreads();
+  if (w == 0 && col < C) {
+    float t = 0.f;
+#pragma unroll
+    for (int k = 0; k < CS_WARPS; ++k) t += s_w[k][lane];
+    out[col] = t;
+  }
 }
 
 // Row chunks of a column reduction: about 1024 CTAs in total, independent of
@@ -443,18 +481,36 @@ int chunks_for(long R, int C) {
   return (int)want;
 }
 
+// 8-column groups per column-sum CTA (a power of two, at most 32).
+int colsum_groups(int C) {
+  int cg = 1;
+  while (cg < 32 && cg * 8 < C) cg *= 2;
+  return cg;
+}
+
+// Row chunks of a column sum: about 1216 CTAs in all (eight per SM of a
+// 152-SM part) with at least 64 rows each, independent of the device so that
+// the summation order and the workspace size are fixed.
+int colsum_chunks(long R, int C) {
+  const int gx = (C + colsum_groups(C) * 8 - 1) / (colsum_groups(C) * 8);
+  long want = (1216 + gx - 1) / gx;
+  want = std::min(want, (R + 63) / 64);
+  return (int)std::max(want, 1L);
+}
+
 template <typename T>
 cudaError_t colsum_impl(const T* X, long R, int C, float* out, float* part, cudaStream_t st) {
-  const int nc = chunks_for(R, C);
+  if (C % 8 != 0 || R < 1) return cudaErrorInvalidValue;
+  const int cg = colsum_groups(C), nc = colsum_chunks(R, C);
   const long rpc = (R + nc - 1) / nc;
-  dim3 grid((C / 8 + EW_THREADS - 1) / EW_THREADS, nc);
+  dim3 grid((C + cg * 8 - 1) / (cg * 8), nc);
   {
     LaunchTimer lt("colsum", st, (double)R * C, (double)R * C * sizeof(T));
-    colsum_part_kernel<T><<<grid, EW_THREADS, 0, st>>>(X, R, C, rpc, part);
+    colsum_part_kernel<T><<<grid, EW_THREADS, 0, st>>>(X, R, C, cg, rpc, part);
   }
   {
     LaunchTimer lt("colsum_final", st, (double)nc * C, 4.0 * nc * C);
-    colsum_final_kernel<<<(C + 7) / 8, 256, 0, st>>>(part, nc, C, out);
+    colsum_final_kernel<<<(C + 31) / 32, 32 * CS_WARPS, 0, st>>>(part, nc, C, out);
   }
   return cudaGetLastError();
 }
@@ -595,7 +651,7 @@ cudaError_t add_f32_bf16(const bf16* a, const float* b, float* out_f, bf16* out_
   return cudaGetLastError();
 }
 
-long colsum_part_elems(long R, int C) { return (long)chunks_for(R, C) * C; }
+long colsum_part_elems(long R, int C) { return (long)colsum_chunks(R, C) * C; }
 
 cudaError_t colsum_bf16(const bf16* X, long R, int C, float* out, float* part, cudaStream_t st) {
   return colsum_impl<bf16>(X, R, C, out, part, st);
