@@ -30,7 +30,7 @@ METRIC = "ProxyFormer layer fwd+bwd tokens/s at L=256K, P=64; % of GB300 rooflin
 UNIT = "tokens/s"
 WORKLOAD = "proxyformer_layer_causal1d_L262144_d1024_h16x64_P64_8x8_gated_bf16_fwd_bwd"
 SAMPLE_L = 2048       # tokens of one reference-arm step (32 proxies)
-BASELINE_L = 65536   # tokens of the cpu_baseline slice (1024 proxies)
+CPU_SLICE_L = 65536   # tokens of the cpu_baseline slice (1024 proxies)
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
@@ -105,16 +105,16 @@ def cpu_baseline_subprocess():
     cores = os.cpu_count() or 1
     env = dict(os.environ, OPENBLAS_NUM_THREADS=str(cores), OMP_NUM_THREADS=str(cores))
     code = ("import json, bench; t = bench.oracle_sample_seconds(%d, 1); print(json.dumps(t))"
-            % BASELINE_L)
+            % CPU_SLICE_L)
     r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, env=env, capture_output=True,
                        text=True, timeout=900)
     if r.returncode != 0:
         return {"value": None, "unit": UNIT, "cores": cores, "kind": "oracle",
                 "sample": "failed: " + r.stderr.strip().splitlines()[-1][:200]}
     t = json.loads(r.stdout.strip().splitlines()[-1])
-    return {"value": BASELINE_L / min(t), "unit": UNIT, "cores": cores, "kind": "oracle",
-            "sample": f"one fwd+bwd of the float64 oracle over a {BASELINE_L}-token slice "
-                      f"({BASELINE_L // 64} proxies) of the same layer shape, {min(t):.1f} s"}
+    return {"value": CPU_SLICE_L / min(t), "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"one fwd+bwd of the float64 oracle over a {CPU_SLICE_L}-token slice "
+                      f"({CPU_SLICE_L // 64} proxies) of the same layer shape, {min(t):.1f} s"}
 
 
 # ------------------------------------------------------------ ranks (N > 1)
