@@ -500,7 +500,8 @@ int colsum_chunks(long R, int C) {
 
 template <typename T>
 cudaError_t colsum_impl(const T* X, long R, int C, float* out, float* part, cudaStream_t st) {
-  if (C % 8 != 0 || R < 1) return cudaErrorInvalidValue;
+  if (C % 8 != 0) return cudaErrorInvalidValue;
+  if (R < 1) return cudaMemsetAsync(out, 0, (size_t)C * sizeof(float), st);  // an empty sum
   const int cg = colsum_groups(C), nc = colsum_chunks(R, C);
   const long rpc = (R + nc - 1) / nc;
   dim3 grid((C + cg * 8 - 1) / (cg * 8), nc);
