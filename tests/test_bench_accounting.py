@@ -1,0 +1,122 @@
+"""bench.py's accounting on the CPU: the algorithmic work that the roofline
+fractions divide by, the compute peak at the sampled clock, and the DRAM
+traffic lookup with its staleness rule.
+
+The layer's FLOPs are re-derived here from the contractions of Alg. 1 one by
+one (compression, the proxy interaction, decompression; every forward GEMM
+has an input-gradient and a weight-gradient GEMM of its own size in the
+backward; the attention backward re-forms S and dP and adds three more
+products), not from the closed form bench.layer_work uses (Eq. complexity),
+so a dropped or double-counted term in either shows up."""
+import os
+
+import pytest
+
+import bench
+import pf_synth as S
+
+
+def _gemm_flops(shapes):
+    return sum(2.0 * M * N * K for M, N, K in shapes)
+
+
+def _layer_gemms(spec):
+    """(M, N, K) of every forward contraction of one sequence (Alg. 1)."""
+    L, d, P = spec.L, spec.d, spec.P
+    m = -(-L // P)
+    if spec.levels == 2:
+        k1, k2 = spec.k1, spec.k2
+        g = [(m * k2, d, k1 * d),          # level-1 compression: groups of k1 tokens
+             (m, d, k2 * d)]               # level-2 compression: groups of k2 level-1 outputs
+        g += [(m, 3 * d, d), (m, d, d)]    # Q, K, V and the output projection
+        g += [(m, k2 * d, d),              # level-2 decompression
+              (m * k2, k1 * d, d)]         # level-1 decompression, one row per k1 tokens
+    else:
+        g = [(m, d, P * d), (m, 3 * d, d), (m, d, d), (m, P * d, d)]
+    return g
+
+
+def _attention_pairs(m, causal):
+    return sum(i + 1 for i in range(m)) if causal else m * m
+
+
+@pytest.mark.parametrize("levels", [1, 2])
+@pytest.mark.parametrize("mode", [0, 1])
+def test_layer_flops_match_the_contractions(levels, mode):
+    kw = dict(k1=8, k2=8) if levels == 2 else {}
+    spec = S.LayerSpec(batch=2, L=262144 if levels == 2 else 65536, d=1024, n_heads=16, P=64,
+                       levels=levels, mode=mode, **kw)
+    m = -(-spec.L // spec.P)
+    lin = _gemm_flops(_layer_gemms(spec))
+    pairs = _attention_pairs(m, causal=(mode == 0))
+    dh, nh = spec.d // spec.n_heads, spec.n_heads
+    att_fwd = nh * pairs * (2 * dh + 2 * dh)                 # S = Q K^T, O = P V
+    att_bwd = nh * pairs * (2 * dh * 5)                      # S again, dP, dV, dQ, dK
+    fwd = spec.batch * (lin + att_fwd)
+    bwd = spec.batch * (2 * lin + att_bwd)                   # dX and dW of every GEMM
+    f_inf, _ = bench.layer_work(spec, train=False)
+    f_train, _ = bench.layer_work(spec, train=True)
+    assert f_inf == pytest.approx(fwd, rel=1e-12)
+    assert f_train == pytest.approx(fwd + bwd, rel=1e-12)
+
+
+def test_headline_work_and_roofline_time():
+    """The benchmark layer (L = 262144, d = 1024, P = 64 as 8 x 8): 3.934
+    TFLOP and 3.52 GB per fwd+bwd step; X, dX_out read and X_out, dX written
+    once, X read once more by the injection and once by the backward, the
+    weights read once per pass and their fp32 gradients written once."""
+    spec = S.spec_c3_layer(64)
+    flops, nbytes = bench.layer_work(spec)
+    assert flops == pytest.approx(3.934e12, rel=1e-3)
+    act = spec.batch * spec.L * spec.d * 2
+    d, k1, k2 = spec.d, spec.k1, spec.k2
+    weights = k1 * d * d + k2 * d * d + 4 * d * d + k2 * d * d + k1 * d * d
+    assert nbytes == pytest.approx(6 * act + 2 * 2 * weights + 4 * weights, rel=1e-12)
+    assert nbytes == pytest.approx(3.52e9, rel=2e-3)
+    # at the measured burst peak the step cannot take less than ~2.04 ms
+    assert flops / 1926.3e12 * 1e3 == pytest.approx(2.042, abs=2e-3)
+
+
+def test_compute_peak_follows_the_sampled_clock():
+    peaks = {"bf16_tflops": 1926.3}
+    assert bench.compute_peak(peaks, None)[0] == 1926.3
+    assert bench.compute_peak(peaks, {"sm_mhz": 2070, "sm_max_mhz": 2070})[0] == 1926.3
+    p, src = bench.compute_peak(peaks, {"sm_mhz": 1035, "sm_max_mhz": 2070})
+    assert p == pytest.approx(1926.3 / 2) and "1035/2070" in src
+    # a sample above the maximum never raises the peak above the burst figure
+    assert bench.compute_peak(peaks, {"sm_mhz": 2100, "sm_max_mhz": 2070})[0] == 1926.3
+
+
+def test_config_entry_takes_the_larger_bound():
+    peaks = {"bf16_tflops": 1000.0, "hbm_gbs": 5000.0}
+    dom = {"kernel": "k"}
+    # 1 TFLOP at 1000 TFLOP/s = 1 ms against 1 GB at 5000 GB/s = 0.2 ms: tensor-bound
+    e = bench.config_entry("m", 1000, 2.0, (1e12, 1e9), dom, peaks, 5)
+    assert e["roofline"]["bound"] == "tensor"
+    assert e["roofline"]["frac"] == pytest.approx(0.5)
+    assert e["value"] == pytest.approx(1000 / 2e-3)
+    # 10 GB at 5000 GB/s = 2 ms against 1 ms of FLOPs: HBM-bound
+    e = bench.config_entry("m", 1000, 4.0, (1e12, 1e10), dom, peaks, 5)
+    assert e["roofline"]["bound"] == "hbm" and e["roofline"]["frac"] == pytest.approx(0.5)
+    # an fp32 workload divides by the measured FFMA peak and says "alu"
+    e = bench.config_entry("m", 1000, 2.0, (50e9, 1e6), dom, peaks, 5, ffma=50.0)
+    assert e["roofline"]["bound"] == "alu" and e["roofline"]["frac"] == pytest.approx(0.5)
+
+
+def test_traffic_lookup_scales_by_tokens_and_drops_stale_captures(tmp_path, monkeypatch):
+    label = "decompress_d1_inject"
+    (tmp_path / "profiles").mkdir()
+    csrc = os.path.join(bench.ROOT, "paper_2608_23463_gb300", "csrc")
+    (tmp_path / "paper_2608_23463_gb300").mkdir()
+    os.symlink(csrc, tmp_path / "paper_2608_23463_gb300" / "csrc")
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    h = bench.source_hash(label)
+    (tmp_path / "profiles" / "traffic.txt").write_text(
+        "# label bytes units hash\n%s 1000 100 %s\ninj_bwd 5 1 0000000000000000\n" % (label, h))
+    assert bench.traffic_from_profile(label, 400) == pytest.approx(4000.0)
+    assert bench.traffic_from_profile("inj_bwd", 1) is None       # captured at other sources
+    assert bench.traffic_from_profile("attn_fwd", 1) is None      # never captured
+    # every label hashes the files that define its kernel
+    assert "gemm_tc.cuh" in bench.kernel_files(label)
+    assert "elementwise.cu" in bench.kernel_files("inj_bwd")
+    assert "attention_tc.cu" in bench.kernel_files("attn_fwd")
