@@ -60,6 +60,29 @@ def test_layer_flops_match_the_contractions(levels, mode):
     assert f_train == pytest.approx(fwd + bwd, rel=1e-12)
 
 
+def test_cross_and_mlp_layer_flops_match_the_contractions():
+    """Gated cross injection (Eq. inj-cross with the gate of Sec. 3.7): the token-query
+    and gate GEMM, the proxies' keys and values, the attention of every token
+    over the proxies of earlier blocks, and the output projection replace the
+    decompression; the single-proxy MLP replaces the attention by two GEMMs."""
+    spec = S.LayerSpec(batch=1, L=262144, d=1024, n_heads=16, P=64, levels=2, k1=8, k2=8,
+                       inject=S.INJ_CROSS)
+    L, d, P, nh = spec.L, spec.d, spec.P, spec.n_heads
+    m = L // P
+    g = _layer_gemms(spec)[:4]                               # compressions, QKV, O
+    g += [(L, d + nh, d), (m, 2 * d, d), (L, d, d)]         # [Q | gate], [K | V], output
+    vis = sum(P * b for b in range(m))                       # token in block b sees b proxies
+    att = 4.0 * d * (_attention_pairs(m, True) + vis)
+    lin = _gemm_flops(g)
+    assert bench.layer_work(spec)[0] == pytest.approx(3 * lin + 3.5 * att, rel=1e-12)
+
+    mlp = S.LayerSpec(batch=1, L=262144, d=1024, n_heads=16, P=64, levels=2, k1=8, k2=8,
+                      interact=S.F_MLP)
+    g = [x for x in _layer_gemms(mlp) if x not in ((m, 3 * d, d), (m, d, d))]
+    g += [(m, 4 * d, d), (m, d, 4 * d)]
+    assert bench.layer_work(mlp)[0] == pytest.approx(3 * _gemm_flops(g), rel=1e-12)
+
+
 def test_headline_work_and_roofline_time():
     """The benchmark layer (L = 262144, d = 1024, P = 64 as 8 x 8): 3.934
     TFLOP and 3.52 GB per fwd+bwd step; X, dX_out read and X_out, dX written
