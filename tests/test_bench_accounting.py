@@ -83,6 +83,19 @@ def test_cross_and_mlp_layer_flops_match_the_contractions():
     assert bench.layer_work(mlp)[0] == pytest.approx(3 * _gemm_flops(g), rel=1e-12)
 
 
+def test_2d_layer_flops_match_the_contractions():
+    """2D layer (Sec. 3.9): each 8 x 8 patch of tokens compressed to a proxy,
+    bidirectional attention over the patch grid, and the decompression to a
+    scale and a shift per token channel (affine injection, 2 P d_fine wide)."""
+    spec = S.spec_c5()
+    d, P = spec.d, spec.P
+    m = spec.L // P
+    g = [(m, d, P * d), (m, 3 * d, d), (m, d, d), (m, 2 * P * d, d)]
+    att = 4.0 * d * m * m
+    expect = spec.batch * (3 * _gemm_flops(g) + 3.5 * att)
+    assert bench.layer_work(spec)[0] == pytest.approx(expect, rel=1e-12)
+
+
 def test_headline_work_and_roofline_time():
     """The benchmark layer (L = 262144, d = 1024, P = 64 as 8 x 8): 3.934
     TFLOP and 3.52 GB per fwd+bwd step; X, dX_out read and X_out, dX written
