@@ -156,3 +156,27 @@ def test_traffic_lookup_scales_by_tokens_and_drops_stale_captures(tmp_path, monk
     assert "gemm_tc.cuh" in bench.kernel_files(label)
     assert "elementwise.cu" in bench.kernel_files("inj_bwd")
     assert "attention_tc.cu" in bench.kernel_files("attn_fwd")
+
+
+@pytest.mark.parametrize("levels", [1, 2])
+def test_one_segment_has_the_work_of_the_layer(levels):
+    """Temporal-distance ratios (Sec. 3.6) with a single segment are the
+    ordinary layer, work included; with several, each segment's compression
+    and decompression at its own ratio plus one attention over all proxies."""
+    kw = dict(k1=8, k2=8) if levels == 2 else {}
+    seg = [(262144, 64, 8, 8)]
+    lay = S.LayerSpec(batch=1, L=262144, d=1024, n_heads=16, P=64, levels=levels, **kw)
+    f, b = bench.segments_work(1024, 16, levels, seg)
+    fl, bl = bench.layer_work(lay)
+    assert f == pytest.approx(fl, rel=1e-12) and b == pytest.approx(bl, rel=1e-12)
+    segs = [(131072, 256, 16, 16), (98304, 64, 8, 8), (32768, 16, 4, 4)]
+    f3, _ = bench.segments_work(1024, 16, 2, segs)
+    m_tot = sum(Ls // Ps for Ls, Ps, _, _ in segs)
+    lin = 0.0
+    for Ls, Ps, a, c in segs:
+        sp = S.LayerSpec(batch=1, L=Ls, d=1024, n_heads=16, P=Ps, levels=2, k1=a, k2=c)
+        lin += _gemm_flops([x for x in _layer_gemms(sp)
+                            if x not in ((Ls // Ps, 3 * 1024, 1024), (Ls // Ps, 1024, 1024))])
+    lin += _gemm_flops([(m_tot, 3 * 1024, 1024), (m_tot, 1024, 1024)])
+    att = 4.0 * 1024 * _attention_pairs(m_tot, True)
+    assert f3 == pytest.approx(3 * lin + 3.5 * att, rel=1e-12)
