@@ -348,11 +348,19 @@ def measure_decode(torch, pf, S, steps: int):
     a1.record(stream)
     torch.cuda.synchronize()
     pf.pf_sync_check(stream.cuda_stream)
+    return spec, ms, ms_direct, a0.elapsed_time(a1), decode_step_bytes(spec, steps), kern
+
+
+def decode_step_bytes(spec, steps: int) -> float:
+    """Algorithmic HBM bytes of one decode step (Sec. 3.8), bf16: the K and V
+    rows of every cached proxy of every sequence, the weights read once
+    (W_qkv, W_o, the alpha MLP's first layer d x d/8), the open block's K and
+    V rows (on average half full over the timed steps), the token in and the
+    output out."""
     B, d, cap = spec.batch, spec.d, spec.capacity
     mean_open = (min(steps, spec.P) + 1) / 2.0
-    step_bytes = (2 * B * cap * d * 2 + (3 * d * d + d * d + d * d // 8) * 2
-                  + B * mean_open * 2 * d * 2 + 2 * B * d * 2)
-    return spec, ms, ms_direct, a0.elapsed_time(a1), step_bytes, kern
+    return (2 * B * cap * d * 2 + (3 * d * d + d * d + d * d // 8) * 2
+            + B * mean_open * 2 * d * 2 + 2 * B * d * 2)
 
 
 def timed_steps(torch, pf, fn, steps: int, warmup: int):

@@ -180,3 +180,16 @@ def test_one_segment_has_the_work_of_the_layer(levels):
     lin += _gemm_flops([(m_tot, 3 * 1024, 1024), (m_tot, 1024, 1024)])
     att = 4.0 * 1024 * _attention_pairs(m_tot, True)
     assert f3 == pytest.approx(3 * lin + 3.5 * att, rel=1e-12)
+
+
+def test_decode_step_bytes():
+    """Decode at the paper's shape (B = 8, d = 2048, 16384 cached proxies):
+    ~1.11 GB per step, almost all of it the cached K and V rows, which every
+    step streams once; the weights add 4.125 d^2 bf16 elements."""
+    spec = S.spec_c4()
+    b = bench.decode_step_bytes(spec, 128)
+    cache = spec.batch * spec.capacity * 2 * spec.d * 2
+    assert b == pytest.approx(1.1105e9, rel=1e-3)
+    assert cache / b > 0.96
+    assert b - bench.decode_step_bytes(spec, 1) == pytest.approx(
+        spec.batch * (32.5 - 1.0) * 2 * spec.d * 2)  # the open block's mean fill
